@@ -1,0 +1,162 @@
+"""fp64 CPU oracle for causal resonant field mixing (ResonatorLM, arxiv 2607.05583).
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+CPU-baseline / reference legs of ``bench.py`` may import this package.  The
+product library (``paper_2607_05583_gb300``) never imports it, and it never
+imports the product: the two share no code.
+
+The arithmetic lives in ``rlm_oracle.c`` (plain C, double precision, optional
+OpenMP over independent channels).  This module only compiles that file with
+gcc and marshals numpy arrays into it.
+
+Functions (all arrays float64, C-contiguous; shapes as in the paper's notation,
+channel innermost):
+
+* ``conv_prefill``   O1: direct O(L^2) causal convolution, Eq. 1-2.
+* ``rec_prefill``    O2: sequential complex recurrence, Eq. 4-5, plus the
+                      prompt's terminal state (Sec. 3.2).
+* ``rec_decode``     one decode step, Eq. 4-5.
+* ``backward_conv``  O3 via the convolution route (chain rule through Eq. 1-2).
+* ``backward_rec``   O3 via the reverse-time Jordan recurrence.
+* ``kernel_table``   K_d[n] of Eq. 1.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "rlm_oracle.c")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD_DIR, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile rlm_oracle.c into oracle/_build/liboracle.so (gcc, -O2, OpenMP)."""
+    os.makedirs(_BUILD_DIR, exist_ok=True)
+    stale = (not os.path.exists(_LIB_PATH)
+             or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC))
+    if force or stale:
+        tmp = _LIB_PATH + f".{os.getpid()}.tmp"
+        cmd = ["gcc", "-O2", "-std=c11", "-fopenmp", "-fPIC", "-shared",
+               _SRC, "-o", tmp, "-lm"]
+        subprocess.check_call(cmd)
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            dp = ctypes.POINTER(ctypes.c_double)
+            L_, I_ = ctypes.c_long, ctypes.c_int
+            lib.oracle_num_threads.restype = I_
+            lib.oracle_kernel_table.argtypes = [I_, I_, dp, dp, dp, dp, L_, dp]
+            lib.oracle_conv_prefill.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp]
+            lib.oracle_rec_prefill.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp, dp]
+            lib.oracle_rec_decode.argtypes = [L_, I_, I_, dp, dp, dp, dp, dp, dp, dp, dp]
+            lib.oracle_backward_conv.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp,
+                                                 dp, dp, dp, dp, dp]
+            lib.oracle_backward_rec.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp,
+                                                dp, dp, dp, dp, dp]
+            _lib = lib
+    return _lib
+
+
+def _f64(a) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=np.float64))
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_double))
+
+
+def _params(decay, freq, amp, phase):
+    ps = [_f64(p) for p in (decay, freq, amp, phase)]
+    D, M = ps[0].shape
+    for p in ps:
+        if p.shape != (D, M):
+            raise ValueError("decay/freq/amp/phase must all be [D][M]")
+    return ps, D, M
+
+
+def num_threads() -> int:
+    return int(_load().oracle_num_threads())
+
+
+def kernel_table(decay, freq, amp, phase, L: int) -> np.ndarray:
+    """K[d][n] = sum_m A exp(-gamma n) cos(omega n + phi), n < L (Eq. 1)."""
+    ps, D, M = _params(decay, freq, amp, phase)
+    K = np.empty((D, L), np.float64)
+    _load().oracle_kernel_table(D, M, *map(_ptr, ps), L, _ptr(K))
+    return K
+
+
+def conv_prefill(x, decay, freq, amp, phase) -> np.ndarray:
+    """O1: y[b,t,d] = sum_{j<=t} K_d[t-j] x[b,j,d] by direct summation (Eq. 2)."""
+    x = _f64(x)
+    ps, D, M = _params(decay, freq, amp, phase)
+    B, L, Dx = x.shape
+    assert Dx == D
+    y = np.empty_like(x)
+    _load().oracle_conv_prefill(B, L, D, M, _ptr(x), *map(_ptr, ps), _ptr(y))
+    return y
+
+
+def rec_prefill(x, decay, freq, amp, phase):
+    """O2: sequential recurrence from a zero state (Eq. 4-5).
+
+    Returns (y [B][L][D], state [B][D][M] complex128)."""
+    x = _f64(x)
+    ps, D, M = _params(decay, freq, amp, phase)
+    B, L, Dx = x.shape
+    assert Dx == D
+    y = np.empty_like(x)
+    st = np.empty((B, D, M, 2), np.float64)
+    _load().oracle_rec_prefill(B, L, D, M, _ptr(x), *map(_ptr, ps), _ptr(y), _ptr(st))
+    return y, st[..., 0] + 1j * st[..., 1]
+
+
+def rec_decode(state, x_t, decay, freq, amp, phase):
+    """One decode step (Eq. 4-5).  state: [B][D][M] complex; x_t: [B][D].
+
+    Returns (y_t [B][D], new state [B][D][M] complex128)."""
+    state = np.asarray(state)
+    x_t = _f64(x_t)
+    ps, D, M = _params(decay, freq, amp, phase)
+    B = x_t.shape[0]
+    sin = np.ascontiguousarray(np.stack([state.real, state.imag], -1), np.float64)
+    sout = np.empty_like(sin)
+    y = np.empty((B, D), np.float64)
+    _load().oracle_rec_decode(B, D, M, _ptr(sin), _ptr(x_t), *map(_ptr, ps),
+                              _ptr(sout), _ptr(y))
+    return y, sout[..., 0] + 1j * sout[..., 1]
+
+
+def _backward(fn, x, dy, decay, freq, amp, phase):
+    x, dy = _f64(x), _f64(dy)
+    ps, D, M = _params(decay, freq, amp, phase)
+    B, L, Dx = x.shape
+    assert Dx == D and dy.shape == x.shape
+    dx = np.empty_like(x)
+    g = [np.empty((D, M), np.float64) for _ in range(4)]
+    fn(B, L, D, M, _ptr(x), _ptr(dy), *map(_ptr, ps), _ptr(dx), *map(_ptr, g))
+    return dx, {"decay": g[0], "freq": g[1], "amp": g[2], "phase": g[3]}
+
+
+def backward_conv(x, dy, decay, freq, amp, phase):
+    """O3 by the convolution route.  Returns (dx, {decay, freq, amp, phase})."""
+    return _backward(_load().oracle_backward_conv, x, dy, decay, freq, amp, phase)
+
+
+def backward_rec(x, dy, decay, freq, amp, phase):
+    """O3 by the reverse-time Jordan recurrence.  Returns (dx, grads dict)."""
+    return _backward(_load().oracle_backward_rec, x, dy, decay, freq, amp, phase)
