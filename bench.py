@@ -1,0 +1,504 @@
+"""Benchmark of the causal resonant field mixing operator on GB300.
+
+Headline (``value``): prefill throughput in Mtok/s at L = 32768 on the long-context
+workload (B=4, L=32768, D=256, M=16, bf16 I/O, fp32 state), inputs resident in HBM,
+L2 flushed (a 512 MiB write) before every timed step.  One step = one
+rlm_mix_prefill call: parameter precompute, intra-chunk Toeplitz contraction,
+inter-chunk carry, state up-projection, epilogue and terminal state.
+
+Also reported on the same line:
+  decode    4096 single-token rlm_mix_decode steps at B=64 (D=256, M=16) after a
+            32768-token prefill, captured in a CUDA graph; tok/s and % of HBM.
+  backward  rlm_mix_backward at B=4, L=32768, D=512, M=32 (bf16 I/O).
+  roofline  achieved algorithmic GB/s of the prefill against the measured HBM peak.
+  e2e       the same prefill metric through the C ABI with pinned HOST buffers
+            (host->device copy of x and device->host copy of y inside the timing).
+  cpu_baseline  the fp64 CPU oracle (sequential recurrence) on the host cores.
+
+``--impl reference`` times the CPU oracle itself as the reference arm.
+Multi-GPU (torchrun, N > 1): every rank runs its own independent batch of the
+same workload (weak scaling, replicas only; the operator has no cross-GPU
+exchange); rank 0 prints value = all ranks' tokens / max time over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "mix prefill Mtok/s at L=32K (% of roofline); decode tok/s at B=64 (% HBM)"
+PREFILL = dict(B=4, L=32768, D=256, M=16)
+DECODE = dict(B=64, L=32768, D=256, M=16, T=4096)
+BACKWARD = dict(B=4, L=32768, D=512, M=32)
+L2_FLUSH_BYTES = 512 << 20
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            pk = json.load(f)
+        return float(pk["hbm_gbs"]), float(pk["bf16_tflops"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, "fallback"
+
+
+def prefill_bytes(B, L, D, M):
+    """Algorithmic HBM bytes of one bf16 prefill: read x, write y (2 B each per
+    token-channel), write the terminal state (8 B per (b,d,m)) and its
+    coefficients (16 B per (d,m)), read the parameters (16 B per (d,m))."""
+    return B * L * D * 4 + B * D * M * 8 + D * M * 32
+
+
+def decode_bytes(B, D, M):
+    """Per decode step: state read+write (16 B per (b,d,m)), token in and out
+    (bf16, 4 B per (b,d)), coefficients (16 B per (d,m))."""
+    return 16 * B * D * M + 4 * B * D + 16 * D * M
+
+
+def backward_bytes(B, L, D, M):
+    """Per backward call: read x and dy, write dx (bf16, 6 B per token-channel),
+    read params and write four gradients (32 B per (d,m))."""
+    return 6 * B * L * D + 32 * D * M
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index=0):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self._t = threading.Thread(target=self._read, daemon=True)
+            self._t.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": mx, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- helpers
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def _barrier_max(t, ws):
+    if ws == 1:
+        return t
+    import torch
+    import torch.distributed as dist
+    v = torch.tensor([t], dtype=torch.float64, device="cuda")
+    dist.all_reduce(v, op=dist.ReduceOp.MAX)
+    return float(v.item())
+
+
+def _barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def _traffic_from_profiles(kernel_tag):
+    """DRAM bytes per launch recorded in profiles/<kernel_tag>.md, valid only while
+    the kernel source hash recorded there matches the current source."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"{kernel_tag}.md")
+    if not os.path.exists(path):
+        return None
+    kv = {}
+    for line in open(path):
+        if line.startswith("- ") and ":" in line:
+            k, v = line[2:].split(":", 1)
+            kv[k.strip()] = v.strip().strip("`")
+    src = kv.get("source")
+    if not src or "dram_bytes_per_full_launch" not in kv:
+        return None
+    try:
+        h = hashlib.sha256(open(os.path.join(ROOT, src), "rb").read()).hexdigest()[:16]
+    except OSError:
+        return None
+    if h != kv.get("source_sha256_16"):
+        return None
+    return float(kv["dram_bytes_per_full_launch"])
+
+
+# ---------------------------------------------------------------- our arm
+def run_ours(args):
+    import torch
+
+    import paper_2607_05583_gb300 as rlm
+    from synth import make_inputs
+
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    dev = torch.device("cuda", local)
+    rlm.load_library()
+    hbm_peak, bf16_peak, peak_kind = _peaks()
+    stream = torch.cuda.current_stream()
+
+    # ---------------- prefill (headline)
+    P = PREFILL
+    inp = make_inputs(P["B"], P["L"], P["D"], P["M"], "bf16", seed=rank)
+    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
+    params = rlm.Params.from_arrays(*inp.params(), device=dev)
+    y = torch.empty_like(x)
+    st = rlm.State.empty(P["B"], P["D"], P["M"], device=dev)
+    wsz = rlm.rlm_prefill_workspace_size(P["B"], P["L"], P["D"], P["M"], torch.bfloat16)
+    work = torch.empty(max(wsz, 256), dtype=torch.uint8, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def step():
+        rlm.rlm_mix_prefill(x, params, y, st, workspace=work)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    n_launch = _count_launches(step)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    _barrier(ws)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        for i in range(args.steps):
+            flush.zero_()
+            starts[i].record(stream)
+            step()
+            ends[i].record(stream)
+        torch.cuda.synchronize()
+    _barrier(ws)
+    times = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    ms = statistics.mean(times)
+    ms_max = _barrier_max(ms, ws)
+    tokens = P["B"] * P["L"]
+    value = ws * tokens / (ms_max * 1e-3) / 1e6
+    alg = prefill_bytes(P["B"], P["L"], P["D"], P["M"])
+    achieved = alg / (ms * 1e-3) / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm_peak,
+                "unit": "GB/s", "frac": round(achieved / hbm_peak, 4),
+                "traffic": _traffic_from_profiles("prefill_tc_long_b4_32k"),
+                "peak_kind": peak_kind, "frac_of_8TBps": round(achieved / 8000.0, 4),
+                "algorithmic_bytes_per_launch": alg,
+                "kernel": "rlm_mix_prefill (whole call)", "median_ms": statistics.median(times)}
+
+    # ---------------- e2e through the C ABI with host buffers
+    xh = torch.from_numpy(inp.x).to(torch.bfloat16).pin_memory()
+    yh = torch.empty_like(xh).pin_memory()
+    for _ in range(2):
+        x.copy_(xh, non_blocking=True)
+        step()
+        yh.copy_(y, non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(3, args.steps // 2)
+    e0.record(stream)
+    for _ in range(reps):
+        x.copy_(xh, non_blocking=True)
+        step()
+        yh.copy_(y, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / reps
+    e2e = {"value": round(tokens / (e2e_ms * 1e-3) / 1e6, 2), "unit": "Mtok/s",
+           "h2d_bytes_per_step": xh.numel() * 2, "d2h_bytes_per_step": yh.numel() * 2}
+    del xh, yh
+
+    # ---------------- per-L sweep (same launch configuration)
+    sweep = {}
+    if not args.quick:
+        for (B, L) in ((1, 8192), (1, 16384), (1, 32768), (4, 8192), (4, 16384)):
+            sweep[f"B{B}_L{L}"] = _time_prefill(rlm, torch, dev, B, L, P["D"], P["M"], flush,
+                                                hbm_peak, reps=max(5, args.steps // 2))
+    sweep[f"B{P['B']}_L{P['L']}"] = {"Mtok_s": round(tokens / (ms * 1e-3) / 1e6, 1),
+                                     "frac": roofline["frac"]}
+    del x, y, work
+
+    # ---------------- decode
+    decode = None if args.quick else _bench_decode(rlm, torch, dev, hbm_peak)
+    # ---------------- backward
+    backward = None if args.quick else _bench_backward(rlm, torch, dev, hbm_peak, args)
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu:
+        cpu = cpu_baseline(seconds=args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 2), "unit": "Mtok/s", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max, 5),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16", "data": "synthetic (seeded N(0,1) drives, paper-range resonator params)",
+            "config": {"workload": "long-context prefill B=4 L=32768 D=256 M=16 bf16 I/O fp32 state",
+                       "B": P["B"], "L": P["L"], "D": P["D"], "M": P["M"],
+                       "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
+                       "l2": "flushed (512 MiB write) before every timed step"},
+            "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": n_launch * args.steps,
+            "clocks": clk.summary(), "sweep": sweep, "decode": decode, "backward": backward,
+        }
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def _count_launches(step):
+    """Kernels of ours that one step launches (counted with the profiler's CUDA
+    activity list, names matched against the library's kernel prefixes)."""
+    import torch
+    from torch.profiler import ProfilerActivity, profile
+    try:
+        with profile(activities=[ProfilerActivity.CUDA]) as prof:
+            step()
+            torch.cuda.synchronize()
+        n = 0
+        for ev in prof.events():
+            name = ev.name or ""
+            if "rlm::" in name or name.startswith("k_") or "rlm" in name:
+                n += 1
+        return n
+    except Exception:
+        return -1
+
+
+def _time_prefill(rlm, torch, dev, B, L, D, M, flush, hbm_peak, reps=5):
+    from synth import make_inputs
+    inp = make_inputs(B, L, D, M, "bf16", seed=1)
+    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
+    p = rlm.Params.from_arrays(*inp.params(), device=dev)
+    y = torch.empty_like(x)
+    st = rlm.State.empty(B, D, M, device=dev)
+    wsz = rlm.rlm_prefill_workspace_size(B, L, D, M, torch.bfloat16)
+    work = torch.empty(max(wsz, 256), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    for _ in range(3):
+        rlm.rlm_mix_prefill(x, p, y, st, workspace=work)
+    ts = []
+    for _ in range(reps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        rlm.rlm_mix_prefill(x, p, y, st, workspace=work)
+        b.record(stream)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    ms = statistics.mean(ts)
+    gbs = prefill_bytes(B, L, D, M) / (ms * 1e-3) / 1e9
+    return {"Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 1), "ms": round(ms, 5),
+            "frac": round(gbs / hbm_peak, 4)}
+
+
+def _bench_decode(rlm, torch, dev, hbm_peak):
+    from synth import make_inputs
+    P = DECODE
+    B, L, D, M, T = P["B"], P["L"], P["D"], P["M"], P["T"]
+    inp = make_inputs(B, L, D, M, "bf16", seed=0, decode_steps=T)
+    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
+    p = rlm.Params.from_arrays(*inp.params(), device=dev)
+    y = torch.empty_like(x)
+    st = rlm.State.empty(B, D, M, device=dev)
+    rlm.rlm_mix_prefill(x, p, y, st)
+    del x, y
+    toks = torch.from_numpy(inp.tokens).to(dev, torch.bfloat16)     # [T][B][D]
+    outs = torch.empty_like(toks)
+    s0 = st.s.clone()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):          # warm up on a side stream before capture
+        for t in range(8):
+            rlm.rlm_mix_decode(toks[t], st, outs[t])
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for t in range(T):
+            rlm.rlm_mix_decode(toks[t], st, outs[t])
+    stream = torch.cuda.current_stream()
+    res = []
+    for rep in range(4):
+        st.s.copy_(s0)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        if rep:
+            res.append(a.elapsed_time(b))
+    ms = statistics.median(res)
+    us_step = ms * 1e3 / T
+    per_step = decode_bytes(B, D, M)
+    gbs = per_step / (us_step * 1e-6) / 1e9
+    return {"workload": "decode B=64 D=256 M=16, 4096 steps after a 32768-token prefill, CUDA graph",
+            "tok_s": round(B * T / (ms * 1e-3), 1), "us_per_step": round(us_step, 4),
+            "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
+            "bytes_per_step": per_step, "launches": T}
+
+
+def _bench_backward(rlm, torch, dev, hbm_peak, args):
+    from synth import make_inputs
+    P = BACKWARD
+    B, L, D, M = P["B"], P["L"], P["D"], P["M"]
+    inp = make_inputs(B, L, D, M, "bf16", seed=0, with_dy=True)
+    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
+    dy = torch.from_numpy(inp.dy).to(dev, torch.bfloat16)
+    p = rlm.Params.from_arrays(*inp.params(), device=dev)
+    dx = torch.empty_like(x)
+    g = rlm.Grads.empty(D, M, device=dev)
+    wsz = rlm.rlm_backward_workspace_size(B, L, D, M, torch.bfloat16)
+    work = torch.empty(max(wsz, 256), dtype=torch.uint8, device=dev)
+    for _ in range(2):
+        rlm.rlm_mix_backward(dy, x, p, dx, g, workspace=work)
+    stream = torch.cuda.current_stream()
+    ts = []
+    for _ in range(3):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        rlm.rlm_mix_backward(dy, x, p, dx, g, workspace=work)
+        b.record(stream)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    ms = statistics.mean(ts)
+    gbs = backward_bytes(B, L, D, M) / (ms * 1e-3) / 1e9
+    return {"workload": "backward B=4 L=32768 D=512 M=32 bf16", "ms": round(ms, 4),
+            "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 2), "achieved_GBps": round(gbs, 1),
+            "frac_hbm": round(gbs / hbm_peak, 4)}
+
+
+# ---------------------------------------------------------------- CPU oracle
+def cpu_baseline(seconds=10.0):
+    """The fp64 oracle's sequential recurrence (as it stands) on the host cores, on
+    a bounded sample of the prefill workload: whole sequences of the B=4, L=32768,
+    D=256, M=16 problem, repeated until about ``seconds`` of CPU time."""
+    import oracle
+    from synth import make_inputs
+    P = PREFILL
+    inp = make_inputs(1, P["L"], P["D"], P["M"], "bf16", seed=0)
+    x64 = inp.x.astype(np.float64)
+    prm = [q.astype(np.float64) for q in inp.params()]
+    oracle.rec_prefill(x64[:, :1024], *prm)          # load/compile outside the timing
+    t0 = time.perf_counter()
+    n = 0
+    while True:
+        oracle.rec_prefill(x64, *prm)
+        n += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": round(n * P["L"] / dt / 1e6, 4), "unit": "Mtok/s", "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": f"{n} x one sequence (B=1, L={P['L']}, D={P['D']}, M={P['M']}) of the "
+                      f"prefill workload through the fp64 sequential recurrence, {dt:.1f} s"}
+
+
+def run_reference(args):
+    """Reference arm: the CPU oracle as it stands, on the host cores."""
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    import oracle
+    from synth import make_inputs
+    P = PREFILL
+    inp = make_inputs(1, P["L"], P["D"], P["M"], "bf16", seed=0)
+    x64 = inp.x.astype(np.float64)
+    prm = [q.astype(np.float64) for q in inp.params()]
+    for _ in range(args.warmup):
+        oracle.rec_prefill(x64[:, :4096], *prm)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle.rec_prefill(x64, *prm)
+    dt = time.perf_counter() - t0
+    val = args.steps * P["L"] / dt / 1e6
+    cpu = {"value": round(val, 4), "unit": "Mtok/s", "cores": oracle.num_threads(), "kind": "oracle",
+           "sample": f"each step one sequence (B=1, L={P['L']}, D={P['D']}, M={P['M']}) of the "
+                     f"prefill workload through the fp64 sequential recurrence"}
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": round(val, 4), "unit": "Mtok/s",
+        "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(dt / args.steps * 1e3, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "long-context prefill B=4 L=32768 D=256 M=16 bf16 I/O fp32 state",
+                   "sample": "B=1 per step"},
+        "cpu_baseline": cpu,
+        "e2e": {"value": round(val, 4), "unit": "Mtok/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0}}), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--quick", action="store_true", help="prefill only (no sweep/decode/backward)")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,183 @@
+/*
+ * rlm.h -- C ABI of the GB300 (sm_103a) causal resonant field mixing library.
+ *
+ * The operator is the attention replacement of ResonatorLM (arxiv 2607.05583):
+ * every channel d of a (B, L, D) token field drives M damped resonators.  With
+ * per-mode decay gamma, frequency omega, amplitude A and phase phi,
+ *
+ *   lambda_dm = exp(-gamma_dm) (cos omega_dm + i sin omega_dm)        (Eq. 5)
+ *   c_dm      = A_dm exp(+i phi_dm)
+ *   K_d[n]    = sum_m A_dm exp(-gamma_dm n) cos(omega_dm n + phi_dm)  (Eq. 1)
+ *   y[b,t,d]  = sum_{j<=t} K_d[t-j] x[b,j,d]                          (Eq. 2)
+ *
+ * which is the same map as the complex recurrence s <- lambda s + x_t,
+ * y_t = sum_m Re(c s) of Sec. 3.3 (Eq. 4), started from a zero state.  The
+ * paper's readout Re(e^{-i phi} s) is taken as Re(e^{+i phi} s) so that decode
+ * agrees with Eq. 1; the paper's single mode per head is the case M = 1, A = 1
+ * with parameters tied across a head's channels.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - All tensor and parameter pointers are DEVICE pointers, 16-byte aligned.
+ *    The caller owns every buffer; the library allocates nothing on any call
+ *    path and keeps no pointer after a call returns.
+ *  - Every call is asynchronous on launch->stream (a cudaStream_t passed as
+ *    void*; NULL is the legacy default stream).
+ *  - Argument checks run on the host before anything is enqueued; a failing
+ *    check returns RLM_ERR_INVALID_ARG or RLM_ERR_UNSUPPORTED and enqueues
+ *    nothing.  rlm_last_error() then describes the failure.
+ *  - A failed kernel launch returns RLM_ERR_CUDA.
+ *  - Kernels that wait on one another (the prefill's cross-block carry) wait a
+ *    bounded number of iterations; on expiry they record RLM_ERR_TIMEOUT in a
+ *    device status word and return without hanging.  rlm_get_device_status()
+ *    reads and clears that word.
+ *  - Shapes: B >= 1, L >= 1, D >= 8 with D % 8 == 0, 1 <= M <= 64.
+ *  - Element types of x, y, dy, dx: RLM_F32 or RLM_BF16 (all four of one call
+ *    share one type).  Parameters, gradients and the decode state are fp32.
+ *  - Inputs and outputs of one call must not overlap.
+ */
+#ifndef RLM_H_
+#define RLM_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define RLM_API __attribute__((visibility("default")))
+#else
+#define RLM_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    RLM_OK = 0,
+    RLM_ERR_INVALID_ARG = 1,  /* bad pointer, shape, dtype, alignment or size   */
+    RLM_ERR_UNSUPPORTED = 2,  /* well-formed but outside what the kernels cover */
+    RLM_ERR_CUDA = 3,         /* a CUDA runtime call or kernel launch failed    */
+    RLM_ERR_TIMEOUT = 4       /* a bounded device-side wait expired             */
+} rlm_status;
+
+typedef enum { RLM_F32 = 0, RLM_BF16 = 1 } rlm_dtype;
+
+/* Resonator parameters (Sec. 3.1 and Eq. 5), each fp32 [D][M] row-major on the
+ * device, in the constrained space (gamma >= 0 and finite, any finite omega,
+ * A and phi).  The paper's softplus/sigmoid reparameterisation lives outside
+ * the operator. */
+typedef struct {
+    const float *decay;   /* gamma_dm */
+    const float *freq;    /* omega_dm */
+    const float *amp;     /* A_dm     */
+    const float *phase;   /* phi_dm   */
+    int D, M;
+} rlm_params;
+
+/* Gradients of a scalar loss with respect to rlm_params; same layout.
+ * Overwritten (not accumulated) by rlm_mix_backward. */
+typedef struct {
+    float *decay, *freq, *amp, *phase;
+    int D, M;
+} rlm_grads;
+
+/* A dense, contiguous [B][L][D] field on the device, channel innermost.
+ * Single-token tensors of decode use L = 1. */
+typedef struct {
+    void *ptr;
+    rlm_dtype dtype;
+    int64_t B, L, D;
+} rlm_tensor;
+
+/* The fixed-size recurrent state of Sec. 3.3 (Eq. 4, "two real tensors", whose
+ * size does not grow with decoded length), stored as interleaved complex fp32:
+ *   s    [B][D][M][2]  (Re, Im) of s_bdm
+ *   coef [D][M][4]     (Re lambda, Im lambda, Re c, Im c) of each mode
+ * The coefficients travel with the state because decode takes no parameters.
+ * rlm_mix_prefill (state_out) and rlm_state_init fill both. */
+typedef struct {
+    float *s;
+    float *coef;
+    int B, D, M;
+} rlm_state;
+
+/* Launch context: the stream, and a caller-owned device workspace of at least
+ * the size the matching *_workspace_size() query returns (256-byte aligned). */
+typedef struct {
+    void *stream;
+    void *workspace;
+    size_t workspace_bytes;
+} rlm_launch;
+
+/* ------------------------------------------------------------------ prefill
+ * Full-sequence causal mixing, Sec. 3.2 (Eq. 2; the paper evaluates it by FFT,
+ * Eq. 3, this library by a chunked complex-diagonal scan with the same result
+ * up to rounding), from a zero initial state.
+ *   x          [B][L][D] input field (F32 or BF16)
+ *   p          resonator parameters, p->D == x->D
+ *   y          [B][L][D] output, same shape and dtype as x; overwritten
+ *   state_out  nullable; if given (state_out->B == B, D, M matching), receives
+ *              the prompt's terminal state s_{L-1} = sum_j lambda^{L-1-j} x_j
+ *              (Sec. 3.2) and the mode coefficients, ready for decode.
+ * BF16 I/O with M == 16 runs on the tcgen05 tensor-core path; other cases run
+ * the fp32 SIMT chunked scan.  Both accumulate the state in fp32. */
+RLM_API rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor *y,
+                           rlm_state *state_out, const rlm_launch *launch);
+
+/* Bytes of workspace rlm_mix_prefill needs for this shape (0 is possible). */
+RLM_API size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype);
+
+/* ------------------------------------------------------------------- decode
+ * One autoregressive step of Sec. 3.3 (Eq. 4-5) for a batch of tokens:
+ *   s_bdm <- lambda_dm s_bdm + x_t[b,d];   y_t[b,d] = sum_m Re(c_dm s_bdm)
+ *   x_t    [B][1][D] input token field (F32 or BF16)
+ *   state  in/out, updated in place (state->B == B, D, M matching)
+ *   y_t    [B][1][D] output, same dtype as x_t
+ * Needs no workspace (launch->workspace may be NULL). */
+RLM_API rlm_status rlm_mix_decode(const rlm_tensor *x_t, rlm_state *state, rlm_tensor *y_t,
+                          const rlm_launch *launch);
+
+/* Zero state->s and fill state->coef from p (for decoding without a prompt). */
+RLM_API rlm_status rlm_state_init(rlm_state *state, const rlm_params *p, const rlm_launch *launch);
+
+/* ----------------------------------------------------------------- backward
+ * Gradients of a scalar loss l through Eq. 2, given dy = dl/dy:
+ *   dx[b,j,d] = sum_{t>=j} K_d[t-j] dy[b,t,d]        (anti-causal mixing)
+ *   with G_dm = sum_{b,j} x_j S_j and P_dm = sum_{b,j} x_j R_j, where
+ *   S_j = sum_{t>=j} lambda^{t-j} dy_t, R_j = sum_{t>=j} (t-j) lambda^{t-j} dy_t:
+ *   dA = Re(e^{i phi} G), dphi = -Im(c G), dgamma = -Re(c P), domega = -Im(c P).
+ *   dy, x   [B][L][D] (same dtype);  dx [B][L][D] output, overwritten
+ *   dparams fp32 [D][M] each, overwritten; summed over batch and time in a
+ *           fixed order (bit-reproducible run to run).
+ * There is no gradient input for state_out: the loss depends on y only. */
+RLM_API rlm_status rlm_mix_backward(const rlm_tensor *dy, const rlm_tensor *x, const rlm_params *p,
+                            rlm_tensor *dx, rlm_grads *dparams, const rlm_launch *launch);
+
+RLM_API size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype);
+
+/* ------------------------------------------------------------------ utility
+ * rlm_validate_params: copies p to the host (synchronous) and checks that every
+ * value is finite and every gamma >= 0 (Sec. 3.1 requires alpha > 0; gamma = 0
+ * is accepted as the undamped limit).  The hot-path calls do not read
+ * parameters on the host, so they do not perform this check. */
+RLM_API rlm_status rlm_validate_params(const rlm_params *p);
+
+/* Synchronises launch->stream, then reports and clears the device status word:
+ * RLM_ERR_TIMEOUT if a bounded wait expired since the last call, else RLM_OK
+ * (or RLM_ERR_CUDA if the stream reports an error). */
+RLM_API rlm_status rlm_get_device_status(const rlm_launch *launch);
+
+/* Static description of a status code. */
+RLM_API const char *rlm_status_string(rlm_status status);
+
+/* Human-readable reason for the last non-OK status returned on this host
+ * thread (valid until the next call on the thread). */
+RLM_API const char *rlm_last_error(void);
+
+/* Library version as major*10000 + minor*100 + patch. */
+RLM_API int rlm_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* RLM_H_ */

@@ -1,0 +1,289 @@
+"""Python binding of the GB300 causal resonant field mixing library (``librlm.so``).
+
+Argument marshalling only: every step of the operator runs in the library's
+CUDA kernels, reached through the C ABI declared in ``include/rlm.h`` with the
+same function names.  PyTorch supplies device memory and the current stream.
+There is no fallback: if the compiled library is missing the calls raise.
+
+Names follow the paper (ResonatorLM, arxiv 2607.05583): x is the drive field
+[B][L][D]; decay gamma, frequency omega, amplitude A and phase phi are the
+per-mode resonator parameters [D][M]; the state is the complex recurrent state
+of Sec. 3.3, [B][D][M] complex fp32 plus its mode coefficients.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+from . import build as _build_mod
+
+__all__ = [
+    "RlmError", "Params", "Grads", "State", "load_library", "library_path",
+    "rlm_mix_prefill", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
+    "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
+    "rlm_validate_params", "rlm_get_device_status", "rlm_status_string",
+    "rlm_version", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
+    "RLM_ERR_CUDA", "RLM_ERR_TIMEOUT", "RLM_F32", "RLM_BF16",
+]
+
+RLM_OK, RLM_ERR_INVALID_ARG, RLM_ERR_UNSUPPORTED, RLM_ERR_CUDA, RLM_ERR_TIMEOUT = range(5)
+RLM_F32, RLM_BF16 = 0, 1
+
+
+class _Tensor(ctypes.Structure):
+    _fields_ = [("ptr", ctypes.c_void_p), ("dtype", ctypes.c_int),
+                ("B", ctypes.c_int64), ("L", ctypes.c_int64), ("D", ctypes.c_int64)]
+
+
+class _Params(ctypes.Structure):
+    _fields_ = [("decay", ctypes.c_void_p), ("freq", ctypes.c_void_p),
+                ("amp", ctypes.c_void_p), ("phase", ctypes.c_void_p),
+                ("D", ctypes.c_int), ("M", ctypes.c_int)]
+
+
+_Grads = _Params
+
+
+class _State(ctypes.Structure):
+    _fields_ = [("s", ctypes.c_void_p), ("coef", ctypes.c_void_p),
+                ("B", ctypes.c_int), ("D", ctypes.c_int), ("M", ctypes.c_int)]
+
+
+class _Launch(ctypes.Structure):
+    _fields_ = [("stream", ctypes.c_void_p), ("workspace", ctypes.c_void_p),
+                ("workspace_bytes", ctypes.c_size_t)]
+
+
+class RlmError(RuntimeError):
+    def __init__(self, status: int, where: str, detail: str):
+        super().__init__(f"{where}: {rlm_status_string(status)}: {detail}")
+        self.status = status
+
+
+_lib = None
+
+
+def library_path() -> str:
+    return _build_mod.LIB
+
+
+def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
+    """Load librlm.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build_mod.LIB
+    if not os.path.exists(path):
+        if not build_if_missing:
+            raise RuntimeError(
+                f"the CUDA library {path} is not built; run "
+                "`python -c 'import __graft_entry__ as g; g.build()'` first")
+        _build_mod.build()
+    lib = ctypes.CDLL(path)
+    P = ctypes.POINTER
+    lib.rlm_mix_prefill.argtypes = [P(_Tensor), P(_Params), P(_Tensor), P(_State), P(_Launch)]
+    lib.rlm_mix_decode.argtypes = [P(_Tensor), P(_State), P(_Tensor), P(_Launch)]
+    lib.rlm_mix_backward.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_Tensor),
+                                     P(_Grads), P(_Launch)]
+    lib.rlm_state_init.argtypes = [P(_State), P(_Params), P(_Launch)]
+    lib.rlm_validate_params.argtypes = [P(_Params)]
+    lib.rlm_get_device_status.argtypes = [P(_Launch)]
+    for f in ("rlm_prefill_workspace_size", "rlm_backward_workspace_size"):
+        getattr(lib, f).argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
+                                    ctypes.c_int, ctypes.c_int]
+        getattr(lib, f).restype = ctypes.c_size_t
+    for f in ("rlm_mix_prefill", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
+              "rlm_validate_params", "rlm_get_device_status"):
+        getattr(lib, f).restype = ctypes.c_int
+    lib.rlm_status_string.argtypes = [ctypes.c_int]
+    lib.rlm_status_string.restype = ctypes.c_char_p
+    lib.rlm_last_error.restype = ctypes.c_char_p
+    lib.rlm_version.restype = ctypes.c_int
+    _lib = lib
+    return lib
+
+
+# --------------------------------------------------------------- containers
+@dataclass
+class Params:
+    """Resonator parameters, each a float32 CUDA tensor [D][M]."""
+    decay: torch.Tensor
+    freq: torch.Tensor
+    amp: torch.Tensor
+    phase: torch.Tensor
+
+    @property
+    def D(self) -> int:
+        return int(self.decay.shape[0])
+
+    @property
+    def M(self) -> int:
+        return int(self.decay.shape[1])
+
+    @classmethod
+    def from_arrays(cls, decay, freq, amp, phase, device="cuda"):
+        t = lambda a: torch.as_tensor(a, dtype=torch.float32).contiguous().to(device)
+        return cls(t(decay), t(freq), t(amp), t(phase))
+
+    def _c(self) -> _Params:
+        return _Params(*(_ptr(t, torch.float32, 2) for t in
+                         (self.decay, self.freq, self.amp, self.phase)), self.D, self.M)
+
+
+@dataclass
+class Grads(Params):
+    """Parameter gradients, same layout as Params (overwritten by backward)."""
+
+    @classmethod
+    def empty(cls, D: int, M: int, device="cuda"):
+        return cls(*(torch.empty(D, M, dtype=torch.float32, device=device) for _ in range(4)))
+
+
+@dataclass
+class State:
+    """Recurrent state of Sec. 3.3: s [B][D][M][2] (Re, Im) and coef [D][M][4]."""
+    s: torch.Tensor
+    coef: torch.Tensor
+
+    @classmethod
+    def empty(cls, B: int, D: int, M: int, device="cuda"):
+        return cls(torch.empty(B, D, M, 2, dtype=torch.float32, device=device),
+                   torch.empty(D, M, 4, dtype=torch.float32, device=device))
+
+    @property
+    def shape(self):
+        B, D, M, _ = self.s.shape
+        return int(B), int(D), int(M)
+
+    def complex(self) -> torch.Tensor:
+        return torch.view_as_complex(self.s.contiguous())
+
+    def _c(self) -> _State:
+        B, D, M = self.shape
+        return _State(_ptr(self.s, torch.float32, 4), _ptr(self.coef, torch.float32, 3), B, D, M)
+
+
+# --------------------------------------------------------------- marshalling
+_DT = {torch.float32: RLM_F32, torch.bfloat16: RLM_BF16}
+
+
+def _ptr(t: torch.Tensor, dtype, ndim) -> int:
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("expected a torch.Tensor")
+    if t.dtype != dtype or t.dim() != ndim or not t.is_contiguous() or not t.is_cuda:
+        raise ValueError(f"expected a contiguous CUDA {dtype} tensor of rank {ndim}, got "
+                         f"{t.dtype} {tuple(t.shape)} on {t.device}")
+    return t.data_ptr()
+
+
+def _field(t: torch.Tensor) -> _Tensor:
+    if t.dtype not in _DT:
+        raise ValueError(f"unsupported dtype {t.dtype}")
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError("fields must be contiguous CUDA tensors")
+    if t.dim() == 3:
+        B, L, D = t.shape
+    elif t.dim() == 2:     # a single token per batch row: [B][D]
+        (B, D), L = t.shape, 1
+    else:
+        raise ValueError(f"fields are [B][L][D] (or [B][D] for one token), got {tuple(t.shape)}")
+    return _Tensor(t.data_ptr(), _DT[t.dtype], B, L, D)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _launch(stream, workspace) -> _Launch:
+    if workspace is None:
+        return _Launch(_stream(stream), None, 0)
+    return _Launch(_stream(stream), workspace.data_ptr(),
+                   workspace.numel() * workspace.element_size())
+
+
+def _check(status: int, where: str):
+    if status != RLM_OK:
+        raise RlmError(status, where, load_library().rlm_last_error().decode())
+
+
+def _workspace(nbytes: int, device) -> torch.Tensor | None:
+    if nbytes == 0:
+        return None
+    return torch.empty(nbytes, dtype=torch.uint8, device=device)
+
+
+# --------------------------------------------------------------- entry points
+def rlm_status_string(status: int) -> str:
+    return load_library().rlm_status_string(status).decode()
+
+
+def rlm_version() -> int:
+    return load_library().rlm_version()
+
+
+def rlm_prefill_workspace_size(B: int, L: int, D: int, M: int, dtype) -> int:
+    return load_library().rlm_prefill_workspace_size(B, L, D, M, _DT.get(dtype, dtype))
+
+
+def rlm_backward_workspace_size(B: int, L: int, D: int, M: int, dtype) -> int:
+    return load_library().rlm_backward_workspace_size(B, L, D, M, _DT.get(dtype, dtype))
+
+
+def rlm_mix_prefill(x: torch.Tensor, params: Params, y: torch.Tensor,
+                    state_out: State | None = None, workspace: torch.Tensor | None = None,
+                    stream=None) -> None:
+    """Causal mixing y = K * x (Eq. 2) from a zero state; optional terminal state.
+
+    ``workspace`` defaults to a fresh buffer of rlm_prefill_workspace_size bytes."""
+    lib = load_library()
+    xt, yt = _field(x), _field(y)
+    if workspace is None:
+        workspace = _workspace(lib.rlm_prefill_workspace_size(xt.B, xt.L, xt.D, params.M, xt.dtype),
+                               x.device)
+    st = state_out._c() if state_out is not None else None
+    _check(lib.rlm_mix_prefill(ctypes.byref(xt), ctypes.byref(params._c()), ctypes.byref(yt),
+                               ctypes.byref(st) if st is not None else None,
+                               ctypes.byref(_launch(stream, workspace))), "rlm_mix_prefill")
+
+
+def rlm_mix_decode(x_t: torch.Tensor, state: State, y_t: torch.Tensor, stream=None) -> None:
+    """One decode step (Eq. 4-5); the state is updated in place."""
+    lib = load_library()
+    xt, yt = _field(x_t), _field(y_t)
+    _check(lib.rlm_mix_decode(ctypes.byref(xt), ctypes.byref(state._c()), ctypes.byref(yt),
+                              ctypes.byref(_launch(stream, None))), "rlm_mix_decode")
+
+
+def rlm_state_init(state: State, params: Params, stream=None) -> None:
+    lib = load_library()
+    _check(lib.rlm_state_init(ctypes.byref(state._c()), ctypes.byref(params._c()),
+                              ctypes.byref(_launch(stream, None))), "rlm_state_init")
+
+
+def rlm_mix_backward(dy: torch.Tensor, x: torch.Tensor, params: Params, dx: torch.Tensor,
+                     dparams: Grads, workspace: torch.Tensor | None = None, stream=None) -> None:
+    """dx and the four parameter gradients of l given dy = dl/dy."""
+    lib = load_library()
+    dyt, xt, dxt = _field(dy), _field(x), _field(dx)
+    if workspace is None:
+        workspace = _workspace(lib.rlm_backward_workspace_size(xt.B, xt.L, xt.D, params.M,
+                                                               xt.dtype), x.device)
+    _check(lib.rlm_mix_backward(ctypes.byref(dyt), ctypes.byref(xt), ctypes.byref(params._c()),
+                                ctypes.byref(dxt), ctypes.byref(dparams._c()),
+                                ctypes.byref(_launch(stream, workspace))), "rlm_mix_backward")
+
+
+def rlm_validate_params(params: Params) -> None:
+    _check(load_library().rlm_validate_params(ctypes.byref(params._c())), "rlm_validate_params")
+
+
+def rlm_get_device_status(stream=None) -> int:
+    """Synchronise the stream and return (and clear) the device status word."""
+    return load_library().rlm_get_device_status(ctypes.byref(_launch(stream, None)))

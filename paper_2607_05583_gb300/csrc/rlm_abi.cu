@@ -1,0 +1,298 @@
+// rlm_abi.cu -- the extern "C" boundary: host-side argument checks, workspace
+// sizing and dispatch to the kernels.  Nothing here allocates device memory.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "rlm_internal.h"
+
+namespace rlm {
+
+static thread_local char g_err[512] = "";
+
+void set_error(const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+}
+
+int sm_count() {
+    static std::mutex mu;
+    static std::vector<int> cache;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+    std::lock_guard<std::mutex> lock(mu);
+    if ((int)cache.size() <= dev) cache.resize(dev + 1, 0);
+    if (cache[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            n = 148;
+        cache[dev] = n;
+    }
+    return cache[dev];
+}
+
+}  // namespace rlm
+
+using namespace rlm;
+
+namespace {
+
+constexpr int kMaxModes = 64;
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+size_t elem_size(rlm_dtype dt) { return dt == RLM_BF16 ? 2 : 4; }
+
+rlm_status fail(rlm_status s, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    set_error("%s", buf);
+    return s;
+}
+
+rlm_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(RLM_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+rlm_status check_tensor(const rlm_tensor *t, const char *name) {
+    if (!t) return fail(RLM_ERR_INVALID_ARG, "%s is NULL", name);
+    if (!t->ptr) return fail(RLM_ERR_INVALID_ARG, "%s->ptr is NULL", name);
+    if (!aligned16(t->ptr)) return fail(RLM_ERR_INVALID_ARG, "%s->ptr is not 16-byte aligned", name);
+    if (t->dtype != RLM_F32 && t->dtype != RLM_BF16)
+        return fail(RLM_ERR_INVALID_ARG, "%s->dtype %d is not RLM_F32 or RLM_BF16", name, (int)t->dtype);
+    if (t->B < 1 || t->L < 1)
+        return fail(RLM_ERR_INVALID_ARG, "%s has B=%lld L=%lld (need >= 1)", name, (long long)t->B,
+                    (long long)t->L);
+    if (t->D < 8 || t->D % 8 != 0)
+        return fail(RLM_ERR_INVALID_ARG, "%s has D=%lld (need D >= 8 and D %% 8 == 0)", name,
+                    (long long)t->D);
+    if (t->D > (1 << 20)) return fail(RLM_ERR_UNSUPPORTED, "%s has D=%lld > 2^20", name, (long long)t->D);
+    if (t->B > 65535) return fail(RLM_ERR_UNSUPPORTED, "%s has B=%lld > 65535", name, (long long)t->B);
+    if (t->L > (int64_t)1 << 30)
+        return fail(RLM_ERR_UNSUPPORTED, "%s has L=%lld > 2^30", name, (long long)t->L);
+    return RLM_OK;
+}
+
+bool same_shape(const rlm_tensor *a, const rlm_tensor *b) {
+    return a->B == b->B && a->L == b->L && a->D == b->D && a->dtype == b->dtype;
+}
+
+size_t tensor_bytes(const rlm_tensor *t) {
+    return (size_t)t->B * (size_t)t->L * (size_t)t->D * elem_size(t->dtype);
+}
+
+bool overlap(const void *a, size_t na, const void *b, size_t nb) {
+    const char *pa = static_cast<const char *>(a), *pb = static_cast<const char *>(b);
+    return pa < pb + nb && pb < pa + na;
+}
+
+rlm_status check_params(const rlm_params *p, int64_t D) {
+    if (!p) return fail(RLM_ERR_INVALID_ARG, "params is NULL");
+    const float *ps[4] = {p->decay, p->freq, p->amp, p->phase};
+    const char *nm[4] = {"decay", "freq", "amp", "phase"};
+    for (int i = 0; i < 4; ++i) {
+        if (!ps[i]) return fail(RLM_ERR_INVALID_ARG, "params->%s is NULL", nm[i]);
+        if (!aligned16(ps[i])) return fail(RLM_ERR_INVALID_ARG, "params->%s is not 16-byte aligned", nm[i]);
+    }
+    if (p->M < 1 || p->M > kMaxModes)
+        return fail(RLM_ERR_INVALID_ARG, "params->M=%d outside 1..%d", p->M, kMaxModes);
+    if (p->D != D) return fail(RLM_ERR_INVALID_ARG, "params->D=%d does not match D=%lld", p->D, (long long)D);
+    return RLM_OK;
+}
+
+rlm_status check_state(const rlm_state *s, int64_t B, int64_t D, int M, const char *name) {
+    if (!s->s || !s->coef) return fail(RLM_ERR_INVALID_ARG, "%s has a NULL s or coef", name);
+    if (!aligned16(s->s) || !aligned16(s->coef))
+        return fail(RLM_ERR_INVALID_ARG, "%s buffers are not 16-byte aligned", name);
+    if (s->B != B || s->D != D || s->M != M)
+        return fail(RLM_ERR_INVALID_ARG, "%s is [B=%d][D=%d][M=%d], expected [%lld][%lld][%d]", name,
+                    s->B, s->D, s->M, (long long)B, (long long)D, M);
+    return RLM_OK;
+}
+
+rlm_status check_workspace(const rlm_launch *ln, size_t need) {
+    if (!ln) return fail(RLM_ERR_INVALID_ARG, "launch is NULL");
+    if (need == 0) return RLM_OK;
+    if (!ln->workspace) return fail(RLM_ERR_INVALID_ARG, "workspace is NULL but %zu bytes are needed", need);
+    if ((reinterpret_cast<uintptr_t>(ln->workspace) & 255u) != 0)
+        return fail(RLM_ERR_INVALID_ARG, "workspace is not 256-byte aligned");
+    if (ln->workspace_bytes < need)
+        return fail(RLM_ERR_INVALID_ARG, "workspace has %zu bytes, %zu needed", ln->workspace_bytes, need);
+    return RLM_OK;
+}
+
+int simt_chunks(int64_t B, int64_t L, int D) {
+    const int C = simt_chunk_len(B, L, D);
+    return (int)((L + C - 1) / C);
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *rlm_status_string(rlm_status s) {
+    switch (s) {
+        case RLM_OK: return "RLM_OK";
+        case RLM_ERR_INVALID_ARG: return "RLM_ERR_INVALID_ARG";
+        case RLM_ERR_UNSUPPORTED: return "RLM_ERR_UNSUPPORTED";
+        case RLM_ERR_CUDA: return "RLM_ERR_CUDA";
+        case RLM_ERR_TIMEOUT: return "RLM_ERR_TIMEOUT";
+    }
+    return "RLM_STATUS_UNKNOWN";
+}
+
+const char *rlm_last_error(void) { return g_err; }
+
+int rlm_version(void) { return 100; }
+
+size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
+    if (B < 1 || L < 1 || D < 1 || M < 1) return 0;
+    if (tc_prefill_supported(B, L, D, M, dtype)) return tc_prefill_ws_bytes(B, L, D, M);
+    return simt_prefill_ws_bytes(B, L, D, M);
+}
+
+size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
+    (void)dtype;
+    if (B < 1 || L < 1 || D < 1 || M < 1) return 0;
+    return simt_backward_ws_bytes(B, L, D, M);
+}
+
+rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor *y,
+                           rlm_state *state_out, const rlm_launch *ln) {
+    rlm_status s;
+    if ((s = check_tensor(x, "x")) != RLM_OK) return s;
+    if ((s = check_tensor(y, "y")) != RLM_OK) return s;
+    if (!same_shape(x, y)) return fail(RLM_ERR_INVALID_ARG, "y must have x's shape and dtype");
+    if (overlap(x->ptr, tensor_bytes(x), y->ptr, tensor_bytes(y)))
+        return fail(RLM_ERR_INVALID_ARG, "x and y overlap");
+    if ((s = check_params(p, x->D)) != RLM_OK) return s;
+    if (state_out && (s = check_state(state_out, x->B, x->D, p->M, "state_out")) != RLM_OK) return s;
+    const int D = (int)x->D, M = p->M;
+    const bool tc = tc_prefill_supported(x->B, x->L, D, M, x->dtype);
+    if (!tc && simt_chunks(x->B, x->L, D) > 65535)
+        return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
+    const size_t need = rlm_prefill_workspace_size(x->B, x->L, D, M, x->dtype);
+    if ((s = check_workspace(ln, need)) != RLM_OK) return s;
+    cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
+    float *so = state_out ? state_out->s : nullptr;
+    float *co = state_out ? state_out->coef : nullptr;
+    cudaError_t e;
+    if (tc)
+        e = tc_prefill(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, so,
+                       co, ln->workspace, st);
+    else
+        e = simt_prefill(x->ptr, y->ptr, x->dtype, x->B, x->L, D, M, p->decay, p->freq, p->amp,
+                         p->phase, so, co, ln->workspace, st);
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_prefill launch");
+    return RLM_OK;
+}
+
+rlm_status rlm_mix_decode(const rlm_tensor *x_t, rlm_state *state, rlm_tensor *y_t,
+                          const rlm_launch *ln) {
+    rlm_status s;
+    if ((s = check_tensor(x_t, "x_t")) != RLM_OK) return s;
+    if ((s = check_tensor(y_t, "y_t")) != RLM_OK) return s;
+    if (x_t->L != 1) return fail(RLM_ERR_INVALID_ARG, "x_t must have L == 1 (got %lld)", (long long)x_t->L);
+    if (!same_shape(x_t, y_t)) return fail(RLM_ERR_INVALID_ARG, "y_t must have x_t's shape and dtype");
+    if (overlap(x_t->ptr, tensor_bytes(x_t), y_t->ptr, tensor_bytes(y_t)))
+        return fail(RLM_ERR_INVALID_ARG, "x_t and y_t overlap");
+    if (!state) return fail(RLM_ERR_INVALID_ARG, "state is NULL");
+    if (state->M < 1 || state->M > kMaxModes)
+        return fail(RLM_ERR_INVALID_ARG, "state->M=%d outside 1..%d", state->M, kMaxModes);
+    if ((s = check_state(state, x_t->B, x_t->D, state->M, "state")) != RLM_OK) return s;
+    if (!ln) return fail(RLM_ERR_INVALID_ARG, "launch is NULL");
+    const size_t sbytes = (size_t)state->B * state->D * state->M * 8;
+    if (overlap(state->s, sbytes, y_t->ptr, tensor_bytes(y_t)) ||
+        overlap(state->s, sbytes, x_t->ptr, tensor_bytes(x_t)))
+        return fail(RLM_ERR_INVALID_ARG, "state overlaps x_t or y_t");
+    cudaError_t e = decode_step(x_t->ptr, y_t->ptr, x_t->dtype, (int)x_t->B, (int)x_t->D, state->M,
+                                state->s, state->coef, static_cast<cudaStream_t>(ln->stream));
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_decode launch");
+    return RLM_OK;
+}
+
+rlm_status rlm_state_init(rlm_state *state, const rlm_params *p, const rlm_launch *ln) {
+    rlm_status s;
+    if (!state) return fail(RLM_ERR_INVALID_ARG, "state is NULL");
+    if ((s = check_params(p, state->D)) != RLM_OK) return s;
+    if (state->B < 1 || state->D < 1) return fail(RLM_ERR_INVALID_ARG, "state has B or D < 1");
+    if ((s = check_state(state, state->B, state->D, p->M, "state")) != RLM_OK) return s;
+    if (!ln) return fail(RLM_ERR_INVALID_ARG, "launch is NULL");
+    cudaError_t e = state_init(state->s, state->coef, state->B, state->D, state->M, p->decay, p->freq,
+                               p->amp, p->phase, static_cast<cudaStream_t>(ln->stream));
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_state_init launch");
+    return RLM_OK;
+}
+
+rlm_status rlm_mix_backward(const rlm_tensor *dy, const rlm_tensor *x, const rlm_params *p,
+                            rlm_tensor *dx, rlm_grads *g, const rlm_launch *ln) {
+    rlm_status s;
+    if ((s = check_tensor(dy, "dy")) != RLM_OK) return s;
+    if ((s = check_tensor(x, "x")) != RLM_OK) return s;
+    if ((s = check_tensor(dx, "dx")) != RLM_OK) return s;
+    if (!same_shape(dy, x) || !same_shape(dx, x))
+        return fail(RLM_ERR_INVALID_ARG, "dy, x and dx must share shape and dtype");
+    if (overlap(dx->ptr, tensor_bytes(dx), x->ptr, tensor_bytes(x)) ||
+        overlap(dx->ptr, tensor_bytes(dx), dy->ptr, tensor_bytes(dy)))
+        return fail(RLM_ERR_INVALID_ARG, "dx overlaps x or dy");
+    if ((s = check_params(p, x->D)) != RLM_OK) return s;
+    if (!g) return fail(RLM_ERR_INVALID_ARG, "dparams is NULL");
+    float *gs[4] = {g->decay, g->freq, g->amp, g->phase};
+    for (int i = 0; i < 4; ++i)
+        if (!gs[i] || !aligned16(gs[i]))
+            return fail(RLM_ERR_INVALID_ARG, "dparams pointer %d is NULL or not 16-byte aligned", i);
+    if (g->D != p->D || g->M != p->M) return fail(RLM_ERR_INVALID_ARG, "dparams shape differs from params");
+    const int D = (int)x->D, M = p->M;
+    if (simt_chunks(x->B, x->L, D) > 65535)
+        return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
+    const size_t need = rlm_backward_workspace_size(x->B, x->L, D, M, x->dtype);
+    if ((s = check_workspace(ln, need)) != RLM_OK) return s;
+    cudaError_t e = simt_backward(dy->ptr, x->ptr, dx->ptr, x->dtype, x->B, x->L, D, M, p->decay,
+                                  p->freq, p->amp, p->phase, g->decay, g->freq, g->amp, g->phase,
+                                  ln->workspace, static_cast<cudaStream_t>(ln->stream));
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_backward launch");
+    return RLM_OK;
+}
+
+rlm_status rlm_validate_params(const rlm_params *p) {
+    if (!p) return fail(RLM_ERR_INVALID_ARG, "params is NULL");
+    rlm_status s;
+    if ((s = check_params(p, p->D)) != RLM_OK) return s;
+    if (p->D < 1) return fail(RLM_ERR_INVALID_ARG, "params->D < 1");
+    const size_t n = (size_t)p->D * p->M;
+    std::vector<float> h(n);
+    const float *ps[4] = {p->decay, p->freq, p->amp, p->phase};
+    const char *nm[4] = {"decay", "freq", "amp", "phase"};
+    for (int i = 0; i < 4; ++i) {
+        cudaError_t e = cudaMemcpy(h.data(), ps[i], n * sizeof(float), cudaMemcpyDeviceToHost);
+        if (e != cudaSuccess) return cuda_fail(e, "rlm_validate_params copy");
+        for (size_t k = 0; k < n; ++k) {
+            if (!std::isfinite(h[k]))
+                return fail(RLM_ERR_INVALID_ARG, "params->%s[%zu] is not finite", nm[i], k);
+            if (i == 0 && h[k] < 0.0f)
+                return fail(RLM_ERR_INVALID_ARG, "params->decay[%zu] = %g < 0", k, (double)h[k]);
+        }
+    }
+    return RLM_OK;
+}
+
+rlm_status rlm_get_device_status(const rlm_launch *ln) {
+    if (!ln) return fail(RLM_ERR_INVALID_ARG, "launch is NULL");
+    int status = RLM_OK;
+    cudaError_t e = read_and_clear_device_status(&status, static_cast<cudaStream_t>(ln->stream));
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_get_device_status");
+    if (status != RLM_OK) return fail((rlm_status)status, "a bounded device-side wait expired");
+    return RLM_OK;
+}
+
+}  // extern "C"

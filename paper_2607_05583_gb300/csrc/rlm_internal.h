@@ -1,0 +1,58 @@
+// rlm_internal.h -- declarations shared by the library's translation units.
+// Host-side only; device helpers live in rlm_device.cuh.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/rlm.h"
+
+namespace rlm {
+
+// Records a human-readable reason for the next rlm_last_error() on this thread.
+void set_error(const char *fmt, ...);
+
+// Multiprocessor count of the current device (cached per device).
+int sm_count();
+
+// ---- SIMT chunked scan (rlm_simt.cu) --------------------------------------
+// Chunk length the SIMT path uses for a problem; workspace and launch agree.
+int simt_chunk_len(int64_t B, int64_t L, int D);
+size_t simt_prefill_ws_bytes(int64_t B, int64_t L, int D, int M);
+size_t simt_backward_ws_bytes(int64_t B, int64_t L, int D, int M);
+
+// y = causal mixing of x (reverse=false) or the anti-causal mixing used by the
+// backward pass for dx (reverse=true: time runs from L-1 down to 0).
+// state_out/coef_out may be null.  ws must hold simt_prefill_ws_bytes().
+cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_t L, int D,
+                         int M, const float *decay, const float *freq, const float *amp,
+                         const float *phase, float *state_out, float *coef_out, void *ws,
+                         cudaStream_t st);
+
+// dx and the four parameter gradients (deterministic reduction).
+cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt, int64_t B,
+                          int64_t L, int D, int M, const float *decay, const float *freq,
+                          const float *amp, const float *phase, float *g_decay,
+                          float *g_freq, float *g_amp, float *g_phase, void *ws,
+                          cudaStream_t st);
+
+// ---- decode (rlm_decode.cu) -----------------------------------------------
+cudaError_t decode_step(const void *x_t, void *y_t, rlm_dtype dt, int B, int D, int M,
+                        float *s, const float *coef, cudaStream_t st);
+cudaError_t state_init(float *s, float *coef, int B, int D, int M, const float *decay,
+                       const float *freq, const float *amp, const float *phase,
+                       cudaStream_t st);
+
+// ---- tcgen05 prefill (rlm_prefill_tc.cu) ------------------------------------
+// True when the tensor-core path covers this problem.
+bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
+size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int M);
+cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int M,
+                       const float *decay, const float *freq, const float *amp,
+                       const float *phase, float *state_out, float *coef_out, void *ws,
+                       cudaStream_t st);
+// Device status word written by bounded waits (RLM_OK or RLM_ERR_TIMEOUT).
+cudaError_t read_and_clear_device_status(int *status, cudaStream_t st);
+
+}  // namespace rlm

@@ -1,0 +1,348 @@
+// rlm_simt.cu -- chunked complex-diagonal scan on the CUDA cores (fp32).
+//
+// Runs the fp32-I/O prefill, every shape the tensor-core path does not cover,
+// and the backward pass.  Three phases, each one launch:
+//
+//  1. chunk-local states: per (b, chunk k, d) and mode m, the state the chunk's
+//     own drives leave at its last token when it starts from zero
+//     (sum_j lambda^(C-1-j) x_j, the chunk form of the terminal state of
+//     Sec. 3.2);
+//  2. inter-chunk carry: per (b, d, m), a sequential scan over chunks,
+//     S_k = lambda^C S_{k-1} + local_k, written back exclusive (the state each
+//     chunk starts from) -- the final S is the prompt's terminal state;
+//  3. chunk output: per (b, k, d), the recurrence of Eq. 4 restarted from the
+//     carried state, with the readout y_t = sum_m Re(c s_t).
+//
+// Chunks are aligned to END at the last token: the first chunk may start at a
+// negative time, whose drives count as zero.  With a zero initial state that
+// leaves every state unchanged, so the carry needs no special last chunk.
+//
+// The backward pass runs the same phases in reverse time on dy (the adjoint of
+// a causal convolution is the anti-causal one) and carries the Jordan partner
+// R of the adjoint state as well, to form G = sum x S and P = sum x R.
+#include <algorithm>
+
+#include "rlm_device.cuh"
+#include "rlm_internal.h"
+
+namespace rlm {
+namespace {
+
+constexpr int kMgFwd = 16;  // modes per thread, forward phases
+constexpr int kMgBwd = 8;   // modes per thread, backward output phase
+constexpr int kBlock = 128;
+
+int threads_per_channel(int M, int mg) {
+    int t = (M + mg - 1) / mg;
+    int p = 1;
+    while (p < t) p <<= 1;
+    return p;
+}
+
+struct ChunkGeom {
+    int C;        // chunk length
+    int nch;      // number of chunks
+    int64_t t0;   // processing time of chunk 0's first token (<= 0)
+};
+
+ChunkGeom geom(int64_t B, int64_t L, int D) {
+    ChunkGeom g;
+    g.C = simt_chunk_len(B, L, D);
+    g.nch = (int)((L + g.C - 1) / g.C);
+    g.t0 = L - (int64_t)g.nch * g.C;
+    return g;
+}
+
+// Phase 1.  Grid (ceil(D*TPC/kBlock), nch, B).
+template <typename T, int MG, bool REV, bool JORDAN>
+__global__ void __launch_bounds__(kBlock) k_chunk_local(
+    const T *__restrict__ x, int64_t L, int D, int M, int tpc, int C, int nch, int64_t t0,
+    const float *__restrict__ decay, const float *__restrict__ freq, float2 *__restrict__ ws_s,
+    float2 *__restrict__ ws_r) {
+    const int gx = blockIdx.x * blockDim.x + threadIdx.x;
+    const int d = gx / tpc, grp = gx % tpc;
+    const int k = blockIdx.y, b = blockIdx.z;
+    if (d >= D) return;
+    float2 lam[MG], s[MG], r[MG];
+#pragma unroll
+    for (int j = 0; j < MG; ++j) {
+        const int m = grp * MG + j;
+        lam[j] = m < M ? lambda_pow(decay[d * M + m], freq[d * M + m], 1.0f) : make_float2(0, 0);
+        s[j] = make_float2(0, 0);
+        r[j] = make_float2(0, 0);
+    }
+    const int64_t tau0 = t0 + (int64_t)k * C;
+    const int i0 = tau0 < 0 ? (int)(-tau0) : 0;
+    for (int i = i0; i < C; ++i) {
+        const int64_t tau = tau0 + i;
+        const int64_t t = REV ? (L - 1 - tau) : tau;
+        const float xv = ld_elem(x + ((int64_t)b * L + t) * D + d);
+#pragma unroll
+        for (int j = 0; j < MG; ++j) {
+            if (JORDAN) r[j] = cmul(lam[j], make_float2(r[j].x + s[j].x, r[j].y + s[j].y));
+            s[j] = cfma(lam[j], s[j], make_float2(xv, 0.0f));
+        }
+    }
+    const int64_t base = (((int64_t)b * nch + k) * D + d) * M;
+#pragma unroll
+    for (int j = 0; j < MG; ++j) {
+        const int m = grp * MG + j;
+        if (m < M) {
+            ws_s[base + m] = s[j];
+            if (JORDAN) ws_r[base + m] = r[j];
+        }
+    }
+}
+
+// Phase 2.  One thread per (b, d, m); grid over B*D*M.
+template <bool JORDAN>
+__global__ void __launch_bounds__(256) k_chunk_carry(
+    int64_t B, int D, int M, int C, int nch, const float *__restrict__ decay,
+    const float *__restrict__ freq, const float *__restrict__ amp, const float *__restrict__ phase,
+    float2 *__restrict__ ws_s, float2 *__restrict__ ws_r, float2 *__restrict__ state_out,
+    float4 *__restrict__ coef_out) {
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= B * D * M) return;
+    const int m = (int)(idx % M);
+    const int d = (int)((idx / M) % D);
+    const int64_t b = idx / ((int64_t)M * D);
+    const int pm = d * M + m;
+    const float2 LC = lambda_pow(decay[pm], freq[pm], (float)C);
+    const float Cf = (float)C;
+    float2 S = make_float2(0, 0), R = make_float2(0, 0);
+    for (int k = 0; k < nch; ++k) {
+        const int64_t off = ((b * nch + k) * D + d) * M + m;
+        const float2 ls = ws_s[off];
+        ws_s[off] = S;
+        if (JORDAN) {
+            const float2 lr = ws_r[off];
+            ws_r[off] = R;
+            R = cfma(LC, make_float2(fmaf(Cf, S.x, R.x), fmaf(Cf, S.y, R.y)), lr);
+        }
+        S = cfma(LC, S, ls);
+    }
+    if (state_out) state_out[idx] = S;
+    if (coef_out && b == 0) {
+        const float2 lam = lambda_pow(decay[pm], freq[pm], 1.0f);
+        const float2 c = mode_coef(amp[pm], phase[pm]);
+        coef_out[pm] = make_float4(lam.x, lam.y, c.x, c.y);
+    }
+}
+
+// Phase 3 (forward).  Grid (ceil(D*TPC/kBlock), nch, B); the TPC threads of a
+// channel split its modes and add their readouts with shuffles.
+template <typename T, int MG, bool REV>
+__global__ void __launch_bounds__(kBlock) k_chunk_output(
+    const T *__restrict__ x, T *__restrict__ y, int64_t L, int D, int M, int tpc, int C, int nch,
+    int64_t t0, const float *__restrict__ decay, const float *__restrict__ freq,
+    const float *__restrict__ amp, const float *__restrict__ phase,
+    const float2 *__restrict__ ws_s) {
+    const int gx = blockIdx.x * blockDim.x + threadIdx.x;
+    const int d = gx / tpc, grp = gx % tpc;
+    const int k = blockIdx.y, b = blockIdx.z;
+    const bool active = d < D;
+    float2 lam[MG], c[MG], s[MG];
+    const int64_t base = (((int64_t)b * nch + k) * D + d) * M;
+#pragma unroll
+    for (int j = 0; j < MG; ++j) {
+        const int m = grp * MG + j;
+        const bool on = active && m < M;
+        lam[j] = on ? lambda_pow(decay[d * M + m], freq[d * M + m], 1.0f) : make_float2(0, 0);
+        c[j] = on ? mode_coef(amp[d * M + m], phase[d * M + m]) : make_float2(0, 0);
+        s[j] = on ? ws_s[base + m] : make_float2(0, 0);
+    }
+    const int64_t tau0 = t0 + (int64_t)k * C;
+    const int i0 = tau0 < 0 ? (int)(-tau0) : 0;
+    for (int i = i0; i < C; ++i) {
+        const int64_t tau = tau0 + i;
+        const int64_t t = REV ? (L - 1 - tau) : tau;
+        const int64_t e = ((int64_t)b * L + t) * D + d;
+        const float xv = active ? ld_elem(x + e) : 0.0f;
+        float acc = 0.0f;
+#pragma unroll
+        for (int j = 0; j < MG; ++j) {
+            s[j] = cfma(lam[j], s[j], make_float2(xv, 0.0f));
+            acc = fmaf(c[j].x, s[j].x, fmaf(-c[j].y, s[j].y, acc));
+        }
+        for (int o = tpc >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (active && grp == 0) st_elem(y + e, acc);
+    }
+}
+
+// Phase 3 (backward).  Reverse time over dy; writes dx and, in place of the
+// carried (S, R), the chunk's partial sums G = sum x S and P = sum x R.
+template <typename T, int MG>
+__global__ void __launch_bounds__(kBlock) k_chunk_backward(
+    const T *__restrict__ dy, const T *__restrict__ x, T *__restrict__ dx, int64_t L, int D,
+    int M, int tpc, int C, int nch, int64_t t0, const float *__restrict__ decay,
+    const float *__restrict__ freq, const float *__restrict__ amp,
+    const float *__restrict__ phase, float2 *__restrict__ ws_s, float2 *__restrict__ ws_r) {
+    const int gx = blockIdx.x * blockDim.x + threadIdx.x;
+    const int d = gx / tpc, grp = gx % tpc;
+    const int k = blockIdx.y, b = blockIdx.z;
+    const bool active = d < D;
+    float2 lam[MG], c[MG], s[MG], r[MG], G[MG], P[MG];
+    const int64_t base = (((int64_t)b * nch + k) * D + d) * M;
+#pragma unroll
+    for (int j = 0; j < MG; ++j) {
+        const int m = grp * MG + j;
+        const bool on = active && m < M;
+        lam[j] = on ? lambda_pow(decay[d * M + m], freq[d * M + m], 1.0f) : make_float2(0, 0);
+        c[j] = on ? mode_coef(amp[d * M + m], phase[d * M + m]) : make_float2(0, 0);
+        s[j] = on ? ws_s[base + m] : make_float2(0, 0);
+        r[j] = on ? ws_r[base + m] : make_float2(0, 0);
+        G[j] = make_float2(0, 0);
+        P[j] = make_float2(0, 0);
+    }
+    const int64_t tau0 = t0 + (int64_t)k * C;
+    const int i0 = tau0 < 0 ? (int)(-tau0) : 0;
+    for (int i = i0; i < C; ++i) {
+        const int64_t t = L - 1 - (tau0 + i);
+        const int64_t e = ((int64_t)b * L + t) * D + d;
+        const float u = active ? ld_elem(dy + e) : 0.0f;
+        const float xv = active ? ld_elem(x + e) : 0.0f;
+        float acc = 0.0f;
+#pragma unroll
+        for (int j = 0; j < MG; ++j) {
+            r[j] = cmul(lam[j], make_float2(r[j].x + s[j].x, r[j].y + s[j].y));
+            s[j] = cfma(lam[j], s[j], make_float2(u, 0.0f));
+            acc = fmaf(c[j].x, s[j].x, fmaf(-c[j].y, s[j].y, acc));
+            G[j].x = fmaf(xv, s[j].x, G[j].x);
+            G[j].y = fmaf(xv, s[j].y, G[j].y);
+            P[j].x = fmaf(xv, r[j].x, P[j].x);
+            P[j].y = fmaf(xv, r[j].y, P[j].y);
+        }
+        for (int o = tpc >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (active && grp == 0) st_elem(dx + e, acc);
+    }
+#pragma unroll
+    for (int j = 0; j < MG; ++j) {
+        const int m = grp * MG + j;
+        if (active && m < M) {
+            ws_s[base + m] = G[j];
+            ws_r[base + m] = P[j];
+        }
+    }
+}
+
+// Phase 4 (backward).  One thread per (d, m): fixed-order sum of the partials
+// over (b, k) in double, then the four gradients.
+__global__ void __launch_bounds__(256) k_grad_reduce(
+    int64_t B, int D, int M, int nch, const float *__restrict__ amp,
+    const float *__restrict__ phase, const float2 *__restrict__ ws_s,
+    const float2 *__restrict__ ws_r, float *__restrict__ g_decay, float *__restrict__ g_freq,
+    float *__restrict__ g_amp, float *__restrict__ g_phase) {
+    const int pm = blockIdx.x * blockDim.x + threadIdx.x;
+    if (pm >= D * M) return;
+    double gr = 0, gi = 0, pr = 0, pi = 0;
+    for (int64_t bk = 0; bk < B * nch; ++bk) {
+        const int64_t off = bk * D * M + pm;
+        const float2 g = ws_s[off], p = ws_r[off];
+        gr += g.x;
+        gi += g.y;
+        pr += p.x;
+        pi += p.y;
+    }
+    double sph, cph;
+    sincos((double)phase[pm], &sph, &cph);
+    const double a = amp[pm];
+    const double cr = a * cph, ci = a * sph;
+    g_amp[pm] = (float)(cph * gr - sph * gi);         // Re(e^{i phi} G)
+    g_phase[pm] = (float)(-(cr * gi + ci * gr));      // -Im(c G)
+    g_decay[pm] = (float)(-(cr * pr - ci * pi));      // -Re(c P)
+    g_freq[pm] = (float)(-(cr * pi + ci * pr));       // -Im(c P)
+}
+
+template <typename T>
+cudaError_t prefill_t(const T *x, T *y, int64_t B, int64_t L, int D, int M, const float *decay,
+                      const float *freq, const float *amp, const float *phase, float *state_out,
+                      float *coef_out, void *ws, cudaStream_t st) {
+    const ChunkGeom g = geom(B, L, D);
+    const int tpc = threads_per_channel(M, kMgFwd);
+    float2 *ws_s = reinterpret_cast<float2 *>(ws);
+    dim3 grid((unsigned)((D * tpc + kBlock - 1) / kBlock), (unsigned)g.nch, (unsigned)B);
+    k_chunk_local<T, kMgFwd, false, false><<<grid, kBlock, 0, st>>>(
+        x, L, D, M, tpc, g.C, g.nch, g.t0, decay, freq, ws_s, nullptr);
+    const int64_t n = B * D * M;
+    k_chunk_carry<false><<<(unsigned)((n + 255) / 256), 256, 0, st>>>(
+        B, D, M, g.C, g.nch, decay, freq, amp, phase, ws_s, nullptr,
+        reinterpret_cast<float2 *>(state_out), reinterpret_cast<float4 *>(coef_out));
+    k_chunk_output<T, kMgFwd, false><<<grid, kBlock, 0, st>>>(
+        x, y, L, D, M, tpc, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s);
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t backward_t(const T *dy, const T *x, T *dx, int64_t B, int64_t L, int D, int M,
+                       const float *decay, const float *freq, const float *amp,
+                       const float *phase, float *gd, float *gf, float *ga, float *gp, void *ws,
+                       cudaStream_t st) {
+    const ChunkGeom g = geom(B, L, D);
+    const int64_t n = B * (int64_t)g.nch * D * M;
+    float2 *ws_s = reinterpret_cast<float2 *>(ws);
+    float2 *ws_r = ws_s + n;
+    const int tpc1 = threads_per_channel(M, kMgFwd);
+    dim3 grid1((unsigned)((D * tpc1 + kBlock - 1) / kBlock), (unsigned)g.nch, (unsigned)B);
+    k_chunk_local<T, kMgFwd, true, true><<<grid1, kBlock, 0, st>>>(
+        dy, L, D, M, tpc1, g.C, g.nch, g.t0, decay, freq, ws_s, ws_r);
+    const int64_t nbdm = B * D * M;
+    k_chunk_carry<true><<<(unsigned)((nbdm + 255) / 256), 256, 0, st>>>(
+        B, D, M, g.C, g.nch, decay, freq, amp, phase, ws_s, ws_r, nullptr, nullptr);
+    const int tpc3 = threads_per_channel(M, kMgBwd);
+    dim3 grid3((unsigned)((D * tpc3 + kBlock - 1) / kBlock), (unsigned)g.nch, (unsigned)B);
+    k_chunk_backward<T, kMgBwd><<<grid3, kBlock, 0, st>>>(
+        dy, x, dx, L, D, M, tpc3, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, ws_r);
+    k_grad_reduce<<<(unsigned)((D * M + 255) / 256), 256, 0, st>>>(
+        B, D, M, g.nch, amp, phase, ws_s, ws_r, gd, gf, ga, gp);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+int simt_chunk_len(int64_t B, int64_t L, int D) {
+    // Enough (b, chunk, channel) threads for about two full waves of 1024
+    // resident threads per SM; chunks of 16..1024 tokens.
+    const int64_t target = (int64_t)sm_count() * 2048;
+    const int64_t per_chunk = std::max<int64_t>(1, B * (int64_t)D);
+    int64_t nch = (target + per_chunk - 1) / per_chunk;
+    nch = std::max<int64_t>(1, nch);
+    int64_t C = (L + nch - 1) / nch;
+    C = std::max<int64_t>(16, std::min<int64_t>(1024, C));
+    return (int)C;
+}
+
+size_t simt_prefill_ws_bytes(int64_t B, int64_t L, int D, int M) {
+    const ChunkGeom g = geom(B, L, D);
+    return (size_t)B * g.nch * D * M * sizeof(float2);
+}
+
+size_t simt_backward_ws_bytes(int64_t B, int64_t L, int D, int M) {
+    return 2 * simt_prefill_ws_bytes(B, L, D, M);
+}
+
+cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_t L, int D,
+                         int M, const float *decay, const float *freq, const float *amp,
+                         const float *phase, float *state_out, float *coef_out, void *ws,
+                         cudaStream_t st) {
+    if (dt == RLM_BF16)
+        return prefill_t(static_cast<const __nv_bfloat16 *>(x), static_cast<__nv_bfloat16 *>(y),
+                         B, L, D, M, decay, freq, amp, phase, state_out, coef_out, ws, st);
+    return prefill_t(static_cast<const float *>(x), static_cast<float *>(y), B, L, D, M, decay,
+                     freq, amp, phase, state_out, coef_out, ws, st);
+}
+
+cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt, int64_t B,
+                          int64_t L, int D, int M, const float *decay, const float *freq,
+                          const float *amp, const float *phase, float *g_decay, float *g_freq,
+                          float *g_amp, float *g_phase, void *ws, cudaStream_t st) {
+    if (dt == RLM_BF16)
+        return backward_t(static_cast<const __nv_bfloat16 *>(dy),
+                          static_cast<const __nv_bfloat16 *>(x), static_cast<__nv_bfloat16 *>(dx),
+                          B, L, D, M, decay, freq, amp, phase, g_decay, g_freq, g_amp, g_phase,
+                          ws, st);
+    return backward_t(static_cast<const float *>(dy), static_cast<const float *>(x),
+                      static_cast<float *>(dx), B, L, D, M, decay, freq, amp, phase, g_decay,
+                      g_freq, g_amp, g_phase, ws, st);
+}
+
+}  // namespace rlm

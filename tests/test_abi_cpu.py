@@ -1,0 +1,173 @@
+"""Host-side checks of the C ABI that need no GPU: the library builds and loads,
+exports every entry point include/rlm.h declares, and rejects bad arguments
+on the host before anything is enqueued (no pointer is dereferenced, so fake
+device addresses are enough)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2607_05583_gb300 as rlm
+from paper_2607_05583_gb300 import build as cbuild
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    cbuild.build()
+    return rlm.load_library()
+
+
+def _declared_entry_points():
+    names = []
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            names += re.findall(r"RLM_API\s+[\w\s\*]+?\b(rlm_\w+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_header_declares_the_boundary():
+    names = _declared_entry_points()
+    for want in ("rlm_mix_prefill", "rlm_mix_decode", "rlm_mix_backward",
+                 "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
+                 "rlm_state_init", "rlm_validate_params", "rlm_get_device_status",
+                 "rlm_status_string", "rlm_last_error"):
+        assert want in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in _declared_entry_points():
+        assert hasattr(lib, name), name
+
+
+def test_sources_target_sm103a_only():
+    assert cbuild.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+def test_status_strings(lib):
+    assert rlm.rlm_status_string(rlm.RLM_OK) == "RLM_OK"
+    assert rlm.rlm_status_string(rlm.RLM_ERR_TIMEOUT) == "RLM_ERR_TIMEOUT"
+    assert rlm.rlm_version() >= 100
+
+
+FAKE = 0x7F0000000000          # 256-byte aligned fake device address, never dereferenced
+
+
+def _t(ptr, B, L, D, dt=rlm.RLM_BF16):
+    return rlm._Tensor(ptr, dt, B, L, D)
+
+
+def _p(D, M, base=FAKE + (1 << 32)):
+    return rlm._Params(base, base + 4096, base + 8192, base + 12288, D, M)
+
+
+def _launch(ws=0, nbytes=0):
+    return rlm._Launch(None, ws or None, nbytes)
+
+
+def _prefill(lib, x, p, y, st=None, ln=None):
+    ln = ln or _launch(FAKE + (1 << 34), 1 << 40)
+    return lib.rlm_mix_prefill(ctypes.byref(x), ctypes.byref(p), ctypes.byref(y),
+                               ctypes.byref(st) if st else None, ctypes.byref(ln))
+
+
+@pytest.mark.parametrize("case", [
+    "null_x", "misaligned_x", "bad_dtype", "d_not_multiple_of_8", "zero_length",
+    "shape_mismatch", "dtype_mismatch", "overlap", "m_zero", "m_too_big", "param_d_mismatch",
+    "misaligned_param", "state_shape", "ws_too_small", "ws_misaligned"])
+def test_prefill_rejects_bad_arguments_on_host(lib, case):
+    B, L, D, M = 2, 100, 64, 16
+    x = _t(FAKE, B, L, D)
+    y = _t(FAKE + (1 << 30), B, L, D)
+    p = _p(D, M)
+    st = None
+    ln = None
+    if case == "null_x":
+        x = _t(0, B, L, D)
+    elif case == "misaligned_x":
+        x = _t(FAKE + 8, B, L, D)
+    elif case == "bad_dtype":
+        x = _t(FAKE, B, L, D, 7)
+    elif case == "d_not_multiple_of_8":
+        x, y, p = _t(FAKE, B, L, 12), _t(FAKE + (1 << 30), B, L, 12), _p(12, M)
+    elif case == "zero_length":
+        x, y = _t(FAKE, B, 0, D), _t(FAKE + (1 << 30), B, 0, D)
+    elif case == "shape_mismatch":
+        y = _t(FAKE + (1 << 30), B, L + 1, D)
+    elif case == "dtype_mismatch":
+        y = _t(FAKE + (1 << 30), B, L, D, rlm.RLM_F32)
+    elif case == "overlap":
+        y = _t(FAKE + 256, B, L, D)
+    elif case == "m_zero":
+        p = _p(D, 0)
+    elif case == "m_too_big":
+        p = _p(D, 65)
+    elif case == "param_d_mismatch":
+        p = _p(D + 8, M)
+    elif case == "misaligned_param":
+        p = _p(D, M, base=FAKE + (1 << 32) + 4)
+    elif case == "state_shape":
+        st = rlm._State(FAKE + (1 << 33), FAKE + (1 << 33) + (1 << 20), B + 1, D, M)
+    elif case == "ws_too_small":
+        ln = _launch(FAKE + (1 << 34), 16)
+    elif case == "ws_misaligned":
+        ln = _launch(FAKE + (1 << 34) + 16, 1 << 40)
+    status = _prefill(lib, x, p, y, st, ln)
+    if case == "ws_too_small" and lib.rlm_prefill_workspace_size(B, L, D, M, rlm.RLM_BF16) <= 16:
+        pytest.skip("this shape needs no workspace")
+    assert status == rlm.RLM_ERR_INVALID_ARG, (case, lib.rlm_last_error())
+    assert lib.rlm_last_error().decode()
+
+
+def test_decode_rejects_bad_arguments_on_host(lib):
+    B, D, M = 4, 64, 16
+    st = rlm._State(FAKE + (1 << 33), FAKE + (1 << 33) + (1 << 20), B, D, M)
+    ln = _launch()
+    call = lambda xt, s, yt: lib.rlm_mix_decode(ctypes.byref(xt), ctypes.byref(s),
+                                                ctypes.byref(yt), ctypes.byref(ln))
+    # L must be 1
+    assert call(_t(FAKE, B, 2, D), st, _t(FAKE + (1 << 30), B, 2, D)) == rlm.RLM_ERR_INVALID_ARG
+    # state batch mismatch
+    bad = rlm._State(st.s, st.coef, B + 1, D, M)
+    assert call(_t(FAKE, B, 1, D), bad, _t(FAKE + (1 << 30), B, 1, D)) == rlm.RLM_ERR_INVALID_ARG
+    # y overlaps the state
+    assert call(_t(FAKE, B, 1, D), st, _t(st.s, B, 1, D)) == rlm.RLM_ERR_INVALID_ARG
+    # M out of range
+    bad = rlm._State(st.s, st.coef, B, D, 0)
+    assert call(_t(FAKE, B, 1, D), bad, _t(FAKE + (1 << 30), B, 1, D)) == rlm.RLM_ERR_INVALID_ARG
+
+
+def test_backward_rejects_bad_arguments_on_host(lib):
+    B, L, D, M = 1, 50, 16, 2
+    dy, x, dx = _t(FAKE, B, L, D), _t(FAKE + (1 << 30), B, L, D), _t(FAKE + (1 << 31), B, L, D)
+    p = _p(D, M)
+    g = rlm._Params(FAKE + (1 << 35), FAKE + (1 << 35) + 4096, FAKE + (1 << 35) + 8192,
+                    FAKE + (1 << 35) + 12288, D, M)
+    ln = _launch(FAKE + (1 << 34), 1 << 40)
+    call = lambda dy, x, dx, g: lib.rlm_mix_backward(ctypes.byref(dy), ctypes.byref(x),
+                                                     ctypes.byref(p), ctypes.byref(dx),
+                                                     ctypes.byref(g), ctypes.byref(ln))
+    assert call(dy, x, _t(x.ptr, B, L, D), g) == rlm.RLM_ERR_INVALID_ARG        # dx aliases x
+    gbad = rlm._Params(g.decay, g.freq, g.amp, g.phase, D, M + 1)
+    assert call(dy, x, dx, gbad) == rlm.RLM_ERR_INVALID_ARG                      # grad shape
+    gnull = rlm._Params(g.decay, 0, g.amp, g.phase, D, M)
+    assert call(dy, x, dx, gnull) == rlm.RLM_ERR_INVALID_ARG
+    assert call(dy, _t(FAKE + (1 << 30), B, L, D, rlm.RLM_F32), dx, g) == rlm.RLM_ERR_INVALID_ARG
+
+
+def test_workspace_queries_are_host_only_and_monotone(lib):
+    a = lib.rlm_prefill_workspace_size(1, 1000, 64, 4, rlm.RLM_F32)
+    b = lib.rlm_prefill_workspace_size(4, 100000, 64, 4, rlm.RLM_F32)
+    assert b >= a
+    assert lib.rlm_backward_workspace_size(2, 5000, 64, 8, rlm.RLM_BF16) > 0
+    assert lib.rlm_prefill_workspace_size(0, 10, 8, 1, rlm.RLM_F32) == 0
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(rlm, "_lib", None)
+    monkeypatch.setattr(cbuild, "LIB", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        rlm.load_library()

@@ -1,0 +1,308 @@
+"""GPU parity: the CUDA path through the C ABI against the fp64 CPU oracle on the
+same seeded inputs, element by element, at sizes the oracle finishes in seconds
+(several chunks/tiles plus ragged tails) and at the full workload sizes on
+sampled channels (channels and batch rows are independent, so a sampled
+channel's oracle result is exact)."""
+import numpy as np
+import pytest
+
+import oracle
+from synth import make_inputs
+from tests._util import TOL, assert_close, rel_errors, to_dev, to_np
+
+torch = pytest.importorskip("torch")
+rlm = pytest.importorskip("paper_2607_05583_gb300")
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2607_05583_gb300 import build
+    build.build()
+    rlm.load_library()
+    yield
+    torch.cuda.synchronize()
+    assert rlm.rlm_get_device_status() == rlm.RLM_OK
+
+
+def _prefill(inp, with_state=True):
+    x = to_dev(inp.x, inp.dtype)
+    p = rlm.Params.from_arrays(*inp.params())
+    y = torch.empty_like(x)
+    st = rlm.State.empty(inp.B, inp.D, inp.M) if with_state else None
+    rlm.rlm_mix_prefill(x, p, y, st)
+    torch.cuda.synchronize()
+    return y, st
+
+
+def _sub(inp, chans):
+    """Oracle inputs restricted to the sampled channels."""
+    return (inp.x[:, :, chans], inp.decay[chans], inp.freq[chans], inp.amp[chans],
+            inp.phase[chans])
+
+
+def _state_err(st, ref, tol, what="state"):
+    s = st.complex().cpu().numpy()
+    assert_close(s.real, ref.real, tol, what + " re")
+    assert_close(s.imag, ref.imag, tol, what + " im")
+
+
+# --------------------------------------------------------------------- prefill
+def test_prefill_tiny_fp32_against_direct_convolution():
+    """fp32 single mixing op: B=1, L=256, D=64, M=4 against the O(L^2) oracle."""
+    inp = make_inputs(1, 256, 64, 4, "f32", seed=0)
+    y, st = _prefill(inp)
+    ref = oracle.conv_prefill(inp.x, *inp.params())
+    assert_close(to_np(y), ref, TOL["f32"], "y")
+    _, st_ref = oracle.rec_prefill(inp.x, *inp.params())
+    _state_err(st, st_ref, TOL["f32"])
+
+
+def test_prefill_layer6m_bf16():
+    """6M-scale layer: B=8, L=2048, D=256, M=16, bf16 I/O, plus the final state."""
+    inp = make_inputs(8, 2048, 256, 16, "bf16", seed=0)
+    y, st = _prefill(inp)
+    ref, st_ref = oracle.rec_prefill(inp.x, *inp.params())
+    assert_close(to_np(y), ref, TOL["bf16"], "y")
+    _state_err(st, st_ref, TOL["bf16"])
+    chans = np.array([0, 37, 128, 255])
+    ref1 = oracle.conv_prefill(*_sub(inp, chans))
+    assert_close(to_np(y)[:, :, chans], ref1, TOL["bf16"], "y vs direct convolution")
+
+
+@pytest.mark.parametrize("B,L,D,M,dtype", [
+    (1, 1, 8, 1, "f32"), (1, 1, 8, 16, "bf16"), (2, 7, 16, 3, "f32"), (3, 65, 24, 16, "bf16"),
+    (1, 1000, 8, 64, "f32"), (2, 2049, 64, 16, "bf16"), (1, 4097, 32, 5, "bf16"),
+    (2, 3000, 40, 33, "f32"), (1, 6143, 256, 16, "bf16"), (3, 2048 * 3 + 17, 64, 16, "bf16"),
+])
+def test_prefill_edge_and_ragged_shapes(B, L, D, M, dtype):
+    inp = make_inputs(B, L, D, M, dtype, seed=B * 1000 + L)
+    y, st = _prefill(inp)
+    ref, st_ref = oracle.rec_prefill(inp.x, *inp.params())
+    assert_close(to_np(y), ref, TOL[dtype], "y")
+    _state_err(st, st_ref, TOL[dtype])
+
+
+@pytest.mark.parametrize("B,L", [(1, 8192), (1, 16384), (1, 32768), (4, 8192), (4, 16384),
+                                 (4, 32768)])
+def test_prefill_long_context_sweep(B, L):
+    """Long-context sweep at the benchmark's launch configuration (D=256, M=16, bf16)."""
+    inp = make_inputs(B, L, 256, 16, "bf16", seed=0)
+    y, st = _prefill(inp)
+    chans = np.array([1, 64, 200, 255])
+    ref, st_ref = oracle.rec_prefill(*_sub(inp, chans))
+    assert_close(to_np(y)[:, :, chans], ref, TOL["bf16"], "y")
+    s = st.complex().cpu().numpy()[:, chans]
+    assert_close(s.real, st_ref.real, TOL["bf16"], "state re")
+    assert_close(s.imag, st_ref.imag, TOL["bf16"], "state im")
+
+
+def test_prefill_is_causal_bit_exact():
+    """I6: perturbing x[t >= t0] leaves y[t < t0] bit-identical on the GPU."""
+    for dtype in ("bf16", "f32"):
+        inp = make_inputs(2, 5000, 64, 16, dtype, seed=5)
+        y1, _ = _prefill(inp, False)
+        x2 = inp.x.copy()
+        x2[:, 3001:] = -x2[:, 3001:] + 1.0
+        inp2 = make_inputs(2, 5000, 64, 16, dtype, seed=5)
+        inp2.x = x2
+        y2, _ = _prefill(inp2, False)
+        a, b = y1.cpu(), y2.cpu()
+        assert torch.equal(a[:, :3001], b[:, :3001])
+        assert not torch.equal(a[:, 3001:], b[:, 3001:])
+
+
+def test_prefill_is_deterministic():
+    inp = make_inputs(2, 4100, 128, 16, "bf16", seed=9)
+    y1, s1 = _prefill(inp)
+    y2, s2 = _prefill(inp)
+    assert torch.equal(y1, y2) and torch.equal(s1.s, s2.s) and torch.equal(s1.coef, s2.coef)
+
+
+def test_prefill_does_not_write_outside_y():
+    inp = make_inputs(2, 777, 64, 16, "bf16", seed=13)
+    x = to_dev(inp.x, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    n = x.numel()
+    guard = 4096
+    buf = torch.full((n + 2 * guard,), 7.0, dtype=torch.bfloat16, device="cuda")
+    y = buf[guard:guard + n].view_as(x)
+    rlm.rlm_mix_prefill(x, p, y)
+    torch.cuda.synchronize()
+    assert torch.all(buf[:guard] == 7.0) and torch.all(buf[guard + n:] == 7.0)
+    ref, _ = oracle.rec_prefill(inp.x, *inp.params())
+    assert_close(to_np(y), ref, TOL["bf16"], "y")
+
+
+def test_linearity_on_gpu():
+    """I9 on the GPU (fp32 I/O): y(2 x1 - 3 x2) = 2 y(x1) - 3 y(x2) to fp32 rounding."""
+    a = make_inputs(1, 3000, 32, 8, "f32", seed=21)
+    b = make_inputs(1, 3000, 32, 8, "f32", seed=22)
+    b.decay, b.freq, b.amp, b.phase = a.decay, a.freq, a.amp, a.phase
+    c = make_inputs(1, 3000, 32, 8, "f32", seed=21)
+    c.x = (2 * a.x - 3 * b.x).astype(np.float32)
+    ya, yb, yc = (to_np(_prefill(i, False)[0]) for i in (a, b, c))
+    assert_close(yc, 2 * ya - 3 * yb, 1e-5, "linearity")
+
+
+# ---------------------------------------------------------------------- decode
+@pytest.mark.parametrize("dtype,M", [("bf16", 16), ("f32", 16), ("f32", 5), ("bf16", 64),
+                                     ("f32", 1)])
+def test_decode_steps_match_oracle(dtype, M):
+    B, L, D, T = 3, 500, 24, 40
+    inp = make_inputs(B, L, D, M, dtype, seed=M, decode_steps=T)
+    _, st = _prefill(inp)
+    ys = []
+    for t in range(T):
+        xt = to_dev(inp.tokens[t], dtype)
+        yt = torch.empty_like(xt)
+        rlm.rlm_mix_decode(xt, st, yt)
+        ys.append(to_np(yt))
+    xcat = np.concatenate([inp.x, inp.tokens.transpose(1, 0, 2)], axis=1)
+    ref, st_ref = oracle.rec_prefill(xcat, *inp.params())
+    assert_close(np.stack(ys, 1), ref[:, L:], TOL[dtype], "y_t")
+    _state_err(st, st_ref, TOL[dtype])
+
+
+def test_prefill_plus_one_decode_equals_longer_prefill_on_gpu():
+    """I3 with both sides on the GPU."""
+    for dtype in ("f32", "bf16"):
+        inp = make_inputs(2, 4097, 64, 16, dtype, seed=3)
+        y_full, st_full = _prefill(inp)
+        short = make_inputs(2, 4097, 64, 16, dtype, seed=3)
+        short.x = inp.x[:, :4096].copy()
+        short.L = 4096
+        _, st = _prefill(short)
+        xt = to_dev(inp.x[:, 4096], dtype)
+        yt = torch.empty_like(xt)
+        rlm.rlm_mix_decode(xt, st, yt)
+        torch.cuda.synchronize()
+        assert_close(to_np(yt), to_np(y_full[:, 4096]), TOL[dtype], "y_L")
+        _state_err(st, st_full.complex().cpu().numpy(), TOL[dtype])
+
+
+@pytest.mark.parametrize("B", [1, 8, 64])
+def test_decode_after_32k_prefill(B):
+    """Decode workload: state from a 32768-token prefill (D=256, M=16), then 4096
+    single-token steps, checked against a prefill of the concatenated sequence
+    (oracle on sampled channels)."""
+    L, D, M, T = 32768, 256, 16, 4096
+    inp = make_inputs(B, L, D, M, "bf16", seed=0, decode_steps=T)
+    _, st = _prefill(inp)
+    toks = to_dev(inp.tokens, "bf16")                  # [T][B][D]
+    out = torch.empty_like(toks)
+    for t in range(T):
+        rlm.rlm_mix_decode(toks[t], st, out[t])
+    torch.cuda.synchronize()
+    chans = np.array([3, 130, 254])
+    xcat = np.concatenate([inp.x[:, :, chans], inp.tokens[:, :, chans].transpose(1, 0, 2)], 1)
+    ref, st_ref = oracle.rec_prefill(xcat, inp.decay[chans], inp.freq[chans], inp.amp[chans],
+                                     inp.phase[chans])
+    got = to_np(out)[:, :, chans].transpose(1, 0, 2)
+    assert_close(got, ref[:, L:], TOL["bf16"], "decode y_t")
+    s = st.complex().cpu().numpy()[:, chans]
+    assert_close(s.real, st_ref.real, TOL["bf16"], "state re")
+
+
+def test_state_init_then_decode_equals_prefill():
+    inp = make_inputs(2, 50, 16, 16, "f32", seed=4)
+    p = rlm.Params.from_arrays(*inp.params())
+    st = rlm.State.empty(2, 16, 16)
+    rlm.rlm_state_init(st, p)
+    ys = []
+    for t in range(50):
+        xt = to_dev(inp.x[:, t], "f32")
+        yt = torch.empty_like(xt)
+        rlm.rlm_mix_decode(xt, st, yt)
+        ys.append(to_np(yt))
+    ref = oracle.conv_prefill(inp.x, *inp.params())
+    assert_close(np.stack(ys, 1), ref, TOL["f32"], "y")
+
+
+def test_zero_drive_decode_energy_decay():
+    """I7 on the GPU: with zero drive |s_t|^2 = exp(-2 gamma t) |s_0|^2."""
+    inp = make_inputs(2, 300, 16, 8, "f32", seed=6)
+    _, st = _prefill(inp)
+    s0 = st.complex().cpu().numpy().copy()
+    z = torch.zeros(2, 16, device="cuda")
+    y = torch.empty_like(z)
+    for _ in range(25):
+        rlm.rlm_mix_decode(z, st, y)
+    s = st.complex().cpu().numpy()
+    want = np.exp(-2 * 25 * inp.decay.astype(np.float64))[None] * np.abs(s0) ** 2
+    np.testing.assert_allclose(np.abs(s) ** 2, want, rtol=2e-5, atol=1e-12)
+
+
+# -------------------------------------------------------------------- backward
+def _backward(inp):
+    x, dy = to_dev(inp.x, inp.dtype), to_dev(inp.dy, inp.dtype)
+    p = rlm.Params.from_arrays(*inp.params())
+    dx = torch.empty_like(x)
+    g = rlm.Grads.empty(inp.D, inp.M)
+    rlm.rlm_mix_backward(dy, x, p, dx, g)
+    torch.cuda.synchronize()
+    return dx, g
+
+
+@pytest.mark.parametrize("B,L,D,M,dtype", [
+    (1, 256, 64, 4, "f32"), (2, 1000, 16, 7, "f32"), (2, 3001, 64, 16, "bf16"),
+    (1, 4096, 32, 32, "bf16"), (1, 1, 8, 1, "f32"),
+])
+def test_backward_matches_oracle(B, L, D, M, dtype):
+    inp = make_inputs(B, L, D, M, dtype, seed=L + M, with_dy=True)
+    dx, g = _backward(inp)
+    dx_ref, g_ref = oracle.backward_rec(inp.x, inp.dy, *inp.params())
+    assert_close(to_np(dx), dx_ref, TOL[dtype], "dx")
+    for k in ("decay", "freq", "amp", "phase"):
+        assert_close(getattr(g, k).cpu().numpy(), g_ref[k], TOL[dtype], "d" + k)
+
+
+def test_backward_training_workload_sampled():
+    """Training path: B=4, L=32768, D=512, M=32, bf16 I/O; dx and all four parameter
+    gradients of sampled channels against the oracle."""
+    inp = make_inputs(4, 32768, 512, 32, "bf16", seed=0, with_dy=True)
+    dx, g = _backward(inp)
+    chans = np.array([0, 101, 333, 511])
+    dx_ref, g_ref = oracle.backward_rec(inp.x[:, :, chans], inp.dy[:, :, chans],
+                                        inp.decay[chans], inp.freq[chans], inp.amp[chans],
+                                        inp.phase[chans])
+    assert_close(to_np(dx)[:, :, chans], dx_ref, TOL["bf16"], "dx")
+    for k in ("decay", "freq", "amp", "phase"):
+        assert_close(getattr(g, k).cpu().numpy()[chans], g_ref[k], TOL["bf16"], "d" + k)
+
+
+def test_backward_is_deterministic():
+    inp = make_inputs(2, 5000, 64, 16, "bf16", seed=8, with_dy=True)
+    dx1, g1 = _backward(inp)
+    dx2, g2 = _backward(inp)
+    assert torch.equal(dx1, dx2)
+    for k in ("decay", "freq", "amp", "phase"):
+        assert torch.equal(getattr(g1, k), getattr(g2, k))
+
+
+def test_backward_gpu_finite_differences_tiny():
+    """Gradients against central differences of the GPU's own fp32 forward at a tiny
+    size (loss sum(dy * y)); loose bound because the forward is fp32."""
+    inp = make_inputs(1, 40, 8, 2, "f32", seed=77, with_dy=True)
+    dx, g = _backward(inp)
+    p0 = [q.astype(np.float64) for q in inp.params()]
+    dy = inp.dy.astype(np.float64)
+
+    def loss(ps):
+        i2 = make_inputs(1, 40, 8, 2, "f32", seed=77)
+        i2.decay, i2.freq, i2.amp, i2.phase = (q.astype(np.float32) for q in ps)
+        y, _ = _prefill(i2, False)
+        return float(np.sum(dy * to_np(y)))
+
+    names = ["decay", "freq", "amp", "phase"]
+    for k, name in enumerate(names):
+        idx = (3, 1)
+        h = 5e-4 if name == "decay" else 1e-3
+        pp = [q.copy() for q in p0]
+        pm = [q.copy() for q in p0]
+        pp[k][idx] += h
+        pm[k][idx] -= h
+        fd = (loss(pp) - loss(pm)) / (2 * h)
+        got = float(getattr(g, name).cpu().numpy()[idx])
+        assert abs(got - fd) <= 2e-2 * max(1.0, abs(fd)), (name, got, fd)
