@@ -85,11 +85,15 @@ class ClockSampler:
         self.lines = []
 
     def __enter__(self):
+        cmd = ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+               "--format=csv,noheader,nounits", "-lms", "200"]
         try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
-                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            # nvidia-smi block-buffers into a pipe; stdbuf makes it line-buffered.
+            import shutil
+            if shutil.which("stdbuf"):
+                cmd = ["stdbuf", "-oL"] + cmd
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
             self._t = threading.Thread(target=self._read, daemon=True)
             self._t.start()
         except Exception:
@@ -212,18 +216,26 @@ def run_ours(args):
         flush.zero_()
         step()
     torch.cuda.synchronize()
-    n_launch = _count_launches(step)
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    _barrier(ws)
-    torch.cuda.synchronize()
     with ClockSampler(local) as clk:
+        # The clock sampler (200 ms period) needs a loaded GPU for longer than the
+        # timed steps last: soak with the same kernel first, then time.
+        t_end = time.perf_counter() + args.soak
+        while time.perf_counter() < t_end:
+            for _ in range(20):
+                step()
+            torch.cuda.synchronize()
+        _barrier(ws)
+        torch.cuda.synchronize()
+        n0 = rlm.rlm_kernels_launched()
         for i in range(args.steps):
             flush.zero_()
             starts[i].record(stream)
             step()
             ends[i].record(stream)
         torch.cuda.synchronize()
+        n_launch = rlm.rlm_kernels_launched() - n0
     _barrier(ws)
     times = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     ms = statistics.mean(times)
@@ -291,32 +303,13 @@ def run_ours(args):
                        "parallelism": f"replicas x{ws}" if ws > 1 else "single GPU",
                        "l2": "flushed (512 MiB write) before every timed step"},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-            "gpu_launches": n_launch * args.steps,
+            "gpu_launches": n_launch,
             "clocks": clk.summary(), "sweep": sweep, "decode": decode, "backward": backward,
         }
         print(json.dumps(line), flush=True)
     if ws > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
-
-
-def _count_launches(step):
-    """Kernels of ours that one step launches (counted with the profiler's CUDA
-    activity list, names matched against the library's kernel prefixes)."""
-    import torch
-    from torch.profiler import ProfilerActivity, profile
-    try:
-        with profile(activities=[ProfilerActivity.CUDA]) as prof:
-            step()
-            torch.cuda.synchronize()
-        n = 0
-        for ev in prof.events():
-            name = ev.name or ""
-            if "rlm::" in name or name.startswith("k_") or "rlm" in name:
-                n += 1
-        return n
-    except Exception:
-        return -1
 
 
 def _time_prefill(rlm, torch, dev, B, L, D, M, flush, hbm_peak, reps=5):
@@ -491,6 +484,8 @@ def main():
     ap.add_argument("--quick", action="store_true", help="prefill only (no sweep/decode/backward)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--soak", type=float, default=1.5,
+                    help="seconds of untimed prefill before the timed steps (clock sampling)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -177,6 +177,10 @@ RLM_API const char *rlm_last_error(void);
 /* Library version as major*10000 + minor*100 + patch. */
 RLM_API int rlm_version(void);
 
+/* Number of kernels this library has launched in this process so far (a
+ * host-side count, incremented at each launch; for accounting in benchmarks). */
+RLM_API unsigned long long rlm_kernels_launched(void);
+
 #ifdef __cplusplus
 }
 #endif

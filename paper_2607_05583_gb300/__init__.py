@@ -25,7 +25,7 @@ __all__ = [
     "rlm_mix_prefill", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
     "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
     "rlm_validate_params", "rlm_get_device_status", "rlm_status_string",
-    "rlm_version", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
+    "rlm_version", "rlm_kernels_launched", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
     "RLM_ERR_CUDA", "RLM_ERR_TIMEOUT", "RLM_F32", "RLM_BF16",
 ]
 
@@ -102,6 +102,7 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.rlm_status_string.restype = ctypes.c_char_p
     lib.rlm_last_error.restype = ctypes.c_char_p
     lib.rlm_version.restype = ctypes.c_int
+    lib.rlm_kernels_launched.restype = ctypes.c_ulonglong
     _lib = lib
     return lib
 
@@ -226,6 +227,11 @@ def rlm_status_string(status: int) -> str:
 
 def rlm_version() -> int:
     return load_library().rlm_version()
+
+
+def rlm_kernels_launched() -> int:
+    """Kernels the library has launched in this process (host-side count)."""
+    return int(load_library().rlm_kernels_launched())
 
 
 def rlm_prefill_workspace_size(B: int, L: int, D: int, M: int, dtype) -> int:

@@ -6,6 +6,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <atomic>
 #include <mutex>
 #include <vector>
 
@@ -14,6 +15,9 @@
 namespace rlm {
 
 static thread_local char g_err[512] = "";
+static std::atomic<unsigned long long> g_launches{0};
+
+void count_launches(int n) { g_launches.fetch_add((unsigned long long)n, std::memory_order_relaxed); }
 
 void set_error(const char *fmt, ...) {
     va_list ap;
@@ -154,6 +158,8 @@ const char *rlm_status_string(rlm_status s) {
 const char *rlm_last_error(void) { return g_err; }
 
 int rlm_version(void) { return 100; }
+
+unsigned long long rlm_kernels_launched(void) { return g_launches.load(std::memory_order_relaxed); }
 
 size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
     if (B < 1 || L < 1 || D < 1 || M < 1) return 0;

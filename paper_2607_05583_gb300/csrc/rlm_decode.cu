@@ -111,6 +111,7 @@ cudaError_t launch_pdl(Kern kern, unsigned grid, cudaStream_t st, Args... args) 
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    count_launches(1);
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
@@ -151,6 +152,7 @@ cudaError_t state_init(float *s, float *coef, int B, int D, int M, const float *
     k_state_init<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(
         reinterpret_cast<float2 *>(s), reinterpret_cast<float4 *>(coef), BDM, D * M, decay, freq,
         amp, phase);
+    count_launches(1);
     return cudaGetLastError();
 }
 

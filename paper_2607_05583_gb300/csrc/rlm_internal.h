@@ -16,6 +16,9 @@ void set_error(const char *fmt, ...);
 // Multiprocessor count of the current device (cached per device).
 int sm_count();
 
+// Adds n to the process-wide count of kernels this library has launched.
+void count_launches(int n);
+
 // ---- SIMT chunked scan (rlm_simt.cu) --------------------------------------
 // Chunk length the SIMT path uses for a problem; workspace and launch agree.
 int simt_chunk_len(int64_t B, int64_t L, int D);

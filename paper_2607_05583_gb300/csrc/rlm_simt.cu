@@ -269,6 +269,7 @@ cudaError_t prefill_t(const T *x, T *y, int64_t B, int64_t L, int D, int M, cons
         reinterpret_cast<float2 *>(state_out), reinterpret_cast<float4 *>(coef_out));
     k_chunk_output<T, kMgFwd, false><<<grid, kBlock, 0, st>>>(
         x, y, L, D, M, tpc, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s);
+    count_launches(3);
     return cudaGetLastError();
 }
 
@@ -294,6 +295,7 @@ cudaError_t backward_t(const T *dy, const T *x, T *dx, int64_t B, int64_t L, int
         dy, x, dx, L, D, M, tpc3, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, ws_r);
     k_grad_reduce<<<(unsigned)((D * M + 255) / 256), 256, 0, st>>>(
         B, D, M, g.nch, amp, phase, ws_s, ws_r, gd, gf, ga, gp);
+    count_launches(4);
     return cudaGetLastError();
 }
 

@@ -111,13 +111,13 @@ def test_prefill_rejects_bad_arguments_on_host(lib, case):
         p = _p(D, M, base=FAKE + (1 << 32) + 4)
     elif case == "state_shape":
         st = rlm._State(FAKE + (1 << 33), FAKE + (1 << 33) + (1 << 20), B + 1, D, M)
-    elif case == "ws_too_small":
-        ln = _launch(FAKE + (1 << 34), 16)
-    elif case == "ws_misaligned":
-        ln = _launch(FAKE + (1 << 34) + 16, 1 << 40)
+    elif case in ("ws_too_small", "ws_misaligned"):
+        # fp32 I/O runs the chunked SIMT path, which needs a workspace
+        x, y = _t(FAKE, B, L, D, rlm.RLM_F32), _t(FAKE + (1 << 30), B, L, D, rlm.RLM_F32)
+        assert lib.rlm_prefill_workspace_size(B, L, D, M, rlm.RLM_F32) > 16
+        ln = (_launch(FAKE + (1 << 34), 16) if case == "ws_too_small"
+              else _launch(FAKE + (1 << 34) + 16, 1 << 40))
     status = _prefill(lib, x, p, y, st, ln)
-    if case == "ws_too_small" and lib.rlm_prefill_workspace_size(B, L, D, M, rlm.RLM_BF16) <= 16:
-        pytest.skip("this shape needs no workspace")
     assert status == rlm.RLM_ERR_INVALID_ARG, (case, lib.rlm_last_error())
     assert lib.rlm_last_error().decode()
 
