@@ -127,6 +127,30 @@ RLM_API rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm
 /* Bytes of workspace rlm_mix_prefill needs for this shape (0 is possible). */
 RLM_API size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype);
 
+/* rlm_mix_prefill_noalloc -- the paper has no counterpart; this entry point
+ * exists for callers that cannot allocate device memory when they call the
+ * library, such as serving runtimes that reserve all device memory up front and
+ * forbid allocation afterwards, or plugin hosts that own every allocation and
+ * cannot hand out a workspace.  It computes what rlm_mix_prefill computes (same
+ * arguments, no workspace) with the chunked-scan kernels, whose scratch lives in
+ * a fixed 64 MiB array that the library itself places in device memory: every
+ * GPU that loads the library holds that array until the process exits.
+ *  - The entry point allocates nothing: no cudaMalloc, cudaFree or allocating
+ *    library routine on any path.
+ *  - Shapes whose scratch would exceed 64 MiB (B * nchunks * D * M * 8 bytes)
+ *    return RLM_ERR_UNSUPPORTED with the needed size in rlm_last_error().
+ *  - The first call on a device looks up the array's device address (one
+ *    cudaGetSymbolAddress with that device current); make that first call
+ *    before any stream capture.
+ *  - All calls share the one array, and it keeps the previous call's contents;
+ *    every scratch element is written before it is read, so nothing needs
+ *    clearing.  Calls whose executions overlap on the GPU (different streams,
+ *    or host threads on one device) race on the array and must be serialised
+ *    by the caller.
+ *  - stream: a cudaStream_t passed as void* (NULL = legacy default stream). */
+RLM_API rlm_status rlm_mix_prefill_noalloc(const rlm_tensor *x, const rlm_params *p, rlm_tensor *y,
+                                           rlm_state *state_out, void *stream);
+
 /* ------------------------------------------------------------------- decode
  * One autoregressive step of Sec. 3.3 (Eq. 4-5) for a batch of tokens:
  *   s_bdm <- lambda_dm s_bdm + x_t[b,d];   y_t[b,d] = sum_m Re(c_dm s_bdm)

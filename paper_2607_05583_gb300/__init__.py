@@ -22,7 +22,7 @@ from . import build as _build_mod
 
 __all__ = [
     "RlmError", "Params", "Grads", "State", "load_library", "library_path",
-    "rlm_mix_prefill", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
+    "rlm_mix_prefill", "rlm_mix_prefill_noalloc", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
     "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
     "rlm_validate_params", "rlm_get_device_status", "rlm_status_string",
     "rlm_version", "rlm_kernels_launched", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
@@ -103,6 +103,9 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.rlm_last_error.restype = ctypes.c_char_p
     lib.rlm_version.restype = ctypes.c_int
     lib.rlm_kernels_launched.restype = ctypes.c_ulonglong
+    lib.rlm_mix_prefill_noalloc.argtypes = [P(_Tensor), P(_Params), P(_Tensor), P(_State),
+                                            ctypes.c_void_p]
+    lib.rlm_mix_prefill_noalloc.restype = ctypes.c_int
     _lib = lib
     return lib
 
@@ -257,6 +260,20 @@ def rlm_mix_prefill(x: torch.Tensor, params: Params, y: torch.Tensor,
     _check(lib.rlm_mix_prefill(ctypes.byref(xt), ctypes.byref(params._c()), ctypes.byref(yt),
                                ctypes.byref(st) if st is not None else None,
                                ctypes.byref(_launch(stream, workspace))), "rlm_mix_prefill")
+
+
+def rlm_mix_prefill_noalloc(x: torch.Tensor, params: Params, y: torch.Tensor,
+                            state_out: State | None = None, stream=None) -> None:
+    """rlm_mix_prefill without a workspace, for callers that cannot allocate device
+    memory: the scratch is the library's fixed 64 MiB device array (see rlm.h).
+    Calls that overlap on the GPU race on that array."""
+    lib = load_library()
+    xt, yt = _field(x), _field(y)
+    st = state_out._c() if state_out is not None else None
+    _check(lib.rlm_mix_prefill_noalloc(ctypes.byref(xt), ctypes.byref(params._c()),
+                                       ctypes.byref(yt),
+                                       ctypes.byref(st) if st is not None else None,
+                                       _stream(stream)), "rlm_mix_prefill_noalloc")
 
 
 def rlm_mix_decode(x_t: torch.Tensor, state: State, y_t: torch.Tensor, stream=None) -> None:
