@@ -16,32 +16,37 @@
 //   D[64:96, n]  = W  (32x64)  X_n      local end state, (Re, Im) of 16 modes
 //   D[0:64, n]  += U  (64x32)  S_{n-1}  up-projection of the carried state
 //
-// T and W share one A operand (rows 0-63 and 64-95 of a 128-row matrix), so a
-// single MMA chain yields both.  The columns of D are the NT = 32 chunks of a
-// 2048-token tile (MMA N = 32).  The carry between chunks is a sequential fp32
-// complex scan in registers: one thread per state row, the two rows (Re, Im) of
-// a mode exchange their values with one warp shuffle per chunk.
+// T and W share one A operand (rows 0-63 and 64-95 of a 128-row matrix) held in
+// TMEM, so a single MMA chain yields both.  The columns of D are the NT = 16
+// chunks of a 1024-token tile (MMA N = 16).  The carry between chunks is a
+// sequential fp32 complex scan in registers: one thread per state row, the two
+// rows (Re, Im) of a mode exchange their values with one warp shuffle per chunk.
 //
 // One CTA owns one batch row b and one group of DG = 8 channels (a 16-byte
 // slice of each token row) and walks the sequence tile by tile, carrying the
 // state in registers, so no CTA waits on another.
 //
-// Data movement per tile (2048 tokens x 8 channels):
-//   TMA (3-D map over [B][L][D], zero fill outside the sequence) -> smem ring
-//   -> ldmatrix.trans / stmatrix into the per-channel K-major B operand (the
-//      positions of a chunk reversed, so the Toeplitz block becomes a Hankel
-//      block; see the A operand layout below)
+// Data movement per tile (1024 tokens x 8 channels):
+//   TMA (3-D map over [B][L][D], zero fill outside the sequence) -> 24-box ring
+//   -> ldmatrix.trans / stmatrix by four transposer warps into the per-channel
+//      K-major B operand (double-buffered; the positions of a chunk reversed so
+//      that the A operand's Toeplitz rows read K[i + p' - 63])
 //   -> tcgen05.mma -> TMEM -> scan warps -> B operand of the up-projection
 //   -> tcgen05.mma -> TMEM -> epilogue warps (fp32 -> bf16, 8 channels packed
 //      into one 16-byte row) -> smem ring -> TMA store.
-// TMEM is double-buffered across tiles (2 x 8 channels x 32 columns).
+// TMEM (512 columns): two accumulator buffers of 8 channels x 16 columns, and
+// the 8 channels' A operands (128 lanes x 32 columns of packed bf16 pairs).
 //
-// Warp roles (16 warps): TMEM lane quarter q = warp % 4 decides which rows of
-// D a warp may read.  Quarters 0-1: epilogue (rows 0-63).  Quarter 2: scan
-// (rows 64-95), two channels per warp.  Quarter 3: TMA producer (warp 3), MMA
-// issuer (warp 7), TMA store issuer (warp 11), transposer (warp 15).
+// Warp roles (19 warps): TMEM lane quarter q = warp % 4 (also the SM
+// sub-partition the warp runs on) decides which rows of D a warp may read.
+// Warps 0,1,4,5,8,9,12,13: epilogue (rows 0-63).  Warps 2, 6 (quarter 2) and
+// 7, 15 (quarter 3): two channels each, end to end -- they issue those
+// channels' MMAs (one tile ahead), scan their states and issue the
+// up-projection; four issuing warps keep the tensor pipe busy where one
+// issuing thread could not.  Warp 3: TMA producer; warp 11: TMA store issuer;
+// warps 10, 14, 16, 17: transposers; warp 18 idle; warp 7 also allocates TMEM.
 //
-// Every wait is bounded: after kWaitLimitNs the waiting thread sets a shared
+// Every wait is bounded: after kWaitLimitCycles the waiting thread sets a shared
 // abort flag and the device status word (RLM_ERR_TIMEOUT); all roles then leave
 // their loops, drain what they issued and the CTA frees its TMEM and returns.
 #include <cuda.h>
@@ -60,63 +65,57 @@ __device__ int g_device_status = 0;
 namespace {
 
 constexpr int kC = 64;                 // chunk length
-constexpr int kNT = 32;                // chunks per tile = MMA N
-constexpr int kTile = kC * kNT;        // 2048 tokens
+constexpr int kNT = 16;                // chunks per tile = MMA N
+constexpr int kTile = kC * kNT;        // 1024 tokens
 constexpr int kDG = 8;                 // channels per CTA
 constexpr int kModes = 16;             // M handled by this kernel
 constexpr int kBox = 256;              // TMA box rows
-constexpr int kBoxes = kTile / kBox;   // 8 per tile
-constexpr int kXSlots = 4;             // x ring depth (boxes)
+constexpr int kBoxes = kTile / kBox;   // 4 per tile
+constexpr int kXSlots = 20;            // x ring depth (boxes)
 constexpr int kYSlots = 2;             // y ring depth (blocks of 8 chunks)
-constexpr int kThreads = 512;
+constexpr int kWarps = 19;
+constexpr int kThreads = kWarps * 32;
 constexpr int kTmemCols = 512;
-constexpr unsigned long long kWaitLimitNs = 1000000000ull;  // 1 s
+constexpr int kTmemA = 256;            // first TMEM column of the A operands
+constexpr long long kWaitLimitCycles = 4000000000ll;  // about 2 s at 2 GHz
 
 // Shared memory map (bytes from a 1024-aligned base).
-constexpr int kAtwStride = 12 * 1024;  // 96 real rows x 128 B; rows 96-127 alias the next buffer
-constexpr int kAuStride = 4096;        // 64 real rows x 64 B;  rows 64-127 alias the next buffer
-constexpr int kBxStride = 4096 + 16;   // 32 rows x 128 B, +16 so stmatrix rows hit distinct banks
-constexpr int kBsLbo = 144, kBsSbo = 576, kBsStride = 4 * kBsSbo;
-constexpr int kOffAtw = 0;
-constexpr int kOffAu = kOffAtw + kDG * kAtwStride;          // 98304
-constexpr int kOffBx = kOffAu + kDG * kAuStride;             // 131072
-constexpr int kOffBs = kOffBx + kDG * kBxStride;             // 163968
-constexpr int kOffX = 182400;                                // 128-aligned
-constexpr int kOffY = kOffX + kXSlots * kBox * 16;           // 198784
-constexpr int kOffBar = kOffY + kYSlots * 512 * 16;          // 215168
-constexpr int kNumBars = 64;
+constexpr int kAuStride = 4096;        // 64 real rows x 64 B; rows 64-127 alias the next buffer
+constexpr int kBxStride = 2048 + 16;   // 16 rows x 128 B, +16 so stmatrix rows hit distinct banks
+constexpr int kBxBuf = kDG * kBxStride;
+constexpr int kBsLbo = 144, kBsSbo = 576, kBsStride = 2 * kBsSbo + 64;  // +64: two channels' rows in disjoint banks
+constexpr int kBsBuf = kDG * kBsStride;
+constexpr int kOffAu = 0;
+constexpr int kOffBx = kOffAu + kDG * kAuStride;             // 32768
+constexpr int kOffBs = kOffBx + 2 * kBxBuf;                  // 65792
+constexpr int kOffSt = kOffBs + 2 * kBsBuf;                  // per scan warp: [2 ch][16 chunks][32 rows] fp32
+constexpr int kStWarp = 2 * 16 * 32 * 4;
+constexpr int kOffX = kOffSt + 4 * kStWarp;
+constexpr int kOffY = kOffX + kXSlots * kBox * 16;
+constexpr int kOffBar = kOffY + kYSlots * 512 * 16;
+constexpr int kNumBars = 128;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;             // + alignment slack
-static_assert(kOffBs + kDG * kBsStride <= kOffX, "smem layout overlap");
 static_assert(kOffX % 128 == 0 && kOffY % 128 == 0, "TMA buffers need 128-byte alignment");
 static_assert(kOffBx + 8 * 64 * 16 * 4 + 8 * 64 * 4 <= kOffX, "prologue scratch does not fit");
 
 // Barrier indices.
-constexpr int kBarXFull = 0;        // [4]
-constexpr int kBarXEmpty = 4;       // [4]
-constexpr int kBarBxFull = 8;
-constexpr int kBarBxEmpty = 9;
-constexpr int kBarTwDone = 10;      // [2][8]
-constexpr int kBarSFull = 26;       // [8]
-constexpr int kBarUDone = 34;       // [2]
-constexpr int kBarDEmpty = 36;      // [2]
-constexpr int kBarYFull = 38;       // [2]
-constexpr int kBarYEmpty = 40;      // [2]
-constexpr int kBarFinal = 42;
+constexpr int kBarXFull = 0;                    // [kXSlots]
+constexpr int kBarXEmpty = kXSlots;             // [kXSlots]
+constexpr int kBarBxFull = 2 * kXSlots;         // [2]
+constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]
+constexpr int kBarTwDone = kBarBxEmpty + 2;     // [2][4]: per buffer, per scan warp
+constexpr int kBarUDone = kBarTwDone + 8;       // [2]
+constexpr int kBarDEmpty = kBarUDone + 2;       // [2]
+constexpr int kBarYFull = kBarDEmpty + 2;       // [2]
+constexpr int kBarYEmpty = kBarYFull + 2;       // [2]
+constexpr int kBarFinal = kBarYEmpty + 2;       // [4]
+static_assert(kBarFinal + 4 <= kNumBars, "too many barriers");
 
-// Instruction descriptor, kind::f16: fp32 accumulate, bf16 A and B, both
-// K-major, M = 128, N = 32.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kNT >> 3) << 17) |
-                            ((uint32_t)(128 >> 4) << 24);
 
 // ------------------------------------------------------------ PTX wrappers
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return (uint32_t)__cvta_generic_to_shared(p);
-}
-__device__ __forceinline__ uint64_t globaltimer() {
-    uint64_t t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
 }
 __device__ __forceinline__ void bar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
@@ -125,6 +124,16 @@ __device__ __forceinline__ bool bar_try(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Non-blocking probe of a phase (unlike try_wait, never suspends the thread).
+__device__ __forceinline__ bool bar_test(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
         : "=r"(ok)
         : "r"(bar), "r"(parity)
         : "memory");
@@ -139,16 +148,24 @@ __device__ __forceinline__ void bar_expect_tx(uint32_t bar, uint32_t bytes) {
 }
 
 // Bounded wait on an mbarrier phase.  Returns false if this CTA aborted.
+// The bound is measured with the SM cycle counter, read only every 1024 failed
+// polls: reading %globaltimer costs about half a microsecond, which would
+// otherwise be added to every wait that does not succeed at once.
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int *abort_flag) {
     if (bar_try(bar, parity)) return true;
-    const uint64_t t0 = globaltimer();
+    long long t0 = 0;
     for (uint32_t it = 1;; ++it) {
         if (bar_try(bar, parity)) return true;
-        if (*abort_flag) return false;
-        if ((it & 63u) == 0 && globaltimer() - t0 > kWaitLimitNs) {
-            *abort_flag = 1;
-            atomicExch(&g_device_status, (int)RLM_ERR_TIMEOUT);
-            return false;
+        if ((it & 1023u) == 0) {
+            if (*abort_flag) return false;
+            const long long now = clock64();
+            if (t0 == 0) {
+                t0 = now;
+            } else if (now - t0 > kWaitLimitCycles) {
+                *abort_flag = 1;
+                atomicExch(&g_device_status, (int)RLM_ERR_TIMEOUT);
+                return false;
+            }
         }
     }
 }
@@ -195,11 +212,22 @@ __device__ __forceinline__ uint64_t umma_desc(uint32_t saddr, uint32_t lbo, uint
     return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
            ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
 }
-__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t accum) {
+// D (TMEM) (+)= A (shared memory) * B (shared memory)^T.
+__device__ __forceinline__ void umma_ss(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                        uint32_t accum) {
     asm volatile(
         "{ .reg .pred p; setp.ne.b32 p, %4, 0;\n"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(d_tmem),
-        "l"(a), "l"(b), "r"(kIdesc), "r"(accum)
+        "l"(a), "l"(b), "r"(idesc), "r"(accum)
+        : "memory");
+}
+// D (TMEM) (+)= A (TMEM: lane = row, column c = K elements 2c, 2c+1) * B (smem)^T.
+__device__ __forceinline__ void umma_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
+                                        uint32_t idesc, uint32_t accum) {
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p; }" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(accum)
         : "memory");
 }
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
@@ -208,18 +236,15 @@ __device__ __forceinline__ void umma_commit(uint32_t bar) {
         : "memory");
 }
 
-#define RLM_TMEM_LD32(taddr, v)                                                                   \
-    asm volatile(                                                                                 \
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13," \
-        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"       \
-        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),   \
-          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),             \
-          "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]),          \
-          "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),          \
-          "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]),          \
-          "=r"(v[31])                                                                             \
-        : "r"(taddr))
-
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+          "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr));
+}
 __device__ __forceinline__ void tmem_ld2(uint32_t taddr, uint32_t &a, uint32_t &b) {
     asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0, %1}, [%2];"
                  : "=r"(a), "=r"(b)
@@ -228,6 +253,21 @@ __device__ __forceinline__ void tmem_ld2(uint32_t taddr, uint32_t &a, uint32_t &
 __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&w)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(
+            taddr),
+        "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7]),
+        "r"(w[8]), "r"(w[9]), "r"(w[10]), "r"(w[11]), "r"(w[12]), "r"(w[13]), "r"(w[14]),
+        "r"(w[15]), "r"(w[16]), "r"(w[17]), "r"(w[18]), "r"(w[19]), "r"(w[20]), "r"(w[21]),
+        "r"(w[22]), "r"(w[23]), "r"(w[24]), "r"(w[25]), "r"(w[26]), "r"(w[27]), "r"(w[28]),
+        "r"(w[29]), "r"(w[30]), "r"(w[31])
+        : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() {
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     uint32_t r;
@@ -235,11 +275,16 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return r;
 }
 
+// Instruction descriptors, kind::f16: fp32 accumulate, bf16 A and B, both K-major,
+// M = 128, N = kNT.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kNT >> 3) << 17) |
+                            ((uint32_t)(128 >> 4) << 24);
+
 struct TcArgs {
     const float *decay, *freq, *amp, *phase;
     float2 *state_out;   // nullable, [B][D][M]
     float4 *coef_out;    // nullable, [D][M]
-    __nv_bfloat16 *y;    // for the plain stores of partially negative boxes
+    __nv_bfloat16 *y;    // for the plain stores of boxes that start before t = 0
     int64_t L;
     int D;
     int ntiles;
@@ -249,9 +294,11 @@ struct TcArgs {
 __global__ void __launch_bounds__(kThreads, 1)
     k_prefill_tc(const __grid_constant__ CUtensorMap tmap_x,
                  const __grid_constant__ CUtensorMap tmap_y, const TcArgs args) {
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>(
-        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    // Align with pointer arithmetic on the __shared__ array (not through an
+    // integer), so the compiler keeps the shared address space and emits
+    // shared-memory loads and stores instead of generic ones.
+    uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const uint32_t sbase = smem_u32(smem);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = blockIdx.x, b = blockIdx.y;
@@ -265,21 +312,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (tid == 0) {
         *abort_flag = 0;
-        for (int i = 0; i < 4; ++i) {
+        for (int i = 0; i < kXSlots; ++i) {
             bar_init(bar(kBarXFull + i), 1);
             bar_init(bar(kBarXEmpty + i), 1);
         }
-        bar_init(bar(kBarBxFull), 1);
-        bar_init(bar(kBarBxEmpty), 1);
-        for (int i = 0; i < 16; ++i) bar_init(bar(kBarTwDone + i), 1);
-        for (int i = 0; i < 8; ++i) bar_init(bar(kBarSFull + i), 1);
         for (int i = 0; i < 2; ++i) {
-            bar_init(bar(kBarUDone + i), 1);
-            bar_init(bar(kBarDEmpty + i), 12);
+            bar_init(bar(kBarBxFull + i), kBoxes);
+            bar_init(bar(kBarBxEmpty + i), 4);
+            bar_init(bar(kBarUDone + i), 4);
+            bar_init(bar(kBarDEmpty + i), 8);
             bar_init(bar(kBarYFull + i), 8);
             bar_init(bar(kBarYEmpty + i), 1);
         }
-        bar_init(bar(kBarFinal), 1);
+        for (int i = 0; i < 8; ++i) bar_init(bar(kBarTwDone + i), 1);
+        for (int i = 0; i < 4; ++i) bar_init(bar(kBarFinal + i), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 7) {
@@ -293,7 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    // The producer starts the first loads before the constants are built.
+    // The producer fills the whole ring before the constants are built.
     const int total_boxes = ntiles * kBoxes;
     int issued = 0;
     if (warp == 3 && lane == 0) {
@@ -307,8 +353,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // ---------------------------------------------------- per-channel constants
-    // Stage 1: thread (c, m, quarter) runs powers lambda^n, n in [16 qn, 16 qn + 16).
-    {
+    // Stage 1: thread (c, m, quarter) runs powers lambda^n, n in [16 qn, 16 qn + 16):
+    // the U rows (Re, -Im of c lambda^(n+1)) and the per-mode terms of K[n].
+    if (tid < 512) {
         float *kt = reinterpret_cast<float *>(smem + kOffBx);  // [8][64][16] scratch
         const int c = tid >> 6, m = (tid >> 2) & 15, qn = tid & 3;
         const int pm = (d0 + c) * kModes + m;
@@ -318,41 +365,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (args.coef_out && b == 0 && qn == 0)
             args.coef_out[pm] = make_float4(lam.x, lam.y, cf.x, cf.y);
         float2 pw = lambda_pow(ga, om, (float)(16 * qn));
-        uint8_t *atw = smem + kOffAtw + c * kAtwStride;
-        uint8_t *au = smem + kOffAu + c * kAuStride;
-        const int wrow = 64 + 2 * m;                 // W rows: Re at 64+2m, Im at 65+2m
-        for (int h = 0; h < 2; ++h) {
-            uint32_t re4[4], im4[4];
-            for (int e = 0; e < 8; e += 2) {
-                const int n = 16 * qn + 8 * h + e;
-                const float2 p0 = pw;
-                const float2 p1 = cmul(pw, lam);
-                re4[e / 2] = pack_bf16x2(p0.x, p1.x);
-                im4[e / 2] = pack_bf16x2(p0.y, p1.y);
-                // K table contributions and U rows for n and n+1
-                kt[(c * 64 + n) * 16 + m] = cf.x * p0.x - cf.y * p0.y;
-                kt[(c * 64 + n + 1) * 16 + m] = cf.x * p1.x - cf.y * p1.y;
-                const float2 q0 = cmul(cf, p1);      // c lambda^(n+1)
-                const float2 p2 = cmul(p1, lam);
-                const float2 q1 = cmul(cf, p2);      // c lambda^(n+2)
-                *reinterpret_cast<uint32_t *>(au + (n / 8) * 512 + (m / 4) * 128 + (n % 8) * 16 +
-                                              ((2 * m) % 8) * 2) = pack_bf16x2(q0.x, -q0.y);
-                *reinterpret_cast<uint32_t *>(au + ((n + 1) / 8) * 512 + (m / 4) * 128 +
-                                              ((n + 1) % 8) * 16 + ((2 * m) % 8) * 2) =
-                    pack_bf16x2(q1.x, -q1.y);
-                pw = p2;
-            }
-            const int kb = 2 * qn + h;
-            *reinterpret_cast<uint4 *>(atw + (wrow / 8) * 1024 + kb * 128 + (wrow % 8) * 16) =
-                make_uint4(re4[0], re4[1], re4[2], re4[3]);
-            *reinterpret_cast<uint4 *>(atw + ((wrow + 1) / 8) * 1024 + kb * 128 +
-                                       ((wrow + 1) % 8) * 16) =
-                make_uint4(im4[0], im4[1], im4[2], im4[3]);
+        uint8_t *au = smem + kOffAu + c * kAuStride + (m / 4) * 128 + ((2 * m) % 8) * 2;
+#pragma unroll 4
+        for (int e = 0; e < 16; ++e) {
+            const int n = 16 * qn + e;
+            kt[(c * 64 + n) * 16 + m] = cf.x * pw.x - cf.y * pw.y;       // Re(c lambda^n)
+            pw = cmul(pw, lam);
+            const float2 q = cmul(cf, pw);                               // c lambda^(n+1)
+            *reinterpret_cast<uint32_t *>(au + (n / 8) * 512 + (n % 8) * 16) = pack_bf16x2(q.x, -q.y);
         }
     }
     __syncthreads();
     // Stage 2: K[c][n] = sum_m Re(c_m lambda_m^n)   (Eq. 1 at integer lags)
-    {
+    if (tid < 512) {
         const float *kt = reinterpret_cast<const float *>(smem + kOffBx);
         float *kf = reinterpret_cast<float *>(smem + kOffBx + 8 * 64 * 16 * 4);
         const int c = tid >> 6, n = tid & 63;
@@ -362,25 +387,48 @@ __global__ void __launch_bounds__(kThreads, 1)
         kf[c * 64 + n] = s;
     }
     __syncthreads();
-    // Stage 3: Toeplitz rows in reversed-position coordinates: T[i][p'] = K[i + p' - 63].
-    {
+    // Stage 3: the A operands into TMEM, row R = 32 q + lane of channels e and e + 4:
+    // rows 0-63   T[R][p'] = K[R + p' - 63]        (Toeplitz, reversed positions)
+    // W[k][p'] = (Re, Im) lambda_m^p' (k = 2m + ri) in rows 64-95 for channels 0-3
+    // and in rows 96-127 for channels 4-7; the other 32 rows are zero.
+    if (warp < 16) {
         const float *kf = reinterpret_cast<const float *>(smem + kOffBx + 8 * 64 * 16 * 4);
-        const int c = tid >> 6, i = tid & 63;
-        uint8_t *atw = smem + kOffAtw + c * kAtwStride;
-        for (int kb = 0; kb < 8; ++kb) {
-            float v[8];
+        const int q = warp & 3, e = warp >> 2;
+        const int R = 32 * q + lane;
+        for (int cc = 0; cc < 2; ++cc) {
+            const int c = e + 4 * cc;
+            uint32_t w[32];
+            if (q < 2) {
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                const int lag = i + 8 * kb + e - 63;
-                v[e] = lag >= 0 ? kf[c * 64 + lag] : 0.0f;
+                for (int k = 0; k < 32; ++k) {
+                    const int l0 = R + 2 * k - 63, l1 = l0 + 1;
+                    w[k] = pack_bf16x2(l0 >= 0 ? kf[c * 64 + l0] : 0.0f, l1 >= 0 ? kf[c * 64 + l1] : 0.0f);
+                }
+            } else if ((q == 2) == (c < 4)) {
+                const int m = lane >> 1, ri = lane & 1;
+                const int pm = (d0 + c) * kModes + m;
+                const float2 lam = lambda_pow(args.decay[pm], args.freq[pm], 1.0f);
+                float2 pw = make_float2(1.0f, 0.0f);
+#pragma unroll
+                for (int k = 0; k < 32; ++k) {
+                    const float2 v0 = pw;
+                    pw = cmul(pw, lam);
+                    const float2 v1 = pw;
+                    pw = cmul(pw, lam);
+                    w[k] = pack_bf16x2(ri ? v0.y : v0.x, ri ? v1.y : v1.x);
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < 32; ++k) w[k] = 0u;
             }
-            *reinterpret_cast<uint4 *>(atw + (i / 8) * 1024 + kb * 128 + (i % 8) * 16) =
-                make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]),
-                           pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+            tmem_st32(tmem + ((uint32_t)(32 * q) << 16) + kTmemA + c * 32, w);
         }
+        tmem_wait_st();
     }
     fence_async_smem();
+    tc_fence_before();
     __syncthreads();
+    tc_fence_after();
 
     const int quarter = warp & 3;
     if (warp == 3) {
@@ -397,105 +445,59 @@ __global__ void __launch_bounds__(kThreads, 1)
                             bar(kBarXFull + slot));
             }
             // Drain: every issued load must land before this CTA may exit.
-            const int first_unconsumed = issued > kXSlots ? issued - kXSlots : 0;
-            for (int k = first_unconsumed; k < issued; ++k) {
+            const int first = issued > kXSlots ? issued - kXSlots : 0;
+            for (int k = first; k < issued; ++k) {
                 const uint32_t slot = k % kXSlots, fill = k / kXSlots;
-                const uint64_t t0 = globaltimer();
+                const long long t0 = clock64();
                 while (!bar_try(bar(kBarXFull + slot), fill & 1))
-                    if (globaltimer() - t0 > kWaitLimitNs) break;
+                    if (clock64() - t0 > kWaitLimitCycles) break;
             }
         }
         __syncwarp();
-    } else if (warp == 15) {
-        // ---------------------------------------------------- transposer
+    } else if (warp == 10 || warp == 14 || warp == 16 || warp == 17) {
+        // ---------------------------------------------------- transposers (box tq of each tile)
+        const int tq = warp == 10 ? 0 : warp == 14 ? 1 : warp - 14;
         for (int j = 0; j < ntiles; ++j) {
-            if (!wait_bar(bar(kBarBxEmpty), (j & 1) ^ 1, abort_flag)) break;
-            bool ok = true;
-            for (int q = 0; q < kBoxes && ok; ++q) {
-                const int qg = j * kBoxes + q;
-                const uint32_t slot = qg % kXSlots;
-                if (!wait_bar(bar(kBarXFull + slot), (qg / kXSlots) & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t xs = sbase + kOffX + slot * (kBox * 16);
-#pragma unroll 2
-                for (int sb = 0; sb < 8; ++sb) {
-                    const uint32_t src = xs + (32 * sb + 8 * (lane >> 3) + (7 - (lane & 7))) * 16;
-                    uint32_t r0, r1, r2, r3;
-                    asm volatile(
-                        "ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-                        : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                        : "r"(src)
-                        : "memory");
-                    const int c = lane & 7, mq = lane >> 3;
-                    const int tb = 32 * q + 4 * sb + mq;      // 8-token block in the tile
-                    const int n = tb >> 3, kb = 7 - (tb & 7);
-                    const uint32_t dst =
-                        sbase + kOffBx + c * kBxStride + (n >> 3) * 1024 + kb * 128 + (n & 7) * 16;
-                    asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1,%2,%3,%4};" ::"r"(
-                                     dst),
-                                 "r"(r0), "r"(r1), "r"(r2), "r"(r3)
-                                 : "memory");
-                }
-                __syncwarp();
-                if (lane == 0) bar_arrive(bar(kBarXEmpty + slot));
+            const int buf = j & 1, use = j >> 1;
+            const int k = j * kBoxes + tq;
+            const uint32_t slot = k % kXSlots;
+            if (!wait_bar(bar(kBarBxEmpty + buf), (use & 1) ^ 1, abort_flag)) break;
+            if (!wait_bar(bar(kBarXFull + slot), (k / kXSlots) & 1, abort_flag)) break;
+            const uint32_t xs = sbase + kOffX + slot * (kBox * 16);
+            uint32_t r[8][4];
+#pragma unroll
+            for (int sb = 0; sb < 8; ++sb) {
+                const uint32_t src = xs + (32 * sb + 8 * (lane >> 3) + (7 - (lane & 7))) * 16;
+                asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                             : "=r"(r[sb][0]), "=r"(r[sb][1]), "=r"(r[sb][2]), "=r"(r[sb][3])
+                             : "r"(src)
+                             : "memory");
             }
-            if (!ok) break;
+            __syncwarp();
+            if (lane == 0) bar_arrive(bar(kBarXEmpty + slot));
+            const int c = lane & 7, mq = lane >> 3;
+            const uint32_t bx = sbase + kOffBx + buf * kBxBuf + c * kBxStride;
+#pragma unroll
+            for (int sb = 0; sb < 8; ++sb) {
+                const int tb = 32 * tq + 4 * sb + mq;    // 8-token block within the tile
+                const int n = tb >> 3, kb = 7 - (tb & 7);
+                const uint32_t dst = bx + (n >> 3) * 1024 + kb * 128 + (n & 7) * 16;
+                asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1,%2,%3,%4};" ::"r"(dst),
+                             "r"(r[sb][0]), "r"(r[sb][1]), "r"(r[sb][2]), "r"(r[sb][3])
+                             : "memory");
+            }
             fence_async_smem();
             __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarBxFull));
+            if (lane == 0) bar_arrive(bar(kBarBxFull + buf));
         }
-    } else if (warp == 7) {
-        // ---------------------------------------------------- MMA issuer
-        if (lane == 0) {
-            for (int j = 0; j < ntiles; ++j) {
-                const int buf = j & 1, use = j >> 1;
-                if (!wait_bar(bar(kBarBxFull), j & 1, abort_flag)) break;
-                if (!wait_bar(bar(kBarDEmpty + buf), (use & 1) ^ 1, abort_flag)) break;
-                tc_fence_after();
-                for (int c = 0; c < kDG; ++c) {
-                    const uint32_t d = tmem + buf * 256 + c * 32;
-                    const uint32_t a0 = sbase + kOffAtw + c * kAtwStride;
-                    const uint32_t b0 = sbase + kOffBx + c * kBxStride;
-#pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        umma_f16(d, umma_desc(a0 + kk * 256, 128, 1024),
-                                 umma_desc(b0 + kk * 256, 128, 1024), kk > 0);
-                    umma_commit(bar(kBarTwDone + buf * 8 + c));
-                }
-                umma_commit(bar(kBarBxEmpty));
-                bool ok = true;
-                for (int c = 0; c < kDG; ++c) {
-                    if (!wait_bar(bar(kBarSFull + c), j & 1, abort_flag)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t d = tmem + buf * 256 + c * 32;
-                    const uint32_t a0 = sbase + kOffAu + c * kAuStride;
-                    const uint32_t b0 = sbase + kOffBs + c * kBsStride;
-#pragma unroll
-                    for (int kk = 0; kk < 2; ++kk)
-                        umma_f16(d, umma_desc(a0 + kk * 256, 128, 512),
-                                 umma_desc(b0 + kk * 2 * kBsLbo, kBsLbo, kBsSbo), 1);
-                }
-                if (!ok) break;
-                umma_commit(bar(kBarUDone + buf));
-            }
-            // Drain: all issued MMAs complete before TMEM is released.
-            umma_commit(bar(kBarFinal));
-            const uint64_t t0 = globaltimer();
-            while (!bar_try(bar(kBarFinal), 0))
-                if (globaltimer() - t0 > kWaitLimitNs) break;
-        }
-        __syncwarp();
+    } else if (warp == 18) {
+        // Idle.
     } else if (warp == 11) {
         // ---------------------------------------------------- y store issuer
         for (int j = 0; j < ntiles; ++j) {
             bool ok = true;
-            for (int nb = 0; nb < 4; ++nb) {
-                const int ng = j * 4 + nb;
+            for (int nb = 0; nb < 2; ++nb) {
+                const int ng = j * 2 + nb;
                 const uint32_t slot = ng % kYSlots;
                 if (!wait_bar(bar(kBarYFull + slot), (ng / kYSlots) & 1, abort_flag)) {
                     ok = false;
@@ -526,53 +528,115 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) break;
         }
         if (lane == 0) tma_store_wait_all();
-    } else if (quarter == 2) {
-        // ---------------------------------------------------- scan (rows 64..95)
-        const int sidx = warp >> 2;                 // 0..3 -> channels 2 sidx, 2 sidx + 1
-        const int r = lane, m = r >> 1, ri = r & 1;
-        float2 LC[2], carry[2];
-        for (int cc = 0; cc < 2; ++cc) {
-            const int pm = (d0 + 2 * sidx + cc) * kModes + m;
-            LC[cc] = lambda_pow(args.decay[pm], args.freq[pm], (float)kC);
-            carry[cc] = make_float2(0.0f, 0.0f);
-        }
-        for (int j = 0; j < ntiles; ++j) {
-            const int buf = j & 1, use = j >> 1;
-            bool ok = true;
-            for (int cc = 0; cc < 2; ++cc) {
-                const int c = 2 * sidx + cc;
-                if (!wait_bar(bar(kBarTwDone + buf * 8 + c), use & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                uint32_t v[32];
-                RLM_TMEM_LD32(tmem + (64u << 16) + buf * 256 + c * 32, v);
-                tmem_wait_ld();
-                uint8_t *bs = smem + kOffBs + c * kBsStride + (m / 4) * kBsLbo + ((2 * m) % 8) * 2;
-                float2 S = carry[cc];
-                const float2 lc = LC[cc];
-#pragma unroll
-                for (int n = 0; n < kNT; ++n) {
-                    const float mine = __uint_as_float(v[n]);
-                    const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
-                    const float2 Ln = ri ? make_float2(other, mine) : make_float2(mine, other);
-                    if ((n >> 4) == ri)
-                        *reinterpret_cast<uint32_t *>(bs + (n >> 3) * kBsSbo + (n & 7) * 16) =
-                            pack_bf16x2(S.x, S.y);
-                    S = cfma(lc, S, Ln);
-                }
-                carry[cc] = S;
-                if (j == ntiles - 1 && args.state_out && ri == 0)
-                    args.state_out[((int64_t)b * D + d0 + c) * kModes + m] = S;
-                fence_async_smem();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) bar_arrive(bar(kBarSFull + c));
+        __syncwarp();
+    } else if (warp == 2 || warp == 6 || warp == 7 || warp == 15) {
+        // ------------------------------------------ scan + MMA issue
+        // Warp sidx owns channels cA = 2 sidx and cB = cA + 1 end to end: it issues
+        // their Toeplitz/state MMAs one tile ahead, scans the chunk states, writes
+        // the carried states and issues the up-projection MMAs.
+        // Channels 0-3 keep their state rows in TMEM lanes 64-95 (warps 2, 6),
+        // channels 4-7 in lanes 96-127 (warps 7, 15), so the scans run on two
+        // SM sub-partitions.
+        const int sidx = warp == 2 ? 0 : warp == 6 ? 1 : warp == 7 ? 2 : 3;
+        const uint32_t st_lane = sidx < 2 ? 64u : 96u;
+        const int cA = 2 * sidx, cB = cA + 1;
+        // After a transpose through shared memory, lane l owns one complex
+        // recurrence: channel ch = l >> 4 of the pair, mode mm = l & 15.
+        const int ch = lane >> 4, mm = lane & 15;
+        const int pmL = (d0 + cA + ch) * kModes + mm;
+        const float2 LC = lambda_pow(args.decay[pmL], args.freq[pmL], (float)kC);
+        float2 S = make_float2(0.0f, 0.0f);
+        float *stage = reinterpret_cast<float *>(smem + kOffSt + sidx * kStWarp);   // [2][16][32]
+        const int bsoff = (cA + ch) * kBsStride + (mm / 4) * kBsLbo + ((2 * mm) % 8) * 2;
+        // Descriptors (advanced by adding byte offsets >> 4 to the address field).
+        const uint64_t dx0 = umma_desc(sbase + kOffBx + cA * kBxStride, 128, 1024);
+        const uint64_t dx1 = umma_desc(sbase + kOffBx + cB * kBxStride, 128, 1024);
+        const uint64_t du0 = umma_desc(sbase + kOffAu + cA * kAuStride, 128, 512);
+        const uint64_t du1 = umma_desc(sbase + kOffAu + cB * kAuStride, 128, 512);
+        const uint64_t ds0 = umma_desc(sbase + kOffBs + cA * kBsStride, kBsLbo, kBsSbo);
+        const uint64_t ds1 = umma_desc(sbase + kOffBs + cB * kBsStride, kBsLbo, kBsSbo);
+        const uint32_t aA = tmem + kTmemA + cA * 32, aB = tmem + kTmemA + cB * 32;
+
+        // Issue the Toeplitz/state MMA chains of tile jn (waits for its drives and
+        // for the epilogue to have drained the accumulator buffer).
+        // With block == false it returns false at once if the inputs are not ready
+        // (the caller then issues after its scan instead).
+        auto issue_tw = [&](int jn, bool block) -> bool {
+            const int bn = jn & 1, un = jn >> 1;
+            if (!block) {
+                const bool ready = bar_test(bar(kBarBxFull + bn), un & 1) &&
+                                   bar_test(bar(kBarDEmpty + bn), (un & 1) ^ 1);
+                if (!__all_sync(0xffffffffu, ready)) return false;
+            } else {
+                if (!wait_bar(bar(kBarBxFull + bn), un & 1, abort_flag)) return false;
+                if (!wait_bar(bar(kBarDEmpty + bn), (un & 1) ^ 1, abort_flag)) return false;
             }
-            if (!ok) break;
-            if (lane == 0) bar_arrive(bar(kBarDEmpty + buf));
+            if (lane == 0) {
+                tc_fence_after();
+                const uint64_t xo = (uint64_t)((bn * kBxBuf) >> 4);
+                const uint32_t dA = tmem + bn * 128 + cA * 16, dB = tmem + bn * 128 + cB * 16;
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) umma_ts(dA, aA + kk * 8, dx0 + xo + kk * 16, kIdesc, kk > 0);
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) umma_ts(dB, aB + kk * 8, dx1 + xo + kk * 16, kIdesc, kk > 0);
+                umma_commit(bar(kBarTwDone + bn * 4 + sidx));
+                umma_commit(bar(kBarBxEmpty + bn));
+            }
+            __syncwarp();
+            return true;
+        };
+
+        bool ok = ntiles > 0 ? issue_tw(0, true) : true;
+        for (int j = 0; j < ntiles && ok; ++j) {
+            const int buf = j & 1, use = j >> 1;
+            const bool early = j + 1 < ntiles && issue_tw(j + 1, false);
+            if (!wait_bar(bar(kBarTwDone + buf * 4 + sidx), use & 1, abort_flag)) break;
+            tc_fence_after();
+            uint32_t vA[16], vB[16];
+            tmem_ld16(tmem + (st_lane << 16) + buf * 128 + cA * 16, vA);
+            tmem_ld16(tmem + (st_lane << 16) + buf * 128 + cB * 16, vB);
+            tmem_wait_ld();
+            // stage[ch][n][row]: lane = state row (2m + Re/Im) of both channels
+#pragma unroll
+            for (int n = 0; n < kNT; ++n) {
+                stage[(0 * 16 + n) * 32 + lane] = __uint_as_float(vA[n]);
+                stage[(1 * 16 + n) * 32 + lane] = __uint_as_float(vB[n]);
+            }
+            __syncwarp();
+            uint8_t *bs = smem + kOffBs + buf * kBsBuf + bsoff;
+#pragma unroll
+            for (int n = 0; n < kNT; ++n) {
+                const float2 Ln = *reinterpret_cast<const float2 *>(&stage[(ch * 16 + n) * 32 + 2 * mm]);
+                *reinterpret_cast<uint32_t *>(bs + (n >> 3) * kBsSbo + (n & 7) * 16) = pack_bf16x2(S.x, S.y);
+                S = cfma(LC, S, Ln);
+            }
+            __syncwarp();
+            if (j == ntiles - 1 && args.state_out)
+                args.state_out[((int64_t)b * D + d0 + cA + ch) * kModes + mm] = S;
+            fence_async_smem();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                tc_fence_after();
+                const uint64_t so = (uint64_t)((buf * kBsBuf) >> 4);
+                const uint32_t dA = tmem + buf * 128 + cA * 16, dB = tmem + buf * 128 + cB * 16;
+#pragma unroll
+                for (int kk = 0; kk < 2; ++kk) umma_ss(dA, du0 + kk * 16, ds0 + so + kk * 18, kIdesc, 1);
+#pragma unroll
+                for (int kk = 0; kk < 2; ++kk) umma_ss(dB, du1 + kk * 16, ds1 + so + kk * 18, kIdesc, 1);
+                umma_commit(bar(kBarUDone + buf));
+            }
+            __syncwarp();
+            if (j + 1 < ntiles && !early && !issue_tw(j + 1, true)) break;
         }
+        // Drain: all MMAs this warp issued complete before TMEM is released.
+        if (lane == 0) {
+            umma_commit(bar(kBarFinal + sidx));
+            const long long t0 = clock64();
+            while (!bar_try(bar(kBarFinal + sidx), 0))
+                if (clock64() - t0 > kWaitLimitCycles) break;
+        }
+        __syncwarp();
     } else {
         // ---------------------------------------------------- epilogue (rows 0..63)
         const int e = warp >> 2;                     // 0..3: chunk pair within a block
@@ -582,14 +646,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!wait_bar(bar(kBarUDone + buf), use & 1, abort_flag)) break;
             tc_fence_after();
             bool ok = true;
-            for (int nb = 0; nb < 4; ++nb) {
-                const int ng = j * 4 + nb;
+            for (int nb = 0; nb < 2; ++nb) {
+                const int ng = j * 2 + nb;
                 const uint32_t slot = ng % kYSlots;
                 const int n0 = 8 * nb + 2 * e;
                 uint32_t v[kDG][2];
 #pragma unroll
                 for (int c = 0; c < kDG; ++c)
-                    tmem_ld2(tmem + ((uint32_t)(32 * quarter) << 16) + buf * 256 + c * 32 + n0,
+                    tmem_ld2(tmem + ((uint32_t)(32 * quarter) << 16) + buf * 128 + c * 16 + n0,
                              v[c][0], v[c][1]);
                 tmem_wait_ld();
                 if (!wait_bar(bar(kBarYEmpty + slot), ((ng / kYSlots) & 1) ^ 1, abort_flag)) {
