@@ -27,8 +27,8 @@
 // state in registers, so no CTA waits on another.
 //
 // Data movement per tile (1024 tokens x 8 channels):
-//   TMA (3-D map over [B][L][D], zero fill outside the sequence) -> 24-box ring
-//   -> ldmatrix.trans / stmatrix by four transposer warps into the per-channel
+//   TMA (3-D map over [B][L][D], zero fill outside the sequence) -> 20-box ring
+//   -> ldmatrix.trans / stmatrix by three transposer warps into the per-channel
 //      K-major B operand (double-buffered; the positions of a chunk reversed so
 //      that the A operand's Toeplitz rows read K[i + p' - 63])
 //   -> tcgen05.mma -> TMEM -> scan warps -> B operand of the up-projection
@@ -37,14 +37,13 @@
 // TMEM (512 columns): two accumulator buffers of 8 channels x 16 columns, and
 // the 8 channels' A operands (128 lanes x 32 columns of packed bf16 pairs).
 //
-// Warp roles (19 warps): TMEM lane quarter q = warp % 4 (also the SM
+// Warp roles (21 warps): TMEM lane quarter q = warp % 4 (also the SM
 // sub-partition the warp runs on) decides which rows of D a warp may read.
-// Warps 0,1,4,5,8,9,12,13: epilogue (rows 0-63).  Warps 2, 6 (quarter 2) and
-// 7, 15 (quarter 3): two channels each, end to end -- they issue those
-// channels' MMAs (one tile ahead), scan their states and issue the
-// up-projection; four issuing warps keep the tensor pipe busy where one
-// issuing thread could not.  Warp 3: TMA producer; warp 11: TMA store issuer;
-// warps 10, 14, 16, 17: transposers; warp 18 idle; warp 7 also allocates TMEM.
+// Warps 0,1,4,5,8,9,12,13: epilogue (rows 0-63).  Warps 2, 6, 10, 14 (quarter
+// 2) and 3, 7, 11, 15 (quarter 3): one channel each, end to end -- issue the
+// channel's MMAs (one tile ahead), scan its states, issue the up-projection.
+// Warps 16-18: transposers; warp 19: TMA producer; warp 20: TMA store issuer
+// and TMEM allocation.
 //
 // Every wait is bounded: after kWaitLimitCycles the waiting thread sets a shared
 // abort flag and the device status word (RLM_ERR_TIMEOUT); all roles then leave
@@ -73,44 +72,47 @@ constexpr int kBox = 256;              // TMA box rows
 constexpr int kBoxes = kTile / kBox;   // 4 per tile
 constexpr int kXSlots = 20;            // x ring depth (boxes)
 constexpr int kYSlots = 2;             // y ring depth (blocks of 8 chunks)
-constexpr int kWarps = 19;
+constexpr int kWarps = 21;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTmemCols = 512;
 constexpr int kTmemA = 256;            // first TMEM column of the A operands
 constexpr long long kWaitLimitCycles = 4000000000ll;  // about 2 s at 2 GHz
+constexpr int kTransposers = 3;
 
 // Shared memory map (bytes from a 1024-aligned base).
 constexpr int kAuStride = 4096;        // 64 real rows x 64 B; rows 64-127 alias the next buffer
 constexpr int kBxStride = 2048 + 16;   // 16 rows x 128 B, +16 so stmatrix rows hit distinct banks
 constexpr int kBxBuf = kDG * kBxStride;
-constexpr int kBsLbo = 144, kBsSbo = 576, kBsStride = 2 * kBsSbo + 64;  // +64: two channels' rows in disjoint banks
+constexpr int kBsLbo = 144, kBsSbo = 576, kBsStride = 2 * kBsSbo + 64;
 constexpr int kBsBuf = kDG * kBsStride;
 constexpr int kOffAu = 0;
 constexpr int kOffBx = kOffAu + kDG * kAuStride;             // 32768
 constexpr int kOffBs = kOffBx + 2 * kBxBuf;                  // 65792
-constexpr int kOffSt = kOffBs + 2 * kBsBuf;                  // per scan warp: [2 ch][16 chunks][32 rows] fp32
-constexpr int kStWarp = 2 * 16 * 32 * 4;
-constexpr int kOffX = kOffSt + 4 * kStWarp;
+constexpr int kOffX = kOffBs + 2 * kBsBuf;                   // 85248
 constexpr int kOffY = kOffX + kXSlots * kBox * 16;
 constexpr int kOffBar = kOffY + kYSlots * 512 * 16;
 constexpr int kNumBars = 128;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;             // + alignment slack
 static_assert(kOffX % 128 == 0 && kOffY % 128 == 0, "TMA buffers need 128-byte alignment");
-static_assert(kOffBx + 8 * 64 * 16 * 4 + 8 * 64 * 4 <= kOffX, "prologue scratch does not fit");
+// Prologue tables (reuse the B-operand region before the first tile):
+constexpr int kOffWtab = kOffBx;                     // [8 ch][32 rows][32 words]: W rows, packed bf16 pairs
+constexpr int kOffTpair = kOffWtab + 8 * 32 * 32 * 4;  // [8 ch][2][64 words]: Toeplitz pairs
+constexpr int kOffKp = kOffTpair + 8 * 2 * 64 * 4;     // [2 halves][8 ch][64] fp32 partial sums of K
+static_assert(kOffKp + 2 * 8 * 64 * 4 <= kOffX, "prologue tables do not fit");
 
 // Barrier indices.
 constexpr int kBarXFull = 0;                    // [kXSlots]
 constexpr int kBarXEmpty = kXSlots;             // [kXSlots]
 constexpr int kBarBxFull = 2 * kXSlots;         // [2]
 constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]
-constexpr int kBarTwDone = kBarBxEmpty + 2;     // [2][4]: per buffer, per scan warp
-constexpr int kBarUDone = kBarTwDone + 8;       // [2]
+constexpr int kBarTwDone = kBarBxEmpty + 2;     // [2][8]: per buffer, per channel
+constexpr int kBarUDone = kBarTwDone + 16;      // [2]
 constexpr int kBarDEmpty = kBarUDone + 2;       // [2]
 constexpr int kBarYFull = kBarDEmpty + 2;       // [2]
 constexpr int kBarYEmpty = kBarYFull + 2;       // [2]
-constexpr int kBarFinal = kBarYEmpty + 2;       // [4]
-static_assert(kBarFinal + 4 <= kNumBars, "too many barriers");
+constexpr int kBarFinal = kBarYEmpty + 2;       // [8]
+static_assert(kBarFinal + 8 <= kNumBars, "too many barriers");
 
 
 // ------------------------------------------------------------ PTX wrappers
@@ -318,17 +320,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int i = 0; i < 2; ++i) {
             bar_init(bar(kBarBxFull + i), kBoxes);
-            bar_init(bar(kBarBxEmpty + i), 4);
-            bar_init(bar(kBarUDone + i), 4);
+            bar_init(bar(kBarBxEmpty + i), kDG);
+            bar_init(bar(kBarUDone + i), kDG);
             bar_init(bar(kBarDEmpty + i), 8);
             bar_init(bar(kBarYFull + i), 8);
             bar_init(bar(kBarYEmpty + i), 1);
         }
-        for (int i = 0; i < 8; ++i) bar_init(bar(kBarTwDone + i), 1);
-        for (int i = 0; i < 4; ++i) bar_init(bar(kBarFinal + i), 1);
+        for (int i = 0; i < 16; ++i) bar_init(bar(kBarTwDone + i), 1);
+        for (int i = 0; i < 8; ++i) bar_init(bar(kBarFinal + i), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 7) {
+    if (warp == 20) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(tmem_slot)),
                      "r"(kTmemCols));
@@ -342,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // The producer fills the whole ring before the constants are built.
     const int total_boxes = ntiles * kBoxes;
     int issued = 0;
-    if (warp == 3 && lane == 0) {
+    if (warp == 19 && lane == 0) {
         for (; issued < total_boxes && issued < kXSlots; ++issued) {
             const int jt = issued / kBoxes, q = issued % kBoxes;
             const uint32_t slot = issued % kXSlots;
@@ -353,10 +355,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // ---------------------------------------------------- per-channel constants
-    // Stage 1: thread (c, m, quarter) runs powers lambda^n, n in [16 qn, 16 qn + 16):
-    // the U rows (Re, -Im of c lambda^(n+1)) and the per-mode terms of K[n].
+    // Stage 1: thread (c, m, qn) runs the powers lambda^n, n in [16 qn, 16 qn + 16),
+    // of mode m of channel c: the U rows (Re, -Im of c lambda^(n+1)), the W-row
+    // words (lambda^n packed in pairs of n), and Re(c lambda^n) summed over the
+    // eight modes of its warp (a fixed shuffle tree) into Kp[half][c][n].
     if (tid < 512) {
-        float *kt = reinterpret_cast<float *>(smem + kOffBx);  // [8][64][16] scratch
         const int c = tid >> 6, m = (tid >> 2) & 15, qn = tid & 3;
         const int pm = (d0 + c) * kModes + m;
         const float ga = args.decay[pm], om = args.freq[pm];
@@ -366,25 +369,54 @@ __global__ void __launch_bounds__(kThreads, 1)
             args.coef_out[pm] = make_float4(lam.x, lam.y, cf.x, cf.y);
         float2 pw = lambda_pow(ga, om, (float)(16 * qn));
         uint8_t *au = smem + kOffAu + c * kAuStride + (m / 4) * 128 + ((2 * m) % 8) * 2;
-#pragma unroll 4
+        uint32_t wre[8], wim[8];
+        float kv[16];
+#pragma unroll
         for (int e = 0; e < 16; ++e) {
             const int n = 16 * qn + e;
-            kt[(c * 64 + n) * 16 + m] = cf.x * pw.x - cf.y * pw.y;       // Re(c lambda^n)
-            pw = cmul(pw, lam);
-            const float2 q = cmul(cf, pw);                               // c lambda^(n+1)
+            kv[e] = cf.x * pw.x - cf.y * pw.y;                          // Re(c lambda^n)
+            const float2 nx = cmul(pw, lam);                             // lambda^(n+1)
+            if ((e & 1) == 0) {
+                wre[e >> 1] = pack_bf16x2(pw.x, nx.x);
+                wim[e >> 1] = pack_bf16x2(pw.y, nx.y);
+            }
+            const float2 q = cmul(cf, nx);                               // c lambda^(n+1)
             *reinterpret_cast<uint32_t *>(au + (n / 8) * 512 + (n % 8) * 16) = pack_bf16x2(q.x, -q.y);
+            pw = nx;
+        }
+        uint4 *wt = reinterpret_cast<uint4 *>(smem + kOffWtab) + (c * 32 + 2 * m) * 8 + 2 * qn;
+        wt[0] = make_uint4(wre[0], wre[1], wre[2], wre[3]);
+        wt[1] = make_uint4(wre[4], wre[5], wre[6], wre[7]);
+        wt[8] = make_uint4(wim[0], wim[1], wim[2], wim[3]);
+        wt[9] = make_uint4(wim[4], wim[5], wim[6], wim[7]);
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+            float v = kv[e];
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            v += __shfl_xor_sync(0xffffffffu, v, 8);
+            v += __shfl_xor_sync(0xffffffffu, v, 16);
+            kv[e] = v;
+        }
+        if ((lane >> 2) == 0) {
+            float *kp = reinterpret_cast<float *>(smem + kOffKp) + ((m >> 3) * 8 + c) * 64 + 16 * qn;
+#pragma unroll
+            for (int e = 0; e < 16; ++e) kp[e] = kv[e];
         }
     }
     __syncthreads();
-    // Stage 2: K[c][n] = sum_m Re(c_m lambda_m^n)   (Eq. 1 at integer lags)
+    // Stage 2: K[c][n] = Kp[0][c][n] + Kp[1][c][n] (Eq. 1 at integer lags), as
+    // zero-padded pair tables kz(i) = K[i - 63] (0 for i < 63):
+    // P0[c][i] = (kz(2i), kz(2i+1)), P1[c][i] = (kz(2i+1), kz(2i+2)).
     if (tid < 512) {
-        const float *kt = reinterpret_cast<const float *>(smem + kOffBx);
-        float *kf = reinterpret_cast<float *>(smem + kOffBx + 8 * 64 * 16 * 4);
-        const int c = tid >> 6, n = tid & 63;
-        float s = 0.0f;
-#pragma unroll
-        for (int m = 0; m < kModes; ++m) s += kt[(c * 64 + n) * 16 + m];
-        kf[c * 64 + n] = s;
+        const float *kp = reinterpret_cast<const float *>(smem + kOffKp);
+        const int c = tid >> 6, i = tid & 63;
+        auto kz = [&](int idx) -> float {
+            const int n = idx - 63;
+            return (n >= 0 && n < 64) ? kp[c * 64 + n] + kp[(8 + c) * 64 + n] : 0.0f;
+        };
+        uint32_t *tp = reinterpret_cast<uint32_t *>(smem + kOffTpair) + c * 128;
+        tp[i] = pack_bf16x2(kz(2 * i), kz(2 * i + 1));
+        tp[64 + i] = pack_bf16x2(kz(2 * i + 1), kz(2 * i + 2));
     }
     __syncthreads();
     // Stage 3: the A operands into TMEM, row R = 32 q + lane of channels e and e + 4:
@@ -392,30 +424,22 @@ __global__ void __launch_bounds__(kThreads, 1)
     // W[k][p'] = (Re, Im) lambda_m^p' (k = 2m + ri) in rows 64-95 for channels 0-3
     // and in rows 96-127 for channels 4-7; the other 32 rows are zero.
     if (warp < 16) {
-        const float *kf = reinterpret_cast<const float *>(smem + kOffBx + 8 * 64 * 16 * 4);
         const int q = warp & 3, e = warp >> 2;
         const int R = 32 * q + lane;
         for (int cc = 0; cc < 2; ++cc) {
             const int c = e + 4 * cc;
             uint32_t w[32];
             if (q < 2) {
+                const uint32_t *tp = reinterpret_cast<const uint32_t *>(smem + kOffTpair) + c * 128 +
+                                     ((R & 1) ? 64 + (R >> 1) : (R >> 1));
 #pragma unroll
-                for (int k = 0; k < 32; ++k) {
-                    const int l0 = R + 2 * k - 63, l1 = l0 + 1;
-                    w[k] = pack_bf16x2(l0 >= 0 ? kf[c * 64 + l0] : 0.0f, l1 >= 0 ? kf[c * 64 + l1] : 0.0f);
-                }
+                for (int k = 0; k < 32; ++k) w[k] = tp[k];
             } else if ((q == 2) == (c < 4)) {
-                const int m = lane >> 1, ri = lane & 1;
-                const int pm = (d0 + c) * kModes + m;
-                const float2 lam = lambda_pow(args.decay[pm], args.freq[pm], 1.0f);
-                float2 pw = make_float2(1.0f, 0.0f);
+                const uint4 *wt = reinterpret_cast<const uint4 *>(smem + kOffWtab) + (c * 32 + lane) * 8;
 #pragma unroll
-                for (int k = 0; k < 32; ++k) {
-                    const float2 v0 = pw;
-                    pw = cmul(pw, lam);
-                    const float2 v1 = pw;
-                    pw = cmul(pw, lam);
-                    w[k] = pack_bf16x2(ri ? v0.y : v0.x, ri ? v1.y : v1.x);
+                for (int k = 0; k < 8; ++k) {
+                    const uint4 v = wt[k];
+                    w[4 * k] = v.x; w[4 * k + 1] = v.y; w[4 * k + 2] = v.z; w[4 * k + 3] = v.w;
                 }
             } else {
 #pragma unroll
@@ -431,7 +455,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
 
     const int quarter = warp & 3;
-    if (warp == 3) {
+    if (warp == 19) {
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
             for (; issued < total_boxes; ++issued) {
@@ -454,14 +478,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         __syncwarp();
-    } else if (warp == 10 || warp == 14 || warp == 16 || warp == 17) {
-        // ---------------------------------------------------- transposers (box tq of each tile)
-        const int tq = warp == 10 ? 0 : warp == 14 ? 1 : warp - 14;
-        for (int j = 0; j < ntiles; ++j) {
+    } else if (warp >= 16 && warp < 16 + kTransposers) {
+        // ---------------------------------------------------- transposers (boxes k = t mod 3)
+        for (int k = warp - 16; k < total_boxes; k += kTransposers) {
+            const int j = k / kBoxes, tq = k % kBoxes;
             const int buf = j & 1, use = j >> 1;
-            const int k = j * kBoxes + tq;
             const uint32_t slot = k % kXSlots;
-            if (!wait_bar(bar(kBarBxEmpty + buf), (use & 1) ^ 1, abort_flag)) break;
             if (!wait_bar(bar(kBarXFull + slot), (k / kXSlots) & 1, abort_flag)) break;
             const uint32_t xs = sbase + kOffX + slot * (kBox * 16);
             uint32_t r[8][4];
@@ -475,6 +497,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             __syncwarp();
             if (lane == 0) bar_arrive(bar(kBarXEmpty + slot));
+            if (!wait_bar(bar(kBarBxEmpty + buf), (use & 1) ^ 1, abort_flag)) break;
             const int c = lane & 7, mq = lane >> 3;
             const uint32_t bx = sbase + kOffBx + buf * kBxBuf + c * kBxStride;
 #pragma unroll
@@ -490,9 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             __syncwarp();
             if (lane == 0) bar_arrive(bar(kBarBxFull + buf));
         }
-    } else if (warp == 18) {
-        // Idle.
-    } else if (warp == 11) {
+    } else if (warp == 20) {
         // ---------------------------------------------------- y store issuer
         for (int j = 0; j < ntiles; ++j) {
             bool ok = true;
@@ -529,38 +550,28 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (lane == 0) tma_store_wait_all();
         __syncwarp();
-    } else if (warp == 2 || warp == 6 || warp == 7 || warp == 15) {
-        // ------------------------------------------ scan + MMA issue
-        // Warp sidx owns channels cA = 2 sidx and cB = cA + 1 end to end: it issues
-        // their Toeplitz/state MMAs one tile ahead, scans the chunk states, writes
-        // the carried states and issues the up-projection MMAs.
-        // Channels 0-3 keep their state rows in TMEM lanes 64-95 (warps 2, 6),
-        // channels 4-7 in lanes 96-127 (warps 7, 15), so the scans run on two
-        // SM sub-partitions.
-        const int sidx = warp == 2 ? 0 : warp == 6 ? 1 : warp == 7 ? 2 : 3;
-        const uint32_t st_lane = sidx < 2 ? 64u : 96u;
-        const int cA = 2 * sidx, cB = cA + 1;
-        // After a transpose through shared memory, lane l owns one complex
-        // recurrence: channel ch = l >> 4 of the pair, mode mm = l & 15.
-        const int ch = lane >> 4, mm = lane & 15;
-        const int pmL = (d0 + cA + ch) * kModes + mm;
-        const float2 LC = lambda_pow(args.decay[pmL], args.freq[pmL], (float)kC);
+    } else if (quarter >= 2) {
+        // ------------------------------------------ one channel: scan + MMA issue
+        // Warps 2, 6, 10, 14 own channels 0-3 (state rows in TMEM lanes 64-95);
+        // warps 3, 7, 11, 15 own channels 4-7 (lanes 96-127).  A warp issues its
+        // channel's Toeplitz/state MMA chain one tile ahead, scans the 16 chunk
+        // states (lane 2m holds mode m: Re from its own row, Im from lane 2m+1)
+        // and issues the up-projection.  Eight issuing threads keep the tensor
+        // pipe fed: one tcgen05.mma occupies its issuing thread ~90 cycles.
+        const int c = (quarter - 2) * 4 + (warp >> 2);
+        const uint32_t st_lane = 32u * (uint32_t)quarter;
+        const int m = lane >> 1, ri = lane & 1;
+        const int pm = (d0 + c) * kModes + m;
+        const float2 LC = lambda_pow(args.decay[pm], args.freq[pm], (float)kC);
         float2 S = make_float2(0.0f, 0.0f);
-        float *stage = reinterpret_cast<float *>(smem + kOffSt + sidx * kStWarp);   // [2][16][32]
-        const int bsoff = (cA + ch) * kBsStride + (mm / 4) * kBsLbo + ((2 * mm) % 8) * 2;
-        // Descriptors (advanced by adding byte offsets >> 4 to the address field).
-        const uint64_t dx0 = umma_desc(sbase + kOffBx + cA * kBxStride, 128, 1024);
-        const uint64_t dx1 = umma_desc(sbase + kOffBx + cB * kBxStride, 128, 1024);
-        const uint64_t du0 = umma_desc(sbase + kOffAu + cA * kAuStride, 128, 512);
-        const uint64_t du1 = umma_desc(sbase + kOffAu + cB * kAuStride, 128, 512);
-        const uint64_t ds0 = umma_desc(sbase + kOffBs + cA * kBsStride, kBsLbo, kBsSbo);
-        const uint64_t ds1 = umma_desc(sbase + kOffBs + cB * kBsStride, kBsLbo, kBsSbo);
-        const uint32_t aA = tmem + kTmemA + cA * 32, aB = tmem + kTmemA + cB * 32;
+        const int bsoff = c * kBsStride + (m / 4) * kBsLbo + ((2 * m) % 8) * 2;
+        const uint64_t dx0 = umma_desc(sbase + kOffBx + c * kBxStride, 128, 1024);
+        const uint64_t du0 = umma_desc(sbase + kOffAu + c * kAuStride, 128, 512);
+        const uint64_t ds0 = umma_desc(sbase + kOffBs + c * kBsStride, kBsLbo, kBsSbo);
+        const uint32_t aT = tmem + kTmemA + c * 32;
 
-        // Issue the Toeplitz/state MMA chains of tile jn (waits for its drives and
-        // for the epilogue to have drained the accumulator buffer).
-        // With block == false it returns false at once if the inputs are not ready
-        // (the caller then issues after its scan instead).
+        // Issue the Toeplitz/state MMA chain of tile jn.  With block == false it
+        // returns false at once if its inputs are not ready yet.
         auto issue_tw = [&](int jn, bool block) -> bool {
             const int bn = jn & 1, un = jn >> 1;
             if (!block) {
@@ -574,12 +585,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (lane == 0) {
                 tc_fence_after();
                 const uint64_t xo = (uint64_t)((bn * kBxBuf) >> 4);
-                const uint32_t dA = tmem + bn * 128 + cA * 16, dB = tmem + bn * 128 + cB * 16;
+                const uint32_t d = tmem + bn * 128 + c * 16;
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk) umma_ts(dA, aA + kk * 8, dx0 + xo + kk * 16, kIdesc, kk > 0);
-#pragma unroll
-                for (int kk = 0; kk < 4; ++kk) umma_ts(dB, aB + kk * 8, dx1 + xo + kk * 16, kIdesc, kk > 0);
-                umma_commit(bar(kBarTwDone + bn * 4 + sidx));
+                for (int kk = 0; kk < 4; ++kk) umma_ts(d, aT + kk * 8, dx0 + xo + kk * 16, kIdesc, kk > 0);
+                umma_commit(bar(kBarTwDone + bn * 8 + c));
                 umma_commit(bar(kBarBxEmpty + bn));
             }
             __syncwarp();
@@ -590,40 +599,32 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int j = 0; j < ntiles && ok; ++j) {
             const int buf = j & 1, use = j >> 1;
             const bool early = j + 1 < ntiles && issue_tw(j + 1, false);
-            if (!wait_bar(bar(kBarTwDone + buf * 4 + sidx), use & 1, abort_flag)) break;
+            if (!wait_bar(bar(kBarTwDone + buf * 8 + c), use & 1, abort_flag)) break;
             tc_fence_after();
-            uint32_t vA[16], vB[16];
-            tmem_ld16(tmem + (st_lane << 16) + buf * 128 + cA * 16, vA);
-            tmem_ld16(tmem + (st_lane << 16) + buf * 128 + cB * 16, vB);
+            uint32_t v[16];
+            tmem_ld16(tmem + (st_lane << 16) + buf * 128 + c * 16, v);
             tmem_wait_ld();
-            // stage[ch][n][row]: lane = state row (2m + Re/Im) of both channels
-#pragma unroll
-            for (int n = 0; n < kNT; ++n) {
-                stage[(0 * 16 + n) * 32 + lane] = __uint_as_float(vA[n]);
-                stage[(1 * 16 + n) * 32 + lane] = __uint_as_float(vB[n]);
-            }
-            __syncwarp();
             uint8_t *bs = smem + kOffBs + buf * kBsBuf + bsoff;
 #pragma unroll
             for (int n = 0; n < kNT; ++n) {
-                const float2 Ln = *reinterpret_cast<const float2 *>(&stage[(ch * 16 + n) * 32 + 2 * mm]);
-                *reinterpret_cast<uint32_t *>(bs + (n >> 3) * kBsSbo + (n & 7) * 16) = pack_bf16x2(S.x, S.y);
-                S = cfma(LC, S, Ln);
+                const float mine = __uint_as_float(v[n]);
+                const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
+                if (ri == 0) {
+                    *reinterpret_cast<uint32_t *>(bs + (n >> 3) * kBsSbo + (n & 7) * 16) = pack_bf16x2(S.x, S.y);
+                    S = cfma(LC, S, make_float2(mine, other));
+                }
             }
-            __syncwarp();
-            if (j == ntiles - 1 && args.state_out)
-                args.state_out[((int64_t)b * D + d0 + cA + ch) * kModes + mm] = S;
+            if (j == ntiles - 1 && args.state_out && ri == 0)
+                args.state_out[((int64_t)b * D + d0 + c) * kModes + m] = S;
             fence_async_smem();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {
                 tc_fence_after();
                 const uint64_t so = (uint64_t)((buf * kBsBuf) >> 4);
-                const uint32_t dA = tmem + buf * 128 + cA * 16, dB = tmem + buf * 128 + cB * 16;
+                const uint32_t d = tmem + buf * 128 + c * 16;
 #pragma unroll
-                for (int kk = 0; kk < 2; ++kk) umma_ss(dA, du0 + kk * 16, ds0 + so + kk * 18, kIdesc, 1);
-#pragma unroll
-                for (int kk = 0; kk < 2; ++kk) umma_ss(dB, du1 + kk * 16, ds1 + so + kk * 18, kIdesc, 1);
+                for (int kk = 0; kk < 2; ++kk) umma_ss(d, du0 + kk * 16, ds0 + so + kk * 18, kIdesc, 1);
                 umma_commit(bar(kBarUDone + buf));
             }
             __syncwarp();
@@ -631,9 +632,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         // Drain: all MMAs this warp issued complete before TMEM is released.
         if (lane == 0) {
-            umma_commit(bar(kBarFinal + sidx));
+            umma_commit(bar(kBarFinal + c));
             const long long t0 = clock64();
-            while (!bar_try(bar(kBarFinal + sidx), 0))
+            while (!bar_try(bar(kBarFinal + c), 0))
                 if (clock64() - t0 > kWaitLimitCycles) break;
         }
         __syncwarp();
@@ -684,7 +685,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 7)
+    if (warp == 20)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(kTmemCols));
 }
