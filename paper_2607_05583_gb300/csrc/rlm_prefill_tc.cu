@@ -71,7 +71,7 @@ constexpr int kModes = 16;             // M handled by this kernel
 constexpr int kBox = 256;              // TMA box rows
 constexpr int kBoxes = kTile / kBox;   // 4 per tile
 constexpr int kXSlots = 20;            // x ring depth (boxes)
-constexpr int kYSlots = 2;             // y ring depth (blocks of 8 chunks)
+constexpr int kYSlots = 4;             // y ring depth (blocks of 8 chunks)
 constexpr int kWarps = 21;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTmemCols = 512;
@@ -95,11 +95,16 @@ constexpr int kNumBars = 128;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;             // + alignment slack
 static_assert(kOffX % 128 == 0 && kOffY % 128 == 0, "TMA buffers need 128-byte alignment");
-// Prologue tables (reuse the B-operand region before the first tile):
-constexpr int kOffWtab = kOffBx;                     // [8 ch][32 rows][32 words]: W rows, packed bf16 pairs
-constexpr int kOffTpair = kOffWtab + 8 * 32 * 32 * 4;  // [8 ch][2][64 words]: Toeplitz pairs
+// Prologue tables, in buffers no other role touches before the prologue ends
+// (the transposers already fill the B operand meanwhile):
+constexpr int kOffWtab = kOffY;                        // [8 ch][32 rows][32 words]: W rows, packed bf16 pairs
+constexpr int kOffTpair = kOffBs;                      // [8 ch][2][64 words]: Toeplitz pairs
 constexpr int kOffKp = kOffTpair + 8 * 2 * 64 * 4;     // [2 halves][8 ch][64] fp32 partial sums of K
+static_assert(8 * 32 * 32 * 4 <= kYSlots * 8192, "W table does not fit the y ring");
 static_assert(kOffKp + 2 * 8 * 64 * 4 <= kOffX, "prologue tables do not fit");
+// Named barrier for the 16 warps that build the constants.
+constexpr int kPrologueBarrier = 1;
+constexpr int kPrologueThreads = 512;
 
 // Barrier indices.
 constexpr int kBarXFull = 0;                    // [kXSlots]
@@ -109,9 +114,9 @@ constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]
 constexpr int kBarTwDone = kBarBxEmpty + 2;     // [2][8]: per buffer, per channel
 constexpr int kBarUDone = kBarTwDone + 16;      // [2]
 constexpr int kBarDEmpty = kBarUDone + 2;       // [2]
-constexpr int kBarYFull = kBarDEmpty + 2;       // [2]
-constexpr int kBarYEmpty = kBarYFull + 2;       // [2]
-constexpr int kBarFinal = kBarYEmpty + 2;       // [8]
+constexpr int kBarYFull = kBarDEmpty + 2;       // [kYSlots]
+constexpr int kBarYEmpty = kBarYFull + kYSlots; // [kYSlots]
+constexpr int kBarFinal = kBarYEmpty + kYSlots; // [8]
 static_assert(kBarFinal + 8 <= kNumBars, "too many barriers");
 
 
@@ -323,6 +328,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             bar_init(bar(kBarBxEmpty + i), kDG);
             bar_init(bar(kBarUDone + i), kDG);
             bar_init(bar(kBarDEmpty + i), 8);
+        }
+        for (int i = 0; i < kYSlots; ++i) {
             bar_init(bar(kBarYFull + i), 8);
             bar_init(bar(kBarYEmpty + i), 1);
         }
@@ -355,6 +362,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // ---------------------------------------------------- per-channel constants
+    // Built by warps 0-15 only (synchronised by a named barrier), while the
+    // transposers, the producer and the store issuer start their work.
     // Stage 1: thread (c, m, qn) runs the powers lambda^n, n in [16 qn, 16 qn + 16),
     // of mode m of channel c: the U rows (Re, -Im of c lambda^(n+1)), the W-row
     // words (lambda^n packed in pairs of n), and Re(c lambda^n) summed over the
@@ -403,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int e = 0; e < 16; ++e) kp[e] = kv[e];
         }
     }
-    __syncthreads();
+    if (warp < 16) asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
     // Stage 2: K[c][n] = Kp[0][c][n] + Kp[1][c][n] (Eq. 1 at integer lags), as
     // zero-padded pair tables kz(i) = K[i - 63] (0 for i < 63):
     // P0[c][i] = (kz(2i), kz(2i+1)), P1[c][i] = (kz(2i+1), kz(2i+2)).
@@ -418,7 +427,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tp[i] = pack_bf16x2(kz(2 * i), kz(2 * i + 1));
         tp[64 + i] = pack_bf16x2(kz(2 * i + 1), kz(2 * i + 2));
     }
-    __syncthreads();
+    if (warp < 16) asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
     // Stage 3: the A operands into TMEM, row R = 32 q + lane of channels e and e + 4:
     // rows 0-63   T[R][p'] = K[R + p' - 63]        (Toeplitz, reversed positions)
     // W[k][p'] = (Re, Im) lambda_m^p' (k = 2m + ri) in rows 64-95 for channels 0-3
@@ -448,11 +457,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_st32(tmem + ((uint32_t)(32 * q) << 16) + kTmemA + c * 32, w);
         }
         tmem_wait_st();
+        fence_async_smem();
+        tc_fence_before();
+        asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
+        tc_fence_after();
     }
-    fence_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
 
     const int quarter = warp & 3;
     if (warp == 19) {
@@ -515,10 +524,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp == 20) {
         // ---------------------------------------------------- y store issuer
-        for (int j = 0; j < ntiles; ++j) {
-            bool ok = true;
-            for (int nb = 0; nb < 2; ++nb) {
-                const int ng = j * 2 + nb;
+        // One bulk group per block of 512 rows; up to kYSlots - 2 groups may still
+        // be reading shared memory while the next block is issued.
+        int ng = 0;
+        bool ok = true;
+        for (int j = 0; j < ntiles && ok; ++j) {
+            for (int nb = 0; nb < 2; ++nb, ++ng) {
                 const uint32_t slot = ng % kYSlots;
                 if (!wait_bar(bar(kBarYFull + slot), (ng / kYSlots) & 1, abort_flag)) {
                     ok = false;
@@ -541,14 +552,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (lane == 0) {
                     tma_store_commit();
-                    tma_store_wait_read();
+                    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(kYSlots - 2) : "memory");
                 }
                 __syncwarp();
-                if (lane == 0) bar_arrive(bar(kBarYEmpty + slot));
+                // Groups up to ng - (kYSlots - 2) have finished reading their slots.
+                const int freed = ng - (kYSlots - 2);
+                if (lane == 0 && freed >= 0) bar_arrive(bar(kBarYEmpty + freed % kYSlots));
             }
-            if (!ok) break;
         }
-        if (lane == 0) tma_store_wait_all();
+        if (lane == 0) {
+            tma_store_wait_read();
+            for (int k = ng - (kYSlots - 2); k < ng; ++k)
+                if (k >= 0) bar_arrive(bar(kBarYEmpty + k % kYSlots));
+            tma_store_wait_all();
+        }
         __syncwarp();
     } else if (quarter >= 2) {
         // ------------------------------------------ one channel: scan + MMA issue
