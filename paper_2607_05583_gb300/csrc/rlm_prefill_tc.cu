@@ -37,13 +37,14 @@
 // TMEM (512 columns): two accumulator buffers of 8 channels x 16 columns, and
 // the 8 channels' A operands (128 lanes x 32 columns of packed bf16 pairs).
 //
-// Warp roles (21 warps): TMEM lane quarter q = warp % 4 (also the SM
+// Warp roles (29 warps): TMEM lane quarter q = warp % 4 (also the SM
 // sub-partition the warp runs on) decides which rows of D a warp may read.
 // Warps 0,1,4,5,8,9,12,13: epilogue (rows 0-63).  Warps 2, 6, 10, 14 (quarter
-// 2) and 3, 7, 11, 15 (quarter 3): one channel each, end to end -- issue the
-// channel's MMAs (one tile ahead), scan its states, issue the up-projection.
-// Warps 16-18: transposers; warp 19: TMA producer; warp 20: TMA store issuer
-// and TMEM allocation.
+// 2) and 3, 7, 11, 15 (quarter 3): scan of one channel each.  Warps 21-28: MMA
+// issue for one channel each -- a tcgen05.mma occupies its issuing thread for
+// ~100 cycles, so eight issuing threads, apart from the scans, keep the tensor
+// pipe fed.  Warps 16-18: transposers; warp 19: TMA producer; warp 20: TMA
+// store issuer and TMEM allocation.
 //
 // Every wait is bounded: after kWaitLimitCycles the waiting thread sets a shared
 // abort flag and the device status word (RLM_ERR_TIMEOUT); all roles then leave
@@ -72,7 +73,7 @@ constexpr int kBox = 256;              // TMA box rows
 constexpr int kBoxes = kTile / kBox;   // 4 per tile
 constexpr int kXSlots = 20;            // x ring depth (boxes)
 constexpr int kYSlots = 4;             // y ring depth (blocks of 8 chunks)
-constexpr int kWarps = 21;
+constexpr int kWarps = 29;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTmemCols = 512;
 constexpr int kTmemA = 256;            // first TMEM column of the A operands
@@ -116,8 +117,10 @@ constexpr int kBarUDone = kBarTwDone + 16;      // [2]
 constexpr int kBarDEmpty = kBarUDone + 2;       // [2]
 constexpr int kBarYFull = kBarDEmpty + 2;       // [kYSlots]
 constexpr int kBarYEmpty = kBarYFull + kYSlots; // [kYSlots]
-constexpr int kBarFinal = kBarYEmpty + kYSlots; // [8]
-static_assert(kBarFinal + 8 <= kNumBars, "too many barriers");
+constexpr int kBarSFull = kBarYEmpty + kYSlots; // [2][8]: carried states written, per buffer and channel
+constexpr int kBarFinal = kBarSFull + 16;       // [8]
+constexpr int kBarConsts = kBarFinal + 8;       // the A operands and U tables are built
+static_assert(kBarConsts < kNumBars, "too many barriers");
 
 
 // ------------------------------------------------------------ PTX wrappers
@@ -131,16 +134,6 @@ __device__ __forceinline__ bool bar_try(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// Non-blocking probe of a phase (unlike try_wait, never suspends the thread).
-__device__ __forceinline__ bool bar_test(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{ .reg .pred p; mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
         : "=r"(ok)
         : "r"(bar), "r"(parity)
         : "memory");
@@ -333,8 +326,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             bar_init(bar(kBarYFull + i), 8);
             bar_init(bar(kBarYEmpty + i), 1);
         }
-        for (int i = 0; i < 16; ++i) bar_init(bar(kBarTwDone + i), 1);
+        for (int i = 0; i < 16; ++i) {
+            bar_init(bar(kBarTwDone + i), 1);
+            bar_init(bar(kBarSFull + i), 1);
+        }
         for (int i = 0; i < 8; ++i) bar_init(bar(kBarFinal + i), 1);
+        bar_init(bar(kBarConsts), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 20) {
@@ -461,6 +458,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
         tc_fence_after();
+        if (tid == 0) bar_arrive(bar(kBarConsts));
     }
 
     const int quarter = warp & 3;
@@ -567,14 +565,57 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_store_wait_all();
         }
         __syncwarp();
+    } else if (warp >= 21) {
+        // ---------------------------------------------------- MMA issuer, one channel
+        // Issues channel c's Toeplitz/state chain of tile j, then the up-projection
+        // of tile j - 1 (whose carried states the scan warp has written by then),
+        // so the tensor pipe always has the next tile's work queued.
+        const int c = warp - 21;
+        const uint64_t dx0 = umma_desc(sbase + kOffBx + c * kBxStride, 128, 1024);
+        const uint64_t du0 = umma_desc(sbase + kOffAu + c * kAuStride, 128, 512);
+        const uint64_t ds0 = umma_desc(sbase + kOffBs + c * kBsStride, kBsLbo, kBsSbo);
+        const uint32_t aT = tmem + kTmemA + c * 32;
+        if (lane == 0 && wait_bar(bar(kBarConsts), 0, abort_flag)) {
+            tc_fence_after();
+            auto issue_u = [&](int jp) -> bool {
+                const int bp = jp & 1;
+                if (!wait_bar(bar(kBarSFull + bp * 8 + c), (jp >> 1) & 1, abort_flag)) return false;
+                tc_fence_after();
+                const uint64_t so = (uint64_t)((bp * kBsBuf) >> 4);
+                const uint32_t d = tmem + bp * 128 + c * 16;
+#pragma unroll
+                for (int kk = 0; kk < 2; ++kk) umma_ss(d, du0 + kk * 16, ds0 + so + kk * 18, kIdesc, 1);
+                umma_commit(bar(kBarUDone + bp));
+                return true;
+            };
+            bool ok = true;
+            for (int j = 0; j < ntiles && ok; ++j) {
+                const int buf = j & 1, use = j >> 1;
+                if (!wait_bar(bar(kBarBxFull + buf), use & 1, abort_flag)) break;
+                if (!wait_bar(bar(kBarDEmpty + buf), (use & 1) ^ 1, abort_flag)) break;
+                tc_fence_after();
+                const uint64_t xo = (uint64_t)((buf * kBxBuf) >> 4);
+                const uint32_t d = tmem + buf * 128 + c * 16;
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) umma_ts(d, aT + kk * 8, dx0 + xo + kk * 16, kIdesc, kk > 0);
+                umma_commit(bar(kBarTwDone + buf * 8 + c));
+                umma_commit(bar(kBarBxEmpty + buf));
+                if (j > 0) ok = issue_u(j - 1);
+            }
+            if (ok && ntiles > 0) issue_u(ntiles - 1);
+            // Drain: all MMAs this thread issued complete before TMEM is released.
+            umma_commit(bar(kBarFinal + c));
+            const long long t0 = clock64();
+            while (!bar_try(bar(kBarFinal + c), 0))
+                if (clock64() - t0 > kWaitLimitCycles) break;
+        }
+        __syncwarp();
     } else if (quarter >= 2) {
-        // ------------------------------------------ one channel: scan + MMA issue
-        // Warps 2, 6, 10, 14 own channels 0-3 (state rows in TMEM lanes 64-95);
-        // warps 3, 7, 11, 15 own channels 4-7 (lanes 96-127).  A warp issues its
-        // channel's Toeplitz/state MMA chain one tile ahead, scans the 16 chunk
-        // states (lane 2m holds mode m: Re from its own row, Im from lane 2m+1)
-        // and issues the up-projection.  Eight issuing threads keep the tensor
-        // pipe fed: one tcgen05.mma occupies its issuing thread ~90 cycles.
+        // ---------------------------------------------------- scan, one channel
+        // Warps 2, 6, 10, 14 own channels 0-3 (state rows in TMEM lanes 64-95),
+        // warps 3, 7, 11, 15 channels 4-7 (lanes 96-127).  Lane 2m holds mode m:
+        // Re from its own row, Im from lane 2m+1.  The carry S_n = lambda^C S_{n-1}
+        // + L_n runs in fp32; S_{n-1} goes to the up-projection's B operand.
         const int c = (quarter - 2) * 4 + (warp >> 2);
         const uint32_t st_lane = 32u * (uint32_t)quarter;
         const int m = lane >> 1, ri = lane & 1;
@@ -582,40 +623,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float2 LC = lambda_pow(args.decay[pm], args.freq[pm], (float)kC);
         float2 S = make_float2(0.0f, 0.0f);
         const int bsoff = c * kBsStride + (m / 4) * kBsLbo + ((2 * m) % 8) * 2;
-        const uint64_t dx0 = umma_desc(sbase + kOffBx + c * kBxStride, 128, 1024);
-        const uint64_t du0 = umma_desc(sbase + kOffAu + c * kAuStride, 128, 512);
-        const uint64_t ds0 = umma_desc(sbase + kOffBs + c * kBsStride, kBsLbo, kBsSbo);
-        const uint32_t aT = tmem + kTmemA + c * 32;
-
-        // Issue the Toeplitz/state MMA chain of tile jn.  With block == false it
-        // returns false at once if its inputs are not ready yet.
-        auto issue_tw = [&](int jn, bool block) -> bool {
-            const int bn = jn & 1, un = jn >> 1;
-            if (!block) {
-                const bool ready = bar_test(bar(kBarBxFull + bn), un & 1) &&
-                                   bar_test(bar(kBarDEmpty + bn), (un & 1) ^ 1);
-                if (!__all_sync(0xffffffffu, ready)) return false;
-            } else {
-                if (!wait_bar(bar(kBarBxFull + bn), un & 1, abort_flag)) return false;
-                if (!wait_bar(bar(kBarDEmpty + bn), (un & 1) ^ 1, abort_flag)) return false;
-            }
-            if (lane == 0) {
-                tc_fence_after();
-                const uint64_t xo = (uint64_t)((bn * kBxBuf) >> 4);
-                const uint32_t d = tmem + bn * 128 + c * 16;
-#pragma unroll
-                for (int kk = 0; kk < 4; ++kk) umma_ts(d, aT + kk * 8, dx0 + xo + kk * 16, kIdesc, kk > 0);
-                umma_commit(bar(kBarTwDone + bn * 8 + c));
-                umma_commit(bar(kBarBxEmpty + bn));
-            }
-            __syncwarp();
-            return true;
-        };
-
-        bool ok = ntiles > 0 ? issue_tw(0, true) : true;
-        for (int j = 0; j < ntiles && ok; ++j) {
+        for (int j = 0; j < ntiles; ++j) {
             const int buf = j & 1, use = j >> 1;
-            const bool early = j + 1 < ntiles && issue_tw(j + 1, false);
             if (!wait_bar(bar(kBarTwDone + buf * 8 + c), use & 1, abort_flag)) break;
             tc_fence_after();
             uint32_t v[16];
@@ -636,44 +645,35 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_async_smem();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) {
-                tc_fence_after();
-                const uint64_t so = (uint64_t)((buf * kBsBuf) >> 4);
-                const uint32_t d = tmem + buf * 128 + c * 16;
-#pragma unroll
-                for (int kk = 0; kk < 2; ++kk) umma_ss(d, du0 + kk * 16, ds0 + so + kk * 18, kIdesc, 1);
-                umma_commit(bar(kBarUDone + buf));
-            }
-            __syncwarp();
-            if (j + 1 < ntiles && !early && !issue_tw(j + 1, true)) break;
+            if (lane == 0) bar_arrive(bar(kBarSFull + buf * 8 + c));
         }
-        // Drain: all MMAs this warp issued complete before TMEM is released.
-        if (lane == 0) {
-            umma_commit(bar(kBarFinal + c));
-            const long long t0 = clock64();
-            while (!bar_try(bar(kBarFinal + c), 0))
-                if (clock64() - t0 > kWaitLimitCycles) break;
-        }
-        __syncwarp();
     } else {
         // ---------------------------------------------------- epilogue (rows 0..63)
-        const int e = warp >> 2;                     // 0..3: chunk pair within a block
+        // Warp (quarter q, e) converts rows 32 q + lane of chunks 2e, 2e+1 (block 0)
+        // and 8 + 2e, 9 + 2e (block 1) for all 8 channels: one 16-byte row per
+        // token into the y ring, one TMEM wait and one proxy fence per tile.
+        const int e = warp >> 2;
         const int i = 32 * quarter + lane;           // position within the chunk
         for (int j = 0; j < ntiles; ++j) {
             const int buf = j & 1, use = j >> 1;
             if (!wait_bar(bar(kBarUDone + buf), use & 1, abort_flag)) break;
             tc_fence_after();
+            uint32_t v[2][kDG][2];
+#pragma unroll
+            for (int nb = 0; nb < 2; ++nb)
+#pragma unroll
+                for (int c = 0; c < kDG; ++c)
+                    tmem_ld2(tmem + ((uint32_t)(32 * quarter) << 16) + buf * 128 + c * 16 + 8 * nb + 2 * e,
+                             v[nb][c][0], v[nb][c][1]);
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) bar_arrive(bar(kBarDEmpty + buf));   // TMEM buffer drained
             bool ok = true;
+#pragma unroll
             for (int nb = 0; nb < 2; ++nb) {
                 const int ng = j * 2 + nb;
                 const uint32_t slot = ng % kYSlots;
-                const int n0 = 8 * nb + 2 * e;
-                uint32_t v[kDG][2];
-#pragma unroll
-                for (int c = 0; c < kDG; ++c)
-                    tmem_ld2(tmem + ((uint32_t)(32 * quarter) << 16) + buf * 128 + c * 16 + n0,
-                             v[c][0], v[c][1]);
-                tmem_wait_ld();
                 if (!wait_bar(bar(kBarYEmpty + slot), ((ng / kYSlots) & 1) ^ 1, abort_flag)) {
                     ok = false;
                     break;
@@ -682,20 +682,20 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
                     uint4 row;
-                    row.x = pack_bf16x2(__uint_as_float(v[0][h]), __uint_as_float(v[1][h]));
-                    row.y = pack_bf16x2(__uint_as_float(v[2][h]), __uint_as_float(v[3][h]));
-                    row.z = pack_bf16x2(__uint_as_float(v[4][h]), __uint_as_float(v[5][h]));
-                    row.w = pack_bf16x2(__uint_as_float(v[6][h]), __uint_as_float(v[7][h]));
+                    row.x = pack_bf16x2(__uint_as_float(v[nb][0][h]), __uint_as_float(v[nb][1][h]));
+                    row.y = pack_bf16x2(__uint_as_float(v[nb][2][h]), __uint_as_float(v[nb][3][h]));
+                    row.z = pack_bf16x2(__uint_as_float(v[nb][4][h]), __uint_as_float(v[nb][5][h]));
+                    row.w = pack_bf16x2(__uint_as_float(v[nb][6][h]), __uint_as_float(v[nb][7][h]));
                     *reinterpret_cast<uint4 *>(ys + ((2 * e + h) * 64 + i) * 16) = row;
                 }
-                fence_async_smem();
-                __syncwarp();
-                if (lane == 0) bar_arrive(bar(kBarYFull + slot));
             }
             if (!ok) break;
-            tc_fence_before();
+            fence_async_smem();
             __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarDEmpty + buf));
+            if (lane == 0) {
+                bar_arrive(bar(kBarYFull + (j * 2) % kYSlots));
+                bar_arrive(bar(kBarYFull + (j * 2 + 1) % kYSlots));
+            }
         }
     }
 
