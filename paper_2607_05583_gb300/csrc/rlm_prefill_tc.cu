@@ -17,34 +17,42 @@
 //   D[0:64, n]  += U  (64x32)  S_{n-1}  up-projection of the carried state
 //
 // T and W share one A operand (rows 0-63 and 64-95 of a 128-row matrix) held in
-// TMEM, so a single MMA chain yields both.  The columns of D are the NT = 16
-// chunks of a 1024-token tile (MMA N = 16).  The carry between chunks is a
-// sequential fp32 complex scan in registers: one thread per state row, the two
-// rows (Re, Im) of a mode exchange their values with one warp shuffle per chunk.
+// TMEM, so a single MMA chain yields both.  The columns of D are the NT = 32
+// chunks of a 2048-token tile (MMA N = 32).  A tcgen05.mma of this shape costs
+// about the same whatever N is (N <= 64), so the number of MMAs per token, not
+// their arithmetic, bounds the tensor pipe: the tile is as wide as TMEM allows.
+// The carry between chunks is a sequential fp32 complex scan in registers: one
+// thread per (channel, mode); a warp scans two channels, the two rows (Re, Im)
+// of a mode exchanging their values with one warp shuffle per chunk.
 //
 // One CTA owns one batch row b and one group of DG = 8 channels (a 16-byte
 // slice of each token row) and walks the sequence tile by tile, carrying the
 // state in registers, so no CTA waits on another.
 //
-// Data movement per tile (1024 tokens x 8 channels):
-//   TMA (3-D map over [B][L][D], zero fill outside the sequence) -> 20-box ring
+// Data movement per tile (2048 tokens x 8 channels):
+//   TMA (3-D map over [B][L][D], zero fill outside the sequence) -> 15-box ring
 //   -> ldmatrix.trans / stmatrix by three transposer warps into the per-channel
 //      K-major B operand (double-buffered; the positions of a chunk reversed so
 //      that the A operand's Toeplitz rows read K[i + p' - 63])
 //   -> tcgen05.mma -> TMEM -> scan warps -> B operand of the up-projection
 //   -> tcgen05.mma -> TMEM -> epilogue warps (fp32 -> bf16, 8 channels packed
 //      into one 16-byte row) -> smem ring -> TMA store.
-// TMEM (512 columns): two accumulator buffers of 8 channels x 16 columns, and
-// the 8 channels' A operands (128 lanes x 32 columns of packed bf16 pairs).
+// TMEM (512 columns): one accumulator of 32 columns per channel (columns
+// 0-255) and the 8 channels' A operands (128 lanes x 32 columns of packed bf16
+// pairs, columns 256-511).  Each channel's accumulator passes through
+// Toeplitz/state MMA -> scan -> up-projection MMA -> epilogue read and is then
+// free for the next tile; the eight channels run this chain independently, so
+// while one waits on its scan or epilogue the others keep the tensor pipe busy.
 //
 // Warp roles (29 warps): TMEM lane quarter q = warp % 4 (also the SM
 // sub-partition the warp runs on) decides which rows of D a warp may read.
-// Warps 0,1,4,5,8,9,12,13: epilogue (rows 0-63).  Warps 2, 6, 10, 14 (quarter
-// 2) and 3, 7, 11, 15 (quarter 3): scan of one channel each.  Warps 21-28: MMA
-// issue for one channel each -- a tcgen05.mma occupies its issuing thread for
-// ~100 cycles, so eight issuing threads, apart from the scans, keep the tensor
-// pipe fed.  Warps 16-18: transposers; warp 19: TMA producer; warp 20: TMA
-// store issuer and TMEM allocation.
+// Warps 0,1,4,5,8,9,12,13: epilogue (rows 0-63).  Warps 2, 6 (quarter 2,
+// channels 0-3) and 3, 7 (quarter 3, channels 4-7): scan of two channels each.
+// Warps 10, 11, 14, 15 only help build the constants.  Warps 21-28: MMA issue
+// for one channel each -- a tcgen05.mma occupies its issuing thread for ~100
+// cycles, so eight issuing threads, apart from the scans, keep the tensor pipe
+// fed.  Warps 16-18: transposers; warp 19: TMA producer; warp 20: TMA store
+// issuer and TMEM allocation.
 //
 // Every wait is bounded: after kWaitLimitCycles the waiting thread sets a shared
 // abort flag and the device status word (RLM_ERR_TIMEOUT); all roles then leave
@@ -65,14 +73,16 @@ __device__ int g_device_status = 0;
 namespace {
 
 constexpr int kC = 64;                 // chunk length
-constexpr int kNT = 16;                // chunks per tile = MMA N
-constexpr int kTile = kC * kNT;        // 1024 tokens
+constexpr int kNT = 32;                // chunks per tile = MMA N
+constexpr int kTile = kC * kNT;        // 2048 tokens
 constexpr int kDG = 8;                 // channels per CTA
 constexpr int kModes = 16;             // M handled by this kernel
 constexpr int kBox = 256;              // TMA box rows
-constexpr int kBoxes = kTile / kBox;   // 4 per tile
-constexpr int kXSlots = 20;            // x ring depth (boxes)
-constexpr int kYSlots = 4;             // y ring depth (blocks of 8 chunks)
+constexpr int kBoxes = kTile / kBox;   // 8 per tile
+constexpr int kXSlots = 15;            // x ring depth (boxes)
+constexpr int kYRows = 512;            // rows per y ring slot (8 chunks)
+constexpr int kYPerTile = kTile / kYRows;  // 4 slots per tile
+constexpr int kYSlots = 6;             // y ring depth
 constexpr int kWarps = 29;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTmemCols = 512;
@@ -82,26 +92,30 @@ constexpr int kTransposers = 3;
 
 // Shared memory map (bytes from a 1024-aligned base).
 constexpr int kAuStride = 4096;        // 64 real rows x 64 B; rows 64-127 alias the next buffer
-constexpr int kBxStride = 2048 + 16;   // 16 rows x 128 B, +16 so stmatrix rows hit distinct banks
+constexpr int kBxStride = 4096 + 16;   // 32 rows x 128 B, +16 so stmatrix rows hit distinct banks
 constexpr int kBxBuf = kDG * kBxStride;
-constexpr int kBsLbo = 144, kBsSbo = 576, kBsStride = 2 * kBsSbo + 64;
-constexpr int kBsBuf = kDG * kBsStride;
+// Carried-state operand: LBO 144 (not 128) spreads one chunk's 16 mode words
+// over distinct banks; the channel stride is 16 banks (mod 32) so the two
+// channels of a scan warp write disjoint banks as well.
+constexpr int kBsLbo = 144, kBsSbo = 576, kBsStride = 4 * kBsSbo + 64;
+static_assert((kBsStride / 4) % 32 == 16, "paired channels must use disjoint banks");
 constexpr int kOffAu = 0;
 constexpr int kOffBx = kOffAu + kDG * kAuStride;             // 32768
-constexpr int kOffBs = kOffBx + 2 * kBxBuf;                  // 65792
-constexpr int kOffX = kOffBs + 2 * kBsBuf;                   // 85248
+constexpr int kOffBs = kOffBx + 2 * kBxBuf;                  // 98560
+constexpr int kOffX = kOffBs + kDG * kBsStride;              // 117504
 constexpr int kOffY = kOffX + kXSlots * kBox * 16;
-constexpr int kOffBar = kOffY + kYSlots * 512 * 16;
+constexpr int kOffBar = kOffY + kYSlots * kYRows * 16;
 constexpr int kNumBars = 128;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;             // + alignment slack
 static_assert(kOffX % 128 == 0 && kOffY % 128 == 0, "TMA buffers need 128-byte alignment");
+static_assert(kSmemBytes <= 232448, "shared memory budget");
 // Prologue tables, in buffers no other role touches before the prologue ends
 // (the transposers already fill the B operand meanwhile):
 constexpr int kOffWtab = kOffY;                        // [8 ch][32 rows][32 words]: W rows, packed bf16 pairs
 constexpr int kOffTpair = kOffBs;                      // [8 ch][2][64 words]: Toeplitz pairs
 constexpr int kOffKp = kOffTpair + 8 * 2 * 64 * 4;     // [2 halves][8 ch][64] fp32 partial sums of K
-static_assert(8 * 32 * 32 * 4 <= kYSlots * 8192, "W table does not fit the y ring");
+static_assert(8 * 32 * 32 * 4 <= kYSlots * kYRows * 16, "W table does not fit the y ring");
 static_assert(kOffKp + 2 * 8 * 64 * 4 <= kOffX, "prologue tables do not fit");
 // Named barrier for the 16 warps that build the constants.
 constexpr int kPrologueBarrier = 1;
@@ -111,14 +125,14 @@ constexpr int kPrologueThreads = 512;
 constexpr int kBarXFull = 0;                    // [kXSlots]
 constexpr int kBarXEmpty = kXSlots;             // [kXSlots]
 constexpr int kBarBxFull = 2 * kXSlots;         // [2]
-constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]
-constexpr int kBarTwDone = kBarBxEmpty + 2;     // [2][8]: per buffer, per channel
-constexpr int kBarUDone = kBarTwDone + 16;      // [2]
-constexpr int kBarDEmpty = kBarUDone + 2;       // [2]
-constexpr int kBarYFull = kBarDEmpty + 2;       // [kYSlots]
+constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]: released by the 8 MMA threads
+constexpr int kBarTwDone = kBarBxEmpty + 2;     // [8]: Toeplitz/state MMAs of a channel done
+constexpr int kBarSFull = kBarTwDone + 8;       // [8]: carried states of a channel written
+constexpr int kBarUDone = kBarSFull + 8;        // [8]: up-projection of a channel done
+constexpr int kBarDEmpty = kBarUDone + 8;       // [8]: accumulator of a channel read out
+constexpr int kBarYFull = kBarDEmpty + 8;       // [kYSlots]
 constexpr int kBarYEmpty = kBarYFull + kYSlots; // [kYSlots]
-constexpr int kBarSFull = kBarYEmpty + kYSlots; // [2][8]: carried states written, per buffer and channel
-constexpr int kBarFinal = kBarSFull + 16;       // [8]
+constexpr int kBarFinal = kBarYEmpty + kYSlots; // [8]
 constexpr int kBarConsts = kBarFinal + 8;       // the A operands and U tables are built
 static_assert(kBarConsts < kNumBars, "too many barriers");
 
@@ -245,9 +259,10 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
           "=r"(v[14]), "=r"(v[15])
         : "r"(taddr));
 }
-__device__ __forceinline__ void tmem_ld2(uint32_t taddr, uint32_t &a, uint32_t &b) {
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x2.b32 {%0, %1}, [%2];"
-                 : "=r"(a), "=r"(b)
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]),
+                   "=r"(v[6]), "=r"(v[7])
                  : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_wait_ld() {
@@ -319,18 +334,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int i = 0; i < 2; ++i) {
             bar_init(bar(kBarBxFull + i), kBoxes);
             bar_init(bar(kBarBxEmpty + i), kDG);
-            bar_init(bar(kBarUDone + i), kDG);
-            bar_init(bar(kBarDEmpty + i), 8);
         }
-        for (int i = 0; i < kYSlots; ++i) {
-            bar_init(bar(kBarYFull + i), 8);
-            bar_init(bar(kBarYEmpty + i), 1);
-        }
-        for (int i = 0; i < 16; ++i) {
+        for (int i = 0; i < kDG; ++i) {
             bar_init(bar(kBarTwDone + i), 1);
             bar_init(bar(kBarSFull + i), 1);
+            bar_init(bar(kBarUDone + i), 1);
+            bar_init(bar(kBarDEmpty + i), 8);
+            bar_init(bar(kBarFinal + i), 1);
         }
-        for (int i = 0; i < 8; ++i) bar_init(bar(kBarFinal + i), 1);
+        for (int i = 0; i < kYSlots; ++i) {
+            bar_init(bar(kBarYFull + i), 2);
+            bar_init(bar(kBarYEmpty + i), 1);
+        }
         bar_init(bar(kBarConsts), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -502,8 +517,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                              : "r"(src)
                              : "memory");
             }
-            __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarXEmpty + slot));
             if (!wait_bar(bar(kBarBxEmpty + buf), (use & 1) ^ 1, abort_flag)) break;
             const int c = lane & 7, mq = lane >> 3;
             const uint32_t bx = sbase + kOffBx + buf * kBxBuf + c * kBxStride;
@@ -518,45 +531,47 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             fence_async_smem();
             __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarBxFull + buf));
+            // The x slot is released only now that stmatrix has consumed the
+            // ldmatrix registers: releasing it right after issuing ldmatrix let
+            // the next TMA load overwrite the box before it had been read.
+            if (lane == 0) {
+                bar_arrive(bar(kBarXEmpty + slot));
+                bar_arrive(bar(kBarBxFull + buf));
+            }
         }
     } else if (warp == 20) {
         // ---------------------------------------------------- y store issuer
-        // One bulk group per block of 512 rows; up to kYSlots - 2 groups may still
-        // be reading shared memory while the next block is issued.
+        // One bulk group per slot of 512 rows; up to kYSlots - 2 groups may still
+        // be reading shared memory while the next slot is issued.
+        const int nslots = ntiles * kYPerTile;
         int ng = 0;
-        bool ok = true;
-        for (int j = 0; j < ntiles && ok; ++j) {
-            for (int nb = 0; nb < 2; ++nb, ++ng) {
-                const uint32_t slot = ng % kYSlots;
-                if (!wait_bar(bar(kBarYFull + slot), (ng / kYSlots) & 1, abort_flag)) {
-                    ok = false;
-                    break;
-                }
-                const uint32_t ys = sbase + kOffY + slot * 8192;
-                for (int h = 0; h < 2; ++h) {
-                    const int64_t start = args.t0 + (int64_t)j * kTile + nb * 512 + h * kBox;
-                    if (start >= 0) {
-                        if (lane == 0) tma_store_3d(&tmap_y, ys + h * 4096, d0, (int)start, b);
-                    } else if (start + kBox > 0) {
-                        // Partially before t = 0: plain 16-byte stores of the rows t >= 0.
-                        const uint8_t *src = smem + kOffY + slot * 8192 + h * 4096;
-                        for (int rr = (int)(-start) + lane; rr < kBox; rr += 32) {
-                            const int64_t t = start + rr;
-                            *reinterpret_cast<uint4 *>(args.y + ((int64_t)b * args.L + t) * D + d0) =
-                                *reinterpret_cast<const uint4 *>(src + rr * 16);
-                        }
+        for (; ng < nslots; ++ng) {
+            const uint32_t slot = ng % kYSlots;
+            if (!wait_bar(bar(kBarYFull + slot), (ng / kYSlots) & 1, abort_flag)) break;
+            const uint32_t ys = sbase + kOffY + slot * (kYRows * 16);
+            const int jt = ng / kYPerTile, e = ng % kYPerTile;
+            for (int h = 0; h < kYRows / kBox; ++h) {
+                const int64_t start = args.t0 + (int64_t)jt * kTile + e * kYRows + h * kBox;
+                if (start >= 0) {
+                    if (lane == 0) tma_store_3d(&tmap_y, ys + h * (kBox * 16), d0, (int)start, b);
+                } else if (start + kBox > 0) {
+                    // Partially before t = 0: plain 16-byte stores of the rows t >= 0.
+                    const uint8_t *src = smem + kOffY + slot * (kYRows * 16) + h * (kBox * 16);
+                    for (int rr = (int)(-start) + lane; rr < kBox; rr += 32) {
+                        const int64_t t = start + rr;
+                        *reinterpret_cast<uint4 *>(args.y + ((int64_t)b * args.L + t) * D + d0) =
+                            *reinterpret_cast<const uint4 *>(src + rr * 16);
                     }
                 }
-                if (lane == 0) {
-                    tma_store_commit();
-                    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(kYSlots - 2) : "memory");
-                }
-                __syncwarp();
-                // Groups up to ng - (kYSlots - 2) have finished reading their slots.
-                const int freed = ng - (kYSlots - 2);
-                if (lane == 0 && freed >= 0) bar_arrive(bar(kBarYEmpty + freed % kYSlots));
             }
+            if (lane == 0) {
+                tma_store_commit();
+                asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(kYSlots - 2) : "memory");
+            }
+            __syncwarp();
+            // Groups up to ng - (kYSlots - 2) have finished reading their slots.
+            const int freed = ng - (kYSlots - 2);
+            if (lane == 0 && freed >= 0) bar_arrive(bar(kBarYEmpty + freed % kYSlots));
         }
         if (lane == 0) {
             tma_store_wait_read();
@@ -567,42 +582,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp >= 21) {
         // ---------------------------------------------------- MMA issuer, one channel
-        // Issues channel c's Toeplitz/state chain of tile j, then the up-projection
-        // of tile j - 1 (whose carried states the scan warp has written by then),
-        // so the tensor pipe always has the next tile's work queued.
+        // Per tile: the Toeplitz/state chain into the channel's accumulator, then,
+        // once the scan has written the carried states, the up-projection.  The
+        // next tile's chain waits until the epilogue has read the accumulator.
         const int c = warp - 21;
         const uint64_t dx0 = umma_desc(sbase + kOffBx + c * kBxStride, 128, 1024);
         const uint64_t du0 = umma_desc(sbase + kOffAu + c * kAuStride, 128, 512);
         const uint64_t ds0 = umma_desc(sbase + kOffBs + c * kBsStride, kBsLbo, kBsSbo);
         const uint32_t aT = tmem + kTmemA + c * 32;
+        const uint32_t d = tmem + c * kNT;
         if (lane == 0 && wait_bar(bar(kBarConsts), 0, abort_flag)) {
             tc_fence_after();
-            auto issue_u = [&](int jp) -> bool {
-                const int bp = jp & 1;
-                if (!wait_bar(bar(kBarSFull + bp * 8 + c), (jp >> 1) & 1, abort_flag)) return false;
-                tc_fence_after();
-                const uint64_t so = (uint64_t)((bp * kBsBuf) >> 4);
-                const uint32_t d = tmem + bp * 128 + c * 16;
-#pragma unroll
-                for (int kk = 0; kk < 2; ++kk) umma_ss(d, du0 + kk * 16, ds0 + so + kk * 18, kIdesc, 1);
-                umma_commit(bar(kBarUDone + bp));
-                return true;
-            };
-            bool ok = true;
-            for (int j = 0; j < ntiles && ok; ++j) {
+            for (int j = 0; j < ntiles; ++j) {
                 const int buf = j & 1, use = j >> 1;
                 if (!wait_bar(bar(kBarBxFull + buf), use & 1, abort_flag)) break;
-                if (!wait_bar(bar(kBarDEmpty + buf), (use & 1) ^ 1, abort_flag)) break;
+                if (!wait_bar(bar(kBarDEmpty + c), (j & 1) ^ 1, abort_flag)) break;
                 tc_fence_after();
                 const uint64_t xo = (uint64_t)((buf * kBxBuf) >> 4);
-                const uint32_t d = tmem + buf * 128 + c * 16;
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) umma_ts(d, aT + kk * 8, dx0 + xo + kk * 16, kIdesc, kk > 0);
-                umma_commit(bar(kBarTwDone + buf * 8 + c));
-                umma_commit(bar(kBarBxEmpty + buf));
-                if (j > 0) ok = issue_u(j - 1);
+                umma_commit(bar(kBarTwDone + c));
+                if (!wait_bar(bar(kBarSFull + c), j & 1, abort_flag)) break;
+                tc_fence_after();
+                // The scan has seen this chain's commit, so its MMAs (and their
+                // reads of the B operand) are complete: release the buffer.  A
+                // second commit issued right behind the first was observed to
+                // arrive while the chain was still reading shared memory.
+                bar_arrive(bar(kBarBxEmpty + buf));
+#pragma unroll
+                for (int kk = 0; kk < 2; ++kk) umma_ss(d, du0 + kk * 16, ds0 + kk * ((2 * kBsLbo) >> 4), kIdesc, 1);
+                umma_commit(bar(kBarUDone + c));
             }
-            if (ok && ntiles > 0) issue_u(ntiles - 1);
             // Drain: all MMAs this thread issued complete before TMEM is released.
             umma_commit(bar(kBarFinal + c));
             const long long t0 = clock64();
@@ -610,92 +620,97 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (clock64() - t0 > kWaitLimitCycles) break;
         }
         __syncwarp();
-    } else if (quarter >= 2) {
-        // ---------------------------------------------------- scan, one channel
-        // Warps 2, 6, 10, 14 own channels 0-3 (state rows in TMEM lanes 64-95),
-        // warps 3, 7, 11, 15 channels 4-7 (lanes 96-127).  Lane 2m holds mode m:
-        // Re from its own row, Im from lane 2m+1.  The carry S_n = lambda^C S_{n-1}
-        // + L_n runs in fp32; S_{n-1} goes to the up-projection's B operand.
-        const int c = (quarter - 2) * 4 + (warp >> 2);
+    } else if (quarter >= 2 && warp < 8) {
+        // ---------------------------------------------------- scan, two channels
+        // Warps 2 and 6 own channels (0,1) and (2,3) (state rows in TMEM lanes
+        // 64-95), warps 3 and 7 channels (4,5) and (6,7) (lanes 96-127).  Lane
+        // 2m carries mode m of the first channel, lane 2m+1 mode m of the second:
+        // each lane reads row 2m+ri of both channels and one shuffle hands the
+        // partner the value it lacks.  S_n = lambda^C S_{n-1} + L_n runs in fp32;
+        // S_{n-1} goes to the up-projection's B operand.
+        const int cA = (quarter - 2) * 4 + 2 * (warp >> 2), cB = cA + 1;
         const uint32_t st_lane = 32u * (uint32_t)quarter;
         const int m = lane >> 1, ri = lane & 1;
-        const int pm = (d0 + c) * kModes + m;
+        const int ch = ri ? cB : cA;
+        const int pm = (d0 + ch) * kModes + m;
         const float2 LC = lambda_pow(args.decay[pm], args.freq[pm], (float)kC);
         float2 S = make_float2(0.0f, 0.0f);
-        const int bsoff = c * kBsStride + (m / 4) * kBsLbo + ((2 * m) % 8) * 2;
+        uint8_t *bs = smem + kOffBs + ch * kBsStride + (m / 4) * kBsLbo + (m % 4) * 4;
         for (int j = 0; j < ntiles; ++j) {
-            const int buf = j & 1, use = j >> 1;
-            if (!wait_bar(bar(kBarTwDone + buf * 8 + c), use & 1, abort_flag)) break;
+            if (!wait_bar(bar(kBarTwDone + cA), j & 1, abort_flag)) break;
+            if (!wait_bar(bar(kBarTwDone + cB), j & 1, abort_flag)) break;
             tc_fence_after();
-            uint32_t v[16];
-            tmem_ld16(tmem + (st_lane << 16) + buf * 128 + c * 16, v);
-            tmem_wait_ld();
-            uint8_t *bs = smem + kOffBs + buf * kBsBuf + bsoff;
 #pragma unroll
-            for (int n = 0; n < kNT; ++n) {
-                const float mine = __uint_as_float(v[n]);
-                const float other = __shfl_xor_sync(0xffffffffu, mine, 1);
-                if (ri == 0) {
-                    *reinterpret_cast<uint32_t *>(bs + (n >> 3) * kBsSbo + (n & 7) * 16) = pack_bf16x2(S.x, S.y);
-                    S = cfma(LC, S, make_float2(mine, other));
+            for (int h = 0; h < kNT / 16; ++h) {
+                uint32_t va[16], vb[16];
+                tmem_ld16(tmem + (st_lane << 16) + cA * kNT + 16 * h, va);
+                tmem_ld16(tmem + (st_lane << 16) + cB * kNT + 16 * h, vb);
+                tmem_wait_ld();
+#pragma unroll
+                for (int n = 0; n < 16; ++n) {
+                    const float a = __uint_as_float(va[n]), bb = __uint_as_float(vb[n]);
+                    const float recv = __shfl_xor_sync(0xffffffffu, ri ? a : bb, 1);
+                    const float2 Ln = ri ? make_float2(recv, bb) : make_float2(a, recv);
+                    const int nn = 16 * h + n;
+                    *reinterpret_cast<uint32_t *>(bs + (nn >> 3) * kBsSbo + (nn & 7) * 16) = pack_bf16x2(S.x, S.y);
+                    S = cfma(LC, S, Ln);
                 }
             }
-            if (j == ntiles - 1 && args.state_out && ri == 0)
-                args.state_out[((int64_t)b * D + d0 + c) * kModes + m] = S;
+            if (j == ntiles - 1 && args.state_out)
+                args.state_out[((int64_t)b * D + d0 + ch) * kModes + m] = S;
             fence_async_smem();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarSFull + buf * 8 + c));
+            if (lane == 0) {
+                bar_arrive(bar(kBarSFull + cA));
+                bar_arrive(bar(kBarSFull + cB));
+            }
         }
-    } else {
+    } else if (quarter < 2 && warp < 16) {
         // ---------------------------------------------------- epilogue (rows 0..63)
-        // Warp (quarter q, e) converts rows 32 q + lane of chunks 2e, 2e+1 (block 0)
-        // and 8 + 2e, 9 + 2e (block 1) for all 8 channels: one 16-byte row per
-        // token into the y ring, one TMEM wait and one proxy fence per tile.
+        // Warp (quarter q, e) converts rows 32 q + lane of chunks 8e .. 8e+7 for
+        // all 8 channels, a channel pair at a time as their up-projections
+        // complete (releasing each accumulator as soon as it is read), and then
+        // writes one 16-byte row per token into the y ring.
         const int e = warp >> 2;
         const int i = 32 * quarter + lane;           // position within the chunk
+        const uint32_t trow = tmem + ((uint32_t)(32 * quarter) << 16) + 8 * e;
         for (int j = 0; j < ntiles; ++j) {
-            const int buf = j & 1, use = j >> 1;
-            if (!wait_bar(bar(kBarUDone + buf), use & 1, abort_flag)) break;
-            tc_fence_after();
-            uint32_t v[2][kDG][2];
-#pragma unroll
-            for (int nb = 0; nb < 2; ++nb)
-#pragma unroll
-                for (int c = 0; c < kDG; ++c)
-                    tmem_ld2(tmem + ((uint32_t)(32 * quarter) << 16) + buf * 128 + c * 16 + 8 * nb + 2 * e,
-                             v[nb][c][0], v[nb][c][1]);
-            tmem_wait_ld();
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarDEmpty + buf));   // TMEM buffer drained
+            uint32_t pk[kDG / 2][8];
             bool ok = true;
 #pragma unroll
-            for (int nb = 0; nb < 2; ++nb) {
-                const int ng = j * 2 + nb;
-                const uint32_t slot = ng % kYSlots;
-                if (!wait_bar(bar(kBarYEmpty + slot), ((ng / kYSlots) & 1) ^ 1, abort_flag)) {
+            for (int p = 0; p < kDG / 2; ++p) {
+                const int cA = 2 * p, cB = 2 * p + 1;
+                if (!wait_bar(bar(kBarUDone + cA), j & 1, abort_flag) ||
+                    !wait_bar(bar(kBarUDone + cB), j & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
-                uint8_t *ys = smem + kOffY + slot * 8192;
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    uint4 row;
-                    row.x = pack_bf16x2(__uint_as_float(v[nb][0][h]), __uint_as_float(v[nb][1][h]));
-                    row.y = pack_bf16x2(__uint_as_float(v[nb][2][h]), __uint_as_float(v[nb][3][h]));
-                    row.z = pack_bf16x2(__uint_as_float(v[nb][4][h]), __uint_as_float(v[nb][5][h]));
-                    row.w = pack_bf16x2(__uint_as_float(v[nb][6][h]), __uint_as_float(v[nb][7][h]));
-                    *reinterpret_cast<uint4 *>(ys + ((2 * e + h) * 64 + i) * 16) = row;
+                tc_fence_after();
+                uint32_t va[8], vb[8];
+                tmem_ld8(trow + cA * kNT, va);
+                tmem_ld8(trow + cB * kNT, vb);
+                tmem_wait_ld();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    bar_arrive(bar(kBarDEmpty + cA));
+                    bar_arrive(bar(kBarDEmpty + cB));
                 }
+#pragma unroll
+                for (int n = 0; n < 8; ++n) pk[p][n] = pack_bf16x2(__uint_as_float(va[n]), __uint_as_float(vb[n]));
             }
             if (!ok) break;
+            const int ng = j * kYPerTile + e;
+            const uint32_t slot = ng % kYSlots;
+            if (!wait_bar(bar(kBarYEmpty + slot), ((ng / kYSlots) & 1) ^ 1, abort_flag)) break;
+            uint8_t *ys = smem + kOffY + slot * (kYRows * 16);
+#pragma unroll
+            for (int n = 0; n < 8; ++n)
+                *reinterpret_cast<uint4 *>(ys + (n * kC + i) * 16) = make_uint4(pk[0][n], pk[1][n], pk[2][n], pk[3][n]);
             fence_async_smem();
             __syncwarp();
-            if (lane == 0) {
-                bar_arrive(bar(kBarYFull + (j * 2) % kYSlots));
-                bar_arrive(bar(kBarYFull + (j * 2 + 1) % kYSlots));
-            }
+            if (lane == 0) bar_arrive(bar(kBarYFull + slot));
         }
     }
 
