@@ -112,10 +112,16 @@ static_assert(kOffX % 128 == 0 && kOffY % 128 == 0, "TMA buffers need 128-byte a
 static_assert(kSmemBytes <= 232448, "shared memory budget");
 // Prologue tables, in buffers no other role touches before the prologue ends
 // (the transposers already fill the B operand meanwhile):
-constexpr int kOffWtab = kOffY;                        // [8 ch][32 rows][32 words]: W rows, packed bf16 pairs
-constexpr int kOffTpair = kOffBs;                      // [8 ch][2][64 words]: Toeplitz pairs
-constexpr int kOffKp = kOffTpair + 8 * 2 * 64 * 4;     // [2 halves][8 ch][64] fp32 partial sums of K
-static_assert(8 * 32 * 32 * 4 <= kYSlots * kYRows * 16, "W table does not fit the y ring");
+// The tables are laid out for conflict-free reads when lane R of a warp fetches
+// word k of row R: the W table is word-major with rows innermost (stride 33
+// words), and the second Toeplitz pair table starts 80 words (16 banks) after the
+// first.
+constexpr int kWtabStride = 33;
+constexpr int kTpairStride = 144;                      // words per channel: P0 at 0, P1 at 80
+constexpr int kOffWtab = kOffY;                        // [8 ch][32 words][33]: W rows, packed bf16 pairs
+constexpr int kOffTpair = kOffBs;                      // [8 ch][144 words]: Toeplitz pairs
+constexpr int kOffKp = kOffTpair + 8 * kTpairStride * 4;  // [2 halves][8 ch][64] fp32 partial sums of K
+static_assert(8 * 32 * kWtabStride * 4 <= kYSlots * kYRows * 16, "W table does not fit the y ring");
 static_assert(kOffKp + 2 * 8 * 64 * 4 <= kOffX, "prologue tables do not fit");
 // Named barrier for the 16 warps that build the constants.
 constexpr int kPrologueBarrier = 1;
@@ -405,11 +411,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             *reinterpret_cast<uint32_t *>(au + (n / 8) * 512 + (n % 8) * 16) = pack_bf16x2(q.x, -q.y);
             pw = nx;
         }
-        uint4 *wt = reinterpret_cast<uint4 *>(smem + kOffWtab) + (c * 32 + 2 * m) * 8 + 2 * qn;
-        wt[0] = make_uint4(wre[0], wre[1], wre[2], wre[3]);
-        wt[1] = make_uint4(wre[4], wre[5], wre[6], wre[7]);
-        wt[8] = make_uint4(wim[0], wim[1], wim[2], wim[3]);
-        wt[9] = make_uint4(wim[4], wim[5], wim[6], wim[7]);
+        uint32_t *wt = reinterpret_cast<uint32_t *>(smem + kOffWtab) + (c * 32 + 8 * qn) * kWtabStride + 2 * m;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            wt[k * kWtabStride] = wre[k];
+            wt[k * kWtabStride + 1] = wim[k];
+        }
 #pragma unroll
         for (int e = 0; e < 16; ++e) {
             float v = kv[e];
@@ -435,9 +442,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int n = idx - 63;
             return (n >= 0 && n < 64) ? kp[c * 64 + n] + kp[(8 + c) * 64 + n] : 0.0f;
         };
-        uint32_t *tp = reinterpret_cast<uint32_t *>(smem + kOffTpair) + c * 128;
+        uint32_t *tp = reinterpret_cast<uint32_t *>(smem + kOffTpair) + c * kTpairStride;
         tp[i] = pack_bf16x2(kz(2 * i), kz(2 * i + 1));
-        tp[64 + i] = pack_bf16x2(kz(2 * i + 1), kz(2 * i + 2));
+        tp[80 + i] = pack_bf16x2(kz(2 * i + 1), kz(2 * i + 2));
     }
     if (warp < 16) asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
     // Stage 3: the A operands into TMEM, row R = 32 q + lane of channels e and e + 4:
@@ -451,17 +458,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int c = e + 4 * cc;
             uint32_t w[32];
             if (q < 2) {
-                const uint32_t *tp = reinterpret_cast<const uint32_t *>(smem + kOffTpair) + c * 128 +
-                                     ((R & 1) ? 64 + (R >> 1) : (R >> 1));
+                const uint32_t *tp = reinterpret_cast<const uint32_t *>(smem + kOffTpair) + c * kTpairStride +
+                                     ((R & 1) ? 80 + (R >> 1) : (R >> 1));
 #pragma unroll
                 for (int k = 0; k < 32; ++k) w[k] = tp[k];
             } else if ((q == 2) == (c < 4)) {
-                const uint4 *wt = reinterpret_cast<const uint4 *>(smem + kOffWtab) + (c * 32 + lane) * 8;
+                const uint32_t *wt = reinterpret_cast<const uint32_t *>(smem + kOffWtab) + c * 32 * kWtabStride + lane;
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    const uint4 v = wt[k];
-                    w[4 * k] = v.x; w[4 * k + 1] = v.y; w[4 * k + 2] = v.z; w[4 * k + 3] = v.w;
-                }
+                for (int k = 0; k < 32; ++k) w[k] = wt[k * kWtabStride];
             } else {
 #pragma unroll
                 for (int k = 0; k < 32; ++k) w[k] = 0u;
