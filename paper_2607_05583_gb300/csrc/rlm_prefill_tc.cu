@@ -16,11 +16,12 @@
 //   D[64:96, n]  = W  (32x64)  X_n      local end state, (Re, Im) of 16 modes
 //   D[0:64, n]  += U  (64x32)  S_{n-1}  up-projection of the carried state
 //
-// T and W share one A operand (rows 0-63 and 64-95 of a 128-row matrix) held in
-// TMEM, so a single MMA chain yields both.  The columns of D are the NT = 32
-// chunks of a 2048-token tile (MMA N = 32).  A tcgen05.mma of this shape costs
-// about the same whatever N is (N <= 64), so the number of MMAs per token, not
-// their arithmetic, bounds the tensor pipe: the tile is as wide as TMEM allows.
+// T and W share one A operand (64 Toeplitz rows and 32 state rows of a
+// 128-row matrix) held in TMEM, so a single MMA chain yields both.  The columns
+// of D are the NT = 32 chunks of a 2048-token tile (MMA N = 32).  A tcgen05.mma
+// of this shape costs about the same whatever N is (N <= 64), so the number of
+// MMAs per token, not their arithmetic, bounds the tensor pipe: the tile is as
+// wide as TMEM allows.
 // The carry between chunks is a sequential fp32 complex scan in registers: one
 // thread per (channel, mode); a warp scans two channels, the two rows (Re, Im)
 // of a mode exchanging their values with one warp shuffle per chunk.
@@ -44,15 +45,23 @@
 // free for the next tile; the eight channels run this chain independently, so
 // while one waits on its scan or epilogue the others keep the tensor pipe busy.
 //
-// Warp roles (29 warps): TMEM lane quarter q = warp % 4 (also the SM
-// sub-partition the warp runs on) decides which rows of D a warp may read.
-// Warps 0,1,4,5,8,9,12,13: epilogue (rows 0-63).  Warps 2, 6 (quarter 2,
-// channels 0-3) and 3, 7 (quarter 3, channels 4-7): scan of two channels each.
-// Warps 10, 11, 14, 15 only help build the constants.  Warps 21-28: MMA issue
-// for one channel each -- a tcgen05.mma occupies its issuing thread for ~100
-// cycles, so eight issuing threads, apart from the scans, keep the tensor pipe
-// fed.  Warps 16-18: transposers; warp 19: TMA producer; warp 20: TMA store
-// issuer and TMEM allocation.
+// TMEM lane quarter q (lanes 32q..32q+31) is readable only by warps with
+// warp % 4 == q, which also run on SM sub-partition q.  The rows of each
+// channel's A operand (and so of its accumulator) are placed so that every
+// quarter carries the same load: quarter c/2 holds channel c's 32 state rows;
+// the Toeplitz rows (positions 0-31, 32-63) sit in quarters 2, 3 for channels
+// 0-3 and in quarters 0, 1 for channels 4-7; the fourth quarter is zero.
+//
+// Warp roles (26 warps):
+//   0-7    epilogue: warp (q = warp % 4, h = warp / 4) converts positions
+//          32 (q % 2) + lane of chunks 16h .. 16h+15 for the four channels whose
+//          Toeplitz rows live in quarter q, into 8-byte halves of the y rows.
+//   8-11   scan: the warp of quarter q carries channels 2q and 2q+1.
+//   12-15  transposers (boxes k = t mod 4); 16 TMA producer; 17 TMA store
+//          issuer and TMEM allocation.
+//   18-25  MMA issue for one channel each -- a tcgen05.mma occupies its issuing
+//          thread for ~100 cycles, so eight issuing threads keep the pipe fed.
+// Warps 0-11 and 18-21 first build the per-channel constants.
 //
 // Every wait is bounded: after kWaitLimitCycles the waiting thread sets a shared
 // abort flag and the device status word (RLM_ERR_TIMEOUT); all roles then leave
@@ -83,15 +92,20 @@ constexpr int kXSlots = 15;            // x ring depth (boxes)
 constexpr int kYRows = 512;            // rows per y ring slot (8 chunks)
 constexpr int kYPerTile = kTile / kYRows;  // 4 slots per tile
 constexpr int kYSlots = 6;             // y ring depth
-constexpr int kWarps = 29;
+constexpr int kWarps = 26;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTmemCols = 512;
 constexpr int kTmemA = 256;            // first TMEM column of the A operands
 constexpr long long kWaitLimitCycles = 4000000000ll;  // about 2 s at 2 GHz
-constexpr int kTransposers = 3;
+constexpr int kTransposers = 4;
 
 // Shared memory map (bytes from a 1024-aligned base).
-constexpr int kAuStride = 4096;        // 64 real rows x 64 B; rows 64-127 alias the next buffer
+// U tables: 64 rows x 64 B per channel, in the order of channels 4-7, 0-3.  The
+// up-projection reads a 128-row A operand whose 64 real rows must meet the
+// channel's Toeplitz lanes: rows 0-63 for channels 4-7 (start at the table),
+// rows 64-127 for channels 0-3 (start one table earlier).  The other 64 rows read
+// a neighbouring table and land in state/zero lanes nobody reads afterwards.
+constexpr int kAuStride = 4096;
 constexpr int kBxStride = 4096 + 16;   // 32 rows x 128 B, +16 so stmatrix rows hit distinct banks
 constexpr int kBxBuf = kDG * kBxStride;
 // Carried-state operand: LBO 144 (not 128) spreads one chunk's 16 mode words
@@ -123,7 +137,7 @@ constexpr int kOffTpair = kOffBs;                      // [8 ch][144 words]: Toe
 constexpr int kOffKp = kOffTpair + 8 * kTpairStride * 4;  // [2 halves][8 ch][64] fp32 partial sums of K
 static_assert(8 * 32 * kWtabStride * 4 <= kYSlots * kYRows * 16, "W table does not fit the y ring");
 static_assert(kOffKp + 2 * 8 * 64 * 4 <= kOffX, "prologue tables do not fit");
-// Named barrier for the 16 warps that build the constants.
+// Named barrier for the 16 warps that build the constants (0-11 and 18-21).
 constexpr int kPrologueBarrier = 1;
 constexpr int kPrologueThreads = 512;
 
@@ -301,6 +315,10 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kNT >> 3) << 17) |
                             ((uint32_t)(128 >> 4) << 24);
 
+__device__ __forceinline__ int au_slot(int c) { return (c + 4) & 7; }
+// First byte (from the U table area) of channel c's 128-row up-projection operand.
+__device__ __forceinline__ int au_operand(int c) { return au_slot(c) * kAuStride - (c < 4 ? kAuStride : 0); }
+
 struct TcArgs {
     const float *decay, *freq, *amp, *phase;
     float2 *state_out;   // nullable, [B][D][M]
@@ -345,17 +363,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             bar_init(bar(kBarTwDone + i), 1);
             bar_init(bar(kBarSFull + i), 1);
             bar_init(bar(kBarUDone + i), 1);
-            bar_init(bar(kBarDEmpty + i), 8);
+            bar_init(bar(kBarDEmpty + i), 4);
             bar_init(bar(kBarFinal + i), 1);
         }
         for (int i = 0; i < kYSlots; ++i) {
-            bar_init(bar(kBarYFull + i), 2);
+            bar_init(bar(kBarYFull + i), 4);
             bar_init(bar(kBarYEmpty + i), 1);
         }
         bar_init(bar(kBarConsts), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 20) {
+    if (warp == 17) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(tmem_slot)),
                      "r"(kTmemCols));
@@ -369,7 +387,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // The producer fills the whole ring before the constants are built.
     const int total_boxes = ntiles * kBoxes;
     int issued = 0;
-    if (warp == 19 && lane == 0) {
+    if (warp == 16 && lane == 0) {
         for (; issued < total_boxes && issued < kXSlots; ++issued) {
             const int jt = issued / kBoxes, q = issued % kBoxes;
             const uint32_t slot = issued % kXSlots;
@@ -380,14 +398,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 
     // ---------------------------------------------------- per-channel constants
-    // Built by warps 0-15 only (synchronised by a named barrier), while the
-    // transposers, the producer and the store issuer start their work.
+    // Built by warps 0-11 and 18-21 (synchronised by a named barrier), while the
+    // transposers, the producer and the store issuer start their work.  Warp
+    // (quarter q, rank e within its quarter) has prologue thread index ptid.
+    const bool builder = warp < 12 || (warp >= 18 && warp < 22);
+    const int pq = warp & 3, pe = warp < 12 ? warp >> 2 : 3;
+    const int ptid = (pe * 4 + pq) * 32 + lane;
     // Stage 1: thread (c, m, qn) runs the powers lambda^n, n in [16 qn, 16 qn + 16),
     // of mode m of channel c: the U rows (Re, -Im of c lambda^(n+1)), the W-row
     // words (lambda^n packed in pairs of n), and Re(c lambda^n) summed over the
     // eight modes of its warp (a fixed shuffle tree) into Kp[half][c][n].
-    if (tid < 512) {
-        const int c = tid >> 6, m = (tid >> 2) & 15, qn = tid & 3;
+    if (builder) {
+        const int c = ptid >> 6, m = (ptid >> 2) & 15, qn = ptid & 3;
         const int pm = (d0 + c) * kModes + m;
         const float ga = args.decay[pm], om = args.freq[pm];
         const float2 lam = lambda_pow(ga, om, 1.0f);
@@ -395,7 +417,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (args.coef_out && b == 0 && qn == 0)
             args.coef_out[pm] = make_float4(lam.x, lam.y, cf.x, cf.y);
         float2 pw = lambda_pow(ga, om, (float)(16 * qn));
-        uint8_t *au = smem + kOffAu + c * kAuStride + (m / 4) * 128 + ((2 * m) % 8) * 2;
+        uint8_t *au = smem + kOffAu + au_slot(c) * kAuStride + (m / 4) * 128 + ((2 * m) % 8) * 2;
         uint32_t wre[8], wim[8];
         float kv[16];
 #pragma unroll
@@ -431,13 +453,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int e = 0; e < 16; ++e) kp[e] = kv[e];
         }
     }
-    if (warp < 16) asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
+    if (builder) asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
     // Stage 2: K[c][n] = Kp[0][c][n] + Kp[1][c][n] (Eq. 1 at integer lags), as
     // zero-padded pair tables kz(i) = K[i - 63] (0 for i < 63):
     // P0[c][i] = (kz(2i), kz(2i+1)), P1[c][i] = (kz(2i+1), kz(2i+2)).
-    if (tid < 512) {
+    if (builder) {
         const float *kp = reinterpret_cast<const float *>(smem + kOffKp);
-        const int c = tid >> 6, i = tid & 63;
+        const int c = ptid >> 6, i = ptid & 63;
         auto kz = [&](int idx) -> float {
             const int n = idx - 63;
             return (n >= 0 && n < 64) ? kp[c * 64 + n] + kp[(8 + c) * 64 + n] : 0.0f;
@@ -446,23 +468,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         tp[i] = pack_bf16x2(kz(2 * i), kz(2 * i + 1));
         tp[80 + i] = pack_bf16x2(kz(2 * i + 1), kz(2 * i + 2));
     }
-    if (warp < 16) asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
-    // Stage 3: the A operands into TMEM, row R = 32 q + lane of channels e and e + 4:
-    // rows 0-63   T[R][p'] = K[R + p' - 63]        (Toeplitz, reversed positions)
-    // W[k][p'] = (Re, Im) lambda_m^p' (k = 2m + ri) in rows 64-95 for channels 0-3
-    // and in rows 96-127 for channels 4-7; the other 32 rows are zero.
-    if (warp < 16) {
-        const int q = warp & 3, e = warp >> 2;
-        const int R = 32 * q + lane;
+    if (builder) asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
+    // Stage 3: the A operands into TMEM, lanes 32 q + lane of channels e and e + 4:
+    //   Toeplitz quarters: T[p][p'] = K[p + p' - 63] (reversed positions) for
+    //     position p = 32 (q % 2) + lane;
+    //   quarter c / 2:     W[k][p'] = (Re, Im) lambda_m^p' for state row k = lane
+    //     (k = 2m + ri);
+    //   the remaining quarter: zero.
+    if (builder) {
+        const int q = pq, e = pe;
         for (int cc = 0; cc < 2; ++cc) {
             const int c = e + 4 * cc;
             uint32_t w[32];
-            if (q < 2) {
+            if ((q >> 1) == (c < 4 ? 1 : 0)) {
+                const int pos = 32 * (q & 1) + lane;
                 const uint32_t *tp = reinterpret_cast<const uint32_t *>(smem + kOffTpair) + c * kTpairStride +
-                                     ((R & 1) ? 80 + (R >> 1) : (R >> 1));
+                                     ((pos & 1) ? 80 + (pos >> 1) : (pos >> 1));
 #pragma unroll
                 for (int k = 0; k < 32; ++k) w[k] = tp[k];
-            } else if ((q == 2) == (c < 4)) {
+            } else if (q == (c >> 1)) {
                 const uint32_t *wt = reinterpret_cast<const uint32_t *>(smem + kOffWtab) + c * 32 * kWtabStride + lane;
 #pragma unroll
                 for (int k = 0; k < 32; ++k) w[k] = wt[k * kWtabStride];
@@ -477,11 +501,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
         tc_fence_after();
-        if (tid == 0) bar_arrive(bar(kBarConsts));
+        if (ptid == 0) bar_arrive(bar(kBarConsts));
     }
 
     const int quarter = warp & 3;
-    if (warp == 19) {
+    if (warp == 16) {
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
             for (; issued < total_boxes; ++issued) {
@@ -504,9 +528,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         __syncwarp();
-    } else if (warp >= 16 && warp < 16 + kTransposers) {
-        // ---------------------------------------------------- transposers (boxes k = t mod 3)
-        for (int k = warp - 16; k < total_boxes; k += kTransposers) {
+    } else if (warp >= 12 && warp < 12 + kTransposers) {
+        // ---------------------------------------------------- transposers (boxes k = t mod 4)
+        for (int k = warp - 12; k < total_boxes; k += kTransposers) {
             const int j = k / kBoxes, tq = k % kBoxes;
             const int buf = j & 1, use = j >> 1;
             const uint32_t slot = k % kXSlots;
@@ -543,7 +567,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 bar_arrive(bar(kBarBxFull + buf));
             }
         }
-    } else if (warp == 20) {
+    } else if (warp == 17) {
         // ---------------------------------------------------- y store issuer
         // One bulk group per slot of 512 rows; up to kYSlots - 2 groups may still
         // be reading shared memory while the next slot is issued.
@@ -584,14 +608,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_store_wait_all();
         }
         __syncwarp();
-    } else if (warp >= 21) {
+    } else if (warp >= 18) {
         // ---------------------------------------------------- MMA issuer, one channel
         // Per tile: the Toeplitz/state chain into the channel's accumulator, then,
         // once the scan has written the carried states, the up-projection.  The
         // next tile's chain waits until the epilogue has read the accumulator.
-        const int c = warp - 21;
+        const int c = warp - 18;
         const uint64_t dx0 = umma_desc(sbase + kOffBx + c * kBxStride, 128, 1024);
-        const uint64_t du0 = umma_desc(sbase + kOffAu + c * kAuStride, 128, 512);
+        const uint64_t du0 = umma_desc(sbase + kOffAu + au_operand(c), 128, 512);
         const uint64_t ds0 = umma_desc(sbase + kOffBs + c * kBsStride, kBsLbo, kBsSbo);
         const uint32_t aT = tmem + kTmemA + c * 32;
         const uint32_t d = tmem + c * kNT;
@@ -624,15 +648,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (clock64() - t0 > kWaitLimitCycles) break;
         }
         __syncwarp();
-    } else if (quarter >= 2 && warp < 8) {
+    } else if (warp >= 8 && warp < 12) {
         // ---------------------------------------------------- scan, two channels
-        // Warps 2 and 6 own channels (0,1) and (2,3) (state rows in TMEM lanes
-        // 64-95), warps 3 and 7 channels (4,5) and (6,7) (lanes 96-127).  Lane
-        // 2m carries mode m of the first channel, lane 2m+1 mode m of the second:
-        // each lane reads row 2m+ri of both channels and one shuffle hands the
-        // partner the value it lacks.  S_n = lambda^C S_{n-1} + L_n runs in fp32;
-        // S_{n-1} goes to the up-projection's B operand.
-        const int cA = (quarter - 2) * 4 + 2 * (warp >> 2), cB = cA + 1;
+        // The warp of quarter q owns channels 2q and 2q+1, whose state rows are
+        // its TMEM lanes.  Lane 2m carries mode m of the first channel, lane 2m+1
+        // mode m of the second: each lane reads row 2m+ri of both channels and one
+        // shuffle hands the partner the value it lacks.  S_n = lambda^C S_{n-1} +
+        // L_n runs in fp32; S_{n-1} goes to the up-projection's B operand.
+        const int cA = 2 * quarter, cB = cA + 1;
         const uint32_t st_lane = 32u * (uint32_t)quarter;
         const int m = lane >> 1, ri = lane & 1;
         const int ch = ri ? cB : cA;
@@ -670,58 +693,73 @@ __global__ void __launch_bounds__(kThreads, 1)
                 bar_arrive(bar(kBarSFull + cB));
             }
         }
-    } else if (quarter < 2 && warp < 16) {
-        // ---------------------------------------------------- epilogue (rows 0..63)
-        // Warp (quarter q, e) converts rows 32 q + lane of chunks 8e .. 8e+7 for
-        // all 8 channels, a channel pair at a time as their up-projections
-        // complete (releasing each accumulator as soon as it is read), and then
-        // writes one 16-byte row per token into the y ring.
-        const int e = warp >> 2;
-        const int i = 32 * quarter + lane;           // position within the chunk
-        const uint32_t trow = tmem + ((uint32_t)(32 * quarter) << 16) + 8 * e;
+    } else if (warp < 8) {
+        // ---------------------------------------------------- epilogue
+        // Warp (quarter q, h) reads its quarter's Toeplitz lanes -- position
+        // pos = 32 (q % 2) + lane of channels c0 .. c0+3 (c0 = 4 in quarters 0, 1
+        // and 0 in quarters 2, 3) -- for chunks 16h .. 16h+15, a channel pair at a
+        // time as its up-projections complete (releasing each accumulator as soon
+        // as it is read), and writes the 8-byte half (channels c0 .. c0+3) of each
+        // token's 16-byte row into the y ring: ring slots 2h and 2h+1 of the tile.
+        const int h = warp >> 2;
+        const int c0 = quarter < 2 ? 4 : 0;
+        const int pos = 32 * (quarter & 1) + lane;
+        const int hb = quarter < 2 ? 8 : 0;
+        const uint32_t trow = tmem + ((uint32_t)(32 * quarter) << 16) + 16 * h;
         for (int j = 0; j < ntiles; ++j) {
-            uint32_t pk[kDG / 2][8];
+            uint32_t pk[2][16];
             bool ok = true;
 #pragma unroll
-            for (int p = 0; p < kDG / 2; ++p) {
-                const int cA = 2 * p, cB = 2 * p + 1;
+            for (int p = 0; p < 2; ++p) {
+                const int cA = c0 + 2 * p, cB = cA + 1;
                 if (!wait_bar(bar(kBarUDone + cA), j & 1, abort_flag) ||
                     !wait_bar(bar(kBarUDone + cB), j & 1, abort_flag)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
-                uint32_t va[8], vb[8];
-                tmem_ld8(trow + cA * kNT, va);
-                tmem_ld8(trow + cB * kNT, vb);
-                tmem_wait_ld();
+#pragma unroll
+                for (int sh = 0; sh < 2; ++sh) {
+                    uint32_t va[8], vb[8];
+                    tmem_ld8(trow + cA * kNT + 8 * sh, va);
+                    tmem_ld8(trow + cB * kNT + 8 * sh, vb);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int n = 0; n < 8; ++n)
+                        pk[p][8 * sh + n] = pack_bf16x2(__uint_as_float(va[n]), __uint_as_float(vb[n]));
+                }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
                     bar_arrive(bar(kBarDEmpty + cA));
                     bar_arrive(bar(kBarDEmpty + cB));
                 }
-#pragma unroll
-                for (int n = 0; n < 8; ++n) pk[p][n] = pack_bf16x2(__uint_as_float(va[n]), __uint_as_float(vb[n]));
             }
             if (!ok) break;
-            const int ng = j * kYPerTile + e;
-            const uint32_t slot = ng % kYSlots;
-            if (!wait_bar(bar(kBarYEmpty + slot), ((ng / kYSlots) & 1) ^ 1, abort_flag)) break;
-            uint8_t *ys = smem + kOffY + slot * (kYRows * 16);
 #pragma unroll
-            for (int n = 0; n < 8; ++n)
-                *reinterpret_cast<uint4 *>(ys + (n * kC + i) * 16) = make_uint4(pk[0][n], pk[1][n], pk[2][n], pk[3][n]);
-            fence_async_smem();
-            __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarYFull + slot));
+            for (int sh = 0; sh < 2; ++sh) {
+                const int ng = j * kYPerTile + 2 * h + sh;
+                const uint32_t slot = ng % kYSlots;
+                if (!wait_bar(bar(kBarYEmpty + slot), ((ng / kYSlots) & 1) ^ 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                uint8_t *ys = smem + kOffY + slot * (kYRows * 16) + hb;
+#pragma unroll
+                for (int n = 0; n < 8; ++n)
+                    *reinterpret_cast<uint2 *>(ys + (n * kC + pos) * 16) = make_uint2(pk[0][8 * sh + n], pk[1][8 * sh + n]);
+                fence_async_smem();
+                __syncwarp();
+                if (lane == 0) bar_arrive(bar(kBarYFull + slot));
+            }
+            if (!ok) break;
         }
     }
 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 20)
+    if (warp == 17)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(kTmemCols));
 }
