@@ -205,6 +205,33 @@ RLM_API int rlm_version(void);
  * host-side count, incremented at each launch; for accounting in benchmarks). */
 RLM_API unsigned long long rlm_kernels_launched(void);
 
+/* rlm_measure_row_io -- a measurement helper with no counterpart in the paper:
+ * it bounds what the prefill's memory access pattern can reach on this GPU.
+ *
+ * The tensor-core prefill gives each CTA one group of 8 bf16 channels, so each
+ * token row it loads from x or stores to y is a 16-byte slice of a [B][L][D] row.
+ * This call launches `ctas` CTAs that stream that pattern and nothing else: CTA k
+ * owns the slice of slice_bytes (16, 32, 64 or 128) bytes at channel
+ * (k % (D / (slice_bytes / 2))) * (slice_bytes / 2) of a [rows][D] bf16 field and
+ * a contiguous range of its rows; it loads 4 KB boxes from `src` with TMA and
+ * stores as many 4 KB boxes to `dst` with TMA.  Together the CTAs load the field
+ * once and store it once (rlm_measure_row_io_bytes gives the exact byte count),
+ * so timing the call on `stream` gives the load+store bandwidth of that slice
+ * width at that CTA count.
+ *
+ * src, dst: device, [rows][D] bf16, 16-byte aligned; dst is overwritten with
+ *   arbitrary bytes (pass scratch memory).
+ * rows: a multiple of 4096 / slice_bytes, below 2^31.  D: a multiple of
+ *   slice_bytes / 2.  ctas: a positive multiple of D / (slice_bytes / 2).
+ * Errors: invalid arguments return RLM_ERR_INVALID_ARG before any launch; a
+ *   launch failure returns RLM_ERR_CUDA.  Waits inside the kernel are bounded
+ *   (about 2 s); a wait that expires shows as a measured time of seconds. */
+RLM_API rlm_status rlm_measure_row_io(const void *src, void *dst, int64_t rows, int D, int slice_bytes,
+                                      int ctas, void *stream);
+/* Bytes rlm_measure_row_io moves (loaded plus stored) for these arguments; 0 if
+ * they are invalid. */
+RLM_API int64_t rlm_measure_row_io_bytes(int64_t rows, int D, int slice_bytes, int ctas);
+
 #ifdef __cplusplus
 }
 #endif

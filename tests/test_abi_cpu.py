@@ -158,6 +158,29 @@ def test_backward_rejects_bad_arguments_on_host(lib):
     assert call(dy, _t(FAKE + (1 << 30), B, L, D, rlm.RLM_F32), dx, g) == rlm.RLM_ERR_INVALID_ARG
 
 
+@pytest.mark.parametrize("rows,D,sb,ctas", [
+    (4096, 256, 24, 128),      # slice width not 16/32/64/128
+    (4096, 250, 16, 125),      # D not a multiple of the slice
+    (4096, 256, 16, 100),      # ctas not a multiple of the slice count
+    (4000, 256, 16, 128),      # rows not a multiple of the box height
+    (256, 256, 16, 64),        # fewer boxes than CTAs need
+])
+def test_row_io_measurement_rejects_bad_arguments_on_host(lib, rows, D, sb, ctas):
+    st = lib.rlm_measure_row_io(FAKE, FAKE + (1 << 30), rows, D, sb, ctas, None)
+    assert st == rlm.RLM_ERR_INVALID_ARG
+    assert lib.rlm_last_error()
+    assert lib.rlm_measure_row_io(None, FAKE, 4096, 256, 16, 128, None) == rlm.RLM_ERR_INVALID_ARG
+    assert lib.rlm_measure_row_io(FAKE + 8, FAKE, 4096, 256, 16, 128, None) == rlm.RLM_ERR_INVALID_ARG
+
+
+def test_row_io_measurement_byte_count(lib):
+    # [131072][256] bf16 in 16-byte slices by 128 CTAs: 4 KB boxes of 256 rows,
+    # 16384 boxes in all, 128 per CTA; loaded once and stored once.
+    assert lib.rlm_measure_row_io_bytes(131072, 256, 16, 128) == 2 * 131072 * 256 * 2
+    assert lib.rlm_measure_row_io_bytes(131072, 256, 32, 128) == 2 * 131072 * 256 * 2
+    assert lib.rlm_measure_row_io_bytes(131072, 250, 16, 128) == 0
+
+
 def test_workspace_queries_are_host_only_and_monotone(lib):
     a = lib.rlm_prefill_workspace_size(1, 1000, 64, 4, rlm.RLM_F32)
     b = lib.rlm_prefill_workspace_size(4, 100000, 64, 4, rlm.RLM_F32)
