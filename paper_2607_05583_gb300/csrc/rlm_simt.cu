@@ -45,6 +45,27 @@ struct ChunkGeom {
     int64_t t0;   // processing time of chunk 0's first token (<= 0)
 };
 
+ChunkGeom geom_c(int64_t L, int C) {
+    ChunkGeom g;
+    g.C = C;
+    g.nch = (int)((L + g.C - 1) / g.C);
+    g.t0 = L - (int64_t)g.nch * g.C;
+    return g;
+}
+
+// The backward pass does ~26 M flop per token-channel in its two per-token
+// phases, so it needs far fewer (b, chunk, channel) tuples than the forward to
+// fill the GPU; longer chunks keep its workspace (16 bytes per (b, chunk, d, m))
+// small enough to stay in L2 and shorten the sequential carry and the reduction.
+int bwd_chunk_len(int64_t B, int64_t L, int D) {
+    const int64_t target = (int64_t)sm_count() * 512;
+    const int64_t per_chunk = std::max<int64_t>(1, B * (int64_t)D);
+    int64_t nch = std::max<int64_t>(1, (target + per_chunk - 1) / per_chunk);
+    int64_t C = (L + nch - 1) / nch;
+    C = std::max<int64_t>(16, std::min<int64_t>(4096, C));
+    return (int)C;
+}
+
 ChunkGeom geom(int64_t B, int64_t L, int D) {
     ChunkGeom g;
     g.C = simt_chunk_len(B, L, D);
@@ -278,7 +299,7 @@ cudaError_t backward_t(const T *dy, const T *x, T *dx, int64_t B, int64_t L, int
                        const float *decay, const float *freq, const float *amp,
                        const float *phase, float *gd, float *gf, float *ga, float *gp, void *ws,
                        cudaStream_t st) {
-    const ChunkGeom g = geom(B, L, D);
+    const ChunkGeom g = geom_c(L, bwd_chunk_len(B, L, D));
     const int64_t n = B * (int64_t)g.nch * D * M;
     float2 *ws_s = reinterpret_cast<float2 *>(ws);
     float2 *ws_r = ws_s + n;
@@ -319,7 +340,8 @@ size_t simt_prefill_ws_bytes(int64_t B, int64_t L, int D, int M) {
 }
 
 size_t simt_backward_ws_bytes(int64_t B, int64_t L, int D, int M) {
-    return 2 * simt_prefill_ws_bytes(B, L, D, M);
+    const ChunkGeom g = geom_c(L, bwd_chunk_len(B, L, D));
+    return 2 * (size_t)B * g.nch * D * M * sizeof(float2);
 }
 
 cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_t L, int D,
