@@ -68,6 +68,7 @@
 // their loops, drain what they issued and the CTA frees its TMEM and returns.
 #include <cuda.h>
 
+#include <algorithm>
 #include <mutex>
 #include <vector>
 
@@ -204,6 +205,29 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
     }
 }
 
+// Bounded wait until *flag >= want (another CTA's release), with acquire
+// semantics for the loads that follow.  Returns false if this CTA aborted.
+__device__ __forceinline__ bool wait_flag(const int *flag, int want, volatile int *abort_flag) {
+    long long t0 = 0;
+    for (uint32_t it = 0;; ++it) {
+        int v;
+        asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(flag) : "memory");
+        if (v >= want) return true;
+        if ((it & 255u) == 0) {
+            if (*abort_flag) return false;
+            const long long now = clock64();
+            if (t0 == 0) {
+                t0 = now;
+            } else if (now - t0 > kWaitLimitCycles) {
+                *abort_flag = 1;
+                atomicExch(&g_device_status, (int)RLM_ERR_TIMEOUT);
+                return false;
+            }
+        }
+        __nanosleep(64);
+    }
+}
+
 __device__ __forceinline__ void fence_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -328,8 +352,16 @@ struct TcArgs {
     int D;
     int ntiles;
     int64_t t0;          // first token of tile 0 (<= 0): tiles end exactly at L-1
+    // Sequence segments (grid z): segment s owns tiles [s * seg_tiles, ...).
+    int nseg, seg_tiles;
+    float2 *seg_state;   // [B][nseg][D][M]: each segment's end state from a zero start
+    int *seg_flag;       // [B][nseg][D / 8]: scan warps that have published (4 = done)
 };
 
+// kSeg: the grid's z dimension splits the sequence into segments.  The
+// unsegmented instance keeps the tile count a kernel parameter (no register
+// holds it), which the per-tile loops' register allocation depends on.
+template <bool kSeg>
 __global__ void __launch_bounds__(kThreads, 1)
     k_prefill_tc(const __grid_constant__ CUtensorMap tmap_x,
                  const __grid_constant__ CUtensorMap tmap_y, const TcArgs args) {
@@ -340,10 +372,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const uint32_t sbase = smem_u32(smem);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int g = blockIdx.x, b = blockIdx.y;
+    const int g = blockIdx.x, b = blockIdx.y, seg = kSeg ? (int)blockIdx.z : 0;
     const int d0 = g * kDG;
     const int D = args.D;
-    const int ntiles = args.ntiles;
+    // Virtual tiles: nA state-only passes over the segment's tiles (every segment
+    // but the last publishes its end state for the later ones), then nB output
+    // passes over the same tiles.
+    const int ja = kSeg ? seg * args.seg_tiles : 0;
+    const int nB = kSeg ? min(args.ntiles, ja + args.seg_tiles) - ja : args.ntiles;
+    const int nA = kSeg && seg < args.nseg - 1 ? nB : 0;
+    const int nV = kSeg ? nA + nB : args.ntiles;
+    auto real_tile = [&](int v) { return ja + (v < nA ? v : v - nA); };
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
     auto bar = [&](int i) { return smem_u32(bars + i); };
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kOffMisc);
@@ -385,11 +424,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = *tmem_slot;
 
     // The producer fills the whole ring before the constants are built.
-    const int total_boxes = ntiles * kBoxes;
+    const int total_boxes = nV * kBoxes;
     int issued = 0;
     if (warp == 16 && lane == 0) {
         for (; issued < total_boxes && issued < kXSlots; ++issued) {
-            const int jt = issued / kBoxes, q = issued % kBoxes;
+            const int jt = real_tile(issued / kBoxes), q = issued % kBoxes;
             const uint32_t slot = issued % kXSlots;
             bar_expect_tx(bar(kBarXFull + slot), kBox * 16);
             tma_load_3d(sbase + kOffX + slot * (kBox * 16), &tmap_x, d0,
@@ -414,7 +453,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float ga = args.decay[pm], om = args.freq[pm];
         const float2 lam = lambda_pow(ga, om, 1.0f);
         const float2 cf = mode_coef(args.amp[pm], args.phase[pm]);
-        if (args.coef_out && b == 0 && qn == 0)
+        if (args.coef_out && b == 0 && seg == 0 && qn == 0)
             args.coef_out[pm] = make_float4(lam.x, lam.y, cf.x, cf.y);
         float2 pw = lambda_pow(ga, om, (float)(16 * qn));
         uint8_t *au = smem + kOffAu + au_slot(c) * kAuStride + (m / 4) * 128 + ((2 * m) % 8) * 2;
@@ -509,7 +548,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
             for (; issued < total_boxes; ++issued) {
-                const int jt = issued / kBoxes, q = issued % kBoxes;
+                const int jt = real_tile(issued / kBoxes), q = issued % kBoxes;
                 const uint32_t slot = issued % kXSlots;
                 const uint32_t fill = issued / kXSlots;
                 if (!wait_bar(bar(kBarXEmpty + slot), (fill & 1) ^ 1, abort_flag)) break;
@@ -571,13 +610,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------- y store issuer
         // One bulk group per slot of 512 rows; up to kYSlots - 2 groups may still
         // be reading shared memory while the next slot is issued.
-        const int nslots = ntiles * kYPerTile;
+        const int nslots = nB * kYPerTile;
         int ng = 0;
         for (; ng < nslots; ++ng) {
             const uint32_t slot = ng % kYSlots;
             if (!wait_bar(bar(kBarYFull + slot), (ng / kYSlots) & 1, abort_flag)) break;
             const uint32_t ys = sbase + kOffY + slot * (kYRows * 16);
-            const int jt = ng / kYPerTile, e = ng % kYPerTile;
+            const int jt = ja + ng / kYPerTile, e = ng % kYPerTile;
             for (int h = 0; h < kYRows / kBox; ++h) {
                 const int64_t start = args.t0 + (int64_t)jt * kTile + e * kYRows + h * kBox;
                 if (start >= 0) {
@@ -612,7 +651,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------- MMA issuer, one channel
         // Per tile: the Toeplitz/state chain into the channel's accumulator, then,
         // once the scan has written the carried states, the up-projection.  The
-        // next tile's chain waits until the epilogue has read the accumulator.
+        // next tile's chain waits until the epilogue has read the accumulator
+        // (after a state-only pass, until the scan has read it).
         const int c = warp - 18;
         const uint64_t dx0 = umma_desc(sbase + kOffBx + c * kBxStride, 128, 1024);
         const uint64_t du0 = umma_desc(sbase + kOffAu + au_operand(c), 128, 512);
@@ -621,22 +661,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t d = tmem + c * kNT;
         if (lane == 0 && wait_bar(bar(kBarConsts), 0, abort_flag)) {
             tc_fence_after();
-            for (int j = 0; j < ntiles; ++j) {
-                const int buf = j & 1, use = j >> 1;
+            for (int v = 0; v < nV; ++v) {
+                const int buf = v & 1, use = v >> 1;
                 if (!wait_bar(bar(kBarBxFull + buf), use & 1, abort_flag)) break;
-                if (!wait_bar(bar(kBarDEmpty + c), (j & 1) ^ 1, abort_flag)) break;
+                if (v > nA && !wait_bar(bar(kBarDEmpty + c), (v - 1 - nA) & 1, abort_flag)) break;
                 tc_fence_after();
                 const uint64_t xo = (uint64_t)((buf * kBxBuf) >> 4);
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) umma_ts(d, aT + kk * 8, dx0 + xo + kk * 16, kIdesc, kk > 0);
                 umma_commit(bar(kBarTwDone + c));
-                if (!wait_bar(bar(kBarSFull + c), j & 1, abort_flag)) break;
+                if (!wait_bar(bar(kBarSFull + c), v & 1, abort_flag)) break;
                 tc_fence_after();
                 // The scan has seen this chain's commit, so its MMAs (and their
                 // reads of the B operand) are complete: release the buffer.  A
                 // second commit issued right behind the first was observed to
                 // arrive while the chain was still reading shared memory.
                 bar_arrive(bar(kBarBxEmpty + buf));
+                if (v < nA) continue;  // state-only pass: no output
 #pragma unroll
                 for (int kk = 0; kk < 2; ++kk) umma_ss(d, du0 + kk * 16, ds0 + kk * ((2 * kBsLbo) >> 4), kIdesc, 1);
                 umma_commit(bar(kBarUDone + c));
@@ -663,9 +704,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float2 LC = lambda_pow(args.decay[pm], args.freq[pm], (float)kC);
         float2 S = make_float2(0.0f, 0.0f);
         uint8_t *bs = smem + kOffBs + ch * kBsStride + (m / 4) * kBsLbo + (m % 4) * 4;
-        for (int j = 0; j < ntiles; ++j) {
-            if (!wait_bar(bar(kBarTwDone + cA), j & 1, abort_flag)) break;
-            if (!wait_bar(bar(kBarTwDone + cB), j & 1, abort_flag)) break;
+        const int64_t seg_row = (int64_t)b * args.nseg;
+        // One tile of the carry: S_n = lambda^C S_{n-1} + L_n over its 32 chunks.
+        auto scan_tile = [&](int v) -> bool {
+            if (!wait_bar(bar(kBarTwDone + cA), v & 1, abort_flag)) return false;
+            if (!wait_bar(bar(kBarTwDone + cB), v & 1, abort_flag)) return false;
             tc_fence_after();
 #pragma unroll
             for (int h = 0; h < kNT / 16; ++h) {
@@ -683,7 +726,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     S = cfma(LC, S, Ln);
                 }
             }
-            if (j == ntiles - 1 && args.state_out)
+            if (v == nV - 1 && (!kSeg || seg == args.nseg - 1) && args.state_out)
                 args.state_out[((int64_t)b * D + d0 + ch) * kModes + m] = S;
             fence_async_smem();
             tc_fence_before();
@@ -692,7 +735,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                 bar_arrive(bar(kBarSFull + cA));
                 bar_arrive(bar(kBarSFull + cB));
             }
+            return true;
+        };
+        bool ok = true;
+        // State-only passes, then (segments with later ones) publish the end state
+        // from a zero start: every lane stores, fences and counts.
+        for (int v = 0; v < nA && ok; ++v) ok = scan_tile(v);
+        if (ok && nA > 0) {
+            args.seg_state[((seg_row + seg) * D + d0 + ch) * kModes + m] = S;
+            __threadfence();
+            atomicAdd(args.seg_flag + (seg_row + seg) * (D / kDG) + g, 1);
         }
+        // Carry in for the output passes: the earlier segments' end states, each
+        // advanced to the end of segment seg - 1 (full segments of seg_tiles tiles).
+        if (kSeg && ok) {
+            S = make_float2(0.0f, 0.0f);
+            for (int r = 0; r < seg; ++r) {
+                if (!wait_flag(args.seg_flag + (seg_row + r) * (D / kDG) + g, 128, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                const float2 lr = __ldcg(args.seg_state + ((seg_row + r) * D + d0 + ch) * kModes + m);
+                const float2 P = lambda_pow(args.decay[pm], args.freq[pm],
+                                            (float)((int64_t)(seg - 1 - r) * args.seg_tiles * kTile));
+                S = cfma(P, lr, S);
+            }
+        }
+        for (int v = nA; v < nV && ok; ++v) ok = scan_tile(v);
     } else if (warp < 8) {
         // ---------------------------------------------------- epilogue
         // Warp (quarter q, h) reads its quarter's Toeplitz lanes -- position
@@ -706,7 +775,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int pos = 32 * (quarter & 1) + lane;
         const int hb = quarter < 2 ? 8 : 0;
         const uint32_t trow = tmem + ((uint32_t)(32 * quarter) << 16) + 16 * h;
-        for (int j = 0; j < ntiles; ++j) {
+        for (int j = 0; j < nB; ++j) {
             uint32_t pk[2][16];
             bool ok = true;
 #pragma unroll
@@ -797,6 +866,29 @@ bool make_field_map(CUtensorMap *map, const void *ptr, int64_t B, int64_t L, int
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Sequence segments: with fewer (batch row, channel group) CTAs than SMs, the
+// sequence is cut into nseg runs of whole tiles so that nseg * B * D / 8 CTAs
+// (at most one per SM, all resident at once) share the work.
+struct Segments {
+    int nseg, seg_tiles;
+};
+
+Segments segments(int64_t B, int64_t L, int D) {
+    const int ntiles = (int)((L + kTile - 1) / kTile);
+    const int64_t ctas = B * (int64_t)(D / kDG);
+    // Segment offsets enter lambda^n with n below 2^24 (exact in fp32).
+    int want = L > ((int64_t)1 << 24) ? 1
+             : (int)std::min<int64_t>(ntiles, std::max<int64_t>(1, sm_count() / std::max<int64_t>(1, ctas)));
+    Segments sg;
+    sg.seg_tiles = (ntiles + want - 1) / want;
+    sg.nseg = (ntiles + sg.seg_tiles - 1) / sg.seg_tiles;
+    return sg;
+}
+
+size_t seg_state_bytes(int64_t B, int nseg, int D) {
+    return ((size_t)B * nseg * D * kModes * sizeof(float2) + 255) / 256 * 256;
+}
+
 }  // namespace
 
 bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
@@ -804,11 +896,15 @@ bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
            L <= ((int64_t)1 << 31) - kTile && D / kDG <= 65535;
 }
 
-size_t tc_prefill_ws_bytes(int64_t, int64_t, int, int) { return 0; }
+size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int) {
+    const Segments sg = segments(B, L, D);
+    if (sg.nseg < 2) return 0;
+    return seg_state_bytes(B, sg.nseg, D) + (size_t)B * sg.nseg * (D / kDG) * sizeof(int);
+}
 
 cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int M,
                        const float *decay, const float *freq, const float *amp,
-                       const float *phase, float *state_out, float *coef_out, void *,
+                       const float *phase, float *state_out, float *coef_out, void *ws,
                        cudaStream_t st) {
     (void)M;
     CUtensorMap mx, my;
@@ -822,8 +918,11 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
         std::lock_guard<std::mutex> lock(mu);
         if ((int)configured.size() <= dev) configured.resize(dev + 1, 0);
         if (!configured[dev]) {
-            cudaError_t e = cudaFuncSetAttribute(k_prefill_tc, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 kSmemBytes);
+            cudaError_t e = cudaFuncSetAttribute(k_prefill_tc<false>,
+                                                 cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(k_prefill_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSmemBytes);
             if (e != cudaSuccess) return e;
             configured[dev] = 1;
         }
@@ -840,10 +939,29 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.D = D;
     a.ntiles = (int)((L + kTile - 1) / kTile);
     a.t0 = L - (int64_t)a.ntiles * kTile;
-    dim3 grid((unsigned)(D / kDG), (unsigned)B);
-    k_prefill_tc<<<grid, kThreads, kSmemBytes, st>>>(mx, my, a);
+    const Segments sg = segments(B, L, D);
+    a.nseg = sg.nseg;
+    a.seg_tiles = sg.seg_tiles;
+    a.seg_state = nullptr;
+    a.seg_flag = nullptr;
+    dim3 grid((unsigned)(D / kDG), (unsigned)B, (unsigned)sg.nseg);
+    if (sg.nseg < 2) {
+        k_prefill_tc<false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, a);
+        count_launches(1);
+        return cudaGetLastError();
+    }
+    // Segments wait on the end states of earlier segments of the same rows: a
+    // cooperative launch guarantees all CTAs are resident together.
+    if (!ws) return cudaErrorInvalidValue;
+    a.seg_state = static_cast<float2 *>(ws);
+    a.seg_flag = reinterpret_cast<int *>(static_cast<char *>(ws) + seg_state_bytes(B, sg.nseg, D));
+    cudaError_t e = cudaMemsetAsync(a.seg_flag, 0, (size_t)B * sg.nseg * (D / kDG) * sizeof(int), st);
+    if (e != cudaSuccess) return e;
+    void *kargs[] = {&mx, &my, &a};
+    e = cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_prefill_tc<true>), grid, dim3(kThreads), kargs,
+                                    (size_t)kSmemBytes, st);
     count_launches(1);
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t read_and_clear_device_status(int *status, cudaStream_t st) {

@@ -75,6 +75,9 @@ def test_prefill_layer6m_bf16():
     (1, 1, 8, 1, "f32"), (1, 1, 8, 16, "bf16"), (2, 7, 16, 3, "f32"), (3, 65, 24, 16, "bf16"),
     (1, 1000, 8, 64, "f32"), (2, 2049, 64, 16, "bf16"), (1, 4097, 32, 5, "bf16"),
     (2, 3000, 40, 33, "f32"), (1, 6143, 256, 16, "bf16"), (3, 2048 * 3 + 17, 64, 16, "bf16"),
+    # few rows: the sequence is split into segments (one per tile; two tiles each
+    # with a shorter last segment)
+    (1, 2048 * 5 + 100, 8, 16, "bf16"), (1, 2048 * 24 + 5, 64, 16, "bf16"),
 ])
 def test_prefill_edge_and_ragged_shapes(B, L, D, M, dtype):
     inp = make_inputs(B, L, D, M, dtype, seed=B * 1000 + L)
