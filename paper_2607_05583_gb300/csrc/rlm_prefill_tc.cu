@@ -69,6 +69,7 @@
 #include <cuda.h>
 
 #include <algorithm>
+#include <atomic>
 #include <mutex>
 #include <vector>
 
@@ -205,14 +206,15 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
     }
 }
 
-// Bounded wait until *flag >= want (another CTA's release), with acquire
+// Bounded wait until *flag == want (another CTA's release), with acquire
 // semantics for the loads that follow.  Returns false if this CTA aborted.
-__device__ __forceinline__ bool wait_flag(const int *flag, int want, volatile int *abort_flag) {
+__device__ __forceinline__ bool wait_flag(const unsigned long long *flag, unsigned long long want,
+                                          volatile int *abort_flag) {
     long long t0 = 0;
     for (uint32_t it = 0;; ++it) {
-        int v;
-        asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(flag) : "memory");
-        if (v >= want) return true;
+        unsigned long long v;
+        asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(flag) : "memory");
+        if (v == want) return true;
         if ((it & 255u) == 0) {
             if (*abort_flag) return false;
             const long long now = clock64();
@@ -355,7 +357,8 @@ struct TcArgs {
     // Sequence segments (grid z): segment s owns tiles [s * seg_tiles, ...).
     int nseg, seg_tiles;
     float2 *seg_state;   // [B][nseg][D][M]: each segment's end state from a zero start
-    int *seg_flag;       // [B][nseg][D / 8]: scan warps that have published (4 = done)
+    unsigned long long *seg_flag;  // [B][nseg][D][M]: == epoch once that state is published
+    unsigned long long epoch;      // distinct for every segmented launch of this process
 };
 
 // kSeg: the grid's z dimension splits the sequence into segments.  The
@@ -383,6 +386,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int nA = kSeg && seg < args.nseg - 1 ? nB : 0;
     const int nV = kSeg ? nA + nB : args.ntiles;
     auto real_tile = [&](int v) { return ja + (v < nA ? v : v - nA); };
+    // Constant builders (warps 0-11 and 18-21) issue their parameter loads first,
+    // so the DRAM latency overlaps the barrier set-up and TMEM allocation.
+    const bool builder = warp < 12 || (warp >= 18 && warp < 22);
+    const int pq = warp & 3, pe = warp < 12 ? warp >> 2 : 3;
+    const int ptid = (pe * 4 + pq) * 32 + lane;
+    float p_decay = 0.0f, p_freq = 0.0f, p_amp = 0.0f, p_phase = 0.0f;
+    if (builder) {
+        const int pm = (d0 + (ptid >> 6)) * kModes + ((ptid >> 2) & 15);
+        p_decay = args.decay[pm];
+        p_freq = args.freq[pm];
+        p_amp = args.amp[pm];
+        p_phase = args.phase[pm];
+    }
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
     auto bar = [&](int i) { return smem_u32(bars + i); };
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kOffMisc);
@@ -440,9 +456,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Built by warps 0-11 and 18-21 (synchronised by a named barrier), while the
     // transposers, the producer and the store issuer start their work.  Warp
     // (quarter q, rank e within its quarter) has prologue thread index ptid.
-    const bool builder = warp < 12 || (warp >= 18 && warp < 22);
-    const int pq = warp & 3, pe = warp < 12 ? warp >> 2 : 3;
-    const int ptid = (pe * 4 + pq) * 32 + lane;
     // Stage 1: thread (c, m, qn) runs the powers lambda^n, n in [16 qn, 16 qn + 16),
     // of mode m of channel c: the U rows (Re, -Im of c lambda^(n+1)), the W-row
     // words (lambda^n packed in pairs of n), and Re(c lambda^n) summed over the
@@ -450,9 +463,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (builder) {
         const int c = ptid >> 6, m = (ptid >> 2) & 15, qn = ptid & 3;
         const int pm = (d0 + c) * kModes + m;
-        const float ga = args.decay[pm], om = args.freq[pm];
+        const float ga = p_decay, om = p_freq;
         const float2 lam = lambda_pow(ga, om, 1.0f);
-        const float2 cf = mode_coef(args.amp[pm], args.phase[pm]);
+        const float2 cf = mode_coef(p_amp, p_phase);
         if (args.coef_out && b == 0 && seg == 0 && qn == 0)
             args.coef_out[pm] = make_float4(lam.x, lam.y, cf.x, cf.y);
         float2 pw = lambda_pow(ga, om, (float)(16 * qn));
@@ -739,23 +752,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         };
         bool ok = true;
         // State-only passes, then (segments with later ones) publish the end state
-        // from a zero start: every lane stores, fences and counts.
+        // from a zero start: every lane stores its state, then releases its flag.
         for (int v = 0; v < nA && ok; ++v) ok = scan_tile(v);
         if (ok && nA > 0) {
-            args.seg_state[((seg_row + seg) * D + d0 + ch) * kModes + m] = S;
-            __threadfence();
-            atomicAdd(args.seg_flag + (seg_row + seg) * (D / kDG) + g, 1);
+            const int64_t at = ((seg_row + seg) * D + d0 + ch) * kModes + m;
+            args.seg_state[at] = S;
+            asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(args.seg_flag + at), "l"(args.epoch)
+                         : "memory");
         }
         // Carry in for the output passes: the earlier segments' end states, each
         // advanced to the end of segment seg - 1 (full segments of seg_tiles tiles).
         if (kSeg && ok) {
             S = make_float2(0.0f, 0.0f);
             for (int r = 0; r < seg; ++r) {
-                if (!wait_flag(args.seg_flag + (seg_row + r) * (D / kDG) + g, 128, abort_flag)) {
+                const int64_t at = ((seg_row + r) * D + d0 + ch) * kModes + m;
+                if (!wait_flag(args.seg_flag + at, args.epoch, abort_flag)) {
                     ok = false;
                     break;
                 }
-                const float2 lr = __ldcg(args.seg_state + ((seg_row + r) * D + d0 + ch) * kModes + m);
+                const float2 lr = __ldcg(args.seg_state + at);
                 const float2 P = lambda_pow(args.decay[pm], args.freq[pm],
                                             (float)((int64_t)(seg - 1 - r) * args.seg_tiles * kTile));
                 S = cfma(P, lr, S);
@@ -899,7 +914,7 @@ bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
 size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int) {
     const Segments sg = segments(B, L, D);
     if (sg.nseg < 2) return 0;
-    return seg_state_bytes(B, sg.nseg, D) + (size_t)B * sg.nseg * (D / kDG) * sizeof(int);
+    return 2 * seg_state_bytes(B, sg.nseg, D);  // states, then their epoch flags
 }
 
 cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int M,
@@ -944,6 +959,7 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.seg_tiles = sg.seg_tiles;
     a.seg_state = nullptr;
     a.seg_flag = nullptr;
+    a.epoch = 0;
     dim3 grid((unsigned)(D / kDG), (unsigned)B, (unsigned)sg.nseg);
     if (sg.nseg < 2) {
         k_prefill_tc<false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, a);
@@ -954,11 +970,13 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     // cooperative launch guarantees all CTAs are resident together.
     if (!ws) return cudaErrorInvalidValue;
     a.seg_state = static_cast<float2 *>(ws);
-    a.seg_flag = reinterpret_cast<int *>(static_cast<char *>(ws) + seg_state_bytes(B, sg.nseg, D));
-    cudaError_t e = cudaMemsetAsync(a.seg_flag, 0, (size_t)B * sg.nseg * (D / kDG) * sizeof(int), st);
-    if (e != cudaSuccess) return e;
+    a.seg_flag = reinterpret_cast<unsigned long long *>(static_cast<char *>(ws) + seg_state_bytes(B, sg.nseg, D));
+    // Flags carry the launch's epoch, so values left by earlier launches (smaller
+    // epochs) never pass for this one and the flags need no clearing.
+    static std::atomic<unsigned long long> epoch{0x5eed0000ull};
+    a.epoch = ++epoch;
     void *kargs[] = {&mx, &my, &a};
-    e = cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_prefill_tc<true>), grid, dim3(kThreads), kargs,
+    cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_prefill_tc<true>), grid, dim3(kThreads), kargs,
                                     (size_t)kSmemBytes, st);
     count_launches(1);
     return e;
