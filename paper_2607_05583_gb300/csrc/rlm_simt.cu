@@ -217,11 +217,17 @@ __global__ void __launch_bounds__(kBlock) k_chunk_backward(
     }
     const int64_t tau0 = t0 + (int64_t)k * C;
     const int i0 = tau0 < 0 ? (int)(-tau0) : 0;
+    // The next token's drives are loaded before this token's arithmetic.
+    auto at = [&](int i) { return ((int64_t)b * L + (L - 1 - (tau0 + i))) * D + d; };
+    float u_next = active && i0 < C ? ld_elem(dy + at(i0)) : 0.0f;
+    float x_next = active && i0 < C ? ld_elem(x + at(i0)) : 0.0f;
     for (int i = i0; i < C; ++i) {
-        const int64_t t = L - 1 - (tau0 + i);
-        const int64_t e = ((int64_t)b * L + t) * D + d;
-        const float u = active ? ld_elem(dy + e) : 0.0f;
-        const float xv = active ? ld_elem(x + e) : 0.0f;
+        const int64_t e = at(i);
+        const float u = u_next, xv = x_next;
+        if (active && i + 1 < C) {
+            u_next = ld_elem(dy + at(i + 1));
+            x_next = ld_elem(x + at(i + 1));
+        }
         float acc = 0.0f;
 #pragma unroll
         for (int j = 0; j < MG; ++j) {
