@@ -181,6 +181,17 @@ def test_row_io_measurement_byte_count(lib):
     assert lib.rlm_measure_row_io_bytes(131072, 250, 16, 128) == 0
 
 
+def test_prefill_workspace_only_when_the_sequence_is_segmented(lib):
+    # The tensor-core prefill splits the sequence when batch rows x channel groups
+    # leave SMs idle; it then needs room for each segment's end state and flag.
+    few = rlm.rlm_prefill_workspace_size(1, 32768, 256, 16, rlm.RLM_BF16)
+    many = rlm.rlm_prefill_workspace_size(64, 32768, 256, 16, rlm.RLM_BF16)
+    assert many == 0
+    assert few > 0 and few % 256 == 0
+    # states and epoch flags: 2 x 8 bytes per (b, segment, d, m)
+    assert few % (2 * 256 * 16 * 8) == 0
+
+
 def test_workspace_queries_are_host_only_and_monotone(lib):
     a = lib.rlm_prefill_workspace_size(1, 1000, 64, 4, rlm.RLM_F32)
     b = lib.rlm_prefill_workspace_size(4, 100000, 64, 4, rlm.RLM_F32)
