@@ -123,6 +123,27 @@ def test_prefill_is_deterministic():
     assert torch.equal(y1, y2) and torch.equal(s1.s, s2.s) and torch.equal(s1.coef, s2.coef)
 
 
+def test_segmented_prefill_reuses_one_workspace():
+    """Few batch rows split the sequence into segments that publish their end
+    states in the workspace (epoch-tagged flags, never cleared): consecutive calls
+    with different inputs and one workspace must each match the oracle."""
+    B, L, D, M = 1, 2048 * 6 + 300, 64, 16
+    assert rlm.rlm_prefill_workspace_size(B, L, D, M, torch.bfloat16) > 0
+    work = torch.empty(rlm.rlm_prefill_workspace_size(B, L, D, M, torch.bfloat16),
+                       dtype=torch.uint8, device="cuda")
+    for seed in (31, 32, 33):
+        inp = make_inputs(B, L, D, M, "bf16", seed=seed)
+        x = to_dev(inp.x, "bf16")
+        p = rlm.Params.from_arrays(*inp.params())
+        y = torch.empty_like(x)
+        st = rlm.State.empty(B, D, M)
+        rlm.rlm_mix_prefill(x, p, y, st, workspace=work)
+        torch.cuda.synchronize()
+        ref, st_ref = oracle.rec_prefill(inp.x, *inp.params())
+        assert_close(to_np(y), ref, TOL["bf16"], f"y (seed {seed})")
+        _state_err(st, st_ref, TOL["bf16"])
+
+
 def test_prefill_does_not_write_outside_y():
     inp = make_inputs(2, 777, 64, 16, "bf16", seed=13)
     x = to_dev(inp.x, "bf16")
