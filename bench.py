@@ -142,11 +142,13 @@ def _dist():
 
 
 def _barrier_max(t, ws):
+    """Maximum of t over the ranks (the job's step time is its slowest rank's)."""
     if ws == 1:
         return t
     import torch
     import torch.distributed as dist
-    v = torch.tensor([t], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    v = torch.tensor([t], dtype=torch.float64, device=dev)
     dist.all_reduce(v, op=dist.ReduceOp.MAX)
     return float(v.item())
 
