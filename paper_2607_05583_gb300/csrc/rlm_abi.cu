@@ -168,8 +168,8 @@ size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype 
 }
 
 size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
-    (void)dtype;
     if (B < 1 || L < 1 || D < 1 || M < 1) return 0;
+    if (tc_backward_supported(B, L, D, M, dtype)) return tc_backward_ws_bytes(B, L, D, M);
     return simt_backward_ws_bytes(B, L, D, M);
 }
 
@@ -259,13 +259,17 @@ rlm_status rlm_mix_backward(const rlm_tensor *dy, const rlm_tensor *x, const rlm
             return fail(RLM_ERR_INVALID_ARG, "dparams pointer %d is NULL or not 16-byte aligned", i);
     if (g->D != p->D || g->M != p->M) return fail(RLM_ERR_INVALID_ARG, "dparams shape differs from params");
     const int D = (int)x->D, M = p->M;
-    if (simt_chunks(x->B, x->L, D) > 65535)
+    const bool tc = tc_backward_supported(x->B, x->L, D, M, x->dtype);
+    if (!tc && simt_chunks(x->B, x->L, D) > 65535)
         return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
     const size_t need = rlm_backward_workspace_size(x->B, x->L, D, M, x->dtype);
     if ((s = check_workspace(ln, need)) != RLM_OK) return s;
-    cudaError_t e = simt_backward(dy->ptr, x->ptr, dx->ptr, x->dtype, x->B, x->L, D, M, p->decay,
-                                  p->freq, p->amp, p->phase, g->decay, g->freq, g->amp, g->phase,
-                                  ln->workspace, static_cast<cudaStream_t>(ln->stream));
+    cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
+    cudaError_t e =
+        tc ? tc_backward(dy->ptr, x->ptr, dx->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp,
+                         p->phase, g->decay, g->freq, g->amp, g->phase, ln->workspace, st)
+           : simt_backward(dy->ptr, x->ptr, dx->ptr, x->dtype, x->B, x->L, D, M, p->decay, p->freq,
+                           p->amp, p->phase, g->decay, g->freq, g->amp, g->phase, ln->workspace, st);
     if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_backward launch");
     return RLM_OK;
 }
@@ -294,9 +298,11 @@ rlm_status rlm_validate_params(const rlm_params *p) {
 
 rlm_status rlm_get_device_status(const rlm_launch *ln) {
     if (!ln) return fail(RLM_ERR_INVALID_ARG, "launch is NULL");
-    int status = RLM_OK;
+    int status = RLM_OK, bwd = RLM_OK;
     cudaError_t e = read_and_clear_device_status(&status, static_cast<cudaStream_t>(ln->stream));
+    if (e == cudaSuccess) e = read_and_clear_bwd_status(&bwd, static_cast<cudaStream_t>(ln->stream));
     if (e != cudaSuccess) return cuda_fail(e, "rlm_get_device_status");
+    if (status == RLM_OK) status = bwd;
     if (status != RLM_OK) return fail((rlm_status)status, "a bounded device-side wait expired");
     return RLM_OK;
 }

@@ -1,0 +1,880 @@
+// rlm_backward_tc.cu -- tcgen05 tensor-core backward pass for bf16 I/O, M <= 32.
+//
+// The loss depends on y = K * x (Eq. 2, K[n] = sum_m Re(c_m lambda_m^n)), so with
+// the adjoint drive dy:
+//
+//   dx[t]  = sum_{s>=t} K[s-t] dy[s]                       anti-causal mixing
+//   G_m    = sum_t x[t] S^_m[t],  S^_m[t] = sum_{s>=t} lambda^(s-t) dy[s]
+//   P_m    = sum_t x[t] R^_m[t],  R^_m[t] = sum_{s>=t} (s-t) lambda^(s-t) dy[s]
+//
+// and the four parameter gradients follow from G and P and c = A e^{i phi}
+// (dA = Re(e^{i phi} G), dphi = -Im(c G), dgamma = -Re(c P), domega = -Im(c P)).
+//
+// Chunked form.  With chunks of C = 64 tokens, position i of chunk k, the state
+// at the start of the following chunk, S^n_k = S^(kC + C), and a = lambda^C:
+//
+//   Dp_k = sum_i lambda^i dy_{k,i}        Dq_k = sum_i i lambda^i dy_{k,i}
+//   Xp_k = sum_i lambda^(C-i) x_{k,i}     Xq_k = sum_i (C-i) lambda^(C-i) x_{k,i}
+//   S^ at chunk start:  S^_k = a S^n_k + Dp_k
+//   R^ at chunk start:  R^_k = a (R^n_k + C S^n_k) + Dq_k
+//   cross-chunk terms:  G += Xp_k S^n_k,  P += Xp_k R^n_k + Xq_k S^n_k
+//   within-chunk terms: G += sum_n lambda^n rho[n],  P += sum_n n lambda^n rho[n],
+//                       rho[n] = sum_k sum_i dy_{k,i+n} x_{k,i}   (0 <= n < C)
+//   dx_{k,i} = sum_{j>=i} K[j-i] dy_{k,j} + sum_m Re(c lambda^(C-i) S^n_k)
+//
+// Every sum over the 64 positions of a chunk is a dense product and runs on the
+// tensor cores (tcgen05.mma, kind::f16, bf16 operands, fp32 accumulators in
+// TMEM), 32 chunks (a 2048-token tile) at a time:
+//
+//   accP = [Vp ; Vq]  (128 x 64) DY       accX = [Vxp ; Vxq] (128 x 64) X
+//          (the Vp and Vxp rows as bf16 high parts plus low parts, M = 64 MMAs:
+//          the gradients are differences of products with the large Jordan
+//          state R^, so single-bf16 powers lambda^i cost up to 2 % in dgamma)
+//   accD = T' (64 x 64) DY + U' (64 x 64) S^n      (T'[i][j] = K[j-i], j >= i)
+//   accQ += DY^T X  over all tiles: Q[i][j] = sum_k dy_{k,i} x_{k,j}, whose
+//           diagonals i - j = n are rho[n]
+//
+// The chunk scan of (S^, R^) runs in reverse time in fp32 registers.
+//
+// Data layout.  The per-channel tables (48 KB) leave room for one channel per
+// CTA, so the backward works on a channel-major copy of x and dy ([B*D][Lp] bf16,
+// Lp = L rounded up to whole tiles, zero past L), written by a transpose kernel:
+// every tile of one channel is then 4 KB of contiguous memory, which TMA loads
+// with the 128-byte swizzle straight into the K-major operand layout.  dx comes
+// out channel-major and a second transpose writes the [B][L][D] field.
+//
+// One CTA = one (batch row, channel), two CTAs per SM (256 TMEM columns each):
+//   warps 0-3  scan: the warp of TMEM quarter q carries modes 8q .. 8q+7.  Lane
+//              2j + ri (ri = Re/Im) reads the Dp and Xp rows of mode 8q + j, lane
+//              16 + 2j + ri its Dq and Xq rows; all four lanes of a mode carry its
+//              complex (S^, R^) redundantly, so the recurrence needs no shuffle on
+//              its critical path.
+//   warps 4-5  dx epilogue (quarters 0, 1: positions 0-63), then the diagonal
+//              sums of Q.
+//   warp 6     TMA producer; warp 7 TMEM allocation and the dx TMA stores;
+//   warp 8     MMA issue: projections; warp 9 MMA issue: T', Q and U'.
+//
+// Every wait is bounded: after kWaitLimitCycles the waiting thread sets a shared
+// abort flag and the device status word (RLM_ERR_TIMEOUT); all roles then leave
+// their loops, drain what they issued, and the CTA frees its TMEM and returns.
+#include <cuda.h>
+
+#include <mutex>
+#include <vector>
+
+#include "rlm_device.cuh"
+#include "rlm_internal.h"
+
+namespace rlm {
+
+// Device status word of this translation unit (RLM_OK or RLM_ERR_TIMEOUT).
+__device__ int g_bwd_status = 0;
+
+namespace {
+
+constexpr int kC = 64;                 // chunk length
+constexpr int kNT = 32;                // chunks per tile
+constexpr int kTile = kC * kNT;        // 2048 tokens
+constexpr int kMaxModes = 32;          // modes the quad layout holds
+constexpr int kWarps = 10;
+constexpr int kThreads = kWarps * 32;
+constexpr int kSlots = 3;              // tile ring depth (dy + x per slot)
+constexpr int kTmemCols = 256;
+constexpr long long kWaitLimitCycles = 4000000000ll;  // about 2 s at 2 GHz
+
+// TMEM columns.
+constexpr int kColP = 0;     // [2] x 32
+constexpr int kColX = 64;    // [2] x 32
+constexpr int kColD = 128;   // [2] x 32
+constexpr int kColQ = 192;   // 64
+
+// Shared memory map (bytes from a 1024-aligned base).
+// Tables, K-major without swizzle (8-row x 16-byte core matrices, LBO 128 between
+// K groups, SBO 1024 between row groups):
+//   U'    (64 rows, K = 64 state rows 2m + ri)  at 0
+//   T'    (64 rows, K = 64 positions)           at 8192
+//   A_P   (128 rows, K = 64 positions)          at 16384
+//   A_X   (128 rows)                            at 32768
+//   A_Plo (64 rows: low parts of the Vp rows)   at 49152
+//   A_Xlo (64 rows: low parts of the Vxp rows)  at 57344
+// A_P / A_X row 32 q + l: l < 16 the (Re, Im) row l % 2 of the Vp (Vxp) part of
+// mode 8 q + l / 2, l >= 16 that of the Vq (Vxq) part of mode 8 q + (l - 16) / 2.
+// Low-part row 16 q + l (l < 16) lands, through the M = 64 accumulator layout
+// (lanes 0-15 of each quarter), on lane 32 q + l: the same Vp (Vxp) row.
+// A 128-row operand starting at U' reads T' as its rows 64-127, one starting at
+// T' reads the first half of A_P: those accumulator rows are never read.
+constexpr int kOffU = 0;
+constexpr int kOffT = 8192;
+constexpr int kOffAP = 16384;
+constexpr int kOffAX = 32768;
+constexpr int kOffAPlo = 49152;
+constexpr int kOffAXlo = 57344;
+constexpr int kOffRing = 65536;                 // [kSlots] x (dy 4 KB, x 4 KB)
+constexpr int kSlotBytes = 8192;
+constexpr int kOffBs = kOffRing + kSlots * kSlotBytes;   // [2] x (hi 4 KB, lo 4 KB)
+constexpr int kOffStage = kOffBs + 2 * 8192;             // 4 KB dx staging
+constexpr int kOffRho = kOffStage + 4096;                // [2 warps][64] fp32
+constexpr int kOffBar = kOffRho + 2 * 64 * 4;
+constexpr int kNumBars = 32;
+constexpr int kOffMisc = kOffBar + kNumBars * 8;
+constexpr int kSmemBytes = kOffMisc + 64 + 1024;         // + alignment slack
+static_assert(kOffRing % 1024 == 0 && kSlotBytes % 1024 == 0, "swizzled tiles need 1024-byte alignment");
+static_assert(kOffStage % 128 == 0, "TMA store source alignment");
+static_assert(2 * (kSmemBytes + 1024) <= 233472, "two CTAs per SM");
+// Prologue scratch (lambda^n for n = 0..64, c, K), in the carried-state and
+// staging buffers, which nobody touches before the prologue ends.
+constexpr int kPwStride = 65;
+constexpr int kOffPw = kOffBs;                                  // [32][65] float2
+constexpr int kOffCf = kOffPw + kMaxModes * kPwStride * 8;      // [32] float2
+constexpr int kOffK = kOffCf + kMaxModes * 8;                   // [64] float
+static_assert(kOffK + 64 * 4 <= kOffRho, "prologue scratch does not fit");
+
+// Barrier indices.
+constexpr int kBarSlotFull = 0;                  // [kSlots]
+constexpr int kBarSlotEmpty = kSlots;            // [kSlots]: scan warp 0 + epilogue warp 4
+constexpr int kBarPXFull = 2 * kSlots;           // [2]: projections committed
+constexpr int kBarPXEmpty = kBarPXFull + 2;      // [2]: 4 scan warps read them
+constexpr int kBarSFull = kBarPXEmpty + 2;       // [2]: 4 scan warps wrote S^n
+constexpr int kBarDFull = kBarSFull + 2;         // [2]: dx accumulator complete
+constexpr int kBarDEmpty = kBarDFull + 2;        // [2]: 2 epilogue warps read it
+constexpr int kBarBsEmpty = kBarDEmpty + 2;      // [2]: S^n operand free again
+constexpr int kBarStageFull = kBarBsEmpty + 2;   // 2 epilogue warps staged dx
+constexpr int kBarStageEmpty = kBarStageFull + 1;// staging buffer stored
+constexpr int kBarQDone = kBarStageEmpty + 1;    // every MMA of warp 9 complete
+constexpr int kBarFinalA = kBarQDone + 1;        // every MMA of warp 8 complete
+static_assert(kBarFinalA < kNumBars, "too many barriers");
+
+// ------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void bar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+__device__ __forceinline__ bool bar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ void bar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void bar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+// Bounded wait on an mbarrier phase; false once this CTA has aborted.
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int *abort_flag) {
+    if (bar_try(bar, parity)) return true;
+    long long t0 = 0;
+    for (uint32_t it = 1;; ++it) {
+        if (bar_try(bar, parity)) return true;
+        if ((it & 1023u) == 0) {
+            if (*abort_flag) return false;
+            const long long now = clock64();
+            if (t0 == 0) {
+                t0 = now;
+            } else if (now - t0 > kWaitLimitCycles) {
+                *abort_flag = 1;
+                atomicExch(&g_bwd_status, (int)RLM_ERR_TIMEOUT);
+                return false;
+            }
+        }
+    }
+}
+// Drain wait (teardown): bounded, no abort check.
+__device__ __forceinline__ void drain_bar(uint32_t bar, uint32_t parity) {
+    const long long t0 = clock64();
+    while (!bar_try(bar, parity))
+        if (clock64() - t0 > kWaitLimitCycles) break;
+}
+__device__ __forceinline__ void fence_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, int c0, int c1,
+                                            int c2, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, uint32_t src, int c0, int c1,
+                                             int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+            reinterpret_cast<uint64_t>(map)),
+        "r"(c0), "r"(c1), "r"(c2), "r"(src)
+        : "memory");
+}
+
+// UMMA shared-memory descriptors (bit 46: descriptor version; bits 61-63: layout).
+// No swizzle, K-major: LBO = byte distance of core matrices adjacent along K,
+// SBO = along M/N.
+__device__ __forceinline__ uint64_t desc_plain(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46);
+}
+// 128-byte swizzle (rows of 128 bytes, 8-row atoms of 1024 bytes).  K-major: SBO =
+// distance of 8-row groups.  MN-major: LBO = distance of 64-element groups along
+// M/N, SBO = distance of 8-row groups along K.
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+__device__ __forceinline__ void umma_ss(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                        uint32_t accum) {
+    asm volatile(
+        "{ .reg .pred p; setp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p; }" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(accum)
+        : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+          "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v) {
+    asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+// Instruction descriptors, kind::f16: fp32 accumulate, bf16 A and B, M = 128.
+// N = 32 with both operands K-major; N = 64 with both MN-major (the Q product).
+constexpr uint32_t kIdescN32 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(32 >> 3) << 17) |
+                               ((uint32_t)(128 >> 4) << 24);
+constexpr uint32_t kIdescN32M64 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(32 >> 3) << 17) |
+                                  ((uint32_t)(64 >> 4) << 24);
+constexpr uint32_t kIdescQ = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | (1u << 16) |
+                             ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+
+// Byte offset of element (row r, k) in a K-major no-swizzle operand with K = 64.
+__host__ __device__ constexpr int kmaj(int r, int k) {
+    return (r >> 3) * 1024 + (k >> 3) * 128 + (r & 7) * 16 + (k & 7) * 2;
+}
+
+struct BwdArgs {
+    const float *decay, *freq, *amp, *phase;
+    float2 *part_g, *part_p;  // [B*D][M]
+    int D, M;
+    int ntiles;               // Lp / kTile
+};
+
+__global__ void __launch_bounds__(kThreads, 2)
+    k_backward_tc(const __grid_constant__ CUtensorMap tmap_dy, const __grid_constant__ CUtensorMap tmap_x,
+                  const __grid_constant__ CUtensorMap tmap_dx, const BwdArgs args) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    const uint32_t sbase = smem_u32(smem);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int row = blockIdx.x;                 // b * D + d
+    const int d = row % args.D;
+    const int M = args.M, ntiles = args.ntiles;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
+    auto bar = [&](int i) { return smem_u32(bars + i); };
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kOffMisc);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + kOffMisc + 16);
+
+    if (tid == 0) {
+        *abort_flag = 0;
+        for (int i = 0; i < kSlots; ++i) {
+            bar_init(bar(kBarSlotFull + i), 1);
+            bar_init(bar(kBarSlotEmpty + i), 2);
+        }
+        for (int i = 0; i < 2; ++i) {
+            bar_init(bar(kBarPXFull + i), 1);
+            bar_init(bar(kBarPXEmpty + i), 4);
+            bar_init(bar(kBarSFull + i), 4);
+            bar_init(bar(kBarDFull + i), 1);
+            bar_init(bar(kBarDEmpty + i), 2);
+            bar_init(bar(kBarBsEmpty + i), 1);
+        }
+        bar_init(bar(kBarStageFull), 2);
+        bar_init(bar(kBarStageEmpty), 1);
+        bar_init(bar(kBarQDone), 1);
+        bar_init(bar(kBarFinalA), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 7) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(kTmemCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    // Tile v of the reverse walk is tile ntiles - 1 - v of the sequence.
+    auto load_tile = [&](int v) {
+        const int slot = v % kSlots;
+        const int chunk0 = (ntiles - 1 - v) * kNT;
+        const uint32_t dst = sbase + kOffRing + slot * kSlotBytes;
+        bar_expect_tx(bar(kBarSlotFull + slot), kSlotBytes);
+        tma_load_3d(dst, &tmap_dy, 0, chunk0, row, bar(kBarSlotFull + slot));
+        tma_load_3d(dst + 4096, &tmap_x, 0, chunk0, row, bar(kBarSlotFull + slot));
+    };
+    int issued = 0;
+    if (warp == 6 && lane == 0)
+        for (; issued < ntiles && issued < kSlots; ++issued) load_tile(issued);
+
+    // ------------------------------------------------------------ constants
+    // Stage 1: lambda^n (n = 0..64) and c for every mode slot (zero past M).
+    float2 *pw = reinterpret_cast<float2 *>(smem + kOffPw);
+    float2 *cf = reinterpret_cast<float2 *>(smem + kOffCf);
+    float *kt = reinterpret_cast<float *>(smem + kOffK);
+    for (int it = tid; it < kMaxModes * kPwStride; it += kThreads) {
+        const int m = it / kPwStride, n = it % kPwStride;
+        pw[it] = m < M ? lambda_pow(args.decay[d * M + m], args.freq[d * M + m], (float)n)
+                       : make_float2(0.0f, 0.0f);
+    }
+    if (tid < kMaxModes)
+        cf[tid] = tid < M ? mode_coef(args.amp[d * M + tid], args.phase[d * M + tid]) : make_float2(0.0f, 0.0f);
+    if (tid < 128) reinterpret_cast<float *>(smem + kOffRho)[tid] = 0.0f;
+    __syncthreads();
+    // Stage 2: K[n] (Eq. 1 at integer lags, modes summed in a fixed order), the
+    // projection tables and the up-projection U'.
+    if (tid < kC) {
+        float s = 0.0f;
+        for (int m = 0; m < kMaxModes; ++m) {
+            const float2 p = pw[m * kPwStride + tid], c = cf[m];
+            s = fmaf(c.x, p.x, fmaf(-c.y, p.y, s));
+        }
+        kt[tid] = s;
+    }
+    for (int it = tid; it < 2 * 128 * 32 + 64 * 32; it += kThreads) {
+        uint32_t word, off;
+        if (it < 2 * 128 * 32) {
+            // A_P / A_X row r = 32 q + l, K pair (k, k + 1); the Vp (Vxp) rows
+            // also write their low parts to row 16 q + l of A_Plo (A_Xlo).
+            const int tab = it >> 12, r = (it >> 5) & 127, k = 2 * (it & 31);
+            const int l = r & 31, m = 8 * (r >> 5) + ((l & 15) >> 1), ri = l & 1;
+            const bool jordan = l >= 16;
+            float v[2];
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int kk = k + e;
+                const int n = tab == 0 ? kk : kC - kk;   // lambda^i  or  lambda^(C-i)
+                const float2 p = pw[m * kPwStride + n];
+                const float w = ri ? p.y : p.x;
+                v[e] = jordan ? (float)n * w : w;
+            }
+            word = pack_bf16x2(v[0], v[1]);
+            off = (tab == 0 ? kOffAP : kOffAX) + kmaj(r, k);
+            if (!jordan) {
+                const uint32_t lo = pack_bf16x2(v[0] - __uint_as_float(word << 16),
+                                                v[1] - __uint_as_float(word & 0xffff0000u));
+                *reinterpret_cast<uint32_t *>(smem + (tab == 0 ? kOffAPlo : kOffAXlo) +
+                                              kmaj(16 * (r >> 5) + l, k)) = lo;
+            }
+        } else {
+            // U'[i][2m + ri]: Re(c lambda^(C-i)), -Im(c lambda^(C-i)).
+            const int j = it - 2 * 128 * 32, i = j >> 5, m = j & 31;
+            const float2 z = cmul(cf[m], pw[m * kPwStride + (kC - i)]);
+            word = pack_bf16x2(z.x, -z.y);
+            off = kOffU + kmaj(i, 2 * m);
+        }
+        *reinterpret_cast<uint32_t *>(smem + off) = word;
+    }
+    __syncthreads();
+    // Stage 3: the transposed Toeplitz block T'[i][j] = K[j - i] (j >= i).
+    for (int it = tid; it < 64 * 32; it += kThreads) {
+        const int i = it >> 5, j = 2 * (it & 31);
+        const float a = j >= i ? kt[j - i] : 0.0f;
+        const float b = j + 1 >= i ? kt[j + 1 - i] : 0.0f;
+        *reinterpret_cast<uint32_t *>(smem + kOffT + kmaj(i, j)) = pack_bf16x2(a, b);
+    }
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+
+    // Scan lanes: mode m = 8 q + (lane % 16) / 2, role s = 2 (lane >= 16) + lane % 2
+    // (0, 1: Re/Im of the Dp and Xp rows; 2, 3: of the Dq and Xq rows); their
+    // (G, P) contributions survive the role loops for the final combination.
+    const int s = ((lane >> 4) << 1) | (lane & 1), m = 8 * (warp & 3) + ((lane & 15) >> 1);
+    const bool on = warp < 4 && m < M;
+    const float gam = on ? args.decay[d * M + m] : 0.0f;
+    const float omg = on ? args.freq[d * M + m] : 0.0f;
+    float gr = 0.0f, gi = 0.0f, pr = 0.0f, pi = 0.0f;
+    if (warp < 4) {
+        // ---------------------------------------------------- reverse chunk scan
+        const int q = warp, base = lane & 14;   // lanes base, base + 1, base + 16, base + 17
+        const float2 a = lambda_pow(gam, omg, (float)kC);
+        float2 S = make_float2(0.0f, 0.0f), R = make_float2(0.0f, 0.0f);
+        float A1 = 0.0f, A2 = 0.0f, A3 = 0.0f, A4 = 0.0f;
+        const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
+        // Word of mode m's (Re, Im) pair in chunk row 0 of the S^n operand; lane
+        // s = 0 writes the bf16 high parts, s = 1 the low parts (second 4 KB).
+        const uint32_t bs_lane = sbase + kOffBs + (m >> 2) * 128 + (m & 3) * 4 + (s == 1 ? 4096 : 0);
+        bool ok = true;
+        for (int v = 0; v < ntiles && ok; ++v) {
+            const int bb = v & 1;
+            if (!wait_bar(bar(kBarPXFull + bb), (v >> 1) & 1, abort_flag)) break;
+            tc_fence_after();
+            if (warp == 0 && lane == 0) bar_arrive(bar(kBarSlotEmpty + v % kSlots));
+            const uint32_t bs = bs_lane + bb * 8192;
+#pragma unroll
+            for (int h = 1; h >= 0; --h) {
+                uint32_t pv[16], xv[16];
+                tmem_ld16(tl + kColP + 32 * bb + 16 * h, pv);
+                tmem_ld16(tl + kColX + 32 * bb + 16 * h, xv);
+                tmem_wait_ld();
+                if (h == 1) {
+                    if (!wait_bar(bar(kBarBsEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                } else {
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) bar_arrive(bar(kBarPXEmpty + bb));
+                }
+#pragma unroll
+                for (int n = 15; n >= 0; --n) {
+                    const int k = 16 * h + n;
+                    const float p = __uint_as_float(pv[n]), x = __uint_as_float(xv[n]);
+                    const float dpr = __shfl_sync(0xffffffffu, p, base);
+                    const float dpi = __shfl_sync(0xffffffffu, p, base + 1);
+                    const float dqr = __shfl_sync(0xffffffffu, p, base + 16);
+                    const float dqi = __shfl_sync(0xffffffffu, p, base + 17);
+                    // Cross-chunk terms with the state entering chunk k from the right.
+                    A1 = fmaf(x, S.x, A1);
+                    A2 = fmaf(x, S.y, A2);
+                    A3 = fmaf(x, R.x, A3);
+                    A4 = fmaf(x, R.y, A4);
+                    if (s < 2) {
+                        uint32_t w = pack_bf16x2(S.x, S.y);
+                        if (s == 1)
+                            w = pack_bf16x2(S.x - __uint_as_float(w << 16),
+                                            S.y - __uint_as_float(w & 0xffff0000u));
+                        st_shared_u32(bs + (k >> 3) * 1024 + (k & 7) * 16, w);
+                    }
+                    const float2 t = make_float2(fmaf((float)kC, S.x, R.x), fmaf((float)kC, S.y, R.y));
+                    R = cfma(a, t, make_float2(dqr, dqi));
+                    S = cfma(a, S, make_float2(dpr, dpi));
+                }
+            }
+            if (!ok) break;
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) bar_arrive(bar(kBarSFull + bb));
+        }
+        // The quad's four partial products as (G, P) contributions of this lane:
+        // lane s holds x-side value s (Re Xp, Im Xp, Re Xq, Im Xq) times S^ (A1,
+        // A2) and R^ (A3, A4).
+        if (s == 0) { gr = A1; gi = A2; pr = A3; pi = A4; }
+        else if (s == 1) { gr = -A2; gi = A1; pr = -A4; pi = A3; }
+        else if (s == 2) { pr = A1; pi = A2; }
+        else { pr = -A2; pi = A1; }
+    } else if (warp < 6) {
+        // ---------------------------------------------------- dx epilogue
+        const int q = warp & 3;   // 0 or 1: positions 32 q + lane
+        const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
+        uint16_t *stage = reinterpret_cast<uint16_t *>(smem + kOffStage) + 32 * q + lane;
+        for (int v = 0; v < ntiles; ++v) {
+            const int bb = v & 1;
+            if (!wait_bar(bar(kBarDFull + bb), (v >> 1) & 1, abort_flag)) break;
+            tc_fence_after();
+            uint32_t r0[16], r1[16];
+            tmem_ld16(tl + kColD + 32 * bb, r0);
+            tmem_ld16(tl + kColD + 32 * bb + 16, r1);
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                bar_arrive(bar(kBarDEmpty + bb));
+                if (warp == 4) {
+                    bar_arrive(bar(kBarBsEmpty + bb));
+                    bar_arrive(bar(kBarSlotEmpty + v % kSlots));
+                }
+            }
+            if (!wait_bar(bar(kBarStageEmpty), (v & 1) ^ 1, abort_flag)) break;
+            uint16_t *st = stage;
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+                st[k * 64] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(r0[k])));
+                st[(k + 16) * 64] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(r1[k])));
+            }
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) bar_arrive(bar(kBarStageFull));
+        }
+        // Diagonal sums of Q (accumulated over the whole sequence): lane i of
+        // quarter q adds Q[i][j], j <= i, to rho_q[i - j].
+        if (wait_bar(bar(kBarQDone), 0, abort_flag)) {
+            tc_fence_after();
+            const int i = 32 * q + lane;
+            float *rho = reinterpret_cast<float *>(smem + kOffRho) + 64 * q;
+            for (int h = 0; h < 2 + 2 * q; ++h) {
+                uint32_t qv[16];
+                tmem_ld16(tl + kColQ + 16 * h, qv);
+                tmem_wait_ld();
+#pragma unroll
+                for (int e = 0; e < 16; ++e) {
+                    const int j = 16 * h + e;
+                    if (j <= i) rho[i - j] += __uint_as_float(qv[e]);
+                    __syncwarp();
+                }
+            }
+        }
+    } else if (warp == 6) {
+        // ---------------------------------------------------- TMA producer
+        if (lane == 0) {
+            for (; issued < ntiles; ++issued) {
+                const int slot = issued % kSlots;
+                if (!wait_bar(bar(kBarSlotEmpty + slot), ((issued / kSlots) & 1) ^ 1, abort_flag)) break;
+                load_tile(issued);
+            }
+            // Drain: every issued load lands before the CTA may exit.
+            for (int k = issued > kSlots ? issued - kSlots : 0; k < issued; ++k)
+                drain_bar(bar(kBarSlotFull + k % kSlots), (k / kSlots) & 1);
+        }
+        __syncwarp();
+    } else if (warp == 7) {
+        // ---------------------------------------------------- dx stores
+        if (lane == 0) {
+            for (int v = 0; v < ntiles; ++v) {
+                if (!wait_bar(bar(kBarStageFull), v & 1, abort_flag)) break;
+                tma_store_3d(&tmap_dx, sbase + kOffStage, 0, (ntiles - 1 - v) * kNT, row);
+                asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+                asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+                bar_arrive(bar(kBarStageEmpty));
+            }
+            asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        }
+        __syncwarp();
+    } else if (warp == 8) {
+        // ---------------------------------------------------- MMA: projections
+        if (lane == 0) {
+            const uint64_t dap = desc_plain(sbase + kOffAP, 128, 1024);
+            const uint64_t dax = desc_plain(sbase + kOffAX, 128, 1024);
+            const uint64_t dapl = desc_plain(sbase + kOffAPlo, 128, 1024);
+            const uint64_t daxl = desc_plain(sbase + kOffAXlo, 128, 1024);
+            for (int v = 0; v < ntiles; ++v) {
+                const int slot = v % kSlots, bb = v & 1;
+                if (!wait_bar(bar(kBarSlotFull + slot), (v / kSlots) & 1, abort_flag)) break;
+                if (!wait_bar(bar(kBarPXEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
+                tc_fence_after();
+                const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
+                const uint64_t ddy = desc_sw128(sdy, 16, 1024), dxx = desc_sw128(sdy + 4096, 16, 1024);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColP + 32 * bb, dap + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColX + 32 * bb, dax + ks * 16, dxx + ks * 2, kIdescN32, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColP + 32 * bb, dapl + ks * 16, ddy + ks * 2, kIdescN32M64, 1u);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColX + 32 * bb, daxl + ks * 16, dxx + ks * 2, kIdescN32M64, 1u);
+                umma_commit(bar(kBarPXFull + bb));
+            }
+            umma_commit(bar(kBarFinalA));
+            drain_bar(bar(kBarFinalA), 0);
+        }
+        __syncwarp();
+    } else {
+        // ---------------------------------------------------- MMA: T', Q, U'
+        if (lane == 0) {
+            const uint64_t dt = desc_plain(sbase + kOffT, 128, 1024);
+            const uint64_t du = desc_plain(sbase + kOffU, 128, 1024);
+            for (int v = 0; v < ntiles; ++v) {
+                const int slot = v % kSlots, bb = v & 1;
+                if (!wait_bar(bar(kBarSlotFull + slot), (v / kSlots) & 1, abort_flag)) break;
+                if (!wait_bar(bar(kBarDEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
+                tc_fence_after();
+                const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
+                const uint64_t ddy = desc_sw128(sdy, 16, 1024);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColD + 32 * bb, dt + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
+                // Q += [DY^T ; X^T] X over this tile's 32 chunks (K = chunks):
+                // MN-major views of the same swizzled tiles; rows 64-127 (X^T X)
+                // are not read.
+                const uint64_t dqa = desc_sw128(sdy, 4096, 1024);
+                const uint64_t dqb = desc_sw128(sdy + 4096, 16, 1024);
+#pragma unroll
+                for (int ks = 0; ks < 2; ++ks)
+                    umma_ss(tmem + kColQ, dqa + ks * (2048 >> 4), dqb + ks * (2048 >> 4), kIdescQ,
+                            (v > 0 || ks > 0) ? 1u : 0u);
+                if (!wait_bar(bar(kBarSFull + bb), (v >> 1) & 1, abort_flag)) break;
+                tc_fence_after();
+                const uint32_t sbs = sbase + kOffBs + bb * 8192;
+                const uint64_t dhi = desc_plain(sbs, 128, 1024), dlo = desc_plain(sbs + 4096, 128, 1024);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dhi + ks * 16, kIdescN32, 1u);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dlo + ks * 16, kIdescN32, 1u);
+                umma_commit(bar(kBarDFull + bb));
+            }
+            umma_commit(bar(kBarQDone));
+            drain_bar(bar(kBarQDone), 0);
+        }
+        __syncwarp();
+    }
+
+    tc_fence_before();
+    __syncthreads();   // every role has left its loop; rho is complete
+    tc_fence_after();
+    if (warp == 7)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(kTmemCols));
+    if (warp < 4) {
+        // Within-chunk terms: lags n = s, s + 4, ... from rho (two partial arrays),
+        // then the quad's sum; lane s = 0 writes mode m's partial (G, P).
+        const float *rho = reinterpret_cast<const float *>(smem + kOffRho);
+#pragma unroll 4
+        for (int e = 0; e < kC / 4; ++e) {
+            const int n = 4 * e + s;
+            const float r = rho[n] + rho[64 + n];
+            const float2 ln = lambda_pow(gam, omg, (float)n);
+            gr = fmaf(r, ln.x, gr);
+            gi = fmaf(r, ln.y, gi);
+            pr = fmaf(r * (float)n, ln.x, pr);
+            pi = fmaf(r * (float)n, ln.y, pi);
+        }
+#pragma unroll
+        for (int o = 1; o <= 16; o <<= 4) {
+            gr += __shfl_xor_sync(0xffffffffu, gr, o);
+            gi += __shfl_xor_sync(0xffffffffu, gi, o);
+            pr += __shfl_xor_sync(0xffffffffu, pr, o);
+            pi += __shfl_xor_sync(0xffffffffu, pi, o);
+        }
+        if (s == 0 && on) {
+            args.part_g[(int64_t)row * M + m] = make_float2(gr, gi);
+            args.part_p[(int64_t)row * M + m] = make_float2(pr, pi);
+        }
+    }
+}
+
+// ------------------------------------------------------------ layout transposes
+// [B][L][D] -> [B*D][Lp] (x and dy; grid z = 2 B), zero for t >= L.
+__global__ void __launch_bounds__(256) k_to_channel_major(const __nv_bfloat16 *__restrict__ x,
+                                                          const __nv_bfloat16 *__restrict__ dy,
+                                                          __nv_bfloat16 *__restrict__ xT,
+                                                          __nv_bfloat16 *__restrict__ dyT, int64_t L,
+                                                          int D, int64_t Lp) {
+    __shared__ uint32_t tile[64][33];   // [token][channel pair]
+    const int64_t t0 = (int64_t)blockIdx.x * 64;
+    const int c0 = blockIdx.y * 64;
+    const int b = blockIdx.z >> 1;
+    const __nv_bfloat16 *src = (blockIdx.z & 1) ? dy : x;
+    __nv_bfloat16 *dst = (blockIdx.z & 1) ? dyT : xT;
+    for (int it = threadIdx.x; it < 512; it += 256) {
+        const int r = it >> 3, vq = it & 7;
+        const int64_t t = t0 + r;
+        const int c = c0 + 8 * vq;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (t < L && c < D) val = __ldg(reinterpret_cast<const uint4 *>(src + ((int64_t)b * L + t) * D + c));
+        tile[r][4 * vq] = val.x;
+        tile[r][4 * vq + 1] = val.y;
+        tile[r][4 * vq + 2] = val.z;
+        tile[r][4 * vq + 3] = val.w;
+    }
+    __syncthreads();
+    for (int it = threadIdx.x; it < 512; it += 256) {
+        const int cr = it >> 3, vq = it & 7;
+        const int c = c0 + cr;
+        if (c >= D) continue;
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const uint32_t a = tile[8 * vq + 2 * e][cr >> 1], bw = tile[8 * vq + 2 * e + 1][cr >> 1];
+            const uint32_t lo = (cr & 1) ? (a >> 16) : (a & 0xffffu);
+            const uint32_t hi = (cr & 1) ? (bw >> 16) : (bw & 0xffffu);
+            w[e] = lo | (hi << 16);
+        }
+        *reinterpret_cast<uint4 *>(dst + ((int64_t)b * D + c) * Lp + t0 + 8 * vq) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+// [B*D][Lp] -> [B][L][D] for t < L.
+__global__ void __launch_bounds__(256) k_to_row_major(const __nv_bfloat16 *__restrict__ dxT,
+                                                      __nv_bfloat16 *__restrict__ dx, int64_t L, int D,
+                                                      int64_t Lp) {
+    __shared__ uint32_t tile[64][33];   // [channel][token pair]
+    const int64_t t0 = (int64_t)blockIdx.x * 64;
+    const int c0 = blockIdx.y * 64;
+    const int b = blockIdx.z;
+    for (int it = threadIdx.x; it < 512; it += 256) {
+        const int cr = it >> 3, vq = it & 7;
+        const int c = c0 + cr;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (c < D) val = __ldg(reinterpret_cast<const uint4 *>(dxT + ((int64_t)b * D + c) * Lp + t0 + 8 * vq));
+        tile[cr][4 * vq] = val.x;
+        tile[cr][4 * vq + 1] = val.y;
+        tile[cr][4 * vq + 2] = val.z;
+        tile[cr][4 * vq + 3] = val.w;
+    }
+    __syncthreads();
+    for (int it = threadIdx.x; it < 512; it += 256) {
+        const int r = it >> 3, vq = it & 7;
+        const int64_t t = t0 + r;
+        const int c = c0 + 8 * vq;
+        if (t >= L || c >= D) continue;
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const uint32_t a = tile[c - c0 + 2 * e][r >> 1], bw = tile[c - c0 + 2 * e + 1][r >> 1];
+            const uint32_t lo = (r & 1) ? (a >> 16) : (a & 0xffffu);
+            const uint32_t hi = (r & 1) ? (bw >> 16) : (bw & 0xffffu);
+            w[e] = lo | (hi << 16);
+        }
+        *reinterpret_cast<uint4 *>(dx + ((int64_t)b * L + t) * D + c) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+// ------------------------------------------------------------ host side
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                   const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                   const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// 3-D map over a channel-major [rows][Lp] bf16 field viewed as (64 positions,
+// Lp / 64 chunks, rows); box = one tile of one row (64 x 32 x 1).
+bool make_chunk_map(CUtensorMap *map, const void *ptr, int64_t rows, int64_t Lp, bool swizzle) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)kC, (cuuint64_t)(Lp / kC), (cuuint64_t)rows};
+    cuuint64_t strides[2] = {(cuuint64_t)kC * 2, (cuuint64_t)Lp * 2};
+    cuuint32_t box[3] = {(cuuint32_t)kC, (cuuint32_t)kNT, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int64_t padded_len(int64_t L) { return (L + kTile - 1) / kTile * kTile; }
+
+size_t field_bytes(int64_t B, int64_t L, int D) {
+    return ((size_t)B * D * padded_len(L) * 2 + 1023) / 1024 * 1024;
+}
+size_t part_bytes(int64_t B, int D, int M) {
+    return ((size_t)B * D * M * sizeof(float2) + 255) / 256 * 256;
+}
+
+}  // namespace
+
+bool tc_backward_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
+    return dt == RLM_BF16 && M >= 1 && M <= kMaxModes && D >= 8 && D % 8 == 0 && B >= 1 && L >= 1 &&
+           L <= ((int64_t)1 << 31) - kTile && B * (int64_t)D <= ((int64_t)1 << 31) - 1 &&
+           2 * B <= 65535;
+}
+
+size_t tc_backward_ws_bytes(int64_t B, int64_t L, int D, int M) {
+    return 3 * field_bytes(B, L, D) + 2 * part_bytes(B, D, M);
+}
+
+cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
+                        const float *decay, const float *freq, const float *amp, const float *phase,
+                        float *g_decay, float *g_freq, float *g_amp, float *g_phase, void *ws,
+                        cudaStream_t st) {
+    if (!ws) return cudaErrorInvalidValue;
+    const int64_t Lp = padded_len(L);
+    char *w = static_cast<char *>(ws);
+    auto *xT = reinterpret_cast<__nv_bfloat16 *>(w);
+    auto *dyT = reinterpret_cast<__nv_bfloat16 *>(w + field_bytes(B, L, D));
+    auto *dxT = reinterpret_cast<__nv_bfloat16 *>(w + 2 * field_bytes(B, L, D));
+    auto *pg = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D));
+    auto *pp = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + part_bytes(B, D, M));
+    const int64_t rows = B * (int64_t)D;
+    CUtensorMap mdy, mx, mdx;
+    if (!make_chunk_map(&mdy, dyT, rows, Lp, true) || !make_chunk_map(&mx, xT, rows, Lp, true) ||
+        !make_chunk_map(&mdx, dxT, rows, Lp, false))
+        return cudaErrorInvalidValue;
+    static std::mutex mu;
+    static std::vector<int> configured;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    {
+        std::lock_guard<std::mutex> lock(mu);
+        if ((int)configured.size() <= dev) configured.resize(dev + 1, 0);
+        if (!configured[dev]) {
+            const cudaError_t e =
+                cudaFuncSetAttribute(k_backward_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+            if (e != cudaSuccess) return e;
+            configured[dev] = 1;
+        }
+    }
+    const unsigned cgroups = (unsigned)((D + 63) / 64);
+    k_to_channel_major<<<dim3((unsigned)(Lp / 64), cgroups, (unsigned)(2 * B)), 256, 0, st>>>(
+        static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp);
+    BwdArgs a;
+    a.decay = decay;
+    a.freq = freq;
+    a.amp = amp;
+    a.phase = phase;
+    a.part_g = pg;
+    a.part_p = pp;
+    a.D = D;
+    a.M = M;
+    a.ntiles = (int)(Lp / kTile);
+    k_backward_tc<<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, mdx, a);
+    k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cgroups, (unsigned)B), 256, 0, st>>>(
+        dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp);
+    count_launches(3);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    return grad_reduce(rows / D, D, M, amp, phase, pg, pp, g_decay, g_freq, g_amp, g_phase, st);
+}
+
+cudaError_t read_and_clear_bwd_status(int *status, cudaStream_t st) {
+    cudaError_t e = cudaMemcpyFromSymbolAsync(status, g_bwd_status, sizeof(int), 0,
+                                              cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return e;
+    if ((e = cudaStreamSynchronize(st)) != cudaSuccess) return e;
+    const int zero = 0;
+    if ((e = cudaMemcpyToSymbolAsync(g_bwd_status, &zero, sizeof(int), 0, cudaMemcpyHostToDevice,
+                                     st)) != cudaSuccess)
+        return e;
+    return cudaStreamSynchronize(st);
+}
+
+}  // namespace rlm

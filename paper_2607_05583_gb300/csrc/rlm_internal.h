@@ -40,6 +40,21 @@ cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt,
                           float *g_freq, float *g_amp, float *g_phase, void *ws,
                           cudaStream_t st);
 
+// Fixed-order (fp64) sum of nparts partial (G, P) arrays of [D][M] each, then the
+// four parameter gradients.
+cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const float *phase,
+                        const float2 *G, const float2 *P, float *g_decay, float *g_freq,
+                        float *g_amp, float *g_phase, cudaStream_t st);
+
+// ---- tcgen05 backward (rlm_backward_tc.cu) -----------------------------------
+bool tc_backward_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
+size_t tc_backward_ws_bytes(int64_t B, int64_t L, int D, int M);
+cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
+                        const float *decay, const float *freq, const float *amp, const float *phase,
+                        float *g_decay, float *g_freq, float *g_amp, float *g_phase, void *ws,
+                        cudaStream_t st);
+cudaError_t read_and_clear_bwd_status(int *status, cudaStream_t st);
+
 // ---- decode (rlm_decode.cu) -----------------------------------------------
 cudaError_t decode_step(const void *x_t, void *y_t, rlm_dtype dt, int B, int D, int M,
                         float *s, const float *coef, cudaStream_t st);

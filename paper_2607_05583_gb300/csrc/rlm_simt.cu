@@ -361,6 +361,15 @@ cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_
                      freq, amp, phase, state_out, coef_out, ws, st);
 }
 
+cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const float *phase,
+                        const float2 *G, const float2 *P, float *g_decay, float *g_freq,
+                        float *g_amp, float *g_phase, cudaStream_t st) {
+    k_grad_reduce<<<(unsigned)((D * M + 255) / 256), 256, 0, st>>>(
+        nparts, D, M, 1, amp, phase, G, P, g_decay, g_freq, g_amp, g_phase);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
 cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt, int64_t B,
                           int64_t L, int D, int M, const float *decay, const float *freq,
                           const float *amp, const float *phase, float *g_decay, float *g_freq,
