@@ -262,8 +262,14 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
     return r;
 }
-__device__ __forceinline__ void st_shared_u32(uint32_t addr, uint32_t v) {
-    asm volatile("st.shared.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+__device__ __forceinline__ void st_shared_u32_if(uint32_t addr, uint32_t v, bool on) {
+    asm volatile("{ .reg .pred p; setp.ne.b32 p, %2, 0; @p st.shared.u32 [%0], %1; }" ::"r"(addr), "r"(v),
+                 "r"((uint32_t)on)
+                 : "memory");
+}
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
+                 : "memory");
 }
 
 // Instruction descriptors, kind::f16: fp32 accumulate, bf16 A and B, M = 128.
@@ -347,70 +353,97 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (; issued < ntiles && issued < kSlots; ++issued) load_tile(issued);
 
     // ------------------------------------------------------------ constants
-    // Stage 1: lambda^n (n = 0..64) and c for every mode slot (zero past M).
+    // Stage 1: lambda^n (n = 0..64) and c for every mode slot (zero past M):
+    // thread (m, g) runs n = 8g .. 8g+7 as one exact power and seven products
+    // (relative error below 1e-6, far inside the low parts' 2^-17).
     float2 *pw = reinterpret_cast<float2 *>(smem + kOffPw);
     float2 *cf = reinterpret_cast<float2 *>(smem + kOffCf);
     float *kt = reinterpret_cast<float *>(smem + kOffK);
-    for (int it = tid; it < kMaxModes * kPwStride; it += kThreads) {
-        const int m = it / kPwStride, n = it % kPwStride;
-        pw[it] = m < M ? lambda_pow(args.decay[d * M + m], args.freq[d * M + m], (float)n)
-                       : make_float2(0.0f, 0.0f);
+    if (tid < kMaxModes * 9) {
+        const int m = tid / 9, g = tid % 9;
+        float2 *o = pw + m * kPwStride + 8 * g;
+        if (m < M) {
+            const float ga = args.decay[d * M + m], om = args.freq[d * M + m];
+            const float2 l1 = lambda_pow(ga, om, 1.0f);
+            float2 z = lambda_pow(ga, om, (float)(8 * g));
+            o[0] = z;
+            if (g < 8) {
+#pragma unroll
+                for (int e = 1; e < 8; ++e) {
+                    z = cmul(z, l1);
+                    o[e] = z;
+                }
+            }
+        } else {
+            for (int e = 0; e < (g < 8 ? 8 : 1); ++e) o[e] = make_float2(0.0f, 0.0f);
+        }
+    } else if (tid >= 288 && tid < 288 + kMaxModes) {
+        const int m = tid - 288;
+        cf[m] = m < M ? mode_coef(args.amp[d * M + m], args.phase[d * M + m]) : make_float2(0.0f, 0.0f);
     }
-    if (tid < kMaxModes)
-        cf[tid] = tid < M ? mode_coef(args.amp[d * M + tid], args.phase[d * M + tid]) : make_float2(0.0f, 0.0f);
     if (tid < 128) reinterpret_cast<float *>(smem + kOffRho)[tid] = 0.0f;
     __syncthreads();
     // Stage 2: K[n] (Eq. 1 at integer lags, modes summed in a fixed order), the
-    // projection tables and the up-projection U'.
+    // projection tables and the up-projection U', one 16-byte core-matrix row
+    // (8 consecutive K elements of one row) per task; consecutive tasks take
+    // consecutive rows, so each quarter-warp's stores fill 128 contiguous bytes.
     if (tid < kC) {
-        float s = 0.0f;
+        float acc = 0.0f;
         for (int m = 0; m < kMaxModes; ++m) {
             const float2 p = pw[m * kPwStride + tid], c = cf[m];
-            s = fmaf(c.x, p.x, fmaf(-c.y, p.y, s));
+            acc = fmaf(c.x, p.x, fmaf(-c.y, p.y, acc));
         }
-        kt[tid] = s;
+        kt[tid] = acc;
     }
-    for (int it = tid; it < 2 * 128 * 32 + 64 * 32; it += kThreads) {
-        uint32_t word, off;
-        if (it < 2 * 128 * 32) {
-            // A_P / A_X row r = 32 q + l, K pair (k, k + 1); the Vp (Vxp) rows
-            // also write their low parts to row 16 q + l of A_Plo (A_Xlo).
-            const int tab = it >> 12, r = (it >> 5) & 127, k = 2 * (it & 31);
+    for (int t = tid; t < 2 * 1024 + 512; t += kThreads) {
+        if (t < 2048) {
+            // A_P (tab 0: lambda^k) / A_X (tab 1: lambda^(C-k)), row r, k = 8 kg .. 8 kg + 7.
+            const int tab = t >> 10, kg = (t >> 7) & 7, r = t & 127;
             const int l = r & 31, m = 8 * (r >> 5) + ((l & 15) >> 1), ri = l & 1;
             const bool jordan = l >= 16;
-            float v[2];
+            uint32_t hi[4], lo[4];
 #pragma unroll
-            for (int e = 0; e < 2; ++e) {
-                const int kk = k + e;
-                const int n = tab == 0 ? kk : kC - kk;   // lambda^i  or  lambda^(C-i)
-                const float2 p = pw[m * kPwStride + n];
-                const float w = ri ? p.y : p.x;
-                v[e] = jordan ? (float)n * w : w;
+            for (int e = 0; e < 4; ++e) {
+                float v[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int kk = 8 * kg + 2 * e + u;
+                    const int n = tab == 0 ? kk : kC - kk;
+                    const float2 p = pw[m * kPwStride + n];
+                    const float w = ri ? p.y : p.x;
+                    v[u] = jordan ? (float)n * w : w;
+                }
+                hi[e] = pack_bf16x2(v[0], v[1]);
+                lo[e] = pack_bf16x2(v[0] - __uint_as_float(hi[e] << 16), v[1] - __uint_as_float(hi[e] & 0xffff0000u));
             }
-            word = pack_bf16x2(v[0], v[1]);
-            off = (tab == 0 ? kOffAP : kOffAX) + kmaj(r, k);
-            if (!jordan) {
-                const uint32_t lo = pack_bf16x2(v[0] - __uint_as_float(word << 16),
-                                                v[1] - __uint_as_float(word & 0xffff0000u));
-                *reinterpret_cast<uint32_t *>(smem + (tab == 0 ? kOffAPlo : kOffAXlo) +
-                                              kmaj(16 * (r >> 5) + l, k)) = lo;
-            }
+            st_shared_v4(sbase + (tab == 0 ? kOffAP : kOffAX) + kmaj(r, 8 * kg), hi[0], hi[1], hi[2], hi[3]);
+            if (!jordan)
+                st_shared_v4(sbase + (tab == 0 ? kOffAPlo : kOffAXlo) + kmaj(16 * (r >> 5) + l, 8 * kg), lo[0], lo[1],
+                             lo[2], lo[3]);
         } else {
-            // U'[i][2m + ri]: Re(c lambda^(C-i)), -Im(c lambda^(C-i)).
-            const int j = it - 2 * 128 * 32, i = j >> 5, m = j & 31;
-            const float2 z = cmul(cf[m], pw[m * kPwStride + (kC - i)]);
-            word = pack_bf16x2(z.x, -z.y);
-            off = kOffU + kmaj(i, 2 * m);
+            // U'[i][2m + ri] = Re(c lambda^(C-i)), -Im(c lambda^(C-i)) for modes 4 kg .. 4 kg + 3.
+            const int u = t - 2048, kg = u >> 6, i = u & 63;
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int m = 4 * kg + e;
+                const float2 z = cmul(cf[m], pw[m * kPwStride + (kC - i)]);
+                w[e] = pack_bf16x2(z.x, -z.y);
+            }
+            st_shared_v4(sbase + kOffU + kmaj(i, 8 * kg), w[0], w[1], w[2], w[3]);
         }
-        *reinterpret_cast<uint32_t *>(smem + off) = word;
     }
     __syncthreads();
     // Stage 3: the transposed Toeplitz block T'[i][j] = K[j - i] (j >= i).
-    for (int it = tid; it < 64 * 32; it += kThreads) {
-        const int i = it >> 5, j = 2 * (it & 31);
-        const float a = j >= i ? kt[j - i] : 0.0f;
-        const float b = j + 1 >= i ? kt[j + 1 - i] : 0.0f;
-        *reinterpret_cast<uint32_t *>(smem + kOffT + kmaj(i, j)) = pack_bf16x2(a, b);
+    for (int t = tid; t < 512; t += kThreads) {
+        const int kg = t >> 6, i = t & 63;
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int j = 8 * kg + 2 * e;
+            w[e] = pack_bf16x2(j >= i ? kt[j - i] : 0.0f, j + 1 >= i ? kt[j + 1 - i] : 0.0f);
+        }
+        st_shared_v4(sbase + kOffT + kmaj(i, 8 * kg), w[0], w[1], w[2], w[3]);
     }
     fence_async_smem();
     tc_fence_before();
@@ -471,13 +504,12 @@ __global__ void __launch_bounds__(kThreads, 2)
                     A2 = fmaf(x, S.y, A2);
                     A3 = fmaf(x, R.x, A3);
                     A4 = fmaf(x, R.y, A4);
-                    if (s < 2) {
-                        uint32_t w = pack_bf16x2(S.x, S.y);
-                        if (s == 1)
-                            w = pack_bf16x2(S.x - __uint_as_float(w << 16),
-                                            S.y - __uint_as_float(w & 0xffff0000u));
-                        st_shared_u32(bs + (k >> 3) * 1024 + (k & 7) * 16, w);
-                    }
+                    // No branch here: a divergent store path per chunk cost more
+                    // than the whole recurrence.
+                    const uint32_t whi = pack_bf16x2(S.x, S.y);
+                    const uint32_t wlo = pack_bf16x2(S.x - __uint_as_float(whi << 16),
+                                                     S.y - __uint_as_float(whi & 0xffff0000u));
+                    st_shared_u32_if(bs + (k >> 3) * 1024 + (k & 7) * 16, (s & 1) ? wlo : whi, s < 2);
                     const float2 t = make_float2(fmaf((float)kC, S.x, R.x), fmaf((float)kC, S.y, R.y));
                     R = cfma(a, t, make_float2(dqr, dqi));
                     S = cfma(a, S, make_float2(dpr, dpi));

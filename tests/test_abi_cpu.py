@@ -200,6 +200,24 @@ def test_workspace_queries_are_host_only_and_monotone(lib):
     assert lib.rlm_prefill_workspace_size(0, 10, 8, 1, rlm.RLM_F32) == 0
 
 
+def test_tensor_core_backward_workspace(lib):
+    # bf16 I/O with M <= 32 runs the tensor-core backward: channel-major copies of
+    # x, dy and dx ([B*D][Lp] bf16, Lp = L rounded up to 2048-token tiles, each
+    # rounded up to 1 KiB) plus the per-(b, d, m) partial sums of G and P.
+    B, L, D, M = 4, 32768, 512, 32
+    field = B * D * L * 2
+    parts = 2 * B * D * M * 8
+    assert rlm.rlm_backward_workspace_size(B, L, D, M, rlm.RLM_BF16) == 3 * field + parts
+    B, L, D, M = 1, 2049, 8, 5
+    field = (B * D * 4096 * 2 + 1023) // 1024 * 1024
+    parts = 2 * ((B * D * M * 8 + 255) // 256 * 256)
+    assert rlm.rlm_backward_workspace_size(B, L, D, M, rlm.RLM_BF16) == 3 * field + parts
+    # fp32 I/O and M > 32 keep the SIMT path and its chunk workspace.
+    assert rlm.rlm_backward_workspace_size(4, 32768, 512, 32, rlm.RLM_F32) < 3 * 4 * 512 * 32768 * 2
+    parts40 = 2 * ((8 * 40 * 8 + 255) // 256 * 256)
+    assert rlm.rlm_backward_workspace_size(1, 2049, 8, 40, rlm.RLM_BF16) != 3 * field + parts40
+
+
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(rlm, "_lib", None)
     monkeypatch.setattr(cbuild, "LIB", str(tmp_path / "missing.so"))

@@ -272,6 +272,14 @@ def _backward(inp):
 @pytest.mark.parametrize("B,L,D,M,dtype", [
     (1, 256, 64, 4, "f32"), (2, 1000, 16, 7, "f32"), (2, 3001, 64, 16, "bf16"),
     (1, 4096, 32, 32, "bf16"), (1, 1, 8, 1, "f32"),
+    # tensor-core path: one token; a ragged tail shorter than a chunk with an odd
+    # mode count; one token past two tiles with M = 31; a slowly decaying mode
+    # whose dgamma is a near-cancelling projection of a large P (needs the
+    # high + low parts of the lambda^i tables)
+    (1, 1, 8, 1, "bf16"), (3, 65, 8, 5, "bf16"), (1, 2 * 2048 + 1, 16, 31, "bf16"),
+    (1, 2100, 8, 32, "bf16"),
+    # bf16 with M > 32 runs the SIMT path
+    (1, 700, 8, 40, "bf16"),
 ])
 def test_backward_matches_oracle(B, L, D, M, dtype):
     inp = make_inputs(B, L, D, M, dtype, seed=L + M, with_dy=True)
