@@ -10,49 +10,55 @@
 // and the four parameter gradients follow from G and P and c = A e^{i phi}
 // (dA = Re(e^{i phi} G), dphi = -Im(c G), dgamma = -Re(c P), domega = -Im(c P)).
 //
-// Chunked form.  With chunks of C = 64 tokens, position i of chunk k, the state
-// at the start of the following chunk, S^n_k = S^(kC + C), and a = lambda^C:
+// Chunked form.  With chunks of C = 64 tokens, position i of chunk k, the pair
+// entering chunk k from the right (S^n_k = S^(kC + C), R^n_k likewise) and
+// a = lambda^C:
 //
 //   Dp_k = sum_i lambda^i dy_{k,i}        Dq_k = sum_i i lambda^i dy_{k,i}
-//   Xp_k = sum_i lambda^(C-i) x_{k,i}     Xq_k = sum_i (C-i) lambda^(C-i) x_{k,i}
 //   S^ at chunk start:  S^_k = a S^n_k + Dp_k
 //   R^ at chunk start:  R^_k = a (R^n_k + C S^n_k) + Dq_k
-//   cross-chunk terms:  G += Xp_k S^n_k,  P += Xp_k R^n_k + Xq_k S^n_k
+//   cross-chunk terms:  G += sum_i lambda^(C-i) E_S[i],
+//                       P += sum_i lambda^(C-i) (E_R[i] + (C-i) E_S[i]),
+//                       E_S[i] = sum_k S^n_k x_{k,i},  E_R[i] = sum_k R^n_k x_{k,i}
 //   within-chunk terms: G += sum_n lambda^n rho[n],  P += sum_n n lambda^n rho[n],
 //                       rho[n] = sum_k sum_i dy_{k,i+n} x_{k,i}   (0 <= n < C)
 //   dx_{k,i} = sum_{j>=i} K[j-i] dy_{k,j} + sum_m Re(c lambda^(C-i) S^n_k)
 //
-// Every sum over the 64 positions of a chunk is a dense product and runs on the
-// tensor cores (tcgen05.mma, kind::f16, bf16 operands, fp32 accumulators in
-// TMEM), 32 chunks (a 2048-token tile) at a time:
+// Every sum over the positions or the chunks of a tile is a dense product and
+// runs on the tensor cores (tcgen05.mma, kind::f16, bf16 operands, fp32
+// accumulators in TMEM), 32 chunks (a 2048-token tile) at a time:
 //
-//   accP = [Vp ; Vq]  (128 x 64) DY       accX = [Vxp ; Vxq] (128 x 64) X
-//          (the Vp and Vxp rows as bf16 high parts plus low parts, M = 64 MMAs:
-//          the gradients are differences of products with the large Jordan
-//          state R^, so single-bf16 powers lambda^i cost up to 2 % in dgamma)
-//   accD = T' (64 x 64) DY + U' (64 x 64) S^n      (T'[i][j] = K[j-i], j >= i)
-//   accQ += DY^T X  over all tiles: Q[i][j] = sum_k dy_{k,i} x_{k,j}, whose
-//           diagonals i - j = n are rho[n]
+//   accP  = [Vp ; Vq] (128 x 64) DY   the lambda^i rows as bf16 high parts plus
+//           low parts (an extra M = 64 product): dgamma = -Re(c P) can be a
+//           near-orthogonal projection of a large P, so single-bf16 powers cost
+//           up to 2 % there
+//   accD  = T' (64 x 64) DY + U' (64 x 64) S^n      (T'[i][j] = K[j-i], j >= i)
+//   accQ += [DY^T ; X^T] X   over all tiles: Q[i][j] = sum_k dy_{k,i} x_{k,j},
+//           whose sub-diagonals i - j = n are rho[n]
+//   accE += [S^n ; R^n] X    over all tiles (K = chunks; the pair as bf16 high
+//           plus low parts): E_S and E_R, weighted by lambda^(C-i) once at the end
 //
-// The chunk scan of (S^, R^) runs in reverse time in fp32 registers.
+// The chunk scan of (S^, R^) runs in reverse time in fp32 registers: the warp
+// of TMEM quarter q carries modes 8q .. 8q+7 with four lanes per mode, lane l
+// reading accumulator row 32q + l (the Re / Im rows of Dp and of Dq); all four
+// carry the mode's complex pair (no shuffle on the recurrence), and each records
+// its own component for row 32q + l of the [S^n ; R^n] operand.
 //
-// Data layout.  The per-channel tables (48 KB) leave room for one channel per
+// Data layout.  The per-channel tables (40 KB) leave room for one channel per
 // CTA, so the backward works on a channel-major copy of x and dy ([B*D][Lp] bf16,
 // Lp = L rounded up to whole tiles, zero past L), written by a transpose kernel:
 // every tile of one channel is then 4 KB of contiguous memory, which TMA loads
-// with the 128-byte swizzle straight into the K-major operand layout.  dx comes
-// out channel-major and a second transpose writes the [B][L][D] field.
+// with the 128-byte swizzle straight into the K-major operand layout.  dx is
+// written channel-major (64-byte runs per warp store) and a second transpose
+// writes the [B][L][D] field.
 //
 // One CTA = one (batch row, channel), two CTAs per SM (256 TMEM columns each):
-//   warps 0-3  scan: the warp of TMEM quarter q carries modes 8q .. 8q+7.  Lane
-//              2j + ri (ri = Re/Im) reads the Dp and Xp rows of mode 8q + j, lane
-//              16 + 2j + ri its Dq and Xq rows; all four lanes of a mode carry its
-//              complex (S^, R^) redundantly, so the recurrence needs no shuffle on
-//              its critical path.
+//   warps 0-3  reverse scan; at the end they read E and form the cross-chunk
+//              (G, P).
 //   warps 4-5  dx epilogue (quarters 0, 1: positions 0-63), then the diagonal
 //              sums of Q.
-//   warp 6     TMA producer; warp 7 TMEM allocation and the dx TMA stores;
-//   warp 8     MMA issue: projections; warp 9 MMA issue: T', Q and U'.
+//   warp 6     TMA producer and TMEM allocation; warp 7 idle.
+//   warp 8     MMA issue: projections and Q; warp 9: T', U' and E.
 //
 // Every wait is bounded: after kWaitLimitCycles the waiting thread sets a shared
 // abort flag and the device status word (RLM_ERR_TIMEOUT); all roles then leave
@@ -75,7 +81,7 @@ namespace {
 constexpr int kC = 64;                 // chunk length
 constexpr int kNT = 32;                // chunks per tile
 constexpr int kTile = kC * kNT;        // 2048 tokens
-constexpr int kMaxModes = 32;          // modes the quad layout holds
+constexpr int kMaxModes = 32;          // one scan lane per mode
 constexpr int kWarps = 10;
 constexpr int kThreads = kWarps * 32;
 constexpr int kSlots = 3;              // tile ring depth (dy + x per slot)
@@ -83,10 +89,10 @@ constexpr int kTmemCols = 256;
 constexpr long long kWaitLimitCycles = 4000000000ll;  // about 2 s at 2 GHz
 
 // TMEM columns.
-constexpr int kColP = 0;     // [2] x 32
-constexpr int kColX = 64;    // [2] x 32
-constexpr int kColD = 128;   // [2] x 32
-constexpr int kColQ = 192;   // 64
+constexpr int kColP = 0;     // [2] x 32: [Vp ; Vq] DY
+constexpr int kColD = 64;    // [2] x 32: dx
+constexpr int kColQ = 128;   // 64: DY^T X over the sequence
+constexpr int kColE = 192;   // 64: [S^n ; R^n] X over the sequence
 
 // Shared memory map (bytes from a 1024-aligned base).
 // Tables, K-major without swizzle (8-row x 16-byte core matrices, LBO 128 between
@@ -94,35 +100,37 @@ constexpr int kColQ = 192;   // 64
 //   U'    (64 rows, K = 64 state rows 2m + ri)  at 0
 //   T'    (64 rows, K = 64 positions)           at 8192
 //   A_P   (128 rows, K = 64 positions)          at 16384
-//   A_X   (128 rows)                            at 32768
-//   A_Plo (64 rows: low parts of the Vp rows)   at 49152
-//   A_Xlo (64 rows: low parts of the Vxp rows)  at 57344
-// A_P / A_X row 32 q + l: l < 16 the (Re, Im) row l % 2 of the Vp (Vxp) part of
-// mode 8 q + l / 2, l >= 16 that of the Vq (Vxq) part of mode 8 q + (l - 16) / 2.
+//   A_Plo (64 rows: low parts of the Vp rows)   at 32768
+// A_P row 32 q + l: l < 16 the (Re, Im) row l % 2 of the Vp part of mode
+// 8 q + l / 2, l >= 16 that of the Vq part of mode 8 q + (l - 16) / 2.
 // Low-part row 16 q + l (l < 16) lands, through the M = 64 accumulator layout
-// (lanes 0-15 of each quarter), on lane 32 q + l: the same Vp (Vxp) row.
+// (lanes 0-15 of each quarter), on lane 32 q + l: the same Vp row.
 // A 128-row operand starting at U' reads T' as its rows 64-127, one starting at
 // T' reads the first half of A_P: those accumulator rows are never read.
 constexpr int kOffU = 0;
 constexpr int kOffT = 8192;
 constexpr int kOffAP = 16384;
-constexpr int kOffAX = 32768;
-constexpr int kOffAPlo = 49152;
-constexpr int kOffAXlo = 57344;
-constexpr int kOffRing = 65536;                 // [kSlots] x (dy 4 KB, x 4 KB)
+constexpr int kOffAPlo = 32768;
+constexpr int kOffRing = 40960;                 // [kSlots] x (dy 4 KB, x 4 KB)
 constexpr int kSlotBytes = 8192;
-constexpr int kOffBs = kOffRing + kSlots * kSlotBytes;   // [2] x (hi 4 KB, lo 4 KB)
-constexpr int kOffStage = kOffBs + 2 * 8192;             // 4 KB dx staging
-constexpr int kOffRho = kOffStage + 4096;                // [2 warps][64] fp32
+// The carried pair [S^n ; R^n] (128 rows x 32 chunks, bf16), high parts then
+// low parts, double-buffered.  Row 32 q + l follows the A_P row layout (S^n for
+// l < 16, R^n for l >= 16).  Element (row r, chunk k) at
+// (r / 8) * 512 + (k / 8) * 128 + (r % 8) * 16 + (k % 8) * 2: the K-major A
+// operand of the E product (LBO 128, SBO 512), and, restricted to the S^n rows of
+// one quarter, the MN-major B operand of the up-projection (N = chunks, SBO 128;
+// K = the 16 S^n rows, LBO 512).
+constexpr int kOffBs = kOffRing + kSlots * kSlotBytes;   // [2] x (hi 8 KB, lo 8 KB)
+constexpr int kBsBuf = 16384;
+constexpr int kOffRho = kOffBs + 2 * kBsBuf;             // [2 warps][64] fp32
 constexpr int kOffBar = kOffRho + 2 * 64 * 4;
 constexpr int kNumBars = 32;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;         // + alignment slack
 static_assert(kOffRing % 1024 == 0 && kSlotBytes % 1024 == 0, "swizzled tiles need 1024-byte alignment");
-static_assert(kOffStage % 128 == 0, "TMA store source alignment");
 static_assert(2 * (kSmemBytes + 1024) <= 233472, "two CTAs per SM");
-// Prologue scratch (lambda^n for n = 0..64, c, K), in the carried-state and
-// staging buffers, which nobody touches before the prologue ends.
+// Prologue scratch (lambda^n for n = 0..64, c, K), in the carried-pair buffers,
+// which nobody touches before the prologue ends.
 constexpr int kPwStride = 65;
 constexpr int kOffPw = kOffBs;                                  // [32][65] float2
 constexpr int kOffCf = kOffPw + kMaxModes * kPwStride * 8;      // [32] float2
@@ -132,17 +140,13 @@ static_assert(kOffK + 64 * 4 <= kOffRho, "prologue scratch does not fit");
 // Barrier indices.
 constexpr int kBarSlotFull = 0;                  // [kSlots]
 constexpr int kBarSlotEmpty = kSlots;            // [kSlots]: scan warp 0 + epilogue warp 4
-constexpr int kBarPXFull = 2 * kSlots;           // [2]: projections committed
-constexpr int kBarPXEmpty = kBarPXFull + 2;      // [2]: 4 scan warps read them
-constexpr int kBarSFull = kBarPXEmpty + 2;       // [2]: 4 scan warps wrote S^n
-constexpr int kBarDFull = kBarSFull + 2;         // [2]: dx accumulator complete
+constexpr int kBarPFull = 2 * kSlots;            // [2]: projections and Q committed
+constexpr int kBarPEmpty = kBarPFull + 2;        // [2]: 4 scan warps read them
+constexpr int kBarSFull = kBarPEmpty + 2;        // [2]: 4 scan warps wrote [S^n ; R^n]
+constexpr int kBarBsEmpty = kBarSFull + 2;       // [2]: U' and E products done with it
+constexpr int kBarDFull = kBarBsEmpty + 2;       // [2]: dx accumulator (and E) complete
 constexpr int kBarDEmpty = kBarDFull + 2;        // [2]: 2 epilogue warps read it
-constexpr int kBarBsEmpty = kBarDEmpty + 2;      // [2]: S^n operand free again
-constexpr int kBarStageFull = kBarBsEmpty + 2;   // 2 epilogue warps staged dx
-constexpr int kBarStageEmpty = kBarStageFull + 1;// staging buffer stored
-constexpr int kBarQDone = kBarStageEmpty + 1;    // every MMA of warp 9 complete
-constexpr int kBarFinalA = kBarQDone + 1;        // every MMA of warp 8 complete
-static_assert(kBarFinalA < kNumBars, "too many barriers");
+static_assert(kBarDEmpty + 2 <= kNumBars, "too many barriers");
 
 // ------------------------------------------------------------ PTX wrappers
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
@@ -151,12 +155,14 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) {
 __device__ __forceinline__ void bar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
 }
+// A waiting thread is suspended until the phase completes or about 0.2 ms pass,
+// so idle roles do not take issue slots from the scan.
 __device__ __forceinline__ bool bar_try(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
-        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
         : "=r"(ok)
-        : "r"(bar), "r"(parity)
+        : "r"(bar), "r"(parity), "r"(200000u)
         : "memory");
     return ok != 0;
 }
@@ -170,19 +176,14 @@ __device__ __forceinline__ void bar_expect_tx(uint32_t bar, uint32_t bytes) {
 // Bounded wait on an mbarrier phase; false once this CTA has aborted.
 __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int *abort_flag) {
     if (bar_try(bar, parity)) return true;
-    long long t0 = 0;
-    for (uint32_t it = 1;; ++it) {
+    const long long t0 = clock64();
+    for (;;) {
         if (bar_try(bar, parity)) return true;
-        if ((it & 1023u) == 0) {
-            if (*abort_flag) return false;
-            const long long now = clock64();
-            if (t0 == 0) {
-                t0 = now;
-            } else if (now - t0 > kWaitLimitCycles) {
-                *abort_flag = 1;
-                atomicExch(&g_bwd_status, (int)RLM_ERR_TIMEOUT);
-                return false;
-            }
+        if (*abort_flag) return false;
+        if (clock64() - t0 > kWaitLimitCycles) {
+            *abort_flag = 1;
+            atomicExch(&g_bwd_status, (int)RLM_ERR_TIMEOUT);
+            return false;
         }
     }
 }
@@ -254,6 +255,12 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
           "=r"(v[14]), "=r"(v[15])
         : "r"(taddr));
 }
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]),
+                   "=r"(v[6]), "=r"(v[7])
+                 : "r"(taddr));
+}
 __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -262,40 +269,59 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
     return r;
 }
-__device__ __forceinline__ void st_shared_u32_if(uint32_t addr, uint32_t v, bool on) {
-    asm volatile("{ .reg .pred p; setp.ne.b32 p, %2, 0; @p st.shared.u32 [%0], %1; }" ::"r"(addr), "r"(v),
-                 "r"((uint32_t)on)
-                 : "memory");
-}
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
     asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
                  : "memory");
 }
 
-// Instruction descriptors, kind::f16: fp32 accumulate, bf16 A and B, M = 128.
-// N = 32 with both operands K-major; N = 64 with both MN-major (the Q product).
-constexpr uint32_t kIdescN32 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(32 >> 3) << 17) |
-                               ((uint32_t)(128 >> 4) << 24);
-constexpr uint32_t kIdescN32M64 = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(32 >> 3) << 17) |
-                                  ((uint32_t)(64 >> 4) << 24);
-constexpr uint32_t kIdescQ = (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | (1u << 16) |
-                             ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+// Instruction descriptors, kind::f16: fp32 accumulate, bf16 A and B (bit 15: A
+// MN-major, bit 16: B MN-major).
+//   kIdescN32    M = 128, N = 32, both K-major          (projections, T')
+//   kIdescN32M64 M = 64,  N = 32, both K-major          (low parts of Vp)
+//   kIdescU      M = 128, N = 32, B MN-major            (up-projection of S^n)
+//   kIdescQ      M = 128, N = 64, both MN-major         (Q)
+//   kIdescE      M = 128, N = 64, B MN-major            (E)
+constexpr uint32_t kIdescBase = (1u << 4) | (1u << 7) | (1u << 10);
+constexpr uint32_t kIdescN32 = kIdescBase | ((uint32_t)(32 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+constexpr uint32_t kIdescN32M64 = kIdescBase | ((uint32_t)(32 >> 3) << 17) | ((uint32_t)(64 >> 4) << 24);
+constexpr uint32_t kIdescU = kIdescN32 | (1u << 16);
+constexpr uint32_t kIdescQ =
+    kIdescBase | (1u << 15) | (1u << 16) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+constexpr uint32_t kIdescE = kIdescBase | (1u << 16) | ((uint32_t)(64 >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
 
-// Byte offset of element (row r, k) in a K-major no-swizzle operand with K = 64.
+// Byte offset of element (row r, k) in a K-major no-swizzle table with K = 64.
 __host__ __device__ constexpr int kmaj(int r, int k) {
     return (r >> 3) * 1024 + (k >> 3) * 128 + (r & 7) * 16 + (k & 7) * 2;
+}
+// Byte offset of row r, chunk group g (chunks 8g .. 8g+7) in a carried-pair buffer.
+__host__ __device__ constexpr int pairoff(int r, int g) { return (r >> 3) * 512 + g * 128 + (r & 7) * 16; }
+
+// Row r of one carried-pair chunk group (chunks 8g .. 8g+7): bf16 high parts
+// into the first 8 KB of the buffer, low parts into the second.
+__device__ __forceinline__ void store_pair_row(uint32_t buf, int r, int g, const float (&v)[8]) {
+    uint32_t h[4], l[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        h[e] = pack_bf16x2(v[2 * e], v[2 * e + 1]);
+        l[e] = pack_bf16x2(v[2 * e] - __uint_as_float(h[e] << 16), v[2 * e + 1] - __uint_as_float(h[e] & 0xffff0000u));
+    }
+    const uint32_t a = buf + pairoff(r, g);
+    st_shared_v4(a, h[0], h[1], h[2], h[3]);
+    st_shared_v4(a + 8192, l[0], l[1], l[2], l[3]);
 }
 
 struct BwdArgs {
     const float *decay, *freq, *amp, *phase;
     float2 *part_g, *part_p;  // [B*D][M]
+    __nv_bfloat16 *dxT;       // [B*D][Lp]
+    int64_t Lp;
     int D, M;
     int ntiles;               // Lp / kTile
 };
 
 __global__ void __launch_bounds__(kThreads, 2)
     k_backward_tc(const __grid_constant__ CUtensorMap tmap_dy, const __grid_constant__ CUtensorMap tmap_x,
-                  const __grid_constant__ CUtensorMap tmap_dx, const BwdArgs args) {
+                  const BwdArgs args) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const uint32_t sbase = smem_u32(smem);
@@ -303,6 +329,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     const int row = blockIdx.x;                 // b * D + d
     const int d = row % args.D;
     const int M = args.M, ntiles = args.ntiles;
+    const int w_prod = 6;
     uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kOffBar);
     auto bar = [&](int i) { return smem_u32(bars + i); };
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kOffMisc);
@@ -315,20 +342,16 @@ __global__ void __launch_bounds__(kThreads, 2)
             bar_init(bar(kBarSlotEmpty + i), 2);
         }
         for (int i = 0; i < 2; ++i) {
-            bar_init(bar(kBarPXFull + i), 1);
-            bar_init(bar(kBarPXEmpty + i), 4);
+            bar_init(bar(kBarPFull + i), 1);
+            bar_init(bar(kBarPEmpty + i), 4);
             bar_init(bar(kBarSFull + i), 4);
+            bar_init(bar(kBarBsEmpty + i), 1);
             bar_init(bar(kBarDFull + i), 1);
             bar_init(bar(kBarDEmpty + i), 2);
-            bar_init(bar(kBarBsEmpty + i), 1);
         }
-        bar_init(bar(kBarStageFull), 2);
-        bar_init(bar(kBarStageEmpty), 1);
-        bar_init(bar(kBarQDone), 1);
-        bar_init(bar(kBarFinalA), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (warp == 7) {
+    if (warp == w_prod) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(tmem_slot)),
                      "r"(kTmemCols));
@@ -349,7 +372,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         tma_load_3d(dst + 4096, &tmap_x, 0, chunk0, row, bar(kBarSlotFull + slot));
     };
     int issued = 0;
-    if (warp == 6 && lane == 0)
+    if (warp == w_prod && lane == 0)
         for (; issued < ntiles && issued < kSlots; ++issued) load_tile(issued);
 
     // ------------------------------------------------------------ constants
@@ -384,7 +407,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (tid < 128) reinterpret_cast<float *>(smem + kOffRho)[tid] = 0.0f;
     __syncthreads();
     // Stage 2: K[n] (Eq. 1 at integer lags, modes summed in a fixed order), the
-    // projection tables and the up-projection U', one 16-byte core-matrix row
+    // projection table and the up-projection U', one 16-byte core-matrix row
     // (8 consecutive K elements of one row) per task; consecutive tasks take
     // consecutive rows, so each quarter-warp's stores fill 128 contiguous bytes.
     if (tid < kC) {
@@ -395,10 +418,11 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
         kt[tid] = acc;
     }
-    for (int t = tid; t < 2 * 1024 + 512; t += kThreads) {
-        if (t < 2048) {
-            // A_P (tab 0: lambda^k) / A_X (tab 1: lambda^(C-k)), row r, k = 8 kg .. 8 kg + 7.
-            const int tab = t >> 10, kg = (t >> 7) & 7, r = t & 127;
+    for (int t = tid; t < 1024 + 512; t += kThreads) {
+        if (t < 1024) {
+            // A_P row r, k = 8 kg .. 8 kg + 7: lambda^k (Vp rows, with low parts) or
+            // k lambda^k (Vq rows).
+            const int kg = t >> 7, r = t & 127;
             const int l = r & 31, m = 8 * (r >> 5) + ((l & 15) >> 1), ri = l & 1;
             const bool jordan = l >= 16;
             uint32_t hi[4], lo[4];
@@ -407,8 +431,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 float v[2];
 #pragma unroll
                 for (int u = 0; u < 2; ++u) {
-                    const int kk = 8 * kg + 2 * e + u;
-                    const int n = tab == 0 ? kk : kC - kk;
+                    const int n = 8 * kg + 2 * e + u;
                     const float2 p = pw[m * kPwStride + n];
                     const float w = ri ? p.y : p.x;
                     v[u] = jordan ? (float)n * w : w;
@@ -416,13 +439,11 @@ __global__ void __launch_bounds__(kThreads, 2)
                 hi[e] = pack_bf16x2(v[0], v[1]);
                 lo[e] = pack_bf16x2(v[0] - __uint_as_float(hi[e] << 16), v[1] - __uint_as_float(hi[e] & 0xffff0000u));
             }
-            st_shared_v4(sbase + (tab == 0 ? kOffAP : kOffAX) + kmaj(r, 8 * kg), hi[0], hi[1], hi[2], hi[3]);
-            if (!jordan)
-                st_shared_v4(sbase + (tab == 0 ? kOffAPlo : kOffAXlo) + kmaj(16 * (r >> 5) + l, 8 * kg), lo[0], lo[1],
-                             lo[2], lo[3]);
+            st_shared_v4(sbase + kOffAP + kmaj(r, 8 * kg), hi[0], hi[1], hi[2], hi[3]);
+            if (!jordan) st_shared_v4(sbase + kOffAPlo + kmaj(16 * (r >> 5) + l, 8 * kg), lo[0], lo[1], lo[2], lo[3]);
         } else {
             // U'[i][2m + ri] = Re(c lambda^(C-i)), -Im(c lambda^(C-i)) for modes 4 kg .. 4 kg + 3.
-            const int u = t - 2048, kg = u >> 6, i = u & 63;
+            const int u = t - 1024, kg = u >> 6, i = u & 63;
             uint32_t w[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
@@ -450,36 +471,33 @@ __global__ void __launch_bounds__(kThreads, 2)
     __syncthreads();
     tc_fence_after();
 
-    // Scan lanes: mode m = 8 q + (lane % 16) / 2, role s = 2 (lane >= 16) + lane % 2
-    // (0, 1: Re/Im of the Dp and Xp rows; 2, 3: of the Dq and Xq rows); their
-    // (G, P) contributions survive the role loops for the final combination.
-    const int s = ((lane >> 4) << 1) | (lane & 1), m = 8 * (warp & 3) + ((lane & 15) >> 1);
-    const bool on = warp < 4 && m < M;
-    const float gam = on ? args.decay[d * M + m] : 0.0f;
-    const float omg = on ? args.freq[d * M + m] : 0.0f;
+    const int last = ntiles - 1;
+    // Scan lanes: lane l of quarter q owns row 32 q + l of the projections and of
+    // [S^n ; R^n] (mode mE = 8 q + (l % 16) / 2; role s = 2 (l >= 16) + l % 2:
+    // Re / Im of Dp and S^n, of Dq and R^n); their cross-chunk (G, P) from E is
+    // kept for the final combination.
+    const int s = ((lane >> 4) << 1) | (lane & 1), mE = 8 * (warp & 3) + ((lane & 15) >> 1);
+    const bool onE = warp < 4 && mE < M;
+    const float gamE = onE ? args.decay[d * M + mE] : 0.0f, omgE = onE ? args.freq[d * M + mE] : 0.0f;
     float gr = 0.0f, gi = 0.0f, pr = 0.0f, pi = 0.0f;
     if (warp < 4) {
         // ---------------------------------------------------- reverse chunk scan
-        const int q = warp, base = lane & 14;   // lanes base, base + 1, base + 16, base + 17
-        const float2 a = lambda_pow(gam, omg, (float)kC);
-        float2 S = make_float2(0.0f, 0.0f), R = make_float2(0.0f, 0.0f);
-        float A1 = 0.0f, A2 = 0.0f, A3 = 0.0f, A4 = 0.0f;
+        const int q = warp, base = lane & 14;   // the mode's rows: base, base + 1, base + 16, base + 17
         const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
-        // Word of mode m's (Re, Im) pair in chunk row 0 of the S^n operand; lane
-        // s = 0 writes the bf16 high parts, s = 1 the low parts (second 4 KB).
-        const uint32_t bs_lane = sbase + kOffBs + (m >> 2) * 128 + (m & 3) * 4 + (s == 1 ? 4096 : 0);
+        const float2 a = lambda_pow(gamE, omgE, (float)kC);
+        float2 S = make_float2(0.0f, 0.0f), R = make_float2(0.0f, 0.0f);
+        const int prow = 32 * q + lane;         // this lane's [S^n ; R^n] row
         bool ok = true;
         for (int v = 0; v < ntiles && ok; ++v) {
             const int bb = v & 1;
-            if (!wait_bar(bar(kBarPXFull + bb), (v >> 1) & 1, abort_flag)) break;
+            if (!wait_bar(bar(kBarPFull + bb), (v >> 1) & 1, abort_flag)) break;
             tc_fence_after();
             if (warp == 0 && lane == 0) bar_arrive(bar(kBarSlotEmpty + v % kSlots));
-            const uint32_t bs = bs_lane + bb * 8192;
+            const uint32_t pb = sbase + kOffBs + bb * kBsBuf;
 #pragma unroll
-            for (int h = 1; h >= 0; --h) {
-                uint32_t pv[16], xv[16];
+            for (int h = 1; h >= 0; --h) {   // chunks 31 .. 0
+                uint32_t pv[16];
                 tmem_ld16(tl + kColP + 32 * bb + 16 * h, pv);
-                tmem_ld16(tl + kColX + 32 * bb + 16 * h, xv);
                 tmem_wait_ld();
                 if (h == 1) {
                     if (!wait_bar(bar(kBarBsEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) {
@@ -489,30 +507,25 @@ __global__ void __launch_bounds__(kThreads, 2)
                 } else {
                     tc_fence_before();
                     __syncwarp();
-                    if (lane == 0) bar_arrive(bar(kBarPXEmpty + bb));
+                    if (lane == 0) bar_arrive(bar(kBarPEmpty + bb));
                 }
 #pragma unroll
-                for (int n = 15; n >= 0; --n) {
-                    const int k = 16 * h + n;
-                    const float p = __uint_as_float(pv[n]), x = __uint_as_float(xv[n]);
-                    const float dpr = __shfl_sync(0xffffffffu, p, base);
-                    const float dpi = __shfl_sync(0xffffffffu, p, base + 1);
-                    const float dqr = __shfl_sync(0xffffffffu, p, base + 16);
-                    const float dqi = __shfl_sync(0xffffffffu, p, base + 17);
-                    // Cross-chunk terms with the state entering chunk k from the right.
-                    A1 = fmaf(x, S.x, A1);
-                    A2 = fmaf(x, S.y, A2);
-                    A3 = fmaf(x, R.x, A3);
-                    A4 = fmaf(x, R.y, A4);
-                    // No branch here: a divergent store path per chunk cost more
-                    // than the whole recurrence.
-                    const uint32_t whi = pack_bf16x2(S.x, S.y);
-                    const uint32_t wlo = pack_bf16x2(S.x - __uint_as_float(whi << 16),
-                                                     S.y - __uint_as_float(whi & 0xffff0000u));
-                    st_shared_u32_if(bs + (k >> 3) * 1024 + (k & 7) * 16, (s & 1) ? wlo : whi, s < 2);
-                    const float2 t = make_float2(fmaf((float)kC, S.x, R.x), fmaf((float)kC, S.y, R.y));
-                    R = cfma(a, t, make_float2(dqr, dqi));
-                    S = cfma(a, S, make_float2(dpr, dpi));
+                for (int g = 1; g >= 0; --g) {
+                    float own[8];
+#pragma unroll
+                    for (int n = 7; n >= 0; --n) {
+                        const float p = __uint_as_float(pv[8 * g + n]);
+                        const float dpr = __shfl_sync(0xffffffffu, p, base);
+                        const float dpi = __shfl_sync(0xffffffffu, p, base + 1);
+                        const float dqr = __shfl_sync(0xffffffffu, p, base + 16);
+                        const float dqi = __shfl_sync(0xffffffffu, p, base + 17);
+                        // The pair entering chunk 16 h + 8 g + n from the right.
+                        own[n] = (s & 2) ? ((s & 1) ? R.y : R.x) : ((s & 1) ? S.y : S.x);
+                        const float2 w = make_float2(fmaf((float)kC, S.x, R.x), fmaf((float)kC, S.y, R.y));
+                        R = cfma(a, w, make_float2(dqr, dqi));
+                        S = cfma(a, S, make_float2(dpr, dpi));
+                    }
+                    store_pair_row(pb, prow, 2 * h + g, own);
                 }
             }
             if (!ok) break;
@@ -520,21 +533,46 @@ __global__ void __launch_bounds__(kThreads, 2)
             __syncwarp();
             if (lane == 0) bar_arrive(bar(kBarSFull + bb));
         }
-        // The quad's four partial products as (G, P) contributions of this lane:
-        // lane s holds x-side value s (Re Xp, Im Xp, Re Xq, Im Xq) times S^ (A1,
-        // A2) and R^ (A3, A4).
-        if (s == 0) { gr = A1; gi = A2; pr = A3; pi = A4; }
-        else if (s == 1) { gr = -A2; gi = A1; pr = -A4; pi = A3; }
-        else if (s == 2) { pr = A1; pi = A2; }
-        else { pr = -A2; pi = A1; }
+        // E = [S^n ; R^n] X over the sequence, complete with the last dx product.
+        if (ok && wait_bar(bar(kBarDFull + (last & 1)), (last >> 1) & 1, abort_flag)) {
+            tc_fence_after();
+            // Weights lambda^(C-i), i = 63 .. 0, by successive products.
+            const float2 l1 = lambda_pow(gamE, omgE, 1.0f);
+            float2 w = l1;
+            float a1 = 0.0f, a2 = 0.0f, a3 = 0.0f, a4 = 0.0f;
+#pragma unroll 1
+            for (int h = 3; h >= 0; --h) {
+                uint32_t ev[16];
+                tmem_ld16(tl + kColE + 16 * h, ev);
+                tmem_wait_ld();
+#pragma unroll
+                for (int e = 15; e >= 0; --e) {
+                    const float x = __uint_as_float(ev[e]);
+                    const float ci = (float)(kC - (16 * h + e));
+                    a1 = fmaf(w.x, x, a1);
+                    a2 = fmaf(w.y, x, a2);
+                    a3 = fmaf(ci * w.x, x, a3);
+                    a4 = fmaf(ci * w.y, x, a4);
+                    w = cmul(w, l1);
+                }
+            }
+            // G = sum w (E_S.re + i E_S.im), P = sum w E_R + sum (C - i) w E_S.
+            if (s == 0) { gr = a1; gi = a2; pr = a3; pi = a4; }
+            else if (s == 1) { gr = -a2; gi = a1; pr = -a4; pi = a3; }
+            else if (s == 2) { pr = a1; pi = a2; }
+            else { pr = -a2; pi = a1; }
+        }
     } else if (warp < 6) {
         // ---------------------------------------------------- dx epilogue
         const int q = warp & 3;   // 0 or 1: positions 32 q + lane
         const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
-        uint16_t *stage = reinterpret_cast<uint16_t *>(smem + kOffStage) + 32 * q + lane;
+        bool ok = true;
         for (int v = 0; v < ntiles; ++v) {
             const int bb = v & 1;
-            if (!wait_bar(bar(kBarDFull + bb), (v >> 1) & 1, abort_flag)) break;
+            if (!wait_bar(bar(kBarDFull + bb), (v >> 1) & 1, abort_flag)) {
+                ok = false;
+                break;
+            }
             tc_fence_after();
             uint32_t r0[16], r1[16];
             tmem_ld16(tl + kColD + 32 * bb, r0);
@@ -549,20 +587,18 @@ __global__ void __launch_bounds__(kThreads, 2)
                     bar_arrive(bar(kBarSlotEmpty + v % kSlots));
                 }
             }
-            if (!wait_bar(bar(kBarStageEmpty), (v & 1) ^ 1, abort_flag)) break;
-            uint16_t *st = stage;
+            // Channel-major dx: each store instruction writes 64 contiguous bytes.
+            __nv_bfloat16 *out = args.dxT + (int64_t)row * args.Lp + (int64_t)(last - v) * kTile + 32 * q + lane;
 #pragma unroll
             for (int k = 0; k < 16; ++k) {
-                st[k * 64] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(r0[k])));
-                st[(k + 16) * 64] = __bfloat16_as_ushort(__float2bfloat16_rn(__uint_as_float(r1[k])));
+                out[k * kC] = __float2bfloat16_rn(__uint_as_float(r0[k]));
+                out[(k + 16) * kC] = __float2bfloat16_rn(__uint_as_float(r1[k]));
             }
-            fence_async_smem();
-            __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarStageFull));
         }
-        // Diagonal sums of Q (accumulated over the whole sequence): lane i of
-        // quarter q adds Q[i][j], j <= i, to rho_q[i - j].
-        if (wait_bar(bar(kBarQDone), 0, abort_flag)) {
+        // Diagonal sums of Q (accumulated over the whole sequence; its last
+        // product precedes the last dx product): lane i of quarter q adds
+        // Q[i][j], j <= i, to rho_q[i - j].
+        if (ok) {
             tc_fence_after();
             const int i = 32 * q + lane;
             float *rho = reinterpret_cast<float *>(smem + kOffRho) + 64 * q;
@@ -578,7 +614,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 }
             }
         }
-    } else if (warp == 6) {
+    } else if (warp == w_prod) {
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
             for (; issued < ntiles; ++issued) {
@@ -591,89 +627,80 @@ __global__ void __launch_bounds__(kThreads, 2)
                 drain_bar(bar(kBarSlotFull + k % kSlots), (k / kSlots) & 1);
         }
         __syncwarp();
-    } else if (warp == 7) {
-        // ---------------------------------------------------- dx stores
-        if (lane == 0) {
-            for (int v = 0; v < ntiles; ++v) {
-                if (!wait_bar(bar(kBarStageFull), v & 1, abort_flag)) break;
-                tma_store_3d(&tmap_dx, sbase + kOffStage, 0, (ntiles - 1 - v) * kNT, row);
-                asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-                asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
-                bar_arrive(bar(kBarStageEmpty));
-            }
-            asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-        }
-        __syncwarp();
     } else if (warp == 8) {
-        // ---------------------------------------------------- MMA: projections
+        // ---------------------------------------------------- MMA: projections and Q
         if (lane == 0) {
             const uint64_t dap = desc_plain(sbase + kOffAP, 128, 1024);
-            const uint64_t dax = desc_plain(sbase + kOffAX, 128, 1024);
             const uint64_t dapl = desc_plain(sbase + kOffAPlo, 128, 1024);
-            const uint64_t daxl = desc_plain(sbase + kOffAXlo, 128, 1024);
-            for (int v = 0; v < ntiles; ++v) {
+            int v = 0;
+            for (; v < ntiles; ++v) {
                 const int slot = v % kSlots, bb = v & 1;
                 if (!wait_bar(bar(kBarSlotFull + slot), (v / kSlots) & 1, abort_flag)) break;
-                if (!wait_bar(bar(kBarPXEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
-                tc_fence_after();
-                const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
-                const uint64_t ddy = desc_sw128(sdy, 16, 1024), dxx = desc_sw128(sdy + 4096, 16, 1024);
-#pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    umma_ss(tmem + kColP + 32 * bb, dap + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
-#pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    umma_ss(tmem + kColX + 32 * bb, dax + ks * 16, dxx + ks * 2, kIdescN32, ks > 0);
-#pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    umma_ss(tmem + kColP + 32 * bb, dapl + ks * 16, ddy + ks * 2, kIdescN32M64, 1u);
-#pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    umma_ss(tmem + kColX + 32 * bb, daxl + ks * 16, dxx + ks * 2, kIdescN32M64, 1u);
-                umma_commit(bar(kBarPXFull + bb));
-            }
-            umma_commit(bar(kBarFinalA));
-            drain_bar(bar(kBarFinalA), 0);
-        }
-        __syncwarp();
-    } else {
-        // ---------------------------------------------------- MMA: T', Q, U'
-        if (lane == 0) {
-            const uint64_t dt = desc_plain(sbase + kOffT, 128, 1024);
-            const uint64_t du = desc_plain(sbase + kOffU, 128, 1024);
-            for (int v = 0; v < ntiles; ++v) {
-                const int slot = v % kSlots, bb = v & 1;
-                if (!wait_bar(bar(kBarSlotFull + slot), (v / kSlots) & 1, abort_flag)) break;
-                if (!wait_bar(bar(kBarDEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
+                if (!wait_bar(bar(kBarPEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
                 tc_fence_after();
                 const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
                 const uint64_t ddy = desc_sw128(sdy, 16, 1024);
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
-                    umma_ss(tmem + kColD + 32 * bb, dt + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
+                    umma_ss(tmem + kColP + 32 * bb, dap + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColP + 32 * bb, dapl + ks * 16, ddy + ks * 2, kIdescN32M64, 1u);
                 // Q += [DY^T ; X^T] X over this tile's 32 chunks (K = chunks):
                 // MN-major views of the same swizzled tiles; rows 64-127 (X^T X)
                 // are not read.
-                const uint64_t dqa = desc_sw128(sdy, 4096, 1024);
-                const uint64_t dqb = desc_sw128(sdy + 4096, 16, 1024);
+                const uint64_t dqa = desc_sw128(sdy, 4096, 1024), dqb = desc_sw128(sdy + 4096, 16, 1024);
 #pragma unroll
                 for (int ks = 0; ks < 2; ++ks)
                     umma_ss(tmem + kColQ, dqa + ks * (2048 >> 4), dqb + ks * (2048 >> 4), kIdescQ,
                             (v > 0 || ks > 0) ? 1u : 0u);
-                if (!wait_bar(bar(kBarSFull + bb), (v >> 1) & 1, abort_flag)) break;
+                umma_commit(bar(kBarPFull + bb));
+            }
+            // Drain: the last group's completion implies all earlier ones.
+            if (v > 0) drain_bar(bar(kBarPFull + ((v - 1) & 1)), ((v - 1) >> 1) & 1);
+        }
+        __syncwarp();
+    } else if (warp == 9) {
+        // ---------------------------------------------------- MMA: T', U', E
+        if (lane == 0) {
+            const uint64_t dt = desc_plain(sbase + kOffT, 128, 1024);
+            const uint64_t du = desc_plain(sbase + kOffU, 128, 1024);
+            int v = 0;
+            for (; v < ntiles; ++v) {
+                const int slot = v % kSlots, bb = v & 1;
+                if (!wait_bar(bar(kBarSlotFull + slot), (v / kSlots) & 1, abort_flag)) break;
+                if (!wait_bar(bar(kBarDEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
                 tc_fence_after();
-                const uint32_t sbs = sbase + kOffBs + bb * 8192;
-                const uint64_t dhi = desc_plain(sbs, 128, 1024), dlo = desc_plain(sbs + 4096, 128, 1024);
+                const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
+                const uint64_t ddy = desc_sw128(sdy, 16, 1024), dxm = desc_sw128(sdy + 4096, 16, 1024);
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
-                    umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dhi + ks * 16, kIdescN32, 1u);
+                    umma_ss(tmem + kColD + 32 * bb, dt + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
+                if (!wait_bar(bar(kBarSFull + bb), (v >> 1) & 1, abort_flag)) {
+                    umma_commit(bar(kBarDFull + bb));   // so that the drain below tracks T'
+                    ++v;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t pb = sbase + kOffBs + bb * kBsBuf;
 #pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dlo + ks * 16, kIdescN32, 1u);
+                for (int part = 0; part < 2; ++part) {   // high parts, then low parts
+                    const uint32_t pp = pb + part * 8192;
+                    // dx += U' S^n: B = the S^n rows of quarter ks (MN-major).
+                    const uint64_t dbu = desc_plain(pp, 512, 128);
+#pragma unroll
+                    for (int ks = 0; ks < 4; ++ks)
+                        umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dbu + ks * (2048 >> 4), kIdescU, 1u);
+                    // E += [S^n ; R^n] X (K = chunks).
+                    const uint64_t dea = desc_plain(pp, 128, 512);
+#pragma unroll
+                    for (int ks = 0; ks < 2; ++ks)
+                        umma_ss(tmem + kColE, dea + ks * (256 >> 4), dxm + ks * (2048 >> 4), kIdescE,
+                                (v > 0 || part > 0 || ks > 0) ? 1u : 0u);
+                }
                 umma_commit(bar(kBarDFull + bb));
             }
-            umma_commit(bar(kBarQDone));
-            drain_bar(bar(kBarQDone), 0);
+            if (v > 0) drain_bar(bar(kBarDFull + ((v - 1) & 1)), ((v - 1) >> 1) & 1);
         }
         __syncwarp();
     }
@@ -681,18 +708,18 @@ __global__ void __launch_bounds__(kThreads, 2)
     tc_fence_before();
     __syncthreads();   // every role has left its loop; rho is complete
     tc_fence_after();
-    if (warp == 7)
+    if (warp == w_prod)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(kTmemCols));
     if (warp < 4) {
         // Within-chunk terms: lags n = s, s + 4, ... from rho (two partial arrays),
-        // then the quad's sum; lane s = 0 writes mode m's partial (G, P).
+        // then the sum over the mode's four lanes; role 0 writes the partials.
         const float *rho = reinterpret_cast<const float *>(smem + kOffRho);
 #pragma unroll 4
         for (int e = 0; e < kC / 4; ++e) {
             const int n = 4 * e + s;
             const float r = rho[n] + rho[64 + n];
-            const float2 ln = lambda_pow(gam, omg, (float)n);
+            const float2 ln = lambda_pow(gamE, omgE, (float)n);
             gr = fmaf(r, ln.x, gr);
             gi = fmaf(r, ln.y, gi);
             pr = fmaf(r * (float)n, ln.x, pr);
@@ -705,9 +732,9 @@ __global__ void __launch_bounds__(kThreads, 2)
             pr += __shfl_xor_sync(0xffffffffu, pr, o);
             pi += __shfl_xor_sync(0xffffffffu, pi, o);
         }
-        if (s == 0 && on) {
-            args.part_g[(int64_t)row * M + m] = make_float2(gr, gi);
-            args.part_p[(int64_t)row * M + m] = make_float2(pr, pi);
+        if (s == 0 && onE) {
+            args.part_g[(int64_t)row * M + mE] = make_float2(gr, gi);
+            args.part_p[(int64_t)row * M + mE] = make_float2(pr, pi);
         }
     }
 }
@@ -810,8 +837,9 @@ EncodeTiledFn encode_fn() {
 }
 
 // 3-D map over a channel-major [rows][Lp] bf16 field viewed as (64 positions,
-// Lp / 64 chunks, rows); box = one tile of one row (64 x 32 x 1).
-bool make_chunk_map(CUtensorMap *map, const void *ptr, int64_t rows, int64_t Lp, bool swizzle) {
+// Lp / 64 chunks, rows); box = one tile of one row (64 x 32 x 1), loaded with the
+// 128-byte swizzle of the UMMA operand layout.
+bool make_chunk_map(CUtensorMap *map, const void *ptr, int64_t rows, int64_t Lp) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)kC, (cuuint64_t)(Lp / kC), (cuuint64_t)rows};
@@ -819,7 +847,7 @@ bool make_chunk_map(CUtensorMap *map, const void *ptr, int64_t rows, int64_t Lp,
     cuuint32_t box[3] = {(cuuint32_t)kC, (cuuint32_t)kNT, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -857,10 +885,8 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     auto *pg = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D));
     auto *pp = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + part_bytes(B, D, M));
     const int64_t rows = B * (int64_t)D;
-    CUtensorMap mdy, mx, mdx;
-    if (!make_chunk_map(&mdy, dyT, rows, Lp, true) || !make_chunk_map(&mx, xT, rows, Lp, true) ||
-        !make_chunk_map(&mdx, dxT, rows, Lp, false))
-        return cudaErrorInvalidValue;
+    CUtensorMap mdy, mx;
+    if (!make_chunk_map(&mdy, dyT, rows, Lp) || !make_chunk_map(&mx, xT, rows, Lp)) return cudaErrorInvalidValue;
     static std::mutex mu;
     static std::vector<int> configured;
     int dev = 0;
@@ -885,10 +911,12 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     a.phase = phase;
     a.part_g = pg;
     a.part_p = pp;
+    a.dxT = dxT;
+    a.Lp = Lp;
     a.D = D;
     a.M = M;
     a.ntiles = (int)(Lp / kTile);
-    k_backward_tc<<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, mdx, a);
+    k_backward_tc<<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a);
     k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cgroups, (unsigned)B), 256, 0, st>>>(
         dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp);
     count_launches(3);
