@@ -84,7 +84,7 @@ constexpr int kTile = kC * kNT;        // 2048 tokens
 constexpr int kMaxModes = 32;          // one scan lane per mode
 constexpr int kWarps = 10;
 constexpr int kThreads = kWarps * 32;
-constexpr int kSlots = 3;              // tile ring depth (dy + x per slot)
+constexpr int kSlots = 4;              // tile ring depth (dy + x per slot)
 constexpr int kTmemCols = 256;
 constexpr long long kWaitLimitCycles = 4000000000ll;  // about 2 s at 2 GHz
 
