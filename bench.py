@@ -16,6 +16,8 @@ Also reported on the same line:
   cpu_baseline  the fp64 CPU oracle (sequential recurrence) on the host cores.
 
 ``--impl reference`` times the CPU oracle itself as the reference arm.
+``--only backward`` runs only the backward measurement and prints its object
+(a diagnostic mode for profiling that path; not the benchmark line).
 Multi-GPU (torchrun, N > 1): every rank runs its own independent batch of the
 same workload (weak scaling, replicas only; the operator has no cross-GPU
 exchange); rank 0 prints value = all ranks' tokens / max time over ranks.
@@ -71,6 +73,14 @@ def backward_bytes(B, L, D, M):
     """Per backward call: read x and dy, write dx (bf16, 6 B per token-channel),
     read params and write four gradients (32 B per (d,m))."""
     return 6 * B * L * D + 32 * D * M
+
+
+def backward_moved_bytes(B, L, D):
+    """DRAM bytes the tensor-core backward's data path moves per call (bf16,
+    L a multiple of 2048): the transpose of x and dy to channel-major (read 4 B,
+    write 4 B per token-channel), the tcgen05 kernel (read 4 B, write 2 B) and
+    the transpose of dx back (read 2 B, write 2 B): 18 B per token-channel."""
+    return 18 * B * L * D
 
 
 # ---------------------------------------------------------------- clocks
@@ -439,9 +449,27 @@ def _bench_backward(rlm, torch, dev, hbm_peak, args):
         ts.append(a.elapsed_time(b))
     ms = statistics.mean(ts)
     gbs = backward_bytes(B, L, D, M) / (ms * 1e-3) / 1e9
+    moved = backward_moved_bytes(B, L, D) / (ms * 1e-3) / 1e9
     return {"workload": "backward B=4 L=32768 D=512 M=32 bf16", "ms": round(ms, 4),
             "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 2), "achieved_GBps": round(gbs, 1),
-            "frac_hbm": round(gbs / hbm_peak, 4)}
+            "frac_hbm": round(gbs / hbm_peak, 4),
+            "data_path": "transpose to channel-major, tcgen05 kernel, transpose back, fixed-order reduction",
+            "moved_GBps": round(moved, 1), "moved_frac_hbm": round(moved / hbm_peak, 4)}
+
+
+def run_backward_only(args):
+    import torch
+
+    import paper_2607_05583_gb300 as rlm
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    rlm.load_library()
+    hbm_peak, _, peak_kind = _peaks()
+    n0 = rlm.rlm_kernels_launched()
+    out = _bench_backward(rlm, torch, dev, hbm_peak, args)
+    out.update({"mode": "backward only", "peak_kind": peak_kind,
+                "gpu_launches": rlm.rlm_kernels_launched() - n0})
+    print(json.dumps(out), flush=True)
 
 
 # ---------------------------------------------------------------- CPU oracle
@@ -512,6 +540,8 @@ def main():
     ap.add_argument("--quick", action="store_true", help="prefill only (no sweep/decode/backward)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--only", default="all", choices=["all", "backward"],
+                    help="backward: run only the backward measurement (diagnostic)")
     ap.add_argument("--soak", type=float, default=1.5,
                     help="seconds of untimed prefill before the timed steps (clock sampling)")
     args = ap.parse_args()
@@ -519,6 +549,8 @@ def main():
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args)
+    elif args.only == "backward":
+        run_backward_only(args)
     else:
         run_ours(args)
 
