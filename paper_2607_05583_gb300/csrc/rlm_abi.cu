@@ -164,6 +164,7 @@ unsigned long long rlm_kernels_launched(void) { return g_launches.load(std::memo
 size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
     if (B < 1 || L < 1 || D < 1 || M < 1) return 0;
     if (tc_prefill_supported(B, L, D, M, dtype)) return tc_prefill_ws_bytes(B, L, D, M);
+    if (tc_prefill_rev_supported(B, L, D, M, dtype)) return tc_prefill_rev_ws_bytes(B, L, D, M);
     return simt_prefill_ws_bytes(B, L, D, M);
 }
 
@@ -185,7 +186,8 @@ rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor 
     if (state_out && (s = check_state(state_out, x->B, x->D, p->M, "state_out")) != RLM_OK) return s;
     const int D = (int)x->D, M = p->M;
     const bool tc = tc_prefill_supported(x->B, x->L, D, M, x->dtype);
-    if (!tc && simt_chunks(x->B, x->L, D) > 65535)
+    const bool rev = !tc && tc_prefill_rev_supported(x->B, x->L, D, M, x->dtype);
+    if (!tc && !rev && simt_chunks(x->B, x->L, D) > 65535)
         return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
     const size_t need = rlm_prefill_workspace_size(x->B, x->L, D, M, x->dtype);
     if ((s = check_workspace(ln, need)) != RLM_OK) return s;
@@ -196,6 +198,9 @@ rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor 
     if (tc)
         e = tc_prefill(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, so,
                        co, ln->workspace, st);
+    else if (rev)
+        e = tc_prefill_rev(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, so,
+                           co, ln->workspace, st);
     else
         e = simt_prefill(x->ptr, y->ptr, x->dtype, x->B, x->L, D, M, p->decay, p->freq, p->amp,
                          p->phase, so, co, ln->workspace, st);

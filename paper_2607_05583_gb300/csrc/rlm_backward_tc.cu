@@ -312,13 +312,20 @@ __device__ __forceinline__ void store_pair_row(uint32_t buf, int r, int g, const
 
 struct BwdArgs {
     const float *decay, *freq, *amp, *phase;
-    float2 *part_g, *part_p;  // [B*D][M]
+    float2 *part_g, *part_p;  // [B*D][M] (backward)
+    float2 *state_out;        // nullable, [B*D][M] (time-reversed prefill)
+    float4 *coef_out;         // nullable, [D][M]   (time-reversed prefill)
     __nv_bfloat16 *dxT;       // [B*D][Lp]
     int64_t Lp;
     int D, M;
     int ntiles;               // Lp / kTile
 };
 
+// kGrad: the backward pass.  !kGrad: the causal prefill of a time-reversed drive
+// (dy = x reversed within [0, L)), which is the same reverse-time scan without the
+// parameter gradients: its output is y reversed, and the adjoint state it ends
+// with, sum_s lambda^s x_{L-1-s}, is the prompt's terminal state (Sec. 3.2).
+template <bool kGrad>
 __global__ void __launch_bounds__(kThreads, 2)
     k_backward_tc(const __grid_constant__ CUtensorMap tmap_dy, const __grid_constant__ CUtensorMap tmap_x,
                   const BwdArgs args) {
@@ -367,9 +374,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         const int slot = v % kSlots;
         const int chunk0 = (ntiles - 1 - v) * kNT;
         const uint32_t dst = sbase + kOffRing + slot * kSlotBytes;
-        bar_expect_tx(bar(kBarSlotFull + slot), kSlotBytes);
+        bar_expect_tx(bar(kBarSlotFull + slot), kGrad ? kSlotBytes : kSlotBytes / 2);
         tma_load_3d(dst, &tmap_dy, 0, chunk0, row, bar(kBarSlotFull + slot));
-        tma_load_3d(dst + 4096, &tmap_x, 0, chunk0, row, bar(kBarSlotFull + slot));
+        if (kGrad) tma_load_3d(dst + 4096, &tmap_x, 0, chunk0, row, bar(kBarSlotFull + slot));
     };
     int issued = 0;
     if (warp == w_prod && lane == 0)
@@ -533,8 +540,18 @@ __global__ void __launch_bounds__(kThreads, 2)
             __syncwarp();
             if (lane == 0) bar_arrive(bar(kBarSFull + bb));
         }
-        // E = [S^n ; R^n] X over the sequence, complete with the last dx product.
-        if (ok && wait_bar(bar(kBarDFull + (last & 1)), (last >> 1) & 1, abort_flag)) {
+        if (!kGrad) {
+            // The adjoint state after the first chunk is the prompt's terminal state.
+            if (ok && s == 0 && onE) {
+                if (args.state_out) args.state_out[(int64_t)row * M + mE] = S;
+                if (args.coef_out && row < args.D) {
+                    const float2 l1 = lambda_pow(gamE, omgE, 1.0f);
+                    const float2 c = mode_coef(args.amp[d * M + mE], args.phase[d * M + mE]);
+                    args.coef_out[d * M + mE] = make_float4(l1.x, l1.y, c.x, c.y);
+                }
+            }
+        } else if (ok && wait_bar(bar(kBarDFull + (last & 1)), (last >> 1) & 1, abort_flag)) {
+            // E = [S^n ; R^n] X over the sequence, complete with the last dx product.
             tc_fence_after();
             // Weights lambda^(C-i), i = 63 .. 0, by successive products.
             const float2 l1 = lambda_pow(gamE, omgE, 1.0f);
@@ -598,7 +615,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         // Diagonal sums of Q (accumulated over the whole sequence; its last
         // product precedes the last dx product): lane i of quarter q adds
         // Q[i][j], j <= i, to rho_q[i - j].
-        if (ok) {
+        if (kGrad && ok) {
             tc_fence_after();
             const int i = 32 * q + lane;
             float *rho = reinterpret_cast<float *>(smem + kOffRho) + 64 * q;
@@ -649,11 +666,13 @@ __global__ void __launch_bounds__(kThreads, 2)
                 // Q += [DY^T ; X^T] X over this tile's 32 chunks (K = chunks):
                 // MN-major views of the same swizzled tiles; rows 64-127 (X^T X)
                 // are not read.
-                const uint64_t dqa = desc_sw128(sdy, 4096, 1024), dqb = desc_sw128(sdy + 4096, 16, 1024);
+                if (kGrad) {
+                    const uint64_t dqa = desc_sw128(sdy, 4096, 1024), dqb = desc_sw128(sdy + 4096, 16, 1024);
 #pragma unroll
-                for (int ks = 0; ks < 2; ++ks)
-                    umma_ss(tmem + kColQ, dqa + ks * (2048 >> 4), dqb + ks * (2048 >> 4), kIdescQ,
-                            (v > 0 || ks > 0) ? 1u : 0u);
+                    for (int ks = 0; ks < 2; ++ks)
+                        umma_ss(tmem + kColQ, dqa + ks * (2048 >> 4), dqb + ks * (2048 >> 4), kIdescQ,
+                                (v > 0 || ks > 0) ? 1u : 0u);
+                }
                 umma_commit(bar(kBarPFull + bb));
             }
             // Drain: the last group's completion implies all earlier ones.
@@ -692,11 +711,13 @@ __global__ void __launch_bounds__(kThreads, 2)
                     for (int ks = 0; ks < 4; ++ks)
                         umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dbu + ks * (2048 >> 4), kIdescU, 1u);
                     // E += [S^n ; R^n] X (K = chunks).
-                    const uint64_t dea = desc_plain(pp, 128, 512);
+                    if (kGrad) {
+                        const uint64_t dea = desc_plain(pp, 128, 512);
 #pragma unroll
-                    for (int ks = 0; ks < 2; ++ks)
-                        umma_ss(tmem + kColE, dea + ks * (256 >> 4), dxm + ks * (2048 >> 4), kIdescE,
-                                (v > 0 || part > 0 || ks > 0) ? 1u : 0u);
+                        for (int ks = 0; ks < 2; ++ks)
+                            umma_ss(tmem + kColE, dea + ks * (256 >> 4), dxm + ks * (2048 >> 4), kIdescE,
+                                    (v > 0 || part > 0 || ks > 0) ? 1u : 0u);
+                    }
                 }
                 umma_commit(bar(kBarDFull + bb));
             }
@@ -711,7 +732,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     if (warp == w_prod)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(kTmemCols));
-    if (warp < 4) {
+    if (kGrad && warp < 4) {
         // Within-chunk terms: lags n = s, s + 4, ... from rho (two partial arrays),
         // then the sum over the mode's four lanes; role 0 writes the partials.
         const float *rho = reinterpret_cast<const float *>(smem + kOffRho);
@@ -740,24 +761,29 @@ __global__ void __launch_bounds__(kThreads, 2)
 }
 
 // ------------------------------------------------------------ layout transposes
-// [B][L][D] -> [B*D][Lp] (x and dy; grid z = 2 B), zero for t >= L.
-__global__ void __launch_bounds__(256) k_to_channel_major(const __nv_bfloat16 *__restrict__ x,
-                                                          const __nv_bfloat16 *__restrict__ dy,
-                                                          __nv_bfloat16 *__restrict__ xT,
-                                                          __nv_bfloat16 *__restrict__ dyT, int64_t L,
-                                                          int D, int64_t Lp) {
-    __shared__ uint32_t tile[64][33];   // [token][channel pair]
+// [B][L][D] -> [B*D][Lp], zero for positions >= L.  Grid z = B * nf: field f of
+// batch row b is (src0, dst0) or (src1, dst1).  rev: position s holds token
+// L - 1 - s (time reversed within [0, L)).
+__global__ void __launch_bounds__(256) k_to_channel_major(const __nv_bfloat16 *__restrict__ src0,
+                                                          const __nv_bfloat16 *__restrict__ src1,
+                                                          __nv_bfloat16 *__restrict__ dst0,
+                                                          __nv_bfloat16 *__restrict__ dst1, int64_t L, int D,
+                                                          int64_t Lp, int nf, int rev) {
+    __shared__ uint32_t tile[64][33];   // [position][channel pair]
     const int64_t t0 = (int64_t)blockIdx.x * 64;
     const int c0 = blockIdx.y * 64;
-    const int b = blockIdx.z >> 1;
-    const __nv_bfloat16 *src = (blockIdx.z & 1) ? dy : x;
-    __nv_bfloat16 *dst = (blockIdx.z & 1) ? dyT : xT;
+    const int b = blockIdx.z / nf, f = blockIdx.z % nf;
+    const __nv_bfloat16 *src = f ? src1 : src0;
+    __nv_bfloat16 *dst = f ? dst1 : dst0;
     for (int it = threadIdx.x; it < 512; it += 256) {
         const int r = it >> 3, vq = it & 7;
-        const int64_t t = t0 + r;
+        const int64_t sp = t0 + r;
         const int c = c0 + 8 * vq;
         uint4 val = make_uint4(0, 0, 0, 0);
-        if (t < L && c < D) val = __ldg(reinterpret_cast<const uint4 *>(src + ((int64_t)b * L + t) * D + c));
+        if (sp < L && c < D) {
+            const int64_t t = rev ? L - 1 - sp : sp;
+            val = __ldg(reinterpret_cast<const uint4 *>(src + ((int64_t)b * L + t) * D + c));
+        }
         tile[r][4 * vq] = val.x;
         tile[r][4 * vq + 1] = val.y;
         tile[r][4 * vq + 2] = val.z;
@@ -780,19 +806,25 @@ __global__ void __launch_bounds__(256) k_to_channel_major(const __nv_bfloat16 *_
     }
 }
 
-// [B*D][Lp] -> [B][L][D] for t < L.
-__global__ void __launch_bounds__(256) k_to_row_major(const __nv_bfloat16 *__restrict__ dxT,
-                                                      __nv_bfloat16 *__restrict__ dx, int64_t L, int D,
-                                                      int64_t Lp) {
-    __shared__ uint32_t tile[64][33];   // [channel][token pair]
+// [B*D][Lp] -> [B][L][D] for tokens t < L, token t read from position t, or from
+// L - 1 - t when rev.  A tile covers 64 tokens x 64 channels; it loads the
+// 8-aligned window of 72 positions that holds its (reversed) positions.
+__global__ void __launch_bounds__(256) k_to_row_major(const __nv_bfloat16 *__restrict__ srcT,
+                                                      __nv_bfloat16 *__restrict__ dst, int64_t L, int D,
+                                                      int64_t Lp, int rev) {
+    __shared__ uint32_t tile[64][37];   // [channel][position pair]
     const int64_t t0 = (int64_t)blockIdx.x * 64;
     const int c0 = blockIdx.y * 64;
     const int b = blockIdx.z;
-    for (int it = threadIdx.x; it < 512; it += 256) {
-        const int cr = it >> 3, vq = it & 7;
+    // First position of the window: t0 itself, or the last 64 tokens' mirror rounded down.
+    const int64_t s_lo = rev ? ((L - t0 - 64) >= 0 ? (L - t0 - 64) & ~(int64_t)7 : -((t0 + 64 - L + 7) & ~(int64_t)7)) : t0;
+    for (int it = threadIdx.x; it < 64 * 9; it += 256) {
+        const int cr = it / 9, vq = it % 9;
         const int c = c0 + cr;
+        const int64_t sp = s_lo + 8 * vq;
         uint4 val = make_uint4(0, 0, 0, 0);
-        if (c < D) val = __ldg(reinterpret_cast<const uint4 *>(dxT + ((int64_t)b * D + c) * Lp + t0 + 8 * vq));
+        if (c < D && sp >= 0 && sp < Lp)
+            val = __ldg(reinterpret_cast<const uint4 *>(srcT + ((int64_t)b * D + c) * Lp + sp));
         tile[cr][4 * vq] = val.x;
         tile[cr][4 * vq + 1] = val.y;
         tile[cr][4 * vq + 2] = val.z;
@@ -804,15 +836,16 @@ __global__ void __launch_bounds__(256) k_to_row_major(const __nv_bfloat16 *__res
         const int64_t t = t0 + r;
         const int c = c0 + 8 * vq;
         if (t >= L || c >= D) continue;
+        const int i = (int)((rev ? L - 1 - t : t) - s_lo);   // 0 <= i < 72
         uint32_t w[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
-            const uint32_t a = tile[c - c0 + 2 * e][r >> 1], bw = tile[c - c0 + 2 * e + 1][r >> 1];
-            const uint32_t lo = (r & 1) ? (a >> 16) : (a & 0xffffu);
-            const uint32_t hi = (r & 1) ? (bw >> 16) : (bw & 0xffffu);
+            const uint32_t a = tile[8 * vq + 2 * e][i >> 1], bw = tile[8 * vq + 2 * e + 1][i >> 1];
+            const uint32_t lo = (i & 1) ? (a >> 16) : (a & 0xffffu);
+            const uint32_t hi = (i & 1) ? (bw >> 16) : (bw & 0xffffu);
             w[e] = lo | (hi << 16);
         }
-        *reinterpret_cast<uint4 *>(dx + ((int64_t)b * L + t) * D + c) = make_uint4(w[0], w[1], w[2], w[3]);
+        *reinterpret_cast<uint4 *>(dst + ((int64_t)b * L + t) * D + c) = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -872,6 +905,46 @@ size_t tc_backward_ws_bytes(int64_t B, int64_t L, int D, int M) {
     return 3 * field_bytes(B, L, D) + 2 * part_bytes(B, D, M);
 }
 
+namespace {
+
+cudaError_t configure_once() {
+    static std::mutex mu;
+    static std::vector<int> configured;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    std::lock_guard<std::mutex> lock(mu);
+    if ((int)configured.size() <= dev) configured.resize(dev + 1, 0);
+    if (!configured[dev]) {
+        cudaError_t e = cudaFuncSetAttribute(k_backward_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(k_backward_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e != cudaSuccess) return e;
+        configured[dev] = 1;
+    }
+    return cudaSuccess;
+}
+
+BwdArgs base_args(const float *decay, const float *freq, const float *amp, const float *phase, __nv_bfloat16 *outT,
+                  int64_t Lp, int D, int M) {
+    BwdArgs a;
+    a.decay = decay;
+    a.freq = freq;
+    a.amp = amp;
+    a.phase = phase;
+    a.part_g = nullptr;
+    a.part_p = nullptr;
+    a.state_out = nullptr;
+    a.coef_out = nullptr;
+    a.dxT = outT;
+    a.Lp = Lp;
+    a.D = D;
+    a.M = M;
+    a.ntiles = (int)(Lp / kTile);
+    return a;
+}
+
+}  // namespace
+
 cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
                         const float *decay, const float *freq, const float *amp, const float *phase,
                         float *g_decay, float *g_freq, float *g_amp, float *g_phase, void *ws,
@@ -887,42 +960,53 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     const int64_t rows = B * (int64_t)D;
     CUtensorMap mdy, mx;
     if (!make_chunk_map(&mdy, dyT, rows, Lp) || !make_chunk_map(&mx, xT, rows, Lp)) return cudaErrorInvalidValue;
-    static std::mutex mu;
-    static std::vector<int> configured;
-    int dev = 0;
-    cudaGetDevice(&dev);
-    {
-        std::lock_guard<std::mutex> lock(mu);
-        if ((int)configured.size() <= dev) configured.resize(dev + 1, 0);
-        if (!configured[dev]) {
-            const cudaError_t e =
-                cudaFuncSetAttribute(k_backward_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
-            if (e != cudaSuccess) return e;
-            configured[dev] = 1;
-        }
-    }
+    cudaError_t e = configure_once();
+    if (e != cudaSuccess) return e;
     const unsigned cgroups = (unsigned)((D + 63) / 64);
     k_to_channel_major<<<dim3((unsigned)(Lp / 64), cgroups, (unsigned)(2 * B)), 256, 0, st>>>(
-        static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp);
-    BwdArgs a;
-    a.decay = decay;
-    a.freq = freq;
-    a.amp = amp;
-    a.phase = phase;
+        static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp, 2, 0);
+    BwdArgs a = base_args(decay, freq, amp, phase, dxT, Lp, D, M);
     a.part_g = pg;
     a.part_p = pp;
-    a.dxT = dxT;
-    a.Lp = Lp;
-    a.D = D;
-    a.M = M;
-    a.ntiles = (int)(Lp / kTile);
-    k_backward_tc<<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a);
+    k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a);
     k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cgroups, (unsigned)B), 256, 0, st>>>(
-        dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp);
+        dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp, 0);
     count_launches(3);
-    cudaError_t e = cudaGetLastError();
+    e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     return grad_reduce(rows / D, D, M, amp, phase, pg, pp, g_decay, g_freq, g_amp, g_phase, st);
+}
+
+bool tc_prefill_rev_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
+    return tc_backward_supported(B, L, D, M, dt);
+}
+
+size_t tc_prefill_rev_ws_bytes(int64_t B, int64_t L, int D, int) { return 2 * field_bytes(B, L, D); }
+
+cudaError_t tc_prefill_rev(const void *x, void *y, int64_t B, int64_t L, int D, int M, const float *decay,
+                           const float *freq, const float *amp, const float *phase, float *state_out,
+                           float *coef_out, void *ws, cudaStream_t st) {
+    if (!ws) return cudaErrorInvalidValue;
+    const int64_t Lp = padded_len(L);
+    char *w = static_cast<char *>(ws);
+    auto *xr = reinterpret_cast<__nv_bfloat16 *>(w);
+    auto *yr = reinterpret_cast<__nv_bfloat16 *>(w + field_bytes(B, L, D));
+    const int64_t rows = B * (int64_t)D;
+    CUtensorMap mx;
+    if (!make_chunk_map(&mx, xr, rows, Lp)) return cudaErrorInvalidValue;
+    cudaError_t e = configure_once();
+    if (e != cudaSuccess) return e;
+    const unsigned cgroups = (unsigned)((D + 63) / 64);
+    k_to_channel_major<<<dim3((unsigned)(Lp / 64), cgroups, (unsigned)B), 256, 0, st>>>(
+        static_cast<const __nv_bfloat16 *>(x), nullptr, xr, nullptr, L, D, Lp, 1, 1);
+    BwdArgs a = base_args(decay, freq, amp, phase, yr, Lp, D, M);
+    a.state_out = reinterpret_cast<float2 *>(state_out);
+    a.coef_out = reinterpret_cast<float4 *>(coef_out);
+    k_backward_tc<false><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mx, mx, a);
+    k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cgroups, (unsigned)B), 256, 0, st>>>(
+        yr, static_cast<__nv_bfloat16 *>(y), L, D, Lp, 1);
+    count_launches(3);
+    return cudaGetLastError();
 }
 
 cudaError_t read_and_clear_bwd_status(int *status, cudaStream_t st) {

@@ -54,6 +54,14 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
                         float *g_decay, float *g_freq, float *g_amp, float *g_phase, void *ws,
                         cudaStream_t st);
 cudaError_t read_and_clear_bwd_status(int *status, cudaStream_t st);
+// The causal prefill (bf16 I/O, M <= 32) as the same reverse-time tcgen05 scan
+// applied to the time-reversed drive; used for the M the tcgen05 prefill does not
+// cover.  state_out / coef_out may be null.
+bool tc_prefill_rev_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
+size_t tc_prefill_rev_ws_bytes(int64_t B, int64_t L, int D, int M);
+cudaError_t tc_prefill_rev(const void *x, void *y, int64_t B, int64_t L, int D, int M, const float *decay,
+                           const float *freq, const float *amp, const float *phase, float *state_out,
+                           float *coef_out, void *ws, cudaStream_t st);
 
 // ---- decode (rlm_decode.cu) -----------------------------------------------
 cudaError_t decode_step(const void *x_t, void *y_t, rlm_dtype dt, int B, int D, int M,

@@ -78,6 +78,12 @@ def test_prefill_layer6m_bf16():
     # few rows: the sequence is split into segments (one per tile; two tiles each
     # with a shorter last segment)
     (1, 2048 * 5 + 100, 8, 16, "bf16"), (1, 2048 * 24 + 5, 64, 16, "bf16"),
+    # bf16 with M != 16 (M <= 32): the time-reversed tcgen05 scan -- one token, a
+    # tail shorter than a chunk, one token past a tile, D not a multiple of 64
+    (1, 1, 8, 3, "bf16"), (2, 65, 16, 32, "bf16"), (1, 2100, 8, 31, "bf16"),
+    (2, 2048 * 2 + 7, 24, 8, "bf16"),
+    # bf16 with M > 32: the SIMT path
+    (1, 500, 8, 40, "bf16"),
 ])
 def test_prefill_edge_and_ragged_shapes(B, L, D, M, dtype):
     inp = make_inputs(B, L, D, M, dtype, seed=B * 1000 + L)
@@ -99,6 +105,37 @@ def test_prefill_long_context_sweep(B, L):
     s = st.complex().cpu().numpy()[:, chans]
     assert_close(s.real, st_ref.real, TOL["bf16"], "state re")
     assert_close(s.imag, st_ref.imag, TOL["bf16"], "state im")
+
+
+def test_prefill_training_shape_m32_sampled():
+    """Forward of the training workload (B=4, L=32768, D=512, M=32, bf16): sampled
+    channels of y and of the terminal state against the oracle."""
+    inp = make_inputs(4, 32768, 512, 32, "bf16", seed=0)
+    y, st = _prefill(inp)
+    chans = np.array([0, 101, 333, 511])
+    ref, st_ref = oracle.rec_prefill(*_sub(inp, chans))
+    assert_close(to_np(y)[:, :, chans], ref, TOL["bf16"], "y")
+    s = st.complex().cpu().numpy()[:, chans]
+    assert_close(s.real, st_ref.real, TOL["bf16"], "state re")
+    assert_close(s.imag, st_ref.imag, TOL["bf16"], "state im")
+    coef = st.coef.cpu().numpy()[chans]
+    lam = np.exp(-inp.decay[chans].astype(np.float64) + 1j * inp.freq[chans].astype(np.float64))
+    np.testing.assert_allclose(coef[..., 0], lam.real, rtol=0, atol=1e-6)
+    np.testing.assert_allclose(coef[..., 1], lam.imag, rtol=0, atol=1e-6)
+
+
+def test_time_reversed_prefill_is_causal_bit_exact():
+    """The M != 16 bf16 prefill runs as a reverse-time scan of the reversed drive;
+    perturbing x[t >= t0] must still leave y[t < t0] bit-identical."""
+    inp = make_inputs(2, 5000, 64, 8, "bf16", seed=6)
+    y1, _ = _prefill(inp, False)
+    inp2 = make_inputs(2, 5000, 64, 8, "bf16", seed=6)
+    inp2.x = inp.x.copy()
+    inp2.x[:, 2999:] = -inp2.x[:, 2999:] + 1.0
+    y2, _ = _prefill(inp2, False)
+    a, b = y1.cpu(), y2.cpu()
+    assert torch.equal(a[:, :2999], b[:, :2999])
+    assert not torch.equal(a[:, 2999:], b[:, 2999:])
 
 
 def test_prefill_is_causal_bit_exact():
