@@ -9,7 +9,8 @@ inter-chunk carry, state up-projection, epilogue and terminal state.
 Also reported on the same line:
   decode    4096 single-token rlm_mix_decode steps at B=64 (D=256, M=16) after a
             32768-token prefill, captured in a CUDA graph; tok/s and % of HBM.
-  backward  rlm_mix_backward at B=4, L=32768, D=512, M=32 (bf16 I/O).
+  backward  rlm_mix_backward at B=4, L=32768, D=512, M=32 (bf16 I/O), with the
+            training step's forward (rlm_mix_prefill) on the same shape.
   roofline  achieved algorithmic GB/s of the prefill against the measured HBM peak.
   e2e       the same prefill metric through the C ABI with pinned HOST buffers
             (host->device copy of x and device->host copy of y inside the timing).
@@ -448,13 +449,32 @@ def _bench_backward(rlm, torch, dev, hbm_peak, args):
         torch.cuda.synchronize()
         ts.append(a.elapsed_time(b))
     ms = statistics.mean(ts)
+    # The training step's forward on the same shape (bf16, M = 32: the tcgen05
+    # reverse scan of the reversed drive).
+    y = torch.empty_like(x)
+    st = rlm.State.empty(B, D, M, device=dev)
+    fw = torch.empty(max(256, rlm.rlm_prefill_workspace_size(B, L, D, M, torch.bfloat16)), dtype=torch.uint8,
+                     device=dev)
+    for _ in range(2):
+        rlm.rlm_mix_prefill(x, p, y, st, workspace=fw)
+    fts = []
+    for _ in range(3):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        rlm.rlm_mix_prefill(x, p, y, st, workspace=fw)
+        b.record(stream)
+        torch.cuda.synchronize()
+        fts.append(a.elapsed_time(b))
+    fms = statistics.mean(fts)
+    del y, st, fw
     gbs = backward_bytes(B, L, D, M) / (ms * 1e-3) / 1e9
     moved = backward_moved_bytes(B, L, D) / (ms * 1e-3) / 1e9
     return {"workload": "backward B=4 L=32768 D=512 M=32 bf16", "ms": round(ms, 4),
             "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 2), "achieved_GBps": round(gbs, 1),
             "frac_hbm": round(gbs / hbm_peak, 4),
             "data_path": "transpose to channel-major, tcgen05 kernel, transpose back, fixed-order reduction",
-            "moved_GBps": round(moved, 1), "moved_frac_hbm": round(moved / hbm_peak, 4)}
+            "moved_GBps": round(moved, 1), "moved_frac_hbm": round(moved / hbm_peak, 4),
+            "forward_ms": round(fms, 4), "forward_plus_backward_ms": round(fms + ms, 4)}
 
 
 def run_backward_only(args):
