@@ -12,9 +12,11 @@ gcc and marshals numpy arrays into it.
 Functions (all arrays float64, C-contiguous; shapes as in the paper's notation,
 channel innermost):
 
-* ``conv_prefill``   O1: direct O(L^2) causal convolution, Eq. 1-2.
-* ``rec_prefill``    O2: sequential complex recurrence, Eq. 4-5, plus the
-                      prompt's terminal state (Sec. 3.2).
+* ``conv_prefill``   O1: direct O(L^2) causal convolution, Eq. 1-2 (plus the
+                      closed-form free response of an initial state).
+* ``rec_prefill``    O2: sequential complex recurrence, Eq. 4-5, from a zero or
+                      given initial state, plus the prompt's terminal state
+                      (Sec. 3.2).
 * ``rec_decode``     one decode step, Eq. 4-5.
 * ``backward_conv``  O3 via the convolution route (chain rule through Eq. 1-2).
 * ``backward_rec``   O3 via the reverse-time Jordan recurrence.
@@ -60,8 +62,8 @@ def _load():
             L_, I_ = ctypes.c_long, ctypes.c_int
             lib.oracle_num_threads.restype = I_
             lib.oracle_kernel_table.argtypes = [I_, I_, dp, dp, dp, dp, L_, dp]
-            lib.oracle_conv_prefill.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp]
-            lib.oracle_rec_prefill.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp, dp]
+            lib.oracle_conv_prefill.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp, dp]
+            lib.oracle_rec_prefill.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp, dp, dp]
             lib.oracle_rec_decode.argtypes = [L_, I_, I_, dp, dp, dp, dp, dp, dp, dp, dp]
             lib.oracle_backward_conv.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp,
                                                  dp, dp, dp, dp, dp]
@@ -100,28 +102,45 @@ def kernel_table(decay, freq, amp, phase, L: int) -> np.ndarray:
     return K
 
 
-def conv_prefill(x, decay, freq, amp, phase) -> np.ndarray:
-    """O1: y[b,t,d] = sum_{j<=t} K_d[t-j] x[b,j,d] by direct summation (Eq. 2)."""
+def _state_pairs(state_in, B, D, M):
+    """[B][D][M] complex -> [B][D][M][2] float64 (Re, Im), or None."""
+    if state_in is None:
+        return None
+    s = np.asarray(state_in)
+    if s.shape != (B, D, M):
+        raise ValueError("state_in must be [B][D][M] complex")
+    return np.ascontiguousarray(np.stack([s.real, s.imag], -1), np.float64)
+
+
+def conv_prefill(x, decay, freq, amp, phase, state_in=None) -> np.ndarray:
+    """O1: y[b,t,d] = sum_{j<=t} K_d[t-j] x[b,j,d] by direct summation (Eq. 2), plus,
+    when state_in ([B][D][M] complex, the state before token 0) is given, its free
+    response sum_m Re(c lambda^(t+1) s) in closed form."""
     x = _f64(x)
     ps, D, M = _params(decay, freq, amp, phase)
     B, L, Dx = x.shape
     assert Dx == D
+    sin = _state_pairs(state_in, B, D, M)
     y = np.empty_like(x)
-    _load().oracle_conv_prefill(B, L, D, M, _ptr(x), *map(_ptr, ps), _ptr(y))
+    _load().oracle_conv_prefill(B, L, D, M, _ptr(x), *map(_ptr, ps),
+                                _ptr(sin) if sin is not None else None, _ptr(y))
     return y
 
 
-def rec_prefill(x, decay, freq, amp, phase):
-    """O2: sequential recurrence from a zero state (Eq. 4-5).
+def rec_prefill(x, decay, freq, amp, phase, state_in=None):
+    """O2: sequential recurrence (Eq. 4-5) from state_in ([B][D][M] complex, the
+    state before token 0), or from a zero state when it is None.
 
     Returns (y [B][L][D], state [B][D][M] complex128)."""
     x = _f64(x)
     ps, D, M = _params(decay, freq, amp, phase)
     B, L, Dx = x.shape
     assert Dx == D
+    sin = _state_pairs(state_in, B, D, M)
     y = np.empty_like(x)
     st = np.empty((B, D, M, 2), np.float64)
-    _load().oracle_rec_prefill(B, L, D, M, _ptr(x), *map(_ptr, ps), _ptr(y), _ptr(st))
+    _load().oracle_rec_prefill(B, L, D, M, _ptr(x), *map(_ptr, ps),
+                               _ptr(sin) if sin is not None else None, _ptr(y), _ptr(st))
     return y, st[..., 0] + 1j * st[..., 1]
 
 

@@ -63,10 +63,15 @@ void oracle_kernel_table(int D, int M, const double *decay, const double *freq,
 }
 
 /* O1: direct O(L^2) causal convolution with the closed-form kernel
- * (Eq. 1 and Eq. 2).  y must hold B*L*D doubles. */
+ * (Eq. 1 and Eq. 2).  y must hold B*L*D doubles.  With state_in
+ * ([B][D][M][2], the state before token 0; NULL = zero), every output also gets
+ * the free response of that state, evaluated in closed form (Eq. 5 powers):
+ * sum_m Re(c_m lambda_m^(t+1) s_m) = sum_m A |s| exp(-gamma (t+1))
+ * cos(omega (t+1) + phi + arg s). */
 void oracle_conv_prefill(long B, long L, int D, int M, const double *x,
                          const double *decay, const double *freq,
-                         const double *amp, const double *phase, double *y)
+                         const double *amp, const double *phase,
+                         const double *state_in, double *y)
 {
     double *K = (double *)malloc(sizeof(double) * (size_t)D * (size_t)L);
     oracle_kernel_table(D, M, decay, freq, amp, phase, L, K);
@@ -78,6 +83,15 @@ void oracle_conv_prefill(long B, long L, int D, int M, const double *x,
                 double acc = 0.0;
                 for (long j = 0; j <= t; ++j)
                     acc += Kd[t - j] * x[((size_t)b * L + j) * D + d];
+                if (state_in)
+                    for (int m = 0; m < M; ++m) {
+                        const size_t pm = (size_t)d * M + m;
+                        const size_t o = (((size_t)b * D + d) * M + m) * 2;
+                        const double mag = hypot(state_in[o], state_in[o + 1]);
+                        const double arg = atan2(state_in[o + 1], state_in[o]);
+                        const double n = (double)(t + 1);
+                        acc += amp[pm] * mag * exp(-decay[pm] * n) * cos(freq[pm] * n + phase[pm] + arg);
+                    }
                 y[((size_t)b * L + t) * D + d] = acc;
             }
         }
@@ -88,14 +102,16 @@ static cplx mode_lambda(double g, double w) { return exp(-g) * (cos(w) + I * sin
 static cplx mode_coef(double a, double p) { return a * (cos(p) + I * sin(p)); }
 
 /* O2: the sequential complex recurrence of Sec. 3.3 (Eq. 4-5), run over the
- * whole prompt from a zero state:  s <- lambda s + x_t,  y_t = sum_m Re(c s).
- * The state after the last token is the prompt's terminal state of Sec. 3.2
- * (the decay-weighted sum of past drives), returned as state[B][D][M][2]
- * (real, imaginary) when state is not NULL. */
+ * whole prompt:  s <- lambda s + x_t,  y_t = sum_m Re(c s), from the state
+ * state_in ([B][D][M][2], the state before token 0) or, when it is NULL, from a
+ * zero state.  The state after the last token is the prompt's terminal state of
+ * Sec. 3.2 (the decay-weighted sum of past drives), returned as
+ * state[B][D][M][2] (real, imaginary) when state is not NULL; it may alias
+ * state_in. */
 void oracle_rec_prefill(long B, long L, int D, int M, const double *x,
                         const double *decay, const double *freq,
-                        const double *amp, const double *phase, double *y,
-                        double *state)
+                        const double *amp, const double *phase,
+                        const double *state_in, double *y, double *state)
 {
 #pragma omp parallel for collapse(2) schedule(static)
     for (long b = 0; b < B; ++b)
@@ -106,14 +122,14 @@ void oracle_rec_prefill(long B, long L, int D, int M, const double *x,
                 size_t pm = (size_t)d * M + m;
                 cplx lam = mode_lambda(decay[pm], freq[pm]);
                 cplx c = mode_coef(amp[pm], phase[pm]);
-                cplx s = 0.0;
+                const size_t o = (((size_t)b * D + d) * M + m) * 2;
+                cplx s = state_in ? state_in[o] + I * state_in[o + 1] : 0.0;
                 for (long t = 0; t < L; ++t) {
                     size_t i = ((size_t)b * L + t) * D + d;
                     s = lam * s + x[i];
                     y[i] += creal(c * s);
                 }
                 if (state) {
-                    size_t o = (((size_t)b * D + d) * M + m) * 2;
                     state[o] = creal(s);
                     state[o + 1] = cimag(s);
                 }

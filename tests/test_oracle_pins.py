@@ -261,6 +261,61 @@ def _loss(x, dy, params):
     return float(np.sum(dy * oracle.conv_prefill(x, *params)))
 
 
+# ------------------------------------------------- prefill from an initial state
+def test_prefill_from_state_continues_the_sequence():
+    """Prefill of x1 || x2 from zero equals prefill of x2 started from the state
+    that x1 leaves (Sec. 3.2 terminal state carried on, Eq. 4-5)."""
+    inp = make_inputs(2, 300, 6, 5, "f32", seed=21)
+    y_all, s_all = oracle.rec_prefill(inp.x, *inp.params())
+    y1, s1 = oracle.rec_prefill(inp.x[:, :123], *inp.params())
+    y2, s2 = oracle.rec_prefill(inp.x[:, 123:], *inp.params(), state_in=s1)
+    np.testing.assert_allclose(y2, y_all[:, 123:], rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(s2, s_all, rtol=1e-11, atol=1e-12)
+
+
+def test_initial_state_routes_agree():
+    """O1 (closed-form free response added to the convolution) against O2 (the
+    recurrence started from the state): independent code."""
+    inp = make_inputs(2, 200, 5, 4, "f32", seed=22)
+    rng = np.random.default_rng(3)
+    s0 = rng.normal(size=(2, 5, 4)) + 1j * rng.normal(size=(2, 5, 4))
+    y_rec, _ = oracle.rec_prefill(inp.x, *inp.params(), state_in=s0)
+    y_conv = oracle.conv_prefill(inp.x, *inp.params(), state_in=s0)
+    np.testing.assert_allclose(y_conv, y_rec, rtol=1e-10, atol=1e-10)
+
+
+def test_free_response_hand_derived():
+    """Zero drive from s = 1: one mode with half-life 10 tokens (gamma = ln2 / 10),
+    omega = pi / 2, A = 2, phi = 0 rings as 2 * 2^(-(t+1)/10) cos(pi (t+1) / 2):
+    0, -2^0.8, 0, 2^0.6 for t = 0..3, and leaves the state 2^(-0.4)."""
+    g = np.array([[math.log(2.0) / 10.0]])
+    w = np.array([[math.pi / 2.0]])
+    a = np.array([[2.0]])
+    ph = np.array([[0.0]])
+    x = np.zeros((1, 4, 1))
+    s0 = np.ones((1, 1, 1), complex)
+    want = np.array([0.0, -2.0 ** 0.8, 0.0, 2.0 ** 0.6])
+    y, st = oracle.rec_prefill(x, g, w, a, ph, state_in=s0)
+    np.testing.assert_allclose(y[0, :, 0], want, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(st[0, 0, 0], 2.0 ** -0.4, rtol=1e-12, atol=1e-12)
+    yc = oracle.conv_prefill(x, g, w, a, ph, state_in=s0)
+    np.testing.assert_allclose(yc[0, :, 0], want, rtol=1e-12, atol=1e-12)
+
+
+def test_zero_initial_state_is_plain_prefill_and_response_is_linear():
+    inp = make_inputs(1, 150, 4, 3, "f32", seed=23)
+    y0, s0 = oracle.rec_prefill(inp.x, *inp.params())
+    z = np.zeros((1, 4, 3), complex)
+    yz, sz = oracle.rec_prefill(inp.x, *inp.params(), state_in=z)
+    assert np.array_equal(y0, yz) and np.array_equal(s0, sz)
+    rng = np.random.default_rng(4)
+    si = rng.normal(size=(1, 4, 3)) + 1j * rng.normal(size=(1, 4, 3))
+    ys, ss = oracle.rec_prefill(inp.x, *inp.params(), state_in=si)
+    yf, sf = oracle.rec_prefill(np.zeros_like(inp.x), *inp.params(), state_in=si)
+    np.testing.assert_allclose(ys, y0 + yf, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(ss, s0 + sf, rtol=1e-12, atol=1e-12)
+
+
 @pytest.mark.parametrize("seed", [41, 43])
 def test_backward_matches_central_finite_differences(seed):
     """I5: both backward routes match central differences of l = sum(dy * y)
