@@ -119,10 +119,26 @@ typedef struct {
  *   state_out  nullable; if given (state_out->B == B, D, M matching), receives
  *              the prompt's terminal state s_{L-1} = sum_j lambda^{L-1-j} x_j
  *              (Sec. 3.2) and the mode coefficients, ready for decode.
- * BF16 I/O with M == 16 runs on the tcgen05 tensor-core path; other cases run
- * the fp32 SIMT chunked scan.  Both accumulate the state in fp32. */
+ * BF16 I/O with M == 16 runs on the tcgen05 tensor-core prefill; BF16 I/O with
+ * another M <= 32 on the tcgen05 reverse-time scan of the reversed drive; other
+ * cases (fp32 I/O, M > 32) on the SIMT chunked scan.  All accumulate the state in
+ * fp32. */
 RLM_API rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor *y,
                            rlm_state *state_out, const rlm_launch *launch);
+
+/* Prefill from a given initial state (chunked or continued prefill: the terminal
+ * state of an earlier prompt, or any state decode has reached), Sec. 3.2-3.3:
+ *   s_{-1} = state_in,  s_t = lambda s_{t-1} + x_t,  y_t = sum_m Re(c_m s_t),
+ * i.e. rlm_mix_prefill's y plus the free response sum_m Re(c_m lambda_m^{t+1} s_in).
+ *   state_in   nullable (NULL = zero state, the same as rlm_mix_prefill); only
+ *              state_in->s ([B][D][M] complex fp32, 16-byte aligned) is read,
+ *              state_in->coef is ignored (p gives the coefficients).  It must
+ *              not overlap y.  state_out may be the same buffer (in-place
+ *              continuation); partial overlap is rejected.
+ * Other arguments, the workspace (rlm_prefill_workspace_size) and the paths
+ * taken are those of rlm_mix_prefill. */
+RLM_API rlm_status rlm_mix_prefill_from(const rlm_tensor *x, const rlm_params *p, const rlm_state *state_in,
+                                        rlm_tensor *y, rlm_state *state_out, const rlm_launch *launch);
 
 /* Bytes of workspace rlm_mix_prefill needs for this shape (0 is possible). */
 RLM_API size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype);

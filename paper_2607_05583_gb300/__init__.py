@@ -22,7 +22,7 @@ from . import build as _build_mod
 
 __all__ = [
     "RlmError", "Params", "Grads", "State", "load_library", "library_path",
-    "rlm_mix_prefill", "rlm_mix_prefill_noalloc", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
+    "rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_prefill_noalloc", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
     "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
     "rlm_validate_params", "rlm_get_device_status", "rlm_status_string",
     "rlm_version", "rlm_kernels_launched", "rlm_measure_row_io", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
@@ -85,6 +85,8 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
     lib = ctypes.CDLL(path)
     P = ctypes.POINTER
     lib.rlm_mix_prefill.argtypes = [P(_Tensor), P(_Params), P(_Tensor), P(_State), P(_Launch)]
+    lib.rlm_mix_prefill_from.argtypes = [P(_Tensor), P(_Params), P(_State), P(_Tensor), P(_State),
+                                         P(_Launch)]
     lib.rlm_mix_decode.argtypes = [P(_Tensor), P(_State), P(_Tensor), P(_Launch)]
     lib.rlm_mix_backward.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_Tensor),
                                      P(_Grads), P(_Launch)]
@@ -95,8 +97,8 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
         getattr(lib, f).argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
                                     ctypes.c_int, ctypes.c_int]
         getattr(lib, f).restype = ctypes.c_size_t
-    for f in ("rlm_mix_prefill", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
-              "rlm_validate_params", "rlm_get_device_status"):
+    for f in ("rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_decode", "rlm_mix_backward",
+              "rlm_state_init", "rlm_validate_params", "rlm_get_device_status"):
         getattr(lib, f).restype = ctypes.c_int
     lib.rlm_status_string.argtypes = [ctypes.c_int]
     lib.rlm_status_string.restype = ctypes.c_char_p
@@ -282,6 +284,25 @@ def rlm_mix_prefill(x: torch.Tensor, params: Params, y: torch.Tensor,
     _check(lib.rlm_mix_prefill(ctypes.byref(xt), ctypes.byref(params._c()), ctypes.byref(yt),
                                ctypes.byref(st) if st is not None else None,
                                ctypes.byref(_launch(stream, workspace))), "rlm_mix_prefill")
+
+
+def rlm_mix_prefill_from(x: torch.Tensor, params: Params, state_in: State | None, y: torch.Tensor,
+                         state_out: State | None = None, workspace: torch.Tensor | None = None,
+                         stream=None) -> None:
+    """Causal mixing from an initial state (chunked or continued prefill): y = K * x
+    plus the free response of ``state_in`` (its ``s``; None = zero state).
+    ``state_out`` may be ``state_in`` itself (in-place continuation)."""
+    lib = load_library()
+    xt, yt = _field(x), _field(y)
+    if workspace is None:
+        workspace = _workspace(lib.rlm_prefill_workspace_size(xt.B, xt.L, xt.D, params.M, xt.dtype),
+                               x.device)
+    si = state_in._c() if state_in is not None else None
+    so = state_out._c() if state_out is not None else None
+    _check(lib.rlm_mix_prefill_from(ctypes.byref(xt), ctypes.byref(params._c()),
+                                    ctypes.byref(si) if si is not None else None, ctypes.byref(yt),
+                                    ctypes.byref(so) if so is not None else None,
+                                    ctypes.byref(_launch(stream, workspace))), "rlm_mix_prefill_from")
 
 
 def rlm_mix_prefill_noalloc(x: torch.Tensor, params: Params, y: torch.Tensor,

@@ -176,6 +176,11 @@ size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype
 
 rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor *y,
                            rlm_state *state_out, const rlm_launch *ln) {
+    return rlm_mix_prefill_from(x, p, nullptr, y, state_out, ln);
+}
+
+rlm_status rlm_mix_prefill_from(const rlm_tensor *x, const rlm_params *p, const rlm_state *state_in,
+                                rlm_tensor *y, rlm_state *state_out, const rlm_launch *ln) {
     rlm_status s;
     if ((s = check_tensor(x, "x")) != RLM_OK) return s;
     if ((s = check_tensor(y, "y")) != RLM_OK) return s;
@@ -184,6 +189,19 @@ rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor 
         return fail(RLM_ERR_INVALID_ARG, "x and y overlap");
     if ((s = check_params(p, x->D)) != RLM_OK) return s;
     if (state_out && (s = check_state(state_out, x->B, x->D, p->M, "state_out")) != RLM_OK) return s;
+    const size_t sbytes = (size_t)x->B * x->D * p->M * 8;
+    if (state_in) {
+        if (!state_in->s || !aligned16(state_in->s))
+            return fail(RLM_ERR_INVALID_ARG, "state_in->s is NULL or not 16-byte aligned");
+        if (state_in->B != x->B || state_in->D != x->D || state_in->M != p->M)
+            return fail(RLM_ERR_INVALID_ARG, "state_in is [B=%d][D=%d][M=%d], expected [%lld][%lld][%d]",
+                        state_in->B, state_in->D, state_in->M, (long long)x->B, (long long)x->D, p->M);
+        if (overlap(state_in->s, sbytes, y->ptr, tensor_bytes(y)))
+            return fail(RLM_ERR_INVALID_ARG, "state_in overlaps y");
+        if (state_out && state_out->s != state_in->s && overlap(state_in->s, sbytes, state_out->s, sbytes))
+            return fail(RLM_ERR_INVALID_ARG, "state_in and state_out overlap without being the same buffer");
+    }
+    const float *sin = state_in ? state_in->s : nullptr;
     const int D = (int)x->D, M = p->M;
     const bool tc = tc_prefill_supported(x->B, x->L, D, M, x->dtype);
     const bool rev = !tc && tc_prefill_rev_supported(x->B, x->L, D, M, x->dtype);
@@ -196,14 +214,14 @@ rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor 
     float *co = state_out ? state_out->coef : nullptr;
     cudaError_t e;
     if (tc)
-        e = tc_prefill(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, so,
+        e = tc_prefill(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so,
                        co, ln->workspace, st);
     else if (rev)
-        e = tc_prefill_rev(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, so,
+        e = tc_prefill_rev(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so,
                            co, ln->workspace, st);
     else
         e = simt_prefill(x->ptr, y->ptr, x->dtype, x->B, x->L, D, M, p->decay, p->freq, p->amp,
-                         p->phase, so, co, ln->workspace, st);
+                         p->phase, sin, so, co, ln->workspace, st);
     if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_prefill launch");
     return RLM_OK;
 }

@@ -313,7 +313,9 @@ __device__ __forceinline__ void store_pair_row(uint32_t buf, int r, int g, const
 struct BwdArgs {
     const float *decay, *freq, *amp, *phase;
     float2 *part_g, *part_p;  // [B*D][M] (backward)
+    const float2 *state_in;   // nullable, [B*D][M] (time-reversed prefill: state before token 0)
     float2 *state_out;        // nullable, [B*D][M] (time-reversed prefill)
+    int64_t L;
     float4 *coef_out;         // nullable, [D][M]   (time-reversed prefill)
     __nv_bfloat16 *dxT;       // [B*D][Lp]
     int64_t Lp;
@@ -325,6 +327,10 @@ struct BwdArgs {
 // (dy = x reversed within [0, L)), which is the same reverse-time scan without the
 // parameter gradients: its output is y reversed, and the adjoint state it ends
 // with, sum_s lambda^s x_{L-1-s}, is the prompt's terminal state (Sec. 3.2).
+// A state s_in before token 0 acts from reversed position L on: lambda^(L-L')
+// s_in joins the pair entering the chunk that ends at L' = L rounded up to a
+// chunk (|lambda^(L-L')| <= exp(63 gamma)), which gives lambda^(t+1) s_in at
+// token t and lambda^L s_in in the end state; positions >= L are never stored.
 template <bool kGrad>
 __global__ void __launch_bounds__(kThreads, 2)
     k_backward_tc(const __grid_constant__ CUtensorMap tmap_dy, const __grid_constant__ CUtensorMap tmap_x,
@@ -494,6 +500,15 @@ __global__ void __launch_bounds__(kThreads, 2)
         const float2 a = lambda_pow(gamE, omgE, (float)kC);
         float2 S = make_float2(0.0f, 0.0f), R = make_float2(0.0f, 0.0f);
         const int prow = 32 * q + lane;         // this lane's [S^n ; R^n] row
+        // State before token 0 (reversed-time prefill): chunk kinj of the walk.
+        float2 inj = make_float2(0.0f, 0.0f);
+        int kinj = -1;
+        if (!kGrad && args.state_in) {
+            const int64_t Lr = (args.L + kC - 1) / kC * kC;
+            kinj = (int)(Lr / kC) - 1;
+            if (onE)
+                inj = cmul(lambda_pow(gamE, omgE, (float)(args.L - Lr)), args.state_in[(int64_t)row * M + mE]);
+        }
         bool ok = true;
         for (int v = 0; v < ntiles && ok; ++v) {
             const int bb = v & 1;
@@ -501,6 +516,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             tc_fence_after();
             if (warp == 0 && lane == 0) bar_arrive(bar(kBarSlotEmpty + v % kSlots));
             const uint32_t pb = sbase + kOffBs + bb * kBsBuf;
+            const int cinj = kinj - (last - v) * kNT;   // chunk of this tile that takes s_in, if any
 #pragma unroll
             for (int h = 1; h >= 0; --h) {   // chunks 31 .. 0
                 uint32_t pv[16];
@@ -527,6 +543,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                         const float dqr = __shfl_sync(0xffffffffu, p, base + 16);
                         const float dqi = __shfl_sync(0xffffffffu, p, base + 17);
                         // The pair entering chunk 16 h + 8 g + n from the right.
+                        if (!kGrad && 16 * h + 8 * g + n == cinj) S = make_float2(S.x + inj.x, S.y + inj.y);
                         own[n] = (s & 2) ? ((s & 1) ? R.y : R.x) : ((s & 1) ? S.y : S.x);
                         const float2 w = make_float2(fmaf((float)kC, S.x, R.x), fmaf((float)kC, S.y, R.y));
                         R = cfma(a, w, make_float2(dqr, dqi));
@@ -933,8 +950,10 @@ BwdArgs base_args(const float *decay, const float *freq, const float *amp, const
     a.phase = phase;
     a.part_g = nullptr;
     a.part_p = nullptr;
+    a.state_in = nullptr;
     a.state_out = nullptr;
     a.coef_out = nullptr;
+    a.L = 0;
     a.dxT = outT;
     a.Lp = Lp;
     a.D = D;
@@ -984,8 +1003,8 @@ bool tc_prefill_rev_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) 
 size_t tc_prefill_rev_ws_bytes(int64_t B, int64_t L, int D, int) { return 2 * field_bytes(B, L, D); }
 
 cudaError_t tc_prefill_rev(const void *x, void *y, int64_t B, int64_t L, int D, int M, const float *decay,
-                           const float *freq, const float *amp, const float *phase, float *state_out,
-                           float *coef_out, void *ws, cudaStream_t st) {
+                           const float *freq, const float *amp, const float *phase, const float *state_in,
+                           float *state_out, float *coef_out, void *ws, cudaStream_t st) {
     if (!ws) return cudaErrorInvalidValue;
     const int64_t Lp = padded_len(L);
     char *w = static_cast<char *>(ws);
@@ -1000,8 +1019,10 @@ cudaError_t tc_prefill_rev(const void *x, void *y, int64_t B, int64_t L, int D, 
     k_to_channel_major<<<dim3((unsigned)(Lp / 64), cgroups, (unsigned)B), 256, 0, st>>>(
         static_cast<const __nv_bfloat16 *>(x), nullptr, xr, nullptr, L, D, Lp, 1, 1);
     BwdArgs a = base_args(decay, freq, amp, phase, yr, Lp, D, M);
+    a.state_in = reinterpret_cast<const float2 *>(state_in);
     a.state_out = reinterpret_cast<float2 *>(state_out);
     a.coef_out = reinterpret_cast<float4 *>(coef_out);
+    a.L = L;
     k_backward_tc<false><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mx, mx, a);
     k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cgroups, (unsigned)B), 256, 0, st>>>(
         yr, static_cast<__nv_bfloat16 *>(y), L, D, Lp, 1);

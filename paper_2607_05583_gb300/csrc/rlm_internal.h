@@ -28,10 +28,12 @@ size_t simt_backward_ws_bytes(int64_t B, int64_t L, int D, int M);
 // y = causal mixing of x (reverse=false) or the anti-causal mixing used by the
 // backward pass for dx (reverse=true: time runs from L-1 down to 0).
 // state_out/coef_out may be null.  ws must hold simt_prefill_ws_bytes().
+// state_in ([B][D][M] complex, the state before token 0), state_out and
+// coef_out may be null; state_out may alias state_in.
 cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_t L, int D,
                          int M, const float *decay, const float *freq, const float *amp,
-                         const float *phase, float *state_out, float *coef_out, void *ws,
-                         cudaStream_t st);
+                         const float *phase, const float *state_in, float *state_out, float *coef_out,
+                         void *ws, cudaStream_t st);
 
 // dx and the four parameter gradients (deterministic reduction).
 cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt, int64_t B,
@@ -60,8 +62,8 @@ cudaError_t read_and_clear_bwd_status(int *status, cudaStream_t st);
 bool tc_prefill_rev_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
 size_t tc_prefill_rev_ws_bytes(int64_t B, int64_t L, int D, int M);
 cudaError_t tc_prefill_rev(const void *x, void *y, int64_t B, int64_t L, int D, int M, const float *decay,
-                           const float *freq, const float *amp, const float *phase, float *state_out,
-                           float *coef_out, void *ws, cudaStream_t st);
+                           const float *freq, const float *amp, const float *phase, const float *state_in,
+                           float *state_out, float *coef_out, void *ws, cudaStream_t st);
 
 // ---- decode (rlm_decode.cu) -----------------------------------------------
 cudaError_t decode_step(const void *x_t, void *y_t, rlm_dtype dt, int B, int D, int M,
@@ -76,8 +78,8 @@ bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
 size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int M);
 cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int M,
                        const float *decay, const float *freq, const float *amp,
-                       const float *phase, float *state_out, float *coef_out, void *ws,
-                       cudaStream_t st);
+                       const float *phase, const float *state_in, float *state_out, float *coef_out,
+                       void *ws, cudaStream_t st);
 // Device status word written by bounded waits (RLM_OK or RLM_ERR_TIMEOUT).
 cudaError_t read_and_clear_device_status(int *status, cudaStream_t st);
 

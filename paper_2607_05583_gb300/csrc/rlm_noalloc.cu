@@ -112,7 +112,7 @@ extern "C" rlm_status rlm_mix_prefill_noalloc(const rlm_tensor *x, const rlm_par
     if (e != cudaSuccess)
         return reject(RLM_ERR_CUDA, "rlm_mix_prefill_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
     e = simt_prefill(x->ptr, y->ptr, x->dtype, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase,
-                     state_out ? state_out->s : nullptr, state_out ? state_out->coef : nullptr, scratch,
+                     nullptr, state_out ? state_out->s : nullptr, state_out ? state_out->coef : nullptr, scratch,
                      static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess)
         return reject(RLM_ERR_CUDA, "rlm_mix_prefill_noalloc launch: %s", cudaGetErrorString(e));

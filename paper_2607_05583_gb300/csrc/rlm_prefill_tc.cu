@@ -347,6 +347,7 @@ __device__ __forceinline__ int au_operand(int c) { return au_slot(c) * kAuStride
 
 struct TcArgs {
     const float *decay, *freq, *amp, *phase;
+    const float2 *state_in;  // [B][D][M], the state before token 0 (kInj instances only)
     float2 *state_out;   // nullable, [B][D][M]
     float4 *coef_out;    // nullable, [D][M]
     __nv_bfloat16 *y;    // for the plain stores of boxes that start before t = 0
@@ -364,7 +365,12 @@ struct TcArgs {
 // kSeg: the grid's z dimension splits the sequence into segments.  The
 // unsegmented instance keeps the tile count a kernel parameter (no register
 // holds it), which the per-tile loops' register allocation depends on.
-template <bool kSeg>
+// kInj: the prefill starts from args.state_in instead of zero.  Token 0 sits at
+// position p of chunk n0 of tile 0 (tiles end at L - 1); lambda^-p s_in is added
+// to the state entering chunk n0, which gives lambda^(i+1-p) s_in at its positions
+// i >= p (those before p are negative times, never stored) and lambda^(64-p) s_in
+// carried on.  |lambda^-p| <= exp(63 gamma) stays bounded.
+template <bool kSeg, bool kInj>
 __global__ void __launch_bounds__(kThreads, 1)
     k_prefill_tc(const __grid_constant__ CUtensorMap tmap_x,
                  const __grid_constant__ CUtensorMap tmap_y, const TcArgs args) {
@@ -716,10 +722,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int pm = (d0 + ch) * kModes + m;
         const float2 LC = lambda_pow(args.decay[pm], args.freq[pm], (float)kC);
         float2 S = make_float2(0.0f, 0.0f);
+        float2 inj = make_float2(0.0f, 0.0f);
+        int n0 = -1;
+        if (kInj) {
+            n0 = (int)((-args.t0) >> 6);
+            const int p = (int)((-args.t0) & 63);
+            inj = cmul(lambda_pow(args.decay[pm], args.freq[pm], (float)(-p)),
+                       args.state_in[((int64_t)b * D + d0 + ch) * kModes + m]);
+        }
         uint8_t *bs = smem + kOffBs + ch * kBsStride + (m / 4) * kBsLbo + (m % 4) * 4;
         const int64_t seg_row = (int64_t)b * args.nseg;
         // One tile of the carry: S_n = lambda^C S_{n-1} + L_n over its 32 chunks.
         auto scan_tile = [&](int v) -> bool {
+            const bool inj_tile = kInj && real_tile(v) == 0;
             if (!wait_bar(bar(kBarTwDone + cA), v & 1, abort_flag)) return false;
             if (!wait_bar(bar(kBarTwDone + cB), v & 1, abort_flag)) return false;
             tc_fence_after();
@@ -735,6 +750,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float recv = __shfl_xor_sync(0xffffffffu, ri ? a : bb, 1);
                     const float2 Ln = ri ? make_float2(recv, bb) : make_float2(a, recv);
                     const int nn = 16 * h + n;
+                    if (kInj && inj_tile && nn == n0) S = make_float2(S.x + inj.x, S.y + inj.y);
                     *reinterpret_cast<uint32_t *>(bs + (nn >> 3) * kBsSbo + (nn & 7) * 16) = pack_bf16x2(S.x, S.y);
                     S = cfma(LC, S, Ln);
                 }
@@ -919,8 +935,8 @@ size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int) {
 
 cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int M,
                        const float *decay, const float *freq, const float *amp,
-                       const float *phase, float *state_out, float *coef_out, void *ws,
-                       cudaStream_t st) {
+                       const float *phase, const float *state_in, float *state_out, float *coef_out,
+                       void *ws, cudaStream_t st) {
     (void)M;
     CUtensorMap mx, my;
     if (!make_field_map(&mx, x, B, L, D) || !make_field_map(&my, y, B, L, D))
@@ -933,10 +949,16 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
         std::lock_guard<std::mutex> lock(mu);
         if ((int)configured.size() <= dev) configured.resize(dev + 1, 0);
         if (!configured[dev]) {
-            cudaError_t e = cudaFuncSetAttribute(k_prefill_tc<false>,
+            cudaError_t e = cudaFuncSetAttribute(k_prefill_tc<false, false>,
                                                  cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
             if (e == cudaSuccess)
-                e = cudaFuncSetAttribute(k_prefill_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                e = cudaFuncSetAttribute(k_prefill_tc<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSmemBytes);
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(k_prefill_tc<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         kSmemBytes);
+            if (e == cudaSuccess)
+                e = cudaFuncSetAttribute(k_prefill_tc<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          kSmemBytes);
             if (e != cudaSuccess) return e;
             configured[dev] = 1;
@@ -947,6 +969,7 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.freq = freq;
     a.amp = amp;
     a.phase = phase;
+    a.state_in = reinterpret_cast<const float2 *>(state_in);
     a.state_out = reinterpret_cast<float2 *>(state_out);
     a.coef_out = reinterpret_cast<float4 *>(coef_out);
     a.y = static_cast<__nv_bfloat16 *>(y);
@@ -962,7 +985,10 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.epoch = 0;
     dim3 grid((unsigned)(D / kDG), (unsigned)B, (unsigned)sg.nseg);
     if (sg.nseg < 2) {
-        k_prefill_tc<false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, a);
+        if (state_in)
+            k_prefill_tc<false, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, a);
+        else
+            k_prefill_tc<false, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, a);
         count_launches(1);
         return cudaGetLastError();
     }
@@ -976,8 +1002,9 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     static std::atomic<unsigned long long> epoch{0x5eed0000ull};
     a.epoch = ++epoch;
     void *kargs[] = {&mx, &my, &a};
-    cudaError_t e = cudaLaunchCooperativeKernel(reinterpret_cast<const void *>(k_prefill_tc<true>), grid, dim3(kThreads), kargs,
-                                    (size_t)kSmemBytes, st);
+    const void *fn = state_in ? reinterpret_cast<const void *>(k_prefill_tc<true, true>)
+                              : reinterpret_cast<const void *>(k_prefill_tc<true, false>);
+    cudaError_t e = cudaLaunchCooperativeKernel(fn, grid, dim3(kThreads), kargs, (size_t)kSmemBytes, st);
     count_launches(1);
     return e;
 }

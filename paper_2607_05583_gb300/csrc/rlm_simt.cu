@@ -116,12 +116,15 @@ __global__ void __launch_bounds__(kBlock) k_chunk_local(
 }
 
 // Phase 2.  One thread per (b, d, m); grid over B*D*M.
+// With state_in (forward only): chunk 0 is entered with the state before token 0
+// (the output phase restarts its recurrence there, at time 0), and that state
+// reaches the end of chunk 0 after C + t0 tokens.
 template <bool JORDAN>
 __global__ void __launch_bounds__(256) k_chunk_carry(
-    int64_t B, int D, int M, int C, int nch, const float *__restrict__ decay,
+    int64_t B, int D, int M, int C, int nch, int64_t t0, const float *__restrict__ decay,
     const float *__restrict__ freq, const float *__restrict__ amp, const float *__restrict__ phase,
-    float2 *__restrict__ ws_s, float2 *__restrict__ ws_r, float2 *__restrict__ state_out,
-    float4 *__restrict__ coef_out) {
+    float2 *__restrict__ ws_s, float2 *__restrict__ ws_r, const float2 *__restrict__ state_in,
+    float2 *__restrict__ state_out, float4 *__restrict__ coef_out) {
     const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= B * D * M) return;
     const int m = (int)(idx % M);
@@ -130,7 +133,8 @@ __global__ void __launch_bounds__(256) k_chunk_carry(
     const int pm = d * M + m;
     const float2 LC = lambda_pow(decay[pm], freq[pm], (float)C);
     const float Cf = (float)C;
-    float2 S = make_float2(0, 0), R = make_float2(0, 0);
+    float2 S = state_in ? state_in[idx] : make_float2(0, 0), R = make_float2(0, 0);
+    const float2 L0 = state_in ? lambda_pow(decay[pm], freq[pm], (float)(C + t0)) : LC;
     for (int k = 0; k < nch; ++k) {
         const int64_t off = ((b * nch + k) * D + d) * M + m;
         const float2 ls = ws_s[off];
@@ -140,7 +144,7 @@ __global__ void __launch_bounds__(256) k_chunk_carry(
             ws_r[off] = R;
             R = cfma(LC, make_float2(fmaf(Cf, S.x, R.x), fmaf(Cf, S.y, R.y)), lr);
         }
-        S = cfma(LC, S, ls);
+        S = cfma(k == 0 ? L0 : LC, S, ls);
     }
     if (state_out) state_out[idx] = S;
     if (coef_out && b == 0) {
@@ -282,8 +286,8 @@ __global__ void __launch_bounds__(256) k_grad_reduce(
 
 template <typename T>
 cudaError_t prefill_t(const T *x, T *y, int64_t B, int64_t L, int D, int M, const float *decay,
-                      const float *freq, const float *amp, const float *phase, float *state_out,
-                      float *coef_out, void *ws, cudaStream_t st) {
+                      const float *freq, const float *amp, const float *phase, const float *state_in,
+                      float *state_out, float *coef_out, void *ws, cudaStream_t st) {
     const ChunkGeom g = geom(B, L, D);
     const int tpc = threads_per_channel(M, kMgFwd);
     float2 *ws_s = reinterpret_cast<float2 *>(ws);
@@ -292,8 +296,9 @@ cudaError_t prefill_t(const T *x, T *y, int64_t B, int64_t L, int D, int M, cons
         x, L, D, M, tpc, g.C, g.nch, g.t0, decay, freq, ws_s, nullptr);
     const int64_t n = B * D * M;
     k_chunk_carry<false><<<(unsigned)((n + 255) / 256), 256, 0, st>>>(
-        B, D, M, g.C, g.nch, decay, freq, amp, phase, ws_s, nullptr,
-        reinterpret_cast<float2 *>(state_out), reinterpret_cast<float4 *>(coef_out));
+        B, D, M, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, nullptr,
+        reinterpret_cast<const float2 *>(state_in), reinterpret_cast<float2 *>(state_out),
+        reinterpret_cast<float4 *>(coef_out));
     k_chunk_output<T, kMgFwd, false><<<grid, kBlock, 0, st>>>(
         x, y, L, D, M, tpc, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s);
     count_launches(3);
@@ -315,7 +320,7 @@ cudaError_t backward_t(const T *dy, const T *x, T *dx, int64_t B, int64_t L, int
         dy, L, D, M, tpc1, g.C, g.nch, g.t0, decay, freq, ws_s, ws_r);
     const int64_t nbdm = B * D * M;
     k_chunk_carry<true><<<(unsigned)((nbdm + 255) / 256), 256, 0, st>>>(
-        B, D, M, g.C, g.nch, decay, freq, amp, phase, ws_s, ws_r, nullptr, nullptr);
+        B, D, M, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, ws_r, nullptr, nullptr, nullptr);
     const int tpc3 = threads_per_channel(M, kMgBwd);
     dim3 grid3((unsigned)((D * tpc3 + kBlock - 1) / kBlock), (unsigned)g.nch, (unsigned)B);
     k_chunk_backward<T, kMgBwd><<<grid3, kBlock, 0, st>>>(
@@ -352,13 +357,13 @@ size_t simt_backward_ws_bytes(int64_t B, int64_t L, int D, int M) {
 
 cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_t L, int D,
                          int M, const float *decay, const float *freq, const float *amp,
-                         const float *phase, float *state_out, float *coef_out, void *ws,
-                         cudaStream_t st) {
+                         const float *phase, const float *state_in, float *state_out, float *coef_out,
+                         void *ws, cudaStream_t st) {
     if (dt == RLM_BF16)
         return prefill_t(static_cast<const __nv_bfloat16 *>(x), static_cast<__nv_bfloat16 *>(y),
-                         B, L, D, M, decay, freq, amp, phase, state_out, coef_out, ws, st);
+                         B, L, D, M, decay, freq, amp, phase, state_in, state_out, coef_out, ws, st);
     return prefill_t(static_cast<const float *>(x), static_cast<float *>(y), B, L, D, M, decay,
-                     freq, amp, phase, state_out, coef_out, ws, st);
+                     freq, amp, phase, state_in, state_out, coef_out, ws, st);
 }
 
 cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const float *phase,

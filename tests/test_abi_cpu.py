@@ -31,7 +31,7 @@ def _declared_entry_points():
 
 def test_header_declares_the_boundary():
     names = _declared_entry_points()
-    for want in ("rlm_mix_prefill", "rlm_mix_decode", "rlm_mix_backward",
+    for want in ("rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_decode", "rlm_mix_backward",
                  "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
                  "rlm_state_init", "rlm_validate_params", "rlm_get_device_status",
                  "rlm_status_string", "rlm_last_error"):
@@ -120,6 +120,31 @@ def test_prefill_rejects_bad_arguments_on_host(lib, case):
     status = _prefill(lib, x, p, y, st, ln)
     assert status == rlm.RLM_ERR_INVALID_ARG, (case, lib.rlm_last_error())
     assert lib.rlm_last_error().decode()
+
+
+def test_prefill_from_rejects_bad_initial_states_on_host(lib):
+    B, L, D, M = 2, 100, 64, 16
+    x = _t(FAKE, B, L, D)
+    y = _t(FAKE + (1 << 30), B, L, D)
+    p = _p(D, M)
+    ln = _launch(FAKE + (1 << 34), 1 << 40)
+    sbase = FAKE + (1 << 36)
+
+    def call(si, so=None):
+        return lib.rlm_mix_prefill_from(ctypes.byref(x), ctypes.byref(p),
+                                        ctypes.byref(si) if si else None, ctypes.byref(y),
+                                        ctypes.byref(so) if so else None, ctypes.byref(ln))
+
+    def state(ptr, b=B, d=D, m=M, coef=0):
+        return rlm._State(ptr, coef, b, d, m)
+
+    assert call(state(0)) == rlm.RLM_ERR_INVALID_ARG                      # NULL s
+    assert call(state(sbase + 8)) == rlm.RLM_ERR_INVALID_ARG              # misaligned s
+    assert call(state(sbase, b=B + 1)) == rlm.RLM_ERR_INVALID_ARG         # batch mismatch
+    assert call(state(sbase, m=M - 1)) == rlm.RLM_ERR_INVALID_ARG         # mode mismatch
+    assert call(state(y.ptr)) == rlm.RLM_ERR_INVALID_ARG                  # overlaps y
+    so = state(sbase + 256, coef=sbase + (1 << 24))                       # partial overlap
+    assert call(state(sbase), so) == rlm.RLM_ERR_INVALID_ARG
 
 
 def test_decode_rejects_bad_arguments_on_host(lib):

@@ -138,6 +138,78 @@ def test_time_reversed_prefill_is_causal_bit_exact():
     assert not torch.equal(a[:, 2999:], b[:, 2999:])
 
 
+def _state_from(inp, s_np):
+    st = rlm.State.empty(inp.B, inp.D, inp.M)
+    st.s.copy_(torch.from_numpy(np.stack([s_np.real, s_np.imag], -1).astype(np.float32)))
+    return st
+
+
+@pytest.mark.parametrize("B,L,D,M,dtype", [
+    (2, 2048 * 2, 64, 16, "bf16"),        # tcgen05 prefill, token 0 at a tile start
+    (8, 5000, 256, 16, "bf16"),           # ... token 0 inside the first tile (ragged)
+    (1, 3000, 16, 16, "bf16"),            # ... segmented sequence, ragged
+    (3, 2048 + 77, 128, 16, "bf16"),      # ... segmented, several rows
+    (2, 1000, 8, 32, "bf16"),             # time-reversed scan, L not a chunk multiple
+    (1, 4096, 16, 7, "bf16"),             # time-reversed scan, L a chunk multiple
+    (2, 1000, 16, 7, "f32"),              # SIMT
+    (1, 500, 8, 40, "bf16"),              # SIMT, bf16 with M > 32
+])
+def test_prefill_from_initial_state_matches_oracle(B, L, D, M, dtype):
+    """Prefill started from a state (chunked / continued prefill) against the
+    oracle's recurrence from the same state; the state is one a 300-token
+    prompt leaves, so its size is that of real use."""
+    inp = make_inputs(B, L, D, M, dtype, seed=L + 7 * M)
+    pre = make_inputs(B, 300, D, M, dtype, seed=1 + M)
+    _, s_in = oracle.rec_prefill(pre.x, *inp.params())
+    x = to_dev(inp.x, dtype)
+    p = rlm.Params.from_arrays(*inp.params())
+    y = torch.empty_like(x)
+    si = _state_from(inp, s_in)
+    so = rlm.State.empty(B, D, M)
+    rlm.rlm_mix_prefill_from(x, p, si, y, so)
+    torch.cuda.synchronize()
+    ref, st_ref = oracle.rec_prefill(inp.x, *inp.params(), state_in=s_in)
+    assert_close(to_np(y), ref, TOL[dtype], "y")
+    _state_err(so, st_ref, TOL[dtype])
+
+
+@pytest.mark.parametrize("M", [16, 32])
+def test_split_prefill_with_in_place_state_equals_whole_prefill(M):
+    """Prefill of x1 then prefill_from(x2) with state_out = state_in (in place)
+    equals one prefill of x1 || x2 (bf16, ragged split)."""
+    inp = make_inputs(2, 6000, 64, M, "bf16", seed=31)
+    x = to_dev(inp.x, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    y_all = torch.empty_like(x)
+    st_all = rlm.State.empty(2, 64, M)
+    rlm.rlm_mix_prefill(x, p, y_all, st_all)
+    x1, x2 = x[:, :2345].contiguous(), x[:, 2345:].contiguous()
+    y1, y2 = torch.empty_like(x1), torch.empty_like(x2)
+    st = rlm.State.empty(2, 64, M)
+    rlm.rlm_mix_prefill(x1, p, y1, st)
+    rlm.rlm_mix_prefill_from(x2, p, st, y2, st)
+    torch.cuda.synchronize()
+    ref, st_ref = oracle.rec_prefill(inp.x, *inp.params())
+    assert_close(to_np(y2), ref[:, 2345:], TOL["bf16"], "y of the continuation")
+    assert_close(to_np(torch.cat([y1, y2], 1)), to_np(y_all), TOL["bf16"], "split vs whole")
+    _state_err(st, st_ref, TOL["bf16"])
+
+
+def test_prefill_from_zero_state_equals_prefill():
+    inp = make_inputs(2, 3000, 64, 16, "bf16", seed=33)
+    x = to_dev(inp.x, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    y0, y1 = torch.empty_like(x), torch.empty_like(x)
+    rlm.rlm_mix_prefill(x, p, y0)
+    z = rlm.State.empty(2, 64, 16)
+    z.s.zero_()
+    rlm.rlm_mix_prefill_from(x, p, z, y1)
+    y2 = torch.empty_like(x)
+    rlm.rlm_mix_prefill_from(x, p, None, y2)
+    torch.cuda.synchronize()
+    assert torch.equal(y0, y1) and torch.equal(y0, y2)
+
+
 def test_prefill_is_causal_bit_exact():
     """I6: perturbing x[t >= t0] leaves y[t < t0] bit-identical on the GPU."""
     for dtype in ("bf16", "f32"):
