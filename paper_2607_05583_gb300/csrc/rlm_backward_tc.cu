@@ -65,6 +65,7 @@
 // their loops, drain what they issued, and the CTA frees its TMEM and returns.
 #include <cuda.h>
 
+#include <algorithm>
 #include <mutex>
 #include <vector>
 
@@ -210,14 +211,6 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map
         "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
         : "memory");
 }
-__device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, uint32_t src, int c0, int c1,
-                                             int c2) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
-            reinterpret_cast<uint64_t>(map)),
-        "r"(c0), "r"(c1), "r"(c2), "r"(src)
-        : "memory");
-}
 
 // UMMA shared-memory descriptors (bit 46: descriptor version; bits 61-63: layout).
 // No swizzle, K-major: LBO = byte distance of core matrices adjacent along K,
@@ -254,12 +247,6 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
           "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
           "=r"(v[14]), "=r"(v[15])
         : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&v)[8]) {
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                 : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]),
-                   "=r"(v[6]), "=r"(v[7])
-                 : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
@@ -316,6 +303,7 @@ struct BwdArgs {
     const float2 *state_in;   // nullable, [B*D][M] (time-reversed prefill: state before token 0)
     float2 *state_out;        // nullable, [B*D][M] (time-reversed prefill)
     int64_t L;
+    int row0;                 // first (b * D + d) row of this launch (0: the whole problem)
     float4 *coef_out;         // nullable, [D][M]   (time-reversed prefill)
     __nv_bfloat16 *dxT;       // [B*D][Lp]
     int64_t Lp;
@@ -339,7 +327,7 @@ __global__ void __launch_bounds__(kThreads, 2)
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const uint32_t sbase = smem_u32(smem);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int row = blockIdx.x;                 // b * D + d
+    const int row = args.row0 + blockIdx.x;     // b * D + d
     const int d = row % args.D;
     const int M = args.M, ntiles = args.ntiles;
     const int w_prod = 6;
@@ -778,26 +766,27 @@ __global__ void __launch_bounds__(kThreads, 2)
 }
 
 // ------------------------------------------------------------ layout transposes
-// [B][L][D] -> [B*D][Lp], zero for positions >= L.  Grid z = B * nf: field f of
-// batch row b is (src0, dst0) or (src1, dst1).  rev: position s holds token
-// L - 1 - s (time reversed within [0, L)).
-__global__ void __launch_bounds__(256) k_to_channel_major(const __nv_bfloat16 *__restrict__ src0,
+// [B][L][D] -> [B*D][Lp], zero for positions >= L.  Grid z = rows * nf: field f of
+// batch row b0 + z / nf is (src0, dst0) or (src1, dst1); channels from c_lo, below
+// c_hi.  rev: position s holds token L - 1 - s (time reversed within [0, L)).
+__global__ void __launch_bounds__(128) k_to_channel_major(const __nv_bfloat16 *__restrict__ src0,
                                                           const __nv_bfloat16 *__restrict__ src1,
                                                           __nv_bfloat16 *__restrict__ dst0,
                                                           __nv_bfloat16 *__restrict__ dst1, int64_t L, int D,
-                                                          int64_t Lp, int nf, int rev) {
+                                                          int64_t Lp, int nf, int rev, int b0, int c_lo,
+                                                          int c_hi) {
     __shared__ uint32_t tile[64][33];   // [position][channel pair]
     const int64_t t0 = (int64_t)blockIdx.x * 64;
-    const int c0 = blockIdx.y * 64;
-    const int b = blockIdx.z / nf, f = blockIdx.z % nf;
+    const int c0 = c_lo + blockIdx.y * 64;
+    const int b = b0 + blockIdx.z / nf, f = blockIdx.z % nf;
     const __nv_bfloat16 *src = f ? src1 : src0;
     __nv_bfloat16 *dst = f ? dst1 : dst0;
-    for (int it = threadIdx.x; it < 512; it += 256) {
+    for (int it = threadIdx.x; it < 512; it += 128) {
         const int r = it >> 3, vq = it & 7;
         const int64_t sp = t0 + r;
         const int c = c0 + 8 * vq;
         uint4 val = make_uint4(0, 0, 0, 0);
-        if (sp < L && c < D) {
+        if (sp < L && c < c_hi) {
             const int64_t t = rev ? L - 1 - sp : sp;
             val = __ldg(reinterpret_cast<const uint4 *>(src + ((int64_t)b * L + t) * D + c));
         }
@@ -807,10 +796,10 @@ __global__ void __launch_bounds__(256) k_to_channel_major(const __nv_bfloat16 *_
         tile[r][4 * vq + 3] = val.w;
     }
     __syncthreads();
-    for (int it = threadIdx.x; it < 512; it += 256) {
+    for (int it = threadIdx.x; it < 512; it += 128) {
         const int cr = it >> 3, vq = it & 7;
         const int c = c0 + cr;
-        if (c >= D) continue;
+        if (c >= c_hi) continue;
         uint32_t w[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -826,21 +815,21 @@ __global__ void __launch_bounds__(256) k_to_channel_major(const __nv_bfloat16 *_
 // [B*D][Lp] -> [B][L][D] for tokens t < L, token t read from position t, or from
 // L - 1 - t when rev.  A tile covers 64 tokens x 64 channels; it loads the
 // 8-aligned window of 72 positions that holds its (reversed) positions.
-__global__ void __launch_bounds__(256) k_to_row_major(const __nv_bfloat16 *__restrict__ srcT,
+__global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__restrict__ srcT,
                                                       __nv_bfloat16 *__restrict__ dst, int64_t L, int D,
-                                                      int64_t Lp, int rev) {
+                                                      int64_t Lp, int rev, int b0, int c_lo, int c_hi) {
     __shared__ uint32_t tile[64][37];   // [channel][position pair]
     const int64_t t0 = (int64_t)blockIdx.x * 64;
-    const int c0 = blockIdx.y * 64;
-    const int b = blockIdx.z;
+    const int c0 = c_lo + blockIdx.y * 64;
+    const int b = b0 + blockIdx.z;
     // First position of the window: t0 itself, or the last 64 tokens' mirror rounded down.
     const int64_t s_lo = rev ? ((L - t0 - 64) >= 0 ? (L - t0 - 64) & ~(int64_t)7 : -((t0 + 64 - L + 7) & ~(int64_t)7)) : t0;
-    for (int it = threadIdx.x; it < 64 * 9; it += 256) {
+    for (int it = threadIdx.x; it < 64 * 9; it += 128) {
         const int cr = it / 9, vq = it % 9;
         const int c = c0 + cr;
         const int64_t sp = s_lo + 8 * vq;
         uint4 val = make_uint4(0, 0, 0, 0);
-        if (c < D && sp >= 0 && sp < Lp)
+        if (c < c_hi && sp >= 0 && sp < Lp)
             val = __ldg(reinterpret_cast<const uint4 *>(srcT + ((int64_t)b * D + c) * Lp + sp));
         tile[cr][4 * vq] = val.x;
         tile[cr][4 * vq + 1] = val.y;
@@ -848,11 +837,11 @@ __global__ void __launch_bounds__(256) k_to_row_major(const __nv_bfloat16 *__res
         tile[cr][4 * vq + 3] = val.w;
     }
     __syncthreads();
-    for (int it = threadIdx.x; it < 512; it += 256) {
+    for (int it = threadIdx.x; it < 512; it += 128) {
         const int r = it >> 3, vq = it & 7;
         const int64_t t = t0 + r;
         const int c = c0 + 8 * vq;
-        if (t >= L || c >= D) continue;
+        if (t >= L || c >= c_hi) continue;
         const int i = (int)((rev ? L - 1 - t : t) - s_lo);   // 0 <= i < 72
         uint32_t w[4];
 #pragma unroll
@@ -953,13 +942,35 @@ BwdArgs base_args(const float *decay, const float *freq, const float *amp, const
     a.state_in = nullptr;
     a.state_out = nullptr;
     a.coef_out = nullptr;
-    a.L = 0;
     a.dxT = outT;
     a.Lp = Lp;
     a.D = D;
     a.M = M;
     a.ntiles = (int)(Lp / kTile);
+    a.L = 0;
+    a.row0 = 0;
     return a;
+}
+
+// One call: transpose in (nf fields: x, or x and dy), the tcgen05 kernel, transpose
+// out, in stream order.  (Running the transposes of one part of the problem beside
+// the tcgen05 kernel of another gained nothing: beside two tcgen05 CTAs an SM has
+// room for one 128-thread transpose block, too few loads in flight to use the
+// DRAM bandwidth the tcgen05 kernel leaves.)
+template <bool kGrad>
+cudaError_t run_layout_and_scan(const CUtensorMap &mdy, const CUtensorMap &mx, BwdArgs a, int64_t B, int64_t L,
+                                int D, int64_t Lp, const __nv_bfloat16 *src0, const __nv_bfloat16 *src1,
+                                __nv_bfloat16 *dst0, __nv_bfloat16 *dst1, int nf, int rev,
+                                const __nv_bfloat16 *outT, __nv_bfloat16 *out, cudaStream_t st) {
+    const unsigned cg = (unsigned)((D + 63) / 64);
+    k_to_channel_major<<<dim3((unsigned)(Lp / 64), cg, (unsigned)(B * nf)), 128, 0, st>>>(
+        src0, src1, dst0, dst1, L, D, Lp, nf, rev, 0, 0, D);
+    a.row0 = 0;
+    k_backward_tc<kGrad><<<(unsigned)(B * D), kThreads, kSmemBytes, st>>>(mdy, mx, a);
+    k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(outT, out, L, D, Lp, rev, 0,
+                                                                                     0, D);
+    count_launches(3);
+    return cudaGetLastError();
 }
 
 }  // namespace
@@ -981,17 +992,12 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     if (!make_chunk_map(&mdy, dyT, rows, Lp) || !make_chunk_map(&mx, xT, rows, Lp)) return cudaErrorInvalidValue;
     cudaError_t e = configure_once();
     if (e != cudaSuccess) return e;
-    const unsigned cgroups = (unsigned)((D + 63) / 64);
-    k_to_channel_major<<<dim3((unsigned)(Lp / 64), cgroups, (unsigned)(2 * B)), 256, 0, st>>>(
-        static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp, 2, 0);
     BwdArgs a = base_args(decay, freq, amp, phase, dxT, Lp, D, M);
     a.part_g = pg;
     a.part_p = pp;
-    k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a);
-    k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cgroups, (unsigned)B), 256, 0, st>>>(
-        dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp, 0);
-    count_launches(3);
-    e = cudaGetLastError();
+    e = run_layout_and_scan<true>(mdy, mx, a, B, L, D, Lp, static_cast<const __nv_bfloat16 *>(x),
+                         static_cast<const __nv_bfloat16 *>(dy), xT, dyT, 2, 0, dxT,
+                         static_cast<__nv_bfloat16 *>(dx), st);
     if (e != cudaSuccess) return e;
     return grad_reduce(rows / D, D, M, amp, phase, pg, pp, g_decay, g_freq, g_amp, g_phase, st);
 }
@@ -1015,19 +1021,13 @@ cudaError_t tc_prefill_rev(const void *x, void *y, int64_t B, int64_t L, int D, 
     if (!make_chunk_map(&mx, xr, rows, Lp)) return cudaErrorInvalidValue;
     cudaError_t e = configure_once();
     if (e != cudaSuccess) return e;
-    const unsigned cgroups = (unsigned)((D + 63) / 64);
-    k_to_channel_major<<<dim3((unsigned)(Lp / 64), cgroups, (unsigned)B), 256, 0, st>>>(
-        static_cast<const __nv_bfloat16 *>(x), nullptr, xr, nullptr, L, D, Lp, 1, 1);
     BwdArgs a = base_args(decay, freq, amp, phase, yr, Lp, D, M);
     a.state_in = reinterpret_cast<const float2 *>(state_in);
     a.state_out = reinterpret_cast<float2 *>(state_out);
     a.coef_out = reinterpret_cast<float4 *>(coef_out);
     a.L = L;
-    k_backward_tc<false><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mx, mx, a);
-    k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cgroups, (unsigned)B), 256, 0, st>>>(
-        yr, static_cast<__nv_bfloat16 *>(y), L, D, Lp, 1);
-    count_launches(3);
-    return cudaGetLastError();
+    return run_layout_and_scan<false>(mx, mx, a, B, L, D, Lp, static_cast<const __nv_bfloat16 *>(x), nullptr, xr, nullptr,
+                             1, 1, yr, static_cast<__nv_bfloat16 *>(y), st);
 }
 
 cudaError_t read_and_clear_bwd_status(int *status, cudaStream_t st) {
