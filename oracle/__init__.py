@@ -66,9 +66,9 @@ def _load():
             lib.oracle_rec_prefill.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp, dp, dp]
             lib.oracle_rec_decode.argtypes = [L_, I_, I_, dp, dp, dp, dp, dp, dp, dp, dp]
             lib.oracle_backward_conv.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp,
-                                                 dp, dp, dp, dp, dp]
+                                                 dp, dp, dp, dp, dp, dp, dp, dp]
             lib.oracle_backward_rec.argtypes = [L_, L_, I_, I_, dp, dp, dp, dp, dp, dp,
-                                                dp, dp, dp, dp, dp]
+                                                dp, dp, dp, dp, dp, dp, dp, dp]
             _lib = lib
     return _lib
 
@@ -160,22 +160,36 @@ def rec_decode(state, x_t, decay, freq, amp, phase):
     return y, sout[..., 0] + 1j * sout[..., 1]
 
 
-def _backward(fn, x, dy, decay, freq, amp, phase):
+def _backward(fn, x, dy, decay, freq, amp, phase, state_in=None, d_state_out=None):
     x, dy = _f64(x), _f64(dy)
     ps, D, M = _params(decay, freq, amp, phase)
     B, L, Dx = x.shape
     assert Dx == D and dy.shape == x.shape
+    sin = _state_pairs(state_in, B, D, M)
+    gout = _state_pairs(d_state_out, B, D, M)
+    want_ds = state_in is not None or d_state_out is not None
+    ds = np.empty((B, D, M, 2), np.float64) if want_ds else None
     dx = np.empty_like(x)
     g = [np.empty((D, M), np.float64) for _ in range(4)]
-    fn(B, L, D, M, _ptr(x), _ptr(dy), *map(_ptr, ps), _ptr(dx), *map(_ptr, g))
-    return dx, {"decay": g[0], "freq": g[1], "amp": g[2], "phase": g[3]}
+    opt = lambda a: _ptr(a) if a is not None else None
+    fn(B, L, D, M, _ptr(x), _ptr(dy), *map(_ptr, ps), opt(sin), opt(gout), _ptr(dx), *map(_ptr, g),
+       opt(ds))
+    out = {"decay": g[0], "freq": g[1], "amp": g[2], "phase": g[3]}
+    if want_ds:
+        out["state_in"] = ds[..., 0] + 1j * ds[..., 1]
+    return dx, out
 
 
-def backward_conv(x, dy, decay, freq, amp, phase):
-    """O3 by the convolution route.  Returns (dx, {decay, freq, amp, phase})."""
-    return _backward(_load().oracle_backward_conv, x, dy, decay, freq, amp, phase)
+def backward_conv(x, dy, decay, freq, amp, phase, state_in=None, d_state_out=None):
+    """O3 by the convolution route.  Returns (dx, {decay, freq, amp, phase}); with
+    state_in (the forward's initial state) and/or d_state_out (the loss gradient of
+    the terminal state, [B][D][M] complex) the dict also holds "state_in", the loss
+    gradient of the initial state."""
+    return _backward(_load().oracle_backward_conv, x, dy, decay, freq, amp, phase, state_in,
+                     d_state_out)
 
 
-def backward_rec(x, dy, decay, freq, amp, phase):
-    """O3 by the reverse-time Jordan recurrence.  Returns (dx, grads dict)."""
-    return _backward(_load().oracle_backward_rec, x, dy, decay, freq, amp, phase)
+def backward_rec(x, dy, decay, freq, amp, phase, state_in=None, d_state_out=None):
+    """O3 by the reverse-time Jordan recurrence.  Same returns as backward_conv."""
+    return _backward(_load().oracle_backward_rec, x, dy, decay, freq, amp, phase, state_in,
+                     d_state_out)

@@ -171,11 +171,29 @@ void oracle_rec_decode(long B, int D, int M, const double *state_in,
  *   dg   = -sum_n rho[n] n A exp(-g n) cos(w n + p)
  *   dw   = -sum_n rho[n] n A exp(-g n) sin(w n + p).
  * Gradients are [D][M] and are overwritten. */
+/* Optional state terms (all [B][D][M][2]; NULL = absent):
+ *   state_in     the state before token 0 of the forward pass (Sec. 3.2-3.3);
+ *   d_state_out  g, the loss gradient w.r.t. (Re, Im) of the terminal state,
+ *                i.e. the loss has the extra term Re(conj(g) s_L);
+ *   d_state_in   output: the loss gradient w.r.t. (Re, Im) of state_in.
+ * Convolution route: every extra term as a direct sum of closed-form powers
+ * (Eq. 5): with n = L-1-j, dx_j += |g| e^{-gamma n} cos(omega n - arg g);
+ * W = sum_t dy_t lambda^(t+1), V = sum_t dy_t (t+1) lambda^(t+1),
+ * J = sum_j (L-1-j) lambda^(L-1-j) x_j + L lambda^L s_in;
+ * G += s_in W, P += s_in V, dgamma -= Re(conj(g) J), domega -= Im(conj(g) J),
+ * d_state_in = conj(c W) + g conj(lambda^L). */
+static cplx lam_pow_closed(double g, double w, double n)
+{
+    return exp(-g * n) * (cos(w * n) + I * sin(w * n));
+}
+
 void oracle_backward_conv(long B, long L, int D, int M, const double *x,
                           const double *dy, const double *decay,
                           const double *freq, const double *amp,
-                          const double *phase, double *dx, double *d_decay,
-                          double *d_freq, double *d_amp, double *d_phase)
+                          const double *phase, const double *state_in,
+                          const double *d_state_out, double *dx, double *d_decay,
+                          double *d_freq, double *d_amp, double *d_phase,
+                          double *d_state_in)
 {
     double *K = (double *)malloc(sizeof(double) * (size_t)D * (size_t)L);
     oracle_kernel_table(D, M, decay, freq, amp, phase, L, K);
@@ -210,6 +228,39 @@ void oracle_backward_conv(long B, long L, int D, int M, const double *x,
                 sg -= rho[n] * (double)n * a * e * cs;
                 sw -= rho[n] * (double)n * a * e * sn;
             }
+            const cplx c = a * (cos(p) + I * sin(p));
+            for (long b = 0; b < B; ++b) {
+                const size_t o = (((size_t)b * D + d) * M + m) * 2;
+                const cplx si = state_in ? state_in[o] + I * state_in[o + 1] : 0.0;
+                const cplx gg = d_state_out ? d_state_out[o] + I * d_state_out[o + 1] : 0.0;
+                cplx W = 0.0, V = 0.0, J = 0.0;
+                for (long t = 0; t < L; ++t) {
+                    const double u = dy[((size_t)b * L + t) * D + d];
+                    const cplx pw = lam_pow_closed(g, w, (double)(t + 1));
+                    W += u * pw;
+                    V += u * (double)(t + 1) * pw;
+                    J += (double)(L - 1 - t) * lam_pow_closed(g, w, (double)(L - 1 - t)) *
+                         x[((size_t)b * L + t) * D + d];
+                }
+                J += (double)L * lam_pow_closed(g, w, (double)L) * si;
+                const cplx Gi = si * W, Pi = si * V;
+                sa += creal((cos(p) + I * sin(p)) * Gi);
+                sp -= cimag(c * Gi);
+                sg -= creal(c * Pi) + creal(conj(gg) * J);
+                sw -= cimag(c * Pi) + cimag(conj(gg) * J);
+                if (d_state_in) {
+                    const cplx ds = conj(c * W) + gg * conj(lam_pow_closed(g, w, (double)L));
+                    d_state_in[o] = creal(ds);
+                    d_state_in[o + 1] = cimag(ds);
+                }
+                if (d_state_out) {
+                    const double mag = cabs(gg), arg = carg(gg);
+                    for (long j = 0; j < L; ++j) {
+                        const double n = (double)(L - 1 - j);
+                        dx[((size_t)b * L + j) * D + d] += mag * exp(-g * n) * cos(w * n - arg);
+                    }
+                }
+            }
             d_amp[pm] = sa;
             d_phase[pm] = sp;
             d_decay[pm] = sg;
@@ -226,11 +277,21 @@ void oracle_backward_conv(long B, long L, int D, int M, const double *x,
  *   R_j = lambda (R_{j+1} + S_{j+1})       (R_j = sum_{t>=j} (t-j) lambda^{t-j} dy_t)
  *   dx_j = sum_m Re(c S_j),  G = sum_{b,j} x_j S_j,  P = sum_{b,j} x_j R_j
  *   dA = Re(e^{i phi} G), dphi = -Im(c G), dgamma = -Re(c P), domega = -Im(c P). */
+/* State terms (see oracle_backward_conv) by recurrences: the terminal-state
+ * gradient is a second adjoint Phi_j = lambda Phi_{j+1}, Phi_{L-1} = conj(g),
+ * read out with coefficient 1 (dx_j += Re Phi_j); J uses the unit adjoint
+ * U_j = lambda U_{j+1} (U_{L-1} = 1) and its Jordan partner
+ * Q_j = lambda (Q_{j+1} + U_{j+1}) (Q_j = (L-1-j) lambda^(L-1-j)): J = sum x Q +
+ * s_in lambda (Q_0 + U_0); with the adjoint pair's end values S_0, R_0:
+ * G += s_in lambda S_0, P += s_in lambda (R_0 + S_0),
+ * d_state_in = conj(c lambda S_0) + g conj(lambda U_0). */
 void oracle_backward_rec(long B, long L, int D, int M, const double *x,
                          const double *dy, const double *decay,
                          const double *freq, const double *amp,
-                         const double *phase, double *dx, double *d_decay,
-                         double *d_freq, double *d_amp, double *d_phase)
+                         const double *phase, const double *state_in,
+                         const double *d_state_out, double *dx, double *d_decay,
+                         double *d_freq, double *d_amp, double *d_phase,
+                         double *d_state_in)
 {
 #pragma omp parallel for schedule(static)
     for (int d = 0; d < D; ++d) {
@@ -241,22 +302,43 @@ void oracle_backward_rec(long B, long L, int D, int M, const double *x,
             size_t pm = (size_t)d * M + m;
             cplx lam = mode_lambda(decay[pm], freq[pm]);
             cplx c = mode_coef(amp[pm], phase[pm]);
-            cplx G = 0.0, P = 0.0;
+            cplx G = 0.0, P = 0.0, GJ = 0.0;
             for (long b = 0; b < B; ++b) {
-                cplx S = 0.0, R = 0.0;
+                const size_t o = (((size_t)b * D + d) * M + m) * 2;
+                const cplx si = state_in ? state_in[o] + I * state_in[o + 1] : 0.0;
+                const cplx gg = d_state_out ? d_state_out[o] + I * d_state_out[o + 1] : 0.0;
+                cplx S = 0.0, R = 0.0, Phi = 0.0, U = 0.0, Q = 0.0, J = 0.0;
                 for (long j = L - 1; j >= 0; --j) {
                     size_t i = ((size_t)b * L + j) * D + d;
                     R = lam * (R + S);
                     S = lam * S + dy[i];
-                    dx[i] += creal(c * S);
+                    if (j == L - 1) {
+                        Phi = conj(gg);
+                        U = 1.0;
+                    } else {
+                        Q = lam * (Q + U);
+                        U = lam * U;
+                        Phi = lam * Phi;
+                    }
+                    dx[i] += creal(c * S) + creal(Phi);
                     G += x[i] * S;
                     P += x[i] * R;
+                    J += x[i] * Q;
+                }
+                J += si * lam * (Q + U);
+                G += si * lam * S;
+                P += si * lam * (R + S);
+                GJ += conj(gg) * J;
+                if (d_state_in) {
+                    const cplx ds = conj(c * lam * S) + gg * conj(lam * U);
+                    d_state_in[o] = creal(ds);
+                    d_state_in[o + 1] = cimag(ds);
                 }
             }
             d_amp[pm] = creal((cos(phase[pm]) + I * sin(phase[pm])) * G);
             d_phase[pm] = -cimag(c * G);
-            d_decay[pm] = -creal(c * P);
-            d_freq[pm] = -cimag(c * P);
+            d_decay[pm] = -creal(c * P) - creal(GJ);
+            d_freq[pm] = -cimag(c * P) - cimag(GJ);
         }
     }
 }

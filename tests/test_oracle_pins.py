@@ -351,6 +351,73 @@ def test_backward_matches_central_finite_differences(seed):
         assert abs(dx_r[idx] - fdx[idx]) < 1e-8
 
 
+def _loss_state(x, dy, params, s_in, g):
+    """l = sum(dy * y) + sum Re(conj(g) s_L) for the prefill from s_in (O2)."""
+    y, sL = oracle.rec_prefill(x, *params, state_in=s_in)
+    return float(np.sum(dy * y) + np.sum(np.real(np.conj(g) * sL)))
+
+
+@pytest.mark.parametrize("seed", [5, 6])
+def test_backward_with_state_terms_matches_central_finite_differences(seed):
+    """Backward of a prefill from an initial state with a loss on its terminal
+    state: both routes against central differences of that loss (in the
+    parameters, in x, and in Re / Im of the initial state)."""
+    inp = make_inputs(1, 29, 2, 2, "f32", seed=seed, with_dy=True)
+    x, dy = inp.x.astype(np.float64), inp.dy.astype(np.float64)
+    params = [p.astype(np.float64) for p in inp.params()]
+    rng = np.random.default_rng(seed)
+    s_in = rng.normal(size=(1, 2, 2)) + 1j * rng.normal(size=(1, 2, 2))
+    g = rng.normal(size=(1, 2, 2)) + 1j * rng.normal(size=(1, 2, 2))
+    outs = [oracle.backward_conv(x, dy, *params, state_in=s_in, d_state_out=g),
+            oracle.backward_rec(x, dy, *params, state_in=s_in, d_state_out=g)]
+    for k, name in enumerate(["decay", "freq", "amp", "phase"]):
+        fd = np.zeros_like(params[k])
+        for idx in np.ndindex(*params[k].shape):
+            h = 1e-6 * max(1.0, abs(params[k][idx]))
+            pp = [q.copy() for q in params]
+            pm = [q.copy() for q in params]
+            pp[k][idx] += h
+            pm[k][idx] -= h
+            fd[idx] = (_loss_state(x, dy, pp, s_in, g) - _loss_state(x, dy, pm, s_in, g)) / (2 * h)
+        scale = max(1.0, np.abs(fd).max())
+        for _, gr in outs:
+            assert np.abs(gr[name] - fd).max() / scale < 2e-7, name
+    for idx in [(0, 0, 0), (0, 7, 1), (0, 28, 0), (0, 28, 1)]:
+        xp, xm = x.copy(), x.copy()
+        xp[idx] += 1e-3
+        xm[idx] -= 1e-3
+        fdx = (_loss_state(xp, dy, params, s_in, g) - _loss_state(xm, dy, params, s_in, g)) / 2e-3
+        for dx, _ in outs:
+            assert abs(dx[idx] - fdx) < 1e-8, idx
+    for idx in np.ndindex(1, 2, 2):
+        for part, unit in (("re", 1.0), ("im", 1j)):
+            sp, sm = s_in.copy(), s_in.copy()
+            sp[idx] += 1e-4 * unit
+            sm[idx] -= 1e-4 * unit
+            fds = (_loss_state(x, dy, params, sp, g) - _loss_state(x, dy, params, sm, g)) / 2e-4
+            for _, gr in outs:
+                got = gr["state_in"][idx].real if part == "re" else gr["state_in"][idx].imag
+                assert abs(got - fds) < 1e-8 * max(1.0, abs(fds)), (idx, part)
+
+
+def test_backward_state_terms_routes_agree_and_vanish_when_zero():
+    inp = make_inputs(2, 300, 3, 4, "f32", seed=41, with_dy=True)
+    rng = np.random.default_rng(9)
+    s_in = rng.normal(size=(2, 3, 4)) + 1j * rng.normal(size=(2, 3, 4))
+    g = rng.normal(size=(2, 3, 4)) + 1j * rng.normal(size=(2, 3, 4))
+    dxc, gc = oracle.backward_conv(inp.x, inp.dy, *inp.params(), state_in=s_in, d_state_out=g)
+    dxr, gr = oracle.backward_rec(inp.x, inp.dy, *inp.params(), state_in=s_in, d_state_out=g)
+    np.testing.assert_allclose(dxc, dxr, rtol=1e-9, atol=1e-9)
+    for k in ("decay", "freq", "amp", "phase", "state_in"):
+        np.testing.assert_allclose(gc[k], gr[k], rtol=1e-9, atol=1e-9 * np.abs(gr[k]).max())
+    z = np.zeros((2, 3, 4), complex)
+    dx0, g0 = oracle.backward_rec(inp.x, inp.dy, *inp.params())
+    dxz, gz = oracle.backward_rec(inp.x, inp.dy, *inp.params(), state_in=z, d_state_out=z)
+    assert np.array_equal(dx0, dxz)
+    for k in ("decay", "freq", "amp", "phase"):
+        assert np.array_equal(g0[k], gz[k])
+
+
 def test_backward_routes_agree():
     inp = make_inputs(2, 211, 4, 5, "f32", seed=47, with_dy=True)
     dx_c, g_c = oracle.backward_conv(inp.x, inp.dy, *inp.params())
