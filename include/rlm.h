@@ -193,6 +193,22 @@ RLM_API rlm_status rlm_state_init(rlm_state *state, const rlm_params *p, const r
 RLM_API rlm_status rlm_mix_backward(const rlm_tensor *dy, const rlm_tensor *x, const rlm_params *p,
                             rlm_tensor *dx, rlm_grads *dparams, const rlm_launch *launch);
 
+/* Backward of rlm_mix_prefill_from (training through a cached state), Sec. 3.2-3.3:
+ * the loss may also depend on the terminal state s_L, and the forward may have
+ * started from state_in.
+ *   state_in     nullable; the forward's initial state (->s read, [B][D][M] complex).
+ *   d_state_out  nullable; g = dl/d(Re s_L) + i dl/d(Im s_L) per (b, d, m) (->s read);
+ *                the loss then has the extra term Re(conj(g) s_L).
+ *   d_state_in   nullable output; dl/d(Re s_in) + i dl/d(Im s_in) (->s written); it
+ *                must not overlap dx, dparams, state_in or d_state_out.
+ * dx and dparams as for rlm_mix_backward, with the state terms included.  Paths:
+ * without d_state_out, bf16 with M <= 32 runs the tcgen05 backward (state_in and
+ * d_state_in are per-(b, d, m) terms at its end); with d_state_out, or fp32, or
+ * M > 32, the SIMT backward.  rlm_backward_workspace_size covers both. */
+RLM_API rlm_status rlm_mix_backward_from(const rlm_tensor *dy, const rlm_tensor *x, const rlm_params *p,
+                                         const rlm_state *state_in, const rlm_state *d_state_out, rlm_tensor *dx,
+                                         rlm_grads *dparams, rlm_state *d_state_in, const rlm_launch *launch);
+
 RLM_API size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype);
 
 /* ------------------------------------------------------------------ utility

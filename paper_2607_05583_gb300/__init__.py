@@ -22,7 +22,8 @@ from . import build as _build_mod
 
 __all__ = [
     "RlmError", "Params", "Grads", "State", "load_library", "library_path",
-    "rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_prefill_noalloc", "rlm_mix_decode", "rlm_mix_backward", "rlm_state_init",
+    "rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_prefill_noalloc", "rlm_mix_decode", "rlm_mix_backward",
+    "rlm_mix_backward_from", "rlm_state_init",
     "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
     "rlm_validate_params", "rlm_get_device_status", "rlm_status_string",
     "rlm_version", "rlm_kernels_launched", "rlm_measure_row_io", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
@@ -90,6 +91,8 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.rlm_mix_decode.argtypes = [P(_Tensor), P(_State), P(_Tensor), P(_Launch)]
     lib.rlm_mix_backward.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_Tensor),
                                      P(_Grads), P(_Launch)]
+    lib.rlm_mix_backward_from.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_State), P(_State),
+                                          P(_Tensor), P(_Grads), P(_State), P(_Launch)]
     lib.rlm_state_init.argtypes = [P(_State), P(_Params), P(_Launch)]
     lib.rlm_validate_params.argtypes = [P(_Params)]
     lib.rlm_get_device_status.argtypes = [P(_Launch)]
@@ -98,7 +101,7 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
                                     ctypes.c_int, ctypes.c_int]
         getattr(lib, f).restype = ctypes.c_size_t
     for f in ("rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_decode", "rlm_mix_backward",
-              "rlm_state_init", "rlm_validate_params", "rlm_get_device_status"):
+              "rlm_mix_backward_from", "rlm_state_init", "rlm_validate_params", "rlm_get_device_status"):
         getattr(lib, f).restype = ctypes.c_int
     lib.rlm_status_string.argtypes = [ctypes.c_int]
     lib.rlm_status_string.restype = ctypes.c_char_p
@@ -344,6 +347,26 @@ def rlm_mix_backward(dy: torch.Tensor, x: torch.Tensor, params: Params, dx: torc
     _check(lib.rlm_mix_backward(ctypes.byref(dyt), ctypes.byref(xt), ctypes.byref(params._c()),
                                 ctypes.byref(dxt), ctypes.byref(dparams._c()),
                                 ctypes.byref(_launch(stream, workspace))), "rlm_mix_backward")
+
+
+def rlm_mix_backward_from(dy: torch.Tensor, x: torch.Tensor, params: Params, state_in: State | None,
+                          d_state_out: State | None, dx: torch.Tensor, dparams: Grads,
+                          d_state_in: State | None = None, workspace: torch.Tensor | None = None,
+                          stream=None) -> None:
+    """Backward of rlm_mix_prefill_from: dx, the parameter gradients and (if
+    ``d_state_in`` is given) the gradient of the initial state, for a loss that may
+    also depend on the terminal state (its gradient ``d_state_out``).  Only the
+    ``s`` buffers of the state arguments are used."""
+    lib = load_library()
+    dyt, xt, dxt = _field(dy), _field(x), _field(dx)
+    if workspace is None:
+        workspace = _workspace(lib.rlm_backward_workspace_size(xt.B, xt.L, xt.D, params.M, xt.dtype),
+                               x.device)
+    opt = lambda st: ctypes.byref(st._c()) if st is not None else None
+    _check(lib.rlm_mix_backward_from(ctypes.byref(dyt), ctypes.byref(xt), ctypes.byref(params._c()),
+                                     opt(state_in), opt(d_state_out), ctypes.byref(dxt),
+                                     ctypes.byref(dparams._c()), opt(d_state_in),
+                                     ctypes.byref(_launch(stream, workspace))), "rlm_mix_backward_from")
 
 
 def rlm_validate_params(params: Params) -> None:

@@ -2,6 +2,7 @@
 // sizing and dispatch to the kernels.  Nothing here allocates device memory.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -140,6 +141,16 @@ int simt_chunks(int64_t B, int64_t L, int D) {
     return (int)((L + C - 1) / C);
 }
 
+// The complex [B][D][M] buffer of an optional state argument (only ->s is used).
+rlm_status check_state_s(const rlm_state *st, int64_t B, int64_t D, int M, const char *name) {
+    if (!st) return RLM_OK;
+    if (!st->s || !aligned16(st->s)) return fail(RLM_ERR_INVALID_ARG, "%s->s is NULL or not 16-byte aligned", name);
+    if (st->B != B || st->D != D || st->M != M)
+        return fail(RLM_ERR_INVALID_ARG, "%s is [B=%d][D=%d][M=%d], expected [%lld][%lld][%d]", name, st->B, st->D,
+                    st->M, (long long)B, (long long)D, M);
+    return RLM_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -170,7 +181,10 @@ size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype 
 
 size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
     if (B < 1 || L < 1 || D < 1 || M < 1) return 0;
-    if (tc_backward_supported(B, L, D, M, dtype)) return tc_backward_ws_bytes(B, L, D, M);
+    // A call with a terminal-state gradient runs the SIMT backward even where the
+    // tcgen05 one applies, so the size covers both.
+    if (tc_backward_supported(B, L, D, M, dtype))
+        return std::max(tc_backward_ws_bytes(B, L, D, M), simt_backward_ws_bytes(B, L, D, M));
     return simt_backward_ws_bytes(B, L, D, M);
 }
 
@@ -265,6 +279,13 @@ rlm_status rlm_state_init(rlm_state *state, const rlm_params *p, const rlm_launc
 
 rlm_status rlm_mix_backward(const rlm_tensor *dy, const rlm_tensor *x, const rlm_params *p,
                             rlm_tensor *dx, rlm_grads *g, const rlm_launch *ln) {
+    return rlm_mix_backward_from(dy, x, p, nullptr, nullptr, dx, g, nullptr, ln);
+}
+
+
+rlm_status rlm_mix_backward_from(const rlm_tensor *dy, const rlm_tensor *x, const rlm_params *p,
+                                 const rlm_state *state_in, const rlm_state *d_state_out, rlm_tensor *dx,
+                                 rlm_grads *g, rlm_state *d_state_in, const rlm_launch *ln) {
     rlm_status s;
     if ((s = check_tensor(dy, "dy")) != RLM_OK) return s;
     if ((s = check_tensor(x, "x")) != RLM_OK) return s;
@@ -281,8 +302,24 @@ rlm_status rlm_mix_backward(const rlm_tensor *dy, const rlm_tensor *x, const rlm
         if (!gs[i] || !aligned16(gs[i]))
             return fail(RLM_ERR_INVALID_ARG, "dparams pointer %d is NULL or not 16-byte aligned", i);
     if (g->D != p->D || g->M != p->M) return fail(RLM_ERR_INVALID_ARG, "dparams shape differs from params");
+    if ((s = check_state_s(state_in, x->B, x->D, p->M, "state_in")) != RLM_OK) return s;
+    if ((s = check_state_s(d_state_out, x->B, x->D, p->M, "d_state_out")) != RLM_OK) return s;
+    if ((s = check_state_s(d_state_in, x->B, x->D, p->M, "d_state_in")) != RLM_OK) return s;
+    if (d_state_in) {
+        const size_t sb = (size_t)x->B * x->D * p->M * 8;
+        if (overlap(d_state_in->s, sb, dx->ptr, tensor_bytes(dx)) ||
+            (state_in && overlap(d_state_in->s, sb, state_in->s, sb)) ||
+            (d_state_out && overlap(d_state_in->s, sb, d_state_out->s, sb)))
+            return fail(RLM_ERR_INVALID_ARG, "d_state_in overlaps dx, state_in or d_state_out");
+        for (int i = 0; i < 4; ++i)
+            if (overlap(d_state_in->s, sb, gs[i], (size_t)p->D * p->M * sizeof(float)))
+                return fail(RLM_ERR_INVALID_ARG, "d_state_in overlaps dparams");
+    }
+    const float *sin = state_in ? state_in->s : nullptr;
+    const float *gout = d_state_out ? d_state_out->s : nullptr;
+    float *dsin = d_state_in ? d_state_in->s : nullptr;
     const int D = (int)x->D, M = p->M;
-    const bool tc = tc_backward_supported(x->B, x->L, D, M, x->dtype);
+    const bool tc = !gout && tc_backward_supported(x->B, x->L, D, M, x->dtype);
     if (!tc && simt_chunks(x->B, x->L, D) > 65535)
         return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
     const size_t need = rlm_backward_workspace_size(x->B, x->L, D, M, x->dtype);
@@ -290,9 +327,10 @@ rlm_status rlm_mix_backward(const rlm_tensor *dy, const rlm_tensor *x, const rlm
     cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
     cudaError_t e =
         tc ? tc_backward(dy->ptr, x->ptr, dx->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp,
-                         p->phase, g->decay, g->freq, g->amp, g->phase, ln->workspace, st)
+                         p->phase, sin, dsin, g->decay, g->freq, g->amp, g->phase, ln->workspace, st)
            : simt_backward(dy->ptr, x->ptr, dx->ptr, x->dtype, x->B, x->L, D, M, p->decay, p->freq,
-                           p->amp, p->phase, g->decay, g->freq, g->amp, g->phase, ln->workspace, st);
+                           p->amp, p->phase, sin, gout, dsin, g->decay, g->freq, g->amp, g->phase,
+                           ln->workspace, st);
     if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_backward launch");
     return RLM_OK;
 }

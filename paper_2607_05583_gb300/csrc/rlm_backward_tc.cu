@@ -305,6 +305,7 @@ struct BwdArgs {
     int64_t L;
     int row0;                 // first (b * D + d) row of this launch (0: the whole problem)
     float4 *coef_out;         // nullable, [D][M]   (time-reversed prefill)
+    float2 *d_state_in;       // nullable, [B*D][M] (backward: gradient of the forward's state_in)
     __nv_bfloat16 *dxT;       // [B*D][Lp]
     int64_t Lp;
     int D, M;
@@ -481,12 +482,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     const bool onE = warp < 4 && mE < M;
     const float gamE = onE ? args.decay[d * M + mE] : 0.0f, omgE = onE ? args.freq[d * M + mE] : 0.0f;
     float gr = 0.0f, gi = 0.0f, pr = 0.0f, pi = 0.0f;
+    // The adjoint pair of the scan lanes; after the last tile it is (S_0, R_0).
+    float2 S = make_float2(0.0f, 0.0f), R = make_float2(0.0f, 0.0f);
     if (warp < 4) {
         // ---------------------------------------------------- reverse chunk scan
         const int q = warp, base = lane & 14;   // the mode's rows: base, base + 1, base + 16, base + 17
         const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
         const float2 a = lambda_pow(gamE, omgE, (float)kC);
-        float2 S = make_float2(0.0f, 0.0f), R = make_float2(0.0f, 0.0f);
         const int prow = 32 * q + lane;         // this lane's [S^n ; R^n] row
         // State before token 0 (reversed-time prefill): chunk kinj of the walk.
         float2 inj = make_float2(0.0f, 0.0f);
@@ -751,6 +753,25 @@ __global__ void __launch_bounds__(kThreads, 2)
             pr = fmaf(r * (float)n, ln.x, pr);
             pi = fmaf(r * (float)n, ln.y, pi);
         }
+        // The forward's initial state s_in (Sec. 3.2-3.3): G += s_in lambda S_0,
+        // P += s_in lambda (R_0 + S_0), added once per mode before the lanes' sum; the
+        // gradient of s_in is conj(c lambda S_0).
+        if (s == 0 && onE && (args.state_in || args.d_state_in)) {
+            const float2 l1 = lambda_pow(gamE, omgE, 1.0f);
+            const float2 ls = cmul(l1, S);
+            if (args.state_in) {
+                const float2 si = args.state_in[(int64_t)row * M + mE];
+                const float2 gin = cmul(si, ls), pin = cmul(si, cmul(l1, make_float2(R.x + S.x, R.y + S.y)));
+                gr += gin.x;
+                gi += gin.y;
+                pr += pin.x;
+                pi += pin.y;
+            }
+            if (args.d_state_in) {
+                const float2 cls = cmul(mode_coef(args.amp[d * M + mE], args.phase[d * M + mE]), ls);
+                args.d_state_in[(int64_t)row * M + mE] = make_float2(cls.x, -cls.y);
+            }
+        }
 #pragma unroll
         for (int o = 1; o <= 16; o <<= 4) {
             gr += __shfl_xor_sync(0xffffffffu, gr, o);
@@ -942,6 +963,7 @@ BwdArgs base_args(const float *decay, const float *freq, const float *amp, const
     a.state_in = nullptr;
     a.state_out = nullptr;
     a.coef_out = nullptr;
+    a.d_state_in = nullptr;
     a.dxT = outT;
     a.Lp = Lp;
     a.D = D;
@@ -977,8 +999,8 @@ cudaError_t run_layout_and_scan(const CUtensorMap &mdy, const CUtensorMap &mx, B
 
 cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
                         const float *decay, const float *freq, const float *amp, const float *phase,
-                        float *g_decay, float *g_freq, float *g_amp, float *g_phase, void *ws,
-                        cudaStream_t st) {
+                        const float *state_in, float *d_state_in, float *g_decay, float *g_freq, float *g_amp,
+                        float *g_phase, void *ws, cudaStream_t st) {
     if (!ws) return cudaErrorInvalidValue;
     const int64_t Lp = padded_len(L);
     char *w = static_cast<char *>(ws);
@@ -995,6 +1017,8 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     BwdArgs a = base_args(decay, freq, amp, phase, dxT, Lp, D, M);
     a.part_g = pg;
     a.part_p = pp;
+    a.state_in = reinterpret_cast<const float2 *>(state_in);
+    a.d_state_in = reinterpret_cast<float2 *>(d_state_in);
     e = run_layout_and_scan<true>(mdy, mx, a, B, L, D, Lp, static_cast<const __nv_bfloat16 *>(x),
                          static_cast<const __nv_bfloat16 *>(dy), xT, dyT, 2, 0, dxT,
                          static_cast<__nv_bfloat16 *>(dx), st);

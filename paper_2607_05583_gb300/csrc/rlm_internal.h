@@ -35,10 +35,13 @@ cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_
                          const float *phase, const float *state_in, float *state_out, float *coef_out,
                          void *ws, cudaStream_t st);
 
-// dx and the four parameter gradients (deterministic reduction).
+// dx and the four parameter gradients (deterministic reduction); optional state
+// terms ([B][D][M] complex, null = absent): the forward's state_in, the loss
+// gradient d_state_out of the terminal state, and the output d_state_in.
 cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt, int64_t B,
                           int64_t L, int D, int M, const float *decay, const float *freq,
-                          const float *amp, const float *phase, float *g_decay,
+                          const float *amp, const float *phase, const float *state_in,
+                          const float *d_state_out, float *d_state_in, float *g_decay,
                           float *g_freq, float *g_amp, float *g_phase, void *ws,
                           cudaStream_t st);
 
@@ -51,10 +54,12 @@ cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const fl
 // ---- tcgen05 backward (rlm_backward_tc.cu) -----------------------------------
 bool tc_backward_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
 size_t tc_backward_ws_bytes(int64_t B, int64_t L, int D, int M);
+// state_in (the forward's initial state) and d_state_in (output) may be null; a
+// terminal-state gradient is not covered here (the SIMT backward takes it).
 cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
                         const float *decay, const float *freq, const float *amp, const float *phase,
-                        float *g_decay, float *g_freq, float *g_amp, float *g_phase, void *ws,
-                        cudaStream_t st);
+                        const float *state_in, float *d_state_in, float *g_decay, float *g_freq, float *g_amp,
+                        float *g_phase, void *ws, cudaStream_t st);
 cudaError_t read_and_clear_bwd_status(int *status, cudaStream_t st);
 // The causal prefill (bf16 I/O, M <= 32) as the same reverse-time tcgen05 scan
 // applied to the time-reversed drive; used for the M the tcgen05 prefill does not

@@ -194,20 +194,39 @@ __global__ void __launch_bounds__(kBlock) k_chunk_output(
     }
 }
 
+// Optional state terms of the backward (all [B][D][M] complex, null = absent).
+struct StateTerms {
+    const float2 *state_in;   // the forward's state before token 0
+    const float2 *g;          // the loss gradient of the terminal state
+    float2 *d_state_in;       // output: the loss gradient of state_in
+    float2 *ws_j;             // with g: per-chunk partials of conj(g) J, next to ws_s / ws_r
+};
+
 // Phase 3 (backward).  Reverse time over dy; writes dx and, in place of the
 // carried (S, R), the chunk's partial sums G = sum x S and P = sum x R.
-template <typename T, int MG>
+// kG (a terminal-state gradient g): the second adjoint Phi_t = lambda^(L-1-t)
+// conj(g) joins dx with readout 1, and J = sum x_t (L-1-t) lambda^(L-1-t) (the unit
+// adjoint U and its Jordan partner Q, both closed-form at the chunk start) gives the
+// partials conj(g) J.  The chunk that ends at token 0 holds S_0 and R_0: it adds the
+// initial state's terms s_in lambda S_0 to G and s_in lambda (R_0 + S_0) to P (and
+// conj(g) L lambda^L s_in to its J partial) and writes the gradient of s_in,
+// conj(c lambda S_0) + g conj(lambda^L).
+template <typename T, int MG, bool kG>
 __global__ void __launch_bounds__(kBlock) k_chunk_backward(
     const T *__restrict__ dy, const T *__restrict__ x, T *__restrict__ dx, int64_t L, int D,
     int M, int tpc, int C, int nch, int64_t t0, const float *__restrict__ decay,
     const float *__restrict__ freq, const float *__restrict__ amp,
-    const float *__restrict__ phase, float2 *__restrict__ ws_s, float2 *__restrict__ ws_r) {
+    const float *__restrict__ phase, float2 *__restrict__ ws_s, float2 *__restrict__ ws_r,
+    const StateTerms stt) {
     const int gx = blockIdx.x * blockDim.x + threadIdx.x;
     const int d = gx / tpc, grp = gx % tpc;
     const int k = blockIdx.y, b = blockIdx.z;
     const bool active = d < D;
     float2 lam[MG], c[MG], s[MG], r[MG], G[MG], P[MG];
+    float2 phi[MG], U[MG], Q[MG], J[MG];
     const int64_t base = (((int64_t)b * nch + k) * D + d) * M;
+    const int64_t tau0 = t0 + (int64_t)k * C;
+    const int i0 = tau0 < 0 ? (int)(-tau0) : 0;
 #pragma unroll
     for (int j = 0; j < MG; ++j) {
         const int m = grp * MG + j;
@@ -218,9 +237,16 @@ __global__ void __launch_bounds__(kBlock) k_chunk_backward(
         r[j] = on ? ws_r[base + m] : make_float2(0, 0);
         G[j] = make_float2(0, 0);
         P[j] = make_float2(0, 0);
+        if (kG) {
+            // At the first position (time L-1-tau, tau = tau0 + i0): lambda^tau.
+            const float n = (float)(tau0 + i0);
+            U[j] = on ? lambda_pow(decay[d * M + m], freq[d * M + m], n) : make_float2(0, 0);
+            Q[j] = make_float2(n * U[j].x, n * U[j].y);
+            const float2 gg = on ? stt.g[((int64_t)b * D + d) * M + m] : make_float2(0, 0);
+            phi[j] = cmul(U[j], make_float2(gg.x, -gg.y));
+            J[j] = make_float2(0, 0);
+        }
     }
-    const int64_t tau0 = t0 + (int64_t)k * C;
-    const int i0 = tau0 < 0 ? (int)(-tau0) : 0;
     // The next token's drives are loaded before this token's arithmetic.
     auto at = [&](int i) { return ((int64_t)b * L + (L - 1 - (tau0 + i))) * D + d; };
     float u_next = active && i0 < C ? ld_elem(dy + at(i0)) : 0.0f;
@@ -242,30 +268,67 @@ __global__ void __launch_bounds__(kBlock) k_chunk_backward(
             G[j].y = fmaf(xv, s[j].y, G[j].y);
             P[j].x = fmaf(xv, r[j].x, P[j].x);
             P[j].y = fmaf(xv, r[j].y, P[j].y);
+            if (kG) {
+                acc += phi[j].x;
+                J[j].x = fmaf(xv, Q[j].x, J[j].x);
+                J[j].y = fmaf(xv, Q[j].y, J[j].y);
+                phi[j] = cmul(lam[j], phi[j]);
+                Q[j] = cmul(lam[j], make_float2(Q[j].x + U[j].x, Q[j].y + U[j].y));
+                U[j] = cmul(lam[j], U[j]);
+            }
         }
         for (int o = tpc >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
         if (active && grp == 0) st_elem(dx + e, acc);
     }
+    const bool first_token = k == nch - 1;   // this chunk ends at token 0
 #pragma unroll
     for (int j = 0; j < MG; ++j) {
         const int m = grp * MG + j;
         if (active && m < M) {
+            const int64_t sm = ((int64_t)b * D + d) * M + m;
+            const float2 gg = kG ? stt.g[sm] : make_float2(0, 0);
+            float2 gj = kG ? cmul(make_float2(gg.x, -gg.y), J[j]) : make_float2(0, 0);
+            if (first_token) {
+                const float2 ls = cmul(lam[j], s[j]);   // lambda S_0
+                if (stt.state_in) {
+                    const float2 si = stt.state_in[sm];
+                    G[j] = cfma(si, ls, G[j]);
+                    P[j] = cfma(si, cmul(lam[j], make_float2(r[j].x + s[j].x, r[j].y + s[j].y)), P[j]);
+                    if (kG) {
+                        const float2 lL = lambda_pow(decay[d * M + m], freq[d * M + m], (float)L);
+                        const float2 jin = cmul(si, lL);
+                        gj = cfma(make_float2(gg.x, -gg.y), make_float2((float)L * jin.x, (float)L * jin.y), gj);
+                    }
+                }
+                if (stt.d_state_in) {
+                    const float2 cl = cmul(c[j], ls);
+                    float2 ds = make_float2(cl.x, -cl.y);
+                    if (kG) {
+                        const float2 lL = lambda_pow(decay[d * M + m], freq[d * M + m], (float)L);
+                        ds = cfma(gg, make_float2(lL.x, -lL.y), ds);
+                    }
+                    stt.d_state_in[sm] = ds;
+                }
+            }
             ws_s[base + m] = G[j];
             ws_r[base + m] = P[j];
+            if (kG) stt.ws_j[base + m] = gj;
         }
     }
 }
 
 // Phase 4 (backward).  One thread per (d, m): fixed-order sum of the partials
 // over (b, k) in double, then the four gradients.
+// ws_j (nullable): partials of conj(g) J from a terminal-state gradient, which
+// add -Re and -Im of their sum to dgamma and domega.
 __global__ void __launch_bounds__(256) k_grad_reduce(
     int64_t B, int D, int M, int nch, const float *__restrict__ amp,
     const float *__restrict__ phase, const float2 *__restrict__ ws_s,
-    const float2 *__restrict__ ws_r, float *__restrict__ g_decay, float *__restrict__ g_freq,
-    float *__restrict__ g_amp, float *__restrict__ g_phase) {
+    const float2 *__restrict__ ws_r, const float2 *__restrict__ ws_j, float *__restrict__ g_decay,
+    float *__restrict__ g_freq, float *__restrict__ g_amp, float *__restrict__ g_phase) {
     const int pm = blockIdx.x * blockDim.x + threadIdx.x;
     if (pm >= D * M) return;
-    double gr = 0, gi = 0, pr = 0, pi = 0;
+    double gr = 0, gi = 0, pr = 0, pi = 0, jr = 0, ji = 0;
     for (int64_t bk = 0; bk < B * nch; ++bk) {
         const int64_t off = bk * D * M + pm;
         const float2 g = ws_s[off], p = ws_r[off];
@@ -273,6 +336,10 @@ __global__ void __launch_bounds__(256) k_grad_reduce(
         gi += g.y;
         pr += p.x;
         pi += p.y;
+        if (ws_j) {
+            jr += ws_j[off].x;
+            ji += ws_j[off].y;
+        }
     }
     double sph, cph;
     sincos((double)phase[pm], &sph, &cph);
@@ -280,8 +347,8 @@ __global__ void __launch_bounds__(256) k_grad_reduce(
     const double cr = a * cph, ci = a * sph;
     g_amp[pm] = (float)(cph * gr - sph * gi);         // Re(e^{i phi} G)
     g_phase[pm] = (float)(-(cr * gi + ci * gr));      // -Im(c G)
-    g_decay[pm] = (float)(-(cr * pr - ci * pi));      // -Re(c P)
-    g_freq[pm] = (float)(-(cr * pi + ci * pr));       // -Im(c P)
+    g_decay[pm] = (float)(-(cr * pr - ci * pi) - jr);   // -Re(c P) - Re(conj(g) J)
+    g_freq[pm] = (float)(-(cr * pi + ci * pr) - ji);    // -Im(c P) - Im(conj(g) J)
 }
 
 template <typename T>
@@ -308,12 +375,18 @@ cudaError_t prefill_t(const T *x, T *y, int64_t B, int64_t L, int D, int M, cons
 template <typename T>
 cudaError_t backward_t(const T *dy, const T *x, T *dx, int64_t B, int64_t L, int D, int M,
                        const float *decay, const float *freq, const float *amp,
-                       const float *phase, float *gd, float *gf, float *ga, float *gp, void *ws,
+                       const float *phase, const float *state_in, const float *d_state_out,
+                       float *d_state_in, float *gd, float *gf, float *ga, float *gp, void *ws,
                        cudaStream_t st) {
     const ChunkGeom g = geom_c(L, bwd_chunk_len(B, L, D));
     const int64_t n = B * (int64_t)g.nch * D * M;
     float2 *ws_s = reinterpret_cast<float2 *>(ws);
     float2 *ws_r = ws_s + n;
+    StateTerms stt;
+    stt.state_in = reinterpret_cast<const float2 *>(state_in);
+    stt.g = reinterpret_cast<const float2 *>(d_state_out);
+    stt.d_state_in = reinterpret_cast<float2 *>(d_state_in);
+    stt.ws_j = d_state_out ? ws_r + n : nullptr;
     const int tpc1 = threads_per_channel(M, kMgFwd);
     dim3 grid1((unsigned)((D * tpc1 + kBlock - 1) / kBlock), (unsigned)g.nch, (unsigned)B);
     k_chunk_local<T, kMgFwd, true, true><<<grid1, kBlock, 0, st>>>(
@@ -323,10 +396,14 @@ cudaError_t backward_t(const T *dy, const T *x, T *dx, int64_t B, int64_t L, int
         B, D, M, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, ws_r, nullptr, nullptr, nullptr);
     const int tpc3 = threads_per_channel(M, kMgBwd);
     dim3 grid3((unsigned)((D * tpc3 + kBlock - 1) / kBlock), (unsigned)g.nch, (unsigned)B);
-    k_chunk_backward<T, kMgBwd><<<grid3, kBlock, 0, st>>>(
-        dy, x, dx, L, D, M, tpc3, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, ws_r);
+    if (d_state_out)
+        k_chunk_backward<T, kMgBwd, true><<<grid3, kBlock, 0, st>>>(
+            dy, x, dx, L, D, M, tpc3, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, ws_r, stt);
+    else
+        k_chunk_backward<T, kMgBwd, false><<<grid3, kBlock, 0, st>>>(
+            dy, x, dx, L, D, M, tpc3, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, ws_r, stt);
     k_grad_reduce<<<(unsigned)((D * M + 255) / 256), 256, 0, st>>>(
-        B, D, M, g.nch, amp, phase, ws_s, ws_r, gd, gf, ga, gp);
+        B, D, M, g.nch, amp, phase, ws_s, ws_r, stt.ws_j, gd, gf, ga, gp);
     count_launches(4);
     return cudaGetLastError();
 }
@@ -352,7 +429,7 @@ size_t simt_prefill_ws_bytes(int64_t B, int64_t L, int D, int M) {
 
 size_t simt_backward_ws_bytes(int64_t B, int64_t L, int D, int M) {
     const ChunkGeom g = geom_c(L, bwd_chunk_len(B, L, D));
-    return 2 * (size_t)B * g.nch * D * M * sizeof(float2);
+    return 3 * (size_t)B * g.nch * D * M * sizeof(float2);   // G, P and conj(g) J partials
 }
 
 cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_t L, int D,
@@ -370,23 +447,24 @@ cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const fl
                         const float2 *G, const float2 *P, float *g_decay, float *g_freq,
                         float *g_amp, float *g_phase, cudaStream_t st) {
     k_grad_reduce<<<(unsigned)((D * M + 255) / 256), 256, 0, st>>>(
-        nparts, D, M, 1, amp, phase, G, P, g_decay, g_freq, g_amp, g_phase);
+        nparts, D, M, 1, amp, phase, G, P, nullptr, g_decay, g_freq, g_amp, g_phase);
     count_launches(1);
     return cudaGetLastError();
 }
 
 cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt, int64_t B,
                           int64_t L, int D, int M, const float *decay, const float *freq,
-                          const float *amp, const float *phase, float *g_decay, float *g_freq,
+                          const float *amp, const float *phase, const float *state_in,
+                          const float *d_state_out, float *d_state_in, float *g_decay, float *g_freq,
                           float *g_amp, float *g_phase, void *ws, cudaStream_t st) {
     if (dt == RLM_BF16)
         return backward_t(static_cast<const __nv_bfloat16 *>(dy),
                           static_cast<const __nv_bfloat16 *>(x), static_cast<__nv_bfloat16 *>(dx),
-                          B, L, D, M, decay, freq, amp, phase, g_decay, g_freq, g_amp, g_phase,
-                          ws, st);
+                          B, L, D, M, decay, freq, amp, phase, state_in, d_state_out, d_state_in, g_decay,
+                          g_freq, g_amp, g_phase, ws, st);
     return backward_t(static_cast<const float *>(dy), static_cast<const float *>(x),
-                      static_cast<float *>(dx), B, L, D, M, decay, freq, amp, phase, g_decay,
-                      g_freq, g_amp, g_phase, ws, st);
+                      static_cast<float *>(dx), B, L, D, M, decay, freq, amp, phase, state_in, d_state_out,
+                      d_state_in, g_decay, g_freq, g_amp, g_phase, ws, st);
 }
 
 }  // namespace rlm

@@ -32,7 +32,7 @@ def _declared_entry_points():
 def test_header_declares_the_boundary():
     names = _declared_entry_points()
     for want in ("rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_decode", "rlm_mix_backward",
-                 "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
+                 "rlm_mix_backward_from", "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
                  "rlm_state_init", "rlm_validate_params", "rlm_get_device_status",
                  "rlm_status_string", "rlm_last_error"):
         assert want in names
@@ -181,6 +181,34 @@ def test_backward_rejects_bad_arguments_on_host(lib):
     gnull = rlm._Params(g.decay, 0, g.amp, g.phase, D, M)
     assert call(dy, x, dx, gnull) == rlm.RLM_ERR_INVALID_ARG
     assert call(dy, _t(FAKE + (1 << 30), B, L, D, rlm.RLM_F32), dx, g) == rlm.RLM_ERR_INVALID_ARG
+
+
+def test_backward_from_rejects_bad_state_arguments_on_host(lib):
+    B, L, D, M = 2, 100, 16, 4
+    dy, x, dx = _t(FAKE, B, L, D), _t(FAKE + (1 << 30), B, L, D), _t(FAKE + (1 << 31), B, L, D)
+    p = _p(D, M)
+    g = rlm._Params(FAKE + (1 << 35), FAKE + (1 << 35) + 4096, FAKE + (1 << 35) + 8192,
+                    FAKE + (1 << 35) + 12288, D, M)
+    ln = _launch(FAKE + (1 << 34), 1 << 40)
+    sbase = FAKE + (1 << 36)
+    ref = lambda st: ctypes.byref(st) if st else None
+
+    def call(si=None, go=None, ds=None):
+        return lib.rlm_mix_backward_from(ctypes.byref(dy), ctypes.byref(x), ctypes.byref(p),
+                                         ref(si), ref(go), ctypes.byref(dx), ctypes.byref(g),
+                                         ref(ds), ctypes.byref(ln))
+
+    def state(ptr, b=B, d=D, m=M):
+        return rlm._State(ptr, 0, b, d, m)
+
+    assert call(state(0)) == rlm.RLM_ERR_INVALID_ARG                       # NULL s
+    assert call(None, state(sbase + 4)) == rlm.RLM_ERR_INVALID_ARG         # misaligned s
+    assert call(state(sbase, b=B + 1)) == rlm.RLM_ERR_INVALID_ARG          # batch mismatch
+    assert call(None, state(sbase, d=D - 1)) == rlm.RLM_ERR_INVALID_ARG    # width mismatch
+    assert call(None, None, state(sbase, m=M + 1)) == rlm.RLM_ERR_INVALID_ARG
+    assert call(None, None, state(dx.ptr)) == rlm.RLM_ERR_INVALID_ARG      # d_state_in overlaps dx
+    assert call(state(sbase), None, state(sbase)) == rlm.RLM_ERR_INVALID_ARG  # ... the state_in
+    assert call(None, None, state(g.decay)) == rlm.RLM_ERR_INVALID_ARG     # ... a gradient
 
 
 @pytest.mark.parametrize("rows,D,sb,ctas", [

@@ -399,6 +399,92 @@ def test_backward_matches_oracle(B, L, D, M, dtype):
         assert_close(getattr(g, k).cpu().numpy(), g_ref[k], TOL[dtype], "d" + k)
 
 
+@pytest.mark.parametrize("B,L,D,M,dtype,with_s,with_g", [
+    # tensor-core backward: state_in, its gradient, no terminal-state gradient
+    (2, 3001, 16, 16, "bf16", True, False),
+    (1, 2 * 2048 + 1, 8, 32, "bf16", True, False),
+    (3, 65, 8, 5, "bf16", True, False),
+    (2, 3001, 16, 16, "bf16", False, False),
+    # SIMT: a terminal-state gradient (any dtype), fp32, bf16 with M > 32
+    (2, 3001, 16, 16, "bf16", True, True),
+    (1, 700, 8, 32, "bf16", False, True),
+    (2, 1000, 16, 7, "f32", True, True),
+    (1, 1, 8, 3, "f32", True, True),
+    (1, 700, 8, 40, "bf16", True, False),
+])
+def test_backward_with_state_terms_matches_oracle(B, L, D, M, dtype, with_s, with_g):
+    """Backward of prefill_from (Sec. 3.2-3.3 with an initial state): dx, the four
+    parameter gradients and the initial-state gradient, for a loss
+    sum(dy * y) + Re<g, state_out>, against the oracle's adjoint recurrence."""
+    inp = make_inputs(B, L, D, M, dtype, seed=L + 3 * M, with_dy=True)
+    rng = np.random.default_rng(L + M)
+    pre = make_inputs(B, 300, D, M, dtype, seed=2 + M)
+    s_in = oracle.rec_prefill(pre.x, *inp.params())[1] if with_s else None
+    g_out = ((rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M)))
+             if with_g else None)
+    x, dy = to_dev(inp.x, dtype), to_dev(inp.dy, dtype)
+    p = rlm.Params.from_arrays(*inp.params())
+    dx = torch.empty_like(x)
+    g = rlm.Grads.empty(D, M)
+    ds = rlm.State.empty(B, D, M)
+    rlm.rlm_mix_backward_from(dy, x, p, _state_from(inp, s_in) if with_s else None,
+                              _state_from(inp, g_out) if with_g else None, dx, g, ds)
+    torch.cuda.synchronize()
+    # a zero initial state leaves the forward unchanged and makes the oracle return
+    # the initial-state gradient
+    s_ref = s_in if with_s else np.zeros((B, D, M), np.complex128)
+    dx_ref, g_ref = oracle.backward_rec(inp.x, inp.dy, *inp.params(), state_in=s_ref,
+                                        d_state_out=g_out)
+    assert_close(to_np(dx), dx_ref, TOL[dtype], "dx")
+    for k in ("decay", "freq", "amp", "phase"):
+        assert_close(getattr(g, k).cpu().numpy(), g_ref[k], TOL[dtype], "d" + k)
+    ds_np = ds.complex().cpu().numpy()
+    want = g_ref["state_in"]
+    for part, got, ref in (("re", ds_np.real, want.real), ("im", ds_np.imag, want.imag)):
+        assert_close(got, ref, TOL[dtype], "dstate_in " + part)
+
+
+def test_backward_from_without_state_terms_equals_backward():
+    """No state arguments: the same kernels and bit-identical results as rlm_mix_backward."""
+    inp = make_inputs(2, 3001, 64, 16, "bf16", seed=12, with_dy=True)
+    dx0, g0 = _backward(inp)
+    x, dy = to_dev(inp.x, "bf16"), to_dev(inp.dy, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    dx1 = torch.empty_like(x)
+    g1 = rlm.Grads.empty(inp.D, inp.M)
+    rlm.rlm_mix_backward_from(dy, x, p, None, None, dx1, g1)
+    torch.cuda.synchronize()
+    assert torch.equal(dx0, dx1)
+    for k in ("decay", "freq", "amp", "phase"):
+        assert torch.equal(getattr(g0, k), getattr(g1, k))
+
+
+def test_split_backward_chains_state_gradients():
+    """Backward through a split sequence x1 || x2: the second half's backward with
+    state_in = state after x1 gives d_state_in, which fed as d_state_out into the
+    first half's backward reproduces the whole sequence's gradients (bf16, fp32
+    terminal-gradient path in the first half)."""
+    B, L, D, M, cut = 2, 5000, 16, 16, 2345
+    inp = make_inputs(B, L, D, M, "bf16", seed=41, with_dy=True)
+    x, dy = to_dev(inp.x, "bf16"), to_dev(inp.dy, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    st = rlm.State.empty(B, D, M)
+    x1, x2 = x[:, :cut].contiguous(), x[:, cut:].contiguous()
+    y1 = torch.empty_like(x1)
+    dy1, dy2 = dy[:, :cut].contiguous(), dy[:, cut:].contiguous()
+    rlm.rlm_mix_prefill(x1, p, y1, st)
+    dx2, g2, ds = torch.empty_like(x2), rlm.Grads.empty(D, M), rlm.State.empty(B, D, M)
+    rlm.rlm_mix_backward_from(dy2, x2, p, st, None, dx2, g2, ds)
+    dx1, g1 = torch.empty_like(x1), rlm.Grads.empty(D, M)
+    rlm.rlm_mix_backward_from(dy1, x1, p, None, ds, dx1, g1)
+    torch.cuda.synchronize()
+    dx_ref, g_ref = oracle.backward_rec(inp.x, inp.dy, *inp.params())
+    assert_close(to_np(torch.cat([dx1, dx2], 1)), dx_ref, TOL["bf16"], "dx")
+    for k in ("decay", "freq", "amp", "phase"):
+        got = getattr(g1, k).cpu().numpy() + getattr(g2, k).cpu().numpy()
+        assert_close(got, g_ref[k], TOL["bf16"], "d" + k)
+
+
 def test_backward_training_workload_sampled():
     """Training path: B=4, L=32768, D=512, M=32, bf16 I/O; dx and all four parameter
     gradients of sampled channels against the oracle."""
