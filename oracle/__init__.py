@@ -21,6 +21,12 @@ channel innermost):
 * ``backward_conv``  O3 via the convolution route (chain rule through Eq. 1-2).
 * ``backward_rec``   O3 via the reverse-time Jordan recurrence.
 * ``kernel_table``   K_d[n] of Eq. 1.
+* ``local_conv``     the local lexical path of Sec. 3.4: causal depthwise
+                      convolution of kernel size K over the drive history.
+* ``mixer_prefill`` / ``mixer_decode``
+                     the mixer output of Sec. 3.4 without head coupling
+                      (lambda_c = 0): z = sigmoid(g) * y + s * l, with y the
+                      resonant mixing above (numpy, fp64).
 """
 from __future__ import annotations
 
@@ -193,3 +199,54 @@ def backward_rec(x, dy, decay, freq, amp, phase, state_in=None, d_state_out=None
     """O3 by the reverse-time Jordan recurrence.  Same returns as backward_conv."""
     return _backward(_load().oracle_backward_rec, x, dy, decay, freq, amp, phase, state_in,
                      d_state_out)
+
+
+# ------------------------------------------------------------------ mixer (Sec. 3.4)
+def sigmoid(v) -> np.ndarray:
+    """The gate nonlinearity gamma = sigma(g) of Sec. 3.1, in fp64."""
+    v = _f64(v)
+    return 1.0 / (1.0 + np.exp(-v))
+
+
+def local_conv(u, conv_w, conv_in=None):
+    """The local lexical path of Sec. 3.4: l_t[d] = sum_{k<K} w[d][k] u_{t-k}[d],
+    a causal depthwise convolution of kernel size K.  Drives before token 0 come
+    from conv_in ([B][K-1][D], oldest first: conv_in[:, K-2] is u_{-1}), or are zero.
+
+    Returns (l [B][L][D], the last K-1 drives of conv_in || u, oldest first)."""
+    u, w = _f64(u), _f64(conv_w)
+    B, L, D = u.shape
+    K = w.shape[1]
+    if w.shape != (D, K):
+        raise ValueError("conv_w must be [D][K]")
+    hist = np.zeros((B, max(K - 1, 0), D)) if conv_in is None else _f64(conv_in)
+    if hist.shape != (B, max(K - 1, 0), D):
+        raise ValueError("conv_in must be [B][K-1][D]")
+    ext = np.concatenate([hist, u], axis=1)          # ext[:, K-1+t] = u_t
+    l = np.zeros((B, L, D))
+    for k in range(K):
+        l += w[:, k][None, None, :] * ext[:, K - 1 - k:K - 1 - k + L, :]
+    tail = ext[:, ext.shape[1] - max(K - 1, 0):, :].copy()
+    return l, tail
+
+
+def mixer_prefill(x, g, decay, freq, amp, phase, conv_w, scale, state_in=None, conv_in=None):
+    """Mixer output over a sequence (Sec. 3.4 with lambda_c = 0):
+    z_t = sigma(g_t) * y_t + s * l_t, y the resonant mixing of the drive x (O2,
+    from state_in) and l the local path over conv_in || x.  g = None means no gate
+    (gamma = 1).  Returns (z, terminal state [B][D][M] complex, last K-1 drives)."""
+    y, st = rec_prefill(x, decay, freq, amp, phase, state_in=state_in)
+    l, tail = local_conv(x, conv_w, conv_in)
+    gate = 1.0 if g is None else sigmoid(g)
+    return gate * y + _f64(scale)[None, None, :] * l, st, tail
+
+
+def mixer_decode(state, conv, x_t, g_t, decay, freq, amp, phase, conv_w, scale):
+    """One decode step of the mixer: the recurrence step (Eq. 4-5) and the local
+    path over the K-1 cached drives.  state [B][D][M] complex, conv [B][K-1][D],
+    x_t and g_t [B][D] (g_t None: no gate).  Returns (z_t, new state, new conv)."""
+    y, st = rec_decode(state, x_t, decay, freq, amp, phase)
+    x_t = _f64(x_t)
+    l, tail = local_conv(x_t[:, None, :], conv_w, conv)
+    gate = 1.0 if g_t is None else sigmoid(g_t)
+    return gate * y + _f64(scale)[None, :] * l[:, 0, :], st, tail

@@ -83,6 +83,41 @@ def make_inputs(B: int, L: int, D: int, M: int, dtype: str = "bf16", seed: int =
     return Inputs(B, L, D, M, dtype, x, decay, freq, amp, phase, dy, tokens)
 
 
+@dataclass
+class MixerInputs:
+    """The mixer wrapper's extra inputs around the resonant operator (Sec. 3.4):
+    the gate pre-activation g (the gate half of the grouped input projection), the
+    local path's depthwise causal kernel w and its channel scale s, and the drive
+    history and gate of decode steps."""
+    K: int
+    g: np.ndarray            # [B][L][D] float32 (bf16-representable for bf16 I/O)
+    conv_w: np.ndarray       # [D][K] float32
+    scale: np.ndarray        # [D] float32
+    conv_in: np.ndarray      # [B][K-1][D] float32: drives before token 0
+    g_tokens: np.ndarray | None = None   # [T][B][D] gate of decode steps
+
+
+def make_mixer_inputs(inp: Inputs, K: int, seed: int = 0) -> MixerInputs:
+    """Draw the mixer's extra inputs for an Inputs instance, from a generator of
+    their own (default_rng([seed, 1])) so the operator's draws are unchanged.
+    g ~ N(0, 1); w ~ N(0, 1/K) (variance 1/K, unit-variance output for unit
+    drives); s ~ U[0.5, 1.5]; the drive history ~ N(0, 1); decode-step gates
+    ~ N(0, 1), one per decode token of inp."""
+    rng = np.random.default_rng([seed, 1])
+    B, L, D = inp.B, inp.L, inp.D
+    g = rng.standard_normal((B, L, D), dtype=np.float32)
+    conv_w = (rng.standard_normal((D, max(K, 0))) / np.sqrt(max(K, 1))).astype(np.float32)
+    scale = rng.uniform(0.5, 1.5, D).astype(np.float32)
+    conv_in = rng.standard_normal((B, max(K - 1, 0), D), dtype=np.float32)
+    T = 0 if inp.tokens is None else inp.tokens.shape[0]
+    g_tokens = rng.standard_normal((T, B, D), dtype=np.float32) if T else None
+    if inp.dtype == "bf16":
+        g = round_to_bf16(g)
+        conv_in = round_to_bf16(conv_in)
+        g_tokens = round_to_bf16(g_tokens) if g_tokens is not None else None
+    return MixerInputs(K, g, conv_w, scale, conv_in, g_tokens)
+
+
 # The workloads, named by what they are (B, L, D, M, dtype).
 WORKLOADS = {
     "tiny_f32_prefill": dict(B=1, L=256, D=64, M=4, dtype="f32"),

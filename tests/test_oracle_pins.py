@@ -438,3 +438,78 @@ def test_backward_dx_is_time_reversed_forward():
 
 def test_oracle_threads_reported():
     assert oracle.num_threads() >= 1
+
+
+# ------------------------------------------------------------------ mixer (Sec. 3.4)
+def _mixer_case(B=2, L=37, D=5, M=3, K=4, seed=3):
+    from synth import make_mixer_inputs
+    inp = make_inputs(B, L, D, M, "f32", seed=seed)
+    return inp, make_mixer_inputs(inp, K, seed=seed)
+
+
+@pytest.mark.parametrize("K", [1, 2, 4, 7])
+def test_local_conv_is_an_fir_filter(K):
+    """The local path against scipy's direct-form FIR filter, run per channel over
+    the drive history followed by the sequence (zero initial conditions)."""
+    inp, mx = _mixer_case(K=K)
+    l, tail = oracle.local_conv(inp.x, mx.conv_w, mx.conv_in)
+    ext = np.concatenate([mx.conv_in.astype(np.float64), inp.x.astype(np.float64)], axis=1)
+    for b in range(inp.B):
+        for d in range(inp.D):
+            want = scipy.signal.lfilter(mx.conv_w[d].astype(np.float64), [1.0], ext[b, :, d])
+            np.testing.assert_allclose(l[b, :, d], want[K - 1:], rtol=1e-13, atol=1e-13)
+    np.testing.assert_array_equal(tail, ext[:, ext.shape[1] - (K - 1):, :])
+
+
+def test_local_conv_unit_lag_is_a_causal_shift():
+    """w = e_k gives l_t = u_{t-k}: the lag runs into the past (a mistaken
+    anti-causal or reversed kernel fails), and the history supplies t < k."""
+    inp, mx = _mixer_case(K=4)
+    for k in range(4):
+        w = np.zeros((inp.D, 4))
+        w[:, k] = 1.0
+        l, _ = oracle.local_conv(inp.x, w, mx.conv_in)
+        np.testing.assert_array_equal(l[:, k:], inp.x[:, :inp.L - k].astype(np.float64))
+        for t in range(k):
+            np.testing.assert_array_equal(l[:, t], mx.conv_in[:, 3 - k + t].astype(np.float64))
+
+
+def test_mixer_reduces_to_its_parts():
+    """sigma is scipy's expit; with zero amplitudes (y = 0) z is s * FIR(x); with a
+    zero local kernel z is expit(g) * y; with no gate z is y + s * l."""
+    import scipy.special
+    inp, mx = _mixer_case()
+    np.testing.assert_allclose(oracle.sigmoid(mx.g), scipy.special.expit(mx.g.astype(np.float64)),
+                               rtol=1e-15)
+    assert oracle.sigmoid(0.0) == 0.5
+    zero_amp = np.zeros_like(inp.amp)
+    z, _, _ = oracle.mixer_prefill(inp.x, mx.g, inp.decay, inp.freq, zero_amp, inp.phase,
+                                   mx.conv_w, mx.scale, conv_in=mx.conv_in)
+    ext = np.concatenate([mx.conv_in, inp.x], axis=1).astype(np.float64)
+    fir = scipy.signal.lfilter(mx.conv_w.astype(np.float64)[0], [1.0], ext[0, :, 0])[mx.K - 1:]
+    np.testing.assert_allclose(z[0, :, 0], mx.scale[0] * fir, rtol=1e-13, atol=1e-13)
+    z, _, _ = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), np.zeros_like(mx.conv_w), mx.scale)
+    y, _ = oracle.conv_prefill(inp.x, *inp.params()), None
+    np.testing.assert_allclose(z, scipy.special.expit(mx.g.astype(np.float64)) * y, rtol=1e-10,
+                               atol=1e-12)
+    z, _, _ = oracle.mixer_prefill(inp.x, None, *inp.params(), mx.conv_w, mx.scale)
+    l, _ = oracle.local_conv(inp.x, mx.conv_w)
+    np.testing.assert_allclose(z, y + mx.scale[None, None, :] * l, rtol=1e-10, atol=1e-12)
+
+
+def test_mixer_split_prefill_and_decode_continue_the_sequence():
+    """Prefill of x1, then prefill of x2 from (state, drive history), then decode
+    steps, reproduce one prefill of the whole sequence: z, state and history."""
+    inp, mx = _mixer_case(L=40, K=3)
+    args = (*inp.params(), mx.conv_w, mx.scale)
+    z, st, tail = oracle.mixer_prefill(inp.x, mx.g, *args, conv_in=mx.conv_in)
+    z1, st1, t1 = oracle.mixer_prefill(inp.x[:, :17], mx.g[:, :17], *args, conv_in=mx.conv_in)
+    z2, st2, t2 = oracle.mixer_prefill(inp.x[:, 17:35], mx.g[:, 17:35], *args, state_in=st1,
+                                       conv_in=t1)
+    np.testing.assert_allclose(np.concatenate([z1, z2], 1), z[:, :35], rtol=1e-10, atol=1e-12)
+    s, c = st2, t2
+    for t in range(35, 40):
+        zt, s, c = oracle.mixer_decode(s, c, inp.x[:, t], mx.g[:, t], *args)
+        np.testing.assert_allclose(zt, z[:, t], rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(s, st, rtol=1e-10, atol=1e-12)
+    np.testing.assert_array_equal(c, tail)
