@@ -211,6 +211,67 @@ RLM_API rlm_status rlm_mix_backward_from(const rlm_tensor *dy, const rlm_tensor 
 
 RLM_API size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype);
 
+/* ------------------------------------------------------------------ mixer
+ * The mixer wrapper of Sec. 3.4 around the operator, with head coupling off
+ * (lambda_c = 0, so the coupled field is y itself):
+ *
+ *   z_t[d] = sigma(g_t[d]) y_t[d] + s[d] l_t[d],   l_t[d] = sum_{k<K} w[d][k] u_{t-k}[d]
+ *
+ * u is the drive (x here), y its resonant mixing (as rlm_mix_prefill_from /
+ * rlm_mix_decode compute it), g the gate pre-activation (the gate half of the
+ * grouped input projection), sigma the logistic function, and l the local
+ * lexical path: a causal depthwise convolution of kernel size K whose output is
+ * scaled channel-wise by s.  The output projection that follows z is outside. */
+#define RLM_MAX_LOCAL_K 8
+
+/* Local lexical path (Sec. 3.4).  conv_w [D][K] fp32: conv_w[d*K + k] multiplies
+ * u_{t-k}[d]; scale [D] fp32 (s).  0 <= K <= RLM_MAX_LOCAL_K; K = 0 means no
+ * local path (conv_w and scale are then not read). */
+typedef struct {
+    const float *conv_w;
+    const float *scale;
+    int D, K;
+} rlm_local;
+
+/* The local path's drive history: the K-1 drives before the next token, oldest
+ * first, [B][K-1][D] in the element type of x: u[(b*(K-1) + j)*D + d] holds
+ * u_{t-K+1+j}[d] when the next token is t.  Unused (may be NULL) when K <= 1. */
+typedef struct {
+    void *u;
+    rlm_dtype dtype;
+    int64_t B;
+    int D, K;
+} rlm_conv_state;
+
+/* Mixer output over a sequence.
+ *   x         [B][L][D] drive (F32 or BF16)
+ *   g         nullable; [B][L][D] gate pre-activation, x's shape and dtype; NULL
+ *             means no gate (sigma(g) taken as 1)
+ *   p         resonator parameters
+ *   local     nullable (no local path) or K = 0
+ *   state_in  nullable; the resonators' state before token 0 (as rlm_mix_prefill_from)
+ *   conv_in   nullable; the drive history before token 0 (zero drives if NULL)
+ *   z         [B][L][D] output, x's shape and dtype; must not overlap x, g, the
+ *             parameters or the states
+ *   state_out nullable; terminal state and coefficients (may alias state_in)
+ *   conv_out  nullable; the history after token L-1 (may alias conv_in exactly)
+ * Workspace: rlm_prefill_workspace_size.  bf16 with M = 16 runs the gate and the
+ * local path inside the tcgen05 prefill's epilogue (one pass: x and g in, z out);
+ * other paths write the mixing into z and finish z with a separate pass. */
+RLM_API rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm_params *p,
+                                     const rlm_local *local, const rlm_state *state_in,
+                                     const rlm_conv_state *conv_in, rlm_tensor *z, rlm_state *state_out,
+                                     rlm_conv_state *conv_out, const rlm_launch *launch);
+
+/* One decode step of the mixer: the recurrence step of rlm_mix_decode, the
+ * gate, and the local path over the cached history, fused in one kernel.
+ *   x_t, g_t [B][1][D] (g_t nullable: no gate); state updated in place; conv
+ *   ([B][K-1][D], required when K >= 2) shifted in place by one token; z_t
+ *   [B][1][D] output.  No workspace. */
+RLM_API rlm_status rlm_mixer_decode(const rlm_tensor *x_t, const rlm_tensor *g_t, rlm_state *state,
+                                    const rlm_local *local, rlm_conv_state *conv, rlm_tensor *z_t,
+                                    const rlm_launch *launch);
+
 /* ------------------------------------------------------------------ utility
  * rlm_validate_params: copies p to the host (synchronous) and checks that every
  * value is finite and every gamma >= 0 (Sec. 3.1 requires alpha > 0; gamma = 0

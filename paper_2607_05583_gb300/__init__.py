@@ -23,7 +23,7 @@ from . import build as _build_mod
 __all__ = [
     "RlmError", "Params", "Grads", "State", "load_library", "library_path",
     "rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_prefill_noalloc", "rlm_mix_decode", "rlm_mix_backward",
-    "rlm_mix_backward_from", "rlm_state_init",
+    "rlm_mix_backward_from", "rlm_state_init", "Local", "ConvState", "rlm_mixer_prefill", "rlm_mixer_decode",
     "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
     "rlm_validate_params", "rlm_get_device_status", "rlm_status_string",
     "rlm_version", "rlm_kernels_launched", "rlm_measure_row_io", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
@@ -51,6 +51,16 @@ _Grads = _Params
 class _State(ctypes.Structure):
     _fields_ = [("s", ctypes.c_void_p), ("coef", ctypes.c_void_p),
                 ("B", ctypes.c_int), ("D", ctypes.c_int), ("M", ctypes.c_int)]
+
+
+class _Local(ctypes.Structure):
+    _fields_ = [("conv_w", ctypes.c_void_p), ("scale", ctypes.c_void_p),
+                ("D", ctypes.c_int), ("K", ctypes.c_int)]
+
+
+class _ConvState(ctypes.Structure):
+    _fields_ = [("u", ctypes.c_void_p), ("dtype", ctypes.c_int), ("B", ctypes.c_int64),
+                ("D", ctypes.c_int), ("K", ctypes.c_int)]
 
 
 class _Launch(ctypes.Structure):
@@ -93,6 +103,10 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
                                      P(_Grads), P(_Launch)]
     lib.rlm_mix_backward_from.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_State), P(_State),
                                           P(_Tensor), P(_Grads), P(_State), P(_Launch)]
+    lib.rlm_mixer_prefill.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_Local), P(_State),
+                                      P(_ConvState), P(_Tensor), P(_State), P(_ConvState), P(_Launch)]
+    lib.rlm_mixer_decode.argtypes = [P(_Tensor), P(_Tensor), P(_State), P(_Local), P(_ConvState),
+                                     P(_Tensor), P(_Launch)]
     lib.rlm_state_init.argtypes = [P(_State), P(_Params), P(_Launch)]
     lib.rlm_validate_params.argtypes = [P(_Params)]
     lib.rlm_get_device_status.argtypes = [P(_Launch)]
@@ -101,7 +115,8 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
                                     ctypes.c_int, ctypes.c_int]
         getattr(lib, f).restype = ctypes.c_size_t
     for f in ("rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_decode", "rlm_mix_backward",
-              "rlm_mix_backward_from", "rlm_state_init", "rlm_validate_params", "rlm_get_device_status"):
+              "rlm_mix_backward_from", "rlm_mixer_prefill", "rlm_mixer_decode", "rlm_state_init",
+              "rlm_validate_params", "rlm_get_device_status"):
         getattr(lib, f).restype = ctypes.c_int
     lib.rlm_status_string.argtypes = [ctypes.c_int]
     lib.rlm_status_string.restype = ctypes.c_char_p
@@ -178,6 +193,49 @@ class State:
     def _c(self) -> _State:
         B, D, M = self.shape
         return _State(_ptr(self.s, torch.float32, 4), _ptr(self.coef, torch.float32, 3), B, D, M)
+
+
+@dataclass
+class Local:
+    """Local lexical path of Sec. 3.4: depthwise causal kernel conv_w [D][K] (conv_w[d][k]
+    multiplies u_{t-k}) and channel scale [D], both float32 CUDA tensors."""
+    conv_w: torch.Tensor
+    scale: torch.Tensor
+
+    @property
+    def K(self) -> int:
+        return int(self.conv_w.shape[1])
+
+    @classmethod
+    def from_arrays(cls, conv_w, scale, device="cuda"):
+        t = lambda a: torch.as_tensor(a, dtype=torch.float32).contiguous().to(device)
+        return cls(t(conv_w), t(scale))
+
+    def _c(self) -> _Local:
+        D, K = self.conv_w.shape
+        if K == 0:
+            return _Local(None, None, int(D), 0)
+        return _Local(_ptr(self.conv_w, torch.float32, 2), _ptr(self.scale, torch.float32, 1), int(D), int(K))
+
+
+@dataclass
+class ConvState:
+    """Drive history of the local path: u [B][K-1][D] in the field's dtype, oldest first."""
+    u: torch.Tensor
+
+    @property
+    def K(self) -> int:
+        return int(self.u.shape[1]) + 1
+
+    @classmethod
+    def empty(cls, B: int, D: int, K: int, dtype=torch.bfloat16, device="cuda"):
+        return cls(torch.empty(B, max(K - 1, 0), D, dtype=dtype, device=device))
+
+    def _c(self) -> _ConvState:
+        if self.u.dtype not in _DT or not self.u.is_cuda or not self.u.is_contiguous() or self.u.dim() != 3:
+            raise ValueError("ConvState.u must be a contiguous CUDA [B][K-1][D] float32 or bfloat16 tensor")
+        B, K1, D = self.u.shape
+        return _ConvState(self.u.data_ptr() if K1 > 0 else None, _DT[self.u.dtype], int(B), int(D), int(K1) + 1)
 
 
 # --------------------------------------------------------------- marshalling
@@ -376,3 +434,37 @@ def rlm_validate_params(params: Params) -> None:
 def rlm_get_device_status(stream=None) -> int:
     """Synchronise the stream and return (and clear) the device status word."""
     return load_library().rlm_get_device_status(ctypes.byref(_launch(stream, None)))
+
+
+def rlm_mixer_prefill(x: torch.Tensor, g: torch.Tensor | None, params: Params, local: Local | None,
+                      z: torch.Tensor, state_in: State | None = None, conv_in: ConvState | None = None,
+                      state_out: State | None = None, conv_out: ConvState | None = None,
+                      workspace: torch.Tensor | None = None, stream=None) -> None:
+    """Mixer output of Sec. 3.4 over a sequence: z = sigmoid(g) * y + s * (w * x), y the
+    resonant mixing of x from ``state_in``; the local path reads its drives before
+    token 0 from ``conv_in``.  ``state_out`` / ``conv_out`` receive the terminal
+    state and drive history (each may be its input, for in-place continuation)."""
+    lib = load_library()
+    xt, zt = _field(x), _field(z)
+    gt = _field(g) if g is not None else None
+    if workspace is None:
+        workspace = _workspace(lib.rlm_prefill_workspace_size(xt.B, xt.L, xt.D, params.M, xt.dtype),
+                               x.device)
+    ref = lambda c: ctypes.byref(c) if c is not None else None
+    opt = lambda o: ref(o._c()) if o is not None else None
+    _check(lib.rlm_mixer_prefill(ctypes.byref(xt), ref(gt), ctypes.byref(params._c()), opt(local), opt(state_in),
+                                 opt(conv_in), ctypes.byref(zt), opt(state_out), opt(conv_out),
+                                 ctypes.byref(_launch(stream, workspace))), "rlm_mixer_prefill")
+
+
+def rlm_mixer_decode(x_t: torch.Tensor, g_t: torch.Tensor | None, state: State, local: Local | None,
+                     conv: ConvState | None, z_t: torch.Tensor, stream=None) -> None:
+    """One mixer decode step: recurrence, gate and local path in one kernel; the state
+    and the drive history advance in place."""
+    lib = load_library()
+    xt, zt = _field(x_t), _field(z_t)
+    gt = _field(g_t) if g_t is not None else None
+    ref = lambda c: ctypes.byref(c) if c is not None else None
+    opt = lambda o: ref(o._c()) if o is not None else None
+    _check(lib.rlm_mixer_decode(ctypes.byref(xt), ref(gt), ctypes.byref(state._c()), opt(local), opt(conv),
+                                ctypes.byref(zt), ctypes.byref(_launch(stream, None))), "rlm_mixer_decode")

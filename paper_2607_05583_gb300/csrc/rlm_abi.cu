@@ -151,6 +151,85 @@ rlm_status check_state_s(const rlm_state *st, int64_t B, int64_t D, int M, const
     return RLM_OK;
 }
 
+// state_in / state_out of a prefill writing the field y: shapes, and no partial
+// overlap (state_out may be state_in itself).
+rlm_status check_prefill_states(const rlm_tensor *x, const rlm_tensor *y, const rlm_params *p,
+                                const rlm_state *state_in, const rlm_state *state_out) {
+    rlm_status s;
+    if (state_out && (s = check_state(state_out, x->B, x->D, p->M, "state_out")) != RLM_OK) return s;
+    const size_t sbytes = (size_t)x->B * x->D * p->M * 8;
+    if (state_in) {
+        if (!state_in->s || !aligned16(state_in->s))
+            return fail(RLM_ERR_INVALID_ARG, "state_in->s is NULL or not 16-byte aligned");
+        if (state_in->B != x->B || state_in->D != x->D || state_in->M != p->M)
+            return fail(RLM_ERR_INVALID_ARG, "state_in is [B=%d][D=%d][M=%d], expected [%lld][%lld][%d]",
+                        state_in->B, state_in->D, state_in->M, (long long)x->B, (long long)x->D, p->M);
+        if (overlap(state_in->s, sbytes, y->ptr, tensor_bytes(y)))
+            return fail(RLM_ERR_INVALID_ARG, "state_in overlaps the output field");
+        if (state_out && state_out->s != state_in->s && overlap(state_in->s, sbytes, state_out->s, sbytes))
+            return fail(RLM_ERR_INVALID_ARG, "state_in and state_out overlap without being the same buffer");
+    }
+    return RLM_OK;
+}
+
+// The prefill path for a problem: the tcgen05 prefill (bf16, M = 16), its
+// time-reversed form (other bf16 M <= 32), else the SIMT scan.
+enum class PrefillPath { kTc, kRev, kSimt };
+
+PrefillPath prefill_path(const rlm_tensor *x, int M) {
+    const int D = (int)x->D;
+    if (tc_prefill_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kTc;
+    if (tc_prefill_rev_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kRev;
+    return PrefillPath::kSimt;
+}
+
+// Launches the mixing of x into y on the chosen path (arguments already checked).
+cudaError_t launch_prefill(PrefillPath path, const rlm_tensor *x, const rlm_params *p, const float *sin,
+                           void *y, float *so, float *co, const rlm_launch *ln) {
+    cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
+    const int D = (int)x->D, M = p->M;
+    switch (path) {
+        case PrefillPath::kTc:
+            return tc_prefill(x->ptr, y, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so, co,
+                              ln->workspace, st);
+        case PrefillPath::kRev:
+            return tc_prefill_rev(x->ptr, y, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so, co,
+                                  ln->workspace, st);
+        default:
+            return simt_prefill(x->ptr, y, x->dtype, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase,
+                                sin, so, co, ln->workspace, st);
+    }
+}
+
+// The mixer's local path: K in range, D matching, weights present when K > 0.
+rlm_status check_local(const rlm_local *lc, int64_t D, int *K) {
+    *K = 0;
+    if (!lc) return RLM_OK;
+    if (lc->K < 0 || lc->K > RLM_MAX_LOCAL_K)
+        return fail(RLM_ERR_INVALID_ARG, "local->K=%d outside 0..%d", lc->K, RLM_MAX_LOCAL_K);
+    if (lc->K == 0) return RLM_OK;
+    if (lc->D != D) return fail(RLM_ERR_INVALID_ARG, "local->D=%d does not match D=%lld", lc->D, (long long)D);
+    if (!lc->conv_w || !lc->scale || !aligned16(lc->conv_w) || !aligned16(lc->scale))
+        return fail(RLM_ERR_INVALID_ARG, "local->conv_w or local->scale is NULL or not 16-byte aligned");
+    *K = lc->K;
+    return RLM_OK;
+}
+
+size_t conv_bytes(int64_t B, int64_t D, int K, rlm_dtype dt) {
+    return K < 2 ? 0 : (size_t)B * (size_t)(K - 1) * (size_t)D * elem_size(dt);
+}
+
+// A drive-history argument (only checked when the local path has K >= 2).
+rlm_status check_conv(const rlm_conv_state *c, int64_t B, int64_t D, int K, rlm_dtype dt, const char *name) {
+    if (!c || K < 2) return RLM_OK;
+    if (!c->u || !aligned16(c->u)) return fail(RLM_ERR_INVALID_ARG, "%s->u is NULL or not 16-byte aligned", name);
+    if (c->B != B || c->D != D || c->K != K || c->dtype != dt)
+        return fail(RLM_ERR_INVALID_ARG, "%s is [B=%lld][K-1=%d][D=%d] of dtype %d, expected [%lld][%d][%lld] of %d",
+                    name, (long long)c->B, c->K - 1, c->D, (int)c->dtype, (long long)B, K - 1, (long long)D,
+                    (int)dt);
+    return RLM_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -202,41 +281,64 @@ rlm_status rlm_mix_prefill_from(const rlm_tensor *x, const rlm_params *p, const 
     if (overlap(x->ptr, tensor_bytes(x), y->ptr, tensor_bytes(y)))
         return fail(RLM_ERR_INVALID_ARG, "x and y overlap");
     if ((s = check_params(p, x->D)) != RLM_OK) return s;
-    if (state_out && (s = check_state(state_out, x->B, x->D, p->M, "state_out")) != RLM_OK) return s;
-    const size_t sbytes = (size_t)x->B * x->D * p->M * 8;
-    if (state_in) {
-        if (!state_in->s || !aligned16(state_in->s))
-            return fail(RLM_ERR_INVALID_ARG, "state_in->s is NULL or not 16-byte aligned");
-        if (state_in->B != x->B || state_in->D != x->D || state_in->M != p->M)
-            return fail(RLM_ERR_INVALID_ARG, "state_in is [B=%d][D=%d][M=%d], expected [%lld][%lld][%d]",
-                        state_in->B, state_in->D, state_in->M, (long long)x->B, (long long)x->D, p->M);
-        if (overlap(state_in->s, sbytes, y->ptr, tensor_bytes(y)))
-            return fail(RLM_ERR_INVALID_ARG, "state_in overlaps y");
-        if (state_out && state_out->s != state_in->s && overlap(state_in->s, sbytes, state_out->s, sbytes))
-            return fail(RLM_ERR_INVALID_ARG, "state_in and state_out overlap without being the same buffer");
-    }
-    const float *sin = state_in ? state_in->s : nullptr;
-    const int D = (int)x->D, M = p->M;
-    const bool tc = tc_prefill_supported(x->B, x->L, D, M, x->dtype);
-    const bool rev = !tc && tc_prefill_rev_supported(x->B, x->L, D, M, x->dtype);
-    if (!tc && !rev && simt_chunks(x->B, x->L, D) > 65535)
+    if ((s = check_prefill_states(x, y, p, state_in, state_out)) != RLM_OK) return s;
+    const PrefillPath path = prefill_path(x, p->M);
+    if (path == PrefillPath::kSimt && simt_chunks(x->B, x->L, (int)x->D) > 65535)
         return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
-    const size_t need = rlm_prefill_workspace_size(x->B, x->L, D, M, x->dtype);
+    const size_t need = rlm_prefill_workspace_size(x->B, x->L, (int)x->D, p->M, x->dtype);
+    if ((s = check_workspace(ln, need)) != RLM_OK) return s;
+    cudaError_t e = launch_prefill(path, x, p, state_in ? state_in->s : nullptr, y->ptr,
+                                   state_out ? state_out->s : nullptr, state_out ? state_out->coef : nullptr, ln);
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_prefill launch");
+    return RLM_OK;
+}
+
+rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm_params *p, const rlm_local *local,
+                             const rlm_state *state_in, const rlm_conv_state *conv_in, rlm_tensor *z,
+                             rlm_state *state_out, rlm_conv_state *conv_out, const rlm_launch *ln) {
+    rlm_status s;
+    if ((s = check_tensor(x, "x")) != RLM_OK) return s;
+    if ((s = check_tensor(z, "z")) != RLM_OK) return s;
+    if (!same_shape(x, z)) return fail(RLM_ERR_INVALID_ARG, "z must have x's shape and dtype");
+    if (g) {
+        if ((s = check_tensor(g, "g")) != RLM_OK) return s;
+        if (!same_shape(x, g)) return fail(RLM_ERR_INVALID_ARG, "g must have x's shape and dtype");
+        if (overlap(g->ptr, tensor_bytes(g), z->ptr, tensor_bytes(z)))
+            return fail(RLM_ERR_INVALID_ARG, "g and z overlap");
+    }
+    if (overlap(x->ptr, tensor_bytes(x), z->ptr, tensor_bytes(z)))
+        return fail(RLM_ERR_INVALID_ARG, "x and z overlap");
+    if ((s = check_params(p, x->D)) != RLM_OK) return s;
+    if ((s = check_prefill_states(x, z, p, state_in, state_out)) != RLM_OK) return s;
+    int K = 0;
+    if ((s = check_local(local, x->D, &K)) != RLM_OK) return s;
+    if ((s = check_conv(conv_in, x->B, x->D, K, x->dtype, "conv_in")) != RLM_OK) return s;
+    if ((s = check_conv(conv_out, x->B, x->D, K, x->dtype, "conv_out")) != RLM_OK) return s;
+    const size_t cb = conv_bytes(x->B, x->D, K, x->dtype);
+    const void *hin = (conv_in && K >= 2) ? conv_in->u : nullptr;
+    void *hout = (conv_out && K >= 2) ? conv_out->u : nullptr;
+    if (hin && overlap(hin, cb, z->ptr, tensor_bytes(z)))
+        return fail(RLM_ERR_INVALID_ARG, "conv_in overlaps z");
+    if (hout) {
+        if (overlap(hout, cb, z->ptr, tensor_bytes(z)) || overlap(hout, cb, x->ptr, tensor_bytes(x)) ||
+            (g && overlap(hout, cb, g->ptr, tensor_bytes(g))))
+            return fail(RLM_ERR_INVALID_ARG, "conv_out overlaps x, g or z");
+        if (hin && hin != hout && overlap(hin, cb, hout, cb))
+            return fail(RLM_ERR_INVALID_ARG, "conv_in and conv_out overlap without being the same buffer");
+    }
+    const PrefillPath path = prefill_path(x, p->M);
+    if (path == PrefillPath::kSimt && simt_chunks(x->B, x->L, (int)x->D) > 65535)
+        return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
+    const size_t need = rlm_prefill_workspace_size(x->B, x->L, (int)x->D, p->M, x->dtype);
     if ((s = check_workspace(ln, need)) != RLM_OK) return s;
     cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
-    float *so = state_out ? state_out->s : nullptr;
-    float *co = state_out ? state_out->coef : nullptr;
-    cudaError_t e;
-    if (tc)
-        e = tc_prefill(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so,
-                       co, ln->workspace, st);
-    else if (rev)
-        e = tc_prefill_rev(x->ptr, y->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so,
-                           co, ln->workspace, st);
-    else
-        e = simt_prefill(x->ptr, y->ptr, x->dtype, x->B, x->L, D, M, p->decay, p->freq, p->amp,
-                         p->phase, sin, so, co, ln->workspace, st);
-    if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_prefill launch");
+    cudaError_t e = launch_prefill(path, x, p, state_in ? state_in->s : nullptr, z->ptr,
+                                   state_out ? state_out->s : nullptr, state_out ? state_out->coef : nullptr, ln);
+    if (e == cudaSuccess && (g || K > 0))
+        e = mixer_epilogue(x->ptr, g ? g->ptr : nullptr, z->ptr, hin, K > 0 ? local->conv_w : nullptr,
+                           K > 0 ? local->scale : nullptr, x->dtype, x->B, x->L, (int)x->D, K, st);
+    if (e == cudaSuccess && hout) e = conv_tail(x->ptr, hin, hout, x->dtype, x->B, x->L, (int)x->D, K, st);
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_mixer_prefill launch");
     return RLM_OK;
 }
 
@@ -261,6 +363,48 @@ rlm_status rlm_mix_decode(const rlm_tensor *x_t, rlm_state *state, rlm_tensor *y
     cudaError_t e = decode_step(x_t->ptr, y_t->ptr, x_t->dtype, (int)x_t->B, (int)x_t->D, state->M,
                                 state->s, state->coef, static_cast<cudaStream_t>(ln->stream));
     if (e != cudaSuccess) return cuda_fail(e, "rlm_mix_decode launch");
+    return RLM_OK;
+}
+
+rlm_status rlm_mixer_decode(const rlm_tensor *x_t, const rlm_tensor *g_t, rlm_state *state, const rlm_local *local,
+                            rlm_conv_state *conv, rlm_tensor *z_t, const rlm_launch *ln) {
+    rlm_status s;
+    if ((s = check_tensor(x_t, "x_t")) != RLM_OK) return s;
+    if ((s = check_tensor(z_t, "z_t")) != RLM_OK) return s;
+    if (x_t->L != 1) return fail(RLM_ERR_INVALID_ARG, "x_t must have L == 1 (got %lld)", (long long)x_t->L);
+    if (!same_shape(x_t, z_t)) return fail(RLM_ERR_INVALID_ARG, "z_t must have x_t's shape and dtype");
+    if (overlap(x_t->ptr, tensor_bytes(x_t), z_t->ptr, tensor_bytes(z_t)))
+        return fail(RLM_ERR_INVALID_ARG, "x_t and z_t overlap");
+    if (g_t) {
+        if ((s = check_tensor(g_t, "g_t")) != RLM_OK) return s;
+        if (!same_shape(x_t, g_t)) return fail(RLM_ERR_INVALID_ARG, "g_t must have x_t's shape and dtype");
+        if (overlap(g_t->ptr, tensor_bytes(g_t), z_t->ptr, tensor_bytes(z_t)))
+            return fail(RLM_ERR_INVALID_ARG, "g_t and z_t overlap");
+    }
+    if (!state) return fail(RLM_ERR_INVALID_ARG, "state is NULL");
+    if (state->M < 1 || state->M > kMaxModes)
+        return fail(RLM_ERR_INVALID_ARG, "state->M=%d outside 1..%d", state->M, kMaxModes);
+    if ((s = check_state(state, x_t->B, x_t->D, state->M, "state")) != RLM_OK) return s;
+    if (!ln) return fail(RLM_ERR_INVALID_ARG, "launch is NULL");
+    const size_t sbytes = (size_t)state->B * state->D * state->M * 8;
+    if (overlap(state->s, sbytes, z_t->ptr, tensor_bytes(z_t)) || overlap(state->s, sbytes, x_t->ptr, tensor_bytes(x_t)) ||
+        (g_t && overlap(state->s, sbytes, g_t->ptr, tensor_bytes(g_t))))
+        return fail(RLM_ERR_INVALID_ARG, "state overlaps x_t, g_t or z_t");
+    int K = 0;
+    if ((s = check_local(local, x_t->D, &K)) != RLM_OK) return s;
+    if (K >= 2 && !conv) return fail(RLM_ERR_INVALID_ARG, "conv is NULL but the local path has K=%d", K);
+    if ((s = check_conv(conv, x_t->B, x_t->D, K, x_t->dtype, "conv")) != RLM_OK) return s;
+    if (K >= 2) {
+        const size_t cb = conv_bytes(x_t->B, x_t->D, K, x_t->dtype);
+        if (overlap(conv->u, cb, z_t->ptr, tensor_bytes(z_t)) || overlap(conv->u, cb, x_t->ptr, tensor_bytes(x_t)) ||
+            (g_t && overlap(conv->u, cb, g_t->ptr, tensor_bytes(g_t))) || overlap(conv->u, cb, state->s, sbytes))
+            return fail(RLM_ERR_INVALID_ARG, "conv overlaps x_t, g_t, z_t or the state");
+    }
+    cudaError_t e = mixer_decode_step(x_t->ptr, g_t ? g_t->ptr : nullptr, z_t->ptr, x_t->dtype, (int)x_t->B,
+                                      (int)x_t->D, state->M, state->s, state->coef, K >= 2 ? conv->u : nullptr,
+                                      K > 0 ? local->conv_w : nullptr, K > 0 ? local->scale : nullptr, K,
+                                      static_cast<cudaStream_t>(ln->stream));
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_mixer_decode launch");
     return RLM_OK;
 }
 

@@ -73,6 +73,22 @@ cudaError_t tc_prefill_rev(const void *x, void *y, int64_t B, int64_t L, int D, 
 // ---- decode (rlm_decode.cu) -----------------------------------------------
 cudaError_t decode_step(const void *x_t, void *y_t, rlm_dtype dt, int B, int D, int M,
                         float *s, const float *coef, cudaStream_t st);
+// The mixer step (Sec. 3.4) fused with the decode step: g_t nullable (no gate);
+// hist [B][K-1][D] drive history shifted in place (unused when K <= 1).
+cudaError_t mixer_decode_step(const void *x_t, const void *g_t, void *z_t, rlm_dtype dt, int B, int D, int M,
+                              float *s, const float *coef, void *hist, const float *conv_w, const float *scale,
+                              int K, cudaStream_t st);
+
+// ---- mixer epilogue for the unfused prefill paths (rlm_mixer.cu) ------------
+// z <- sigma(g) z + s * (w * u) in place (g nullable; K = 0: no local path), the
+// drives before token 0 from hist ([B][K-1][D], nullable = zeros).
+cudaError_t mixer_epilogue(const void *x, const void *g, void *z, const void *hist, const float *conv_w,
+                           const float *scale, rlm_dtype dt, int64_t B, int64_t L, int D, int K,
+                           cudaStream_t st);
+// out = the last K-1 drives of hist || x (out may alias hist; no-op for K < 2).
+cudaError_t conv_tail(const void *x, const void *hist, void *out, rlm_dtype dt, int64_t B, int64_t L, int D,
+                      int K, cudaStream_t st);
+
 cudaError_t state_init(float *s, float *coef, int B, int D, int M, const float *decay,
                        const float *freq, const float *amp, const float *phase,
                        cudaStream_t st);

@@ -32,7 +32,7 @@ def _declared_entry_points():
 def test_header_declares_the_boundary():
     names = _declared_entry_points()
     for want in ("rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_decode", "rlm_mix_backward",
-                 "rlm_mix_backward_from", "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
+                 "rlm_mix_backward_from", "rlm_mixer_prefill", "rlm_mixer_decode", "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
                  "rlm_state_init", "rlm_validate_params", "rlm_get_device_status",
                  "rlm_status_string", "rlm_last_error"):
         assert want in names
@@ -209,6 +209,49 @@ def test_backward_from_rejects_bad_state_arguments_on_host(lib):
     assert call(None, None, state(dx.ptr)) == rlm.RLM_ERR_INVALID_ARG      # d_state_in overlaps dx
     assert call(state(sbase), None, state(sbase)) == rlm.RLM_ERR_INVALID_ARG  # ... the state_in
     assert call(None, None, state(g.decay)) == rlm.RLM_ERR_INVALID_ARG     # ... a gradient
+
+
+RLM_MAX_K = 8
+
+
+def test_mixer_rejects_bad_arguments_on_host(lib):
+    B, L, D, M, K = 2, 100, 16, 4, 4
+    x, z = _t(FAKE, B, L, D), _t(FAKE + (1 << 30), B, L, D)
+    g = _t(FAKE + (1 << 31), B, L, D)
+    p = _p(D, M)
+    ln = _launch(FAKE + (1 << 34), 1 << 40)
+    wbase = FAKE + (1 << 37)
+    cbase = FAKE + (1 << 38)
+    ref = lambda v: ctypes.byref(v) if v is not None else None
+
+    def local(k=K, d=D, w=wbase):
+        return rlm._Local(w, w + 4096, d, k)
+
+    def conv(ptr=cbase, b=B, d=D, k=K, dt=rlm.RLM_BF16):
+        return rlm._ConvState(ptr, dt, b, d, k)
+
+    def call(gt=g, lc=None, cin=None, zt=z, cout=None):
+        return lib.rlm_mixer_prefill(ctypes.byref(x), ref(gt), ctypes.byref(p), ref(lc), None, ref(cin),
+                                     ctypes.byref(zt), None, ref(cout), ctypes.byref(ln))
+
+    assert call(lc=local(k=RLM_MAX_K + 1)) == rlm.RLM_ERR_INVALID_ARG          # K too large
+    assert call(lc=local(k=-1)) == rlm.RLM_ERR_INVALID_ARG
+    assert call(lc=local(d=D + 8)) == rlm.RLM_ERR_INVALID_ARG                  # D mismatch
+    assert call(lc=local(w=0)) == rlm.RLM_ERR_INVALID_ARG                      # NULL weights
+    assert call(gt=_t(FAKE + (1 << 31), B, L + 1, D)) == rlm.RLM_ERR_INVALID_ARG   # g shape
+    assert call(gt=_t(z.ptr, B, L, D)) == rlm.RLM_ERR_INVALID_ARG               # g overlaps z
+    assert call(lc=local(), cin=conv(k=K + 1)) == rlm.RLM_ERR_INVALID_ARG       # history shape
+    assert call(lc=local(), cin=conv(dt=rlm.RLM_F32)) == rlm.RLM_ERR_INVALID_ARG  # history dtype
+    assert call(lc=local(), cin=conv(ptr=cbase + 8)) == rlm.RLM_ERR_INVALID_ARG   # misaligned
+    assert call(lc=local(), cin=conv(), cout=conv(ptr=cbase + 64)) == rlm.RLM_ERR_INVALID_ARG  # partial overlap
+    assert call(lc=local(), cout=conv(ptr=z.ptr)) == rlm.RLM_ERR_INVALID_ARG     # history overlaps z
+    st = rlm._State(FAKE + (1 << 33), FAKE + (1 << 33) + (1 << 20), B, D, M)
+    x1, z1 = _t(FAKE, B, 1, D), _t(FAKE + (1 << 30), B, 1, D)
+    dec = lambda lc, cv: lib.rlm_mixer_decode(ctypes.byref(x1), None, ctypes.byref(st), ref(lc), ref(cv),
+                                              ctypes.byref(z1), ctypes.byref(ln))
+    assert dec(local(), None) == rlm.RLM_ERR_INVALID_ARG                         # history required for K >= 2
+    assert dec(local(), conv(b=B + 1)) == rlm.RLM_ERR_INVALID_ARG
+    assert dec(local(), conv(ptr=st.s)) == rlm.RLM_ERR_INVALID_ARG               # history overlaps the state
 
 
 @pytest.mark.parametrize("rows,D,sb,ctas", [

@@ -1,0 +1,196 @@
+"""GPU parity of the mixer wrapper (Sec. 3.4: gate and local path around the
+operator) through the C ABI against the fp64 oracle, on every prefill path and
+in decode."""
+import numpy as np
+import pytest
+
+import oracle
+from synth import make_inputs, make_mixer_inputs
+from tests._util import TOL, assert_close, to_dev, to_np
+
+torch = pytest.importorskip("torch")
+rlm = pytest.importorskip("paper_2607_05583_gb300")
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2607_05583_gb300 import build
+    build.build()
+    rlm.load_library()
+    yield
+    torch.cuda.synchronize()
+    assert rlm.rlm_get_device_status() == rlm.RLM_OK
+
+
+def _state_from(B, D, M, s_np):
+    st = rlm.State.empty(B, D, M)
+    st.s.copy_(torch.from_numpy(np.stack([s_np.real, s_np.imag], -1).astype(np.float32)))
+    return st
+
+
+def _run_prefill(inp, mx, with_g=True, with_hist=True, s_in=None):
+    dt = inp.dtype
+    x = to_dev(inp.x, dt)
+    g = to_dev(mx.g, dt) if with_g else None
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale) if mx.K > 0 else None
+    cin = rlm.ConvState(to_dev(mx.conv_in, dt)) if with_hist and mx.K > 0 else None
+    cout = rlm.ConvState.empty(inp.B, inp.D, max(mx.K, 1), dtype=x.dtype) if mx.K > 0 else None
+    si = _state_from(inp.B, inp.D, inp.M, s_in) if s_in is not None else None
+    so = rlm.State.empty(inp.B, inp.D, inp.M)
+    z = torch.empty_like(x)
+    rlm.rlm_mixer_prefill(x, g, p, local, z, state_in=si, conv_in=cin, state_out=so, conv_out=cout)
+    torch.cuda.synchronize()
+    return z, so, cout
+
+
+def _check_prefill(inp, mx, z, so, cout, with_g, with_hist, s_in=None):
+    tol = TOL[inp.dtype]
+    zr, sr, tr = oracle.mixer_prefill(inp.x, mx.g if with_g else None, *inp.params(), mx.conv_w, mx.scale,
+                                      state_in=s_in, conv_in=mx.conv_in if with_hist else None)
+    assert_close(to_np(z), zr, tol, "z")
+    s = so.complex().cpu().numpy()
+    assert_close(s.real, sr.real, tol, "state re")
+    assert_close(s.imag, sr.imag, tol, "state im")
+    if cout is not None and mx.K > 1:
+        np.testing.assert_array_equal(to_np(cout.u), tr)   # the history is a copy: bit-exact
+
+
+@pytest.mark.parametrize("B,L,D,M,K,dtype,with_g,with_hist", [
+    (2, 2 * 2048 + 77, 64, 16, 4, "bf16", True, True),    # tcgen05 prefill (M = 16), ragged tail
+    (1, 3000, 16, 16, 8, "bf16", True, False),             # ... segmented sequence, K = 8, zero history
+    (3, 1000, 32, 16, 1, "bf16", False, False),            # ... no gate, pointwise local path
+    (2, 1000, 8, 16, 0, "bf16", True, False),              # ... gate only
+    (2, 1000, 8, 32, 4, "bf16", True, True),               # time-reversed tcgen05 prefill
+    (2, 1000, 16, 7, 3, "f32", True, True),                # SIMT, fp32
+    (1, 500, 8, 40, 2, "bf16", True, True),                # SIMT, bf16 with M > 32
+    (1, 5, 8, 16, 8, "bf16", True, True),                  # L shorter than the history
+])
+def test_mixer_prefill_matches_oracle(B, L, D, M, K, dtype, with_g, with_hist):
+    inp = make_inputs(B, L, D, M, dtype, seed=L + K)
+    mx = make_mixer_inputs(inp, K, seed=L + K)
+    z, so, cout = _run_prefill(inp, mx, with_g, with_hist)
+    _check_prefill(inp, mx, z, so, cout, with_g, with_hist)
+
+
+def test_mixer_prefill_from_state_matches_oracle():
+    inp = make_inputs(2, 3001, 64, 16, "bf16", seed=5)
+    mx = make_mixer_inputs(inp, 4, seed=5)
+    pre = make_inputs(2, 300, 64, 16, "bf16", seed=6)
+    _, s_in = oracle.rec_prefill(pre.x, *inp.params())
+    z, so, cout = _run_prefill(inp, mx, True, True, s_in=s_in)
+    _check_prefill(inp, mx, z, so, cout, True, True, s_in=s_in)
+
+
+def test_mixer_without_gate_or_local_path_is_the_mixing():
+    inp = make_inputs(2, 3000, 64, 16, "bf16", seed=9)
+    x = to_dev(inp.x, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    y, z = torch.empty_like(x), torch.empty_like(x)
+    rlm.rlm_mix_prefill(x, p, y)
+    rlm.rlm_mixer_prefill(x, None, p, None, z)
+    torch.cuda.synchronize()
+    assert torch.equal(y, z)
+
+
+@pytest.mark.parametrize("M", [16, 32])
+def test_mixer_split_prefill_in_place_equals_whole(M):
+    """Prefill of x1, then of x2 continuing from the state and drive history, both
+    updated in place, equals one prefill of x1 || x2."""
+    B, L, D, K, cut = 2, 5000, 64, 4, 2345
+    inp = make_inputs(B, L, D, M, "bf16", seed=21)
+    mx = make_mixer_inputs(inp, K, seed=21)
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    st = rlm.State.empty(B, D, M)
+    cs = rlm.ConvState.empty(B, D, K, dtype=torch.bfloat16)
+    x1, x2 = x[:, :cut].contiguous(), x[:, cut:].contiguous()
+    g1, g2 = g[:, :cut].contiguous(), g[:, cut:].contiguous()
+    z1, z2 = torch.empty_like(x1), torch.empty_like(x2)
+    rlm.rlm_mixer_prefill(x1, g1, p, local, z1, state_out=st, conv_out=cs)
+    rlm.rlm_mixer_prefill(x2, g2, p, local, z2, state_in=st, conv_in=cs, state_out=st, conv_out=cs)
+    torch.cuda.synchronize()
+    zr, sr, tr = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), mx.conv_w, mx.scale)
+    assert_close(to_np(torch.cat([z1, z2], 1)), zr, TOL["bf16"], "z")
+    s = st.complex().cpu().numpy()
+    assert_close(s.real, sr.real, TOL["bf16"], "state re")
+    np.testing.assert_array_equal(to_np(cs.u), tr)
+
+
+@pytest.mark.parametrize("dtype,M,K", [("bf16", 16, 4), ("f32", 7, 3), ("bf16", 40, 8), ("bf16", 16, 1)])
+def test_mixer_decode_continues_the_prefill(dtype, M, K):
+    """Prefill of 300 tokens then 40 fused mixer decode steps reproduce the oracle's
+    mixer output over all 340 tokens, and the final state and history."""
+    B, D, L0, T = 3, 32, 300, 40
+    inp = make_inputs(B, L0 + T, D, M, dtype, seed=M + K)
+    mx = make_mixer_inputs(inp, K, seed=M + K)
+    x, g = to_dev(inp.x, dtype), to_dev(mx.g, dtype)
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    st = rlm.State.empty(B, D, M)
+    cs = rlm.ConvState.empty(B, D, K, dtype=x.dtype)
+    z0 = torch.empty_like(x[:, :L0])
+    rlm.rlm_mixer_prefill(x[:, :L0].contiguous(), g[:, :L0].contiguous(), p, local, z0, state_out=st, conv_out=cs)
+    zs = []
+    for t in range(L0, L0 + T):
+        zt = torch.empty_like(x[:, t])
+        rlm.rlm_mixer_decode(x[:, t].contiguous(), g[:, t].contiguous(), st, local, cs, zt)
+        zs.append(zt)
+    torch.cuda.synchronize()
+    zr, sr, tr = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), mx.conv_w, mx.scale)
+    assert_close(to_np(z0), zr[:, :L0], TOL[dtype], "prefill z")
+    assert_close(to_np(torch.stack(zs, 1)), zr[:, L0:], TOL[dtype], "decode z")
+    s = st.complex().cpu().numpy()
+    assert_close(s.real, sr.real, TOL[dtype], "state re")
+    if K > 1:
+        np.testing.assert_array_equal(to_np(cs.u), tr)
+
+
+def test_mixer_decode_without_gate_or_local_path_is_the_decode():
+    inp = make_inputs(4, 1, 64, 16, "bf16", seed=2)
+    x = to_dev(inp.x[:, 0], "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    s1, s2 = rlm.State.empty(4, 64, 16), rlm.State.empty(4, 64, 16)
+    rlm.rlm_state_init(s1, p)
+    rlm.rlm_state_init(s2, p)
+    y, z = torch.empty_like(x), torch.empty_like(x)
+    for _ in range(3):
+        rlm.rlm_mix_decode(x, s1, y)
+        rlm.rlm_mixer_decode(x, None, s2, None, None, z)
+    torch.cuda.synchronize()
+    assert torch.equal(y, z) and torch.equal(s1.s, s2.s)
+
+
+def test_mixer_prefill_is_causal_bit_exact():
+    """Changing x and g from token t0 on leaves z before t0 bit-identical."""
+    inp = make_inputs(2, 4100, 64, 16, "bf16", seed=4)
+    mx = make_mixer_inputs(inp, 4, seed=4)
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    z1, z2 = torch.empty_like(x), torch.empty_like(x)
+    rlm.rlm_mixer_prefill(x, g, p, local, z1)
+    t0 = 2049
+    x2, g2 = x.clone(), g.clone()
+    x2[:, t0:] = torch.randn_like(x2[:, t0:])
+    g2[:, t0:] = torch.randn_like(g2[:, t0:])
+    rlm.rlm_mixer_prefill(x2, g2, p, local, z2)
+    torch.cuda.synchronize()
+    assert torch.equal(z1[:, :t0], z2[:, :t0])
+    assert not torch.equal(z1[:, t0:], z2[:, t0:])
+
+
+def test_mixer_prefill_long_context_sampled():
+    """The long-context workload shape (B=4, L=32768, D=256, M=16, K=4, bf16) on
+    sampled channels against the oracle."""
+    inp = make_inputs(4, 32768, 256, 16, "bf16", seed=0)
+    mx = make_mixer_inputs(inp, 4, seed=0)
+    z, so, cout = _run_prefill(inp, mx, True, True)
+    ch = np.array([0, 7, 8, 129, 255])
+    zr, sr, tr = oracle.mixer_prefill(inp.x[:, :, ch], mx.g[:, :, ch], inp.decay[ch], inp.freq[ch], inp.amp[ch],
+                                      inp.phase[ch], mx.conv_w[ch], mx.scale[ch], conv_in=mx.conv_in[:, :, ch])
+    assert_close(to_np(z)[:, :, ch], zr, TOL["bf16"], "z")
+    np.testing.assert_array_equal(to_np(cout.u)[:, :, ch], tr)
