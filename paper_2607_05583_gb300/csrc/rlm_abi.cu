@@ -191,7 +191,7 @@ cudaError_t launch_prefill(PrefillPath path, const rlm_tensor *x, const rlm_para
     switch (path) {
         case PrefillPath::kTc:
             return tc_prefill(x->ptr, y, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so, co,
-                              ln->workspace, st);
+                              nullptr, ln->workspace, st);
         case PrefillPath::kRev:
             return tc_prefill_rev(x->ptr, y, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so, co,
                                   ln->workspace, st);
@@ -332,9 +332,18 @@ rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm
     const size_t need = rlm_prefill_workspace_size(x->B, x->L, (int)x->D, p->M, x->dtype);
     if ((s = check_workspace(ln, need)) != RLM_OK) return s;
     cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
-    cudaError_t e = launch_prefill(path, x, p, state_in ? state_in->s : nullptr, z->ptr,
-                                   state_out ? state_out->s : nullptr, state_out ? state_out->coef : nullptr, ln);
-    if (e == cudaSuccess && (g || K > 0))
+    const bool fused = (g || K > 0) && path == PrefillPath::kTc && tc_mixer_fused(x->B, x->L, (int)x->D, p->M, x->dtype);
+    cudaError_t e;
+    if (fused) {
+        const TcMix mix{g ? g->ptr : nullptr, hin, K > 0 ? local->conv_w : nullptr, K > 0 ? local->scale : nullptr, K};
+        e = tc_prefill(x->ptr, z->ptr, x->B, x->L, (int)x->D, p->M, p->decay, p->freq, p->amp, p->phase,
+                       state_in ? state_in->s : nullptr, state_out ? state_out->s : nullptr,
+                       state_out ? state_out->coef : nullptr, &mix, ln->workspace, st);
+    } else {
+        e = launch_prefill(path, x, p, state_in ? state_in->s : nullptr, z->ptr, state_out ? state_out->s : nullptr,
+                           state_out ? state_out->coef : nullptr, ln);
+    }
+    if (e == cudaSuccess && !fused && (g || K > 0))
         e = mixer_epilogue(x->ptr, g ? g->ptr : nullptr, z->ptr, hin, K > 0 ? local->conv_w : nullptr,
                            K > 0 ? local->scale : nullptr, x->dtype, x->B, x->L, (int)x->D, K, st);
     if (e == cudaSuccess && hout) e = conv_tail(x->ptr, hin, hout, x->dtype, x->B, x->L, (int)x->D, K, st);

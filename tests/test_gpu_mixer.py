@@ -194,3 +194,101 @@ def test_mixer_prefill_long_context_sampled():
                                       inp.phase[ch], mx.conv_w[ch], mx.scale[ch], conv_in=mx.conv_in[:, :, ch])
     assert_close(to_np(z)[:, :, ch], zr, TOL["bf16"], "z")
     np.testing.assert_array_equal(to_np(cout.u)[:, :, ch], tr)
+
+
+# ---- the fused tcgen05 epilogue (bf16, M = 16, unsegmented: >= 77 channel groups x rows)
+def _launches(fn):
+    before = rlm.rlm_kernels_launched()
+    fn()
+    torch.cuda.synchronize()
+    return rlm.rlm_kernels_launched() - before
+
+
+@pytest.mark.parametrize("B,L,D,K,with_g,with_hist", [
+    (2, 2 * 2048 + 77, 512, 4, True, True),    # ragged, three tiles, token 0 inside tile 0
+    (1, 3 * 2048, 1024, 8, True, True),        # tiles aligned with the sequence, K = 8
+    (2, 2048 + 3, 512, 2, False, True),        # local path only
+    (2, 4000, 512, 0, True, False),            # gate only
+])
+def test_fused_mixer_prefill_matches_oracle(B, L, D, K, with_g, with_hist):
+    inp = make_inputs(B, L, D, 16, "bf16", seed=L + D + K)
+    mx = make_mixer_inputs(inp, K, seed=L + K)
+    out = {}
+
+    def run():
+        out["r"] = _run_prefill(inp, mx, with_g, with_hist)
+
+    n = _launches(run)
+    # one fused prefill launch (+ the history tail when K >= 2); the unfused route
+    # would add an epilogue launch
+    assert n == 1 + (1 if K >= 2 else 0), n
+    z, so, cout = out["r"]
+    _check_prefill(inp, mx, z, so, cout, with_g, with_hist)
+
+
+def test_fused_mixer_prefill_from_state_and_split_in_place():
+    B, L, D, K, cut = 2, 6000, 512, 4, 2345
+    inp = make_inputs(B, L, D, 16, "bf16", seed=77)
+    mx = make_mixer_inputs(inp, K, seed=77)
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    st = rlm.State.empty(B, D, 16)
+    cs = rlm.ConvState(to_dev(mx.conv_in, "bf16"))
+    x1, x2 = x[:, :cut].contiguous(), x[:, cut:].contiguous()
+    g1, g2 = g[:, :cut].contiguous(), g[:, cut:].contiguous()
+    z1, z2 = torch.empty_like(x1), torch.empty_like(x2)
+    rlm.rlm_mixer_prefill(x1, g1, p, local, z1, conv_in=cs, state_out=st, conv_out=cs)
+    n = _launches(lambda: rlm.rlm_mixer_prefill(x2, g2, p, local, z2, state_in=st, conv_in=cs, state_out=st,
+                                                conv_out=cs))
+    assert n == 2
+    zr, sr, tr = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), mx.conv_w, mx.scale, conv_in=mx.conv_in)
+    assert_close(to_np(torch.cat([z1, z2], 1)), zr, TOL["bf16"], "z")
+    s = st.complex().cpu().numpy()
+    assert_close(s.real, sr.real, TOL["bf16"], "state re")
+    assert_close(s.imag, sr.imag, TOL["bf16"], "state im")
+    np.testing.assert_array_equal(to_np(cs.u), tr)
+
+
+def test_fused_mixer_prefill_is_causal_bit_exact():
+    inp = make_inputs(2, 4100, 512, 16, "bf16", seed=14)
+    mx = make_mixer_inputs(inp, 8, seed=14)
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    z1, z2 = torch.empty_like(x), torch.empty_like(x)
+    rlm.rlm_mixer_prefill(x, g, p, local, z1)
+    for t0 in (2048, 2049, 4095):
+        x2, g2 = x.clone(), g.clone()
+        x2[:, t0:] = torch.randn_like(x2[:, t0:])
+        g2[:, t0:] = torch.randn_like(g2[:, t0:])
+        rlm.rlm_mixer_prefill(x2, g2, p, local, z2)
+        torch.cuda.synchronize()
+        assert torch.equal(z1[:, :t0], z2[:, :t0]), t0
+        assert not torch.equal(z1[:, t0:], z2[:, t0:])
+
+
+def test_fused_and_unfused_mixer_agree():
+    """The same problem through the fused epilogue (D = 512) and, channel group by
+    channel group, through the unfused route (each 64-channel slice is segmented):
+    within one bf16 rounding of z."""
+    inp = make_inputs(2, 3000, 512, 16, "bf16", seed=3)
+    mx = make_mixer_inputs(inp, 4, seed=3)
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    hist = to_dev(mx.conv_in, "bf16")
+    zf = torch.empty_like(x)
+    rlm.rlm_mixer_prefill(x, g, p, local, zf, conv_in=rlm.ConvState(hist))
+    zu = torch.empty_like(x)
+    for c0 in range(0, 512, 64):
+        sl = slice(c0, c0 + 64)
+        ps = rlm.Params(*(t[sl].contiguous() for t in (p.decay, p.freq, p.amp, p.phase)))
+        ls = rlm.Local(local.conv_w[sl].contiguous(), local.scale[sl].contiguous())
+        zs = torch.empty_like(x[:, :, sl].contiguous())
+        rlm.rlm_mixer_prefill(x[:, :, sl].contiguous(), g[:, :, sl].contiguous(), ps, ls, zs,
+                              conv_in=rlm.ConvState(hist[:, :, sl].contiguous()))
+        zu[:, :, sl] = zs
+    torch.cuda.synchronize()
+    d = (zf.float() - zu.float()).abs().max().item()
+    assert d <= 2.0 ** -6 * zu.float().abs().max().item(), d
