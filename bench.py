@@ -44,6 +44,7 @@ METRIC = "mix prefill Mtok/s at L=32K (% of roofline); decode tok/s at B=64 (% H
 PREFILL = dict(B=4, L=32768, D=256, M=16)
 DECODE = dict(B=64, L=32768, D=256, M=16, T=4096)
 BACKWARD = dict(B=4, L=32768, D=512, M=32)
+MIXER = dict(B=4, L=32768, D=256, M=16, K=4, decode_B=64, T=4096)
 L2_FLUSH_BYTES = 512 << 20
 
 
@@ -68,6 +69,20 @@ def decode_bytes(B, D, M):
     """Per decode step: state read+write (16 B per (b,d,m)), token in and out
     (bf16, 4 B per (b,d)), coefficients (16 B per (d,m))."""
     return 16 * B * D * M + 4 * B * D + 16 * D * M
+
+
+def mixer_prefill_bytes(B, L, D, M, K):
+    """Algorithmic HBM bytes of one fused mixer prefill (Sec. 3.4): read x and g,
+    write z (bf16, 6 B per token-channel), the state and parameters as for the
+    prefill, the drive history in and out (2 B per (b, k, d)) and the local-path
+    weights (4 B per (d, k) and per d)."""
+    return prefill_bytes(B, L, D, M) + 2 * B * L * D + 2 * 2 * B * (K - 1) * D + 4 * D * (K + 1)
+
+
+def mixer_decode_bytes(B, D, M, K):
+    """Per mixer decode step: the decode step's bytes, the gate (2 B per (b,d)),
+    the drive history read and written (4 B per (b, k, d)) and the weights."""
+    return decode_bytes(B, D, M) + 2 * B * D + 4 * B * (K - 1) * D + 4 * D * (K + 1)
 
 
 def backward_bytes(B, L, D, M):
@@ -301,6 +316,8 @@ def run_ours(args):
     decode = None if args.quick else _bench_decode(rlm, torch, dev, hbm_peak)
     # ---------------- backward
     backward = None if args.quick else _bench_backward(rlm, torch, dev, hbm_peak, args)
+    # ---------------- mixer wrapper (gate + local path, fused)
+    mixer = None if args.quick else _bench_mixer(rlm, torch, dev, hbm_peak, flush, ms)
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu:
@@ -318,7 +335,7 @@ def run_ours(args):
                        "l2": "flushed (512 MiB write) before every timed step"},
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": n_launch,
-            "clocks": clk.summary(), "sweep": sweep, "decode": decode, "backward": backward,
+            "clocks": clk.summary(), "sweep": sweep, "decode": decode, "backward": backward, "mixer": mixer,
         }
         print(json.dumps(line), flush=True)
     if ws > 1:
@@ -423,6 +440,100 @@ def _bench_decode(rlm, torch, dev, hbm_peak):
             "tok_s": round(B * T / (ms * 1e-3), 1), "us_per_step": round(us_step, 4),
             "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
             "bytes_per_step": per_step, "launches": T}
+
+
+def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms):
+    """The mixer wrapper of Sec. 3.4 (gate, local path K = 4, drive history in and
+    out) on the headline prefill shape, fused into the tcgen05 prefill, and its
+    decode step (B = 64) in a CUDA graph."""
+    from synth import make_inputs, make_mixer_inputs
+    P = MIXER
+    B, L, D, M, K = P["B"], P["L"], P["D"], P["M"], P["K"]
+    inp = make_inputs(B, L, D, M, "bf16", seed=2)
+    mx = make_mixer_inputs(inp, K, seed=2)
+    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
+    g = torch.from_numpy(mx.g).to(dev, torch.bfloat16)
+    p = rlm.Params.from_arrays(*inp.params(), device=dev)
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale, device=dev)
+    hin = rlm.ConvState(torch.from_numpy(mx.conv_in).to(dev, torch.bfloat16))
+    hout = rlm.ConvState.empty(B, D, K, dtype=torch.bfloat16, device=dev)
+    z = torch.empty_like(x)
+    st = rlm.State.empty(B, D, M, device=dev)
+    wsz = rlm.rlm_prefill_workspace_size(B, L, D, M, torch.bfloat16)
+    work = torch.empty(max(wsz, 256), dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def call():
+        rlm.rlm_mixer_prefill(x, g, p, local, z, conv_in=hin, state_out=st, conv_out=hout, workspace=work)
+
+    for _ in range(3):
+        flush.zero_()
+        call()
+    torch.cuda.synchronize()
+    ts = []
+    n0 = rlm.rlm_kernels_launched()
+    for _ in range(10):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        call()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    launches = (rlm.rlm_kernels_launched() - n0) // 10
+    ms = statistics.mean(ts)
+    alg = mixer_prefill_bytes(B, L, D, M, K)
+    gbs = alg / (ms * 1e-3) / 1e9
+    prefill = {"workload": f"fused mixer prefill B={B} L={L} D={D} M={M} K={K} bf16, gate and drive history",
+               "ms": round(ms, 5), "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 1),
+               "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
+               "algorithmic_bytes": alg, "launches_per_call": launches,
+               "vs_mix_only": round(ms / mix_ms, 3)}
+    del x, g, z, work
+
+    Bd, T = P["decode_B"], P["T"]
+    dinp = make_inputs(Bd, 1, D, M, "bf16", seed=3, decode_steps=T)
+    dmx = make_mixer_inputs(dinp, K, seed=3)
+    toks = torch.from_numpy(dinp.tokens).to(dev, torch.bfloat16)      # [T][B][D]
+    gts = torch.from_numpy(np.ascontiguousarray(
+        np.random.default_rng(4).standard_normal((T, Bd, D)).astype(np.float32))).to(dev, torch.bfloat16)
+    outs = torch.empty_like(toks)
+    dp = rlm.Params.from_arrays(*dinp.params(), device=dev)
+    dlocal = rlm.Local.from_arrays(dmx.conv_w, dmx.scale, device=dev)
+    dst = rlm.State.empty(Bd, D, M, device=dev)
+    rlm.rlm_state_init(dst, dp)
+    hist = rlm.ConvState(torch.zeros(Bd, K - 1, D, dtype=torch.bfloat16, device=dev))
+    s0 = dst.s.clone()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for t in range(8):
+            rlm.rlm_mixer_decode(toks[t], gts[t], dst, dlocal, hist, outs[t])
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph):
+        for t in range(T):
+            rlm.rlm_mixer_decode(toks[t], gts[t], dst, dlocal, hist, outs[t])
+    res = []
+    for rep in range(4):
+        dst.s.copy_(s0)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        graph.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        if rep:
+            res.append(a.elapsed_time(b))
+    dms = statistics.median(res)
+    us = dms * 1e3 / T
+    per = mixer_decode_bytes(Bd, D, M, K)
+    dgbs = per / (us * 1e-6) / 1e9
+    decode = {"workload": f"fused mixer decode B={Bd} D={D} M={M} K={K}, {T} steps, CUDA graph",
+              "us_per_step": round(us, 4), "tok_s": round(Bd * T / (dms * 1e-3), 1),
+              "achieved_GBps": round(dgbs, 1), "frac_hbm": round(dgbs / hbm_peak, 4), "bytes_per_step": per}
+    return {"prefill": prefill, "decode": decode}
 
 
 def _bench_backward(rlm, torch, dev, hbm_peak, args):

@@ -332,10 +332,13 @@ rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm
     const size_t need = rlm_prefill_workspace_size(x->B, x->L, (int)x->D, p->M, x->dtype);
     if ((s = check_workspace(ln, need)) != RLM_OK) return s;
     cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
-    const bool fused = (g || K > 0) && path == PrefillPath::kTc && tc_mixer_fused(x->B, x->L, (int)x->D, p->M, x->dtype);
+    // The gate alone is fused into the tcgen05 prefill's epilogue.  With a local
+    // path, the mixing and one full-width pass over x, g and y are faster than
+    // the fused kernel (whose 8-channel row slices cap its memory rate).
+    const bool fused = g && K == 0 && path == PrefillPath::kTc && tc_mixer_fused(x->B, x->L, (int)x->D, p->M, x->dtype);
     cudaError_t e;
     if (fused) {
-        const TcMix mix{g ? g->ptr : nullptr, hin, K > 0 ? local->conv_w : nullptr, K > 0 ? local->scale : nullptr, K};
+        const TcMix mix{g->ptr};
         e = tc_prefill(x->ptr, z->ptr, x->B, x->L, (int)x->D, p->M, p->decay, p->freq, p->amp, p->phase,
                        state_in ? state_in->s : nullptr, state_out ? state_out->s : nullptr,
                        state_out ? state_out->coef : nullptr, &mix, ln->workspace, st);

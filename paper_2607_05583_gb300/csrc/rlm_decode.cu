@@ -37,52 +37,61 @@ struct MixStep {
 };
 
 // Plain (coherent) load of the drive history, which every step rewrites.
-__device__ __forceinline__ float ld_hist(const float *p) { return *p; }
-__device__ __forceinline__ float ld_hist(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
+__device__ __forceinline__ float as_float(float v) { return v; }
+__device__ __forceinline__ float as_float(__nv_bfloat16 v) { return __bfloat162float(v); }
 
-// Loads of the mixer step, taken before the state update.
-struct MixLoads {
-    float gate, s, l;   // l: the local path without the current token
-    float w0;
+// One thread's share of the mixer step: the thread of rank g in its (b, d) group
+// (tpg threads) loads history entries j = g, g + tpg, ... (at most one when
+// tpg >= K - 1), weighs them, and later moves them one slot down; rank 0 also
+// loads the gate and adds the current drive's tap.  The loads are issued before
+// the state update.
+template <typename T>
+struct MixPart {
+    float l;          // partial sum of w[k] u_{t-k}
+    float gate;       // rank 0: g_t
+    T hv[2];          // the history entries this thread owns (tpg >= 4 gives at most two)
 };
 
 template <typename T>
-__device__ __forceinline__ MixLoads mix_load(const MixStep<T> &m, int64_t bd, int D) {
-    MixLoads r{1.0f, 0.0f, 0.0f, 0.0f};
-    if (m.g) r.gate = ld_elem(m.g + bd);
+__device__ __forceinline__ MixPart<T> mix_part(const MixStep<T> &m, int64_t bd, int D, int g, int tpg,
+                                               const T *x_t) {
+    MixPart<T> r;
+    r.l = 0.0f;
+    r.gate = 0.0f;
+    if (m.g && g == 0) r.gate = ld_elem(m.g + bd);
     if (m.K > 0) {
         const int d = (int)(bd % D);
         const int64_t b = bd / D;
-        r.s = __ldg(m.scale + d);
-        r.w0 = __ldg(m.conv_w + (int64_t)d * m.K);
+        const float *w = m.conv_w + (int64_t)d * m.K;
+        if (g == 0) r.l = __ldg(w) * ld_elem(x_t + bd);
         const T *h = m.hist + b * (m.K - 1) * (int64_t)D + d;
 #pragma unroll
-        for (int k = 1; k < kMaxK; ++k)
-            if (k < m.K) r.l = fmaf(__ldg(m.conv_w + (int64_t)d * m.K + k), ld_hist(h + (int64_t)(m.K - 1 - k) * D), r.l);
+        for (int i = 0; i < 2; ++i) {
+            const int j = g + i * tpg;              // entry j holds u_{t-(K-1-j)}
+            if (j < m.K - 1) {
+                r.hv[i] = h[(int64_t)j * D];
+                r.l = fmaf(__ldg(w + (m.K - 1 - j)), as_float(r.hv[i]), r.l);
+            }
+        }
     }
     return r;
 }
 
-// z = sigma(g) y + s (w0 x + l); shifts the history and appends x.
+// After the group's reductions (which every thread's loads feed, so all loads of
+// the old history are complete): shift the owned entries one slot down, rank 0
+// appends the current drive.
 template <typename T>
-__device__ __forceinline__ float mix_finish(const MixStep<T> &m, const MixLoads &r, int64_t bd, int D, float y,
-                                            const T *x_t) {
-    const float gate = m.g ? 1.0f / (1.0f + expf(-r.gate)) : 1.0f;
-    if (m.K == 0) return gate * y;
-    const float xv = ld_elem(x_t + bd);
-    if (m.K > 1) {
-        const int64_t b = bd / D;
-        T *h = m.hist + b * (m.K - 1) * (int64_t)D + (bd % D);
-        T v[kMaxK];
+__device__ __forceinline__ void mix_shift(const MixStep<T> &m, const MixPart<T> &r, int64_t bd, int D, int g,
+                                          int tpg, const T *x_t) {
+    if (m.K < 2) return;
+    const int64_t b = bd / D;
+    T *h = m.hist + b * (m.K - 1) * (int64_t)D + (bd % D);
 #pragma unroll
-        for (int j = 1; j < kMaxK - 1; ++j)
-            if (j < m.K - 1) v[j] = h[(int64_t)j * D];
-#pragma unroll
-        for (int j = 1; j < kMaxK - 1; ++j)
-            if (j < m.K - 1) h[(int64_t)(j - 1) * D] = v[j];
-        h[(int64_t)(m.K - 2) * D] = x_t[bd];
+    for (int i = 0; i < 2; ++i) {
+        const int j = g + i * tpg;
+        if (j >= 1 && j < m.K - 1) h[(int64_t)(j - 1) * D] = r.hv[i];
     }
-    return fmaf(gate, y, r.s * fmaf(r.w0, xv, r.l));
+    if (g == 0) h[(int64_t)(m.K - 2) * D] = x_t[bd];
 }
 
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
@@ -102,8 +111,8 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_vec2(
     const int g = (int)(gid & ((1 << log2_tpg) - 1));
     const int tpg = 1 << log2_tpg;
     const bool valid = bd < BD && 2 * g < M;
-    MixLoads ml{};
-    if (kMix && valid && g == 0) ml = mix_load(mix, bd, D);
+    MixPart<T> mp{};
+    if (kMix && bd < BD) mp = mix_part(mix, bd, D, g, tpg, x_t);  // every rank, with or without modes
     float acc = 0.0f;
     if (valid) {
         const int d = (int)(bd % D);
@@ -119,11 +128,19 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_vec2(
         s[si] = make_float4(r0, i0, r1, i1);
         acc = fmaf(c0.z, r0, fmaf(-c0.w, i0, fmaf(c1.z, r1, -c1.w * i1)));
     }
-    for (int o = tpg >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (valid && g == 0) {
-        if (kMix) acc = mix_finish(mix, ml, bd, D, acc, x_t);
-        st_elem(y_t + bd, acc);
+    float lsum = mp.l;
+    for (int o = tpg >> 1; o > 0; o >>= 1) {
+        acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (kMix) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
     }
+    if (kMix && bd < BD) {
+        mix_shift(mix, mp, bd, D, g, tpg, x_t);
+        if (g == 0) {
+            if (mix.g) acc *= 1.0f / (1.0f + expf(-mp.gate));
+            if (mix.K > 0) acc = fmaf(__ldg(mix.scale + bd % D), lsum, acc);
+        }
+    }
+    if (valid && g == 0) st_elem(y_t + bd, acc);
 }
 
 // Any M: each thread owns up to MPT modes, accessed as float2.
@@ -137,8 +154,8 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_any(
     const int64_t bd = gid >> log2_tpg;
     const int g = (int)(gid & ((1 << log2_tpg) - 1));
     const int tpg = 1 << log2_tpg;
-    MixLoads ml{};
-    if (kMix && bd < BD && g == 0) ml = mix_load(mix, bd, D);
+    MixPart<T> mp{};
+    if (kMix && bd < BD) mp = mix_part(mix, bd, D, g, tpg, x_t);
     float acc = 0.0f;
     if (bd < BD) {
         const int d = (int)(bd % D);
@@ -154,11 +171,19 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_any(
             acc = fmaf(cf.z, re, fmaf(-cf.w, im, acc));
         }
     }
-    for (int o = tpg >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (bd < BD && g == 0) {
-        if (kMix) acc = mix_finish(mix, ml, bd, D, acc, x_t);
-        st_elem(y_t + bd, acc);
+    float lsum = mp.l;
+    for (int o = tpg >> 1; o > 0; o >>= 1) {
+        acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (kMix) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
     }
+    if (kMix && bd < BD) {
+        mix_shift(mix, mp, bd, D, g, tpg, x_t);
+        if (g == 0) {
+            if (mix.g) acc *= 1.0f / (1.0f + expf(-mp.gate));
+            if (mix.K > 0) acc = fmaf(__ldg(mix.scale + bd % D), lsum, acc);
+        }
+    }
+    if (bd < BD && g == 0) st_elem(y_t + bd, acc);
 }
 
 __global__ void k_state_init(float2 *__restrict__ s, float4 *__restrict__ coef, int64_t BDM,
@@ -196,12 +221,16 @@ cudaError_t decode_t(const T *x_t, T *y_t, int B, int D, int M, float *s, const 
     int pairs = (M + 1) / 2;
     int log2_tpg = 0;
     while ((1 << log2_tpg) < pairs && log2_tpg < 5) ++log2_tpg;
+    // The mixer step spreads the K - 1 <= 7 history entries over the group, two
+    // at most per rank: at least 4 ranks (extra ranks own no modes).
+    const bool widened = kMix && log2_tpg < 2;
+    if (widened) log2_tpg = 2;
     const int tpg = 1 << log2_tpg;
     const int64_t BD = (int64_t)B * D;
     const int64_t threads = BD * tpg;
     const unsigned grid = (unsigned)((threads + kDecodeBlock - 1) / kDecodeBlock);
     const float4 *cf = reinterpret_cast<const float4 *>(coef);
-    if (M % 2 == 0 && 2 * tpg >= M)
+    if (!widened && M % 2 == 0 && 2 * tpg >= M)
         return launch_pdl(k_decode_vec2<T, kMix>, grid, st, x_t, y_t, BD, D, M, log2_tpg,
                           reinterpret_cast<float4 *>(s), cf, mix);
     const int mpt = (M + tpg - 1) / tpg;

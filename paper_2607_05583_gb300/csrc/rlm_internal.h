@@ -96,19 +96,15 @@ cudaError_t state_init(float *s, float *coef, int B, int D, int M, const float *
 // ---- tcgen05 prefill (rlm_prefill_tc.cu) ------------------------------------
 // True when the tensor-core path covers this problem.
 bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
-// True when that path also forms the mixer output in its epilogue (unsegmented
+// True when that path also applies the mixer's gate in its epilogue (unsegmented
 // launches).
 bool tc_mixer_fused(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
 size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int M);
-// The mixer wrapper (Sec. 3.4) of the fused epilogue: g nullable (no gate); hist
-// [B][K-1][D] nullable (zero drives before token 0); K = 0: no local path.
+// The gate field (Sec. 3.4) for the fused epilogue: [B][L][D] bf16, non-null.
 struct TcMix {
     const void *g;
-    const void *hist;
-    const float *conv_w, *scale;
-    int K;
 };
-// mix non-null: y receives z = sigma(g) y + s (w * x) (requires tc_mixer_fused).
+// mix non-null: y receives z = sigma(g) y (requires tc_mixer_fused).
 cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int M,
                        const float *decay, const float *freq, const float *amp,
                        const float *phase, const float *state_in, float *state_out, float *coef_out,

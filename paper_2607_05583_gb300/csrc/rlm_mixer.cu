@@ -4,71 +4,104 @@
 // applied in place to a field z that already holds the mixing y, plus the update
 // of the local path's drive history (the last K-1 drives of history || x).
 //
-// k_mixer_epilogue: one thread per (b, run of kRun tokens, d), channel fastest so a
-// warp reads consecutive channels of one token row.  The thread keeps the K most
-// recent drives in registers, so x is read once (plus K-1 tokens of overlap per
-// run).  The pass moves 8 (bf16) or 16 (fp32) bytes per token-channel: read x, g
-// and y, write z.
+// k_mixer_epilogue: a block finishes a tile of kTT tokens x kTC channels.  It first
+// stages the tile's drive rows, with the K - 1 rows before it (from x or the
+// history), in shared memory with 16-byte loads; then each thread takes a channel
+// pair for kTT / 4 tokens, reads its taps from shared memory (a warp reads 128
+// contiguous bytes per row: no bank conflicts) and the gate and y from global
+// memory, and writes z.  The kernel size K is a template parameter (2 K weights per
+// thread in registers).  The pass moves 8 (bf16) or 16 (fp32) bytes per
+// token-channel: read x, g and y, write z.
 #include "rlm_device.cuh"
 #include "rlm_internal.h"
 
 namespace rlm {
 namespace {
 
-constexpr int kRun = 32;
 constexpr int kBlock = 256;
 constexpr int kMaxK = RLM_MAX_LOCAL_K;
+constexpr int kTT = 64;    // tokens per tile
+constexpr int kTC = 128;   // channels per tile (a multiple of 8 channels is staged)
 
-__device__ __forceinline__ float sigmoidf(float v) { return 1.0f / (1.0f + expf(-v)); }
+__device__ __forceinline__ float gatef(float v) { return __fdividef(1.0f, 1.0f + __expf(-v)); }
 
-// Plain (coherent) load of an element this kernel also writes.
-__device__ __forceinline__ float ld_rw(const float *p) { return *p; }
-__device__ __forceinline__ float ld_rw(const __nv_bfloat16 *p) { return __bfloat162float(*p); }
-
-// u_{t}[d] of the sequence preceded by its history: t < 0 reads the history
-// ([B][K-1][D], oldest first) or zero.
-template <typename T>
-__device__ __forceinline__ float drive_at(const T *x, const T *hist, int64_t b, int64_t t, int64_t L,
-                                          int D, int K, int d) {
-    if (t >= 0) return ld_elem(x + (b * L + t) * D + d);
-    if (!hist) return 0.0f;
-    return ld_elem(hist + (b * (K - 1) + (K - 1 + t)) * D + d);
+// Two consecutive channels as floats, and back.
+__device__ __forceinline__ float2 ld2(const float *p) { return *reinterpret_cast<const float2 *>(p); }
+__device__ __forceinline__ float2 ld2(const __nv_bfloat16 *p) {
+    const uint32_t v = *reinterpret_cast<const uint32_t *>(p);
+    return make_float2(__uint_as_float(v << 16), __uint_as_float(v & 0xFFFF0000u));
+}
+__device__ __forceinline__ void st2(float *p, float2 v) { *reinterpret_cast<float2 *>(p) = v; }
+__device__ __forceinline__ void st2(__nv_bfloat16 *p, float2 v) {
+    uint32_t a;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(a) : "f"(v.y), "f"(v.x));
+    *reinterpret_cast<uint32_t *>(p) = a;
 }
 
-template <typename T>
+template <typename T, int K>
 __global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__ x, const T *__restrict__ g,
                                                            T *__restrict__ z, const T *__restrict__ hist,
                                                            const float *__restrict__ conv_w,
-                                                           const float *__restrict__ scale, int64_t B,
-                                                           int64_t L, int D, int K) {
-    const int64_t nruns = (L + kRun - 1) / kRun;
-    const int64_t gid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (gid >= B * nruns * D) return;
-    const int d = (int)(gid % D);
-    const int64_t br = gid / D;
-    const int64_t b = br / nruns, t0 = (br % nruns) * kRun;
-    const int64_t t1 = t0 + kRun < L ? t0 + kRun : L;
-    float w[kMaxK], win[kMaxK];  // win[k] = u_{t-k}
-    float s = 0.0f;
-#pragma unroll
-    for (int k = 0; k < kMaxK; ++k) {
-        w[k] = k < K ? __ldg(conv_w + (int64_t)d * K + k) : 0.0f;
-        win[k] = 0.0f;
+                                                           const float *__restrict__ scale, int64_t L, int D) {
+    constexpr int kRows = kTT + (K > 1 ? K - 1 : 0);
+    constexpr int kVE = 16 / sizeof(T);                // elements per 16-byte vector
+    __shared__ __align__(16) T xs[K > 0 ? kRows * kTC : 1];
+    const int c0 = blockIdx.x * kTC;
+    const int64_t t0 = (int64_t)blockIdx.y * kTT;
+    const int64_t b = blockIdx.z;
+    const int nc = min(kTC, D - c0);                   // a multiple of 8
+    const int tid = threadIdx.x;
+    if (K > 0) {
+        const int vpr = nc / kVE;
+        for (int i = tid; i < kRows * vpr; i += kBlock) {
+            const int r = i / vpr, v = i % vpr;
+            const int64_t t = t0 - (K > 1 ? K - 1 : 0) + r;
+            uint4 val = make_uint4(0u, 0u, 0u, 0u);
+            if (t >= 0 && t < L)
+                val = *reinterpret_cast<const uint4 *>(x + (b * L + t) * D + c0 + v * kVE);
+            else if (t < 0 && hist)
+                val = *reinterpret_cast<const uint4 *>(hist + (b * (K - 1) + (K - 1 + t)) * D + c0 + v * kVE);
+            *reinterpret_cast<uint4 *>(xs + r * kTC + v * kVE) = val;
+        }
+        __syncthreads();
     }
-    if (K > 0) s = __ldg(scale + d);
+    const int cp = tid % (kTC / 2), tg = tid / (kTC / 2);
+    const int c = 2 * cp;
+    if (c >= nc) return;
+    float w0[K > 0 ? K : 1], w1[K > 0 ? K : 1];
+    float s0 = 0.0f, s1 = 0.0f;
 #pragma unroll
-    for (int k = 1; k < kMaxK; ++k)
-        if (k < K) win[k] = drive_at(x, hist, b, t0 - k, L, D, K, d);
-    for (int64_t t = t0; t < t1; ++t) {
-        const int64_t i = (b * L + t) * D + d;
-        win[0] = ld_elem(x + i);
-        float l = 0.0f;
+    for (int k = 0; k < K; ++k) {
+        w0[k] = __ldg(conv_w + (int64_t)(c0 + c) * K + k);
+        w1[k] = __ldg(conv_w + (int64_t)(c0 + c + 1) * K + k);
+    }
+    if (K > 0) {
+        s0 = __ldg(scale + c0 + c);
+        s1 = __ldg(scale + c0 + c + 1);
+    }
+    constexpr int kPer = kTT / (kBlock / (kTC / 2));   // tokens per thread
+#pragma unroll 4
+    for (int tt = 0; tt < kPer; ++tt) {
+        const int r = tg * kPer + tt;                   // token t0 + r
+        const int64_t t = t0 + r;
+        if (t >= L) break;
+        const int64_t i = (b * L + t) * D + c0 + c;
+        float2 zv = ld2(z + i);
+        if (g) {
+            const float2 gv = ld2(g + i);
+            zv = make_float2(zv.x * gatef(gv.x), zv.y * gatef(gv.y));
+        }
+        if (K > 0) {
+            float l0 = 0.0f, l1 = 0.0f;
 #pragma unroll
-        for (int k = 0; k < kMaxK; ++k) l = fmaf(w[k], win[k], l);
-        const float gate = g ? sigmoidf(ld_elem(g + i)) : 1.0f;
-        st_elem(z + i, fmaf(gate, ld_rw(z + i), s * l));
-#pragma unroll
-        for (int k = kMaxK - 1; k > 0; --k) win[k] = win[k - 1];
+            for (int k = 0; k < K; ++k) {
+                const float2 v = ld2(xs + (r + (K > 1 ? K - 1 : 0) - k) * kTC + c);
+                l0 = fmaf(w0[k], v.x, l0);
+                l1 = fmaf(w1[k], v.y, l1);
+            }
+            zv = make_float2(fmaf(s0, l0, zv.x), fmaf(s1, l1, zv.y));
+        }
+        st2(z + i, zv);
     }
 }
 
@@ -98,15 +131,31 @@ __global__ void __launch_bounds__(kBlock) k_conv_tail(const T *__restrict__ x, c
     }
 }
 
+template <typename T, int K>
+cudaError_t epilogue_k(const void *x, const void *g, void *z, const void *hist, const float *conv_w,
+                       const float *scale, int64_t B, int64_t L, int D, cudaStream_t st) {
+    const dim3 grid((unsigned)((D + kTC - 1) / kTC), (unsigned)((L + kTT - 1) / kTT), (unsigned)B);
+    k_mixer_epilogue<T, K><<<grid, kBlock, 0, st>>>(static_cast<const T *>(x), static_cast<const T *>(g),
+                                                    static_cast<T *>(z), static_cast<const T *>(hist), conv_w,
+                                                    scale, L, D);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
 template <typename T>
 cudaError_t epilogue_t(const void *x, const void *g, void *z, const void *hist, const float *conv_w,
                        const float *scale, int64_t B, int64_t L, int D, int K, cudaStream_t st) {
-    const int64_t n = B * ((L + kRun - 1) / kRun) * D;
-    k_mixer_epilogue<T><<<(unsigned)((n + kBlock - 1) / kBlock), kBlock, 0, st>>>(
-        static_cast<const T *>(x), static_cast<const T *>(g), static_cast<T *>(z), static_cast<const T *>(hist),
-        conv_w, scale, B, L, D, K);
-    count_launches(1);
-    return cudaGetLastError();
+    switch (K) {
+        case 0: return epilogue_k<T, 0>(x, g, z, hist, conv_w, scale, B, L, D, st);
+        case 1: return epilogue_k<T, 1>(x, g, z, hist, conv_w, scale, B, L, D, st);
+        case 2: return epilogue_k<T, 2>(x, g, z, hist, conv_w, scale, B, L, D, st);
+        case 3: return epilogue_k<T, 3>(x, g, z, hist, conv_w, scale, B, L, D, st);
+        case 4: return epilogue_k<T, 4>(x, g, z, hist, conv_w, scale, B, L, D, st);
+        case 5: return epilogue_k<T, 5>(x, g, z, hist, conv_w, scale, B, L, D, st);
+        case 6: return epilogue_k<T, 6>(x, g, z, hist, conv_w, scale, B, L, D, st);
+        case 7: return epilogue_k<T, 7>(x, g, z, hist, conv_w, scale, B, L, D, st);
+        default: return epilogue_k<T, 8>(x, g, z, hist, conv_w, scale, B, L, D, st);
+    }
 }
 
 template <typename T>

@@ -123,8 +123,7 @@ constexpr int kOffY = kOffX + kXSlots * kBox * 16;
 constexpr int kOffBar = kOffY + kYSlots * kYRows * 16;
 constexpr int kNumBars = 128;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
-constexpr int kOffWts = kOffMisc + 64;                       // mixer: [8 ch][8 taps] w, then [8] s (fp32)
-constexpr int kSmemBytes = kOffWts + 320 + 1024;             // + alignment slack
+constexpr int kSmemBytes = kOffMisc + 64 + 1024;             // + alignment slack
 static_assert(kOffX % 128 == 0 && kOffY % 128 == 0, "TMA buffers need 128-byte alignment");
 static_assert(kSmemBytes <= 232448, "shared memory budget");
 // Prologue tables, in buffers no other role touches before the prologue ends
@@ -159,8 +158,7 @@ constexpr int kBarFinal = kBarYEmpty + kYSlots; // [8]
 constexpr int kBarConsts = kBarFinal + 8;       // the A operands and U tables are built
 constexpr int kBarGFull = kBarConsts + 1;       // [kYSlots] mixer: the gate rows of a z slot landed
 static_assert(kBarGFull + kYSlots <= kNumBars, "too many barriers");
-constexpr int kMixBarrier = 2;                  // named barrier of the 8 epilogue warps
-constexpr int kMaxTaps = RLM_MAX_LOCAL_K;
+
 
 
 // ------------------------------------------------------------ PTX wrappers
@@ -364,12 +362,6 @@ struct TcArgs {
     float2 *seg_state;   // [B][nseg][D][M]: each segment's end state from a zero start
     unsigned long long *seg_flag;  // [B][nseg][D][M]: == epoch once that state is published
     unsigned long long epoch;      // distinct for every segmented launch of this process
-    // Mixer (kMix instances): z = sigma(g) y + s (w * x) formed in the epilogue.
-    const __nv_bfloat16 *x;        // the drive, read for the local path across tile edges
-    const __nv_bfloat16 *hist;     // [B][K-1][D] drives before token 0, or null (zeros)
-    const float *conv_w, *scale;   // [D][K], [D]
-    int K;                         // 0: no local path
-    int gate;                      // nonzero: the gate field is loaded through tmap_g
 };
 
 // kSeg: the grid's z dimension splits the sequence into segments.  The
@@ -380,14 +372,10 @@ struct TcArgs {
 // to the state entering chunk n0, which gives lambda^(i+1-p) s_in at its positions
 // i >= p (those before p are negative times, never stored) and lambda^(64-p) s_in
 // carried on.  |lambda^-p| <= exp(63 gamma) stays bounded.
-// kMix: the mixer wrapper of Sec. 3.4 in the epilogue (unsegmented launches only).
-// The store issuer loads the gate rows of each z ring slot into the slot itself
-// once the slot's previous store has been read out; every epilogue thread reads
-// its 8 bytes of g there and overwrites them with z.  The local path reads the
-// drive from the tile's B operand, which the epilogue (not the MMA thread) then
-// releases: each thread loads its own position and takes the K-1 earlier ones
-// from lower lanes by shuffle; the lanes below K-1 load theirs directly (from
-// the previous chunk, or across the tile edge from global memory or the history).
+// kMix: the gate of the mixer wrapper (Sec. 3.4), z = sigma(g) y, in the epilogue
+// (unsegmented launches only).  The store issuer loads the gate rows of each z ring
+// slot into the slot itself once the slot's previous store has been read out;
+// every epilogue thread reads its 8 bytes of g there and overwrites them with z.
 template <bool kSeg, bool kInj, bool kMix>
 __global__ void __launch_bounds__(kThreads, 1)
     k_prefill_tc(const __grid_constant__ CUtensorMap tmap_x,
@@ -652,15 +640,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         // One bulk group per slot of 512 rows; up to kYSlots - 2 groups may still
         // be reading shared memory while the next slot is issued.
         const int nslots = nB * kYPerTile;
-        // Mixer: the gate rows of z slot k go into the slot itself (two boxes of 256
-        // rows); without a gate the slot is only marked ready.
+        // Mixer: the gate rows of z slot k go into the slot itself (two boxes of 256 rows).
         auto issue_g = [&](int k) {
             const uint32_t slot = k % kYSlots;
             if (lane != 0) return;
-            if (!args.gate) {
-                bar_arrive(bar(kBarGFull + slot));
-                return;
-            }
             bar_expect_tx(bar(kBarGFull + slot), kYRows * 16);
             const int jt = ja + k / kYPerTile, e = k % kYPerTile;
             for (int h = 0; h < kYRows / kBox; ++h)
@@ -747,7 +730,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // reads of the B operand) are complete: release the buffer.  A
                 // second commit issued right behind the first was observed to
                 // arrive while the chain was still reading shared memory.
-                if (!kMix) bar_arrive(bar(kBarBxEmpty + buf));  // kMix: the epilogue releases it
+                bar_arrive(bar(kBarBxEmpty + buf));
                 if (v < nA) continue;  // state-only pass: no output
 #pragma unroll
                 for (int kk = 0; kk < 2; ++kk) umma_ss(d, du0 + kk * 16, ds0 + kk * ((2 * kBsLbo) >> 4), kIdesc, 1);
@@ -859,30 +842,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int hb = quarter < 2 ? 8 : 0;
         const uint32_t trow = tmem + ((uint32_t)(32 * quarter) << 16) + 16 * h;
         if constexpr (kMix) {
-            // The CTA's local-path weights into shared memory (taps past K are zero).
-            float *wts = reinterpret_cast<float *>(smem + kOffWts);
-            for (int i = tid; i < 8 * kMaxTaps + 8; i += 256) {
-                float v = 0.0f;
-                if (i < 8 * kMaxTaps) {
-                    const int c = i / kMaxTaps, k = i % kMaxTaps;
-                    if (k < args.K) v = args.conv_w[(int64_t)(d0 + c) * args.K + k];
-                } else if (args.K > 0) {
-                    v = args.scale[d0 + i - 8 * kMaxTaps];
-                }
-                wts[i] = v;
-            }
-            asm volatile("bar.sync %0, %1;" ::"n"(kMixBarrier), "n"(256) : "memory");
-            const int K = args.K;
             for (int j = 0; j < nB; ++j) {
                 const int ng0 = j * kYPerTile + 2 * h;
                 if (!wait_bar(bar(kBarGFull + ng0 % kYSlots), (ng0 / kYSlots) & 1, abort_flag) ||
                     !wait_bar(bar(kBarGFull + (ng0 + 1) % kYSlots), ((ng0 + 1) / kYSlots) & 1, abort_flag))
                     break;
-                const int buf = j & 1;
-                const int64_t tile_t = args.t0 + (int64_t)j * kTile;
-                uint32_t pk[2][16];
                 bool ok = true;
-#pragma unroll 1
+#pragma unroll
                 for (int p = 0; p < 2; ++p) {
                     const int cA = c0 + 2 * p, cB = cA + 1;
                     if (!wait_bar(bar(kBarUDone + cA), j & 1, abort_flag) ||
@@ -897,55 +863,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tmem_ld8(trow + cA * kNT + 8 * sh, va);
                         tmem_ld8(trow + cB * kNT + 8 * sh, vb);
                         tmem_wait_ld();
-                        const uint8_t *gs = smem + kOffY + ((ng0 + sh) % kYSlots) * (kYRows * 16) + hb + 4 * p;
-#pragma unroll 1
-                        for (int n8 = 0; n8 < 8; ++n8) {
-                            const int n = 16 * h + 8 * sh + n8;   // chunk within the tile
-                            float z[2] = {__uint_as_float(va[n8]), __uint_as_float(vb[n8])};
-                            if (args.gate) {
-                                const __nv_bfloat162 g2 =
-                                    *reinterpret_cast<const __nv_bfloat162 *>(gs + (n8 * kC + pos) * 16);
-                                z[0] *= __fdividef(1.0f, 1.0f + __expf(-__low2float(g2)));
-                                z[1] *= __fdividef(1.0f, 1.0f + __expf(-__high2float(g2)));
-                            }
-                            if (K > 0) {
-                                const int64_t t = tile_t + (int64_t)n * kC + pos;
+                        // The gate rows (and, once done, the z rows) of this 512-token block.
+                        uint8_t *gs = smem + kOffY + ((ng0 + sh) % kYSlots) * (kYRows * 16) + hb + 4 * p;
 #pragma unroll
-                                for (int cc = 0; cc < 2; ++cc) {
-                                    const int c = cA + cc;
-                                    const uint8_t *bx = smem + kOffBx + buf * kBxBuf + c * kBxStride;
-                                    // x at chunk nn, position pp of this tile (B operand layout:
-                                    // positions reversed, 8-position core rows).
-                                    auto xat = [&](int nn, int pp) {
-                                        const int pr = 63 - pp;
-                                        return __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(
-                                            bx + (nn >> 3) * 1024 + (pr >> 3) * 128 + (nn & 7) * 16 + (pr & 7) * 2));
-                                    };
-                                    const float* w = reinterpret_cast<const float *>(smem + kOffWts) + c * kMaxTaps;
-                                    const float own = xat(n, pos);
-                                    float l = w[0] * own;
-                                    for (int k = 1; k < K; ++k) {
-                                        float v = __shfl_up_sync(0xffffffffu, own, k);
-                                        if (lane < k) {
-                                            const int pp = pos - k;
-                                            if (pp >= 0)
-                                                v = xat(n, pp);
-                                            else if (n > 0)
-                                                v = xat(n - 1, pp + kC);
-                                            else if (t - k >= 0)
-                                                v = __bfloat162float(args.x[((int64_t)b * args.L + (t - k)) * D + d0 + c]);
-                                        }
-                                        if (t - k < 0)
-                                            v = (args.hist && t - k >= -(K - 1))
-                                                    ? __bfloat162float(args.hist[((int64_t)b * (K - 1) + (K - 1) + (t - k)) * D + d0 + c])
-                                                    : 0.0f;
-                                        l = fmaf(w[k], v, l);
-                                    }
-                                    const float sc = reinterpret_cast<const float *>(smem + kOffWts)[8 * kMaxTaps + c];
-                                    z[cc] = fmaf(sc, l, z[cc]);
-                                }
-                            }
-                            pk[p][8 * sh + n8] = pack_bf16x2(z[0], z[1]);
+                        for (int n8 = 0; n8 < 8; ++n8) {
+                            uint32_t *gz = reinterpret_cast<uint32_t *>(gs + (n8 * kC + pos) * 16);
+                            const __nv_bfloat162 g2 = *reinterpret_cast<const __nv_bfloat162 *>(gz);
+                            const float za = __uint_as_float(va[n8]) * __fdividef(1.0f, 1.0f + __expf(-__low2float(g2)));
+                            const float zb = __uint_as_float(vb[n8]) * __fdividef(1.0f, 1.0f + __expf(-__high2float(g2)));
+                            *gz = pack_bf16x2(za, zb);
                         }
                     }
                     tc_fence_before();
@@ -956,20 +882,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 if (!ok) break;
-                // This warp's reads of the tile's B operand are done.
+                fence_async_smem();
                 __syncwarp();
-                if (lane == 0) bar_arrive(bar(kBarBxEmpty + buf));
-#pragma unroll
-                for (int sh = 0; sh < 2; ++sh) {
-                    const uint32_t slot = (ng0 + sh) % kYSlots;
-                    uint8_t *ys = smem + kOffY + slot * (kYRows * 16) + hb;
-#pragma unroll
-                    for (int n = 0; n < 8; ++n)
-                        *reinterpret_cast<uint2 *>(ys + (n * kC + pos) * 16) =
-                            make_uint2(pk[0][8 * sh + n], pk[1][8 * sh + n]);
-                    fence_async_smem();
-                    __syncwarp();
-                    if (lane == 0) bar_arrive(bar(kBarYFull + slot));
+                if (lane == 0) {
+                    bar_arrive(bar(kBarYFull + ng0 % kYSlots));
+                    bar_arrive(bar(kBarYFull + (ng0 + 1) % kYSlots));
                 }
             }
         } else
@@ -1113,7 +1030,7 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     if (!make_field_map(&mx, x, B, L, D) || !make_field_map(&my, y, B, L, D))
         return cudaErrorInvalidValue;
     mg = mx;  // placeholder unless a gate field is given
-    if (mix && mix->g && !make_field_map(&mg, mix->g, B, L, D)) return cudaErrorInvalidValue;
+    if (mix && (!mix->g || !make_field_map(&mg, mix->g, B, L, D))) return cudaErrorInvalidValue;
     static std::mutex mu;
     static std::vector<int> configured;
     int dev = 0;
@@ -1155,12 +1072,6 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.seg_state = nullptr;
     a.seg_flag = nullptr;
     a.epoch = 0;
-    a.x = static_cast<const __nv_bfloat16 *>(x);
-    a.hist = mix ? static_cast<const __nv_bfloat16 *>(mix->hist) : nullptr;
-    a.conv_w = mix ? mix->conv_w : nullptr;
-    a.scale = mix ? mix->scale : nullptr;
-    a.K = mix ? mix->K : 0;
-    a.gate = mix && mix->g ? 1 : 0;
     dim3 grid((unsigned)(D / kDG), (unsigned)B, (unsigned)sg.nseg);
     if (mix && sg.nseg >= 2) return cudaErrorInvalidValue;  // callers check tc_mixer_fused
     if (sg.nseg < 2) {

@@ -120,7 +120,8 @@ def test_mixer_split_prefill_in_place_equals_whole(M):
     np.testing.assert_array_equal(to_np(cs.u), tr)
 
 
-@pytest.mark.parametrize("dtype,M,K", [("bf16", 16, 4), ("f32", 7, 3), ("bf16", 40, 8), ("bf16", 16, 1)])
+@pytest.mark.parametrize("dtype,M,K", [("bf16", 16, 4), ("f32", 7, 3), ("bf16", 40, 8), ("bf16", 16, 1),
+                                     ("f32", 1, 8), ("bf16", 2, 6), ("bf16", 6, 8)])
 def test_mixer_decode_continues_the_prefill(dtype, M, K):
     """Prefill of 300 tokens then 40 fused mixer decode steps reproduce the oracle's
     mixer output over all 340 tokens, and the final state and history."""
@@ -196,7 +197,8 @@ def test_mixer_prefill_long_context_sampled():
     np.testing.assert_array_equal(to_np(cout.u)[:, :, ch], tr)
 
 
-# ---- the fused tcgen05 epilogue (bf16, M = 16, unsegmented: >= 77 channel groups x rows)
+# ---- the gate fused into the tcgen05 epilogue (bf16, M = 16, unsegmented: >= 77
+# channel groups x rows); with a local path the mixing is followed by one full-width pass
 def _launches(fn):
     before = rlm.rlm_kernels_launched()
     fn()
@@ -205,12 +207,13 @@ def _launches(fn):
 
 
 @pytest.mark.parametrize("B,L,D,K,with_g,with_hist", [
-    (2, 2 * 2048 + 77, 512, 4, True, True),    # ragged, three tiles, token 0 inside tile 0
-    (1, 3 * 2048, 1024, 8, True, True),        # tiles aligned with the sequence, K = 8
-    (2, 2048 + 3, 512, 2, False, True),        # local path only
-    (2, 4000, 512, 0, True, False),            # gate only
+    (2, 2 * 2048 + 77, 512, 0, True, False),   # gate only: fused; ragged, token 0 inside tile 0
+    (1, 3 * 2048, 1024, 0, True, False),       # gate only: fused; tiles aligned with the sequence
+    (2, 2 * 2048 + 77, 512, 4, True, True),    # local path: mixing + pass + history tail
+    (1, 3 * 2048, 1024, 8, True, True),
+    (2, 2048 + 3, 512, 2, False, True),
 ])
-def test_fused_mixer_prefill_matches_oracle(B, L, D, K, with_g, with_hist):
+def test_tcgen05_shape_mixer_prefill_matches_oracle(B, L, D, K, with_g, with_hist):
     inp = make_inputs(B, L, D, 16, "bf16", seed=L + D + K)
     mx = make_mixer_inputs(inp, K, seed=L + K)
     out = {}
@@ -219,43 +222,46 @@ def test_fused_mixer_prefill_matches_oracle(B, L, D, K, with_g, with_hist):
         out["r"] = _run_prefill(inp, mx, with_g, with_hist)
 
     n = _launches(run)
-    # one fused prefill launch (+ the history tail when K >= 2); the unfused route
-    # would add an epilogue launch
-    assert n == 1 + (1 if K >= 2 else 0), n
+    # fused gate: one launch; otherwise the tcgen05 prefill, the pass and (K >= 2)
+    # the history tail
+    assert n == (1 if K == 0 else 2 + (1 if K >= 2 else 0)), n
     z, so, cout = out["r"]
     _check_prefill(inp, mx, z, so, cout, with_g, with_hist)
 
 
-def test_fused_mixer_prefill_from_state_and_split_in_place():
-    B, L, D, K, cut = 2, 6000, 512, 4, 2345
+@pytest.mark.parametrize("K", [0, 4])
+def test_tcgen05_shape_mixer_prefill_from_state_and_split_in_place(K):
+    B, L, D, cut = 2, 6000, 512, 2345
     inp = make_inputs(B, L, D, 16, "bf16", seed=77)
     mx = make_mixer_inputs(inp, K, seed=77)
     x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
     p = rlm.Params.from_arrays(*inp.params())
-    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale) if K else None
     st = rlm.State.empty(B, D, 16)
-    cs = rlm.ConvState(to_dev(mx.conv_in, "bf16"))
+    cs = rlm.ConvState(to_dev(mx.conv_in, "bf16")) if K else None
     x1, x2 = x[:, :cut].contiguous(), x[:, cut:].contiguous()
     g1, g2 = g[:, :cut].contiguous(), g[:, cut:].contiguous()
     z1, z2 = torch.empty_like(x1), torch.empty_like(x2)
     rlm.rlm_mixer_prefill(x1, g1, p, local, z1, conv_in=cs, state_out=st, conv_out=cs)
-    n = _launches(lambda: rlm.rlm_mixer_prefill(x2, g2, p, local, z2, state_in=st, conv_in=cs, state_out=st,
-                                                conv_out=cs))
-    assert n == 2
-    zr, sr, tr = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), mx.conv_w, mx.scale, conv_in=mx.conv_in)
+    rlm.rlm_mixer_prefill(x2, g2, p, local, z2, state_in=st, conv_in=cs, state_out=st, conv_out=cs)
+    torch.cuda.synchronize()
+    zr, sr, tr = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), mx.conv_w, mx.scale,
+                                      conv_in=mx.conv_in if K else None)
     assert_close(to_np(torch.cat([z1, z2], 1)), zr, TOL["bf16"], "z")
     s = st.complex().cpu().numpy()
     assert_close(s.real, sr.real, TOL["bf16"], "state re")
     assert_close(s.imag, sr.imag, TOL["bf16"], "state im")
-    np.testing.assert_array_equal(to_np(cs.u), tr)
+    if K:
+        np.testing.assert_array_equal(to_np(cs.u), tr)
 
 
-def test_fused_mixer_prefill_is_causal_bit_exact():
+@pytest.mark.parametrize("K", [0, 8])
+def test_tcgen05_shape_mixer_prefill_is_causal_bit_exact(K):
     inp = make_inputs(2, 4100, 512, 16, "bf16", seed=14)
-    mx = make_mixer_inputs(inp, 8, seed=14)
+    mx = make_mixer_inputs(inp, K, seed=14)
     x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
     p = rlm.Params.from_arrays(*inp.params())
-    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale) if K else None
     z1, z2 = torch.empty_like(x), torch.empty_like(x)
     rlm.rlm_mixer_prefill(x, g, p, local, z1)
     for t0 in (2048, 2049, 4095):
@@ -268,26 +274,23 @@ def test_fused_mixer_prefill_is_causal_bit_exact():
         assert not torch.equal(z1[:, t0:], z2[:, t0:])
 
 
-def test_fused_and_unfused_mixer_agree():
-    """The same problem through the fused epilogue (D = 512) and, channel group by
-    channel group, through the unfused route (each 64-channel slice is segmented):
-    within one bf16 rounding of z."""
+def test_fused_and_unfused_gate_agree():
+    """The gate through the fused epilogue (D = 512) and, 64 channels at a time,
+    through the segmented prefill and the separate pass: within one bf16 rounding
+    of z (the unfused route rounds y before the gate)."""
     inp = make_inputs(2, 3000, 512, 16, "bf16", seed=3)
-    mx = make_mixer_inputs(inp, 4, seed=3)
+    mx = make_mixer_inputs(inp, 0, seed=3)
     x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
     p = rlm.Params.from_arrays(*inp.params())
-    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
-    hist = to_dev(mx.conv_in, "bf16")
     zf = torch.empty_like(x)
-    rlm.rlm_mixer_prefill(x, g, p, local, zf, conv_in=rlm.ConvState(hist))
+    assert _launches(lambda: rlm.rlm_mixer_prefill(x, g, p, None, zf)) == 1
     zu = torch.empty_like(x)
     for c0 in range(0, 512, 64):
         sl = slice(c0, c0 + 64)
         ps = rlm.Params(*(t[sl].contiguous() for t in (p.decay, p.freq, p.amp, p.phase)))
-        ls = rlm.Local(local.conv_w[sl].contiguous(), local.scale[sl].contiguous())
         zs = torch.empty_like(x[:, :, sl].contiguous())
-        rlm.rlm_mixer_prefill(x[:, :, sl].contiguous(), g[:, :, sl].contiguous(), ps, ls, zs,
-                              conv_in=rlm.ConvState(hist[:, :, sl].contiguous()))
+        assert _launches(lambda: rlm.rlm_mixer_prefill(x[:, :, sl].contiguous(), g[:, :, sl].contiguous(), ps,
+                                                       None, zs)) == 2
         zu[:, :, sl] = zs
     torch.cuda.synchronize()
     d = (zf.float() - zu.float()).abs().max().item()
