@@ -72,11 +72,12 @@ def decode_bytes(B, D, M):
 
 
 def mixer_prefill_bytes(B, L, D, M, K):
-    """Algorithmic HBM bytes of one fused mixer prefill (Sec. 3.4): read x and g,
-    write z (bf16, 6 B per token-channel), the state and parameters as for the
-    prefill, the drive history in and out (2 B per (b, k, d)) and the local-path
-    weights (4 B per (d, k) and per d)."""
-    return prefill_bytes(B, L, D, M) + 2 * B * L * D + 2 * 2 * B * (K - 1) * D + 4 * D * (K + 1)
+    """Algorithmic HBM bytes of one mixer prefill (Sec. 3.4): read x and g, write z
+    (bf16, 6 B per token-channel), the state and parameters as for the prefill,
+    and with a local path (K > 0) the drive history in and out (2 B per (b, k, d))
+    and its weights (4 B per (d, k) and per d)."""
+    extra = 2 * 2 * B * (K - 1) * D + 4 * D * (K + 1) if K > 0 else 0
+    return prefill_bytes(B, L, D, M) + 2 * B * L * D + extra
 
 
 def mixer_decode_bytes(B, D, M, K):
@@ -442,10 +443,11 @@ def _bench_decode(rlm, torch, dev, hbm_peak):
             "bytes_per_step": per_step, "launches": T}
 
 
-def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms):
-    """The mixer wrapper of Sec. 3.4 (gate, local path K = 4, drive history in and
-    out) on the headline prefill shape, fused into the tcgen05 prefill, and its
-    decode step (B = 64) in a CUDA graph."""
+def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
+    """The mixer wrapper of Sec. 3.4 on the headline prefill shape: the gate alone
+    (fused into the tcgen05 prefill) and the gate with the local path K = 4 and
+    drive history (the prefill, then one full-width pass); and the fused decode
+    step (B = 64) in a CUDA graph."""
     from synth import make_inputs, make_mixer_inputs
     P = MIXER
     B, L, D, M, K = P["B"], P["L"], P["D"], P["M"], P["K"]
@@ -463,33 +465,44 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms):
     work = torch.empty(max(wsz, 256), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
-    def call():
-        rlm.rlm_mixer_prefill(x, g, p, local, z, conv_in=hin, state_out=st, conv_out=hout, workspace=work)
+    def measure(kk):
+        loc = local if kk else None
 
-    for _ in range(3):
-        flush.zero_()
-        call()
-    torch.cuda.synchronize()
-    ts = []
-    n0 = rlm.rlm_kernels_launched()
-    for _ in range(10):
-        flush.zero_()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        call()
-        b.record(stream)
+        def call():
+            rlm.rlm_mixer_prefill(x, g, p, loc, z, conv_in=hin if kk else None, state_out=st,
+                                  conv_out=hout if kk else None, workspace=work)
+
+        for _ in range(3):
+            flush.zero_()
+            call()
         torch.cuda.synchronize()
-        ts.append(a.elapsed_time(b))
-    launches = (rlm.rlm_kernels_launched() - n0) // 10
-    ms = statistics.mean(ts)
-    alg = mixer_prefill_bytes(B, L, D, M, K)
-    gbs = alg / (ms * 1e-3) / 1e9
-    prefill = {"workload": f"fused mixer prefill B={B} L={L} D={D} M={M} K={K} bf16, gate and drive history",
-               "ms": round(ms, 5), "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 1),
-               "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
-               "algorithmic_bytes": alg, "launches_per_call": launches,
-               "vs_mix_only": round(ms / mix_ms, 3)}
+        ts = []
+        n0 = rlm.rlm_kernels_launched()
+        for _ in range(10):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            call()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        launches = (rlm.rlm_kernels_launched() - n0) // 10
+        ms = statistics.mean(ts)
+        alg = mixer_prefill_bytes(B, L, D, M, kk)
+        gbs = alg / (ms * 1e-3) / 1e9
+        what = "gate fused into the tcgen05 prefill" if kk == 0 else \
+            f"gate and local path K={kk} with drive history: prefill then one full-width pass"
+        return {"workload": f"mixer prefill B={B} L={L} D={D} M={M} bf16, {what}",
+                "ms": round(ms, 5), "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 1),
+                "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
+                "algorithmic_bytes": alg, "launches_per_call": launches,
+                "vs_mix_only": round(ms / mix_ms, 3)}
+
+    prefill_gate = measure(0)
+    prefill = measure(K)
     del x, g, z, work
+    if not with_decode:
+        return {"prefill_gate": prefill_gate, "prefill": prefill}
 
     Bd, T = P["decode_B"], P["T"]
     dinp = make_inputs(Bd, 1, D, M, "bf16", seed=3, decode_steps=T)
@@ -533,7 +546,7 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms):
     decode = {"workload": f"fused mixer decode B={Bd} D={D} M={M} K={K}, {T} steps, CUDA graph",
               "us_per_step": round(us, 4), "tok_s": round(Bd * T / (dms * 1e-3), 1),
               "achieved_GBps": round(dgbs, 1), "frac_hbm": round(dgbs / hbm_peak, 4), "bytes_per_step": per}
-    return {"prefill": prefill, "decode": decode}
+    return {"prefill_gate": prefill_gate, "prefill": prefill, "decode": decode}
 
 
 def _bench_backward(rlm, torch, dev, hbm_peak, args):
@@ -599,6 +612,41 @@ def run_backward_only(args):
     n0 = rlm.rlm_kernels_launched()
     out = _bench_backward(rlm, torch, dev, hbm_peak, args)
     out.update({"mode": "backward only", "peak_kind": peak_kind,
+                "gpu_launches": rlm.rlm_kernels_launched() - n0})
+    print(json.dumps(out), flush=True)
+
+
+def run_mixer_only(args):
+    """The mixer prefill measurements alone (used for their ncu captures)."""
+    import torch
+
+    import paper_2607_05583_gb300 as rlm
+    from synth import make_inputs
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    rlm.load_library()
+    hbm_peak, _, peak_kind = _peaks()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    P = MIXER
+    inp = make_inputs(P["B"], P["L"], P["D"], P["M"], "bf16", seed=2)
+    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
+    p = rlm.Params.from_arrays(*inp.params(), device=dev)
+    y = torch.empty_like(x)
+    for _ in range(3):
+        rlm.rlm_mix_prefill(x, p, y)
+    ts = []
+    for _ in range(5):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        rlm.rlm_mix_prefill(x, p, y)
+        b.record()
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b))
+    del x, y
+    n0 = rlm.rlm_kernels_launched()
+    out = _bench_mixer(rlm, torch, dev, hbm_peak, flush, statistics.mean(ts), with_decode=False)
+    out.update({"mode": "mixer prefill only", "peak_kind": peak_kind,
                 "gpu_launches": rlm.rlm_kernels_launched() - n0})
     print(json.dumps(out), flush=True)
 
@@ -671,8 +719,8 @@ def main():
     ap.add_argument("--quick", action="store_true", help="prefill only (no sweep/decode/backward)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
-    ap.add_argument("--only", default="all", choices=["all", "backward"],
-                    help="backward: run only the backward measurement (diagnostic)")
+    ap.add_argument("--only", default="all", choices=["all", "backward", "mixer"],
+                    help="backward / mixer: run only that measurement (diagnostic, ncu captures)")
     ap.add_argument("--soak", type=float, default=1.5,
                     help="seconds of untimed prefill before the timed steps (clock sampling)")
     args = ap.parse_args()
@@ -682,6 +730,8 @@ def main():
         run_reference(args)
     elif args.only == "backward":
         run_backward_only(args)
+    elif args.only == "mixer":
+        run_mixer_only(args)
     else:
         run_ours(args)
 
