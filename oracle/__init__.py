@@ -23,10 +23,13 @@ channel innermost):
 * ``kernel_table``   K_d[n] of Eq. 1.
 * ``local_conv``     the local lexical path of Sec. 3.4: causal depthwise
                       convolution of kernel size K over the drive history.
+* ``coupling_matrix`` / ``couple_heads``
+                     head coupling of Sec. 3.4: C = I + lambda_c / sqrt(H) tanh(C~),
+                      ybar_g = sum_h C_gh y_h over head-major channels.
 * ``mixer_prefill`` / ``mixer_decode``
-                     the mixer output of Sec. 3.4 without head coupling
-                      (lambda_c = 0): z = sigmoid(g) * y + s * l, with y the
-                      resonant mixing above (numpy, fp64).
+                     the mixer output of Sec. 3.4: z = sigmoid(g) * ybar + s * l,
+                      with ybar the (optionally coupled) resonant mixing above
+                      (numpy, fp64).
 """
 from __future__ import annotations
 
@@ -230,22 +233,53 @@ def local_conv(u, conv_w, conv_in=None):
     return l, tail
 
 
-def mixer_prefill(x, g, decay, freq, amp, phase, conv_w, scale, state_in=None, conv_in=None):
-    """Mixer output over a sequence (Sec. 3.4 with lambda_c = 0):
-    z_t = sigma(g_t) * y_t + s * l_t, y the resonant mixing of the drive x (O2,
-    from state_in) and l the local path over conv_in || x.  g = None means no gate
-    (gamma = 1).  Returns (z, terminal state [B][D][M] complex, last K-1 drives)."""
+def coupling_matrix(c_raw, lambda_c) -> np.ndarray:
+    """C = I + (lambda_c / sqrt(H)) tanh(C~) of Sec. 3.4, for C~ = c_raw [H][H]."""
+    c = _f64(c_raw)
+    H = c.shape[0]
+    if c.shape != (H, H):
+        raise ValueError("c_raw must be [H][H]")
+    return np.eye(H) + (float(lambda_c) / np.sqrt(H)) * np.tanh(c)
+
+
+def couple_heads(y, C) -> np.ndarray:
+    """ybar[..., g*dh + i] = sum_h C[g, h] y[..., h*dh + i] (Sec. 3.4): the channels of
+    a token are the H heads' dh channels, head-major (d = h*dh + i)."""
+    y, C = _f64(y), _f64(C)
+    H = C.shape[0]
+    D = y.shape[-1]
+    if D % H:
+        raise ValueError("D must be a multiple of H")
+    dh = D // H
+    out = np.zeros_like(y)
+    for g in range(H):
+        for h in range(H):
+            out[..., g * dh:(g + 1) * dh] += C[g, h] * y[..., h * dh:(h + 1) * dh]
+    return out
+
+
+def mixer_prefill(x, g, decay, freq, amp, phase, conv_w, scale, state_in=None, conv_in=None, coupling=None):
+    """Mixer output over a sequence (Sec. 3.4): z_t = sigma(g_t) * ybar_t + s * l_t,
+    ybar the resonant mixing of the drive x (O2, from state_in), coupled across
+    heads when coupling = (c_raw [H][H], lambda_c) is given, and l the local path
+    over conv_in || x.  g = None means no gate (gamma = 1).  Returns (z, terminal
+    state [B][D][M] complex, last K-1 drives)."""
     y, st = rec_prefill(x, decay, freq, amp, phase, state_in=state_in)
+    if coupling is not None:
+        y = couple_heads(y, coupling_matrix(*coupling))
     l, tail = local_conv(x, conv_w, conv_in)
     gate = 1.0 if g is None else sigmoid(g)
     return gate * y + _f64(scale)[None, None, :] * l, st, tail
 
 
-def mixer_decode(state, conv, x_t, g_t, decay, freq, amp, phase, conv_w, scale):
-    """One decode step of the mixer: the recurrence step (Eq. 4-5) and the local
-    path over the K-1 cached drives.  state [B][D][M] complex, conv [B][K-1][D],
-    x_t and g_t [B][D] (g_t None: no gate).  Returns (z_t, new state, new conv)."""
+def mixer_decode(state, conv, x_t, g_t, decay, freq, amp, phase, conv_w, scale, coupling=None):
+    """One decode step of the mixer: the recurrence step (Eq. 4-5), the head
+    coupling (if given), the gate and the local path over the K-1 cached drives.
+    state [B][D][M] complex, conv [B][K-1][D], x_t and g_t [B][D] (g_t None: no
+    gate).  Returns (z_t, new state, new conv)."""
     y, st = rec_decode(state, x_t, decay, freq, amp, phase)
+    if coupling is not None:
+        y = couple_heads(y, coupling_matrix(*coupling))
     x_t = _f64(x_t)
     l, tail = local_conv(x_t[:, None, :], conv_w, conv)
     gate = 1.0 if g_t is None else sigmoid(g_t)

@@ -513,3 +513,45 @@ def test_mixer_split_prefill_and_decode_continue_the_sequence():
         np.testing.assert_allclose(zt, z[:, t], rtol=1e-10, atol=1e-12)
     np.testing.assert_allclose(s, st, rtol=1e-10, atol=1e-12)
     np.testing.assert_array_equal(c, tail)
+
+
+def test_coupling_hand_derived_two_heads():
+    """H = 2, dh = 1: C = [[1, l/sqrt2 tanh a], [l/sqrt2 tanh b, 1]] applied to one
+    token (a transposed C or a dropped identity fails)."""
+    a, b_, lam = 0.7, -1.3, 0.5
+    C = oracle.coupling_matrix([[0.0, a], [b_, 0.0]], lam)
+    k = lam / math.sqrt(2.0)
+    np.testing.assert_allclose(C, [[1.0, k * math.tanh(a)], [k * math.tanh(b_), 1.0]], rtol=1e-15)
+    y = np.array([[[2.0, -3.0]]])
+    yb = oracle.couple_heads(y, C)
+    np.testing.assert_allclose(yb[0, 0], [2.0 + k * math.tanh(a) * -3.0, k * math.tanh(b_) * 2.0 - 3.0], rtol=1e-15)
+
+
+def test_coupling_is_a_head_major_einsum_and_identity_when_off():
+    rng = np.random.default_rng(5)
+    H, dh = 4, 3
+    y = rng.standard_normal((2, 7, H * dh))
+    c_raw = rng.standard_normal((H, H))
+    C = oracle.coupling_matrix(c_raw, 0.8)
+    want = np.einsum("gh,blhi->blgi", C, y.reshape(2, 7, H, dh)).reshape(2, 7, H * dh)
+    np.testing.assert_allclose(oracle.couple_heads(y, C), want, rtol=1e-13, atol=1e-14)
+    # a field living in head 1 only spreads to head g with weight C[g, 1]
+    y1 = np.zeros_like(y)
+    y1[..., dh:2 * dh] = y[..., dh:2 * dh]
+    out = oracle.couple_heads(y1, C)
+    for g in range(H):
+        np.testing.assert_allclose(out[..., g * dh:(g + 1) * dh], C[g, 1] * y[..., dh:2 * dh], rtol=1e-13)
+    np.testing.assert_array_equal(oracle.couple_heads(y, oracle.coupling_matrix(c_raw, 0.0)), y)
+    np.testing.assert_array_equal(oracle.couple_heads(y, oracle.coupling_matrix(np.zeros((H, H)), 0.9)), y)
+
+
+def test_coupled_mixer_decode_continues_the_prefill():
+    inp, mx = _mixer_case(B=2, L=30, D=6, M=2, K=3)
+    cp = (np.random.default_rng(1).standard_normal((3, 3)), 0.6)
+    args = (*inp.params(), mx.conv_w, mx.scale)
+    z, st, tail = oracle.mixer_prefill(inp.x, mx.g, *args, conv_in=mx.conv_in, coupling=cp)
+    z1, s, c = oracle.mixer_prefill(inp.x[:, :25], mx.g[:, :25], *args, conv_in=mx.conv_in, coupling=cp)
+    np.testing.assert_allclose(z1, z[:, :25], rtol=1e-12, atol=1e-12)
+    for t in range(25, 30):
+        zt, s, c = oracle.mixer_decode(s, c, inp.x[:, t], mx.g[:, t], *args, coupling=cp)
+        np.testing.assert_allclose(zt, z[:, t], rtol=1e-10, atol=1e-12)
