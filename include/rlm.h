@@ -212,17 +212,27 @@ RLM_API rlm_status rlm_mix_backward_from(const rlm_tensor *dy, const rlm_tensor 
 RLM_API size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype);
 
 /* ------------------------------------------------------------------ mixer
- * The mixer wrapper of Sec. 3.4 around the operator, with head coupling off
- * (lambda_c = 0, so the coupled field is y itself):
+ * The mixer wrapper of Sec. 3.4 around the operator:
  *
- *   z_t[d] = sigma(g_t[d]) y_t[d] + s[d] l_t[d],   l_t[d] = sum_{k<K} w[d][k] u_{t-k}[d]
+ *   z_t[d] = sigma(g_t[d]) ybar_t[d] + s[d] l_t[d],   l_t[d] = sum_{k<K} w[d][k] u_{t-k}[d]
  *
+ * ybar is y coupled across heads (below), or y itself without coupling.
  * u is the drive (x here), y its resonant mixing (as rlm_mix_prefill_from /
  * rlm_mix_decode compute it), g the gate pre-activation (the gate half of the
  * grouped input projection), sigma the logistic function, and l the local
  * lexical path: a causal depthwise convolution of kernel size K whose output is
  * scaled channel-wise by s.  The output projection that follows z is outside. */
 #define RLM_MAX_LOCAL_K 8
+
+/* Head coupling (Sec. 3.4): C = I + (lambda_c / sqrt(H)) tanh(c_raw) mixes the H
+ * heads of each token, ybar[g*dh + i] = sum_h C[g][h] y[h*dh + i] with dh = D / H:
+ * the D channels are the heads' dh channels, head-major.  c_raw [H][H] fp32
+ * row-major; 1 <= H <= 64, D % H == 0, D <= 8192; lambda_c = 0 is the identity. */
+typedef struct {
+    const float *c_raw;
+    float lambda_c;
+    int H;
+} rlm_coupling;
 
 /* Local lexical path (Sec. 3.4).  conv_w [D][K] fp32: conv_w[d*K + k] multiplies
  * u_{t-k}[d]; scale [D] fp32 (s).  0 <= K <= RLM_MAX_LOCAL_K; K = 0 means no
@@ -249,28 +259,33 @@ typedef struct {
  *             means no gate (sigma(g) taken as 1)
  *   p         resonator parameters
  *   local     nullable (no local path) or K = 0
+ *   coupling  nullable (no coupling)
  *   state_in  nullable; the resonators' state before token 0 (as rlm_mix_prefill_from)
  *   conv_in   nullable; the drive history before token 0 (zero drives if NULL)
  *   z         [B][L][D] output, x's shape and dtype; must not overlap x, g, the
  *             parameters or the states
  *   state_out nullable; terminal state and coefficients (may alias state_in)
  *   conv_out  nullable; the history after token L-1 (may alias conv_in exactly)
- * Workspace: rlm_prefill_workspace_size.  bf16 with M = 16 runs the gate and the
- * local path inside the tcgen05 prefill's epilogue (one pass: x and g in, z out);
- * other paths write the mixing into z and finish z with a separate pass. */
+ * Workspace: rlm_prefill_workspace_size.  With a gate only (no local path, no
+ * coupling), bf16 with M = 16 applies the gate inside the tcgen05 prefill's
+ * epilogue (one pass: x and g in, z out); otherwise the mixing is written into z,
+ * coupled in place (one pass over whole token rows) if asked, and finished by one
+ * full-width pass over x, g and z. */
 RLM_API rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm_params *p,
-                                     const rlm_local *local, const rlm_state *state_in,
+                                     const rlm_local *local, const rlm_coupling *coupling, const rlm_state *state_in,
                                      const rlm_conv_state *conv_in, rlm_tensor *z, rlm_state *state_out,
                                      rlm_conv_state *conv_out, const rlm_launch *launch);
 
 /* One decode step of the mixer: the recurrence step of rlm_mix_decode, the
- * gate, and the local path over the cached history, fused in one kernel.
+ * gate, and the local path over the cached history, fused in one kernel (with
+ * coupling: the recurrence step, then one kernel per batch row for the coupling,
+ * the gate and the local path).
  *   x_t, g_t [B][1][D] (g_t nullable: no gate); state updated in place; conv
  *   ([B][K-1][D], required when K >= 2) shifted in place by one token; z_t
  *   [B][1][D] output.  No workspace. */
 RLM_API rlm_status rlm_mixer_decode(const rlm_tensor *x_t, const rlm_tensor *g_t, rlm_state *state,
-                                    const rlm_local *local, rlm_conv_state *conv, rlm_tensor *z_t,
-                                    const rlm_launch *launch);
+                                    const rlm_local *local, const rlm_coupling *coupling, rlm_conv_state *conv,
+                                    rlm_tensor *z_t, const rlm_launch *launch);
 
 /* ------------------------------------------------------------------ utility
  * rlm_validate_params: copies p to the host (synchronous) and checks that every

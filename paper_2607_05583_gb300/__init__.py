@@ -23,7 +23,8 @@ from . import build as _build_mod
 __all__ = [
     "RlmError", "Params", "Grads", "State", "load_library", "library_path",
     "rlm_mix_prefill", "rlm_mix_prefill_from", "rlm_mix_prefill_noalloc", "rlm_mix_decode", "rlm_mix_backward",
-    "rlm_mix_backward_from", "rlm_state_init", "Local", "ConvState", "rlm_mixer_prefill", "rlm_mixer_decode",
+    "rlm_mix_backward_from", "rlm_state_init", "Local", "ConvState", "Coupling", "rlm_mixer_prefill",
+    "rlm_mixer_decode",
     "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
     "rlm_validate_params", "rlm_get_device_status", "rlm_status_string",
     "rlm_version", "rlm_kernels_launched", "rlm_measure_row_io", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
@@ -56,6 +57,10 @@ class _State(ctypes.Structure):
 class _Local(ctypes.Structure):
     _fields_ = [("conv_w", ctypes.c_void_p), ("scale", ctypes.c_void_p),
                 ("D", ctypes.c_int), ("K", ctypes.c_int)]
+
+
+class _Coupling(ctypes.Structure):
+    _fields_ = [("c_raw", ctypes.c_void_p), ("lambda_c", ctypes.c_float), ("H", ctypes.c_int)]
 
 
 class _ConvState(ctypes.Structure):
@@ -103,9 +108,9 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
                                      P(_Grads), P(_Launch)]
     lib.rlm_mix_backward_from.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_State), P(_State),
                                           P(_Tensor), P(_Grads), P(_State), P(_Launch)]
-    lib.rlm_mixer_prefill.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_Local), P(_State),
+    lib.rlm_mixer_prefill.argtypes = [P(_Tensor), P(_Tensor), P(_Params), P(_Local), P(_Coupling), P(_State),
                                       P(_ConvState), P(_Tensor), P(_State), P(_ConvState), P(_Launch)]
-    lib.rlm_mixer_decode.argtypes = [P(_Tensor), P(_Tensor), P(_State), P(_Local), P(_ConvState),
+    lib.rlm_mixer_decode.argtypes = [P(_Tensor), P(_Tensor), P(_State), P(_Local), P(_Coupling), P(_ConvState),
                                      P(_Tensor), P(_Launch)]
     lib.rlm_state_init.argtypes = [P(_State), P(_Params), P(_Launch)]
     lib.rlm_validate_params.argtypes = [P(_Params)]
@@ -216,6 +221,23 @@ class Local:
         if K == 0:
             return _Local(None, None, int(D), 0)
         return _Local(_ptr(self.conv_w, torch.float32, 2), _ptr(self.scale, torch.float32, 1), int(D), int(K))
+
+
+@dataclass
+class Coupling:
+    """Head coupling of Sec. 3.4: raw matrix c_raw [H][H] (float32 CUDA tensor) and
+    strength lambda_c; C = I + lambda_c / sqrt(H) tanh(c_raw) mixes the heads of
+    head-major channels."""
+    c_raw: torch.Tensor
+    lambda_c: float
+
+    @classmethod
+    def from_arrays(cls, c_raw, lambda_c, device="cuda"):
+        return cls(torch.as_tensor(c_raw, dtype=torch.float32).contiguous().to(device), float(lambda_c))
+
+    def _c(self) -> _Coupling:
+        H = int(self.c_raw.shape[0])
+        return _Coupling(_ptr(self.c_raw, torch.float32, 2), float(self.lambda_c), H)
 
 
 @dataclass
@@ -439,7 +461,8 @@ def rlm_get_device_status(stream=None) -> int:
 def rlm_mixer_prefill(x: torch.Tensor, g: torch.Tensor | None, params: Params, local: Local | None,
                       z: torch.Tensor, state_in: State | None = None, conv_in: ConvState | None = None,
                       state_out: State | None = None, conv_out: ConvState | None = None,
-                      workspace: torch.Tensor | None = None, stream=None) -> None:
+                      workspace: torch.Tensor | None = None, stream=None,
+                      coupling: Coupling | None = None) -> None:
     """Mixer output of Sec. 3.4 over a sequence: z = sigmoid(g) * y + s * (w * x), y the
     resonant mixing of x from ``state_in``; the local path reads its drives before
     token 0 from ``conv_in``.  ``state_out`` / ``conv_out`` receive the terminal
@@ -452,13 +475,14 @@ def rlm_mixer_prefill(x: torch.Tensor, g: torch.Tensor | None, params: Params, l
                                x.device)
     ref = lambda c: ctypes.byref(c) if c is not None else None
     opt = lambda o: ref(o._c()) if o is not None else None
-    _check(lib.rlm_mixer_prefill(ctypes.byref(xt), ref(gt), ctypes.byref(params._c()), opt(local), opt(state_in),
+    _check(lib.rlm_mixer_prefill(ctypes.byref(xt), ref(gt), ctypes.byref(params._c()), opt(local), opt(coupling),
+                                 opt(state_in),
                                  opt(conv_in), ctypes.byref(zt), opt(state_out), opt(conv_out),
                                  ctypes.byref(_launch(stream, workspace))), "rlm_mixer_prefill")
 
 
 def rlm_mixer_decode(x_t: torch.Tensor, g_t: torch.Tensor | None, state: State, local: Local | None,
-                     conv: ConvState | None, z_t: torch.Tensor, stream=None) -> None:
+                     conv: ConvState | None, z_t: torch.Tensor, stream=None, coupling: Coupling | None = None) -> None:
     """One mixer decode step: recurrence, gate and local path in one kernel; the state
     and the drive history advance in place."""
     lib = load_library()
@@ -466,5 +490,6 @@ def rlm_mixer_decode(x_t: torch.Tensor, g_t: torch.Tensor | None, state: State, 
     gt = _field(g_t) if g_t is not None else None
     ref = lambda c: ctypes.byref(c) if c is not None else None
     opt = lambda o: ref(o._c()) if o is not None else None
-    _check(lib.rlm_mixer_decode(ctypes.byref(xt), ref(gt), ctypes.byref(state._c()), opt(local), opt(conv),
+    _check(lib.rlm_mixer_decode(ctypes.byref(xt), ref(gt), ctypes.byref(state._c()), opt(local), opt(coupling),
+                                opt(conv),
                                 ctypes.byref(zt), ctypes.byref(_launch(stream, None))), "rlm_mixer_decode")

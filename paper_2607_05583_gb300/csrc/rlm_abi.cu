@@ -215,6 +215,19 @@ rlm_status check_local(const rlm_local *lc, int64_t D, int *K) {
     return RLM_OK;
 }
 
+// Head coupling: H heads dividing D, a finite strength, the raw matrix present.
+rlm_status check_coupling(const rlm_coupling *cp, int64_t D) {
+    if (!cp) return RLM_OK;
+    if (cp->H < 1 || cp->H > 64) return fail(RLM_ERR_INVALID_ARG, "coupling->H=%d outside 1..64", cp->H);
+    if (D % cp->H != 0)
+        return fail(RLM_ERR_INVALID_ARG, "D=%lld is not a multiple of coupling->H=%d", (long long)D, cp->H);
+    if (D > 8192) return fail(RLM_ERR_UNSUPPORTED, "head coupling supports D <= 8192 (got %lld)", (long long)D);
+    if (!cp->c_raw || !aligned16(cp->c_raw))
+        return fail(RLM_ERR_INVALID_ARG, "coupling->c_raw is NULL or not 16-byte aligned");
+    if (!std::isfinite(cp->lambda_c)) return fail(RLM_ERR_INVALID_ARG, "coupling->lambda_c is not finite");
+    return RLM_OK;
+}
+
 size_t conv_bytes(int64_t B, int64_t D, int K, rlm_dtype dt) {
     return K < 2 ? 0 : (size_t)B * (size_t)(K - 1) * (size_t)D * elem_size(dt);
 }
@@ -294,7 +307,7 @@ rlm_status rlm_mix_prefill_from(const rlm_tensor *x, const rlm_params *p, const 
 }
 
 rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm_params *p, const rlm_local *local,
-                             const rlm_state *state_in, const rlm_conv_state *conv_in, rlm_tensor *z,
+                             const rlm_coupling *coupling, const rlm_state *state_in, const rlm_conv_state *conv_in, rlm_tensor *z,
                              rlm_state *state_out, rlm_conv_state *conv_out, const rlm_launch *ln) {
     rlm_status s;
     if ((s = check_tensor(x, "x")) != RLM_OK) return s;
@@ -312,6 +325,7 @@ rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm
     if ((s = check_prefill_states(x, z, p, state_in, state_out)) != RLM_OK) return s;
     int K = 0;
     if ((s = check_local(local, x->D, &K)) != RLM_OK) return s;
+    if ((s = check_coupling(coupling, x->D)) != RLM_OK) return s;
     if ((s = check_conv(conv_in, x->B, x->D, K, x->dtype, "conv_in")) != RLM_OK) return s;
     if ((s = check_conv(conv_out, x->B, x->D, K, x->dtype, "conv_out")) != RLM_OK) return s;
     const size_t cb = conv_bytes(x->B, x->D, K, x->dtype);
@@ -335,7 +349,8 @@ rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm
     // The gate alone is fused into the tcgen05 prefill's epilogue.  With a local
     // path, the mixing and one full-width pass over x, g and y are faster than
     // the fused kernel (whose 8-channel row slices cap its memory rate).
-    const bool fused = g && K == 0 && path == PrefillPath::kTc && tc_mixer_fused(x->B, x->L, (int)x->D, p->M, x->dtype);
+    const bool fused = g && K == 0 && !coupling && path == PrefillPath::kTc &&
+                       tc_mixer_fused(x->B, x->L, (int)x->D, p->M, x->dtype);
     cudaError_t e;
     if (fused) {
         const TcMix mix{g->ptr};
@@ -346,6 +361,8 @@ rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm
         e = launch_prefill(path, x, p, state_in ? state_in->s : nullptr, z->ptr, state_out ? state_out->s : nullptr,
                            state_out ? state_out->coef : nullptr, ln);
     }
+    if (e == cudaSuccess && coupling)
+        e = couple_heads(z->ptr, x->dtype, coupling->c_raw, coupling->lambda_c, coupling->H, x->B, x->L, (int)x->D, st);
     if (e == cudaSuccess && !fused && (g || K > 0))
         e = mixer_epilogue(x->ptr, g ? g->ptr : nullptr, z->ptr, hin, K > 0 ? local->conv_w : nullptr,
                            K > 0 ? local->scale : nullptr, x->dtype, x->B, x->L, (int)x->D, K, st);
@@ -379,7 +396,7 @@ rlm_status rlm_mix_decode(const rlm_tensor *x_t, rlm_state *state, rlm_tensor *y
 }
 
 rlm_status rlm_mixer_decode(const rlm_tensor *x_t, const rlm_tensor *g_t, rlm_state *state, const rlm_local *local,
-                            rlm_conv_state *conv, rlm_tensor *z_t, const rlm_launch *ln) {
+                            const rlm_coupling *coupling, rlm_conv_state *conv, rlm_tensor *z_t, const rlm_launch *ln) {
     rlm_status s;
     if ((s = check_tensor(x_t, "x_t")) != RLM_OK) return s;
     if ((s = check_tensor(z_t, "z_t")) != RLM_OK) return s;
@@ -404,6 +421,7 @@ rlm_status rlm_mixer_decode(const rlm_tensor *x_t, const rlm_tensor *g_t, rlm_st
         return fail(RLM_ERR_INVALID_ARG, "state overlaps x_t, g_t or z_t");
     int K = 0;
     if ((s = check_local(local, x_t->D, &K)) != RLM_OK) return s;
+    if ((s = check_coupling(coupling, x_t->D)) != RLM_OK) return s;
     if (K >= 2 && !conv) return fail(RLM_ERR_INVALID_ARG, "conv is NULL but the local path has K=%d", K);
     if ((s = check_conv(conv, x_t->B, x_t->D, K, x_t->dtype, "conv")) != RLM_OK) return s;
     if (K >= 2) {
@@ -412,10 +430,22 @@ rlm_status rlm_mixer_decode(const rlm_tensor *x_t, const rlm_tensor *g_t, rlm_st
             (g_t && overlap(conv->u, cb, g_t->ptr, tensor_bytes(g_t))) || overlap(conv->u, cb, state->s, sbytes))
             return fail(RLM_ERR_INVALID_ARG, "conv overlaps x_t, g_t, z_t or the state");
     }
-    cudaError_t e = mixer_decode_step(x_t->ptr, g_t ? g_t->ptr : nullptr, z_t->ptr, x_t->dtype, (int)x_t->B,
-                                      (int)x_t->D, state->M, state->s, state->coef, K >= 2 ? conv->u : nullptr,
-                                      K > 0 ? local->conv_w : nullptr, K > 0 ? local->scale : nullptr, K,
-                                      static_cast<cudaStream_t>(ln->stream));
+    cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
+    cudaError_t e;
+    if (coupling) {
+        // The recurrence step writes y_t into z_t; one block per batch row then
+        // couples the heads and applies the gate and the local path.
+        e = decode_step(x_t->ptr, z_t->ptr, x_t->dtype, (int)x_t->B, (int)x_t->D, state->M, state->s, state->coef, st);
+        if (e == cudaSuccess)
+            e = mixer_finish_coupled(x_t->ptr, g_t ? g_t->ptr : nullptr, z_t->ptr, K >= 2 ? conv->u : nullptr,
+                                     K > 0 ? local->conv_w : nullptr, K > 0 ? local->scale : nullptr, K,
+                                     coupling->c_raw, coupling->lambda_c, coupling->H, x_t->dtype, (int)x_t->B,
+                                     (int)x_t->D, st);
+    } else {
+        e = mixer_decode_step(x_t->ptr, g_t ? g_t->ptr : nullptr, z_t->ptr, x_t->dtype, (int)x_t->B, (int)x_t->D,
+                              state->M, state->s, state->coef, K >= 2 ? conv->u : nullptr,
+                              K > 0 ? local->conv_w : nullptr, K > 0 ? local->scale : nullptr, K, st);
+    }
     if (e != cudaSuccess) return cuda_fail(e, "rlm_mixer_decode launch");
     return RLM_OK;
 }

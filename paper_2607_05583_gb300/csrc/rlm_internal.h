@@ -85,6 +85,15 @@ cudaError_t mixer_decode_step(const void *x_t, const void *g_t, void *z_t, rlm_d
 cudaError_t mixer_epilogue(const void *x, const void *g, void *z, const void *hist, const float *conv_w,
                            const float *scale, rlm_dtype dt, int64_t B, int64_t L, int D, int K,
                            cudaStream_t st);
+// Head coupling (Sec. 3.4) in place over z [B][L][D]: ybar = C y per token,
+// C = I + lambda_c / sqrt(H) tanh(c_raw), channels head-major.
+cudaError_t couple_heads(void *z, rlm_dtype dt, const float *c_raw, float lambda_c, int H, int64_t B, int64_t L,
+                         int D, cudaStream_t st);
+// One mixer decode step after the recurrence step wrote y_t into z_t: coupling,
+// gate (g_t nullable), local path (K = 0: none) with the history shift.
+cudaError_t mixer_finish_coupled(const void *x_t, const void *g_t, void *z_t, void *hist, const float *conv_w,
+                                 const float *scale, int K, const float *c_raw, float lambda_c, int H, rlm_dtype dt,
+                                 int B, int D, cudaStream_t st);
 // out = the last K-1 drives of hist || x (out may alias hist; no-op for K < 2).
 cudaError_t conv_tail(const void *x, const void *hist, void *out, rlm_dtype dt, int64_t B, int64_t L, int D,
                       int K, cudaStream_t st);

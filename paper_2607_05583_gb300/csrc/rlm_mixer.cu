@@ -12,6 +12,8 @@
 // memory, and writes z.  The kernel size K is a template parameter (2 K weights per
 // thread in registers).  The pass moves 8 (bf16) or 16 (fp32) bytes per
 // token-channel: read x, g and y, write z.
+#include <algorithm>
+
 #include "rlm_device.cuh"
 #include "rlm_internal.h"
 
@@ -105,6 +107,87 @@ __global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__
     }
 }
 
+// Head coupling (Sec. 3.4): C = I + (lambda_c / sqrt(H)) tanh(c_raw), built per
+// block in shared memory.
+__device__ __forceinline__ void build_coupling(float *C, const float *c_raw, float lam, int H) {
+    const float k = lam * rsqrtf((float)H);
+    for (int i = threadIdx.x; i < H * H; i += blockDim.x)
+        C[i] = (i / H == i % H ? 1.0f : 0.0f) + k * tanhf(__ldg(c_raw + i));
+}
+
+__device__ __forceinline__ float as_f(float v) { return v; }
+__device__ __forceinline__ float as_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+
+// k_couple: ybar = C y in place over z.  A block stages `rows` whole token rows of
+// one batch row (16-byte loads) and writes them back coupled; a warp covers
+// consecutive channels of one head, so its reads of each source head are
+// contiguous in shared memory.
+template <typename T>
+__global__ void __launch_bounds__(kBlock) k_couple(T *z, const float *__restrict__ c_raw, float lam, int H,
+                                                   int64_t L, int D, int rows) {
+    extern __shared__ __align__(16) uint8_t sm[];
+    float *C = reinterpret_cast<float *>(sm);
+    T *ys = reinterpret_cast<T *>(sm + ((H * H * 4 + 15) & ~15));
+    const int64_t b = blockIdx.y, t0 = (int64_t)blockIdx.x * rows;
+    const int n = (int)(L - t0 < rows ? L - t0 : rows);
+    T *zb = z + (b * L + t0) * D;
+    build_coupling(C, c_raw, lam, H);
+    constexpr int kVE = 16 / sizeof(T);
+    for (int i = threadIdx.x; i < n * D / kVE; i += kBlock)
+        reinterpret_cast<uint4 *>(ys)[i] = reinterpret_cast<const uint4 *>(zb)[i];
+    __syncthreads();
+    const int dh = D / H;
+    for (int i = threadIdx.x; i < n * D; i += kBlock) {
+        const int t = i / D, d = i % D, gh = d / dh, j = d % dh;
+        const T *row = ys + (int64_t)t * D + j;
+        const float *Cg = C + gh * H;
+        float acc = 0.0f;
+        for (int h = 0; h < H; ++h) acc = fmaf(Cg[h], as_f(row[h * dh]), acc);
+        st_elem(zb + i, acc);
+    }
+}
+
+// k_mixer_finish: one decode step's mixer for one batch row, after the recurrence
+// step wrote y_t into z_t: coupling, gate, local path (the thread of channel d
+// owns its history column, so it reads it all before shifting it).
+template <typename T>
+__global__ void __launch_bounds__(kBlock) k_mixer_finish(const T *__restrict__ x_t, const T *__restrict__ g_t,
+                                                         T *__restrict__ z_t, T *hist,
+                                                         const float *__restrict__ conv_w,
+                                                         const float *__restrict__ scale, int K,
+                                                         const float *__restrict__ c_raw, float lam, int H, int D) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" :::);
+    extern __shared__ __align__(16) uint8_t sm[];
+    float *C = reinterpret_cast<float *>(sm);
+    float *ys = C + ((H * H + 3) & ~3);
+    const int64_t b = blockIdx.x;
+    build_coupling(C, c_raw, lam, H);
+    for (int d = threadIdx.x; d < D; d += kBlock) ys[d] = as_f(z_t[b * D + d]);
+    __syncthreads();
+    const int dh = D / H;
+    for (int d = threadIdx.x; d < D; d += kBlock) {
+        const int gh = d / dh, j = d % dh;
+        float v = 0.0f;
+        for (int h = 0; h < H; ++h) v = fmaf(C[gh * H + h], ys[h * dh + j], v);
+        if (g_t) v *= gatef(as_f(g_t[b * D + d]));
+        if (K > 0) {
+            const float xv = as_f(x_t[b * D + d]);
+            float l = __ldg(conv_w + (int64_t)d * K) * xv;
+            T *hc = hist + b * (K - 1) * (int64_t)D + d;    // entry j: u_{t-(K-1-j)}
+            T hv[kMaxK];
+            for (int j2 = 0; j2 < K - 1; ++j2) {
+                hv[j2] = hc[(int64_t)j2 * D];
+                l = fmaf(__ldg(conv_w + (int64_t)d * K + (K - 1 - j2)), as_f(hv[j2]), l);
+            }
+            for (int j2 = 1; j2 < K - 1; ++j2) hc[(int64_t)(j2 - 1) * D] = hv[j2];
+            if (K > 1) hc[(int64_t)(K - 2) * D] = x_t[b * D + d];
+            v = fmaf(__ldg(scale + d), l, v);
+        }
+        st_elem(z_t + b * D + d, v);
+    }
+}
+
 // The history after the last token: entry j is element L + j of history || x.
 // One thread per (b, d) reads all K-1 values before writing, so out may alias in.
 template <typename T>
@@ -175,6 +258,51 @@ cudaError_t mixer_epilogue(const void *x, const void *g, void *z, const void *hi
                            cudaStream_t st) {
     if (dt == RLM_BF16) return epilogue_t<__nv_bfloat16>(x, g, z, hist, conv_w, scale, B, L, D, K, st);
     return epilogue_t<float>(x, g, z, hist, conv_w, scale, B, L, D, K, st);
+}
+
+namespace {
+template <typename T>
+cudaError_t couple_t(void *z, const float *c_raw, float lam, int H, int64_t B, int64_t L, int D, cudaStream_t st) {
+    // Whole rows of one batch row per block, up to 16 KB of them.
+    const int rows = (int)std::max<int64_t>(1, std::min<int64_t>(64, 16384 / ((int64_t)D * sizeof(T))));
+    const size_t smem = ((H * H * 4 + 15) & ~15) + (size_t)rows * D * sizeof(T);
+    const dim3 grid((unsigned)((L + rows - 1) / rows), (unsigned)B);
+    k_couple<T><<<grid, kBlock, smem, st>>>(static_cast<T *>(z), c_raw, lam, H, L, D, rows);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t finish_t(const void *x_t, const void *g_t, void *z_t, void *hist, const float *conv_w, const float *scale,
+                     int K, const float *c_raw, float lam, int H, int B, int D, cudaStream_t st) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)B);
+    cfg.blockDim = dim3(kBlock);
+    cfg.dynamicSmemBytes = ((H * H + 3) & ~3) * 4 + (size_t)D * 4;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    count_launches(1);
+    return cudaLaunchKernelEx(&cfg, k_mixer_finish<T>, static_cast<const T *>(x_t), static_cast<const T *>(g_t),
+                              static_cast<T *>(z_t), static_cast<T *>(hist), conv_w, scale, K, c_raw, lam, H, D);
+}
+}  // namespace
+
+cudaError_t couple_heads(void *z, rlm_dtype dt, const float *c_raw, float lambda_c, int H, int64_t B, int64_t L,
+                         int D, cudaStream_t st) {
+    if (dt == RLM_BF16) return couple_t<__nv_bfloat16>(z, c_raw, lambda_c, H, B, L, D, st);
+    return couple_t<float>(z, c_raw, lambda_c, H, B, L, D, st);
+}
+
+cudaError_t mixer_finish_coupled(const void *x_t, const void *g_t, void *z_t, void *hist, const float *conv_w,
+                                 const float *scale, int K, const float *c_raw, float lambda_c, int H, rlm_dtype dt,
+                                 int B, int D, cudaStream_t st) {
+    if (dt == RLM_BF16)
+        return finish_t<__nv_bfloat16>(x_t, g_t, z_t, hist, conv_w, scale, K, c_raw, lambda_c, H, B, D, st);
+    return finish_t<float>(x_t, g_t, z_t, hist, conv_w, scale, K, c_raw, lambda_c, H, B, D, st);
 }
 
 cudaError_t conv_tail(const void *x, const void *hist, void *out, rlm_dtype dt, int64_t B, int64_t L, int D,

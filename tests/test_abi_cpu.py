@@ -230,8 +230,8 @@ def test_mixer_rejects_bad_arguments_on_host(lib):
     def conv(ptr=cbase, b=B, d=D, k=K, dt=rlm.RLM_BF16):
         return rlm._ConvState(ptr, dt, b, d, k)
 
-    def call(gt=g, lc=None, cin=None, zt=z, cout=None):
-        return lib.rlm_mixer_prefill(ctypes.byref(x), ref(gt), ctypes.byref(p), ref(lc), None, ref(cin),
+    def call(gt=g, lc=None, cin=None, zt=z, cout=None, cp=None):
+        return lib.rlm_mixer_prefill(ctypes.byref(x), ref(gt), ctypes.byref(p), ref(lc), ref(cp), None, ref(cin),
                                      ctypes.byref(zt), None, ref(cout), ctypes.byref(ln))
 
     assert call(lc=local(k=RLM_MAX_K + 1)) == rlm.RLM_ERR_INVALID_ARG          # K too large
@@ -245,9 +245,14 @@ def test_mixer_rejects_bad_arguments_on_host(lib):
     assert call(lc=local(), cin=conv(ptr=cbase + 8)) == rlm.RLM_ERR_INVALID_ARG   # misaligned
     assert call(lc=local(), cin=conv(), cout=conv(ptr=cbase + 64)) == rlm.RLM_ERR_INVALID_ARG  # partial overlap
     assert call(lc=local(), cout=conv(ptr=z.ptr)) == rlm.RLM_ERR_INVALID_ARG     # history overlaps z
+    cpl = lambda h=4, ptr=wbase + 8192, lam=0.5: rlm._Coupling(ptr, lam, h)
+    assert call(cp=cpl(h=3)) == rlm.RLM_ERR_INVALID_ARG                          # D % H != 0
+    assert call(cp=cpl(h=65)) == rlm.RLM_ERR_INVALID_ARG                         # H > 64
+    assert call(cp=cpl(ptr=0)) == rlm.RLM_ERR_INVALID_ARG                        # no matrix
+    assert call(cp=cpl(lam=float("nan"))) == rlm.RLM_ERR_INVALID_ARG             # strength not finite
     st = rlm._State(FAKE + (1 << 33), FAKE + (1 << 33) + (1 << 20), B, D, M)
     x1, z1 = _t(FAKE, B, 1, D), _t(FAKE + (1 << 30), B, 1, D)
-    dec = lambda lc, cv: lib.rlm_mixer_decode(ctypes.byref(x1), None, ctypes.byref(st), ref(lc), ref(cv),
+    dec = lambda lc, cv: lib.rlm_mixer_decode(ctypes.byref(x1), None, ctypes.byref(st), ref(lc), None, ref(cv),
                                               ctypes.byref(z1), ctypes.byref(ln))
     assert dec(local(), None) == rlm.RLM_ERR_INVALID_ARG                         # history required for K >= 2
     assert dec(local(), conv(b=B + 1)) == rlm.RLM_ERR_INVALID_ARG

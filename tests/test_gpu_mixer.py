@@ -295,3 +295,78 @@ def test_fused_and_unfused_gate_agree():
     torch.cuda.synchronize()
     d = (zf.float() - zu.float()).abs().max().item()
     assert d <= 2.0 ** -6 * zu.float().abs().max().item(), d
+
+
+# ---- head coupling (NEXT 3): C = I + lambda_c/sqrt(H) tanh(C~) before the gate
+def _coupling(H, seed, lam=0.7):
+    return np.random.default_rng(seed).standard_normal((H, H)), lam
+
+
+@pytest.mark.parametrize("B,L,D,M,K,H,dtype,with_g", [
+    (2, 3001, 64, 16, 4, 8, "bf16", True),          # tcgen05 prefill (segmented), K = 4
+    (2, 2 * 2048 + 77, 512, 16, 0, 8, "bf16", True), # unsegmented shape: the gate is not fused with coupling
+    (2, 1000, 16, 7, 3, 4, "f32", True),             # SIMT, fp32
+    (1, 700, 8, 40, 2, 2, "bf16", False),            # SIMT, bf16 with M > 32, no gate
+    (2, 1000, 32, 32, 0, 1, "bf16", True),           # time-reversed prefill, H = 1 (a scalar gain)
+])
+def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
+    inp = make_inputs(B, L, D, M, dtype, seed=L + H)
+    mx = make_mixer_inputs(inp, K, seed=L + H)
+    c_raw, lam = _coupling(H, H)
+    x = to_dev(inp.x, dtype)
+    g = to_dev(mx.g, dtype) if with_g else None
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale) if K else None
+    cin = rlm.ConvState(to_dev(mx.conv_in, dtype)) if K else None
+    so = rlm.State.empty(B, D, M)
+    z = torch.empty_like(x)
+    rlm.rlm_mixer_prefill(x, g, p, local, z, conv_in=cin, state_out=so,
+                          coupling=rlm.Coupling.from_arrays(c_raw, lam))
+    torch.cuda.synchronize()
+    zr, sr, _ = oracle.mixer_prefill(inp.x, mx.g if with_g else None, *inp.params(), mx.conv_w, mx.scale,
+                                     conv_in=mx.conv_in if K else None, coupling=(c_raw, lam))
+    assert_close(to_np(z), zr, TOL[dtype], "z")
+    s = so.complex().cpu().numpy()
+    assert_close(s.real, sr.real, TOL[dtype], "state re")
+
+
+@pytest.mark.parametrize("dtype,M,K,H", [("bf16", 16, 4, 8), ("f32", 7, 3, 4), ("bf16", 16, 0, 2), ("bf16", 2, 8, 16)])
+def test_coupled_mixer_decode_continues_the_prefill(dtype, M, K, H):
+    B, D, L0, T = 3, 64, 300, 30
+    inp = make_inputs(B, L0 + T, D, M, dtype, seed=M + K + H)
+    mx = make_mixer_inputs(inp, K, seed=M + K + H)
+    c_raw, lam = _coupling(H, 3 * H)
+    cp = rlm.Coupling.from_arrays(c_raw, lam)
+    x, g = to_dev(inp.x, dtype), to_dev(mx.g, dtype)
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale) if K else None
+    st = rlm.State.empty(B, D, M)
+    cs = rlm.ConvState.empty(B, D, max(K, 1), dtype=x.dtype)
+    z0 = torch.empty_like(x[:, :L0])
+    rlm.rlm_mixer_prefill(x[:, :L0].contiguous(), g[:, :L0].contiguous(), p, local, z0, state_out=st,
+                          conv_out=cs if K else None, coupling=cp)
+    zs = []
+    for t in range(L0, L0 + T):
+        zt = torch.empty_like(x[:, t])
+        rlm.rlm_mixer_decode(x[:, t].contiguous(), g[:, t].contiguous(), st, local, cs if K else None, zt,
+                             coupling=cp)
+        zs.append(zt)
+    torch.cuda.synchronize()
+    zr, sr, tr = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), mx.conv_w, mx.scale, coupling=(c_raw, lam))
+    assert_close(to_np(z0), zr[:, :L0], TOL[dtype], "prefill z")
+    assert_close(to_np(torch.stack(zs, 1)), zr[:, L0:], TOL[dtype], "decode z")
+    if K > 1:
+        np.testing.assert_array_equal(to_np(cs.u), tr)
+
+
+def test_zero_strength_coupling_is_no_coupling():
+    inp = make_inputs(2, 3001, 64, 16, "bf16", seed=6)
+    mx = make_mixer_inputs(inp, 4, seed=6)
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    z0, z1 = torch.empty_like(x), torch.empty_like(x)
+    rlm.rlm_mixer_prefill(x, g, p, local, z0)
+    rlm.rlm_mixer_prefill(x, g, p, local, z1, coupling=rlm.Coupling.from_arrays(np.ones((8, 8)), 0.0))
+    torch.cuda.synchronize()
+    assert torch.equal(z0, z1)
