@@ -44,7 +44,7 @@ METRIC = "mix prefill Mtok/s at L=32K (% of roofline); decode tok/s at B=64 (% H
 PREFILL = dict(B=4, L=32768, D=256, M=16)
 DECODE = dict(B=64, L=32768, D=256, M=16, T=4096)
 BACKWARD = dict(B=4, L=32768, D=512, M=32)
-MIXER = dict(B=4, L=32768, D=256, M=16, K=4, decode_B=64, T=4096)
+MIXER = dict(B=4, L=32768, D=256, M=16, K=4, H=8, decode_B=64, T=4096)
 L2_FLUSH_BYTES = 512 << 20
 
 
@@ -465,12 +465,15 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
     work = torch.empty(max(wsz, 256), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
-    def measure(kk):
+    H = P["H"]
+    coupling = rlm.Coupling.from_arrays(np.random.default_rng(5).standard_normal((H, H)), 0.5, device=dev)
+
+    def measure(kk, cp=None):
         loc = local if kk else None
 
         def call():
             rlm.rlm_mixer_prefill(x, g, p, loc, z, conv_in=hin if kk else None, state_out=st,
-                                  conv_out=hout if kk else None, workspace=work)
+                                  conv_out=hout if kk else None, workspace=work, coupling=cp)
 
         for _ in range(3):
             flush.zero_()
@@ -488,10 +491,12 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
             ts.append(a.elapsed_time(b))
         launches = (rlm.rlm_kernels_launched() - n0) // 10
         ms = statistics.mean(ts)
-        alg = mixer_prefill_bytes(B, L, D, M, kk)
+        alg = mixer_prefill_bytes(B, L, D, M, kk) + (4 * H * H if cp is not None else 0)
         gbs = alg / (ms * 1e-3) / 1e9
         what = "gate fused into the tcgen05 prefill" if kk == 0 else \
             f"gate and local path K={kk} with drive history: prefill then one full-width pass"
+        if cp is not None:
+            what = f"head coupling H={H}, " + what.replace("prefill then one", "prefill, a coupling pass, then one")
         return {"workload": f"mixer prefill B={B} L={L} D={D} M={M} bf16, {what}",
                 "ms": round(ms, 5), "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 1),
                 "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
@@ -500,9 +505,10 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
 
     prefill_gate = measure(0)
     prefill = measure(K)
+    prefill_coupled = measure(K, coupling)
     del x, g, z, work
     if not with_decode:
-        return {"prefill_gate": prefill_gate, "prefill": prefill}
+        return {"prefill_gate": prefill_gate, "prefill": prefill, "prefill_coupled": prefill_coupled}
 
     Bd, T = P["decode_B"], P["T"]
     dinp = make_inputs(Bd, 1, D, M, "bf16", seed=3, decode_steps=T)
@@ -528,25 +534,37 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
     with torch.cuda.graph(graph):
         for t in range(T):
             rlm.rlm_mixer_decode(toks[t], gts[t], dst, dlocal, hist, outs[t])
-    res = []
-    for rep in range(4):
-        dst.s.copy_(s0)
-        torch.cuda.synchronize()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        graph.replay()
-        b.record(stream)
-        torch.cuda.synchronize()
-        if rep:
-            res.append(a.elapsed_time(b))
-    dms = statistics.median(res)
-    us = dms * 1e3 / T
+    def replay_us(gr):
+        res = []
+        for rep in range(4):
+            dst.s.copy_(s0)
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            gr.replay()
+            b.record(stream)
+            torch.cuda.synchronize()
+            if rep:
+                res.append(a.elapsed_time(b))
+        return statistics.median(res) * 1e3 / T
+
+    us = replay_us(graph)
     per = mixer_decode_bytes(Bd, D, M, K)
     dgbs = per / (us * 1e-6) / 1e9
     decode = {"workload": f"fused mixer decode B={Bd} D={D} M={M} K={K}, {T} steps, CUDA graph",
-              "us_per_step": round(us, 4), "tok_s": round(Bd * T / (dms * 1e-3), 1),
+              "us_per_step": round(us, 4), "tok_s": round(Bd * T / (us * 1e-6), 1),
               "achieved_GBps": round(dgbs, 1), "frac_hbm": round(dgbs / hbm_peak, 4), "bytes_per_step": per}
-    return {"prefill_gate": prefill_gate, "prefill": prefill, "decode": decode}
+    dcp = rlm.Coupling.from_arrays(np.random.default_rng(6).standard_normal((H, H)), 0.5, device=dev)
+    graph_c = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph_c):
+        for t in range(T):
+            rlm.rlm_mixer_decode(toks[t], gts[t], dst, dlocal, hist, outs[t], coupling=dcp)
+    uc = replay_us(graph_c)
+    decode_coupled = {"workload": f"mixer decode with head coupling H={H}, B={Bd} D={D} M={M} K={K}: recurrence "
+                                  f"step, then one block per batch row; {T} steps, CUDA graph",
+                      "us_per_step": round(uc, 4), "tok_s": round(Bd * T / (uc * 1e-6), 1), "launches_per_step": 2}
+    return {"prefill_gate": prefill_gate, "prefill": prefill, "prefill_coupled": prefill_coupled, "decode": decode,
+            "decode_coupled": decode_coupled}
 
 
 def _bench_backward(rlm, torch, dev, hbm_peak, args):

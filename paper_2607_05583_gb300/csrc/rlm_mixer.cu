@@ -147,6 +147,78 @@ __global__ void __launch_bounds__(kBlock) k_couple(T *z, const float *__restrict
     }
 }
 
+// k_couple_small: the same for H <= 16 heads without staging: a thread owns kV
+// consecutive in-head positions j of one token, loads its H head vectors (a warp
+// reads consecutive j, so each head's load is contiguous), forms all H outputs
+// with C from shared memory (broadcast reads) and writes them.
+constexpr int kSmallH = 16;
+
+template <typename T, int kV> struct VecIO;
+template <typename T> struct VecIO<T, 1> {
+    __device__ static void load(const T *p, float (&v)[1]) { v[0] = as_f(*p); }
+    __device__ static void store(T *p, const float (&v)[1]) { st_elem(p, v[0]); }
+};
+template <> struct VecIO<__nv_bfloat16, 4> {
+    __device__ static void load(const __nv_bfloat16 *p, float (&v)[4]) {
+        const uint2 u = *reinterpret_cast<const uint2 *>(p);
+        v[0] = __uint_as_float(u.x << 16); v[1] = __uint_as_float(u.x & 0xFFFF0000u);
+        v[2] = __uint_as_float(u.y << 16); v[3] = __uint_as_float(u.y & 0xFFFF0000u);
+    }
+    __device__ static void store(__nv_bfloat16 *p, const float (&v)[4]) {
+        uint32_t a, b;
+        asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(a) : "f"(v[1]), "f"(v[0]));
+        asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(b) : "f"(v[3]), "f"(v[2]));
+        *reinterpret_cast<uint2 *>(p) = make_uint2(a, b);
+    }
+};
+template <> struct VecIO<float, 4> {
+    __device__ static void load(const float *p, float (&v)[4]) {
+        const float4 u = *reinterpret_cast<const float4 *>(p);
+        v[0] = u.x; v[1] = u.y; v[2] = u.z; v[3] = u.w;
+    }
+    __device__ static void store(float *p, const float (&v)[4]) {
+        *reinterpret_cast<float4 *>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    }
+};
+
+template <typename T, int kV>
+__global__ void __launch_bounds__(kBlock) k_couple_small(T *z, const float *__restrict__ c_raw, float lam, int H,
+                                                         int64_t rows, int D) {
+    __shared__ float C[kSmallH * kSmallH];
+    build_coupling(C, c_raw, lam, H);
+    __syncthreads();
+    const int dh = D / H, nj = dh / kV;
+    const int64_t i = (int64_t)blockIdx.x * kBlock + threadIdx.x;
+    if (i >= rows * nj) return;
+    const int64_t r = i / nj;
+    const int j = (int)(i % nj) * kV;
+    T *row = z + r * D + j;
+    float y[kSmallH][kV];
+#pragma unroll
+    for (int h = 0; h < kSmallH; ++h) {
+        if (h < H) {
+            VecIO<T, kV>::load(row + h * dh, y[h]);
+        } else {
+#pragma unroll
+            for (int e = 0; e < kV; ++e) y[h][e] = 0.0f;
+        }
+    }
+#pragma unroll
+    for (int gh = 0; gh < kSmallH; ++gh) {
+        if (gh >= H) break;
+        float acc[kV];
+#pragma unroll
+        for (int e = 0; e < kV; ++e) acc[e] = 0.0f;
+#pragma unroll
+        for (int h = 0; h < kSmallH; ++h) {
+            const float c = C[gh * H + (h < H ? h : 0)];
+#pragma unroll
+            for (int e = 0; e < kV; ++e) acc[e] = fmaf(c, y[h][e], acc[e]);
+        }
+        VecIO<T, kV>::store(row + gh * dh, acc);
+    }
+}
+
 // k_mixer_finish: one decode step's mixer for one batch row, after the recurrence
 // step wrote y_t into z_t: coupling, gate, local path (the thread of channel d
 // owns its history column, so it reads it all before shifting it).
@@ -263,6 +335,17 @@ cudaError_t mixer_epilogue(const void *x, const void *g, void *z, const void *hi
 namespace {
 template <typename T>
 cudaError_t couple_t(void *z, const float *c_raw, float lam, int H, int64_t B, int64_t L, int D, cudaStream_t st) {
+    if (H <= kSmallH) {
+        const int dh = D / H;
+        const int64_t n = B * L * (dh % 4 == 0 ? dh / 4 : dh);
+        const unsigned grid = (unsigned)((n + kBlock - 1) / kBlock);
+        if (dh % 4 == 0)
+            k_couple_small<T, 4><<<grid, kBlock, 0, st>>>(static_cast<T *>(z), c_raw, lam, H, B * L, D);
+        else
+            k_couple_small<T, 1><<<grid, kBlock, 0, st>>>(static_cast<T *>(z), c_raw, lam, H, B * L, D);
+        count_launches(1);
+        return cudaGetLastError();
+    }
     // Whole rows of one batch row per block, up to 16 KB of them.
     const int rows = (int)std::max<int64_t>(1, std::min<int64_t>(64, 16384 / ((int64_t)D * sizeof(T))));
     const size_t smem = ((H * H * 4 + 15) & ~15) + (size_t)rows * D * sizeof(T);

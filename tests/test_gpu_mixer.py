@@ -308,6 +308,8 @@ def _coupling(H, seed, lam=0.7):
     (2, 1000, 16, 7, 3, 4, "f32", True),             # SIMT, fp32
     (1, 700, 8, 40, 2, 2, "bf16", False),            # SIMT, bf16 with M > 32, no gate
     (2, 1000, 32, 32, 0, 1, "bf16", True),           # time-reversed prefill, H = 1 (a scalar gain)
+    (2, 1000, 24, 16, 4, 8, "bf16", True),           # head width 3: one position per thread
+    (2, 1000, 64, 16, 2, 32, "f32", True),           # 32 heads: whole rows staged in shared memory
 ])
 def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
     inp = make_inputs(B, L, D, M, dtype, seed=L + H)
