@@ -319,6 +319,8 @@ def run_ours(args):
     backward = None if args.quick else _bench_backward(rlm, torch, dev, hbm_peak, args)
     # ---------------- mixer wrapper (gate + local path, fused)
     mixer = None if args.quick else _bench_mixer(rlm, torch, dev, hbm_peak, flush, ms)
+    # ---------------- the paper's tied heads, and its FFT evaluation as the comparison
+    paper_form = None if args.quick else _bench_tied_and_fft(rlm, torch, dev, hbm_peak, flush)
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu:
@@ -337,6 +339,7 @@ def run_ours(args):
             "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": n_launch,
             "clocks": clk.summary(), "sweep": sweep, "decode": decode, "backward": backward, "mixer": mixer,
+            "paper_form": paper_form,
         }
         print(json.dumps(line), flush=True)
     if ws > 1:
@@ -565,6 +568,67 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
                       "us_per_step": round(uc, 4), "tok_s": round(Bd * T / (uc * 1e-6), 1), "launches_per_step": 2}
     return {"prefill_gate": prefill_gate, "prefill": prefill, "prefill_coupled": prefill_coupled, "decode": decode,
             "decode_coupled": decode_coupled}
+
+
+def _bench_tied_and_fft(rlm, torch, dev, hbm_peak, flush):
+    """The paper's tied heads (Sec. 3.1: H = 8 heads x 32 channels, one mode, no
+    amplitude) on the long-context shape through the library (the tcgen05 prefill
+    with M = 1), and the paper's own evaluation of Eq. 2 by FFT (Eq. 3: zero
+    padding to a power of two; cuFFT through torch.fft in fp32) on the same drive
+    and kernels, timed as the prior-art comparison and checked against the
+    library's output."""
+    B, L, H, dh = 4, 32768, 8, 32
+    D = H * dh
+    rng = np.random.default_rng(9)
+    alpha = np.exp(rng.uniform(np.log(1e-3), np.log(0.3), H)).astype(np.float32)
+    omega = rng.uniform(0.0, np.pi, H).astype(np.float32)
+    phi = rng.uniform(-np.pi, np.pi, H).astype(np.float32)
+    x = torch.randn(B, L, D, device=dev).to(torch.bfloat16)
+    p = rlm.Params.tied_heads(alpha, omega, phi, dh, device=dev)
+    y = torch.empty_like(x)
+    stream = torch.cuda.current_stream()
+
+    def timed(fn, reps=8):
+        for _ in range(3):
+            flush.zero_()
+            fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(reps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        return statistics.mean(ts)
+
+    ms = timed(lambda: rlm.rlm_mix_prefill(x, p, y))
+    alg = prefill_bytes(B, L, D, 1)
+    tied = {"workload": f"tied heads B={B} L={L} H={H} d_h={dh} (one mode per head, A = 1), bf16",
+            "ms": round(ms, 5), "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 1),
+            "frac_hbm": round(alg / (ms * 1e-3) / 1e9 / hbm_peak, 4)}
+    nfft = 1 << (2 * L - 1).bit_length()
+    n = torch.arange(L, device=dev, dtype=torch.float32)
+    a_t, w_t, f_t = (torch.from_numpy(v).to(dev)[:, None] for v in (alpha, omega, phi))
+    k = torch.exp(-a_t * n) * torch.cos(w_t * n + f_t)                       # [H][L], Sec. 3.1
+    out = {}
+
+    def fft_route():
+        kf = torch.fft.rfft(k, nfft)
+        xf = torch.fft.rfft(x.float().view(B, L, H, dh).permute(0, 2, 3, 1), nfft)
+        yh = torch.fft.irfft(xf * kf[None, :, None, :], nfft)[..., :L]
+        out["y"] = yh.permute(0, 3, 1, 2).reshape(B, L, D).to(torch.bfloat16)
+
+    fms = timed(fft_route, reps=4)
+    d = (out["y"].float() - y.float()).norm() / y.float().norm()
+    fft = {"workload": "the same problem by Eq. 3: rfft of drive and kernels (zero padded to "
+                       f"{nfft}), product, irfft, fp32 (cuFFT through torch.fft)",
+           "ms": round(fms, 4), "Mtok_s": round(B * L / (fms * 1e-3) / 1e6, 1),
+           "rel_l2_vs_library": round(float(d), 6), "library_speedup": round(fms / ms, 1)}
+    del x, y, out
+    return {"tied_heads": tied, "fft_eq3": fft}
 
 
 def _bench_backward(rlm, torch, dev, hbm_peak, args):

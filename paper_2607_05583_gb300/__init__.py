@@ -162,6 +162,17 @@ class Params:
         t = lambda a: torch.as_tensor(a, dtype=torch.float32).contiguous().to(device)
         return cls(t(decay), t(freq), t(amp), t(phase))
 
+    @classmethod
+    def tied_heads(cls, decay, freq, phase, d_h: int, device="cuda"):
+        """The paper's parameterisation (Sec. 3.1): one damped mode per head, no
+        amplitude (A = 1), shared by the head's d_h channels (head-major).  decay,
+        freq, phase: [H].  Gives [H * d_h][1] parameters, which the bf16 prefill
+        runs on its tcgen05 path (M = 1)."""
+        t = lambda a: torch.as_tensor(a, dtype=torch.float32).reshape(-1).repeat_interleave(d_h)
+        dec, fr, ph = t(decay), t(freq), t(phase)
+        amp = torch.ones_like(dec)
+        return cls(*(v.reshape(-1, 1).contiguous().to(device) for v in (dec, fr, amp, ph)))
+
     def _c(self) -> _Params:
         return _Params(*(_ptr(t, torch.float32, 2) for t in
                          (self.decay, self.freq, self.amp, self.phase)), self.D, self.M)

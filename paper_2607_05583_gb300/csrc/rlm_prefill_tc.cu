@@ -87,7 +87,7 @@ constexpr int kC = 64;                 // chunk length
 constexpr int kNT = 32;                // chunks per tile = MMA N
 constexpr int kTile = kC * kNT;        // 2048 tokens
 constexpr int kDG = 8;                 // channels per CTA
-constexpr int kModes = 16;             // M handled by this kernel
+constexpr int kModes = 16;             // modes per channel in the kernel's tables (M <= 16 is padded)
 constexpr int kBox = 256;              // TMA box rows
 constexpr int kBoxes = kTile / kBox;   // 8 per tile
 constexpr int kXSlots = 15;            // x ring depth (boxes)
@@ -355,6 +355,7 @@ struct TcArgs {
     __nv_bfloat16 *y;    // for the plain stores of boxes that start before t = 0
     int64_t L;
     int D;
+    int M;               // modes per channel, 1..16; modes M..15 are padding (amplitude 0, never stored)
     int ntiles;
     int64_t t0;          // first token of tile 0 (<= 0): tiles end exactly at L-1
     // Sequence segments (grid z): segment s owns tiles [s * seg_tiles, ...).
@@ -406,8 +407,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int pq = warp & 3, pe = warp < 12 ? warp >> 2 : 3;
     const int ptid = (pe * 4 + pq) * 32 + lane;
     float p_decay = 0.0f, p_freq = 0.0f, p_amp = 0.0f, p_phase = 0.0f;
-    if (builder) {
-        const int pm = (d0 + (ptid >> 6)) * kModes + ((ptid >> 2) & 15);
+    if (builder && ((ptid >> 2) & 15) < args.M) {
+        const int pm = (d0 + (ptid >> 6)) * args.M + ((ptid >> 2) & 15);
         p_decay = args.decay[pm];
         p_freq = args.freq[pm];
         p_amp = args.amp[pm];
@@ -478,11 +479,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // eight modes of its warp (a fixed shuffle tree) into Kp[half][c][n].
     if (builder) {
         const int c = ptid >> 6, m = (ptid >> 2) & 15, qn = ptid & 3;
-        const int pm = (d0 + c) * kModes + m;
+        const int pm = (d0 + c) * args.M + m;
         const float ga = p_decay, om = p_freq;
         const float2 lam = lambda_pow(ga, om, 1.0f);
         const float2 cf = mode_coef(p_amp, p_phase);
-        if (args.coef_out && b == 0 && seg == 0 && qn == 0)
+        if (args.coef_out && b == 0 && seg == 0 && qn == 0 && m < args.M)
             args.coef_out[pm] = make_float4(lam.x, lam.y, cf.x, cf.y);
         float2 pw = lambda_pow(ga, om, (float)(16 * qn));
         uint8_t *au = smem + kOffAu + au_slot(c) * kAuStride + (m / 4) * 128 + ((2 * m) % 8) * 2;
@@ -754,16 +755,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t st_lane = 32u * (uint32_t)quarter;
         const int m = lane >> 1, ri = lane & 1;
         const int ch = ri ? cB : cA;
-        const int pm = (d0 + ch) * kModes + m;
-        const float2 LC = lambda_pow(args.decay[pm], args.freq[pm], (float)kC);
+        const bool mreal = m < args.M;                       // padded modes: gamma = omega = 0, never stored
+        const int pm = (d0 + ch) * args.M + m;
+        const float m_decay = mreal ? args.decay[pm] : 0.0f, m_freq = mreal ? args.freq[pm] : 0.0f;
+        const float2 LC = lambda_pow(m_decay, m_freq, (float)kC);
         float2 S = make_float2(0.0f, 0.0f);
         float2 inj = make_float2(0.0f, 0.0f);
         int n0 = -1;
         if (kInj) {
             n0 = (int)((-args.t0) >> 6);
             const int p = (int)((-args.t0) & 63);
-            inj = cmul(lambda_pow(args.decay[pm], args.freq[pm], (float)(-p)),
-                       args.state_in[((int64_t)b * D + d0 + ch) * kModes + m]);
+            if (mreal)
+                inj = cmul(lambda_pow(m_decay, m_freq, (float)(-p)), args.state_in[((int64_t)b * D + d0 + ch) * args.M + m]);
         }
         uint8_t *bs = smem + kOffBs + ch * kBsStride + (m / 4) * kBsLbo + (m % 4) * 4;
         const int64_t seg_row = (int64_t)b * args.nseg;
@@ -790,8 +793,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     S = cfma(LC, S, Ln);
                 }
             }
-            if (v == nV - 1 && (!kSeg || seg == args.nseg - 1) && args.state_out)
-                args.state_out[((int64_t)b * D + d0 + ch) * kModes + m] = S;
+            if (v == nV - 1 && (!kSeg || seg == args.nseg - 1) && args.state_out && mreal)
+                args.state_out[((int64_t)b * D + d0 + ch) * args.M + m] = S;
             fence_async_smem();
             tc_fence_before();
             __syncwarp();
@@ -822,8 +825,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 const float2 lr = __ldcg(args.seg_state + at);
-                const float2 P = lambda_pow(args.decay[pm], args.freq[pm],
-                                            (float)((int64_t)(seg - 1 - r) * args.seg_tiles * kTile));
+                const float2 P = lambda_pow(m_decay, m_freq, (float)((int64_t)(seg - 1 - r) * args.seg_tiles * kTile));
                 S = cfma(P, lr, S);
             }
         }
@@ -1007,7 +1009,7 @@ size_t seg_state_bytes(int64_t B, int nseg, int D) {
 }  // namespace
 
 bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
-    return dt == RLM_BF16 && M == kModes && D % kDG == 0 && B >= 1 && B <= 65535 && L >= 1 &&
+    return dt == RLM_BF16 && M >= 1 && M <= kModes && D % kDG == 0 && B >= 1 && B <= 65535 && L >= 1 &&
            L <= ((int64_t)1 << 31) - kTile && D / kDG <= 65535;
 }
 
@@ -1025,7 +1027,6 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
                        const float *decay, const float *freq, const float *amp,
                        const float *phase, const float *state_in, float *state_out, float *coef_out,
                        const TcMix *mix, void *ws, cudaStream_t st) {
-    (void)M;
     CUtensorMap mx, my, mg;
     if (!make_field_map(&mx, x, B, L, D) || !make_field_map(&my, y, B, L, D))
         return cudaErrorInvalidValue;
@@ -1064,6 +1065,7 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.y = static_cast<__nv_bfloat16 *>(y);
     a.L = L;
     a.D = D;
+    a.M = M;
     a.ntiles = (int)((L + kTile - 1) / kTile);
     a.t0 = L - (int64_t)a.ntiles * kTile;
     const Segments sg = segments(B, L, D);

@@ -78,10 +78,14 @@ def test_prefill_layer6m_bf16():
     # few rows: the sequence is split into segments (one per tile; two tiles each
     # with a shorter last segment)
     (1, 2048 * 5 + 100, 8, 16, "bf16"), (1, 2048 * 24 + 5, 64, 16, "bf16"),
-    # bf16 with M != 16 (M <= 32): the time-reversed tcgen05 scan -- one token, a
-    # tail shorter than a chunk, one token past a tile, D not a multiple of 64
-    (1, 1, 8, 3, "bf16"), (2, 65, 16, 32, "bf16"), (1, 2100, 8, 31, "bf16"),
-    (2, 2048 * 2 + 7, 24, 8, "bf16"),
+    # bf16 with M < 16: the tcgen05 prefill with the modes padded to 16 (one token,
+    # D not a multiple of 64, the paper's single mode per channel, segmented and not)
+    (1, 1, 8, 3, "bf16"), (2, 2048 * 2 + 7, 24, 8, "bf16"), (1, 2048 * 3, 64, 1, "bf16"),
+    (4, 2048 + 5, 256, 1, "bf16"), (1, 3000, 8, 15, "bf16"),
+    # bf16 with 16 < M <= 32: the time-reversed tcgen05 scan -- one token, a tail
+    # shorter than a chunk, one token past a tile, D not a multiple of 64
+    (1, 1, 8, 17, "bf16"), (2, 65, 16, 32, "bf16"), (1, 2100, 8, 31, "bf16"),
+    (2, 2048 * 2 + 7, 24, 20, "bf16"),
     # bf16 with M > 32: the SIMT path
     (1, 500, 8, 40, "bf16"),
 ])
@@ -125,11 +129,11 @@ def test_prefill_training_shape_m32_sampled():
 
 
 def test_time_reversed_prefill_is_causal_bit_exact():
-    """The M != 16 bf16 prefill runs as a reverse-time scan of the reversed drive;
-    perturbing x[t >= t0] must still leave y[t < t0] bit-identical."""
-    inp = make_inputs(2, 5000, 64, 8, "bf16", seed=6)
+    """The bf16 prefill with 16 < M <= 32 runs as a reverse-time scan of the reversed
+    drive; perturbing x[t >= t0] must still leave y[t < t0] bit-identical."""
+    inp = make_inputs(2, 5000, 64, 24, "bf16", seed=6)
     y1, _ = _prefill(inp, False)
-    inp2 = make_inputs(2, 5000, 64, 8, "bf16", seed=6)
+    inp2 = make_inputs(2, 5000, 64, 24, "bf16", seed=6)
     inp2.x = inp.x.copy()
     inp2.x[:, 2999:] = -inp2.x[:, 2999:] + 1.0
     y2, _ = _prefill(inp2, False)
@@ -150,7 +154,9 @@ def _state_from(inp, s_np):
     (1, 3000, 16, 16, "bf16"),            # ... segmented sequence, ragged
     (3, 2048 + 77, 128, 16, "bf16"),      # ... segmented, several rows
     (2, 1000, 8, 32, "bf16"),             # time-reversed scan, L not a chunk multiple
-    (1, 4096, 16, 7, "bf16"),             # time-reversed scan, L a chunk multiple
+    (1, 4096, 16, 20, "bf16"),            # time-reversed scan, L a chunk multiple
+    (1, 4096, 16, 7, "bf16"),             # tcgen05 prefill, 7 modes padded to 16 (segmented)
+    (4, 3001, 256, 1, "bf16"),            # ... one mode per channel, unsegmented
     (2, 1000, 16, 7, "f32"),              # SIMT
     (1, 500, 8, 40, "bf16"),              # SIMT, bf16 with M > 32
 ])
@@ -533,3 +539,26 @@ def test_backward_gpu_finite_differences_tiny():
         fd = (loss(pp) - loss(pm)) / (2 * h)
         got = float(getattr(g, name).cpu().numpy()[idx])
         assert abs(got - fd) <= 2e-2 * max(1.0, abs(fd)), (name, got, fd)
+
+
+def test_tied_heads_match_the_paper_kernel():
+    """The paper's heads (one mode, A = 1, parameters shared by the head's channels)
+    through Params.tied_heads: y against the direct convolution with
+    k_h[t] = exp(-alpha_h t) cos(omega_h t + phi_h) (Sec. 3.1), per head."""
+    H, d_h, B, L = 8, 32, 2, 3000
+    rng = np.random.default_rng(17)
+    alpha = np.exp(rng.uniform(np.log(1e-3), np.log(0.3), H)).astype(np.float32)
+    omega = rng.uniform(0.0, np.pi, H).astype(np.float32)
+    phi = rng.uniform(-np.pi, np.pi, H).astype(np.float32)
+    inp = make_inputs(B, L, H * d_h, 1, "bf16", seed=18)
+    p = rlm.Params.tied_heads(alpha, omega, phi, d_h)
+    x = to_dev(inp.x, "bf16")
+    y = torch.empty_like(x)
+    rlm.rlm_mix_prefill(x, p, y)
+    torch.cuda.synchronize()
+    n = np.arange(L, dtype=np.float64)
+    for h in (0, 3, 7):
+        k = np.exp(-np.float64(alpha[h]) * n) * np.cos(np.float64(omega[h]) * n + np.float64(phi[h]))
+        for c in (h * d_h, h * d_h + d_h - 1):
+            ref = np.stack([np.convolve(inp.x[b, :, c].astype(np.float64), k)[:L] for b in range(B)])
+            assert_close(to_np(y)[:, :, c], ref, TOL["bf16"], f"head {h} channel {c}")
