@@ -753,10 +753,57 @@ def cpu_baseline(seconds=10.0):
         if time.perf_counter() - t0 >= seconds:
             break
     dt = time.perf_counter() - t0
-    return {"value": round(n * P["L"] / dt / 1e6, 4), "unit": "Mtok/s", "cores": oracle.num_threads(),
-            "kind": "oracle",
-            "sample": f"{n} x one sequence (B=1, L={P['L']}, D={P['D']}, M={P['M']}) of the "
-                      f"prefill workload through the fp64 sequential recurrence, {dt:.1f} s"}
+    out = {"value": round(n * P["L"] / dt / 1e6, 4), "unit": "Mtok/s", "cores": oracle.num_threads(),
+           "kind": "oracle",
+           "sample": f"{n} x one sequence (B=1, L={P['L']}, D={P['D']}, M={P['M']}) of the "
+                     f"prefill workload through the fp64 sequential recurrence, {dt:.1f} s"}
+    out["other_workloads"] = _cpu_other_workloads(seconds=max(1.0, seconds / 4))
+    return out
+
+
+def _cpu_other_workloads(seconds):
+    """The oracle on the other workloads, each for about ``seconds``: the 6M layer's
+    prefill (O2), decode steps at B = 64 (O2's step), and the O(L^2) direct
+    convolution (O1) at L = 8192 on a sample of channels (the analogue of the
+    paper's quadratic causal reference)."""
+    import oracle
+    from synth import make_inputs
+
+    def loop(fn):
+        t0 = time.perf_counter()
+        n = 0
+        while True:
+            fn()
+            n += 1
+            if time.perf_counter() - t0 >= seconds:
+                return n, time.perf_counter() - t0
+
+    res = {}
+    inp = make_inputs(8, 2048, 256, 16, "bf16", seed=0)
+    x64, prm = inp.x.astype(np.float64), [q.astype(np.float64) for q in inp.params()]
+    n, dt = loop(lambda: oracle.rec_prefill(x64, *prm))
+    res["layer6m_prefill_B8_L2048"] = {"Mtok_s": round(n * 8 * 2048 / dt / 1e6, 4),
+                                       "sample": f"{n} calls of the whole problem, {dt:.1f} s"}
+    dec = make_inputs(64, 1, 256, 16, "bf16", seed=0)
+    _, st = oracle.rec_prefill(dec.x.astype(np.float64), *[q.astype(np.float64) for q in dec.params()])
+    xt = dec.x[:, 0].astype(np.float64)
+    dprm = [q.astype(np.float64) for q in dec.params()]
+    box = {"s": st}
+
+    def step():
+        _, box["s"] = oracle.rec_decode(box["s"], xt, *dprm)
+
+    n, dt = loop(step)
+    res["decode_B64"] = {"tok_s": round(n * 64 / dt, 1), "us_per_step": round(dt / n * 1e6, 1),
+                         "sample": f"{n} steps, {dt:.1f} s"}
+    ch = 16
+    conv = make_inputs(1, 8192, ch, 16, "bf16", seed=0)
+    cx, cprm = conv.x.astype(np.float64), [q.astype(np.float64) for q in conv.params()]
+    n, dt = loop(lambda: oracle.conv_prefill(cx, *cprm))
+    # scale to the full 256 channels: channels are independent work
+    res["direct_convolution_L8192"] = {"Mtok_s_at_D256": round(n * 8192 * ch / 256 / dt / 1e6, 6),
+                                       "sample": f"{n} calls on {ch} of 256 channels, {dt:.1f} s"}
+    return res
 
 
 def run_reference(args):
