@@ -309,12 +309,19 @@ def run_ours(args):
         for (B, L) in ((1, 8192), (1, 16384), (1, 32768), (4, 8192), (4, 16384)):
             sweep[f"B{B}_L{L}"] = _time_prefill(rlm, torch, dev, B, L, P["D"], P["M"], flush,
                                                 hbm_peak, reps=max(5, args.steps // 2))
+        # the 6M layer's prefill (B = 8, L = 2048)
+        sweep["layer6m_B8_L2048"] = _time_prefill(rlm, torch, dev, 8, 2048, P["D"], P["M"], flush,
+                                                  hbm_peak, reps=max(5, args.steps // 2))
     sweep[f"B{P['B']}_L{P['L']}"] = {"Mtok_s": round(tokens / (ms * 1e-3) / 1e6, 1),
                                      "frac": roofline["frac"]}
     del x, y, work
 
     # ---------------- decode
     decode = None if args.quick else _bench_decode(rlm, torch, dev, hbm_peak)
+    if decode is not None:
+        decode["other_batch_sizes"] = {f"B{b}": {k: v for k, v in _bench_decode(rlm, torch, dev, hbm_peak, B=b).items()
+                                                 if k in ("tok_s", "us_per_step", "frac_hbm")}
+                                       for b in (1, 8)}
     # ---------------- backward
     backward = None if args.quick else _bench_backward(rlm, torch, dev, hbm_peak, args)
     # ---------------- mixer wrapper (gate + local path, fused)
@@ -399,10 +406,11 @@ def _time_prefill(rlm, torch, dev, B, L, D, M, flush, hbm_peak, reps=5):
             "frac": round(gbs / hbm_peak, 4)}
 
 
-def _bench_decode(rlm, torch, dev, hbm_peak):
+def _bench_decode(rlm, torch, dev, hbm_peak, B=None):
     from synth import make_inputs
     P = DECODE
-    B, L, D, M, T = P["B"], P["L"], P["D"], P["M"], P["T"]
+    B = P["B"] if B is None else B
+    L, D, M, T = P["L"], P["D"], P["M"], P["T"]
     inp = make_inputs(B, L, D, M, "bf16", seed=0, decode_steps=T)
     x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
     p = rlm.Params.from_arrays(*inp.params(), device=dev)
@@ -440,7 +448,7 @@ def _bench_decode(rlm, torch, dev, hbm_peak):
     us_step = ms * 1e3 / T
     per_step = decode_bytes(B, D, M)
     gbs = per_step / (us_step * 1e-6) / 1e9
-    return {"workload": "decode B=64 D=256 M=16, 4096 steps after a 32768-token prefill, CUDA graph",
+    return {"workload": f"decode B={B} D={D} M={M}, {T} steps after a {L}-token prefill, CUDA graph",
             "tok_s": round(B * T / (ms * 1e-3), 1), "us_per_step": round(us_step, 4),
             "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
             "bytes_per_step": per_step, "launches": T}
