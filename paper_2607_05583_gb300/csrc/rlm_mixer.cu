@@ -181,10 +181,13 @@ template <> struct VecIO<float, 4> {
     }
 };
 
-template <typename T, int kV>
-__global__ void __launch_bounds__(kBlock) k_couple_small(T *z, const float *__restrict__ c_raw, float lam, int H,
+// kHc = H when it is a compile-time 2, 4, 8 or 16 (loops unrolled, C rows read as
+// 16-byte vectors); 0 for any other H <= 16.
+template <typename T, int kV, int kHc>
+__global__ void __launch_bounds__(kBlock) k_couple_small(T *z, const float *__restrict__ c_raw, float lam, int H_rt,
                                                          int64_t rows, int D) {
-    __shared__ float C[kSmallH * kSmallH];
+    __shared__ __align__(16) float C[kSmallH * kSmallH];
+    const int H = kHc ? kHc : H_rt;
     build_coupling(C, c_raw, lam, H);
     __syncthreads();
     const int dh = D / H, nj = dh / kV;
@@ -193,10 +196,11 @@ __global__ void __launch_bounds__(kBlock) k_couple_small(T *z, const float *__re
     const int64_t r = i / nj;
     const int j = (int)(i % nj) * kV;
     T *row = z + r * D + j;
-    float y[kSmallH][kV];
+    constexpr int kHm = kHc ? kHc : kSmallH;
+    float y[kHm][kV];
 #pragma unroll
-    for (int h = 0; h < kSmallH; ++h) {
-        if (h < H) {
+    for (int h = 0; h < kHm; ++h) {
+        if (kHc || h < H) {
             VecIO<T, kV>::load(row + h * dh, y[h]);
         } else {
 #pragma unroll
@@ -204,16 +208,28 @@ __global__ void __launch_bounds__(kBlock) k_couple_small(T *z, const float *__re
         }
     }
 #pragma unroll
-    for (int gh = 0; gh < kSmallH; ++gh) {
-        if (gh >= H) break;
+    for (int gh = 0; gh < kHm; ++gh) {
+        if (!kHc && gh >= H) break;
         float acc[kV];
 #pragma unroll
         for (int e = 0; e < kV; ++e) acc[e] = 0.0f;
+        if constexpr (kHc >= 4) {
 #pragma unroll
-        for (int h = 0; h < kSmallH; ++h) {
-            const float c = C[gh * H + (h < H ? h : 0)];
+            for (int h4 = 0; h4 < kHc; h4 += 4) {
+                const float4 c4 = *reinterpret_cast<const float4 *>(C + gh * kHc + h4);
+                const float cs[4] = {c4.x, c4.y, c4.z, c4.w};
 #pragma unroll
-            for (int e = 0; e < kV; ++e) acc[e] = fmaf(c, y[h][e], acc[e]);
+                for (int q = 0; q < 4; ++q)
+#pragma unroll
+                    for (int e = 0; e < kV; ++e) acc[e] = fmaf(cs[q], y[h4 + q][e], acc[e]);
+            }
+        } else {
+#pragma unroll
+            for (int h = 0; h < kHm; ++h) {
+                const float c = C[gh * H + (kHc || h < H ? h : 0)];
+#pragma unroll
+                for (int e = 0; e < kV; ++e) acc[e] = fmaf(c, y[h][e], acc[e]);
+            }
         }
         VecIO<T, kV>::store(row + gh * dh, acc);
     }
@@ -339,10 +355,18 @@ cudaError_t couple_t(void *z, const float *c_raw, float lam, int H, int64_t B, i
         const int dh = D / H;
         const int64_t n = B * L * (dh % 4 == 0 ? dh / 4 : dh);
         const unsigned grid = (unsigned)((n + kBlock - 1) / kBlock);
-        if (dh % 4 == 0)
-            k_couple_small<T, 4><<<grid, kBlock, 0, st>>>(static_cast<T *>(z), c_raw, lam, H, B * L, D);
-        else
-            k_couple_small<T, 1><<<grid, kBlock, 0, st>>>(static_cast<T *>(z), c_raw, lam, H, B * L, D);
+        T *zt = static_cast<T *>(z);
+        if (dh % 4 == 0) {
+            switch (H) {
+                case 2: k_couple_small<T, 4, 2><<<grid, kBlock, 0, st>>>(zt, c_raw, lam, H, B * L, D); break;
+                case 4: k_couple_small<T, 4, 4><<<grid, kBlock, 0, st>>>(zt, c_raw, lam, H, B * L, D); break;
+                case 8: k_couple_small<T, 4, 8><<<grid, kBlock, 0, st>>>(zt, c_raw, lam, H, B * L, D); break;
+                case 16: k_couple_small<T, 4, 16><<<grid, kBlock, 0, st>>>(zt, c_raw, lam, H, B * L, D); break;
+                default: k_couple_small<T, 4, 0><<<grid, kBlock, 0, st>>>(zt, c_raw, lam, H, B * L, D); break;
+            }
+        } else {
+            k_couple_small<T, 1, 0><<<grid, kBlock, 0, st>>>(zt, c_raw, lam, H, B * L, D);
+        }
         count_launches(1);
         return cudaGetLastError();
     }

@@ -310,6 +310,8 @@ def _coupling(H, seed, lam=0.7):
     (2, 1000, 32, 32, 0, 1, "bf16", True),           # time-reversed prefill, H = 1 (a scalar gain)
     (2, 1000, 24, 16, 4, 8, "bf16", True),           # head width 3: one position per thread
     (2, 1000, 64, 16, 2, 32, "f32", True),           # 32 heads: whole rows staged in shared memory
+    (2, 3001, 64, 16, 4, 16, "bf16", True),          # 16 heads (the largest unrolled case)
+    (1, 700, 48, 16, 3, 12, "bf16", True),           # 12 heads: H not unrolled, head width 4
 ])
 def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
     inp = make_inputs(B, L, D, M, dtype, seed=L + H)
