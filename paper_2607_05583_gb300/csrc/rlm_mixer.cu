@@ -40,6 +40,17 @@ __device__ __forceinline__ void st2(__nv_bfloat16 *p, float2 v) {
     *reinterpret_cast<uint32_t *>(p) = a;
 }
 
+// Two consecutive channels as loaded (4 bytes of bf16 or 8 bytes of fp32).
+template <typename T> struct Raw2;
+template <> struct Raw2<float> { using type = float2; };
+template <> struct Raw2<__nv_bfloat16> { using type = uint32_t; };
+__device__ __forceinline__ float2 ld_raw2(const float *p) { return *reinterpret_cast<const float2 *>(p); }
+__device__ __forceinline__ uint32_t ld_raw2(const __nv_bfloat16 *p) { return *reinterpret_cast<const uint32_t *>(p); }
+__device__ __forceinline__ float2 raw_f2(float2 v) { return v; }
+__device__ __forceinline__ float2 raw_f2(uint32_t v) {
+    return make_float2(__uint_as_float(v << 16), __uint_as_float(v & 0xFFFF0000u));
+}
+
 template <typename T, int K>
 __global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__ x, const T *__restrict__ g,
                                                            T *__restrict__ z, const T *__restrict__ hist,
@@ -47,12 +58,28 @@ __global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__
                                                            const float *__restrict__ scale, int64_t L, int D) {
     constexpr int kRows = kTT + (K > 1 ? K - 1 : 0);
     constexpr int kVE = 16 / sizeof(T);                // elements per 16-byte vector
+    constexpr int kPer = kTT / (kBlock / (kTC / 2));   // tokens per thread
     __shared__ __align__(16) T xs[K > 0 ? kRows * kTC : 1];
     const int c0 = blockIdx.x * kTC;
     const int64_t t0 = (int64_t)blockIdx.y * kTT;
     const int64_t b = blockIdx.z;
     const int nc = min(kTC, D - c0);                   // a multiple of 8
     const int tid = threadIdx.x;
+    const int cp = tid % (kTC / 2), tg = tid / (kTC / 2);
+    const int c = 2 * cp;
+    const bool active = c < nc;
+    // This thread's y and gate for all its tokens, requested before the drive
+    // tile is staged, so the block waits on memory once.
+    typename Raw2<T>::type zr[kPer], gr[kPer];
+#pragma unroll
+    for (int tt = 0; tt < kPer; ++tt) {
+        const int64_t t = t0 + tg * kPer + tt;
+        if (active && t < L) {
+            const int64_t i = (b * L + t) * D + c0 + c;
+            zr[tt] = ld_raw2(z + i);
+            if (g) gr[tt] = ld_raw2(g + i);
+        }
+    }
     if (K > 0) {
         const int vpr = nc / kVE;
         for (int i = tid; i < kRows * vpr; i += kBlock) {
@@ -67,9 +94,7 @@ __global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__
         }
         __syncthreads();
     }
-    const int cp = tid % (kTC / 2), tg = tid / (kTC / 2);
-    const int c = 2 * cp;
-    if (c >= nc) return;
+    if (!active) return;
     float w0[K > 0 ? K : 1], w1[K > 0 ? K : 1];
     float s0 = 0.0f, s1 = 0.0f;
 #pragma unroll
@@ -81,17 +106,15 @@ __global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__
         s0 = __ldg(scale + c0 + c);
         s1 = __ldg(scale + c0 + c + 1);
     }
-    constexpr int kPer = kTT / (kBlock / (kTC / 2));   // tokens per thread
-#pragma unroll 4
+#pragma unroll
     for (int tt = 0; tt < kPer; ++tt) {
         const int r = tg * kPer + tt;                   // token t0 + r
         const int64_t t = t0 + r;
         if (t >= L) break;
-        const int64_t i = (b * L + t) * D + c0 + c;
-        float2 zv = ld2(z + i);
+        float2 o = raw_f2(zr[tt]);
         if (g) {
-            const float2 gv = ld2(g + i);
-            zv = make_float2(zv.x * gatef(gv.x), zv.y * gatef(gv.y));
+            const float2 gv = raw_f2(gr[tt]);
+            o = make_float2(o.x * gatef(gv.x), o.y * gatef(gv.y));
         }
         if (K > 0) {
             float l0 = 0.0f, l1 = 0.0f;
@@ -101,9 +124,9 @@ __global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__
                 l0 = fmaf(w0[k], v.x, l0);
                 l1 = fmaf(w1[k], v.y, l1);
             }
-            zv = make_float2(fmaf(s0, l0, zv.x), fmaf(s1, l1, zv.y));
+            o = make_float2(fmaf(s0, l0, o.x), fmaf(s1, l1, o.y));
         }
-        st2(z + i, zv);
+        st2(z + (b * L + t) * D + c0 + c, o);
     }
 }
 
