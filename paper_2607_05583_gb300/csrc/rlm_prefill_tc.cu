@@ -355,7 +355,10 @@ struct TcArgs {
     __nv_bfloat16 *y;    // for the plain stores of boxes that start before t = 0
     int64_t L;
     int D;
-    int M;               // modes per channel, 1..16; modes M..15 are padding (amplitude 0, never stored)
+    int M;               // modes of this pass, 1..16; modes M..15 are padding (amplitude 0, never stored)
+    int m0, Mt;          // first mode of this pass; modes per channel in the parameter/state layouts
+    int add;             // kMix: the slot holds y so far (earlier passes); z = that + this pass's y
+                         // (otherwise the slot holds the gate: z = sigma(g) y)
     int ntiles;
     int64_t t0;          // first token of tile 0 (<= 0): tiles end exactly at L-1
     // Sequence segments (grid z): segment s owns tiles [s * seg_tiles, ...).
@@ -373,10 +376,13 @@ struct TcArgs {
 // to the state entering chunk n0, which gives lambda^(i+1-p) s_in at its positions
 // i >= p (those before p are negative times, never stored) and lambda^(64-p) s_in
 // carried on.  |lambda^-p| <= exp(63 gamma) stays bounded.
-// kMix: the gate of the mixer wrapper (Sec. 3.4), z = sigma(g) y, in the epilogue
-// (unsegmented launches only).  The store issuer loads the gate rows of each z ring
-// slot into the slot itself once the slot's previous store has been read out;
-// every epilogue thread reads its 8 bytes of g there and overwrites them with z.
+// kMix: a second field is loaded into the z ring and combined in the epilogue
+// (unsegmented launches only): the gate of the mixer wrapper (Sec. 3.4),
+// z = sigma(g) y, or (args.add, for M > 16 in passes of 16 modes) the output of
+// the earlier passes, z = y_before + y.  The store issuer loads the field's rows
+// of each z ring slot into the slot itself once the slot's previous store has
+// been read out; every epilogue thread reads its 8 bytes there and overwrites them
+// with z.
 template <bool kSeg, bool kInj, bool kMix>
 __global__ void __launch_bounds__(kThreads, 1)
     k_prefill_tc(const __grid_constant__ CUtensorMap tmap_x,
@@ -408,7 +414,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int ptid = (pe * 4 + pq) * 32 + lane;
     float p_decay = 0.0f, p_freq = 0.0f, p_amp = 0.0f, p_phase = 0.0f;
     if (builder && ((ptid >> 2) & 15) < args.M) {
-        const int pm = (d0 + (ptid >> 6)) * args.M + ((ptid >> 2) & 15);
+        const int pm = (d0 + (ptid >> 6)) * args.Mt + args.m0 + ((ptid >> 2) & 15);
         p_decay = args.decay[pm];
         p_freq = args.freq[pm];
         p_amp = args.amp[pm];
@@ -479,7 +485,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // eight modes of its warp (a fixed shuffle tree) into Kp[half][c][n].
     if (builder) {
         const int c = ptid >> 6, m = (ptid >> 2) & 15, qn = ptid & 3;
-        const int pm = (d0 + c) * args.M + m;
+        const int pm = (d0 + c) * args.Mt + args.m0 + m;
         const float ga = p_decay, om = p_freq;
         const float2 lam = lambda_pow(ga, om, 1.0f);
         const float2 cf = mode_coef(p_amp, p_phase);
@@ -756,7 +762,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int m = lane >> 1, ri = lane & 1;
         const int ch = ri ? cB : cA;
         const bool mreal = m < args.M;                       // padded modes: gamma = omega = 0, never stored
-        const int pm = (d0 + ch) * args.M + m;
+        const int pm = (d0 + ch) * args.Mt + args.m0 + m;
         const float m_decay = mreal ? args.decay[pm] : 0.0f, m_freq = mreal ? args.freq[pm] : 0.0f;
         const float2 LC = lambda_pow(m_decay, m_freq, (float)kC);
         float2 S = make_float2(0.0f, 0.0f);
@@ -766,7 +772,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             n0 = (int)((-args.t0) >> 6);
             const int p = (int)((-args.t0) & 63);
             if (mreal)
-                inj = cmul(lambda_pow(m_decay, m_freq, (float)(-p)), args.state_in[((int64_t)b * D + d0 + ch) * args.M + m]);
+                inj = cmul(lambda_pow(m_decay, m_freq, (float)(-p)), args.state_in[((int64_t)b * D + d0 + ch) * args.Mt + args.m0 + m]);
         }
         uint8_t *bs = smem + kOffBs + ch * kBsStride + (m / 4) * kBsLbo + (m % 4) * 4;
         const int64_t seg_row = (int64_t)b * args.nseg;
@@ -794,7 +800,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
             if (v == nV - 1 && (!kSeg || seg == args.nseg - 1) && args.state_out && mreal)
-                args.state_out[((int64_t)b * D + d0 + ch) * args.M + m] = S;
+                args.state_out[((int64_t)b * D + d0 + ch) * args.Mt + args.m0 + m] = S;
             fence_async_smem();
             tc_fence_before();
             __syncwarp();
@@ -871,8 +877,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int n8 = 0; n8 < 8; ++n8) {
                             uint32_t *gz = reinterpret_cast<uint32_t *>(gs + (n8 * kC + pos) * 16);
                             const __nv_bfloat162 g2 = *reinterpret_cast<const __nv_bfloat162 *>(gz);
-                            const float za = __uint_as_float(va[n8]) * __fdividef(1.0f, 1.0f + __expf(-__low2float(g2)));
-                            const float zb = __uint_as_float(vb[n8]) * __fdividef(1.0f, 1.0f + __expf(-__high2float(g2)));
+                            float za = __uint_as_float(va[n8]), zb = __uint_as_float(vb[n8]);
+                            if (args.add) {
+                                za += __low2float(g2);
+                                zb += __high2float(g2);
+                            } else {
+                                za *= __fdividef(1.0f, 1.0f + __expf(-__low2float(g2)));
+                                zb *= __fdividef(1.0f, 1.0f + __expf(-__high2float(g2)));
+                            }
                             *gz = pack_bf16x2(za, zb);
                         }
                     }
@@ -1009,12 +1021,17 @@ size_t seg_state_bytes(int64_t B, int nseg, int D) {
 }  // namespace
 
 bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
-    return dt == RLM_BF16 && M >= 1 && M <= kModes && D % kDG == 0 && B >= 1 && B <= 65535 && L >= 1 &&
-           L <= ((int64_t)1 << 31) - kTile && D / kDG <= 65535;
+    const bool shape = dt == RLM_BF16 && M >= 1 && D % kDG == 0 && B >= 1 && B <= 65535 && L >= 1 &&
+                       L <= ((int64_t)1 << 31) - kTile && D / kDG <= 65535;
+    if (!shape) return false;
+    if (M <= kModes) return true;
+    // More modes: passes of 16 modes, each later one adding to the output of the
+    // earlier ones through the z ring (unsegmented launches only).
+    return M <= 4 * kModes && segments(B, L, D).nseg < 2;
 }
 
 bool tc_mixer_fused(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
-    return tc_prefill_supported(B, L, D, M, dt) && segments(B, L, D).nseg < 2;
+    return M <= kModes && tc_prefill_supported(B, L, D, M, dt) && segments(B, L, D).nseg < 2;
 }
 
 size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int) {
@@ -1065,7 +1082,10 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.y = static_cast<__nv_bfloat16 *>(y);
     a.L = L;
     a.D = D;
-    a.M = M;
+    a.M = std::min(M, kModes);
+    a.m0 = 0;
+    a.Mt = M;
+    a.add = 0;
     a.ntiles = (int)((L + kTile - 1) / kTile);
     a.t0 = L - (int64_t)a.ntiles * kTile;
     const Segments sg = segments(B, L, D);
@@ -1075,20 +1095,31 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.seg_flag = nullptr;
     a.epoch = 0;
     dim3 grid((unsigned)(D / kDG), (unsigned)B, (unsigned)sg.nseg);
-    if (mix && sg.nseg >= 2) return cudaErrorInvalidValue;  // callers check tc_mixer_fused
+    const int npass = (M + kModes - 1) / kModes;
+    if ((mix || npass > 1) && sg.nseg >= 2) return cudaErrorInvalidValue;  // callers check support
+    if (mix && npass > 1) return cudaErrorInvalidValue;
     if (sg.nseg < 2) {
-        if (mix) {
-            if (state_in)
-                k_prefill_tc<false, true, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, mg, a);
-            else
-                k_prefill_tc<false, false, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, mg, a);
-        } else if (state_in) {
-            k_prefill_tc<false, true, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, mg, a);
-        } else {
-            k_prefill_tc<false, false, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, mg, a);
+        for (int p = 0; p < npass; ++p) {
+            a.m0 = p * kModes;
+            a.M = std::min(kModes, M - a.m0);
+            a.add = p > 0;
+            // Later passes load the output so far into the z ring and add to it.
+            const CUtensorMap &m2 = p > 0 ? my : mg;
+            if (mix || p > 0) {
+                if (state_in)
+                    k_prefill_tc<false, true, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+                else
+                    k_prefill_tc<false, false, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+            } else if (state_in) {
+                k_prefill_tc<false, true, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+            } else {
+                k_prefill_tc<false, false, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+            }
+            count_launches(1);
+            const cudaError_t e = cudaGetLastError();
+            if (e != cudaSuccess) return e;
         }
-        count_launches(1);
-        return cudaGetLastError();
+        return cudaSuccess;
     }
     // Segments wait on the end states of earlier segments of the same rows: a
     // cooperative launch guarantees all CTAs are resident together.

@@ -562,3 +562,39 @@ def test_tied_heads_match_the_paper_kernel():
         for c in (h * d_h, h * d_h + d_h - 1):
             ref = np.stack([np.convolve(inp.x[b, :, c].astype(np.float64), k)[:L] for b in range(B)])
             assert_close(to_np(y)[:, :, c], ref, TOL["bf16"], f"head {h} channel {c}")
+
+
+@pytest.mark.parametrize("B,L,D,M,with_state_in", [
+    (2, 3000, 512, 32, False),        # two passes of 16 modes (128 CTAs: unsegmented)
+    (1, 2048 + 5, 1024, 40, True),    # three passes, the last with 8 modes; from an initial state
+    (2, 4100, 512, 64, True),         # four passes
+    (4, 2048 * 2, 512, 17, False),    # a second pass with one mode
+])
+def test_multi_pass_prefill_matches_oracle(B, L, D, M, with_state_in):
+    """bf16 with M > 16 on unsegmented shapes: passes of 16 modes, each later pass
+    adding to the output of the earlier ones; y, the terminal state and the mode
+    coefficients of every mode on sampled channels against the oracle."""
+    inp = make_inputs(B, L, D, M, "bf16", seed=M + L)
+    s_in = None
+    if with_state_in:
+        pre = make_inputs(B, 200, D, M, "bf16", seed=M)
+        s_in = oracle.rec_prefill(pre.x, *inp.params())[1]
+    x = to_dev(inp.x, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    y = torch.empty_like(x)
+    so = rlm.State.empty(B, D, M)
+    n0 = rlm.rlm_kernels_launched()
+    rlm.rlm_mix_prefill_from(x, p, _state_from(inp, s_in) if with_state_in else None, y, so)
+    torch.cuda.synchronize()
+    assert rlm.rlm_kernels_launched() - n0 == (M + 15) // 16
+    ch = np.array([0, 9, D // 2 + 3, D - 1])
+    ref, st_ref = oracle.rec_prefill(inp.x[:, :, ch], inp.decay[ch], inp.freq[ch], inp.amp[ch], inp.phase[ch],
+                                     state_in=s_in[:, ch] if with_state_in else None)
+    assert_close(to_np(y)[:, :, ch], ref, TOL["bf16"], "y")
+    s = so.complex().cpu().numpy()[:, ch]
+    assert_close(s.real, st_ref.real, TOL["bf16"], "state re")
+    assert_close(s.imag, st_ref.imag, TOL["bf16"], "state im")
+    coef = so.coef.cpu().numpy()[ch]
+    lam = np.exp(-inp.decay[ch].astype(np.float64) + 1j * inp.freq[ch].astype(np.float64))
+    np.testing.assert_allclose(coef[..., 0], lam.real, rtol=0, atol=1e-6)
+    np.testing.assert_allclose(coef[..., 1], lam.imag, rtol=0, atol=1e-6)
