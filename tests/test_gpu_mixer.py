@@ -229,6 +229,23 @@ def test_tcgen05_shape_mixer_prefill_matches_oracle(B, L, D, K, with_g, with_his
     _check_prefill(inp, mx, z, so, cout, with_g, with_hist)
 
 
+@pytest.mark.parametrize("M,K", [(32, 4), (24, 0)])
+def test_multi_pass_mixer_prefill_matches_oracle(M, K):
+    """M > 16 on an unsegmented shape: the prefill in passes of 16 modes, then the
+    mixer pass (the gate is not fused with several passes)."""
+    inp = make_inputs(2, 3000, 512, M, "bf16", seed=M + K)
+    mx = make_mixer_inputs(inp, K, seed=M)
+    out = {}
+
+    def run():
+        out["r"] = _run_prefill(inp, mx, True, K > 0)
+
+    n = _launches(run)
+    assert n == 2 + 1 + (1 if K >= 2 else 0), n
+    z, so, cout = out["r"]
+    _check_prefill(inp, mx, z, so, cout, True, K > 0)
+
+
 @pytest.mark.parametrize("K", [0, 4])
 def test_tcgen05_shape_mixer_prefill_from_state_and_split_in_place(K):
     B, L, D, cut = 2, 6000, 512, 2345
