@@ -24,6 +24,7 @@ constexpr int kBlock = 256;
 constexpr int kMaxK = RLM_MAX_LOCAL_K;
 constexpr int kTT = 64;    // tokens per tile
 constexpr int kTC = 128;   // channels per tile (a multiple of 8 channels is staged)
+constexpr int kEB = 256;   // threads per block of the mixer pass
 
 __device__ __forceinline__ float gatef(float v) { return __fdividef(1.0f, 1.0f + __expf(-v)); }
 
@@ -52,13 +53,13 @@ __device__ __forceinline__ float2 raw_f2(uint32_t v) {
 }
 
 template <typename T, int K>
-__global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__ x, const T *__restrict__ g,
+__global__ void __launch_bounds__(kEB) k_mixer_epilogue(const T *__restrict__ x, const T *__restrict__ g,
                                                            T *__restrict__ z, const T *__restrict__ hist,
                                                            const float *__restrict__ conv_w,
                                                            const float *__restrict__ scale, int64_t L, int D) {
     constexpr int kRows = kTT + (K > 1 ? K - 1 : 0);
     constexpr int kVE = 16 / sizeof(T);                // elements per 16-byte vector
-    constexpr int kPer = kTT / (kBlock / (kTC / 2));   // tokens per thread
+    constexpr int kPer = kTT / (kEB / (kTC / 2));      // tokens per thread
     __shared__ __align__(16) T xs[K > 0 ? kRows * kTC : 1];
     const int c0 = blockIdx.x * kTC;
     const int64_t t0 = (int64_t)blockIdx.y * kTT;
@@ -82,7 +83,7 @@ __global__ void __launch_bounds__(kBlock) k_mixer_epilogue(const T *__restrict__
     }
     if (K > 0) {
         const int vpr = nc / kVE;
-        for (int i = tid; i < kRows * vpr; i += kBlock) {
+        for (int i = tid; i < kRows * vpr; i += kEB) {
             const int r = i / vpr, v = i % vpr;
             const int64_t t = t0 - (K > 1 ? K - 1 : 0) + r;
             uint4 val = make_uint4(0u, 0u, 0u, 0u);
@@ -329,7 +330,7 @@ template <typename T, int K>
 cudaError_t epilogue_k(const void *x, const void *g, void *z, const void *hist, const float *conv_w,
                        const float *scale, int64_t B, int64_t L, int D, cudaStream_t st) {
     const dim3 grid((unsigned)((D + kTC - 1) / kTC), (unsigned)((L + kTT - 1) / kTT), (unsigned)B);
-    k_mixer_epilogue<T, K><<<grid, kBlock, 0, st>>>(static_cast<const T *>(x), static_cast<const T *>(g),
+    k_mixer_epilogue<T, K><<<grid, kEB, 0, st>>>(static_cast<const T *>(x), static_cast<const T *>(g),
                                                     static_cast<T *>(z), static_cast<const T *>(hist), conv_w,
                                                     scale, L, D);
     count_launches(1);
