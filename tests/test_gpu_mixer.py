@@ -329,6 +329,7 @@ def _coupling(H, seed, lam=0.7):
     (2, 1000, 64, 16, 2, 32, "f32", True),           # 32 heads: whole rows staged in shared memory
     (2, 3001, 64, 16, 4, 16, "bf16", True),          # 16 heads (the largest unrolled case)
     (1, 700, 48, 16, 3, 12, "bf16", True),           # 12 heads: H not unrolled, head width 4
+    (1, 50, 8, 4, 2, 8, "f32", True),                # one channel per head
 ])
 def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
     inp = make_inputs(B, L, D, M, dtype, seed=L + H)
@@ -351,9 +352,10 @@ def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
     assert_close(s.real, sr.real, TOL[dtype], "state re")
 
 
-@pytest.mark.parametrize("dtype,M,K,H", [("bf16", 16, 4, 8), ("f32", 7, 3, 4), ("bf16", 16, 0, 2), ("bf16", 2, 8, 16)])
-def test_coupled_mixer_decode_continues_the_prefill(dtype, M, K, H):
-    B, D, L0, T = 3, 64, 300, 30
+@pytest.mark.parametrize("dtype,M,K,H,B", [("bf16", 16, 4, 8, 3), ("f32", 7, 3, 4, 3), ("bf16", 16, 0, 2, 3),
+                                       ("bf16", 2, 8, 16, 3), ("bf16", 16, 4, 8, 1)])
+def test_coupled_mixer_decode_continues_the_prefill(dtype, M, K, H, B):
+    D, L0, T = 64, 300, 30
     inp = make_inputs(B, L0 + T, D, M, dtype, seed=M + K + H)
     mx = make_mixer_inputs(inp, K, seed=M + K + H)
     c_raw, lam = _coupling(H, 3 * H)

@@ -598,3 +598,17 @@ def test_multi_pass_prefill_matches_oracle(B, L, D, M, with_state_in):
     lam = np.exp(-inp.decay[ch].astype(np.float64) + 1j * inp.freq[ch].astype(np.float64))
     np.testing.assert_allclose(coef[..., 0], lam.real, rtol=0, atol=1e-6)
     np.testing.assert_allclose(coef[..., 1], lam.imag, rtol=0, atol=1e-6)
+
+
+def test_prefill_million_token_sequence():
+    """One sequence of 2^20 + 3 tokens (B = 1, D = 8, M = 16, bf16): the segmented
+    tcgen05 prefill with its longest segment offsets, y on sampled stretches and
+    the terminal state against the oracle's recurrence over the whole sequence."""
+    L = (1 << 20) + 3
+    inp = make_inputs(1, L, 8, 16, "bf16", seed=20)
+    y, st = _prefill(inp)
+    ref, st_ref = oracle.rec_prefill(inp.x, *inp.params())
+    yn = to_np(y)
+    for a in (0, 2048 * 100 + 7, L - 5000):
+        assert_close(yn[:, a:a + 5000], ref[:, a:a + 5000], TOL["bf16"], f"y at {a}")
+    _state_err(st, st_ref, TOL["bf16"])
