@@ -24,7 +24,6 @@ namespace rlm {
 namespace {
 
 constexpr int kDecodeBlock = 256;
-constexpr int kMaxK = RLM_MAX_LOCAL_K;
 
 // The mixer's per-step inputs (null g: no gate; K = 0: no local path).
 template <typename T>
@@ -95,6 +94,20 @@ __device__ __forceinline__ void mix_shift(const MixStep<T> &m, const MixPart<T> 
 }
 
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Moves the line holding p into L2 without reading it into the thread: safe before
+// the dependency wait even if the previous grid writes the line (L2 is where the
+// writes land), and it overlaps the token's DRAM latency with the wait.
+__device__ __forceinline__ void prefetch_l2(const void *p) {
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+// The step's fresh inputs (token and gate rows: one line per 64 (b, d) pairs).
+template <typename T>
+__device__ __forceinline__ void prefetch_step(const T *x_t, const MixStep<T> &mix, bool is_mix, int64_t bd,
+                                              int64_t BD, int g) {
+    if (g != 0 || bd >= BD || (bd & 63) != 0) return;
+    prefetch_l2(x_t + bd);
+    if (is_mix && mix.g) prefetch_l2(mix.g + bd);
+}
 __device__ __forceinline__ void pdl_launch_dependents() {
     asm volatile("griddepcontrol.launch_dependents;" :::);
 }
@@ -104,11 +117,12 @@ template <typename T, bool kMix>
 __global__ void __launch_bounds__(kDecodeBlock) k_decode_vec2(
     const T *__restrict__ x_t, T *__restrict__ y_t, int64_t BD, int D, int M, int log2_tpg,
     float4 *__restrict__ s, const float4 *__restrict__ coef, MixStep<T> mix) {
-    pdl_wait();
-    pdl_launch_dependents();
     const int64_t gid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t bd = gid >> log2_tpg;
     const int g = (int)(gid & ((1 << log2_tpg) - 1));
+    prefetch_step(x_t, mix, kMix, bd, BD, g);
+    pdl_wait();
+    pdl_launch_dependents();
     const int tpg = 1 << log2_tpg;
     const bool valid = bd < BD && 2 * g < M;
     MixPart<T> mp{};
@@ -148,11 +162,12 @@ template <typename T, bool kMix>
 __global__ void __launch_bounds__(kDecodeBlock) k_decode_any(
     const T *__restrict__ x_t, T *__restrict__ y_t, int64_t BD, int D, int M, int log2_tpg,
     int mpt, float2 *__restrict__ s, const float4 *__restrict__ coef, MixStep<T> mix) {
-    pdl_wait();
-    pdl_launch_dependents();
     const int64_t gid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     const int64_t bd = gid >> log2_tpg;
     const int g = (int)(gid & ((1 << log2_tpg) - 1));
+    prefetch_step(x_t, mix, kMix, bd, BD, g);
+    pdl_wait();
+    pdl_launch_dependents();
     const int tpg = 1 << log2_tpg;
     MixPart<T> mp{};
     if (kMix && bd < BD) mp = mix_part(mix, bd, D, g, tpg, x_t);
