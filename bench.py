@@ -710,6 +710,29 @@ def _bench_backward(rlm, torch, dev, hbm_peak, args):
         fts.append(a.elapsed_time(b))
     fms = statistics.mean(fts)
     del y, st, fw
+    # Backward with the state terms of a segmented training step: an initial state
+    # (its gradient returned) keeps the tcgen05 route; a terminal-state gradient as
+    # well takes the SIMT backward.
+    gen = torch.Generator(device="cpu").manual_seed(1)
+    s_in, ds_out, ds_in = (rlm.State.empty(B, D, M, device=dev) for _ in range(3))
+    s_in.s.copy_(torch.randn(B, D, M, 2, generator=gen))
+    ds_out.s.copy_(torch.randn(B, D, M, 2, generator=gen))
+
+    def _timed(fn):
+        fn()
+        out = []
+        for _ in range(3):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            out.append(a.elapsed_time(b))
+        return statistics.mean(out)
+
+    ms_init = _timed(lambda: rlm.rlm_mix_backward_from(dy, x, p, s_in, None, dx, g, ds_in, workspace=work))
+    ms_term = _timed(lambda: rlm.rlm_mix_backward_from(dy, x, p, s_in, ds_out, dx, g, ds_in, workspace=work))
+    del s_in, ds_out, ds_in
     gbs = backward_bytes(B, L, D, M) / (ms * 1e-3) / 1e9
     moved = backward_moved_bytes(B, L, D) / (ms * 1e-3) / 1e9
     return {"workload": "backward B=4 L=32768 D=512 M=32 bf16", "ms": round(ms, 4),
@@ -717,7 +740,10 @@ def _bench_backward(rlm, torch, dev, hbm_peak, args):
             "frac_hbm": round(gbs / hbm_peak, 4),
             "data_path": "transpose to channel-major, tcgen05 kernel, transpose back, fixed-order reduction",
             "moved_GBps": round(moved, 1), "moved_frac_hbm": round(moved / hbm_peak, 4),
-            "forward_ms": round(fms, 4), "forward_plus_backward_ms": round(fms + ms, 4)}
+            "forward_ms": round(fms, 4), "forward_plus_backward_ms": round(fms + ms, 4),
+            "with_state_in_ms": round(ms_init, 4),
+            "with_state_in_and_d_state_out_ms": round(ms_term, 4),
+            "state_terms_route": "state_in: tcgen05; d_state_out: SIMT chunked scan"}
 
 
 def run_backward_only(args):
