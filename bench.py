@@ -486,8 +486,9 @@ def _bench_decode(rlm, torch, dev, hbm_peak, B=None):
 def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
     """The mixer wrapper of Sec. 3.4 on the headline prefill shape: the gate alone
     (fused into the tcgen05 prefill) and the gate with the local path K = 4 and
-    drive history (the prefill, then one full-width pass); and the fused decode
-    step (B = 64) in a CUDA graph."""
+    drive history (the prefill, then one pass over whole-row tiles that also
+    applies the head coupling when there is one); and the fused decode step
+    (B = 64) in a CUDA graph."""
     from synth import make_inputs, make_mixer_inputs
     P = MIXER
     B, L, D, M, K = P["B"], P["L"], P["D"], P["M"], P["K"]
@@ -534,9 +535,9 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
         alg = mixer_prefill_bytes(B, L, D, M, kk) + (4 * H * H if cp is not None else 0)
         gbs = alg / (ms * 1e-3) / 1e9
         what = "gate fused into the tcgen05 prefill" if kk == 0 else \
-            f"gate and local path K={kk} with drive history: prefill then one full-width pass"
+            f"gate and local path K={kk} with drive history: prefill then one whole-row pass"
         if cp is not None:
-            what = f"head coupling H={H}, " + what.replace("prefill then one", "prefill, a coupling pass, then one")
+            what = f"head coupling H={H}, " + what.replace("one whole-row pass", "one whole-row pass with the coupling")
         return {"workload": f"mixer prefill B={B} L={L} D={D} M={M} bf16, {what}",
                 "ms": round(ms, 5), "Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 1),
                 "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),

@@ -361,11 +361,22 @@ rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm
         e = launch_prefill(path, x, p, state_in ? state_in->s : nullptr, z->ptr, state_out ? state_out->s : nullptr,
                            state_out ? state_out->coef : nullptr, ln);
     }
-    if (e == cudaSuccess && coupling)
-        e = couple_heads(z->ptr, x->dtype, coupling->c_raw, coupling->lambda_c, coupling->H, x->B, x->L, (int)x->D, st);
-    if (e == cudaSuccess && !fused && (g || K > 0))
-        e = mixer_epilogue(x->ptr, g ? g->ptr : nullptr, z->ptr, hin, K > 0 ? local->conv_w : nullptr,
-                           K > 0 ? local->scale : nullptr, x->dtype, x->B, x->L, (int)x->D, K, st);
+    const int H = coupling ? coupling->H : 0;
+    if (e == cudaSuccess && !fused && (g || K > 0 || coupling)) {
+        if (mixer_stream_supported(x->dtype, (int)x->D, H)) {
+            // Coupling, gate and local path in one pass over whole-row tiles.
+            e = mixer_stream(x->ptr, g ? g->ptr : nullptr, z->ptr, hin, K > 0 ? local->conv_w : nullptr,
+                             K > 0 ? local->scale : nullptr, K, coupling ? coupling->c_raw : nullptr,
+                             coupling ? coupling->lambda_c : 0.0f, H, x->dtype, x->B, x->L, (int)x->D, st);
+        } else {
+            if (coupling)
+                e = couple_heads(z->ptr, x->dtype, coupling->c_raw, coupling->lambda_c, H, x->B, x->L, (int)x->D,
+                                 st);
+            if (e == cudaSuccess && (g || K > 0))
+                e = mixer_epilogue(x->ptr, g ? g->ptr : nullptr, z->ptr, hin, K > 0 ? local->conv_w : nullptr,
+                                   K > 0 ? local->scale : nullptr, x->dtype, x->B, x->L, (int)x->D, K, st);
+        }
+    }
     if (e == cudaSuccess && hout) e = conv_tail(x->ptr, hin, hout, x->dtype, x->B, x->L, (int)x->D, K, st);
     if (e != cudaSuccess) return cuda_fail(e, "rlm_mixer_prefill launch");
     return RLM_OK;
@@ -545,11 +556,13 @@ rlm_status rlm_validate_params(const rlm_params *p) {
 
 rlm_status rlm_get_device_status(const rlm_launch *ln) {
     if (!ln) return fail(RLM_ERR_INVALID_ARG, "launch is NULL");
-    int status = RLM_OK, bwd = RLM_OK;
+    int status = RLM_OK, bwd = RLM_OK, mix = RLM_OK;
     cudaError_t e = read_and_clear_device_status(&status, static_cast<cudaStream_t>(ln->stream));
     if (e == cudaSuccess) e = read_and_clear_bwd_status(&bwd, static_cast<cudaStream_t>(ln->stream));
+    if (e == cudaSuccess) e = read_and_clear_mixer_status(&mix, static_cast<cudaStream_t>(ln->stream));
     if (e != cudaSuccess) return cuda_fail(e, "rlm_get_device_status");
     if (status == RLM_OK) status = bwd;
+    if (status == RLM_OK) status = mix;
     if (status != RLM_OK) return fail((rlm_status)status, "a bounded device-side wait expired");
     return RLM_OK;
 }

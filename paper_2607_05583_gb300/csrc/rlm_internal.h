@@ -94,6 +94,15 @@ cudaError_t couple_heads(void *z, rlm_dtype dt, const float *c_raw, float lambda
 cudaError_t mixer_finish_coupled(const void *x_t, const void *g_t, void *z_t, void *hist, const float *conv_w,
                                  const float *scale, int K, const float *c_raw, float lambda_c, int H, rlm_dtype dt,
                                  int B, int D, cudaStream_t st);
+// The whole mixer pass after the mixing, z <- sigma(g) (C z) + s (w * u) in place,
+// as one persistent kernel on whole-row tiles (rlm_mixer_stream.cu); g nullable,
+// K = 0 (no local path), H = 0 (no coupling; c_raw unused).  Covers the shapes
+// for which mixer_stream_supported() holds.
+bool mixer_stream_supported(rlm_dtype dt, int D, int H);
+cudaError_t mixer_stream(const void *x, const void *g, void *z, const void *hist, const float *conv_w,
+                         const float *scale, int K, const float *c_raw, float lambda_c, int H, rlm_dtype dt,
+                         int64_t B, int64_t L, int D, cudaStream_t st);
+cudaError_t read_and_clear_mixer_status(int *status, cudaStream_t st);
 // out = the last K-1 drives of hist || x (out may alias hist; no-op for K < 2).
 cudaError_t conv_tail(const void *x, const void *hist, void *out, rlm_dtype dt, int64_t B, int64_t L, int D,
                       int K, cudaStream_t st);

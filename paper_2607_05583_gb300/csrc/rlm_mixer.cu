@@ -16,6 +16,7 @@
 
 #include "rlm_device.cuh"
 #include "rlm_internal.h"
+#include "rlm_mixer.cuh"
 
 namespace rlm {
 namespace {
@@ -25,8 +26,6 @@ constexpr int kMaxK = RLM_MAX_LOCAL_K;
 constexpr int kTT = 64;    // tokens per tile
 constexpr int kTC = 128;   // channels per tile (a multiple of 8 channels is staged)
 constexpr int kEB = 256;   // threads per block of the mixer pass
-
-__device__ __forceinline__ float gatef(float v) { return __fdividef(1.0f, 1.0f + __expf(-v)); }
 
 // Two consecutive channels as floats, and back.
 __device__ __forceinline__ float2 ld2(const float *p) { return *reinterpret_cast<const float2 *>(p); }
@@ -129,14 +128,6 @@ __global__ void __launch_bounds__(kEB) k_mixer_epilogue(const T *__restrict__ x,
         }
         st2(z + (b * L + t) * D + c0 + c, o);
     }
-}
-
-// Head coupling (Sec. 3.4): C = I + (lambda_c / sqrt(H)) tanh(c_raw), built per
-// block in shared memory.
-__device__ __forceinline__ void build_coupling(float *C, const float *c_raw, float lam, int H) {
-    const float k = lam * rsqrtf((float)H);
-    for (int i = threadIdx.x; i < H * H; i += blockDim.x)
-        C[i] = (i / H == i % H ? 1.0f : 0.0f) + k * tanhf(__ldg(c_raw + i));
 }
 
 __device__ __forceinline__ float as_f(float v) { return v; }

@@ -67,6 +67,9 @@ def _check_prefill(inp, mx, z, so, cout, with_g, with_hist, s_in=None):
     (2, 1000, 16, 7, 3, "f32", True, True),                # SIMT, fp32
     (1, 500, 8, 40, 2, "bf16", True, True),                # SIMT, bf16 with M > 32
     (1, 5, 8, 16, 8, "bf16", True, True),                  # L shorter than the history
+    (1, 700, 2048, 16, 4, "bf16", True, True),             # 4 KB rows: the channel-pair pass instead
+    (1, 300, 1024, 7, 3, "f32", True, False),              # ... and in fp32
+    (1, 130, 16, 16, 8, "bf16", True, True),               # 64-token tiles: the history rows of tile 2
 ])
 def test_mixer_prefill_matches_oracle(B, L, D, M, K, dtype, with_g, with_hist):
     inp = make_inputs(B, L, D, M, dtype, seed=L + K)
@@ -330,6 +333,11 @@ def _coupling(H, seed, lam=0.7):
     (2, 3001, 64, 16, 4, 16, "bf16", True),          # 16 heads (the largest unrolled case)
     (1, 700, 48, 16, 3, 12, "bf16", True),           # 12 heads: H not unrolled, head width 4
     (1, 50, 8, 4, 2, 8, "f32", True),                # one channel per head
+    (2, 1000, 128, 16, 4, 16, "bf16", True),         # 16 heads of width 8: coupling in the whole-row pass
+    (2, 1000, 96, 16, 4, 12, "bf16", True),          # 12 heads of width 8: separate passes
+    (2, 700, 64, 7, 3, 4, "f32", True),              # ... fp32, 4 heads
+    (2, 600, 64, 16, 0, 4, "bf16", False),           # coupling alone, in the whole-row pass
+    (1, 300, 1024, 16, 2, 8, "f32", True),           # 4 KB rows: separate coupling and mixer passes
 ])
 def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
     inp = make_inputs(B, L, D, M, dtype, seed=L + H)
@@ -380,6 +388,25 @@ def test_coupled_mixer_decode_continues_the_prefill(dtype, M, K, H, B):
     assert_close(to_np(torch.stack(zs, 1)), zr[:, L0:], TOL[dtype], "decode z")
     if K > 1:
         np.testing.assert_array_equal(to_np(cs.u), tr)
+
+
+@pytest.mark.parametrize("D,H,passes", [(256, 8, 1), (64, 16, 1), (96, 12, 2), (2048, 8, 2)])
+def test_coupled_mixer_prefill_launches(D, H, passes):
+    """Coupling, gate and local path after the mixing: one whole-row pass where
+    the rows fit (at most 2 KB), H is 1, 2, 4, 8 or 16 and each head is a
+    multiple of 4 channels wide; else a coupling pass and a channel-pair pass;
+    then the history tail."""
+    inp = make_inputs(1, 300, D, 16, "bf16", seed=D + H)
+    mx = make_mixer_inputs(inp, 4, seed=D + H)
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    cin = rlm.ConvState(to_dev(mx.conv_in, "bf16"))
+    cout = rlm.ConvState.empty(1, D, 4, dtype=x.dtype)
+    z = torch.empty_like(x)
+    cp = rlm.Coupling.from_arrays(*_coupling(H, H))
+    n = _launches(lambda: rlm.rlm_mixer_prefill(x, g, p, local, z, conv_in=cin, conv_out=cout, coupling=cp))
+    assert n == 1 + passes + 1, n
 
 
 def test_zero_strength_coupling_is_no_coupling():
