@@ -712,8 +712,8 @@ def _bench_backward(rlm, torch, dev, hbm_peak, args):
     fms = statistics.mean(fts)
     del y, st, fw
     # Backward with the state terms of a segmented training step: an initial state
-    # (its gradient returned) keeps the tcgen05 route; a terminal-state gradient as
-    # well takes the SIMT backward.
+    # (its gradient returned), and a terminal-state gradient as well (a second pass
+    # of the tcgen05 kernel).
     gen = torch.Generator(device="cpu").manual_seed(1)
     s_in, ds_out, ds_in = (rlm.State.empty(B, D, M, device=dev) for _ in range(3))
     s_in.s.copy_(torch.randn(B, D, M, 2, generator=gen))
@@ -744,7 +744,8 @@ def _bench_backward(rlm, torch, dev, hbm_peak, args):
             "forward_ms": round(fms, 4), "forward_plus_backward_ms": round(fms + ms, 4),
             "with_state_in_ms": round(ms_init, 4),
             "with_state_in_and_d_state_out_ms": round(ms_term, 4),
-            "state_terms_route": "state_in: tcgen05; d_state_out: SIMT chunked scan"}
+            "state_terms_route": "tcgen05; d_state_out adds a second pass of the same kernel on a unit "
+                                 "drive at token L-1 read through c = conj(d_state_out)"}
 
 
 def run_backward_only(args):

@@ -273,10 +273,7 @@ size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype 
 
 size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
     if (B < 1 || L < 1 || D < 1 || M < 1) return 0;
-    // A call with a terminal-state gradient runs the SIMT backward even where the
-    // tcgen05 one applies, so the size covers both.
-    if (tc_backward_supported(B, L, D, M, dtype))
-        return std::max(tc_backward_ws_bytes(B, L, D, M), simt_backward_ws_bytes(B, L, D, M));
+    if (tc_backward_supported(B, L, D, M, dtype)) return tc_backward_ws_bytes(B, L, D, M);
     return simt_backward_ws_bytes(B, L, D, M);
 }
 
@@ -516,7 +513,7 @@ rlm_status rlm_mix_backward_from(const rlm_tensor *dy, const rlm_tensor *x, cons
     const float *gout = d_state_out ? d_state_out->s : nullptr;
     float *dsin = d_state_in ? d_state_in->s : nullptr;
     const int D = (int)x->D, M = p->M;
-    const bool tc = !gout && tc_backward_supported(x->B, x->L, D, M, x->dtype);
+    const bool tc = tc_backward_supported(x->B, x->L, D, M, x->dtype);
     if (!tc && simt_chunks(x->B, x->L, D) > 65535)
         return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
     const size_t need = rlm_backward_workspace_size(x->B, x->L, D, M, x->dtype);
@@ -524,7 +521,7 @@ rlm_status rlm_mix_backward_from(const rlm_tensor *dy, const rlm_tensor *x, cons
     cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
     cudaError_t e =
         tc ? tc_backward(dy->ptr, x->ptr, dx->ptr, x->B, x->L, D, M, p->decay, p->freq, p->amp,
-                         p->phase, sin, dsin, g->decay, g->freq, g->amp, g->phase, ln->workspace, st)
+                         p->phase, sin, gout, dsin, g->decay, g->freq, g->amp, g->phase, ln->workspace, st)
            : simt_backward(dy->ptr, x->ptr, dx->ptr, x->dtype, x->B, x->L, D, M, p->decay, p->freq,
                            p->amp, p->phase, sin, gout, dsin, g->decay, g->freq, g->amp, g->phase,
                            ln->workspace, st);

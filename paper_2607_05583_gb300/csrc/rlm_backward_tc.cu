@@ -306,6 +306,10 @@ struct BwdArgs {
     int row0;                 // first (b * D + d) row of this launch (0: the whole problem)
     float4 *coef_out;         // nullable, [D][M]   (time-reversed prefill)
     float2 *d_state_in;       // nullable, [B*D][M] (backward: gradient of the forward's state_in)
+    // nullable, [B*D][M]: the terminal-state pass (a unit drive at token L-1 read
+    // through c = conj(cconj[b * D + d][m]) per batch row); it writes c P as its P
+    // partial and adds to d_state_in.
+    const float2 *cconj;
     __nv_bfloat16 *dxT;       // [B*D][Lp]
     int64_t Lp;
     int D, M;
@@ -404,7 +408,9 @@ __global__ void __launch_bounds__(kThreads, 2)
         }
     } else if (tid >= 288 && tid < 288 + kMaxModes) {
         const int m = tid - 288;
-        cf[m] = m < M ? mode_coef(args.amp[d * M + m], args.phase[d * M + m]) : make_float2(0.0f, 0.0f);
+        cf[m] = m >= M ? make_float2(0.0f, 0.0f)
+                : args.cconj ? conj2(args.cconj[(int64_t)row * M + m])
+                             : mode_coef(args.amp[d * M + m], args.phase[d * M + m]);
     }
     if (tid < 128) reinterpret_cast<float *>(smem + kOffRho)[tid] = 0.0f;
     __syncthreads();
@@ -768,8 +774,15 @@ __global__ void __launch_bounds__(kThreads, 2)
                 pi += pin.y;
             }
             if (args.d_state_in) {
-                const float2 cls = cmul(mode_coef(args.amp[d * M + mE], args.phase[d * M + mE]), ls);
-                args.d_state_in[(int64_t)row * M + mE] = make_float2(cls.x, -cls.y);
+                const float2 c = args.cconj ? conj2(args.cconj[(int64_t)row * M + mE])
+                                            : mode_coef(args.amp[d * M + mE], args.phase[d * M + mE]);
+                const float2 cls = cmul(c, ls);
+                float2 ds = make_float2(cls.x, -cls.y);
+                if (args.cconj) {
+                    const float2 prev = args.d_state_in[(int64_t)row * M + mE];
+                    ds = make_float2(prev.x + ds.x, prev.y + ds.y);
+                }
+                args.d_state_in[(int64_t)row * M + mE] = ds;
             }
         }
 #pragma unroll
@@ -780,8 +793,10 @@ __global__ void __launch_bounds__(kThreads, 2)
             pi += __shfl_xor_sync(0xffffffffu, pi, o);
         }
         if (s == 0 && onE) {
+            float2 pp = make_float2(pr, pi);
+            if (args.cconj) pp = cmul(conj2(args.cconj[(int64_t)row * M + mE]), pp);   // conj(g) J
             args.part_g[(int64_t)row * M + mE] = make_float2(gr, gi);
-            args.part_p[(int64_t)row * M + mE] = make_float2(pr, pi);
+            args.part_p[(int64_t)row * M + mE] = pp;
         }
     }
 }
@@ -836,9 +851,11 @@ __global__ void __launch_bounds__(128) k_to_channel_major(const __nv_bfloat16 *_
 // [B*D][Lp] -> [B][L][D] for tokens t < L, token t read from position t, or from
 // L - 1 - t when rev.  A tile covers 64 tokens x 64 channels; it loads the
 // 8-aligned window of 72 positions that holds its (reversed) positions.
+// acc: add to what dst holds (one more bf16 rounding) instead of overwriting it.
 __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__restrict__ srcT,
                                                       __nv_bfloat16 *__restrict__ dst, int64_t L, int D,
-                                                      int64_t Lp, int rev, int b0, int c_lo, int c_hi) {
+                                                      int64_t Lp, int rev, int b0, int c_lo, int c_hi,
+                                                      int acc) {
     __shared__ uint32_t tile[64][37];   // [channel][position pair]
     const int64_t t0 = (int64_t)blockIdx.x * 64;
     const int c0 = c_lo + blockIdx.y * 64;
@@ -872,7 +889,18 @@ __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__res
             const uint32_t hi = (i & 1) ? (bw >> 16) : (bw & 0xffffu);
             w[e] = lo | (hi << 16);
         }
-        *reinterpret_cast<uint4 *>(dst + ((int64_t)b * L + t) * D + c) = make_uint4(w[0], w[1], w[2], w[3]);
+        uint4 *out = reinterpret_cast<uint4 *>(dst + ((int64_t)b * L + t) * D + c);
+        if (acc) {
+            const uint4 o = *out;
+            const uint32_t ov[4] = {o.x, o.y, o.z, o.w};
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float lo = __uint_as_float(w[e] << 16) + __uint_as_float(ov[e] << 16);
+                const float hi = __uint_as_float(w[e] & 0xffff0000u) + __uint_as_float(ov[e] & 0xffff0000u);
+                asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(w[e]) : "f"(hi), "f"(lo));
+            }
+        }
+        *out = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -929,7 +957,7 @@ bool tc_backward_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
 }
 
 size_t tc_backward_ws_bytes(int64_t B, int64_t L, int D, int M) {
-    return 3 * field_bytes(B, L, D) + 2 * part_bytes(B, D, M);
+    return 3 * field_bytes(B, L, D) + 4 * part_bytes(B, D, M);   // + the terminal-state pass's partials
 }
 
 namespace {
@@ -964,6 +992,7 @@ BwdArgs base_args(const float *decay, const float *freq, const float *amp, const
     a.state_out = nullptr;
     a.coef_out = nullptr;
     a.d_state_in = nullptr;
+    a.cconj = nullptr;
     a.dxT = outT;
     a.Lp = Lp;
     a.D = D;
@@ -990,17 +1019,24 @@ cudaError_t run_layout_and_scan(const CUtensorMap &mdy, const CUtensorMap &mx, B
     a.row0 = 0;
     k_backward_tc<kGrad><<<(unsigned)(B * D), kThreads, kSmemBytes, st>>>(mdy, mx, a);
     k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(outT, out, L, D, Lp, rev, 0,
-                                                                                     0, D);
+                                                                                     0, D, 0);
     count_launches(3);
     return cudaGetLastError();
 }
 
 }  // namespace
 
+// The terminal-state pass's drive: 1 at token L-1 of every row, 0 elsewhere
+// (the rows were zeroed before).
+__global__ void k_unit_last(__nv_bfloat16 *dT, int64_t rows, int64_t Lp, int64_t L) {
+    const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (r < rows) dT[r * Lp + (L - 1)] = __float2bfloat16_rn(1.0f);
+}
+
 cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
                         const float *decay, const float *freq, const float *amp, const float *phase,
-                        const float *state_in, float *d_state_in, float *g_decay, float *g_freq, float *g_amp,
-                        float *g_phase, void *ws, cudaStream_t st) {
+                        const float *state_in, const float *d_state_out, float *d_state_in, float *g_decay,
+                        float *g_freq, float *g_amp, float *g_phase, void *ws, cudaStream_t st) {
     if (!ws) return cudaErrorInvalidValue;
     const int64_t Lp = padded_len(L);
     char *w = static_cast<char *>(ws);
@@ -1009,6 +1045,8 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     auto *dxT = reinterpret_cast<__nv_bfloat16 *>(w + 2 * field_bytes(B, L, D));
     auto *pg = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D));
     auto *pp = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + part_bytes(B, D, M));
+    auto *pg2 = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + 2 * part_bytes(B, D, M));
+    auto *pj = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + 3 * part_bytes(B, D, M));
     const int64_t rows = B * (int64_t)D;
     CUtensorMap mdy, mx;
     if (!make_chunk_map(&mdy, dyT, rows, Lp) || !make_chunk_map(&mx, xT, rows, Lp)) return cudaErrorInvalidValue;
@@ -1023,7 +1061,29 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
                          static_cast<const __nv_bfloat16 *>(dy), xT, dyT, 2, 0, dxT,
                          static_cast<__nv_bfloat16 *>(dx), st);
     if (e != cudaSuccess) return e;
-    return grad_reduce(rows / D, D, M, amp, phase, pg, pp, g_decay, g_freq, g_amp, g_phase, st);
+    if (d_state_out) {
+        // A terminal-state gradient g adds Re(conj(g) lambda^(L-1-t)) to dx_t,
+        // conj(g) J to the decay / frequency products and g conj(lambda^L) to the
+        // gradient of s_in (Sec. 3.2-3.3).  These are exactly what the same
+        // backward gives for a unit drive at token L-1 read through c = conj(g)
+        // (per batch row): its dx, c P (P = J with the s_in term) and
+        // conj(c lambda S_0).  So a second pass runs on that drive, reusing the
+        // channel-major x, and its dx is added to the first.
+        if ((e = cudaMemsetAsync(dyT, 0, (size_t)rows * Lp * 2, st)) != cudaSuccess) return e;
+        k_unit_last<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(dyT, rows, Lp, L);
+        BwdArgs a2 = a;
+        a2.part_g = pg2;
+        a2.part_p = pj;
+        a2.cconj = reinterpret_cast<const float2 *>(d_state_out);
+        k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a2);
+        const unsigned cg = (unsigned)((D + 63) / 64);
+        k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(
+            dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp, 0, 0, 0, D, 1);
+        count_launches(3);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    return grad_reduce(rows / D, D, M, amp, phase, pg, pp, d_state_out ? pj : nullptr, g_decay, g_freq, g_amp,
+                       g_phase, st);
 }
 
 bool tc_prefill_rev_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {

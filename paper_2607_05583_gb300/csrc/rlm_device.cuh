@@ -29,6 +29,7 @@ __device__ __forceinline__ void st_elem<__nv_bfloat16>(__nv_bfloat16 *p, float v
 __device__ __forceinline__ float2 cmul(float2 a, float2 b) {
     return make_float2(fmaf(a.x, b.x, -a.y * b.y), fmaf(a.x, b.y, a.y * b.x));
 }
+__device__ __forceinline__ float2 conj2(float2 a) { return make_float2(a.x, -a.y); }
 // a*b + c
 __device__ __forceinline__ float2 cfma(float2 a, float2 b, float2 c) {
     return make_float2(fmaf(a.x, b.x, fmaf(-a.y, b.y, c.x)), fmaf(a.x, b.y, fmaf(a.y, b.x, c.y)));

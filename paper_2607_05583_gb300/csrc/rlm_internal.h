@@ -46,20 +46,21 @@ cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt,
                           cudaStream_t st);
 
 // Fixed-order (fp64) sum of nparts partial (G, P) arrays of [D][M] each, then the
-// four parameter gradients.
+// four parameter gradients.  J (nullable): nparts partials of conj(g) J from a
+// terminal-state gradient g, whose sum's -Re and -Im join dgamma and domega.
 cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const float *phase,
-                        const float2 *G, const float2 *P, float *g_decay, float *g_freq,
+                        const float2 *G, const float2 *P, const float2 *J, float *g_decay, float *g_freq,
                         float *g_amp, float *g_phase, cudaStream_t st);
 
 // ---- tcgen05 backward (rlm_backward_tc.cu) -----------------------------------
 bool tc_backward_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
 size_t tc_backward_ws_bytes(int64_t B, int64_t L, int D, int M);
-// state_in (the forward's initial state) and d_state_in (output) may be null; a
-// terminal-state gradient is not covered here (the SIMT backward takes it).
+// state_in (the forward's initial state), d_state_out (the loss gradient of the
+// terminal state) and d_state_in (output) may be null.
 cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
                         const float *decay, const float *freq, const float *amp, const float *phase,
-                        const float *state_in, float *d_state_in, float *g_decay, float *g_freq, float *g_amp,
-                        float *g_phase, void *ws, cudaStream_t st);
+                        const float *state_in, const float *d_state_out, float *d_state_in, float *g_decay,
+                        float *g_freq, float *g_amp, float *g_phase, void *ws, cudaStream_t st);
 cudaError_t read_and_clear_bwd_status(int *status, cudaStream_t st);
 // The causal prefill (bf16 I/O, M <= 32) as the same reverse-time tcgen05 scan
 // applied to the time-reversed drive; used for the M the tcgen05 prefill does not

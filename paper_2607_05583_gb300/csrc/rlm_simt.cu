@@ -444,10 +444,10 @@ cudaError_t simt_prefill(const void *x, void *y, rlm_dtype dt, int64_t B, int64_
 }
 
 cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const float *phase,
-                        const float2 *G, const float2 *P, float *g_decay, float *g_freq,
+                        const float2 *G, const float2 *P, const float2 *J, float *g_decay, float *g_freq,
                         float *g_amp, float *g_phase, cudaStream_t st) {
     k_grad_reduce<<<(unsigned)((D * M + 255) / 256), 256, 0, st>>>(
-        nparts, D, M, 1, amp, phase, G, P, nullptr, g_decay, g_freq, g_amp, g_phase);
+        nparts, D, M, 1, amp, phase, G, P, J, g_decay, g_freq, g_amp, g_phase);
     count_launches(1);
     return cudaGetLastError();
 }

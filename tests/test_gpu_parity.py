@@ -406,17 +406,22 @@ def test_backward_matches_oracle(B, L, D, M, dtype):
 
 
 @pytest.mark.parametrize("B,L,D,M,dtype,with_s,with_g", [
-    # tensor-core backward: state_in, its gradient, no terminal-state gradient
+    # tensor-core backward: state_in and its gradient
     (2, 3001, 16, 16, "bf16", True, False),
     (1, 2 * 2048 + 1, 8, 32, "bf16", True, False),
     (3, 65, 8, 5, "bf16", True, False),
     (2, 3001, 16, 16, "bf16", False, False),
-    # SIMT: a terminal-state gradient (any dtype), fp32, bf16 with M > 32
+    # ... with a terminal-state gradient (the second pass on a unit drive at L-1)
     (2, 3001, 16, 16, "bf16", True, True),
     (1, 700, 8, 32, "bf16", False, True),
+    (3, 65, 8, 5, "bf16", True, True),
+    (1, 2 * 2048, 8, 32, "bf16", True, True),
+    (2, 1, 8, 16, "bf16", True, True),
+    # SIMT: fp32, bf16 with M > 32
     (2, 1000, 16, 7, "f32", True, True),
     (1, 1, 8, 3, "f32", True, True),
     (1, 700, 8, 40, "bf16", True, False),
+    (1, 700, 8, 40, "bf16", True, True),
 ])
 def test_backward_with_state_terms_matches_oracle(B, L, D, M, dtype, with_s, with_g):
     """Backward of prefill_from (Sec. 3.2-3.3 with an initial state): dx, the four
@@ -450,6 +455,34 @@ def test_backward_with_state_terms_matches_oracle(B, L, D, M, dtype, with_s, wit
         assert_close(got, ref, TOL[dtype], "dstate_in " + part)
 
 
+@pytest.mark.parametrize("decay_scale,L", [(1.0, 3001), (40.0, 2077)])
+def test_terminal_gradient_with_silent_modes_matches_oracle(decay_scale, L):
+    """A terminal-state gradient reaches modes with zero amplitude (c = 0: they add
+    nothing to y, but the terminal state still depends on them), and fast decays
+    with a ragged sequence end (the tensor-core route's second pass)."""
+    B, D, M = 2, 16, 16
+    inp = make_inputs(B, L, D, M, "bf16", seed=L, with_dy=True)
+    decay, freq, amp, phase = (a.copy() for a in inp.params())
+    amp[:, ::3] = 0.0
+    decay *= decay_scale
+    rng = np.random.default_rng(L)
+    g_out = rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M))
+    s_in = rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M))
+    x, dy = to_dev(inp.x, "bf16"), to_dev(inp.dy, "bf16")
+    p = rlm.Params.from_arrays(decay, freq, amp, phase)
+    dx, g, ds = torch.empty_like(x), rlm.Grads.empty(D, M), rlm.State.empty(B, D, M)
+    rlm.rlm_mix_backward_from(dy, x, p, _state_from(inp, s_in), _state_from(inp, g_out), dx, g, ds)
+    torch.cuda.synchronize()
+    dx_ref, g_ref = oracle.backward_rec(inp.x, inp.dy, decay, freq, amp, phase, state_in=s_in,
+                                        d_state_out=g_out)
+    assert_close(to_np(dx), dx_ref, TOL["bf16"], "dx")
+    for k in ("decay", "freq", "amp", "phase"):
+        assert_close(getattr(g, k).cpu().numpy(), g_ref[k], TOL["bf16"], "d" + k)
+    ds_np = ds.complex().cpu().numpy()
+    assert_close(ds_np.real, g_ref["state_in"].real, TOL["bf16"], "dstate_in re")
+    assert_close(ds_np.imag, g_ref["state_in"].imag, TOL["bf16"], "dstate_in im")
+
+
 def test_backward_from_without_state_terms_equals_backward():
     """No state arguments: the same kernels and bit-identical results as rlm_mix_backward."""
     inp = make_inputs(2, 3001, 64, 16, "bf16", seed=12, with_dy=True)
@@ -468,8 +501,8 @@ def test_backward_from_without_state_terms_equals_backward():
 def test_split_backward_chains_state_gradients():
     """Backward through a split sequence x1 || x2: the second half's backward with
     state_in = state after x1 gives d_state_in, which fed as d_state_out into the
-    first half's backward reproduces the whole sequence's gradients (bf16, fp32
-    terminal-gradient path in the first half)."""
+    first half's backward reproduces the whole sequence's gradients (bf16; the
+    first half's backward takes the terminal-state gradient)."""
     B, L, D, M, cut = 2, 5000, 16, 16, 2345
     inp = make_inputs(B, L, D, M, "bf16", seed=41, with_dy=True)
     x, dy = to_dev(inp.x, "bf16"), to_dev(inp.dy, "bf16")
