@@ -136,7 +136,11 @@ RLM_API rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm
  *              not overlap y.  state_out may be the same buffer (in-place
  *              continuation); partial overlap is rejected.
  * Other arguments, the workspace (rlm_prefill_workspace_size) and the paths
- * taken are those of rlm_mix_prefill. */
+ * taken are those of rlm_mix_prefill.  Range: on the time-reversed tcgen05 path
+ * (bf16, 16 < M <= 32, few batch rows and channel groups) with L not a multiple of
+ * 64, state_in enters as lambda^(L - L') s_in, L' = L rounded up to 64, whose
+ * modulus exp(decay (L' - L)) exceeds fp32 for decays above 88 / 63 (a half-life
+ * under half a token); keep decays below that there. */
 RLM_API rlm_status rlm_mix_prefill_from(const rlm_tensor *x, const rlm_params *p, const rlm_state *state_in,
                                         rlm_tensor *y, rlm_state *state_out, const rlm_launch *launch);
 
