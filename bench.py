@@ -327,9 +327,33 @@ def run_ours(args):
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / reps
+    # The same schedule without the prefill: what the host link alone allows with
+    # both directions busy (the bound on e2e; the prefill hides under the copies).
+    def copy_steps(n):
+        for s_ in (s_in, s_out):
+            s_.wait_stream(stream)
+        for i in range(n):
+            k = i % 2
+            with torch.cuda.stream(s_in):
+                xs[k].copy_(xh, non_blocking=True)
+            with torch.cuda.stream(s_out):
+                yhs[k].copy_(ys[k], non_blocking=True)
+        for s_ in (s_in, s_out):
+            stream.wait_stream(s_)
+
+    copy_steps(3)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    copy_steps(reps)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    copy_ms = e0.elapsed_time(e1) / reps
     e2e = {"value": round(tokens / (e2e_ms * 1e-3) / 1e6, 2), "unit": "Mtok/s",
            "h2d_bytes_per_step": xh.numel() * 2, "d2h_bytes_per_step": yhs[0].numel() * 2,
-           "schedule": "copy-in, prefill and copy-out of consecutive steps overlapped on three streams"}
+           "schedule": "copy-in, prefill and copy-out of consecutive steps overlapped on three streams",
+           "copy_only_ms_per_step": round(copy_ms, 4),
+           "link_GBps_each_way": round(xh.numel() * 2 / (copy_ms * 1e-3) / 1e9, 1),
+           "frac_of_copy_only": round(copy_ms / e2e_ms, 4)}
     del xh, yhs, xs, ys
 
     # ---------------- per-L sweep (same launch configuration)
