@@ -58,11 +58,11 @@ def _peaks():
         return 6800.0, 1900.0, "fallback"
 
 
-def prefill_bytes(B, L, D, M):
-    """Algorithmic HBM bytes of one bf16 prefill: read x, write y (2 B each per
-    token-channel), write the terminal state (8 B per (b,d,m)) and its
-    coefficients (16 B per (d,m)), read the parameters (16 B per (d,m))."""
-    return B * L * D * 4 + B * D * M * 8 + D * M * 32
+def prefill_bytes(B, L, D, M, elem=2):
+    """Algorithmic HBM bytes of one prefill: read x, write y (elem = 2 B each per
+    token-channel in bf16, 4 in fp32), write the terminal state (8 B per (b,d,m))
+    and its coefficients (16 B per (d,m)), read the parameters (16 B per (d,m))."""
+    return B * L * D * 2 * elem + B * D * M * 8 + D * M * 32
 
 
 def decode_bytes(B, D, M):
@@ -365,6 +365,10 @@ def run_ours(args):
         # the 6M layer's prefill (B = 8, L = 2048)
         sweep["layer6m_B8_L2048"] = _time_prefill(rlm, torch, dev, 8, 2048, P["D"], P["M"], flush,
                                                   hbm_peak, reps=max(5, args.steps // 2))
+        # fp32 I/O on the headline shape (the SIMT chunked scan; 8 B per token-channel)
+        sweep[f"fp32_B{P['B']}_L{P['L']}"] = _time_prefill(rlm, torch, dev, P["B"], P["L"], P["D"], P["M"],
+                                                           flush, hbm_peak, reps=max(5, args.steps // 2),
+                                                           dtype="f32")
     sweep[f"B{P['B']}_L{P['L']}"] = {"Mtok_s": round(tokens / (ms * 1e-3) / 1e6, 1),
                                      "frac": roofline["frac"]}
     del x, y, work
@@ -432,14 +436,14 @@ def _io_ceiling(rlm, torch, x, y, flush, stream, P, achieved, reps=5):
     return out
 
 
-def _time_prefill(rlm, torch, dev, B, L, D, M, flush, hbm_peak, reps=5):
+def _time_prefill(rlm, torch, dev, B, L, D, M, flush, hbm_peak, reps=5, dtype="bf16"):
     from synth import make_inputs
-    inp = make_inputs(B, L, D, M, "bf16", seed=1)
-    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
+    inp = make_inputs(B, L, D, M, dtype, seed=1)
+    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16 if dtype == "bf16" else torch.float32)
     p = rlm.Params.from_arrays(*inp.params(), device=dev)
     y = torch.empty_like(x)
     st = rlm.State.empty(B, D, M, device=dev)
-    wsz = rlm.rlm_prefill_workspace_size(B, L, D, M, torch.bfloat16)
+    wsz = rlm.rlm_prefill_workspace_size(B, L, D, M, x.dtype)
     work = torch.empty(max(wsz, 256), dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
     for _ in range(3):
@@ -454,7 +458,7 @@ def _time_prefill(rlm, torch, dev, B, L, D, M, flush, hbm_peak, reps=5):
         torch.cuda.synchronize()
         ts.append(a.elapsed_time(b))
     ms = statistics.mean(ts)
-    gbs = prefill_bytes(B, L, D, M) / (ms * 1e-3) / 1e9
+    gbs = prefill_bytes(B, L, D, M, 2 if dtype == "bf16" else 4) / (ms * 1e-3) / 1e9
     return {"Mtok_s": round(B * L / (ms * 1e-3) / 1e6, 1), "ms": round(ms, 5),
             "frac": round(gbs / hbm_peak, 4)}
 
@@ -617,17 +621,20 @@ def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
     per = mixer_decode_bytes(Bd, D, M, K)
     dgbs = per / (us * 1e-6) / 1e9
     decode = {"workload": f"fused mixer decode B={Bd} D={D} M={M} K={K}, {T} steps, CUDA graph",
-              "us_per_step": round(us, 4), "tok_s": round(Bd * T / (us * 1e-6), 1),
+              "us_per_step": round(us, 4), "tok_s": round(Bd / (us * 1e-6), 1),
               "achieved_GBps": round(dgbs, 1), "frac_hbm": round(dgbs / hbm_peak, 4), "bytes_per_step": per}
     dcp = rlm.Coupling.from_arrays(np.random.default_rng(6).standard_normal((H, H)), 0.5, device=dev)
     graph_c = torch.cuda.CUDAGraph()
+    n0 = rlm.rlm_kernels_launched()
     with torch.cuda.graph(graph_c):
         for t in range(T):
             rlm.rlm_mixer_decode(toks[t], gts[t], dst, dlocal, hist, outs[t], coupling=dcp)
+    lps = (rlm.rlm_kernels_launched() - n0) / T
     uc = replay_us(graph_c)
-    decode_coupled = {"workload": f"mixer decode with head coupling H={H}, B={Bd} D={D} M={M} K={K}: recurrence "
-                                  f"step, then one block per batch row; {T} steps, CUDA graph",
-                      "us_per_step": round(uc, 4), "tok_s": round(Bd * T / (uc * 1e-6), 1), "launches_per_step": 2}
+    decode_coupled = {"workload": f"mixer decode with head coupling H={H}, B={Bd} D={D} M={M} K={K}: one block "
+                                  f"per batch row (recurrence step, coupling, gate, local path); {T} steps, "
+                                  f"CUDA graph",
+                      "us_per_step": round(uc, 4), "tok_s": round(Bd / (uc * 1e-6), 1), "launches_per_step": lps}
     return {"prefill_gate": prefill_gate, "prefill": prefill, "prefill_coupled": prefill_coupled, "decode": decode,
             "decode_coupled": decode_coupled}
 

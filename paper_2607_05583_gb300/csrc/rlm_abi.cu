@@ -440,7 +440,15 @@ rlm_status rlm_mixer_decode(const rlm_tensor *x_t, const rlm_tensor *g_t, rlm_st
     }
     cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
     cudaError_t e;
-    if (coupling) {
+    if (mixer_decode_coupled_supported((int)x_t->D, state->M)) {
+        // One launch, one block per batch row: recurrence step, coupling (if any),
+        // gate, local path.
+        e = mixer_decode_coupled(x_t->ptr, g_t ? g_t->ptr : nullptr, z_t->ptr, x_t->dtype, (int)x_t->B,
+                                 (int)x_t->D, state->M, state->s, state->coef, K >= 2 ? conv->u : nullptr,
+                                 K > 0 ? local->conv_w : nullptr, K > 0 ? local->scale : nullptr, K,
+                                 coupling ? coupling->c_raw : nullptr, coupling ? coupling->lambda_c : 0.0f,
+                                 coupling ? coupling->H : 0, st);
+    } else if (coupling) {
         // The recurrence step writes y_t into z_t; one block per batch row then
         // couples the heads and applies the gate and the local path.
         e = decode_step(x_t->ptr, z_t->ptr, x_t->dtype, (int)x_t->B, (int)x_t->D, state->M, state->s, state->coef, st);

@@ -19,6 +19,7 @@
 // latency when decode steps are issued back to back or captured in a graph.
 #include "rlm_device.cuh"
 #include "rlm_internal.h"
+#include "rlm_mixer.cuh"
 
 namespace rlm {
 namespace {
@@ -230,6 +231,116 @@ cudaError_t launch_pdl(Kern kern, unsigned grid, cudaStream_t st, Args... args) 
     return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+// One decode step with head coupling (Sec. 3.4) in a single launch, one block per
+// batch row, for rows of at most 512 channels and 4096 modes.  Right after the
+// dependency wait every load of the step is issued at once: the thread of channel
+// d (threadIdx.x) takes its token, gate, drive history and conv weights, and every
+// thread takes its (at most four) float4 mode pairs of the row's state slab with
+// their coefficients -- consecutive threads on consecutive pairs, so the M / 2
+// threads of a channel form one aligned shuffle group.  Phase 1 updates the
+// states and puts each channel's readout y_t[d] in shared memory (fp32); after
+// the block barrier, phase 2 forms (C y_t)[d], applies the gate and the local
+// path, shifts the history and writes z_t[d].  C depends on the parameters only,
+// so it is built before the wait.  H = 0: no coupling (the mixer step alone).
+constexpr int kCoupledBlock = 512;
+constexpr int kCoupledIters = 4;               // mode pairs per thread
+constexpr int kCoupledMaxModesPerRow = 2 * kCoupledIters * kCoupledBlock;   // D * M <= 4096
+constexpr int kHistMax = RLM_MAX_LOCAL_K - 1;
+
+template <typename T>
+__global__ void __launch_bounds__(kCoupledBlock, 1) k_decode_coupled(
+    const T *__restrict__ x_t, T *__restrict__ z_t, int D, int M, float4 *__restrict__ s,
+    const float4 *__restrict__ coef, MixStep<T> mix, const float *__restrict__ c_raw, float lam, int H) {
+    extern __shared__ __align__(16) float smf[];
+    float *C = smf;                              // [H][H]
+    float *ys = smf + ((H * H + 3) & ~3);        // [D]
+    const int64_t b = blockIdx.x;
+    if (H > 0) build_coupling(C, c_raw, lam, H);
+    pdl_wait();
+    pdl_launch_dependents();
+    const T *xb = x_t + b * D;
+    // ---- loads: phase 2's inputs (channel d2) ...
+    const int d2 = threadIdx.x, K = mix.K;
+    const bool ch = d2 < D;
+    T xraw = T(0.0f), hv[kHistMax];
+    float gv = 0.0f, sc = 0.0f, w0 = 0.0f, wj[kHistMax];   // wj[j]: the weight of history entry j
+    T *hc = mix.hist + b * (K > 1 ? K - 1 : 0) * (int64_t)D + d2;
+    if (ch) {
+        xraw = xb[d2];
+        if (mix.g) gv = ld_elem(mix.g + b * D + d2);
+        if (K > 0) {
+            sc = __ldg(mix.scale + d2);
+            w0 = __ldg(mix.conv_w + (int64_t)d2 * K);
+#pragma unroll
+            for (int j = 0; j < kHistMax; ++j) {
+                if (j < K - 1) {
+                    hv[j] = hc[(int64_t)j * D];
+                    wj[j] = __ldg(mix.conv_w + (int64_t)d2 * K + (K - 1 - j));
+                }
+            }
+        }
+    }
+    // ... and phase 1's states, coefficients and tokens.
+    const int pairs = M / 2;                     // a power of two, at most 32
+    const int lp = __ffs(pairs) - 1;
+    const int n4 = D * pairs;
+    float4 *sb = s + b * n4;
+    float4 stv[kCoupledIters], c0v[kCoupledIters], c1v[kCoupledIters];
+    float xv[kCoupledIters];
+#pragma unroll
+    for (int k = 0; k < kCoupledIters; ++k) {
+        const int i = (int)threadIdx.x + k * kCoupledBlock;
+        const int d = i >> lp, g = i & (pairs - 1);
+        if (i < n4) {
+            xv[k] = ld_elem(xb + d);
+            stv[k] = sb[i];
+            c0v[k] = __ldg(coef + (int64_t)d * M + 2 * g);
+            c1v[k] = __ldg(coef + (int64_t)d * M + 2 * g + 1);
+        }
+    }
+    // ---- phase 1: every thread runs every iteration, so whole warps shuffle
+#pragma unroll
+    for (int k = 0; k < kCoupledIters; ++k) {
+        const int i = (int)threadIdx.x + k * kCoupledBlock;
+        const bool on = i < n4;
+        const int d = i >> lp, g = i & (pairs - 1);
+        float acc = 0.0f;
+        if (on) {
+            const float4 st = stv[k], c0 = c0v[k], c1 = c1v[k];
+            const float r0 = fmaf(c0.x, st.x, fmaf(-c0.y, st.y, xv[k]));
+            const float i0 = fmaf(c0.x, st.y, c0.y * st.x);
+            const float r1 = fmaf(c1.x, st.z, fmaf(-c1.y, st.w, xv[k]));
+            const float i1 = fmaf(c1.x, st.w, c1.y * st.z);
+            sb[i] = make_float4(r0, i0, r1, i1);
+            acc = fmaf(c0.z, r0, fmaf(-c0.w, i0, fmaf(c1.z, r1, -c1.w * i1)));
+        }
+        for (int o = pairs >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (on && g == 0) ys[d] = acc;
+    }
+    __syncthreads();
+    // ---- phase 2
+    if (!ch) return;
+    float v = ys[d2];
+    if (H > 0) {
+        const int dh = D / H, gh = d2 / dh, jh = d2 % dh;
+        v = 0.0f;
+        for (int h = 0; h < H; ++h) v = fmaf(C[gh * H + h], ys[h * dh + jh], v);
+    }
+    if (mix.g) v *= gatef(gv);
+    if (K > 0) {
+        float l = w0 * as_float(xraw);
+#pragma unroll
+        for (int j = 0; j < kHistMax; ++j)
+            if (j < K - 1) l = fmaf(wj[j], as_float(hv[j]), l);
+#pragma unroll
+        for (int j = 1; j < kHistMax; ++j)
+            if (j < K - 1) hc[(int64_t)(j - 1) * D] = hv[j];
+        if (K > 1) hc[(int64_t)(K - 2) * D] = xraw;
+        v = fmaf(sc, l, v);
+    }
+    st_elem(z_t + b * D + d2, v);
+}
+
 template <typename T, bool kMix>
 cudaError_t decode_t(const T *x_t, T *y_t, int B, int D, int M, float *s, const float *coef,
                      MixStep<T> mix, cudaStream_t st) {
@@ -275,6 +386,39 @@ cudaError_t mixer_decode_step(const void *x_t, const void *g_t, void *z_t, rlm_d
     const MixStep<float> m{static_cast<const float *>(g_t), static_cast<float *>(hist), conv_w, scale, K};
     return decode_t<float, true>(static_cast<const float *>(x_t), static_cast<float *>(z_t), B, D, M, s, coef, m,
                                  st);
+}
+
+bool mixer_decode_coupled_supported(int D, int M) {
+    const int pairs = M / 2;
+    return M % 2 == 0 && pairs >= 1 && pairs <= 32 && (pairs & (pairs - 1)) == 0 && D <= kCoupledBlock &&
+           (int64_t)D * M <= kCoupledMaxModesPerRow;
+}
+
+cudaError_t mixer_decode_coupled(const void *x_t, const void *g_t, void *z_t, rlm_dtype dt, int B, int D, int M,
+                                 float *s, const float *coef, void *hist, const float *conv_w, const float *scale,
+                                 int K, const float *c_raw, float lambda_c, int H, cudaStream_t st) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)B);
+    cfg.blockDim = dim3(kCoupledBlock);
+    cfg.dynamicSmemBytes = (size_t)(((H * H + 3) & ~3) + D) * sizeof(float);
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    count_launches(1);
+    float4 *s4 = reinterpret_cast<float4 *>(s);
+    const float4 *cf = reinterpret_cast<const float4 *>(coef);
+    if (dt == RLM_BF16) {
+        using T = __nv_bfloat16;
+        const MixStep<T> m{static_cast<const T *>(g_t), static_cast<T *>(hist), conv_w, scale, K};
+        return cudaLaunchKernelEx(&cfg, k_decode_coupled<T>, static_cast<const T *>(x_t), static_cast<T *>(z_t), D,
+                                  M, s4, cf, m, c_raw, lambda_c, H);
+    }
+    const MixStep<float> m{static_cast<const float *>(g_t), static_cast<float *>(hist), conv_w, scale, K};
+    return cudaLaunchKernelEx(&cfg, k_decode_coupled<float>, static_cast<const float *>(x_t),
+                              static_cast<float *>(z_t), D, M, s4, cf, m, c_raw, lambda_c, H);
 }
 
 cudaError_t state_init(float *s, float *coef, int B, int D, int M, const float *decay,

@@ -80,6 +80,14 @@ cudaError_t mixer_decode_step(const void *x_t, const void *g_t, void *z_t, rlm_d
                               float *s, const float *coef, void *hist, const float *conv_w, const float *scale,
                               int K, cudaStream_t st);
 
+// The mixer step in one launch, one block per batch row: recurrence step, C y_t
+// (H = 0: no coupling, c_raw unused), gate and local path (with the history
+// shift).  Covers M even with M / 2 a power of two, D <= 512 and D * M <= 4096.
+bool mixer_decode_coupled_supported(int D, int M);
+cudaError_t mixer_decode_coupled(const void *x_t, const void *g_t, void *z_t, rlm_dtype dt, int B, int D, int M,
+                                 float *s, const float *coef, void *hist, const float *conv_w, const float *scale,
+                                 int K, const float *c_raw, float lambda_c, int H, cudaStream_t st);
+
 // ---- mixer epilogue for the unfused prefill paths (rlm_mixer.cu) ------------
 // z <- sigma(g) z + s * (w * u) in place (g nullable; K = 0: no local path), the
 // drives before token 0 from hist ([B][K-1][D], nullable = zeros).

@@ -360,10 +360,17 @@ def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
     assert_close(s.real, sr.real, TOL[dtype], "state re")
 
 
-@pytest.mark.parametrize("dtype,M,K,H,B", [("bf16", 16, 4, 8, 3), ("f32", 7, 3, 4, 3), ("bf16", 16, 0, 2, 3),
-                                       ("bf16", 2, 8, 16, 3), ("bf16", 16, 4, 8, 1)])
-def test_coupled_mixer_decode_continues_the_prefill(dtype, M, K, H, B):
-    D, L0, T = 64, 300, 30
+@pytest.mark.parametrize("dtype,M,K,H,B,D,launches", [
+    # one launch per step (M / 2 a power of two, D <= 512, D * M <= 4096): one block per batch row
+    ("bf16", 16, 4, 8, 3, 64, 1), ("bf16", 16, 0, 2, 3, 64, 1), ("bf16", 2, 8, 16, 3, 64, 1),
+    ("bf16", 16, 4, 8, 1, 64, 1), ("f32", 16, 3, 4, 3, 64, 1), ("bf16", 64, 4, 8, 2, 64, 1),
+    ("bf16", 8, 8, 16, 2, 512, 1),
+    # two launches: the recurrence step, then coupling, gate and local path
+    ("f32", 7, 3, 4, 3, 64, 2), ("bf16", 12, 2, 4, 2, 64, 2), ("bf16", 32, 4, 8, 2, 512, 2),
+    ("bf16", 64, 4, 8, 2, 128, 2),
+])
+def test_coupled_mixer_decode_continues_the_prefill(dtype, M, K, H, B, D, launches):
+    L0, T = 300, 30
     inp = make_inputs(B, L0 + T, D, M, dtype, seed=M + K + H)
     mx = make_mixer_inputs(inp, K, seed=M + K + H)
     c_raw, lam = _coupling(H, 3 * H)
@@ -377,12 +384,14 @@ def test_coupled_mixer_decode_continues_the_prefill(dtype, M, K, H, B):
     rlm.rlm_mixer_prefill(x[:, :L0].contiguous(), g[:, :L0].contiguous(), p, local, z0, state_out=st,
                           conv_out=cs if K else None, coupling=cp)
     zs = []
+    n0 = rlm.rlm_kernels_launched()
     for t in range(L0, L0 + T):
         zt = torch.empty_like(x[:, t])
         rlm.rlm_mixer_decode(x[:, t].contiguous(), g[:, t].contiguous(), st, local, cs if K else None, zt,
                              coupling=cp)
         zs.append(zt)
     torch.cuda.synchronize()
+    assert rlm.rlm_kernels_launched() - n0 == launches * T
     zr, sr, tr = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), mx.conv_w, mx.scale, coupling=(c_raw, lam))
     assert_close(to_np(z0), zr[:, :L0], TOL[dtype], "prefill z")
     assert_close(to_np(torch.stack(zs, 1)), zr[:, L0:], TOL[dtype], "decode z")
