@@ -361,6 +361,9 @@ struct TcArgs {
                          // (otherwise the slot holds the gate: z = sigma(g) y)
     int ntiles;
     int64_t t0;          // first token of tile 0 (<= 0): tiles end exactly at L-1
+    // Unsegmented launches: grid y covers batch rows in groups of bpc; a CTA runs
+    // its rows' tiles back to back as one stream (one prologue for all of them).
+    int B, bpc;
     // Sequence segments (grid z): segment s owns tiles [s * seg_tiles, ...).
     int nseg, seg_tiles;
     float2 *seg_state;   // [B][nseg][D][M]: each segment's end state from a zero start
@@ -368,9 +371,11 @@ struct TcArgs {
     unsigned long long epoch;      // distinct for every segmented launch of this process
 };
 
-// kSeg: the grid's z dimension splits the sequence into segments.  The
-// unsegmented instance keeps the tile count a kernel parameter (no register
-// holds it), which the per-tile loops' register allocation depends on.
+// kMode: kPlain, one CTA per (channel group, batch row); kSegmented (kSeg), the
+// grid's z dimension splits the sequence into segments; kPacked (kPack), a CTA
+// runs args.bpc batch rows of its channel group back to back.  The plain instance
+// keeps the tile count a kernel parameter (no register holds it), which the
+// per-tile loops' register allocation depends on.
 // kInj: the prefill starts from args.state_in instead of zero.  Token 0 sits at
 // position p of chunk n0 of tile 0 (tiles end at L - 1); lambda^-p s_in is added
 // to the state entering chunk n0, which gives lambda^(i+1-p) s_in at its positions
@@ -383,11 +388,14 @@ struct TcArgs {
 // of each z ring slot into the slot itself once the slot's previous store has
 // been read out; every epilogue thread reads its 8 bytes there and overwrites them
 // with z.
-template <bool kSeg, bool kInj, bool kMix>
+enum : int { kPlain = 0, kSegmented = 1, kPacked = 2 };
+
+template <int kMode, bool kInj, bool kMix>
 __global__ void __launch_bounds__(kThreads, 1)
     k_prefill_tc(const __grid_constant__ CUtensorMap tmap_x,
                  const __grid_constant__ CUtensorMap tmap_y, const __grid_constant__ CUtensorMap tmap_g,
                  const TcArgs args) {
+    constexpr bool kSeg = kMode == kSegmented, kPack = kMode == kPacked;
     static_assert(!(kSeg && kMix), "the mixer epilogue is not built for segmented launches");
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // Align with pointer arithmetic on the __shared__ array (not through an
@@ -396,17 +404,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     const uint32_t sbase = smem_u32(smem);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int g = blockIdx.x, b = blockIdx.y, seg = kSeg ? (int)blockIdx.z : 0;
+    const int g = blockIdx.x, seg = kSeg ? (int)blockIdx.z : 0;
+    const int b = kPack ? (int)blockIdx.y * args.bpc : (int)blockIdx.y;   // the CTA's (first) batch row
     const int d0 = g * kDG;
     const int D = args.D;
-    // Virtual tiles: nA state-only passes over the segment's tiles (every segment
-    // but the last publishes its end state for the later ones), then nB output
-    // passes over the same tiles.
+    // Virtual tiles.  Segmented: nA state-only passes over the segment's tiles
+    // (every segment but the last publishes its end state for the later ones),
+    // then nB output passes over the same tiles.  Packed: the tiles of the CTA's
+    // batch rows, row after row (v -> row b + v / ntiles, tile v % ntiles).
     const int ja = kSeg ? seg * args.seg_tiles : 0;
-    const int nB = kSeg ? min(args.ntiles, ja + args.seg_tiles) - ja : args.ntiles;
+    const int nB = kSeg ? min(args.ntiles, ja + args.seg_tiles) - ja
+                        : kPack ? min(args.bpc, args.B - b) * args.ntiles : args.ntiles;
     const int nA = kSeg && seg < args.nseg - 1 ? nB : 0;
-    const int nV = kSeg ? nA + nB : args.ntiles;
-    auto real_tile = [&](int v) { return ja + (v < nA ? v : v - nA); };
+    const int nV = kSeg ? nA + nB : kPack ? nB : args.ntiles;
+    auto real_tile = [&](int v) { return kPack ? v % args.ntiles : ja + (v < nA ? v : v - nA); };
+    auto row_of = [&](int v) { return kPack ? b + v / args.ntiles : b; };
     // Constant builders (warps 0-11 and 18-21) issue their parameter loads first,
     // so the DRAM latency overlaps the barrier set-up and TMEM allocation.
     const bool builder = warp < 12 || (warp >= 18 && warp < 22);
@@ -467,11 +479,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     int issued = 0;
     if (warp == 16 && lane == 0) {
         for (; issued < total_boxes && issued < kXSlots; ++issued) {
-            const int jt = real_tile(issued / kBoxes), q = issued % kBoxes;
+            const int jt = real_tile(issued / kBoxes), q = issued % kBoxes, bq = row_of(issued / kBoxes);
             const uint32_t slot = issued % kXSlots;
             bar_expect_tx(bar(kBarXFull + slot), kBox * 16);
             tma_load_3d(sbase + kOffX + slot * (kBox * 16), &tmap_x, d0,
-                        (int)(args.t0 + (int64_t)jt * kTile + q * kBox), b, bar(kBarXFull + slot));
+                        (int)(args.t0 + (int64_t)jt * kTile + q * kBox), bq, bar(kBarXFull + slot));
         }
     }
 
@@ -584,13 +596,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------- TMA producer
         if (lane == 0) {
             for (; issued < total_boxes; ++issued) {
-                const int jt = real_tile(issued / kBoxes), q = issued % kBoxes;
+                const int jt = real_tile(issued / kBoxes), q = issued % kBoxes, bq = row_of(issued / kBoxes);
                 const uint32_t slot = issued % kXSlots;
                 const uint32_t fill = issued / kXSlots;
                 if (!wait_bar(bar(kBarXEmpty + slot), (fill & 1) ^ 1, abort_flag)) break;
                 bar_expect_tx(bar(kBarXFull + slot), kBox * 16);
                 tma_load_3d(sbase + kOffX + slot * (kBox * 16), &tmap_x, d0,
-                            (int)(args.t0 + (int64_t)jt * kTile + q * kBox), b,
+                            (int)(args.t0 + (int64_t)jt * kTile + q * kBox), bq,
                             bar(kBarXFull + slot));
             }
             // Drain: every issued load must land before this CTA may exit.
@@ -652,10 +664,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t slot = k % kYSlots;
             if (lane != 0) return;
             bar_expect_tx(bar(kBarGFull + slot), kYRows * 16);
-            const int jt = ja + k / kYPerTile, e = k % kYPerTile;
+            const int vq = k / kYPerTile, e = k % kYPerTile;
+            const int jt = kPack ? vq % args.ntiles : ja + vq, bq = row_of(vq);
             for (int h = 0; h < kYRows / kBox; ++h)
                 tma_load_3d(sbase + kOffY + slot * (kYRows * 16) + h * (kBox * 16), &tmap_g, d0,
-                            (int)(args.t0 + (int64_t)jt * kTile + e * kYRows + h * kBox), b, bar(kBarGFull + slot));
+                            (int)(args.t0 + (int64_t)jt * kTile + e * kYRows + h * kBox), bq, bar(kBarGFull + slot));
         };
         // The prologue keeps its W table in the z ring until the constants are built.
         if (kMix && wait_bar(bar(kBarConsts), 0, abort_flag))
@@ -665,17 +678,18 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t slot = ng % kYSlots;
             if (!wait_bar(bar(kBarYFull + slot), (ng / kYSlots) & 1, abort_flag)) break;
             const uint32_t ys = sbase + kOffY + slot * (kYRows * 16);
-            const int jt = ja + ng / kYPerTile, e = ng % kYPerTile;
+            const int vq = ng / kYPerTile, e = ng % kYPerTile;
+            const int jt = kPack ? vq % args.ntiles : ja + vq, bq = row_of(vq);
             for (int h = 0; h < kYRows / kBox; ++h) {
                 const int64_t start = args.t0 + (int64_t)jt * kTile + e * kYRows + h * kBox;
                 if (start >= 0) {
-                    if (lane == 0) tma_store_3d(&tmap_y, ys + h * (kBox * 16), d0, (int)start, b);
+                    if (lane == 0) tma_store_3d(&tmap_y, ys + h * (kBox * 16), d0, (int)start, bq);
                 } else if (start + kBox > 0) {
                     // Partially before t = 0: plain 16-byte stores of the rows t >= 0.
                     const uint8_t *src = smem + kOffY + slot * (kYRows * 16) + h * (kBox * 16);
                     for (int rr = (int)(-start) + lane; rr < kBox; rr += 32) {
                         const int64_t t = start + rr;
-                        *reinterpret_cast<uint4 *>(args.y + ((int64_t)b * args.L + t) * D + d0) =
+                        *reinterpret_cast<uint4 *>(args.y + ((int64_t)bq * args.L + t) * D + d0) =
                             *reinterpret_cast<const uint4 *>(src + rr * 16);
                     }
                 }
@@ -771,14 +785,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (kInj) {
             n0 = (int)((-args.t0) >> 6);
             const int p = (int)((-args.t0) & 63);
-            if (mreal)
+            if (!kPack && mreal)
                 inj = cmul(lambda_pow(m_decay, m_freq, (float)(-p)), args.state_in[((int64_t)b * D + d0 + ch) * args.Mt + args.m0 + m]);
         }
         uint8_t *bs = smem + kOffBs + ch * kBsStride + (m / 4) * kBsLbo + (m % 4) * 4;
         const int64_t seg_row = (int64_t)b * args.nseg;
         // One tile of the carry: S_n = lambda^C S_{n-1} + L_n over its 32 chunks.
         auto scan_tile = [&](int v) -> bool {
-            const bool inj_tile = kInj && real_tile(v) == 0;
+            const bool row_start = real_tile(v) == 0;
+            const bool inj_tile = kInj && row_start;
+            if (kPack && row_start) {
+                S = make_float2(0.0f, 0.0f);   // a new batch row starts from zero (or its own s_in)
+                if (kInj && mreal)
+                    inj = cmul(lambda_pow(m_decay, m_freq, (float)(-(int)((-args.t0) & 63))),
+                               args.state_in[((int64_t)row_of(v) * D + d0 + ch) * args.Mt + args.m0 + m]);
+            }
             if (!wait_bar(bar(kBarTwDone + cA), v & 1, abort_flag)) return false;
             if (!wait_bar(bar(kBarTwDone + cB), v & 1, abort_flag)) return false;
             tc_fence_after();
@@ -799,8 +820,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     S = cfma(LC, S, Ln);
                 }
             }
-            if (v == nV - 1 && (!kSeg || seg == args.nseg - 1) && args.state_out && mreal)
-                args.state_out[((int64_t)b * D + d0 + ch) * args.Mt + args.m0 + m] = S;
+            if ((kPack ? real_tile(v) == args.ntiles - 1 : v == nV - 1 && (!kSeg || seg == args.nseg - 1)) &&
+                args.state_out && mreal)
+                args.state_out[((int64_t)row_of(v) * D + d0 + ch) * args.Mt + args.m0 + m] = S;
             fence_async_smem();
             tc_fence_before();
             __syncwarp();
@@ -1040,6 +1062,46 @@ size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int) {
     return 2 * seg_state_bytes(B, sg.nseg, D);  // states, then their epoch flags
 }
 
+template <int kMode>
+void launch_unsegmented(bool field, bool inj, dim3 grid, const CUtensorMap &mx, const CUtensorMap &my,
+                        const CUtensorMap &m2, const TcArgs &a, cudaStream_t st) {
+    if (field) {
+        if (inj)
+            k_prefill_tc<kMode, true, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+        else
+            k_prefill_tc<kMode, false, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+    } else if (inj) {
+        k_prefill_tc<kMode, true, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+    } else {
+        k_prefill_tc<kMode, false, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+    }
+}
+
+// Batch rows per CTA of an unsegmented launch.  One CTA per SM (shared memory
+// and TMEM), so a grid of more CTAs than SMs runs in waves, each paying the
+// CTAs' prologue and pipeline fill again.  That cost is exposed only when a CTA
+// has few tiles (with more, the producer fills the ring while the constants are
+// built): measured at D = 256, about 6 tiles' worth for a one-tile CTA.  A CTA
+// that runs several rows saves it, at a few per cent per tile (measured 5 % at
+// D = 512, M = 32).  The count minimising waves * (max(0, 6 - tiles) + rows *
+// tiles * cost) is taken.
+int rows_per_cta(int64_t B, int D, int ntiles) {
+    const int64_t groups = D / kDG, sms = sm_count();
+    const double fill = std::max(0, 6 - ntiles);
+    int best = 1;
+    double best_t = 0.0;
+    for (int64_t r = 1; r <= B; ++r) {
+        const int64_t ctas = groups * ((B + r - 1) / r);
+        const double t = (double)((ctas + sms - 1) / sms) * (fill + (double)r * ntiles * (r > 1 ? 1.05 : 1.0));
+        if (r == 1 || t < best_t - 1e-9) {
+            best = (int)r;
+            best_t = t;
+        }
+        if (ctas <= sms) break;        // one wave: more rows per CTA only lengthen it
+    }
+    return best;
+}
+
 cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int M,
                        const float *decay, const float *freq, const float *amp,
                        const float *phase, const float *state_in, float *state_out, float *coef_out,
@@ -1057,12 +1119,16 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
         std::lock_guard<std::mutex> lock(mu);
         if ((int)configured.size() <= dev) configured.resize(dev + 1, 0);
         if (!configured[dev]) {
-            const void *fns[] = {reinterpret_cast<const void *>(k_prefill_tc<false, false, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<true, false, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<false, true, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<true, true, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<false, false, true>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<false, true, true>)};
+            const void *fns[] = {reinterpret_cast<const void *>(k_prefill_tc<kPlain, false, false>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kSegmented, false, false>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, true, false>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kSegmented, true, false>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, false, true>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, true, true>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, false, false>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, true, false>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, false, true>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, true, true>)};
             cudaError_t e = cudaSuccess;
             for (const void *f : fns)
                 if (e == cudaSuccess)
@@ -1094,7 +1160,9 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.seg_state = nullptr;
     a.seg_flag = nullptr;
     a.epoch = 0;
-    dim3 grid((unsigned)(D / kDG), (unsigned)B, (unsigned)sg.nseg);
+    a.B = (int)B;
+    a.bpc = sg.nseg < 2 ? rows_per_cta(B, D, a.ntiles) : 1;
+    dim3 grid((unsigned)(D / kDG), (unsigned)((B + a.bpc - 1) / a.bpc), (unsigned)sg.nseg);
     const int npass = (M + kModes - 1) / kModes;
     if ((mix || npass > 1) && sg.nseg >= 2) return cudaErrorInvalidValue;  // callers check support
     if (mix && npass > 1) return cudaErrorInvalidValue;
@@ -1105,15 +1173,10 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
             a.add = p > 0;
             // Later passes load the output so far into the z ring and add to it.
             const CUtensorMap &m2 = p > 0 ? my : mg;
-            if (mix || p > 0) {
-                if (state_in)
-                    k_prefill_tc<false, true, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
-                else
-                    k_prefill_tc<false, false, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
-            } else if (state_in) {
-                k_prefill_tc<false, true, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+            if (a.bpc > 1) {
+                launch_unsegmented<kPacked>(mix || p > 0, state_in != nullptr, grid, mx, my, m2, a, st);
             } else {
-                k_prefill_tc<false, false, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+                launch_unsegmented<kPlain>(mix || p > 0, state_in != nullptr, grid, mx, my, m2, a, st);
             }
             count_launches(1);
             const cudaError_t e = cudaGetLastError();
@@ -1131,8 +1194,8 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     static std::atomic<unsigned long long> epoch{0x5eed0000ull};
     a.epoch = ++epoch;
     void *kargs[] = {&mx, &my, &mg, &a};
-    const void *fn = state_in ? reinterpret_cast<const void *>(k_prefill_tc<true, true, false>)
-                              : reinterpret_cast<const void *>(k_prefill_tc<true, false, false>);
+    const void *fn = state_in ? reinterpret_cast<const void *>(k_prefill_tc<kSegmented, true, false>)
+                              : reinterpret_cast<const void *>(k_prefill_tc<kSegmented, false, false>);
     cudaError_t e = cudaLaunchCooperativeKernel(fn, grid, dim3(kThreads), kargs, (size_t)kSmemBytes, st);
     count_launches(1);
     return e;

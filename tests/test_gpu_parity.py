@@ -71,6 +71,45 @@ def test_prefill_layer6m_bf16():
     assert_close(to_np(y)[:, :, chans], ref1, TOL["bf16"], "y vs direct convolution")
 
 
+@pytest.mark.parametrize("B,L,D,M,with_state_in,bitwise", [
+    (8, 2048, 256, 16, False, True),          # the 6M layer: two rows per CTA, one wave
+    (9, 700, 256, 7, True, True),             # three rows per CTA, padded modes, an initial state
+    (3, 2048 * 2 + 77, 2048, 16, True, True), # more channel groups than SMs: three rows per CTA, ragged
+    (5, 2048 + 3, 512, 32, False, False),     # two mode passes, rows in CTAs of three (a partial last one)
+])
+def test_packed_rows_prefill(B, L, D, M, with_state_in, bitwise):
+    """Where the (batch row, channel group) CTAs would take more than one wave, a
+    CTA runs several rows' tiles back to back (one prologue).  Against the oracle,
+    and bit for bit against prefilling each row alone where that call is
+    unsegmented too (y and the terminal state)."""
+    inp = make_inputs(B, L, D, M, "bf16", seed=B * 100 + L)
+    rng = np.random.default_rng(L)
+    s_in = (rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M))) if with_state_in else None
+    x = to_dev(inp.x, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    y, st = torch.empty_like(x), rlm.State.empty(B, D, M)
+    si = None
+    if with_state_in:
+        si = rlm.State.empty(B, D, M)
+        si.s.copy_(torch.from_numpy(np.stack([s_in.real, s_in.imag], -1).astype(np.float32)))
+    rlm.rlm_mix_prefill_from(x, p, si, y, st)
+    torch.cuda.synchronize()
+    ref, st_ref = oracle.rec_prefill(inp.x, *inp.params(), state_in=s_in)
+    assert_close(to_np(y), ref, TOL["bf16"], "y")
+    _state_err(st, st_ref, TOL["bf16"])
+    if bitwise:
+        for b in range(B):
+            yb, stb = torch.empty_like(x[b:b + 1]), rlm.State.empty(1, D, M)
+            sib = None
+            if with_state_in:
+                sib = rlm.State.empty(1, D, M)
+                sib.s.copy_(si.s[b:b + 1])
+            rlm.rlm_mix_prefill_from(x[b:b + 1].contiguous(), p, sib, yb, stb)
+            torch.cuda.synchronize()
+            assert torch.equal(yb[0], y[b]), b
+            assert torch.equal(stb.s[0], st.s[b]), b
+
+
 @pytest.mark.parametrize("B,L,D,M,dtype", [
     (1, 1, 8, 1, "f32"), (1, 1, 8, 16, "bf16"), (2, 7, 16, 3, "f32"), (3, 65, 24, 16, "bf16"),
     (1, 1000, 8, 64, "f32"), (2, 2049, 64, 16, "bf16"), (1, 4097, 32, 5, "bf16"),
