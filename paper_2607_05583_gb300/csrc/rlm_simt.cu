@@ -31,6 +31,8 @@ namespace {
 constexpr int kMgFwd = 16;  // modes per thread, forward phases
 constexpr int kMgBwd = 8;   // modes per thread, backward output phase
 constexpr int kBlock = 128;
+constexpr int kTokBlock = 8;   // drives loaded ahead per thread in the per-token loops
+constexpr int kCarryBlock = 64; // threads per block of the carry (one per (b, d, m): spread over all SMs)
 
 int threads_per_channel(int M, int mg) {
     int t = (M + mg - 1) / mg;
@@ -94,14 +96,23 @@ __global__ void __launch_bounds__(kBlock) k_chunk_local(
     }
     const int64_t tau0 = t0 + (int64_t)k * C;
     const int i0 = tau0 < 0 ? (int)(-tau0) : 0;
-    for (int i = i0; i < C; ++i) {
-        const int64_t tau = tau0 + i;
-        const int64_t t = REV ? (L - 1 - tau) : tau;
-        const float xv = ld_elem(x + ((int64_t)b * L + t) * D + d);
+    // kTokBlock tokens' drives are loaded before their updates run.
+    for (int i = i0; i < C; i += kTokBlock) {
+        float xs[kTokBlock];
 #pragma unroll
-        for (int j = 0; j < MG; ++j) {
-            if (JORDAN) r[j] = cmul(lam[j], make_float2(r[j].x + s[j].x, r[j].y + s[j].y));
-            s[j] = cfma(lam[j], s[j], make_float2(xv, 0.0f));
+        for (int u = 0; u < kTokBlock; ++u) {
+            const int64_t tau = tau0 + i + u;
+            const int64_t t = REV ? (L - 1 - tau) : tau;
+            xs[u] = i + u < C ? ld_elem(x + ((int64_t)b * L + t) * D + d) : 0.0f;
+        }
+#pragma unroll
+        for (int u = 0; u < kTokBlock; ++u) {
+            if (i + u >= C) break;
+#pragma unroll
+            for (int j = 0; j < MG; ++j) {
+                if (JORDAN) r[j] = cmul(lam[j], make_float2(r[j].x + s[j].x, r[j].y + s[j].y));
+                s[j] = cfma(lam[j], s[j], make_float2(xs[u], 0.0f));
+            }
         }
     }
     const int64_t base = (((int64_t)b * nch + k) * D + d) * M;
@@ -120,7 +131,7 @@ __global__ void __launch_bounds__(kBlock) k_chunk_local(
 // (the output phase restarts its recurrence there, at time 0), and that state
 // reaches the end of chunk 0 after C + t0 tokens.
 template <bool JORDAN>
-__global__ void __launch_bounds__(256) k_chunk_carry(
+__global__ void __launch_bounds__(kCarryBlock) k_chunk_carry(
     int64_t B, int D, int M, int C, int nch, int64_t t0, const float *__restrict__ decay,
     const float *__restrict__ freq, const float *__restrict__ amp, const float *__restrict__ phase,
     float2 *__restrict__ ws_s, float2 *__restrict__ ws_r, const float2 *__restrict__ state_in,
@@ -135,16 +146,32 @@ __global__ void __launch_bounds__(256) k_chunk_carry(
     const float Cf = (float)C;
     float2 S = state_in ? state_in[idx] : make_float2(0, 0), R = make_float2(0, 0);
     const float2 L0 = state_in ? lambda_pow(decay[pm], freq[pm], (float)(C + t0)) : LC;
-    for (int k = 0; k < nch; ++k) {
-        const int64_t off = ((b * nch + k) * D + d) * M + m;
-        const float2 ls = ws_s[off];
-        ws_s[off] = S;
-        if (JORDAN) {
-            const float2 lr = ws_r[off];
-            ws_r[off] = R;
-            R = cfma(LC, make_float2(fmaf(Cf, S.x, R.x), fmaf(Cf, S.y, R.y)), lr);
+    // The chunks' partials are read kCarryBatch at a time before the recurrence
+    // runs over them (each slot is then overwritten with the state entering its
+    // chunk), so a thread waits on memory once per batch, not once per chunk.
+    constexpr int kCB = JORDAN ? 16 : 32;
+    const int64_t stride = (int64_t)D * M;
+    const int64_t off0 = (b * nch * D + d) * M + m;   // chunk 0; chunk k at off0 + k * stride
+    for (int k0 = 0; k0 < nch; k0 += kCB) {
+        float2 lsv[kCB], lrv[JORDAN ? kCB : 1];
+#pragma unroll
+        for (int j = 0; j < kCB; ++j) {
+            if (k0 + j < nch) {
+                lsv[j] = ws_s[off0 + (k0 + j) * stride];
+                if (JORDAN) lrv[j] = ws_r[off0 + (k0 + j) * stride];
+            }
         }
-        S = cfma(k == 0 ? L0 : LC, S, ls);
+#pragma unroll
+        for (int j = 0; j < kCB; ++j) {
+            if (k0 + j >= nch) break;
+            const int64_t off = off0 + (k0 + j) * stride;
+            ws_s[off] = S;
+            if (JORDAN) {
+                ws_r[off] = R;
+                R = cfma(LC, make_float2(fmaf(Cf, S.x, R.x), fmaf(Cf, S.y, R.y)), lrv[j]);
+            }
+            S = cfma(k0 + j == 0 ? L0 : LC, S, lsv[j]);
+        }
     }
     if (state_out) state_out[idx] = S;
     if (coef_out && b == 0) {
@@ -178,19 +205,28 @@ __global__ void __launch_bounds__(kBlock) k_chunk_output(
     }
     const int64_t tau0 = t0 + (int64_t)k * C;
     const int i0 = tau0 < 0 ? (int)(-tau0) : 0;
-    for (int i = i0; i < C; ++i) {
+    auto at = [&](int i) {
         const int64_t tau = tau0 + i;
-        const int64_t t = REV ? (L - 1 - tau) : tau;
-        const int64_t e = ((int64_t)b * L + t) * D + d;
-        const float xv = active ? ld_elem(x + e) : 0.0f;
-        float acc = 0.0f;
+        return ((int64_t)b * L + (REV ? (L - 1 - tau) : tau)) * D + d;
+    };
+    // kTokBlock tokens' drives are loaded before their updates run (the trip
+    // counts are uniform across the warp, so every lane reaches the shuffles).
+    for (int i = i0; i < C; i += kTokBlock) {
+        float xs[kTokBlock];
 #pragma unroll
-        for (int j = 0; j < MG; ++j) {
-            s[j] = cfma(lam[j], s[j], make_float2(xv, 0.0f));
-            acc = fmaf(c[j].x, s[j].x, fmaf(-c[j].y, s[j].y, acc));
+        for (int u = 0; u < kTokBlock; ++u) xs[u] = active && i + u < C ? ld_elem(x + at(i + u)) : 0.0f;
+#pragma unroll
+        for (int u = 0; u < kTokBlock; ++u) {
+            if (i + u >= C) break;
+            float acc = 0.0f;
+#pragma unroll
+            for (int j = 0; j < MG; ++j) {
+                s[j] = cfma(lam[j], s[j], make_float2(xs[u], 0.0f));
+                acc = fmaf(c[j].x, s[j].x, fmaf(-c[j].y, s[j].y, acc));
+            }
+            for (int o = tpc >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+            if (active && grp == 0) st_elem(y + at(i + u), acc);
         }
-        for (int o = tpc >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-        if (active && grp == 0) st_elem(y + e, acc);
     }
 }
 
@@ -362,7 +398,7 @@ cudaError_t prefill_t(const T *x, T *y, int64_t B, int64_t L, int D, int M, cons
     k_chunk_local<T, kMgFwd, false, false><<<grid, kBlock, 0, st>>>(
         x, L, D, M, tpc, g.C, g.nch, g.t0, decay, freq, ws_s, nullptr);
     const int64_t n = B * D * M;
-    k_chunk_carry<false><<<(unsigned)((n + 255) / 256), 256, 0, st>>>(
+    k_chunk_carry<false><<<(unsigned)((n + kCarryBlock - 1) / kCarryBlock), kCarryBlock, 0, st>>>(
         B, D, M, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, nullptr,
         reinterpret_cast<const float2 *>(state_in), reinterpret_cast<float2 *>(state_out),
         reinterpret_cast<float4 *>(coef_out));
@@ -392,7 +428,7 @@ cudaError_t backward_t(const T *dy, const T *x, T *dx, int64_t B, int64_t L, int
     k_chunk_local<T, kMgFwd, true, true><<<grid1, kBlock, 0, st>>>(
         dy, L, D, M, tpc1, g.C, g.nch, g.t0, decay, freq, ws_s, ws_r);
     const int64_t nbdm = B * D * M;
-    k_chunk_carry<true><<<(unsigned)((nbdm + 255) / 256), 256, 0, st>>>(
+    k_chunk_carry<true><<<(unsigned)((nbdm + kCarryBlock - 1) / kCarryBlock), kCarryBlock, 0, st>>>(
         B, D, M, g.C, g.nch, g.t0, decay, freq, amp, phase, ws_s, ws_r, nullptr, nullptr, nullptr);
     const int tpc3 = threads_per_channel(M, kMgBwd);
     dim3 grid3((unsigned)((D * tpc3 + kBlock - 1) / kBlock), (unsigned)g.nch, (unsigned)B);
