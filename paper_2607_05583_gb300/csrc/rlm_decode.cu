@@ -264,7 +264,7 @@ __global__ void __launch_bounds__(kCoupledBlock, 1) k_decode_coupled(
     const bool ch = d2 < D;
     T xraw = T(0.0f), hv[kHistMax];
     float gv = 0.0f, sc = 0.0f, w0 = 0.0f, wj[kHistMax];   // wj[j]: the weight of history entry j
-    T *hc = mix.hist + b * (K > 1 ? K - 1 : 0) * (int64_t)D + d2;
+    T *hc = K > 1 ? mix.hist + b * (K - 1) * (int64_t)D + d2 : nullptr;   // used only when K > 1
     if (ch) {
         xraw = xb[d2];
         if (mix.g) gv = ld_elem(mix.g + b * D + d2);
