@@ -379,6 +379,7 @@ def run_ours(args):
         decode["other_batch_sizes"] = {f"B{b}": {k: v for k, v in _bench_decode(rlm, torch, dev, hbm_peak, B=b).items()
                                                  if k in ("tok_s", "us_per_step", "frac_hbm")}
                                        for b in (1, 8)}
+        decode["large_batch"] = _bench_decode_large_batch(rlm, torch, dev, hbm_peak)
     # ---------------- backward
     backward = None if args.quick else _bench_backward(rlm, torch, dev, hbm_peak, args)
     # ---------------- mixer wrapper (gate + local path, fused)
@@ -509,6 +510,56 @@ def _bench_decode(rlm, torch, dev, hbm_peak, B=None):
             "tok_s": round(B * T / (ms * 1e-3), 1), "us_per_step": round(us_step, 4),
             "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4),
             "bytes_per_step": per_step, "launches": T}
+
+
+def _bench_decode_large_batch(rlm, torch, dev, hbm_peak, B=8192, T=64):
+    """The decode kernel where moving the state, not latency, sets the step time:
+    B = 8192 (a 256 MiB fp32 state, above the L2 size, read and written every
+    step).  The state is seeded with N(0, 1) values (rlm_state_init, then a fill)
+    instead of a 32768-token prefill, which at this batch would need 137 GB of
+    drive."""
+    from synth import make_inputs
+    P = DECODE
+    D, M = P["D"], P["M"]
+    inp = make_inputs(1, 1, D, M, "bf16", seed=0)
+    p = rlm.Params.from_arrays(*inp.params(), device=dev)
+    st = rlm.State.empty(B, D, M, device=dev)
+    rlm.rlm_state_init(st, p)
+    gen = torch.Generator(device="cpu").manual_seed(3)
+    s0 = torch.randn(B, D, M, 2, generator=gen).to(dev)
+    toks = torch.randn(T, B, D, generator=gen).to(dev, torch.bfloat16)
+    outs = torch.empty_like(toks)
+    st.s.copy_(s0)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        for t in range(8):
+            rlm.rlm_mix_decode(toks[t], st, outs[t])
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for t in range(T):
+            rlm.rlm_mix_decode(toks[t], st, outs[t])
+    stream = torch.cuda.current_stream()
+    res = []
+    for rep in range(4):
+        st.s.copy_(s0)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        g.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        if rep:
+            res.append(a.elapsed_time(b))
+    us_step = statistics.median(res) * 1e3 / T
+    per_step = decode_bytes(B, D, M)
+    gbs = per_step / (us_step * 1e-6) / 1e9
+    return {"workload": f"decode B={B} D={D} M={M}, {T} steps from a seeded state, CUDA graph (beyond the "
+                        f"configured batch sizes: the bandwidth-bound regime of the same kernel)",
+            "us_per_step": round(us_step, 4), "tok_s": round(B / (us_step * 1e-6), 1),
+            "achieved_GBps": round(gbs, 1), "frac_hbm": round(gbs / hbm_peak, 4), "bytes_per_step": per_step}
 
 
 def _bench_mixer(rlm, torch, dev, hbm_peak, flush, mix_ms, with_decode=True):
