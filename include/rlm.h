@@ -272,17 +272,21 @@ typedef struct {
  *   state_out nullable; terminal state and coefficients (may alias state_in)
  *   conv_out  nullable; the history after token L-1 (may alias conv_in exactly)
  * Workspace: rlm_prefill_workspace_size.  With a gate only (no local path, no
- * coupling), bf16 with M = 16 applies the gate inside the tcgen05 prefill's
- * epilogue (one pass: x and g in, z out); otherwise the mixing is written into z,
- * coupled in place (one pass over whole token rows) if asked, and finished by one
- * full-width pass over x, g and z. */
+ * coupling), bf16 with M <= 16 on unsegmented shapes applies the gate inside the
+ * tcgen05 prefill's epilogue (one pass: x and g in, z out).  Otherwise the mixing
+ * is written into z and one persistent pass over whole-row tiles applies the
+ * coupling, the gate and the local path (rows of at most 2 KB; H in {1, 2, 4, 8,
+ * 16} with D / H a multiple of 4); other shapes take a coupling pass and a
+ * channel-pair pass. */
 RLM_API rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm_params *p,
                                      const rlm_local *local, const rlm_coupling *coupling, const rlm_state *state_in,
                                      const rlm_conv_state *conv_in, rlm_tensor *z, rlm_state *state_out,
                                      rlm_conv_state *conv_out, const rlm_launch *launch);
 
 /* One decode step of the mixer: the recurrence step of rlm_mix_decode, the
- * gate, and the local path over the cached history, fused in one kernel (with
+ * coupling, the gate, and the local path over the cached history.  One kernel,
+ * one block per batch row, where D <= 512, D * M <= 4096 and M / 2 is a power of
+ * two; otherwise the decode kernel with the gate and the local path fused (with
  * coupling: the recurrence step, then one kernel per batch row for the coupling,
  * the gate and the local path).
  *   x_t, g_t [B][1][D] (g_t nullable: no gate); state updated in place; conv
