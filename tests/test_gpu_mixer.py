@@ -215,6 +215,8 @@ def _launches(fn):
     (2, 2 * 2048 + 77, 512, 4, True, True),    # local path: mixing + pass + history tail
     (1, 3 * 2048, 1024, 8, True, True),
     (2, 2048 + 3, 512, 2, False, True),
+    (8, 2048, 256, 0, True, False),            # gate only, two batch rows per CTA (the 6M layer)
+    (9, 700, 256, 0, True, False),             # ... three rows per CTA, one tile each
 ])
 def test_tcgen05_shape_mixer_prefill_matches_oracle(B, L, D, K, with_g, with_hist):
     inp = make_inputs(B, L, D, 16, "bf16", seed=L + D + K)
@@ -292,6 +294,27 @@ def test_tcgen05_shape_mixer_prefill_is_causal_bit_exact(K):
         torch.cuda.synchronize()
         assert torch.equal(z1[:, :t0], z2[:, :t0]), t0
         assert not torch.equal(z1[:, t0:], z2[:, t0:])
+
+
+def test_packed_rows_gate_from_state_matches_oracle():
+    """The gate in the epilogue of a prefill whose CTAs run several batch rows
+    (B = 9, L = 700, D = 256: three rows per CTA), each row from its own initial
+    state."""
+    B, L, D, M = 9, 700, 256, 16
+    inp = make_inputs(B, L, D, M, "bf16", seed=77)
+    mx = make_mixer_inputs(inp, 0, seed=77)
+    rng = np.random.default_rng(77)
+    s_in = rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M))
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    so, z = rlm.State.empty(B, D, M), torch.empty_like(x)
+    assert _launches(lambda: rlm.rlm_mixer_prefill(x, g, p, None, z, state_in=_state_from(B, D, M, s_in),
+                                                   state_out=so)) == 1
+    zr, sr, _ = oracle.mixer_prefill(inp.x, mx.g, *inp.params(), mx.conv_w, mx.scale, state_in=s_in)
+    assert_close(to_np(z), zr, TOL["bf16"], "z")
+    s = so.complex().cpu().numpy()
+    assert_close(s.real, sr.real, TOL["bf16"], "state re")
+    assert_close(s.imag, sr.imag, TOL["bf16"], "state im")
 
 
 def test_fused_and_unfused_gate_agree():
