@@ -4,7 +4,7 @@ One nvcc invocation per translation unit (run in parallel), one link step.
 Target: sm_103a only (``-gencode arch=compute_103a,code=sm_103a``); the CUDA
 runtime is linked statically and the driver API is reached at run time through
 ``cudaGetDriverEntryPoint``, so the library loads on a machine without a GPU
-driver (for the symbol checks) and needs only the driver on the GPU machine.
+driver (for the symbol checks) and needs only the driver where it runs kernels.
 """
 from __future__ import annotations
 
