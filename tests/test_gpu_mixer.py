@@ -361,6 +361,7 @@ def _coupling(H, seed, lam=0.7):
     (2, 700, 64, 7, 3, 4, "f32", True),              # ... fp32, 4 heads
     (2, 600, 64, 16, 0, 4, "bf16", False),           # coupling alone, in the whole-row pass
     (1, 300, 1024, 16, 2, 8, "f32", True),           # 4 KB rows: separate coupling and mixer passes
+    (1, 300, 8192, 16, 4, 64, "bf16", True),         # the largest coupling: D = 8192, 64 heads of 128
 ])
 def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
     inp = make_inputs(B, L, D, M, dtype, seed=L + H)
@@ -391,6 +392,7 @@ def test_coupled_mixer_prefill_matches_oracle(B, L, D, M, K, H, dtype, with_g):
     # two launches: the recurrence step, then coupling, gate and local path
     ("f32", 7, 3, 4, 3, 64, 2), ("bf16", 12, 2, 4, 2, 64, 2), ("bf16", 32, 4, 8, 2, 512, 2),
     ("bf16", 64, 4, 8, 2, 128, 2),
+    ("bf16", 16, 4, 64, 2, 8192, 2),                 # the largest coupling (48 KB of C and y_t per block)
 ])
 def test_coupled_mixer_decode_continues_the_prefill(dtype, M, K, H, B, D, launches):
     L0, T = 300, 30
