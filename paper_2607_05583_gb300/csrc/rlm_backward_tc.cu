@@ -310,6 +310,7 @@ struct BwdArgs {
     // through c = conj(cconj[b * D + d][m]) per batch row); it writes c P as its P
     // partial and adds to d_state_in.
     const float2 *cconj;
+    int acc_dx;               // add this pass's dx to what dxT holds (the terminal-state pass)
     __nv_bfloat16 *dxT;       // [B*D][Lp]
     int64_t Lp;
     int D, M;
@@ -619,10 +620,25 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             // Channel-major dx: each store instruction writes 64 contiguous bytes.
             __nv_bfloat16 *out = args.dxT + (int64_t)row * args.Lp + (int64_t)(last - v) * kTile + 32 * q + lane;
+            if (args.acc_dx) {
+                // Added to the first pass's dx (16 loads issued before their adds).
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {
-                out[k * kC] = __float2bfloat16_rn(__uint_as_float(r0[k]));
-                out[(k + 16) * kC] = __float2bfloat16_rn(__uint_as_float(r1[k]));
+                for (int hf = 0; hf < 2; ++hf) {
+                    const uint32_t *rv = hf ? r1 : r0;
+                    __nv_bfloat16 *oh = out + 16 * hf * kC;
+                    __nv_bfloat16 prev[16];
+#pragma unroll
+                    for (int k = 0; k < 16; ++k) prev[k] = oh[k * kC];
+#pragma unroll
+                    for (int k = 0; k < 16; ++k)
+                        oh[k * kC] = __float2bfloat16_rn(__bfloat162float(prev[k]) + __uint_as_float(rv[k]));
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    out[k * kC] = __float2bfloat16_rn(__uint_as_float(r0[k]));
+                    out[(k + 16) * kC] = __float2bfloat16_rn(__uint_as_float(r1[k]));
+                }
             }
         }
         // Diagonal sums of Q (accumulated over the whole sequence; its last
@@ -851,11 +867,9 @@ __global__ void __launch_bounds__(128) k_to_channel_major(const __nv_bfloat16 *_
 // [B*D][Lp] -> [B][L][D] for tokens t < L, token t read from position t, or from
 // L - 1 - t when rev.  A tile covers 64 tokens x 64 channels; it loads the
 // 8-aligned window of 72 positions that holds its (reversed) positions.
-// acc: add to what dst holds (one more bf16 rounding) instead of overwriting it.
 __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__restrict__ srcT,
                                                       __nv_bfloat16 *__restrict__ dst, int64_t L, int D,
-                                                      int64_t Lp, int rev, int b0, int c_lo, int c_hi,
-                                                      int acc) {
+                                                      int64_t Lp, int rev, int b0, int c_lo, int c_hi) {
     __shared__ uint32_t tile[64][37];   // [channel][position pair]
     const int64_t t0 = (int64_t)blockIdx.x * 64;
     const int c0 = c_lo + blockIdx.y * 64;
@@ -889,18 +903,7 @@ __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__res
             const uint32_t hi = (i & 1) ? (bw >> 16) : (bw & 0xffffu);
             w[e] = lo | (hi << 16);
         }
-        uint4 *out = reinterpret_cast<uint4 *>(dst + ((int64_t)b * L + t) * D + c);
-        if (acc) {
-            const uint4 o = *out;
-            const uint32_t ov[4] = {o.x, o.y, o.z, o.w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const float lo = __uint_as_float(w[e] << 16) + __uint_as_float(ov[e] << 16);
-                const float hi = __uint_as_float(w[e] & 0xffff0000u) + __uint_as_float(ov[e] & 0xffff0000u);
-                asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(w[e]) : "f"(hi), "f"(lo));
-            }
-        }
-        *out = make_uint4(w[0], w[1], w[2], w[3]);
+        *reinterpret_cast<uint4 *>(dst + ((int64_t)b * L + t) * D + c) = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -993,6 +996,7 @@ BwdArgs base_args(const float *decay, const float *freq, const float *amp, const
     a.coef_out = nullptr;
     a.d_state_in = nullptr;
     a.cconj = nullptr;
+    a.acc_dx = 0;
     a.dxT = outT;
     a.Lp = Lp;
     a.D = D;
@@ -1019,7 +1023,7 @@ cudaError_t run_layout_and_scan(const CUtensorMap &mdy, const CUtensorMap &mx, B
     a.row0 = 0;
     k_backward_tc<kGrad><<<(unsigned)(B * D), kThreads, kSmemBytes, st>>>(mdy, mx, a);
     k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(outT, out, L, D, Lp, rev, 0,
-                                                                                     0, D, 0);
+                                                                                     0, D);
     count_launches(3);
     return cudaGetLastError();
 }
@@ -1057,29 +1061,36 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     a.part_p = pp;
     a.state_in = reinterpret_cast<const float2 *>(state_in);
     a.d_state_in = reinterpret_cast<float2 *>(d_state_in);
-    e = run_layout_and_scan<true>(mdy, mx, a, B, L, D, Lp, static_cast<const __nv_bfloat16 *>(x),
-                         static_cast<const __nv_bfloat16 *>(dy), xT, dyT, 2, 0, dxT,
-                         static_cast<__nv_bfloat16 *>(dx), st);
-    if (e != cudaSuccess) return e;
-    if (d_state_out) {
+    if (!d_state_out) {
+        e = run_layout_and_scan<true>(mdy, mx, a, B, L, D, Lp, static_cast<const __nv_bfloat16 *>(x),
+                                      static_cast<const __nv_bfloat16 *>(dy), xT, dyT, 2, 0, dxT,
+                                      static_cast<__nv_bfloat16 *>(dx), st);
+        if (e != cudaSuccess) return e;
+    } else {
         // A terminal-state gradient g adds Re(conj(g) lambda^(L-1-t)) to dx_t,
         // conj(g) J to the decay / frequency products and g conj(lambda^L) to the
         // gradient of s_in (Sec. 3.2-3.3).  These are exactly what the same
         // backward gives for a unit drive at token L-1 read through c = conj(g)
         // (per batch row): its dx, c P (P = J with the s_in term) and
-        // conj(c lambda S_0).  So a second pass runs on that drive, reusing the
-        // channel-major x, and its dx is added to the first.
+        // conj(c lambda S_0).  So a second pass of the kernel runs on that drive,
+        // reusing the channel-major x and adding its dx to the first pass's in
+        // the channel-major buffer; one transpose then writes the sum.
+        const unsigned cg = (unsigned)((D + 63) / 64);
+        k_to_channel_major<<<dim3((unsigned)(Lp / 64), cg, (unsigned)(B * 2)), 128, 0, st>>>(
+            static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp, 2, 0,
+            0, 0, D);
+        k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a);
         if ((e = cudaMemsetAsync(dyT, 0, (size_t)rows * Lp * 2, st)) != cudaSuccess) return e;
         k_unit_last<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(dyT, rows, Lp, L);
         BwdArgs a2 = a;
         a2.part_g = pg2;
         a2.part_p = pj;
         a2.cconj = reinterpret_cast<const float2 *>(d_state_out);
+        a2.acc_dx = 1;
         k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a2);
-        const unsigned cg = (unsigned)((D + 63) / 64);
         k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(
-            dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp, 0, 0, 0, D, 1);
-        count_launches(3);
+            dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp, 0, 0, 0, D);
+        count_launches(5);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     return grad_reduce(rows / D, D, M, amp, phase, pg, pp, d_state_out ? pj : nullptr, g_decay, g_freq, g_amp,
