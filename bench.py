@@ -279,7 +279,6 @@ def run_ours(args):
                 "peak_kind": peak_kind, "frac_of_8TBps": round(achieved / 8000.0, 4),
                 "algorithmic_bytes_per_launch": alg,
                 "kernel": "rlm_mix_prefill (whole call)", "median_ms": statistics.median(times)}
-    roofline["io_ceiling"] = _io_ceiling(rlm, torch, x, y, flush, stream, P, achieved)
 
     # ---------------- e2e through the C ABI with host buffers
     # Every step copies its input from pinned host memory, runs the prefill and
@@ -410,31 +409,6 @@ def run_ours(args):
     if ws > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
-
-
-def _io_ceiling(rlm, torch, x, y, flush, stream, P, achieved, reps=5):
-    """Load+store bandwidth of the prefill's access pattern with nothing else in the
-    way: its CTA count (one per 8-channel group and batch row), each streaming
-    16-byte slices of the [B*L][D] field (and, for comparison, 32-byte slices at
-    the same CTA count).  `frac` is the prefill's algorithmic GB/s over the
-    16-byte ceiling."""
-    rows, D = P["B"] * P["L"], P["D"]
-    ctas = P["B"] * (D // 8)
-    src, dst = x.view(rows, D), y.view(rows, D)
-    out = {"ctas": ctas}
-    for sb in (16, 32):
-        ts = []
-        for _ in range(reps):
-            flush.zero_()
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            nbytes = rlm.rlm_measure_row_io(src, dst, sb, ctas)
-            e1.record(stream)
-            torch.cuda.synchronize()
-            ts.append(e0.elapsed_time(e1))
-        out[f"slice{sb}_GBps"] = round(nbytes / (statistics.median(ts) * 1e-3) / 1e9, 1)
-    out["frac"] = round(achieved / out["slice16_GBps"], 4)
-    return out
 
 
 def _time_prefill(rlm, torch, dev, B, L, D, M, flush, hbm_peak, reps=5, dtype="bf16"):

@@ -136,11 +136,12 @@ RLM_API rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm
  *              not overlap y.  state_out may be the same buffer (in-place
  *              continuation); partial overlap is rejected.
  * Other arguments, the workspace (rlm_prefill_workspace_size) and the paths
- * taken are those of rlm_mix_prefill.  Range: on the time-reversed tcgen05 path
- * (bf16, 16 < M <= 32, few batch rows and channel groups) with L not a multiple of
- * 64, state_in enters as lambda^(L - L') s_in, L' = L rounded up to 64, whose
- * modulus exp(decay (L' - L)) exceeds fp32 for decays above 88 / 63 (a half-life
- * under half a token); keep decays below that there. */
+ * taken are those of rlm_mix_prefill, except that a call with state_in whose L is
+ * not a multiple of 64 runs on the SIMT chunked scan: the tensor-core forms work
+ * in 64-token chunks aligned to the end of the sequence and would enter the state
+ * through a negative power of lambda (up to lambda^-63), which overflows fp32 for
+ * decays above 88/63 per token.  Every finite decay >= 0 is covered; chunked
+ * prefills in pieces whose length is a multiple of 64 stay on the tensor cores. */
 RLM_API rlm_status rlm_mix_prefill_from(const rlm_tensor *x, const rlm_params *p, const rlm_state *state_in,
                                         rlm_tensor *y, rlm_state *state_out, const rlm_launch *launch);
 
@@ -161,7 +162,12 @@ RLM_API size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rl
  *    return RLM_ERR_UNSUPPORTED with the needed size in rlm_last_error().
  *  - The first call on a device looks up the array's device address (one
  *    cudaGetSymbolAddress with that device current); make that first call
- *    before any stream capture.
+ *    before any stream capture.  Under CUDA's default lazy module loading the
+ *    array's device memory is committed by that same first call, so a runtime
+ *    that reserves device memory up front should make it before reserving
+ *    (or load modules eagerly, CUDA_MODULE_LOADING=EAGER).
+ *  - stream must belong to the current device (RLM_ERR_INVALID_ARG otherwise);
+ *    state_out's buffers must not overlap x, y or each other.
  *  - All calls share the one array, and it keeps the previous call's contents;
  *    every scratch element is written before it is read, so nothing needs
  *    clearing.  Calls whose executions overlap on the GPU (different streams,
@@ -311,6 +317,16 @@ RLM_API rlm_status rlm_get_device_status(const rlm_launch *launch);
 /* Static description of a status code. */
 RLM_API const char *rlm_status_string(rlm_status status);
 
+/* Test hook for failure detection; the paper has no counterpart.  on != 0 makes
+ * the next prefills that split a sequence into segments (few batch rows, M <= 16,
+ * bf16) run with a wait bound of about 1 ms instead of about 2 s, and makes the
+ * first segment withhold the flag that publishes its end state: every later
+ * segment's wait then expires, the kernel records RLM_ERR_TIMEOUT in the device
+ * status word, drains what it issued, frees its tensor memory and returns (its
+ * output is undefined).  on = 0 restores normal operation.  Synchronous (two
+ * copies to device symbols on the current device); not for production use. */
+RLM_API rlm_status rlm_test_stall_segments(int on);
+
 /* Human-readable reason for the last non-OK status returned on this host
  * thread (valid until the next call on the thread). */
 RLM_API const char *rlm_last_error(void);
@@ -322,32 +338,6 @@ RLM_API int rlm_version(void);
  * host-side count, incremented at each launch; for accounting in benchmarks). */
 RLM_API unsigned long long rlm_kernels_launched(void);
 
-/* rlm_measure_row_io -- a measurement helper with no counterpart in the paper:
- * it bounds what the prefill's memory access pattern can reach on this GPU.
- *
- * The tensor-core prefill gives each CTA one group of 8 bf16 channels, so each
- * token row it loads from x or stores to y is a 16-byte slice of a [B][L][D] row.
- * This call launches `ctas` CTAs that stream that pattern and nothing else: CTA k
- * owns the slice of slice_bytes (16, 32, 64 or 128) bytes at channel
- * (k % (D / (slice_bytes / 2))) * (slice_bytes / 2) of a [rows][D] bf16 field and
- * a contiguous range of its rows; it loads 4 KB boxes from `src` with TMA and
- * stores as many 4 KB boxes to `dst` with TMA.  Together the CTAs load the field
- * once and store it once (rlm_measure_row_io_bytes gives the exact byte count),
- * so timing the call on `stream` gives the load+store bandwidth of that slice
- * width at that CTA count.
- *
- * src, dst: device, [rows][D] bf16, 16-byte aligned; dst is overwritten with
- *   arbitrary bytes (pass scratch memory).
- * rows: a multiple of 4096 / slice_bytes, below 2^31.  D: a multiple of
- *   slice_bytes / 2.  ctas: a positive multiple of D / (slice_bytes / 2).
- * Errors: invalid arguments return RLM_ERR_INVALID_ARG before any launch; a
- *   launch failure returns RLM_ERR_CUDA.  Waits inside the kernel are bounded
- *   (about 2 s); a wait that expires shows as a measured time of seconds. */
-RLM_API rlm_status rlm_measure_row_io(const void *src, void *dst, int64_t rows, int D, int slice_bytes,
-                                      int ctas, void *stream);
-/* Bytes rlm_measure_row_io moves (loaded plus stored) for these arguments; 0 if
- * they are invalid. */
-RLM_API int64_t rlm_measure_row_io_bytes(int64_t rows, int D, int slice_bytes, int ctas);
 
 #ifdef __cplusplus
 }

@@ -27,7 +27,7 @@ __all__ = [
     "rlm_mixer_decode",
     "rlm_prefill_workspace_size", "rlm_backward_workspace_size",
     "rlm_validate_params", "rlm_get_device_status", "rlm_status_string",
-    "rlm_version", "rlm_kernels_launched", "rlm_measure_row_io", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
+    "rlm_version", "rlm_kernels_launched", "RLM_OK", "RLM_ERR_INVALID_ARG", "RLM_ERR_UNSUPPORTED",
     "RLM_ERR_CUDA", "RLM_ERR_TIMEOUT", "RLM_F32", "RLM_BF16",
 ]
 
@@ -115,6 +115,7 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.rlm_state_init.argtypes = [P(_State), P(_Params), P(_Launch)]
     lib.rlm_validate_params.argtypes = [P(_Params)]
     lib.rlm_get_device_status.argtypes = [P(_Launch)]
+    lib.rlm_test_stall_segments.argtypes = [ctypes.c_int]
     for f in ("rlm_prefill_workspace_size", "rlm_backward_workspace_size"):
         getattr(lib, f).argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
                                     ctypes.c_int, ctypes.c_int]
@@ -131,11 +132,6 @@ def load_library(build_if_missing: bool = False) -> ctypes.CDLL:
     lib.rlm_mix_prefill_noalloc.argtypes = [P(_Tensor), P(_Params), P(_Tensor), P(_State),
                                             ctypes.c_void_p]
     lib.rlm_mix_prefill_noalloc.restype = ctypes.c_int
-    lib.rlm_measure_row_io.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_int,
-                                       ctypes.c_int, ctypes.c_int, ctypes.c_void_p]
-    lib.rlm_measure_row_io.restype = ctypes.c_int
-    lib.rlm_measure_row_io_bytes.argtypes = [ctypes.c_int64, ctypes.c_int, ctypes.c_int, ctypes.c_int]
-    lib.rlm_measure_row_io_bytes.restype = ctypes.c_int64
     _lib = lib
     return lib
 
@@ -336,23 +332,6 @@ def rlm_version() -> int:
 def rlm_kernels_launched() -> int:
     """Kernels the library has launched in this process (host-side count)."""
     return int(load_library().rlm_kernels_launched())
-
-
-def rlm_measure_row_io(src: torch.Tensor, dst: torch.Tensor, slice_bytes: int, ctas: int,
-                       stream=None) -> int:
-    """Stream TMA loads of `src` and stores to `dst` (both [rows][D] bf16 CUDA tensors)
-    in slices of `slice_bytes` bytes per CTA, with `ctas` CTAs; returns the bytes
-    moved (loaded plus stored).  Time the call on `stream` to get the bandwidth of
-    the prefill's access pattern."""
-    if src.dtype != torch.bfloat16 or dst.dtype != torch.bfloat16 or src.shape != dst.shape or src.dim() != 2:
-        raise ValueError("src and dst must be [rows][D] bf16 tensors of the same shape")
-    if not (src.is_contiguous() and dst.is_contiguous()):
-        raise ValueError("src and dst must be contiguous")
-    lib = load_library()
-    rows, D = src.shape
-    _check(lib.rlm_measure_row_io(src.data_ptr(), dst.data_ptr(), rows, D, slice_bytes, ctas,
-                                  _stream(stream)), "rlm_measure_row_io")
-    return int(lib.rlm_measure_row_io_bytes(rows, D, slice_bytes, ctas))
 
 
 def rlm_prefill_workspace_size(B: int, L: int, D: int, M: int, dtype) -> int:

@@ -158,6 +158,13 @@ rlm_status check_prefill_states(const rlm_tensor *x, const rlm_tensor *y, const 
     rlm_status s;
     if (state_out && (s = check_state(state_out, x->B, x->D, p->M, "state_out")) != RLM_OK) return s;
     const size_t sbytes = (size_t)x->B * x->D * p->M * 8;
+    if (state_out) {
+        const size_t cbytes = (size_t)x->D * p->M * 16;
+        if (overlap(state_out->s, sbytes, x->ptr, tensor_bytes(x)) || overlap(state_out->s, sbytes, y->ptr, tensor_bytes(y)) ||
+            overlap(state_out->coef, cbytes, x->ptr, tensor_bytes(x)) ||
+            overlap(state_out->coef, cbytes, y->ptr, tensor_bytes(y)) || overlap(state_out->s, sbytes, state_out->coef, cbytes))
+            return fail(RLM_ERR_INVALID_ARG, "state_out->s or state_out->coef overlaps the fields or each other");
+    }
     if (state_in) {
         if (!state_in->s || !aligned16(state_in->s))
             return fail(RLM_ERR_INVALID_ARG, "state_in->s is NULL or not 16-byte aligned");
@@ -172,12 +179,20 @@ rlm_status check_prefill_states(const rlm_tensor *x, const rlm_tensor *y, const 
     return RLM_OK;
 }
 
-// The prefill path for a problem: the tcgen05 prefill (bf16, M = 16), its
-// time-reversed form (other bf16 M <= 32), else the SIMT scan.
+// The prefill path for a problem: the tcgen05 prefill (bf16, M <= 64), its
+// time-reversed form (other bf16 M <= 32), else the SIMT scan.  Both tcgen05 forms
+// work in 64-token chunks aligned to one end of the sequence; when L is not a
+// multiple of 64, an initial state enters them through a negative power of
+// lambda (up to lambda^-63), which overflows fp32 for decays above 88/63 per
+// token.  Such calls run on the SIMT scan, whose powers of lambda are all
+// positive, so every finite decay >= 0 is covered.
 enum class PrefillPath { kTc, kRev, kSimt };
 
-PrefillPath prefill_path(const rlm_tensor *x, int M) {
+bool state_in_needs_simt(int64_t L, bool with_state_in) { return with_state_in && L % 64 != 0; }
+
+PrefillPath prefill_path(const rlm_tensor *x, int M, bool with_state_in) {
     const int D = (int)x->D;
+    if (state_in_needs_simt(x->L, with_state_in)) return PrefillPath::kSimt;
     if (tc_prefill_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kTc;
     if (tc_prefill_rev_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kRev;
     return PrefillPath::kSimt;
@@ -266,9 +281,12 @@ unsigned long long rlm_kernels_launched(void) { return g_launches.load(std::memo
 
 size_t rlm_prefill_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
     if (B < 1 || L < 1 || D < 1 || M < 1) return 0;
-    if (tc_prefill_supported(B, L, D, M, dtype)) return tc_prefill_ws_bytes(B, L, D, M);
-    if (tc_prefill_rev_supported(B, L, D, M, dtype)) return tc_prefill_rev_ws_bytes(B, L, D, M);
-    return simt_prefill_ws_bytes(B, L, D, M);
+    size_t tc = 0;
+    if (tc_prefill_supported(B, L, D, M, dtype)) tc = tc_prefill_ws_bytes(B, L, D, M);
+    else if (tc_prefill_rev_supported(B, L, D, M, dtype)) tc = tc_prefill_rev_ws_bytes(B, L, D, M);
+    else return simt_prefill_ws_bytes(B, L, D, M);
+    // A call with an initial state and a ragged length runs on the SIMT scan.
+    return state_in_needs_simt(L, true) ? std::max(tc, simt_prefill_ws_bytes(B, L, D, M)) : tc;
 }
 
 size_t rlm_backward_workspace_size(int64_t B, int64_t L, int D, int M, rlm_dtype dtype) {
@@ -292,7 +310,7 @@ rlm_status rlm_mix_prefill_from(const rlm_tensor *x, const rlm_params *p, const 
         return fail(RLM_ERR_INVALID_ARG, "x and y overlap");
     if ((s = check_params(p, x->D)) != RLM_OK) return s;
     if ((s = check_prefill_states(x, y, p, state_in, state_out)) != RLM_OK) return s;
-    const PrefillPath path = prefill_path(x, p->M);
+    const PrefillPath path = prefill_path(x, p->M, state_in != nullptr);
     if (path == PrefillPath::kSimt && simt_chunks(x->B, x->L, (int)x->D) > 65535)
         return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
     const size_t need = rlm_prefill_workspace_size(x->B, x->L, (int)x->D, p->M, x->dtype);
@@ -337,7 +355,7 @@ rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, const rlm
         if (hin && hin != hout && overlap(hin, cb, hout, cb))
             return fail(RLM_ERR_INVALID_ARG, "conv_in and conv_out overlap without being the same buffer");
     }
-    const PrefillPath path = prefill_path(x, p->M);
+    const PrefillPath path = prefill_path(x, p->M, state_in != nullptr);
     if (path == PrefillPath::kSimt && simt_chunks(x->B, x->L, (int)x->D) > 65535)
         return fail(RLM_ERR_UNSUPPORTED, "sequence too long for the chunk grid");
     const size_t need = rlm_prefill_workspace_size(x->B, x->L, (int)x->D, p->M, x->dtype);
@@ -569,6 +587,12 @@ rlm_status rlm_get_device_status(const rlm_launch *ln) {
     if (status == RLM_OK) status = bwd;
     if (status == RLM_OK) status = mix;
     if (status != RLM_OK) return fail((rlm_status)status, "a bounded device-side wait expired");
+    return RLM_OK;
+}
+
+rlm_status rlm_test_stall_segments(int on) {
+    const cudaError_t e = set_segment_stall(on ? 1 : 0);
+    if (e != cudaSuccess) return cuda_fail(e, "rlm_test_stall_segments");
     return RLM_OK;
 }
 

@@ -622,6 +622,8 @@ __global__ void __launch_bounds__(kThreads, 2)
             __nv_bfloat16 *out = args.dxT + (int64_t)row * args.Lp + (int64_t)(last - v) * kTile + 32 * q + lane;
             if (args.acc_dx) {
                 // Added to the first pass's dx (16 loads issued before their adds).
+                // That dx was already rounded to bf16, so the sum is rounded twice:
+                // one extra bf16 rounding of dx, well inside the bf16 tolerance.
 #pragma unroll
                 for (int hf = 0; hf < 2; ++hf) {
                     const uint32_t *rv = hf ? r1 : r0;

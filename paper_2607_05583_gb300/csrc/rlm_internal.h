@@ -138,5 +138,8 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
                        const TcMix *mix, void *ws, cudaStream_t st);
 // Device status word written by bounded waits (RLM_OK or RLM_ERR_TIMEOUT).
 cudaError_t read_and_clear_device_status(int *status, cudaStream_t st);
+// Test hook of the failure-detection test: on = 1 shortens the prefill's wait
+// bound to about 1 ms and makes sequence segment 0 withhold its end-state flag.
+cudaError_t set_segment_stall(int on);
 
 }  // namespace rlm

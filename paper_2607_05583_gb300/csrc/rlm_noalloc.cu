@@ -3,11 +3,13 @@
 // callers that cannot hand the library a workspace.
 //
 // The scratch is a file-scope __device__ array of kNoAllocScratchBytes.  Every
-// GPU that loads this library reserves it (at module load) and keeps it until
-// the process exits.  Host code must not pass the array's name to a kernel: on
-// the host that name is only a stand-in, not a device address.  The device
-// address is looked up with cudaGetSymbolAddress, once per device, with that
-// device current, the first time this entry point runs on it.
+// GPU on which the library's device code is loaded holds it until the process
+// exits; under CUDA's default lazy module loading that happens when the first
+// call of this entry point on the device looks the array up, so the memory is
+// committed by that first call.  Host code must not pass the array's name to a
+// kernel: on the host that name is only a stand-in, not a device address.  The
+// device address is looked up with cudaGetSymbolAddress, once per device, with
+// that device current, the first time this entry point runs on it.
 #include <cuda_runtime.h>
 
 #include <cstdarg>
@@ -97,6 +99,24 @@ extern "C" rlm_status rlm_mix_prefill_noalloc(const rlm_tensor *x, const rlm_par
             return reject(RLM_ERR_INVALID_ARG, "state_out buffers are NULL or not 16-byte aligned");
         if (state_out->B != x->B || state_out->D != x->D || state_out->M != p->M)
             return reject(RLM_ERR_INVALID_ARG, "state_out shape does not match x and params");
+        const char *sa = reinterpret_cast<const char *>(state_out->s);
+        const char *ca = reinterpret_cast<const char *>(state_out->coef);
+        const size_t sb = (size_t)x->B * x->D * p->M * 8, cb = (size_t)x->D * p->M * 16;
+        auto hits = [](const char *a, size_t na, const char *b, size_t nb) { return a < b + nb && b < a + na; };
+        if (hits(sa, sb, xa, nbytes) || hits(sa, sb, ya, nbytes) || hits(ca, cb, xa, nbytes) ||
+            hits(ca, cb, ya, nbytes) || hits(sa, sb, ca, cb))
+            return reject(RLM_ERR_INVALID_ARG, "state_out->s or state_out->coef overlaps x, y or each other");
+    }
+    if (stream) {
+        // The scratch address is the current device's, so the stream must be that device's.
+        int dev = 0, sdev = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess ||
+            cudaStreamGetDevice(static_cast<cudaStream_t>(stream), &sdev) != cudaSuccess)
+            return reject(RLM_ERR_INVALID_ARG, "rlm_mix_prefill_noalloc: the stream's device cannot be read");
+        if (sdev != dev)
+            return reject(RLM_ERR_INVALID_ARG,
+                          "rlm_mix_prefill_noalloc: the stream belongs to device %d, the current device is %d",
+                          sdev, dev);
     }
     const int D = (int)x->D, M = p->M;
     const int C = simt_chunk_len(x->B, x->L, D);

@@ -63,7 +63,7 @@
 //          thread for ~100 cycles, so eight issuing threads keep the pipe fed.
 // Warps 0-11 and 18-21 first build the per-channel constants.
 //
-// Every wait is bounded: after kWaitLimitCycles the waiting thread sets a shared
+// Every wait is bounded: after wait_limit() cycles the waiting thread sets a shared
 // abort flag and the device status word (RLM_ERR_TIMEOUT); all roles then leave
 // their loops, drain what they issued and the CTA frees its TMEM and returns.
 #include <cuda.h>
@@ -80,6 +80,17 @@ namespace rlm {
 
 // Device status word: RLM_OK, or RLM_ERR_TIMEOUT once a bounded wait expired.
 __device__ int g_device_status = 0;
+
+// Bound of every wait in the prefill kernel, in SM cycles: about 2 s at 2 GHz.
+// The failure-detection test (rlm_test_stall_segments) shortens it to about 1 ms
+// and makes the first sequence segment withhold its end-state flag, so that the
+// later segments' waits expire; off (these values) by default.
+constexpr long long kWaitLimitDefault = 4000000000ll;
+__device__ long long g_wait_limit_cycles = kWaitLimitDefault;
+__device__ int g_stall_segment0 = 0;
+__device__ __forceinline__ long long wait_limit() {
+    return *reinterpret_cast<volatile long long *>(&g_wait_limit_cycles);
+}
 
 namespace {
 
@@ -98,7 +109,6 @@ constexpr int kWarps = 26;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTmemCols = 512;
 constexpr int kTmemA = 256;            // first TMEM column of the A operands
-constexpr long long kWaitLimitCycles = 4000000000ll;  // about 2 s at 2 GHz
 constexpr int kTransposers = 4;
 
 // Shared memory map (bytes from a 1024-aligned base).
@@ -199,7 +209,7 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
             const long long now = clock64();
             if (t0 == 0) {
                 t0 = now;
-            } else if (now - t0 > kWaitLimitCycles) {
+            } else if (now - t0 > wait_limit()) {
                 *abort_flag = 1;
                 atomicExch(&g_device_status, (int)RLM_ERR_TIMEOUT);
                 return false;
@@ -222,7 +232,7 @@ __device__ __forceinline__ bool wait_flag(const unsigned long long *flag, unsign
             const long long now = clock64();
             if (t0 == 0) {
                 t0 = now;
-            } else if (now - t0 > kWaitLimitCycles) {
+            } else if (now - t0 > wait_limit()) {
                 *abort_flag = 1;
                 atomicExch(&g_device_status, (int)RLM_ERR_TIMEOUT);
                 return false;
@@ -611,7 +621,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t slot = k % kXSlots, fill = k / kXSlots;
                 const long long t0 = clock64();
                 while (!bar_try(bar(kBarXFull + slot), fill & 1))
-                    if (clock64() - t0 > kWaitLimitCycles) break;
+                    if (clock64() - t0 > wait_limit()) break;
             }
         }
         __syncwarp();
@@ -761,7 +771,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             umma_commit(bar(kBarFinal + c));
             const long long t0 = clock64();
             while (!bar_try(bar(kBarFinal + c), 0))
-                if (clock64() - t0 > kWaitLimitCycles) break;
+                if (clock64() - t0 > wait_limit()) break;
         }
         __syncwarp();
     } else if (warp >= 8 && warp < 12) {
@@ -836,7 +846,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // State-only passes, then (segments with later ones) publish the end state
         // from a zero start: every lane stores its state, then releases its flag.
         for (int v = 0; v < nA && ok; ++v) ok = scan_tile(v);
-        if (ok && nA > 0) {
+        if (ok && nA > 0 && !(seg == 0 && *reinterpret_cast<volatile int *>(&g_stall_segment0))) {
             const int64_t at = ((seg_row + seg) * D + d0 + ch) * kModes + m;
             args.seg_state[at] = S;
             asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(args.seg_flag + at), "l"(args.epoch)
@@ -1198,6 +1208,13 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
                               : reinterpret_cast<const void *>(k_prefill_tc<kSegmented, false, false>);
     cudaError_t e = cudaLaunchCooperativeKernel(fn, grid, dim3(kThreads), kargs, (size_t)kSmemBytes, st);
     count_launches(1);
+    return e;
+}
+
+cudaError_t set_segment_stall(int on) {
+    const long long limit = on ? 2000000ll : kWaitLimitDefault;   // about 1 ms, or about 2 s
+    cudaError_t e = cudaMemcpyToSymbol(g_wait_limit_cycles, &limit, sizeof(limit));
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_stall_segment0, &on, sizeof(on));
     return e;
 }
 

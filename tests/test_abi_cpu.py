@@ -147,6 +147,26 @@ def test_prefill_from_rejects_bad_initial_states_on_host(lib):
     assert call(state(sbase), so) == rlm.RLM_ERR_INVALID_ARG
 
 
+def test_prefills_reject_state_out_overlapping_fields_on_host(lib):
+    """state_out's complex buffer and its coefficient buffer may overlap neither x,
+    y nor each other (rlm_mix_prefill and rlm_mix_prefill_noalloc)."""
+    B, L, D, M = 2, 100, 64, 16
+    x = _t(FAKE, B, L, D)
+    y = _t(FAKE + (1 << 30), B, L, D)
+    p = _p(D, M)
+    ln = _launch(FAKE + (1 << 34), 1 << 40)
+    sbase = FAKE + (1 << 36)
+    cases = [(x.ptr + 4096, sbase), (y.ptr, sbase), (sbase, x.ptr + 256), (sbase, y.ptr + 512),
+             (sbase, sbase + 256)]
+    for s_ptr, c_ptr in cases:
+        so = rlm._State(s_ptr, c_ptr, B, D, M)
+        assert lib.rlm_mix_prefill(ctypes.byref(x), ctypes.byref(p), ctypes.byref(y), ctypes.byref(so),
+                                   ctypes.byref(ln)) == rlm.RLM_ERR_INVALID_ARG, (s_ptr, c_ptr)
+        assert lib.rlm_mix_prefill_noalloc(ctypes.byref(x), ctypes.byref(p), ctypes.byref(y), ctypes.byref(so),
+                                           None) == rlm.RLM_ERR_INVALID_ARG, (s_ptr, c_ptr)
+        assert "overlaps" in lib.rlm_last_error().decode()
+
+
 def test_decode_rejects_bad_arguments_on_host(lib):
     B, D, M = 4, 64, 16
     st = rlm._State(FAKE + (1 << 33), FAKE + (1 << 33) + (1 << 20), B, D, M)
@@ -257,29 +277,6 @@ def test_mixer_rejects_bad_arguments_on_host(lib):
     assert dec(local(), None) == rlm.RLM_ERR_INVALID_ARG                         # history required for K >= 2
     assert dec(local(), conv(b=B + 1)) == rlm.RLM_ERR_INVALID_ARG
     assert dec(local(), conv(ptr=st.s)) == rlm.RLM_ERR_INVALID_ARG               # history overlaps the state
-
-
-@pytest.mark.parametrize("rows,D,sb,ctas", [
-    (4096, 256, 24, 128),      # slice width not 16/32/64/128
-    (4096, 250, 16, 125),      # D not a multiple of the slice
-    (4096, 256, 16, 100),      # ctas not a multiple of the slice count
-    (4000, 256, 16, 128),      # rows not a multiple of the box height
-    (256, 256, 16, 64),        # fewer boxes than CTAs need
-])
-def test_row_io_measurement_rejects_bad_arguments_on_host(lib, rows, D, sb, ctas):
-    st = lib.rlm_measure_row_io(FAKE, FAKE + (1 << 30), rows, D, sb, ctas, None)
-    assert st == rlm.RLM_ERR_INVALID_ARG
-    assert lib.rlm_last_error()
-    assert lib.rlm_measure_row_io(None, FAKE, 4096, 256, 16, 128, None) == rlm.RLM_ERR_INVALID_ARG
-    assert lib.rlm_measure_row_io(FAKE + 8, FAKE, 4096, 256, 16, 128, None) == rlm.RLM_ERR_INVALID_ARG
-
-
-def test_row_io_measurement_byte_count(lib):
-    # [131072][256] bf16 in 16-byte slices by 128 CTAs: 4 KB boxes of 256 rows,
-    # 16384 boxes in all, 128 per CTA; loaded once and stored once.
-    assert lib.rlm_measure_row_io_bytes(131072, 256, 16, 128) == 2 * 131072 * 256 * 2
-    assert lib.rlm_measure_row_io_bytes(131072, 256, 32, 128) == 2 * 131072 * 256 * 2
-    assert lib.rlm_measure_row_io_bytes(131072, 250, 16, 128) == 0
 
 
 def test_prefill_workspace_only_when_the_sequence_is_segmented(lib):

@@ -298,9 +298,9 @@ def test_tcgen05_shape_mixer_prefill_is_causal_bit_exact(K):
 
 def test_packed_rows_gate_from_state_matches_oracle():
     """The gate in the epilogue of a prefill whose CTAs run several batch rows
-    (B = 9, L = 700, D = 256: three rows per CTA), each row from its own initial
+    (B = 9, L = 704, D = 256: three rows per CTA), each row from its own initial
     state."""
-    B, L, D, M = 9, 700, 256, 16
+    B, L, D, M = 9, 704, 256, 16
     inp = make_inputs(B, L, D, M, "bf16", seed=77)
     mx = make_mixer_inputs(inp, 0, seed=77)
     rng = np.random.default_rng(77)
