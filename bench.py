@@ -819,6 +819,107 @@ def run_backward_only(args):
     print(json.dumps(out), flush=True)
 
 
+def run_kernels_only(args):
+    """One representative workload per kernel that the headline path does not
+    time, for their ncu captures: each case runs 3 warm-up and 5 timed calls (L2
+    flushed before each) and the line reports its mean time and algorithmic
+    bytes.  Cases and the kernels they launch:
+      fp32_prefill        B=4 L=32768 D=256 M=16 fp32: k_chunk_local, k_chunk_carry, k_chunk_output
+      decode_b64 / b1     one plain decode step: k_decode_tile (B=64), k_decode_vec2 (B=1)
+      mixer_decode_b64    coupled mixer step H=8 K=4 (D=256): k_decode_coupled
+      mixer_prefill_d2048 coupled mixer prefill B=1 L=32768 D=2048 H=8 K=4 (4 KB rows):
+                          k_prefill_tc, k_couple_small, k_mixer_epilogue, k_mixer_tail
+      mixer_decode_d2048  coupled mixer step B=64 D=2048 H=8 K=4: k_decode_vec2 (mixer), k_mixer_finish"""
+    import torch
+
+    import paper_2607_05583_gb300 as rlm
+    from synth import make_inputs, make_mixer_inputs
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    rlm.load_library()
+    hbm_peak, _, peak_kind = _peaks()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+    out = {}
+
+    def timed(name, fn, alg_bytes):
+        for _ in range(3):
+            flush.zero_()
+            fn()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(5):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            ts.append(a.elapsed_time(b))
+        ms = statistics.mean(ts)
+        gbs = alg_bytes / (ms * 1e-3) / 1e9
+        out[name] = {"ms": round(ms, 5), "algorithmic_bytes": alg_bytes, "achieved_GBps": round(gbs, 1),
+                     "frac_hbm": round(gbs / hbm_peak, 4)}
+
+    # fp32 prefill on the SIMT chunked scan
+    B, L, D, M = 4, 32768, 256, 16
+    inp = make_inputs(B, L, D, M, "f32", seed=1)
+    x = torch.from_numpy(inp.x).to(dev)
+    p = rlm.Params.from_arrays(*inp.params(), device=dev)
+    y = torch.empty_like(x)
+    st = rlm.State.empty(B, D, M, device=dev)
+    work = torch.empty(max(rlm.rlm_prefill_workspace_size(B, L, D, M, torch.float32), 256), dtype=torch.uint8,
+                       device=dev)
+    timed("fp32_prefill", lambda: rlm.rlm_mix_prefill(x, p, y, st, workspace=work), prefill_bytes(B, L, D, M, 4))
+    del x, y, work
+
+    # plain decode steps
+    for Bd in (64, 1):
+        dinp = make_inputs(Bd, 1, D, M, "bf16", seed=3, decode_steps=2)
+        dp = rlm.Params.from_arrays(*dinp.params(), device=dev)
+        dst = rlm.State.empty(Bd, D, M, device=dev)
+        rlm.rlm_state_init(dst, dp)
+        tok = torch.from_numpy(dinp.tokens[0]).to(dev, torch.bfloat16)
+        yt = torch.empty_like(tok)
+        timed(f"decode_b{Bd}", lambda: rlm.rlm_mix_decode(tok, dst, yt), decode_bytes(Bd, D, M))
+
+    # coupled mixer decode step, fused (D = 256) and with the finishing pass (D = 2048)
+    H, K = 8, 4
+    for Dm in (256, 2048):
+        Bd = 64
+        dinp = make_inputs(Bd, 1, Dm, M, "bf16", seed=4, decode_steps=2)
+        dmx = make_mixer_inputs(dinp, K, seed=4)
+        dp = rlm.Params.from_arrays(*dinp.params(), device=dev)
+        dst = rlm.State.empty(Bd, Dm, M, device=dev)
+        rlm.rlm_state_init(dst, dp)
+        loc = rlm.Local.from_arrays(dmx.conv_w, dmx.scale, device=dev)
+        cp = rlm.Coupling.from_arrays(np.random.default_rng(5).standard_normal((H, H)), 0.5, device=dev)
+        hist = rlm.ConvState(torch.zeros(Bd, K - 1, Dm, dtype=torch.bfloat16, device=dev))
+        tok = torch.from_numpy(dinp.tokens[0]).to(dev, torch.bfloat16)
+        gt = torch.randn(Bd, 1, Dm, device=dev).to(torch.bfloat16).view_as(tok)
+        zt = torch.empty_like(tok)
+        name = "mixer_decode_b64" if Dm == 256 else "mixer_decode_d2048"
+        alg = decode_bytes(Bd, Dm, M) + 2 * Bd * Dm * (K - 1) * 2 + 2 * Bd * Dm
+        timed(name, lambda: rlm.rlm_mixer_decode(tok, gt, dst, loc, hist, zt, coupling=cp), alg)
+
+    # coupled mixer prefill on 4 KB rows (the separate coupling and channel-pair passes)
+    B, L, Dm = 1, 32768, 2048
+    inp = make_inputs(B, L, Dm, M, "bf16", seed=6)
+    mx = make_mixer_inputs(inp, K, seed=6)
+    x = torch.from_numpy(inp.x).to(dev, torch.bfloat16)
+    g = torch.from_numpy(mx.g).to(dev, torch.bfloat16)
+    p = rlm.Params.from_arrays(*inp.params(), device=dev)
+    loc = rlm.Local.from_arrays(mx.conv_w, mx.scale, device=dev)
+    cp = rlm.Coupling.from_arrays(np.random.default_rng(7).standard_normal((H, H)), 0.5, device=dev)
+    z = torch.empty_like(x)
+    work = torch.empty(max(rlm.rlm_prefill_workspace_size(B, L, Dm, M, torch.bfloat16), 256), dtype=torch.uint8,
+                       device=dev)
+    timed("mixer_prefill_d2048",
+          lambda: rlm.rlm_mixer_prefill(x, g, p, loc, z, workspace=work, coupling=cp),
+          mixer_prefill_bytes(B, L, Dm, M, K) + 4 * H * H)
+    print(json.dumps({"kernels_only": out, "peak_GBps": hbm_peak, "peak_kind": peak_kind}), flush=True)
+
+
 def run_mixer_only(args):
     """The mixer prefill measurements alone (used for their ncu captures)."""
     import torch
@@ -969,8 +1070,8 @@ def main():
     ap.add_argument("--quick", action="store_true", help="prefill only (no sweep/decode/backward)")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU-oracle baseline")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
-    ap.add_argument("--only", default="all", choices=["all", "backward", "mixer"],
-                    help="backward / mixer: run only that measurement (diagnostic, ncu captures)")
+    ap.add_argument("--only", default="all", choices=["all", "backward", "mixer", "kernels"],
+                    help="backward / mixer / kernels: run only that measurement (diagnostic, ncu captures)")
     ap.add_argument("--soak", type=float, default=1.5,
                     help="seconds of untimed prefill before the timed steps (clock sampling)")
     args = ap.parse_args()
@@ -982,6 +1083,8 @@ def main():
         run_backward_only(args)
     elif args.only == "mixer":
         run_mixer_only(args)
+    elif args.only == "kernels":
+        run_kernels_only(args)
     else:
         run_ours(args)
 
