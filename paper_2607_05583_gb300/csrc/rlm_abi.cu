@@ -180,13 +180,14 @@ rlm_status check_prefill_states(const rlm_tensor *x, const rlm_tensor *y, const 
 }
 
 // The prefill path for a problem: the tcgen05 prefill (bf16, M <= 64), its
-// time-reversed form (other bf16 M <= 32), else the SIMT scan.  Both tcgen05 forms
+// time-reversed form (other bf16 M <= 32), the tcgen05 prefill for fp32 I/O
+// (M <= 16, zero initial state), else the SIMT scan.  Both bf16 tcgen05 forms
 // work in 64-token chunks aligned to one end of the sequence; when L is not a
 // multiple of 64, an initial state enters them through a negative power of
 // lambda (up to lambda^-63), which overflows fp32 for decays above 88/63 per
 // token.  Such calls run on the SIMT scan, whose powers of lambda are all
 // positive, so every finite decay >= 0 is covered.
-enum class PrefillPath { kTc, kRev, kSimt };
+enum class PrefillPath { kTc, kRev, kTc32, kSimt };
 
 bool state_in_needs_simt(int64_t L, bool with_state_in) { return with_state_in && L % 64 != 0; }
 
@@ -195,6 +196,7 @@ PrefillPath prefill_path(const rlm_tensor *x, int M, bool with_state_in) {
     if (state_in_needs_simt(x->L, with_state_in)) return PrefillPath::kSimt;
     if (tc_prefill_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kTc;
     if (tc_prefill_rev_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kRev;
+    if (!with_state_in && tc32_prefill_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kTc32;
     return PrefillPath::kSimt;
 }
 
@@ -210,6 +212,9 @@ cudaError_t launch_prefill(PrefillPath path, const rlm_tensor *x, const rlm_para
         case PrefillPath::kRev:
             return tc_prefill_rev(x->ptr, y, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase, sin, so, co,
                                   ln->workspace, st);
+        case PrefillPath::kTc32:
+            return tc32_prefill(static_cast<const float *>(x->ptr), static_cast<float *>(y), x->B, x->L, D, M,
+                                p->decay, p->freq, p->amp, p->phase, so, co, st);
         default:
             return simt_prefill(x->ptr, y, x->dtype, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase,
                                 sin, so, co, ln->workspace, st);
@@ -579,13 +584,15 @@ rlm_status rlm_validate_params(const rlm_params *p) {
 
 rlm_status rlm_get_device_status(const rlm_launch *ln) {
     if (!ln) return fail(RLM_ERR_INVALID_ARG, "launch is NULL");
-    int status = RLM_OK, bwd = RLM_OK, mix = RLM_OK;
+    int status = RLM_OK, bwd = RLM_OK, mix = RLM_OK, t32 = RLM_OK;
     cudaError_t e = read_and_clear_device_status(&status, static_cast<cudaStream_t>(ln->stream));
     if (e == cudaSuccess) e = read_and_clear_bwd_status(&bwd, static_cast<cudaStream_t>(ln->stream));
     if (e == cudaSuccess) e = read_and_clear_mixer_status(&mix, static_cast<cudaStream_t>(ln->stream));
+    if (e == cudaSuccess) e = read_and_clear_tc32_status(&t32, static_cast<cudaStream_t>(ln->stream));
     if (e != cudaSuccess) return cuda_fail(e, "rlm_get_device_status");
     if (status == RLM_OK) status = bwd;
     if (status == RLM_OK) status = mix;
+    if (status == RLM_OK) status = t32;
     if (status != RLM_OK) return fail((rlm_status)status, "a bounded device-side wait expired");
     return RLM_OK;
 }
