@@ -22,9 +22,11 @@
 // 4 channels is 16 bytes, the same slice of the [B][L][D] row as the bf16
 // kernel's 8 channels, so loads and stores have the bf16 kernel's granularity
 // with twice its bytes per token-channel.
-// TMEM (512 columns): channel c's accumulator at columns 32 c (32 chunks); its
-// A operands hi / lo (128 lanes x 32 columns of packed bf16 pairs) at columns
-// 256 + 64 c and 256 + 64 c + 32.
+// TMEM (512 columns): two accumulator buffers (tile v uses buffer v & 1), channel
+// c's at columns 128 b + 32 c (32 chunks); its A operands hi / lo (128 lanes x 32
+// columns of packed bf16 pairs) at columns 256 + 64 c and 256 + 64 c + 32.  With
+// two buffers the chain of one tile (the Toeplitz/state MMAs) runs while the
+// scan, up-projection and epilogue of the tile before still hold the other.
 // Rows of channel c's accumulator (= TMEM lanes): its Toeplitz rows (positions
 // 0-31, 32-63) in quarters 2, 3 for channels 0, 1 and in quarters 0, 1 for
 // channels 2, 3; its 32 state rows (2 m + ri) in quarter c; zeros in the last
@@ -40,7 +42,9 @@
 //   12-15  transposers (boxes k = t mod 4): fp32 token rows -> hi / lo K-major
 //          B operands.
 //   16     TMA producer; 17 TMA store issuer and TMEM allocation.
-//   18-21  MMA issue for one channel each.
+//   18-21  MMA issue for one channel each: the thread polls the inputs of the
+//          next Toeplitz/state chain and of the next up-projection and issues
+//          whichever is ready.
 // Warps 0-7 first build the per-channel constants.
 //
 // Every wait is bounded (about 2 s): the waiting thread then sets a shared abort
@@ -70,7 +74,7 @@ constexpr int kDG = 4;                 // channels per CTA
 constexpr int kModes = 16;             // modes per channel in the tables (M <= 16 is padded)
 constexpr int kBox = 256;              // TMA box rows (16 bytes each)
 constexpr int kBoxes = kTile / kBox;   // 8 per tile
-constexpr int kXSlots = 13;            // x ring depth (boxes)
+constexpr int kXSlots = 15;            // x ring depth (boxes)
 constexpr int kYRows = 512;            // rows per y ring slot (8 chunks)
 constexpr int kYPerTile = kTile / kYRows;
 constexpr int kYSlots = 6;
@@ -90,11 +94,12 @@ constexpr int kTransposers = 4;
 constexpr int kAuStride = 4096;
 constexpr int kAuPart = kDG * kAuStride;           // 16 KB: the hi tables, then the lo tables
 // B operand of a channel's drives (one part): K = 64 positions (reversed) x
-// N = 32 chunks, K-major core matrices of 8 chunks x 16 B.  LBO = 144 (not 128)
-// spreads a transposer warp's 16-byte stores over distinct banks.
-constexpr int kBxLbo = 144, kBxSbo = 8 * kBxLbo;    // 1152
-constexpr int kBxPart = 4 * kBxSbo;                 // 4608 bytes per channel and part
-constexpr int kBxBuf = kDG * 2 * kBxPart;           // 36864: [channel][hi, lo]
+// N = 32 chunks, K-major core matrices of 8 chunks x 16 B.  The parts are 4096 +
+// 16 bytes apart, so the 8 rows one stmatrix writes (hi and lo of the 4
+// channels) land in distinct banks.
+constexpr int kBxLbo = 128, kBxSbo = 1024;
+constexpr int kBxPart = 4 * kBxSbo + 16;            // 4112 bytes per channel and part
+constexpr int kBxBuf = kDG * 2 * kBxPart;           // 32896: [channel][hi, lo]
 // Carried-state operand (one part): K = 32 (Re, Im of 16 modes) x N = 32 chunks.
 // LBO 144 spreads a chunk's 16 mode words over distinct banks; the lo part sits
 // 16 banks after the hi part, so the two lanes of a mode write disjoint banks.
@@ -104,7 +109,7 @@ constexpr int kBsStride = 2 * kBsPart;              // per channel: hi, lo
 constexpr int kOffAu = 0;
 constexpr int kOffBx = kOffAu + 2 * kAuPart;                 // 32768
 constexpr int kOffBs = kOffBx + 2 * kBxBuf;                  // 106496
-constexpr int kOffX = kOffBs + kDG * kBsStride;              // 125440
+constexpr int kOffX = kOffBs + kDG * kBsStride;
 constexpr int kOffY = kOffX + kXSlots * kBox * 16;
 constexpr int kOffBar = kOffY + kYSlots * kYRows * 16;
 constexpr int kNumBars = 96;
@@ -132,12 +137,14 @@ constexpr int kPrologueThreads = 256;
 constexpr int kBarXFull = 0;                    // [kXSlots]
 constexpr int kBarXEmpty = kXSlots;             // [kXSlots]
 constexpr int kBarBxFull = 2 * kXSlots;         // [2]
-constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]: released by the 4 MMA threads
-constexpr int kBarTwDone = kBarBxEmpty + 2;     // [4]: Toeplitz/state MMAs of a channel done
-constexpr int kBarSFull = kBarTwDone + kDG;     // [4]: carried states of a channel written
-constexpr int kBarUDone = kBarSFull + kDG;      // [4]: up-projection of a channel done
-constexpr int kBarDEmpty = kBarUDone + kDG;     // [4]: accumulator of a channel read out
-constexpr int kBarYFull = kBarDEmpty + kDG;     // [kYSlots]
+constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]: released by the 4 scan warps
+// Per channel c and accumulator buffer b (index 2 c + b), each completing once
+// per tile of its buffer:
+constexpr int kBarTwDone = kBarBxEmpty + 2;     // [4][2]: Toeplitz/state MMAs done
+constexpr int kBarSFull = kBarTwDone + 2 * kDG; // [4][2]: carried states written
+constexpr int kBarUDone = kBarSFull + 2 * kDG;  // [4][2]: up-projection done
+constexpr int kBarDEmpty = kBarUDone + 2 * kDG; // [4][2]: accumulator read out
+constexpr int kBarYFull = kBarDEmpty + 2 * kDG; // [kYSlots]
 constexpr int kBarYEmpty = kBarYFull + kYSlots; // [kYSlots]
 constexpr int kBarFinal = kBarYEmpty + kYSlots; // [4]
 constexpr int kBarConsts = kBarFinal + kDG;     // the A operands and U tables are built
@@ -154,6 +161,16 @@ __device__ __forceinline__ bool bar_try(uint32_t bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Non-blocking test of an mbarrier phase (for a thread that polls several).
+__device__ __forceinline__ bool bar_test(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
         : "=r"(ok)
         : "r"(bar), "r"(parity)
         : "memory");
@@ -361,13 +378,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             bar_init(bar(kBarBxFull + i), kBoxes);
             bar_init(bar(kBarBxEmpty + i), kDG);
         }
-        for (int i = 0; i < kDG; ++i) {
+        for (int i = 0; i < 2 * kDG; ++i) {
             bar_init(bar(kBarTwDone + i), 1);
             bar_init(bar(kBarSFull + i), 1);
             bar_init(bar(kBarUDone + i), 1);
             bar_init(bar(kBarDEmpty + i), 4);
-            bar_init(bar(kBarFinal + i), 1);
         }
+        for (int i = 0; i < kDG; ++i) bar_init(bar(kBarFinal + i), 1);
         for (int i = 0; i < kYSlots; ++i) {
             bar_init(bar(kBarYFull + i), 4);
             bar_init(bar(kBarYEmpty + i), 1);
@@ -533,40 +550,62 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp >= 12 && warp < 12 + kTransposers) {
         // ---------------------------------------------------- transposers (boxes k = t mod 4)
-        // Lane l takes tokens 8 l .. 8 l + 7 of the box: 8 token rows of 4 fp32
-        // channels, i.e. one K group (8 positions) of chunk n for every channel,
-        // written reversed (position p -> p' = 63 - p) as hi and lo bf16 parts.
+        // Per 8-token block (one K group of one chunk): ldmatrix.trans of the 8
+        // token rows (in reversed order, so positions come out as p' = 63 - p)
+        // gives thread t the half-word k = t / 4 (half k % 2 of channel k / 2) of
+        // two tokens; one shuffle with thread t ^ 4 joins the two halves into the
+        // fp32 values.  The thread of the even half then holds the bf16 high parts
+        // of its channel's two positions, the thread of the odd half the low
+        // parts: exactly row k of an 8 x 8 matrix whose rows are (channel, part),
+        // which stmatrix writes into the 8 B operands (4 channels x hi, lo).
         for (int k = warp - 12; k < total_boxes; k += kTransposers) {
             const int j = k / kBoxes, tq = k % kBoxes;
             const int buf = j & 1, use = j >> 1;
             const uint32_t slot = k % kXSlots;
             if (!wait_bar(bar(kBarXFull + slot), (k / kXSlots) & 1, abort_flag)) break;
-            const float4 *xs = reinterpret_cast<const float4 *>(smem + kOffX + slot * (kBox * 16)) + 8 * lane;
-            float4 r[8];
+            const uint32_t xs = sbase + kOffX + slot * (kBox * 16);
+            uint32_t r[8][4];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) r[i] = xs[i];
+            for (int sb = 0; sb < 8; ++sb) {
+                const uint32_t src = xs + (32 * sb + 8 * (lane >> 3) + (7 - (lane & 7))) * 16;
+                asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+                             : "=r"(r[sb][0]), "=r"(r[sb][1]), "=r"(r[sb][2]), "=r"(r[sb][3])
+                             : "r"(src)
+                             : "memory");
+            }
+            // Join the halves and split into bf16 parts (even half: hi, odd: lo).
+            const bool odd = (lane >> 2) & 1;
+#pragma unroll
+            for (int sb = 0; sb < 8; ++sb) {
+#pragma unroll
+                for (int mq = 0; mq < 4; ++mq) {
+                    const uint32_t mine = r[sb][mq];
+                    const uint32_t other = __shfl_xor_sync(0xffffffffu, mine, 4);
+                    const uint32_t lo16 = odd ? other : mine, hi16 = odd ? mine : other;
+                    const float fa = __uint_as_float(__byte_perm(lo16, hi16, 0x5410));
+                    const float fb = __uint_as_float(__byte_perm(lo16, hi16, 0x7632));
+                    const float ha = bf16_hi(fa), hb = bf16_hi(fb);
+                    r[sb][mq] = odd ? pack_bf16x2(fa - ha, fb - hb) : pack_bf16x2(ha, hb);
+                }
+            }
             if (!wait_bar(bar(kBarBxEmpty + buf), (use & 1) ^ 1, abort_flag)) break;
-            const int tb = 32 * tq + lane;                        // 8-token block within the tile
-            const int n = tb >> 3, kb = 7 - (tb & 7);
-            uint8_t *bx = smem + kOffBx + buf * kBxBuf + (n >> 3) * kBxSbo + kb * kBxLbo + (n & 7) * 16;
-            auto emit = [&](int c, float v0, float v1, float v2, float v3, float v4, float v5, float v6, float v7) {
-                // K order within the group: k % 8 = 7 - (token % 8).
-                uint4 h, l;
-                split_pack(v7, v6, h.x, l.x);
-                split_pack(v5, v4, h.y, l.y);
-                split_pack(v3, v2, h.z, l.z);
-                split_pack(v1, v0, h.w, l.w);
-                *reinterpret_cast<uint4 *>(bx + c * 2 * kBxPart) = h;
-                *reinterpret_cast<uint4 *>(bx + c * 2 * kBxPart + kBxPart) = l;
-            };
-            emit(0, r[0].x, r[1].x, r[2].x, r[3].x, r[4].x, r[5].x, r[6].x, r[7].x);
-            emit(1, r[0].y, r[1].y, r[2].y, r[3].y, r[4].y, r[5].y, r[6].y, r[7].y);
-            emit(2, r[0].z, r[1].z, r[2].z, r[3].z, r[4].z, r[5].z, r[6].z, r[7].z);
-            emit(3, r[0].w, r[1].w, r[2].w, r[3].w, r[4].w, r[5].w, r[6].w, r[7].w);
+            // stmatrix row address: thread t gives row t % 8 = (channel, part) of
+            // matrix t / 8, i.e. of token block 32 tq + 4 sb + t / 8.
+            const int rr = lane & 7, mq = lane >> 3;
+            const uint32_t bx = sbase + kOffBx + buf * kBxBuf + ((rr >> 1) * 2 + (rr & 1)) * kBxPart;
+#pragma unroll
+            for (int sb = 0; sb < 8; ++sb) {
+                const int tb = 32 * tq + 4 * sb + mq;    // 8-token block within the tile
+                const int n = tb >> 3, kb = 7 - (tb & 7);
+                const uint32_t dst = bx + (n >> 3) * kBxSbo + kb * kBxLbo + (n & 7) * 16;
+                asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1,%2,%3,%4};" ::"r"(dst),
+                             "r"(r[sb][0]), "r"(r[sb][1]), "r"(r[sb][2]), "r"(r[sb][3])
+                             : "memory");
+            }
             fence_async_smem();
             __syncwarp();
-            // The x slot is released only now that the stores have consumed the
-            // loaded registers.
+            // The x slot is released only now that stmatrix has consumed the
+            // ldmatrix registers.
             if (lane == 0) {
                 bar_arrive(bar(kBarXEmpty + slot));
                 bar_arrive(bar(kBarBxFull + buf));
@@ -613,10 +652,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp >= 18) {
         // ---------------------------------------------------- MMA issuer, one channel
-        // Per tile: the Toeplitz/state chain (hi hi + hi lo + lo hi) into the
-        // channel's accumulator, then, once the scan has written the carried
-        // states, the up-projection (same three terms).  The next tile's chain
-        // waits until the epilogue has read the accumulator.
+        // Tile v uses accumulator buffer v & 1 (and B-operand buffer v & 1).  The
+        // thread issues whichever is ready: the Toeplitz/state chain of tile tw
+        // (hi hi + hi lo + lo hi; its B operand full and its buffer's previous tile,
+        // tw - 2, read out by the epilogue) or the up-projection of tile uu (same
+        // three terms) once the scan has written that tile's carried states.  tw
+        // stays at most two tiles ahead of uu, so no barrier runs a phase ahead of
+        // this thread.
         const int c = warp - 18;
         const uint64_t dxh = umma_desc(sbase + kOffBx + c * 2 * kBxPart, kBxLbo, kBxSbo);
         const uint64_t dxl = umma_desc(sbase + kOffBx + c * 2 * kBxPart + kBxPart, kBxLbo, kBxSbo);
@@ -625,36 +667,64 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint64_t dsh = umma_desc(sbase + kOffBs + c * kBsStride, kBsLbo, kBsSbo);
         const uint64_t dsl = umma_desc(sbase + kOffBs + c * kBsStride + kBsPart, kBsLbo, kBsSbo);
         const uint32_t aH = tmem + kTmemA + c * 64, aL = aH + 32;
-        const uint32_t d = tmem + c * kNT;
         constexpr uint64_t kXStep = (2 * kBxLbo) >> 4;     // 16 K elements of the drive operand
         constexpr uint64_t kSStep = (2 * kBsLbo) >> 4;     // 16 K elements of the state operand
         if (lane == 0 && wait_bar(bar(kBarConsts), 0, abort_flag)) {
             tc_fence_after();
-            for (int v = 0; v < nV; ++v) {
-                const int buf = v & 1, use = v >> 1;
-                if (!wait_bar(bar(kBarBxFull + buf), use & 1, abort_flag)) break;
-                if (v > 0 && !wait_bar(bar(kBarDEmpty + c), (v - 1) & 1, abort_flag)) break;
-                tc_fence_after();
-                const uint64_t xo = (uint64_t)((buf * kBxBuf) >> 4);
+            int tw = 0, uu = 0;
+            long long t_idle = 0;
+            uint32_t polls = 0;
+            while (uu < nV) {
+                bool progress = false;
+                if (uu < tw) {
+                    const int bb = uu & 1, u = uu >> 1;
+                    if (bar_test(bar(kBarSFull + 2 * c + bb), u & 1)) {
+                        tc_fence_after();
+                        const uint32_t d = tmem + bb * 128 + c * kNT;
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk) umma_ts(d, aH + kk * 8, dxh + xo + kk * kXStep, kIdesc, kk > 0);
+                        for (int kk = 0; kk < 2; ++kk) umma_ss(d, duh + kk * 16, dsh + kk * kSStep, kIdesc, 1);
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk) umma_ts(d, aH + kk * 8, dxl + xo + kk * kXStep, kIdesc, 1);
+                        for (int kk = 0; kk < 2; ++kk) umma_ss(d, duh + kk * 16, dsl + kk * kSStep, kIdesc, 1);
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk) umma_ts(d, aL + kk * 8, dxh + xo + kk * kXStep, kIdesc, 1);
-                umma_commit(bar(kBarTwDone + c));
-                if (!wait_bar(bar(kBarSFull + c), v & 1, abort_flag)) break;
-                tc_fence_after();
-                // The scan has seen this chain's commit, so its MMAs (and their
-                // reads of the B operand) are complete: release the buffer.
-                bar_arrive(bar(kBarBxEmpty + buf));
+                        for (int kk = 0; kk < 2; ++kk) umma_ss(d, dul + kk * 16, dsh + kk * kSStep, kIdesc, 1);
+                        umma_commit(bar(kBarUDone + 2 * c + bb));
+                        ++uu;
+                        progress = true;
+                    }
+                }
+                if (tw < nV && tw < uu + 2) {
+                    const int bb = tw & 1, u = tw >> 1;
+                    if (bar_test(bar(kBarBxFull + bb), u & 1) &&
+                        (tw < 2 || bar_test(bar(kBarDEmpty + 2 * c + bb), (u - 1) & 1))) {
+                        tc_fence_after();
+                        const uint64_t xo = (uint64_t)((bb * kBxBuf) >> 4);
+                        const uint32_t d = tmem + bb * 128 + c * kNT;
 #pragma unroll
-                for (int kk = 0; kk < 2; ++kk) umma_ss(d, duh + kk * 16, dsh + kk * kSStep, kIdesc, 1);
+                        for (int kk = 0; kk < 4; ++kk) umma_ts(d, aH + kk * 8, dxh + xo + kk * kXStep, kIdesc, kk > 0);
 #pragma unroll
-                for (int kk = 0; kk < 2; ++kk) umma_ss(d, duh + kk * 16, dsl + kk * kSStep, kIdesc, 1);
+                        for (int kk = 0; kk < 4; ++kk) umma_ts(d, aH + kk * 8, dxl + xo + kk * kXStep, kIdesc, 1);
 #pragma unroll
-                for (int kk = 0; kk < 2; ++kk) umma_ss(d, dul + kk * 16, dsh + kk * kSStep, kIdesc, 1);
-                umma_commit(bar(kBarUDone + c));
+                        for (int kk = 0; kk < 4; ++kk) umma_ts(d, aL + kk * 8, dxh + xo + kk * kXStep, kIdesc, 1);
+                        umma_commit(bar(kBarTwDone + 2 * c + bb));
+                        ++tw;
+                        progress = true;
+                    }
+                }
+                if (progress) {
+                    t_idle = 0;
+                    polls = 0;
+                } else if ((++polls & 255u) == 0) {
+                    // Bounded like wait_bar: give up after kWaitLimitCycles without progress.
+                    if (*abort_flag) break;
+                    const long long now = clock64();
+                    if (t_idle == 0) {
+                        t_idle = now;
+                    } else if (now - t_idle > kWaitLimitCycles) {
+                        *abort_flag = 1;
+                        atomicExch(&g_tc32_status, (int)RLM_ERR_TIMEOUT);
+                        break;
+                    }
+                }
             }
             // Drain: all MMAs this thread issued complete before TMEM is released.
             umma_commit(bar(kBarFinal + c));
@@ -680,13 +750,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         float2 S = make_float2(0.0f, 0.0f);
         uint8_t *bs = smem + kOffBs + ch * kBsStride + ri * kBsPart + (m / 4) * kBsLbo + (m % 4) * 4;
         for (int v = 0; v < nV; ++v) {
+            const int bb = v & 1, u = v >> 1;
             if (kPack && real_tile(v) == 0) S = make_float2(0.0f, 0.0f);   // a new batch row starts from zero
-            if (!wait_bar(bar(kBarTwDone + ch), v & 1, abort_flag)) break;
+            if (!wait_bar(bar(kBarTwDone + 2 * ch + bb), u & 1, abort_flag)) break;
+            // The chain of tile v has completed, so its reads of B-operand buffer
+            // v & 1 are done: release it (one arrival per channel).
+            if (lane == 0) bar_arrive(bar(kBarBxEmpty + bb));
+            // The carried-state operand is single-buffered: tile v - 1's
+            // up-projection must have read it before it is rewritten.
+            if (v > 0 && !wait_bar(bar(kBarUDone + 2 * ch + (bb ^ 1)), ((v - 1) >> 1) & 1, abort_flag)) break;
             tc_fence_after();
 #pragma unroll
             for (int h = 0; h < kNT / 16; ++h) {
                 uint32_t va[16];
-                tmem_ld16(tmem + (st_lane << 16) + ch * kNT + 16 * h, va);
+                tmem_ld16(tmem + (st_lane << 16) + bb * 128 + ch * kNT + 16 * h, va);
                 tmem_wait_ld();
 #pragma unroll
                 for (int n = 0; n < 16; ++n) {
@@ -705,7 +782,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_async_smem();
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) bar_arrive(bar(kBarSFull + ch));
+            if (lane == 0) bar_arrive(bar(kBarSFull + 2 * ch + bb));
         }
     } else if (warp < 8) {
         // ---------------------------------------------------- epilogue
@@ -720,19 +797,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int hb = quarter < 2 ? 8 : 0;
         const uint32_t trow = tmem + ((uint32_t)(32 * quarter) << 16) + 16 * h;
         for (int j = 0; j < nV; ++j) {
-            if (!wait_bar(bar(kBarUDone + c0), j & 1, abort_flag) ||
-                !wait_bar(bar(kBarUDone + c0 + 1), j & 1, abort_flag))
+            const int bb = j & 1, u = j >> 1;
+            if (!wait_bar(bar(kBarUDone + 2 * c0 + bb), u & 1, abort_flag) ||
+                !wait_bar(bar(kBarUDone + 2 * (c0 + 1) + bb), u & 1, abort_flag))
                 break;
             tc_fence_after();
             uint32_t va[16], vb[16];
-            tmem_ld16(trow + c0 * kNT, va);
-            tmem_ld16(trow + (c0 + 1) * kNT, vb);
+            tmem_ld16(trow + bb * 128 + c0 * kNT, va);
+            tmem_ld16(trow + bb * 128 + (c0 + 1) * kNT, vb);
             tmem_wait_ld();
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {
-                bar_arrive(bar(kBarDEmpty + c0));
-                bar_arrive(bar(kBarDEmpty + c0 + 1));
+                bar_arrive(bar(kBarDEmpty + 2 * c0 + bb));
+                bar_arrive(bar(kBarDEmpty + 2 * (c0 + 1) + bb));
             }
             bool ok = true;
 #pragma unroll
