@@ -148,10 +148,14 @@ constexpr int kOffWtab = kOffY;                        // [8 ch][32 words][33]: 
 constexpr int kOffTpair = kOffBs;                      // [8 ch][144 words]: Toeplitz pairs
 constexpr int kOffKp = kOffTpair + 8 * kTpairStride * 4;  // [2 halves][8 ch][64] fp32 partial sums of K
 static_assert(8 * 32 * kWtabStride * 4 <= kYSlots * kYRows * 16, "W table does not fit the y ring");
-static_assert(kOffKp + 2 * 8 * 64 * 4 <= kOffX, "prologue tables do not fit");
-// Named barrier for the 16 warps that build the constants (0-11 and 18-21).
+// [8 ch][kModes][5] float2: lambda, c, lambda^2, lambda^4, lambda^8 of each mode.
+constexpr int kOffLtab = kOffKp + 2 * 8 * 64 * 4;
+static_assert(kOffLtab + 8 * 16 * 5 * 8 <= kOffX, "prologue tables do not fit");
+// Named barriers: the 16 warps that build the constants (0-11 and 18-21); the
+// CTA's set-up, which the TMA producer warp only arrives at.
 constexpr int kPrologueBarrier = 1;
 constexpr int kPrologueThreads = 512;
+constexpr int kSetupBarrier = 2;
 
 // Barrier indices.
 constexpr int kBarXFull = 0;                    // [kXSlots]
@@ -429,14 +433,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int nV = kSeg ? nA + nB : kPack ? nB : args.ntiles;
     auto real_tile = [&](int v) { return kPack ? v % args.ntiles : ja + (v < nA ? v : v - nA); };
     auto row_of = [&](int v) { return kPack ? b + v / args.ntiles : b; };
-    // Constant builders (warps 0-11 and 18-21) issue their parameter loads first,
-    // so the DRAM latency overlaps the barrier set-up and TMEM allocation.
+    // Constant builders: warps 0-11 and 18-21.  The first 128 of them (one per
+    // (channel, mode)) form each mode's powers once for all builders and issue
+    // their parameter loads first, so the DRAM latency overlaps the set-up.
+    // (Computing these powers in warps 22-25 instead, the MMA issuers of channels
+    // 4-7, made the steady state slower: 47.8 against 45.7 us at B = 4, L = 32768.)
     const bool builder = warp < 12 || (warp >= 18 && warp < 22);
     const int pq = warp & 3, pe = warp < 12 ? warp >> 2 : 3;
     const int ptid = (pe * 4 + pq) * 32 + lane;
+    const bool lpow = builder && ptid < 128;
+    const int l_c = ptid >> 4, l_m = ptid & 15;
     float p_decay = 0.0f, p_freq = 0.0f, p_amp = 0.0f, p_phase = 0.0f;
-    if (builder && ((ptid >> 2) & 15) < args.M) {
-        const int pm = (d0 + (ptid >> 6)) * args.Mt + args.m0 + ((ptid >> 2) & 15);
+    if (lpow && l_m < args.M) {
+        const int pm = (d0 + l_c) * args.Mt + args.m0 + l_m;
         p_decay = args.decay[pm];
         p_freq = args.freq[pm];
         p_amp = args.amp[pm];
@@ -447,107 +456,145 @@ __global__ void __launch_bounds__(kThreads, 1)
     volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kOffMisc);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + kOffMisc + 16);
 
-    if (tid == 0) {
-        *abort_flag = 0;
-        for (int i = 0; i < kXSlots; ++i) {
-            bar_init(bar(kBarXFull + i), 1);
-            bar_init(bar(kBarXEmpty + i), 1);
-        }
-        for (int i = 0; i < 2; ++i) {
-            bar_init(bar(kBarBxFull + i), kBoxes);
-            bar_init(bar(kBarBxEmpty + i), kDG);
-        }
-        for (int i = 0; i < kDG; ++i) {
-            bar_init(bar(kBarTwDone + i), 1);
-            bar_init(bar(kBarSFull + i), 1);
-            bar_init(bar(kBarUDone + i), 1);
-            bar_init(bar(kBarDEmpty + i), 4);
-            bar_init(bar(kBarFinal + i), 1);
-        }
-        for (int i = 0; i < kYSlots; ++i) {
-            bar_init(bar(kBarYFull + i), 4);
-            bar_init(bar(kBarYEmpty + i), 1);
-        }
-        bar_init(bar(kBarConsts), 1);
-        if (kMix)
-            for (int i = 0; i < kYSlots; ++i) bar_init(bar(kBarGFull + i), 1);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    if (warp == 17) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         smem_u32(tmem_slot)),
-                     "r"(kTmemCols));
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *tmem_slot;
-
-    // The producer fills the whole ring before the constants are built.
+    // Set-up.  The TMA producer warp initialises the x ring's barriers, arrives
+    // at the set-up barrier without waiting for it and fills the whole ring at
+    // once (issuing a TMA load blocks its thread while the previous box is being
+    // processed, so it must not hold up the others).  Thread 0 initialises the
+    // other barriers, warp 17 allocates TMEM.
     const int total_boxes = nV * kBoxes;
     int issued = 0;
-    if (warp == 16 && lane == 0) {
-        for (; issued < total_boxes && issued < kXSlots; ++issued) {
-            const int jt = real_tile(issued / kBoxes), q = issued % kBoxes, bq = row_of(issued / kBoxes);
-            const uint32_t slot = issued % kXSlots;
-            bar_expect_tx(bar(kBarXFull + slot), kBox * 16);
-            tma_load_3d(sbase + kOffX + slot * (kBox * 16), &tmap_x, d0,
-                        (int)(args.t0 + (int64_t)jt * kTile + q * kBox), bq, bar(kBarXFull + slot));
+    uint32_t tmem = 0;
+    if (warp == 16) {
+        if (lane == 0) {
+            *abort_flag = 0;
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmap_x)) : "memory");
+            for (int i = 0; i < kXSlots; ++i) {
+                bar_init(bar(kBarXFull + i), 1);
+                bar_init(bar(kBarXEmpty + i), 1);
+            }
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            fence_async_smem();
         }
+        __syncwarp();
+        asm volatile("bar.arrive %0, %1;" ::"n"(kSetupBarrier), "n"(kThreads) : "memory");
+        if (lane == 0) {
+            for (; issued < total_boxes && issued < kXSlots; ++issued) {
+                const int jt = real_tile(issued / kBoxes), q = issued % kBoxes, bq = row_of(issued / kBoxes);
+                const uint32_t slot = issued % kXSlots;
+                bar_expect_tx(bar(kBarXFull + slot), kBox * 16);
+                tma_load_3d(sbase + kOffX + slot * (kBox * 16), &tmap_x, d0,
+                            (int)(args.t0 + (int64_t)jt * kTile + q * kBox), bq, bar(kBarXFull + slot));
+            }
+        }
+    } else {
+        if (tid == 0) {
+            for (int i = 0; i < 2; ++i) {
+                bar_init(bar(kBarBxFull + i), kBoxes);
+                bar_init(bar(kBarBxEmpty + i), kDG);
+            }
+            for (int i = 0; i < kDG; ++i) {
+                bar_init(bar(kBarTwDone + i), 1);
+                bar_init(bar(kBarSFull + i), 1);
+                bar_init(bar(kBarUDone + i), 1);
+                bar_init(bar(kBarDEmpty + i), 4);
+                bar_init(bar(kBarFinal + i), 1);
+            }
+            for (int i = 0; i < kYSlots; ++i) {
+                bar_init(bar(kBarYFull + i), 4);
+                bar_init(bar(kBarYEmpty + i), 1);
+            }
+            bar_init(bar(kBarConsts), 1);
+            if (kMix)
+                for (int i = 0; i < kYSlots; ++i) bar_init(bar(kBarGFull + i), 1);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        if (warp == 17) {
+            if (lane == 0) {
+                asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmap_y)) : "memory");
+                if (kMix) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmap_g)) : "memory");
+            }
+            __syncwarp();
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             smem_u32(tmem_slot)),
+                         "r"(kTmemCols));
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+        }
+        tc_fence_before();
+        asm volatile("bar.sync %0, %1;" ::"n"(kSetupBarrier), "n"(kThreads) : "memory");
+        tc_fence_after();
+        tmem = *tmem_slot;
+    }
+
+    // Per-mode powers (builder threads 0-127, one per (channel, mode)): lambda and c
+    // in full fp32 accuracy (also the mode coefficients for decode), lambda^2,
+    // lambda^4 and lambda^8 by squaring.
+    if (lpow) {
+        const float2 lam = lambda_pow(p_decay, p_freq, 1.0f);
+        const float2 cf = mode_coef(p_amp, p_phase);
+        if (args.coef_out && b == 0 && seg == 0 && l_m < args.M)
+            args.coef_out[(d0 + l_c) * args.Mt + args.m0 + l_m] = make_float4(lam.x, lam.y, cf.x, cf.y);
+        const float2 l2 = cmul(lam, lam), l4 = cmul(l2, l2), l8 = cmul(l4, l4);
+        float2 *lt = reinterpret_cast<float2 *>(smem + kOffLtab) + (l_c * kModes + l_m) * 5;
+        lt[0] = lam;
+        lt[1] = cf;
+        lt[2] = l2;
+        lt[3] = l4;
+        lt[4] = l8;
     }
 
     // ---------------------------------------------------- per-channel constants
     // Built by warps 0-11 and 18-21 (synchronised by a named barrier), while the
     // transposers, the producer and the store issuer start their work.  Warp
     // (quarter q, rank e within its quarter) has prologue thread index ptid.
-    // Stage 1: thread (c, m, qn) runs the powers lambda^n, n in [16 qn, 16 qn + 16),
-    // of mode m of channel c: the U rows (Re, -Im of c lambda^(n+1)), the W-row
-    // words (lambda^n packed in pairs of n), and Re(c lambda^n) summed over the
-    // eight modes of its warp (a fixed shuffle tree) into Kp[half][c][n].
+    // Stage 1: builder warp bw (channel c = bw / 2) runs the powers lambda^n of
+    // its modes m = 4 (bw % 2) + lane % 4 + 8 j at the positions n = q8 + 8 e
+    // (q8 = lane / 4, e < 8), by a recurrence with step lambda^8.  Per power it
+    // writes the U row word (Re, -Im of c lambda^(n+1)), for even n the W-row
+    // words (lambda^n, lambda^(n+1) packed), and adds Re(c lambda^n) to its
+    // partial sum of K[n].  A warp's U stores cover every (n mod 8, m mod 4) pair,
+    // i.e. 32 distinct banks.  The partial sums are reduced over the warp's four
+    // lanes of equal q8 (a fixed shuffle tree) into Kp[bw % 2][c][n].
     if (builder) {
-        const int c = ptid >> 6, m = (ptid >> 2) & 15, qn = ptid & 3;
-        const int pm = (d0 + c) * args.Mt + args.m0 + m;
-        const float ga = p_decay, om = p_freq;
-        const float2 lam = lambda_pow(ga, om, 1.0f);
-        const float2 cf = mode_coef(p_amp, p_phase);
-        if (args.coef_out && b == 0 && seg == 0 && qn == 0 && m < args.M)
-            args.coef_out[pm] = make_float4(lam.x, lam.y, cf.x, cf.y);
-        float2 pw = lambda_pow(ga, om, (float)(16 * qn));
-        uint8_t *au = smem + kOffAu + au_slot(c) * kAuStride + (m / 4) * 128 + ((2 * m) % 8) * 2;
-        uint32_t wre[8], wim[8];
-        float kv[16];
+        asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
+        const int c = ptid >> 6, q8 = lane >> 2;
+        const int mb = 4 * ((ptid >> 5) & 1) + (lane & 3);
+        float kv[8];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
-            const int n = 16 * qn + e;
-            kv[e] = cf.x * pw.x - cf.y * pw.y;                          // Re(c lambda^n)
-            const float2 nx = cmul(pw, lam);                             // lambda^(n+1)
-            if ((e & 1) == 0) {
-                wre[e >> 1] = pack_bf16x2(pw.x, nx.x);
-                wim[e >> 1] = pack_bf16x2(pw.y, nx.y);
+        for (int e = 0; e < 8; ++e) kv[e] = 0.0f;
+#pragma unroll
+        for (int j = 0; j < kModes / 8; ++j) {
+            const int m = mb + 8 * j;
+            const float2 *lt = reinterpret_cast<const float2 *>(smem + kOffLtab) + (c * kModes + m) * 5;
+            const float2 lam = lt[0], cf = lt[1], l2 = lt[2], l4 = lt[3], l8 = lt[4];
+            float2 pw = (q8 & 1) ? lam : make_float2(1.0f, 0.0f);      // lambda^q8
+            if (q8 & 2) pw = cmul(pw, l2);
+            if (q8 & 4) pw = cmul(pw, l4);
+            uint8_t *au = smem + kOffAu + au_slot(c) * kAuStride + (m / 4) * 128 + (m % 4) * 4 + q8 * 16;
+            uint32_t *wt = reinterpret_cast<uint32_t *>(smem + kOffWtab) + (c * 32 + (q8 >> 1)) * kWtabStride + 2 * m;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                kv[e] = fmaf(cf.x, pw.x, fmaf(-cf.y, pw.y, kv[e]));        // += Re(c lambda^n)
+                const float2 nx = cmul(pw, lam);                             // lambda^(n+1)
+                if ((q8 & 1) == 0) {
+                    wt[4 * e * kWtabStride] = pack_bf16x2(pw.x, nx.x);
+                    wt[4 * e * kWtabStride + 1] = pack_bf16x2(pw.y, nx.y);
+                }
+                const float2 q = cmul(cf, nx);                               // c lambda^(n+1)
+                *reinterpret_cast<uint32_t *>(au + e * 512) = pack_bf16x2(q.x, -q.y);
+                pw = cmul(pw, l8);
             }
-            const float2 q = cmul(cf, nx);                               // c lambda^(n+1)
-            *reinterpret_cast<uint32_t *>(au + (n / 8) * 512 + (n % 8) * 16) = pack_bf16x2(q.x, -q.y);
-            pw = nx;
-        }
-        uint32_t *wt = reinterpret_cast<uint32_t *>(smem + kOffWtab) + (c * 32 + 8 * qn) * kWtabStride + 2 * m;
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            wt[k * kWtabStride] = wre[k];
-            wt[k * kWtabStride + 1] = wim[k];
         }
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
+        for (int e = 0; e < 8; ++e) {
             float v = kv[e];
-            v += __shfl_xor_sync(0xffffffffu, v, 4);
-            v += __shfl_xor_sync(0xffffffffu, v, 8);
-            v += __shfl_xor_sync(0xffffffffu, v, 16);
+            v += __shfl_xor_sync(0xffffffffu, v, 1);
+            v += __shfl_xor_sync(0xffffffffu, v, 2);
             kv[e] = v;
         }
-        if ((lane >> 2) == 0) {
-            float *kp = reinterpret_cast<float *>(smem + kOffKp) + ((m >> 3) * 8 + c) * 64 + 16 * qn;
+        if ((lane & 3) == 0) {
+            float *kp = reinterpret_cast<float *>(smem + kOffKp) + (((ptid >> 5) & 1) * 8 + c) * 64 + q8;
 #pragma unroll
-            for (int e = 0; e < 16; ++e) kp[e] = kv[e];
+            for (int e = 0; e < 8; ++e) kp[8 * e] = kv[e];
         }
     }
     if (builder) asm volatile("bar.sync %0, %1;" ::"n"(kPrologueBarrier), "n"(kPrologueThreads) : "memory");
