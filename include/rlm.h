@@ -119,10 +119,15 @@ typedef struct {
  *   state_out  nullable; if given (state_out->B == B, D, M matching), receives
  *              the prompt's terminal state s_{L-1} = sum_j lambda^{L-1-j} x_j
  *              (Sec. 3.2) and the mode coefficients, ready for decode.
- * BF16 I/O with M == 16 runs on the tcgen05 tensor-core prefill; BF16 I/O with
- * another M <= 32 on the tcgen05 reverse-time scan of the reversed drive; other
- * cases (fp32 I/O, M > 32) on the SIMT chunked scan.  All accumulate the state in
- * fp32. */
+ * Paths (all accumulate the state in fp32):
+ *  - BF16, M <= 16: the tcgen05 tensor-core prefill (modes past M padded);
+ *  - BF16, 16 < M <= 32: its 32-mode instance, one launch, where the shape needs
+ *    no sequence segments (B * D / 8 of at least about the SM count); else the
+ *    tcgen05 reverse-time scan of the reversed drive;
+ *  - BF16, 32 < M <= 64 without segments: passes of 16 modes, each adding to y;
+ *  - FP32, M <= 16, zero initial state: the tensor-core prefill with each
+ *    product split into bf16 high and low parts (three MMAs);
+ *  - other cases: the SIMT chunked scan. */
 RLM_API rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor *y,
                            rlm_state *state_out, const rlm_launch *launch);
 

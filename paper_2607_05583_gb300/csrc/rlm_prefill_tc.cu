@@ -57,7 +57,7 @@
 //          32 (q % 2) + lane of chunks 16h .. 16h+15 for the four channels whose
 //          Toeplitz rows live in quarter q, into 8-byte halves of the y rows.
 //   8-11   scan: the warp of quarter q carries channels 2q and 2q+1.
-//   12-15  transposers (boxes k = t mod 4); 16 TMA producer; 17 TMA store
+//   12-15  transposers (ring slot s: warp 12 + s mod 4); 16 TMA producer; 17 TMA store
 //          issuer and TMEM allocation.
 //   18-25  MMA issue for one channel each -- a tcgen05.mma occupies its issuing
 //          thread for ~100 cycles, so eight issuing threads keep the pipe fed.
@@ -98,80 +98,91 @@ constexpr int kC = 64;                 // chunk length
 constexpr int kNT = 32;                // chunks per tile = MMA N
 constexpr int kTile = kC * kNT;        // 2048 tokens
 constexpr int kDG = 8;                 // channels per CTA
-constexpr int kModes = 16;             // modes per channel in the kernel's tables (M <= 16 is padded)
 constexpr int kBox = 256;              // TMA box rows
 constexpr int kBoxes = kTile / kBox;   // 8 per tile
-constexpr int kXSlots = 15;            // x ring depth (boxes)
 constexpr int kYRows = 512;            // rows per y ring slot (8 chunks)
 constexpr int kYPerTile = kTile / kYRows;  // 4 slots per tile
-constexpr int kYSlots = 6;             // y ring depth
 constexpr int kWarps = 26;
 constexpr int kThreads = kWarps * 32;
 constexpr int kTmemCols = 512;
 constexpr int kTmemA = 256;            // first TMEM column of the A operands
 constexpr int kTransposers = 4;
-
-// Shared memory map (bytes from a 1024-aligned base).
-// U tables: 64 rows x 64 B per channel, in the order of channels 4-7, 0-3.  The
-// up-projection reads a 128-row A operand whose 64 real rows must meet the
-// channel's Toeplitz lanes: rows 0-63 for channels 4-7 (start at the table),
-// rows 64-127 for channels 0-3 (start one table earlier).  The other 64 rows read
-// a neighbouring table and land in state/zero lanes nobody reads afterwards.
-constexpr int kAuStride = 4096;
 constexpr int kBxStride = 4096 + 16;   // 32 rows x 128 B, +16 so stmatrix rows hit distinct banks
 constexpr int kBxBuf = kDG * kBxStride;
 // Carried-state operand: LBO 144 (not 128) spreads one chunk's 16 mode words
 // over distinct banks; the channel stride is 16 banks (mod 32) so the two
 // channels of a scan warp write disjoint banks as well.
-constexpr int kBsLbo = 144, kBsSbo = 576, kBsStride = 4 * kBsSbo + 64;
-static_assert((kBsStride / 4) % 32 == 16, "paired channels must use disjoint banks");
-constexpr int kOffAu = 0;
-constexpr int kOffBx = kOffAu + kDG * kAuStride;             // 32768
-constexpr int kOffBs = kOffBx + 2 * kBxBuf;                  // 98560
-constexpr int kOffX = kOffBs + kDG * kBsStride;              // 117504
-constexpr int kOffY = kOffX + kXSlots * kBox * 16;
-constexpr int kOffBar = kOffY + kYSlots * kYRows * 16;
-constexpr int kNumBars = 128;
-constexpr int kOffMisc = kOffBar + kNumBars * 8;
-constexpr int kSmemBytes = kOffMisc + 64 + 1024;             // + alignment slack
-static_assert(kOffX % 128 == 0 && kOffY % 128 == 0, "TMA buffers need 128-byte alignment");
-static_assert(kSmemBytes <= 232448, "shared memory budget");
+constexpr int kBsLbo = 144;
 // Prologue tables, in buffers no other role touches before the prologue ends
-// (the transposers already fill the B operand meanwhile):
-// The tables are laid out for conflict-free reads when lane R of a warp fetches
-// word k of row R: the W table is word-major with rows innermost (stride 33
-// words), and the second Toeplitz pair table starts 80 words (16 banks) after the
-// first.
+// (the transposers already fill the B operand meanwhile).  They are laid out for
+// conflict-free reads when lane R of a warp fetches word k of row R: the W table
+// is word-major with rows innermost (stride 33 words), and the second Toeplitz
+// pair table starts 80 words (16 banks) after the first.
 constexpr int kWtabStride = 33;
-constexpr int kTpairStride = 144;                      // words per channel: P0 at 0, P1 at 80
-constexpr int kOffWtab = kOffY;                        // [8 ch][32 words][33]: W rows, packed bf16 pairs
-constexpr int kOffTpair = kOffBs;                      // [8 ch][144 words]: Toeplitz pairs
-constexpr int kOffKp = kOffTpair + 8 * kTpairStride * 4;  // [2 halves][8 ch][64] fp32 partial sums of K
-static_assert(8 * 32 * kWtabStride * 4 <= kYSlots * kYRows * 16, "W table does not fit the y ring");
-// [8 ch][kModes][5] float2: lambda, c, lambda^2, lambda^4, lambda^8 of each mode.
-constexpr int kOffLtab = kOffKp + 2 * 8 * 64 * 4;
-static_assert(kOffLtab + 8 * 16 * 5 * 8 <= kOffX, "prologue tables do not fit");
+constexpr int kTpairStride = 144;      // words per channel: P0 at 0, P1 at 80
 // Named barriers: the 16 warps that build the constants (0-11 and 18-21); the
 // CTA's set-up, which the TMA producer warp only arrives at.
 constexpr int kPrologueBarrier = 1;
 constexpr int kPrologueThreads = 512;
 constexpr int kSetupBarrier = 2;
 
-// Barrier indices.
-constexpr int kBarXFull = 0;                    // [kXSlots]
-constexpr int kBarXEmpty = kXSlots;             // [kXSlots]
-constexpr int kBarBxFull = 2 * kXSlots;         // [2]
-constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]: released by the 8 MMA threads
-constexpr int kBarTwDone = kBarBxEmpty + 2;     // [8]: Toeplitz/state MMAs of a channel done
-constexpr int kBarSFull = kBarTwDone + 8;       // [8]: carried states of a channel written
-constexpr int kBarUDone = kBarSFull + 8;        // [8]: up-projection of a channel done
-constexpr int kBarDEmpty = kBarUDone + 8;       // [8]: accumulator of a channel read out
-constexpr int kBarYFull = kBarDEmpty + 8;       // [kYSlots]
-constexpr int kBarYEmpty = kBarYFull + kYSlots; // [kYSlots]
-constexpr int kBarFinal = kBarYEmpty + kYSlots; // [8]
-constexpr int kBarConsts = kBarFinal + 8;       // the A operands and U tables are built
-constexpr int kBarGFull = kBarConsts + 1;       // [kYSlots] mixer: the gate rows of a z slot landed
-static_assert(kBarGFull + kYSlots <= kNumBars, "too many barriers");
+// Layout of one kernel instance: kModes = 16 or 32 modes per channel in its
+// tables (fewer are padded).  With 32 modes the A operand's fourth TMEM quarter
+// holds the state rows of modes 16-31, the U tables and the carried-state
+// operand double, and the x and y rings shrink to fit shared memory.
+template <int kModes>
+struct Cfg {
+    static_assert(kModes == 16 || kModes == 32, "16 or 32 modes per instance");
+    static constexpr int kXSlots = kModes == 16 ? 15 : 7;   // x ring depth (boxes)
+    static constexpr int kYSlots = kModes == 16 ? 6 : 4;    // y ring depth
+    // U tables: 64 rows x 2 kModes bf16 per channel (K-major core matrices: 8 rows
+    // x 16 B, K groups 128 B apart, row groups kAuSbo apart), in the order of
+    // channels 4-7, 0-3.  The up-projection reads a 128-row A operand whose 64
+    // real rows must meet the channel's Toeplitz lanes: rows 0-63 for channels
+    // 4-7 (start at the table), rows 64-127 for channels 0-3 (start one table
+    // earlier).  The other 64 rows read a neighbouring table and land in state
+    // lanes nobody reads afterwards.
+    static constexpr int kAuSbo = 32 * kModes;
+    static constexpr int kAuStride = 8 * kAuSbo;
+    static constexpr int kBsSbo = (kModes / 4) * kBsLbo;
+    static constexpr int kBsStride = 4 * kBsSbo + 64;
+    static_assert((kBsStride / 4) % 32 == 16, "paired channels must use disjoint banks");
+    static constexpr int kOffAu = 0;
+    static constexpr int kOffBx = kOffAu + kDG * kAuStride;
+    static constexpr int kOffBs = kOffBx + 2 * kBxBuf;
+    static constexpr int kOffX = kOffBs + kDG * kBsStride;
+    static constexpr int kOffY = kOffX + kXSlots * kBox * 16;
+    static constexpr int kOffBar = kOffY + kYSlots * kYRows * 16;
+    static constexpr int kNumBars = 96;
+    static constexpr int kOffMisc = kOffBar + kNumBars * 8;
+    static constexpr int kSmemBytes = kOffMisc + 64 + 1024;        // + alignment slack
+    static_assert(kOffX % 128 == 0 && kOffY % 128 == 0, "TMA buffers need 128-byte alignment");
+    static_assert(kSmemBytes <= 232448, "shared memory budget");
+    // Prologue tables.  The W table (16 modes only; with 32 the W rows are formed
+    // in registers) lives in the y ring, the others in the carried-state buffers.
+    static constexpr int kOffWtab = kOffY;                          // [8 ch][32 words][33]
+    static constexpr int kOffTpair = kOffBs;                        // [8 ch][144 words]: Toeplitz pairs
+    static constexpr int kOffKp = kOffTpair + 8 * kTpairStride * 4; // [2 halves][8 ch][64] fp32 partial sums of K
+    // [8 ch][kModes][5] float2: lambda, c, lambda^2, lambda^4, lambda^8 of each mode.
+    static constexpr int kOffLtab = kOffKp + 2 * 8 * 64 * 4;
+    static_assert(kModes != 16 || 8 * 32 * kWtabStride * 4 <= kYSlots * kYRows * 16, "W table does not fit the y ring");
+    static_assert(kOffLtab + 8 * kModes * 5 * 8 <= kOffX, "prologue tables do not fit");
+    // Barrier indices.
+    static constexpr int kBarXFull = 0;                    // [kXSlots]
+    static constexpr int kBarXEmpty = kXSlots;             // [kXSlots]
+    static constexpr int kBarBxFull = 2 * kXSlots;         // [2]
+    static constexpr int kBarBxEmpty = kBarBxFull + 2;     // [2]: released by the 8 MMA threads
+    static constexpr int kBarTwDone = kBarBxEmpty + 2;     // [8]: Toeplitz/state MMAs of a channel done
+    static constexpr int kBarSFull = kBarTwDone + 8;       // [8]: carried states of a channel written
+    static constexpr int kBarUDone = kBarSFull + 8;        // [8]: up-projection of a channel done
+    static constexpr int kBarDEmpty = kBarUDone + 8;       // [8]: accumulator of a channel read out
+    static constexpr int kBarYFull = kBarDEmpty + 8;       // [kYSlots]
+    static constexpr int kBarYEmpty = kBarYFull + kYSlots; // [kYSlots]
+    static constexpr int kBarFinal = kBarYEmpty + kYSlots; // [8]
+    static constexpr int kBarConsts = kBarFinal + 8;       // the A operands and U tables are built
+    static constexpr int kBarGFull = kBarConsts + 1;       // [kYSlots] mixer: the gate rows of a z slot landed
+    static_assert(kBarGFull + kYSlots <= kNumBars, "too many barriers");
+};
 
 
 
@@ -359,7 +370,7 @@ constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(kNT
 
 __device__ __forceinline__ int au_slot(int c) { return (c + 4) & 7; }
 // First byte (from the U table area) of channel c's 128-row up-projection operand.
-__device__ __forceinline__ int au_operand(int c) { return au_slot(c) * kAuStride - (c < 4 ? kAuStride : 0); }
+__device__ __forceinline__ int au_operand(int c, int stride) { return au_slot(c) * stride - (c < 4 ? stride : 0); }
 
 struct TcArgs {
     const float *decay, *freq, *amp, *phase;
@@ -369,7 +380,7 @@ struct TcArgs {
     __nv_bfloat16 *y;    // for the plain stores of boxes that start before t = 0
     int64_t L;
     int D;
-    int M;               // modes of this pass, 1..16; modes M..15 are padding (amplitude 0, never stored)
+    int M;               // modes of this pass, 1..kModes; modes M.. are padding (amplitude 0, never stored)
     int m0, Mt;          // first mode of this pass; modes per channel in the parameter/state layouts
     int add;             // kMix: the slot holds y so far (earlier passes); z = that + this pass's y
                          // (otherwise the slot holds the gate: z = sigma(g) y)
@@ -404,13 +415,26 @@ struct TcArgs {
 // with z.
 enum : int { kPlain = 0, kSegmented = 1, kPacked = 2 };
 
-template <int kMode, bool kInj, bool kMix>
+// kModes: 16, or 32 (kPlain and kPacked without the mixer field only).
+template <int kMode, bool kInj, bool kMix, int kModes>
 __global__ void __launch_bounds__(kThreads, 1)
     k_prefill_tc(const __grid_constant__ CUtensorMap tmap_x,
                  const __grid_constant__ CUtensorMap tmap_y, const __grid_constant__ CUtensorMap tmap_g,
                  const TcArgs args) {
     constexpr bool kSeg = kMode == kSegmented, kPack = kMode == kPacked;
     static_assert(!(kSeg && kMix), "the mixer epilogue is not built for segmented launches");
+    static_assert(kModes == 16 || (!kSeg && !kMix), "32 modes: plain or packed launches without a second field");
+    using Cf = Cfg<kModes>;
+    constexpr int kXSlots = Cf::kXSlots, kYSlots = Cf::kYSlots, kAuStride = Cf::kAuStride, kAuSbo = Cf::kAuSbo;
+    constexpr int kBsSbo = Cf::kBsSbo, kBsStride = Cf::kBsStride;
+    constexpr int kOffAu = Cf::kOffAu, kOffBx = Cf::kOffBx, kOffBs = Cf::kOffBs, kOffX = Cf::kOffX, kOffY = Cf::kOffY;
+    constexpr int kOffBar = Cf::kOffBar, kOffMisc = Cf::kOffMisc, kOffWtab = Cf::kOffWtab, kOffTpair = Cf::kOffTpair;
+    constexpr int kOffKp = Cf::kOffKp, kOffLtab = Cf::kOffLtab;
+    constexpr int kBarXFull = Cf::kBarXFull, kBarXEmpty = Cf::kBarXEmpty, kBarBxFull = Cf::kBarBxFull;
+    constexpr int kBarBxEmpty = Cf::kBarBxEmpty, kBarTwDone = Cf::kBarTwDone, kBarSFull = Cf::kBarSFull;
+    constexpr int kBarUDone = Cf::kBarUDone, kBarDEmpty = Cf::kBarDEmpty, kBarYFull = Cf::kBarYFull;
+    constexpr int kBarYEmpty = Cf::kBarYEmpty, kBarFinal = Cf::kBarFinal, kBarConsts = Cf::kBarConsts;
+    constexpr int kBarGFull = Cf::kBarGFull;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // Align with pointer arithmetic on the __shared__ array (not through an
     // integer), so the compiler keeps the shared address space and emits
@@ -441,8 +465,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const bool builder = warp < 12 || (warp >= 18 && warp < 22);
     const int pq = warp & 3, pe = warp < 12 ? warp >> 2 : 3;
     const int ptid = (pe * 4 + pq) * 32 + lane;
-    const bool lpow = builder && ptid < 128;
-    const int l_c = ptid >> 4, l_m = ptid & 15;
+    const bool lpow = builder && ptid < 8 * kModes;
+    const int l_c = ptid / kModes, l_m = ptid % kModes;
     float p_decay = 0.0f, p_freq = 0.0f, p_amp = 0.0f, p_phase = 0.0f;
     if (lpow && l_m < args.M) {
         const int pm = (d0 + l_c) * args.Mt + args.m0 + l_m;
@@ -494,7 +518,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             for (int i = 0; i < kDG; ++i) {
                 bar_init(bar(kBarTwDone + i), 1);
-                bar_init(bar(kBarSFull + i), 1);
+                bar_init(bar(kBarSFull + i), kModes / 16);   // with 32 modes: two scan warps
                 bar_init(bar(kBarUDone + i), 1);
                 bar_init(bar(kBarDEmpty + i), 4);
                 bar_init(bar(kBarFinal + i), 1);
@@ -575,12 +599,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int e = 0; e < 8; ++e) {
                 kv[e] = fmaf(cf.x, pw.x, fmaf(-cf.y, pw.y, kv[e]));        // += Re(c lambda^n)
                 const float2 nx = cmul(pw, lam);                             // lambda^(n+1)
-                if ((q8 & 1) == 0) {
+                if (kModes == 16 && (q8 & 1) == 0) {
                     wt[4 * e * kWtabStride] = pack_bf16x2(pw.x, nx.x);
                     wt[4 * e * kWtabStride + 1] = pack_bf16x2(pw.y, nx.y);
                 }
                 const float2 q = cmul(cf, nx);                               // c lambda^(n+1)
-                *reinterpret_cast<uint32_t *>(au + e * 512) = pack_bf16x2(q.x, -q.y);
+                *reinterpret_cast<uint32_t *>(au + e * kAuSbo) = pack_bf16x2(q.x, -q.y);
                 pw = cmul(pw, l8);
             }
         }
@@ -618,7 +642,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     //     position p = 32 (q % 2) + lane;
     //   quarter c / 2:     W[k][p'] = (Re, Im) lambda_m^p' for state row k = lane
     //     (k = 2m + ri);
-    //   the remaining quarter: zero.
+    //   the remaining quarter, (c / 2) ^ 1: zero, or with 32 modes the W rows of
+    //     modes 16-31 (row k = lane for mode 16 + k / 2).
+    // With 32 modes the W rows are formed here, by the recurrence lambda^(p'+1) =
+    // lambda^p' lambda from the per-mode table (the 16-mode instance reads the W
+    // table written in stage 1).
     if (builder) {
         const int q = pq, e = pe;
         for (int cc = 0; cc < 2; ++cc) {
@@ -630,10 +658,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                                      ((pos & 1) ? 80 + (pos >> 1) : (pos >> 1));
 #pragma unroll
                 for (int k = 0; k < 32; ++k) w[k] = tp[k];
-            } else if (q == (c >> 1)) {
+            } else if (kModes == 16 && q == (c >> 1)) {
                 const uint32_t *wt = reinterpret_cast<const uint32_t *>(smem + kOffWtab) + c * 32 * kWtabStride + lane;
 #pragma unroll
                 for (int k = 0; k < 32; ++k) w[k] = wt[k * kWtabStride];
+            } else if (kModes == 32) {
+                const int m = (lane >> 1) + (q == (c >> 1) ? 0 : 16), ri = lane & 1;
+                const float2 lam = reinterpret_cast<const float2 *>(smem + kOffLtab)[(c * kModes + m) * 5];
+                float2 pw = make_float2(1.0f, 0.0f);
+#pragma unroll
+                for (int k = 0; k < 32; ++k) {
+                    const float2 nx = cmul(pw, lam);
+                    w[k] = ri ? pack_bf16x2(pw.y, nx.y) : pack_bf16x2(pw.x, nx.x);
+                    pw = cmul(nx, lam);
+                }
             } else {
 #pragma unroll
                 for (int k = 0; k < 32; ++k) w[k] = 0u;
@@ -673,8 +711,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         __syncwarp();
     } else if (warp >= 12 && warp < 12 + kTransposers) {
-        // ---------------------------------------------------- transposers (boxes k = t mod 4)
-        for (int k = warp - 12; k < total_boxes; k += kTransposers) {
+        // ---------------------------------------------------- transposers (ring slot s: warp 12 + s mod 4)
+        // Each ring slot belongs to one transposer warp (slot s to warp s mod 4), so
+        // a warp waits on a slot's full barrier only after it has itself consumed
+        // the slot's previous box.  With boxes dealt round-robin instead, a warp
+        // could wait for box k while box k - kXSlots (consumed by another warp) had
+        // not landed yet; its parity wait then matched the phase of box k - 2 kXSlots
+        // and passed at once (intermittent wrong tiles and launch failures with the
+        // 7-slot ring of the 32-mode instance).
+        const int tw = warp - 12;
+        for (int k = tw; k < total_boxes;) {
+            const int kn = (k % kXSlots) + kTransposers < kXSlots ? k + kTransposers
+                                                                 : k - (k % kXSlots) + kXSlots + tw;
             const int j = k / kBoxes, tq = k % kBoxes;
             const int buf = j & 1, use = j >> 1;
             const uint32_t slot = k % kXSlots;
@@ -710,6 +758,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 bar_arrive(bar(kBarXEmpty + slot));
                 bar_arrive(bar(kBarBxFull + buf));
             }
+            k = kn;
         }
     } else if (warp == 17) {
         // ---------------------------------------------------- y store issuer
@@ -787,7 +836,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // (after a state-only pass, until the scan has read it).
         const int c = warp - 18;
         const uint64_t dx0 = umma_desc(sbase + kOffBx + c * kBxStride, 128, 1024);
-        const uint64_t du0 = umma_desc(sbase + kOffAu + au_operand(c), 128, 512);
+        const uint64_t du0 = umma_desc(sbase + kOffAu + au_operand(c, kAuStride), 128, kAuSbo);
         const uint64_t ds0 = umma_desc(sbase + kOffBs + c * kBsStride, kBsLbo, kBsSbo);
         const uint32_t aT = tmem + kTmemA + c * 32;
         const uint32_t d = tmem + c * kNT;
@@ -811,7 +860,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 bar_arrive(bar(kBarBxEmpty + buf));
                 if (v < nA) continue;  // state-only pass: no output
 #pragma unroll
-                for (int kk = 0; kk < 2; ++kk) umma_ss(d, du0 + kk * 16, ds0 + kk * ((2 * kBsLbo) >> 4), kIdesc, 1);
+                for (int kk = 0; kk < kModes / 8; ++kk)
+                    umma_ss(d, du0 + kk * 16, ds0 + kk * ((2 * kBsLbo) >> 4), kIdesc, 1);
                 umma_commit(bar(kBarUDone + c));
             }
             // Drain: all MMAs this thread issued complete before TMEM is released.
@@ -823,6 +873,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
     } else if (warp >= 8 && warp < 12) {
         // ---------------------------------------------------- scan, two channels
+        if constexpr (kModes == 16) {
         // The warp of quarter q owns channels 2q and 2q+1, whose state rows are
         // its TMEM lanes.  Lane 2m carries mode m of the first channel, lane 2m+1
         // mode m of the second: each lane reads row 2m+ri of both channels and one
@@ -915,6 +966,96 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         for (int v = nA; v < nV && ok; ++v) ok = scan_tile(v);
+        } else {
+        // With 32 modes quarter q holds the state rows of modes 0-15 of channels
+        // 2q, 2q+1 and of modes 16-31 of channels 2 (q ^ 1), 2 (q ^ 1) + 1, so each
+        // channel's carried states come from two scan warps (SFull counts two).
+        // Both warps of a quarter pair {q, q ^ 1} scan the channel pair of the even
+        // quarter first and that of the odd quarter second, each as one chain of
+        // 32 chunks like the 16-mode scan, so a pair's up-projection waits only for
+        // that pair's scans.  Pass k covers channels 2 pr, 2 pr + 1 with pr =
+        // 2 (q / 2) + k, at modes mo + m (mo = 0 if pr == q, else 16); lane 2m + ri
+        // carries mode mo + m of channel 2 pr + ri.
+        const uint32_t st_lane = 32u * (uint32_t)quarter;
+        const int m = lane >> 1, ri = lane & 1;
+        int chk[2], mok[2];
+        bool realk[2];
+        float deck[2], frqk[2];
+        float2 LCk[2], Sk[2], injk[2];
+        uint32_t bsk[2];
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+            const int pr = ((quarter >> 1) << 1) + k;
+            chk[k] = 2 * pr + ri;
+            mok[k] = pr == quarter ? 0 : 16;
+            realk[k] = mok[k] + m < args.M;
+            const int pm = (d0 + chk[k]) * args.Mt + args.m0 + mok[k] + m;
+            deck[k] = realk[k] ? args.decay[pm] : 0.0f;
+            frqk[k] = realk[k] ? args.freq[pm] : 0.0f;
+            LCk[k] = lambda_pow(deck[k], frqk[k], (float)kC);
+            Sk[k] = injk[k] = make_float2(0.0f, 0.0f);
+            bsk[k] = sbase + kOffBs + chk[k] * kBsStride + ((mok[k] + m) / 4) * kBsLbo + (m % 4) * 4;
+        }
+        const int n0 = kInj ? (int)((-args.t0) >> 6) : -1;
+        auto load_inj = [&](int row) {
+            const float p = (float)(-(int)((-args.t0) & 63));
+#pragma unroll
+            for (int k = 0; k < 2; ++k)
+                injk[k] = realk[k] ? cmul(lambda_pow(deck[k], frqk[k], p),
+                                          args.state_in[((int64_t)row * D + d0 + chk[k]) * args.Mt + args.m0 + mok[k] + m])
+                                   : make_float2(0.0f, 0.0f);
+        };
+        if (kInj && !kPack) load_inj(b);
+        bool ok = true;
+        for (int v = 0; v < nV && ok; ++v) {
+            const bool row_start = real_tile(v) == 0;
+            const bool inj_tile = kInj && row_start;
+            if (kPack && row_start) {
+                Sk[0] = Sk[1] = make_float2(0.0f, 0.0f);
+                if (kInj) load_inj(row_of(v));
+            }
+#pragma unroll
+            for (int k = 0; k < 2; ++k) {
+                const int cA = 2 * (((quarter >> 1) << 1) + k), cB = cA + 1;
+                if (!wait_bar(bar(kBarTwDone + cA), v & 1, abort_flag) ||
+                    !wait_bar(bar(kBarTwDone + cB), v & 1, abort_flag)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                float2 S = Sk[k];
+#pragma unroll
+                for (int h = 0; h < kNT / 16; ++h) {
+                    uint32_t va[16], vb[16];
+                    tmem_ld16(tmem + (st_lane << 16) + cA * kNT + 16 * h, va);
+                    tmem_ld16(tmem + (st_lane << 16) + cB * kNT + 16 * h, vb);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int n = 0; n < 16; ++n) {
+                        const float a = __uint_as_float(va[n]), bb = __uint_as_float(vb[n]);
+                        const float recv = __shfl_xor_sync(0xffffffffu, ri ? a : bb, 1);
+                        const float2 Ln = ri ? make_float2(recv, bb) : make_float2(a, recv);
+                        const int nn = 16 * h + n;
+                        if (kInj && inj_tile && nn == n0) S = make_float2(S.x + injk[k].x, S.y + injk[k].y);
+                        asm volatile("st.shared.b32 [%0], %1;" ::"r"(bsk[k] + (nn >> 3) * kBsSbo + (nn & 7) * 16),
+                                     "r"(pack_bf16x2(S.x, S.y))
+                                     : "memory");
+                        S = cfma(LCk[k], S, Ln);
+                    }
+                }
+                Sk[k] = S;
+                if ((kPack ? real_tile(v) == args.ntiles - 1 : v == nV - 1) && args.state_out && realk[k])
+                    args.state_out[((int64_t)row_of(v) * D + d0 + chk[k]) * args.Mt + args.m0 + mok[k] + m] = S;
+                fence_async_smem();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) {
+                    bar_arrive(bar(kBarSFull + cA));
+                    bar_arrive(bar(kBarSFull + cB));
+                }
+            }
+        }
+        }
     } else if (warp < 8) {
         // ---------------------------------------------------- epilogue
         // Warp (quarter q, h) reads its quarter's Toeplitz lanes -- position
@@ -1074,6 +1215,10 @@ bool make_field_map(CUtensorMap *map, const void *ptr, int64_t B, int64_t L, int
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Modes per channel of the segmented and mixer instances (their tables and the
+// segment-state layout); plain and packed launches also come with 32.
+constexpr int kModes16 = 16;
+
 // Sequence segments: with fewer (batch row, channel group) CTAs than SMs, the
 // sequence is cut into nseg runs of whole tiles so that nseg * B * D / 8 CTAs
 // (at most one per SM, all resident at once) share the work.
@@ -1094,7 +1239,7 @@ Segments segments(int64_t B, int64_t L, int D) {
 }
 
 size_t seg_state_bytes(int64_t B, int nseg, int D) {
-    return ((size_t)B * nseg * D * kModes * sizeof(float2) + 255) / 256 * 256;
+    return ((size_t)B * nseg * D * kModes16 * sizeof(float2) + 255) / 256 * 256;
 }
 
 }  // namespace
@@ -1103,14 +1248,15 @@ bool tc_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
     const bool shape = dt == RLM_BF16 && M >= 1 && D % kDG == 0 && B >= 1 && B <= 65535 && L >= 1 &&
                        L <= ((int64_t)1 << 31) - kTile && D / kDG <= 65535;
     if (!shape) return false;
-    if (M <= kModes) return true;
-    // More modes: passes of 16 modes, each later one adding to the output of the
-    // earlier ones through the z ring (unsegmented launches only).
-    return M <= 4 * kModes && segments(B, L, D).nseg < 2;
+    if (M <= kModes16) return true;
+    // More modes (unsegmented launches only): up to 32 in one launch of the
+    // 32-mode instance; beyond, passes of 16 modes, each later one adding to the
+    // output of the earlier ones through the z ring.
+    return M <= 4 * kModes16 && segments(B, L, D).nseg < 2;
 }
 
 bool tc_mixer_fused(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
-    return M <= kModes && tc_prefill_supported(B, L, D, M, dt) && segments(B, L, D).nseg < 2;
+    return M <= kModes16 && tc_prefill_supported(B, L, D, M, dt) && segments(B, L, D).nseg < 2;
 }
 
 size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int) {
@@ -1122,16 +1268,27 @@ size_t tc_prefill_ws_bytes(int64_t B, int64_t L, int D, int) {
 template <int kMode>
 void launch_unsegmented(bool field, bool inj, dim3 grid, const CUtensorMap &mx, const CUtensorMap &my,
                         const CUtensorMap &m2, const TcArgs &a, cudaStream_t st) {
+    constexpr int sm = Cfg<16>::kSmemBytes;
     if (field) {
         if (inj)
-            k_prefill_tc<kMode, true, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+            k_prefill_tc<kMode, true, true, 16><<<grid, kThreads, sm, st>>>(mx, my, m2, a);
         else
-            k_prefill_tc<kMode, false, true><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+            k_prefill_tc<kMode, false, true, 16><<<grid, kThreads, sm, st>>>(mx, my, m2, a);
     } else if (inj) {
-        k_prefill_tc<kMode, true, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+        k_prefill_tc<kMode, true, false, 16><<<grid, kThreads, sm, st>>>(mx, my, m2, a);
     } else {
-        k_prefill_tc<kMode, false, false><<<grid, kThreads, kSmemBytes, st>>>(mx, my, m2, a);
+        k_prefill_tc<kMode, false, false, 16><<<grid, kThreads, sm, st>>>(mx, my, m2, a);
     }
+}
+
+template <int kMode>
+void launch_unsegmented32(bool inj, dim3 grid, const CUtensorMap &mx, const CUtensorMap &my, const TcArgs &a,
+                          cudaStream_t st) {
+    constexpr int sm = Cfg<32>::kSmemBytes;
+    if (inj)
+        k_prefill_tc<kMode, true, false, 32><<<grid, kThreads, sm, st>>>(mx, my, mx, a);
+    else
+        k_prefill_tc<kMode, false, false, 32><<<grid, kThreads, sm, st>>>(mx, my, mx, a);
 }
 
 // Batch rows per CTA of an unsegmented launch.  One CTA per SM (shared memory
@@ -1176,20 +1333,27 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
         std::lock_guard<std::mutex> lock(mu);
         if ((int)configured.size() <= dev) configured.resize(dev + 1, 0);
         if (!configured[dev]) {
-            const void *fns[] = {reinterpret_cast<const void *>(k_prefill_tc<kPlain, false, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kSegmented, false, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, true, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kSegmented, true, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, false, true>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, true, true>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, false, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, true, false>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, false, true>),
-                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, true, true>)};
+            const void *fns[] = {reinterpret_cast<const void *>(k_prefill_tc<kPlain, false, false, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kSegmented, false, false, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, true, false, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kSegmented, true, false, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, false, true, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPlain, true, true, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, false, false, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, true, false, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, false, true, 16>),
+                                 reinterpret_cast<const void *>(k_prefill_tc<kPacked, true, true, 16>)};
+            const void *fns32[] = {reinterpret_cast<const void *>(k_prefill_tc<kPlain, false, false, 32>),
+                                   reinterpret_cast<const void *>(k_prefill_tc<kPlain, true, false, 32>),
+                                   reinterpret_cast<const void *>(k_prefill_tc<kPacked, false, false, 32>),
+                                   reinterpret_cast<const void *>(k_prefill_tc<kPacked, true, false, 32>)};
             cudaError_t e = cudaSuccess;
             for (const void *f : fns)
                 if (e == cudaSuccess)
-                    e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+                    e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<16>::kSmemBytes);
+            for (const void *f : fns32)
+                if (e == cudaSuccess)
+                    e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg<32>::kSmemBytes);
             if (e != cudaSuccess) return e;
             configured[dev] = 1;
         }
@@ -1205,7 +1369,7 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.y = static_cast<__nv_bfloat16 *>(y);
     a.L = L;
     a.D = D;
-    a.M = std::min(M, kModes);
+    a.M = std::min(M, kModes16);
     a.m0 = 0;
     a.Mt = M;
     a.add = 0;
@@ -1220,13 +1384,24 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     a.B = (int)B;
     a.bpc = sg.nseg < 2 ? rows_per_cta(B, D, a.ntiles) : 1;
     dim3 grid((unsigned)(D / kDG), (unsigned)((B + a.bpc - 1) / a.bpc), (unsigned)sg.nseg);
-    const int npass = (M + kModes - 1) / kModes;
-    if ((mix || npass > 1) && sg.nseg >= 2) return cudaErrorInvalidValue;  // callers check support
-    if (mix && npass > 1) return cudaErrorInvalidValue;
+    // 16 < M <= 32: one launch of the 32-mode instance (unsegmented, no gate).
+    const bool m32 = M > kModes16 && M <= 2 * kModes16;
+    const int npass = m32 ? 1 : (M + kModes16 - 1) / kModes16;
+    if ((mix || M > kModes16) && sg.nseg >= 2) return cudaErrorInvalidValue;  // callers check support
+    if (mix && M > kModes16) return cudaErrorInvalidValue;
+    if (m32) {
+        a.M = M;
+        if (a.bpc > 1)
+            launch_unsegmented32<kPacked>(state_in != nullptr, grid, mx, my, a, st);
+        else
+            launch_unsegmented32<kPlain>(state_in != nullptr, grid, mx, my, a, st);
+        count_launches(1);
+        return cudaGetLastError();
+    }
     if (sg.nseg < 2) {
         for (int p = 0; p < npass; ++p) {
-            a.m0 = p * kModes;
-            a.M = std::min(kModes, M - a.m0);
+            a.m0 = p * kModes16;
+            a.M = std::min(kModes16, M - a.m0);
             a.add = p > 0;
             // Later passes load the output so far into the z ring and add to it.
             const CUtensorMap &m2 = p > 0 ? my : mg;
@@ -1251,9 +1426,9 @@ cudaError_t tc_prefill(const void *x, void *y, int64_t B, int64_t L, int D, int 
     static std::atomic<unsigned long long> epoch{0x5eed0000ull};
     a.epoch = ++epoch;
     void *kargs[] = {&mx, &my, &mg, &a};
-    const void *fn = state_in ? reinterpret_cast<const void *>(k_prefill_tc<kSegmented, true, false>)
-                              : reinterpret_cast<const void *>(k_prefill_tc<kSegmented, false, false>);
-    cudaError_t e = cudaLaunchCooperativeKernel(fn, grid, dim3(kThreads), kargs, (size_t)kSmemBytes, st);
+    const void *fn = state_in ? reinterpret_cast<const void *>(k_prefill_tc<kSegmented, true, false, 16>)
+                              : reinterpret_cast<const void *>(k_prefill_tc<kSegmented, false, false, 16>);
+    cudaError_t e = cudaLaunchCooperativeKernel(fn, grid, dim3(kThreads), kargs, (size_t)Cfg<16>::kSmemBytes, st);
     count_launches(1);
     return e;
 }

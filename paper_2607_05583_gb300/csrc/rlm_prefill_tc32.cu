@@ -39,7 +39,7 @@
 //          quarter q, chunks 16h .. 16h+15, into the 8-byte half of each 16-byte
 //          y row.
 //   8-11   scan: the warp of quarter q carries channel q.
-//   12-15  transposers (boxes k = t mod 4): fp32 token rows -> hi / lo K-major
+//   12-15  transposers (ring slot s: warp 12 + s mod 4): fp32 token rows -> hi / lo K-major
 //          B operands.
 //   16     TMA producer; 17 TMA store issuer and TMEM allocation.
 //   18-21  MMA issue for one channel each: the thread polls the inputs of the
@@ -549,7 +549,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         __syncwarp();
     } else if (warp >= 12 && warp < 12 + kTransposers) {
-        // ---------------------------------------------------- transposers (boxes k = t mod 4)
+        // ---------------------------------------------------- transposers (ring slot s: warp 12 + s mod 4)
         // Per 8-token block (one K group of one chunk): ldmatrix.trans of the 8
         // token rows (in reversed order, so positions come out as p' = 63 - p)
         // gives thread t the half-word k = t / 4 (half k % 2 of channel k / 2) of
@@ -558,7 +558,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         // of its channel's two positions, the thread of the odd half the low
         // parts: exactly row k of an 8 x 8 matrix whose rows are (channel, part),
         // which stmatrix writes into the 8 B operands (4 channels x hi, lo).
-        for (int k = warp - 12; k < total_boxes; k += kTransposers) {
+        // Each ring slot belongs to one transposer warp, so a warp waits on a slot's
+        // full barrier only after it has itself consumed the slot's previous box (a
+        // parity wait must never be two phases ahead of the barrier).
+        const int tw = warp - 12;
+        for (int k = tw; k < total_boxes;) {
+            const int kn = (k % kXSlots) + kTransposers < kXSlots ? k + kTransposers
+                                                                 : k - (k % kXSlots) + kXSlots + tw;
             const int j = k / kBoxes, tq = k % kBoxes;
             const int buf = j & 1, use = j >> 1;
             const uint32_t slot = k % kXSlots;
@@ -610,6 +616,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 bar_arrive(bar(kBarXEmpty + slot));
                 bar_arrive(bar(kBarBxFull + buf));
             }
+            k = kn;
         }
     } else if (warp == 17) {
         // ---------------------------------------------------- y store issuer

@@ -234,10 +234,11 @@ def test_tcgen05_shape_mixer_prefill_matches_oracle(B, L, D, K, with_g, with_his
     _check_prefill(inp, mx, z, so, cout, with_g, with_hist)
 
 
-@pytest.mark.parametrize("M,K", [(32, 4), (24, 0)])
+@pytest.mark.parametrize("M,K", [(32, 4), (24, 0), (40, 4)])
 def test_multi_pass_mixer_prefill_matches_oracle(M, K):
-    """M > 16 on an unsegmented shape: the prefill in passes of 16 modes, then the
-    mixer pass (the gate is not fused with several passes)."""
+    """M > 16 on an unsegmented shape: the prefill (one launch of the 32-mode
+    instance for M <= 32, else passes of 16 modes), then the mixer pass (the gate
+    is not fused with more than 16 modes)."""
     inp = make_inputs(2, 3000, 512, M, "bf16", seed=M + K)
     mx = make_mixer_inputs(inp, K, seed=M)
     out = {}
@@ -246,7 +247,8 @@ def test_multi_pass_mixer_prefill_matches_oracle(M, K):
         out["r"] = _run_prefill(inp, mx, True, K > 0)
 
     n = _launches(run)
-    assert n == 2 + 1 + (1 if K >= 2 else 0), n
+    passes = 1 if M <= 32 else (M + 15) // 16
+    assert n == passes + 1 + (1 if K >= 2 else 0), n
     z, so, cout = out["r"]
     _check_prefill(inp, mx, z, so, cout, True, K > 0)
 

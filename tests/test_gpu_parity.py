@@ -76,7 +76,9 @@ def test_prefill_layer6m_bf16():
     (9, 704, 256, 7, True, True),             # three rows per CTA, padded modes, an initial state
     (3, 2048 * 2 + 64, 2048, 16, True, True), # more channel groups than SMs: three rows per CTA, ragged tile
     (3, 2048 * 2 + 77, 2048, 16, True, False), # L not a multiple of 64 with a state: the SIMT scan
-    (5, 2048 + 3, 512, 32, False, False),     # two mode passes, rows in CTAs of three (a partial last one)
+    (5, 2048 + 3, 512, 32, False, False),     # 32 modes in one launch, rows in CTAs of three (a partial last one)
+    (6, 2048 * 2 + 64, 1024, 24, True, True), # 32-mode instance: modes 24-31 padded, an initial state
+    (9, 704, 512, 32, False, True),           # 32-mode instance, one tile per row
 ])
 def test_packed_rows_prefill(B, L, D, M, with_state_in, bitwise):
     """Where the (batch row, channel group) CTAs would take more than one wave, a
@@ -126,6 +128,10 @@ def test_packed_rows_prefill(B, L, D, M, with_state_in, bitwise):
     # shorter than a chunk, one token past a tile, D not a multiple of 64
     (1, 1, 8, 17, "bf16"), (2, 65, 16, 32, "bf16"), (1, 2100, 8, 31, "bf16"),
     (2, 2048 * 2 + 7, 24, 20, "bf16"),
+    # bf16 with 16 < M <= 32 on unsegmented shapes: the 32-mode tcgen05 instance
+    # (several tiles and a ragged first tile; 17 modes; a packed launch)
+    (4, 2048 * 2 + 100, 160, 20, "bf16"), (1, 2048 + 1, 1024, 17, "bf16"),
+    (2, 3 * 2048 + 17, 640, 32, "bf16"),
     # bf16 with M > 32: the SIMT path
     (1, 500, 8, 40, "bf16"),
 ])
@@ -204,6 +210,8 @@ def _state_from(inp, s_np):
     (4, 3001, 256, 1, "bf16"),            # ... one mode per channel, unsegmented
     (2, 1000, 16, 7, "f32"),              # SIMT
     (1, 500, 8, 40, "bf16"),              # SIMT, bf16 with M > 32
+    (2, 4096, 640, 32, "bf16"),           # 32-mode tcgen05 instance, two rows per CTA
+    (1, 2048 * 2 + 64 * 3, 1024, 24, "bf16"),  # ... one row per CTA, token 0 inside the first tile
 ])
 def test_prefill_from_initial_state_matches_oracle(B, L, D, M, dtype):
     """Prefill started from a state (chunked / continued prefill) against the
@@ -679,15 +687,17 @@ def test_tied_heads_match_the_paper_kernel():
 
 
 @pytest.mark.parametrize("B,L,D,M,with_state_in", [
-    (2, 3000, 512, 32, False),        # two passes of 16 modes (128 CTAs: unsegmented)
+    (2, 3000, 512, 32, False),        # one launch of the 32-mode instance (128 CTAs: unsegmented)
     (1, 2048 + 64, 1024, 40, True),   # three passes, the last with 8 modes; from an initial state
     (2, 4160, 512, 64, True),         # four passes
-    (4, 2048 * 2, 512, 17, False),    # a second pass with one mode
+    (4, 2048 * 2, 512, 17, False),    # the 32-mode instance with 15 padded modes
+    (2, 2048 * 2, 512, 33, False),    # three passes, the last with one mode
 ])
 def test_multi_pass_prefill_matches_oracle(B, L, D, M, with_state_in):
-    """bf16 with M > 16 on unsegmented shapes: passes of 16 modes, each later pass
-    adding to the output of the earlier ones; y, the terminal state and the mode
-    coefficients of every mode on sampled channels against the oracle."""
+    """bf16 with M > 16 on unsegmented shapes: one launch of the 32-mode instance
+    for M <= 32, else passes of 16 modes, each later pass adding to the output of
+    the earlier ones; y, the terminal state and the mode coefficients of every
+    mode on sampled channels against the oracle."""
     inp = make_inputs(B, L, D, M, "bf16", seed=M + L)
     s_in = None
     if with_state_in:
@@ -700,7 +710,7 @@ def test_multi_pass_prefill_matches_oracle(B, L, D, M, with_state_in):
     n0 = rlm.rlm_kernels_launched()
     rlm.rlm_mix_prefill_from(x, p, _state_from(inp, s_in) if with_state_in else None, y, so)
     torch.cuda.synchronize()
-    assert rlm.rlm_kernels_launched() - n0 == (M + 15) // 16
+    assert rlm.rlm_kernels_launched() - n0 == (1 if M <= 32 else (M + 15) // 16)
     ch = np.array([0, 9, D // 2 + 3, D - 1])
     ref, st_ref = oracle.rec_prefill(inp.x[:, :, ch], inp.decay[ch], inp.freq[ch], inp.amp[ch], inp.phase[ch],
                                      state_in=s_in[:, ch] if with_state_in else None)
