@@ -19,8 +19,8 @@
 // it), which hides most of the per-step launch latency when decode steps are
 // issued back to back or captured in a graph.
 //
-// Batches of two or more rows without the mixer take k_decode_tile, whose blocks
-// cover 8 batch rows of the same channels so the coefficient rows come from L1.
+// The plain step (no mixer) takes k_decode_tile, whose blocks cover 8 or 16
+// batch rows of the same channels so the coefficient rows come from L1.
 #include "rlm_device.cuh"
 #include "rlm_internal.h"
 #include "rlm_mixer.cuh"
@@ -162,20 +162,25 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_vec2(
     if (valid && g == 0) st_elem(y_t + bd, acc);
 }
 
-// The plain step (no mixer) for batches, M even with one mode pair per thread:
-// a block of 8 warps covers the same 32 / tpg channels for 8 batch rows (warp w
-// takes row 8 * blockIdx.y + w), so the coefficient rows that every batch row
-// needs are fetched from L2 once per block and then hit in L1.  Within a warp the
-// lanes cover consecutive (channel, pair) slots of one row: one contiguous 512-byte
-// state access per warp.
-template <typename T>
-__global__ void __launch_bounds__(kDecodeBlock) k_decode_tile(
+// The plain step (no mixer), M even with one mode pair per thread: a block of R
+// warps covers the same 32 / tpg channels for R batch rows (warp w takes row
+// R * blockIdx.y + w), so the coefficient rows that every batch row needs are
+// fetched from L2 once per block and then hit in L1.  Within a warp the lanes
+// cover consecutive (channel, pair) slots of one row: one contiguous 512-byte
+// state access per warp.  R = 16 for batches of 16 to 256 rows, else 8: in a
+// CUDA graph of steps at D = 256, M = 16, B = 64 took 1.82 us per step with
+// R = 16 against 1.97 (R = 8), 1.99 (R = 12), 1.97 (R = 24) and 2.03 (R = 32);
+// B = 8 took 1.16 with R = 8 and 1.29 with R = 16; B = 8192 (state above the L2
+// size, bandwidth-bound) 88.5 with R = 8 and 93.4 with R = 16.  A single row
+// (B = 1) took 1.05 us here against 1.37 on k_decode_vec2.
+template <typename T, int R>
+__global__ void __launch_bounds__(R * 32) k_decode_tile(
     const T *__restrict__ x_t, T *__restrict__ y_t, int B, int D, int M, int log2_tpg,
     float4 *__restrict__ s, const float4 *__restrict__ coef) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int g = lane & ((1 << log2_tpg) - 1);
     const int d = blockIdx.x * (32 >> log2_tpg) + (lane >> log2_tpg);
-    const int b = blockIdx.y * (kDecodeBlock / 32) + warp;
+    const int b = blockIdx.y * R + warp;
     const bool on = b < B && d < D && 2 * g < M;
     const int64_t bd = (int64_t)b * D + d;
     if (on && g == 0 && (d & 63) == 0) prefetch_l2(x_t + bd);
@@ -260,10 +265,10 @@ __global__ void k_state_init(float2 *__restrict__ s, float4 *__restrict__ coef, 
 }
 
 template <typename Kern, typename... Args>
-cudaError_t launch_pdl(Kern kern, dim3 grid, cudaStream_t st, Args... args) {
+cudaError_t launch_pdl_block(Kern kern, dim3 grid, int block, cudaStream_t st, Args... args) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
-    cfg.blockDim = dim3(kDecodeBlock);
+    cfg.blockDim = dim3(block);
     cfg.dynamicSmemBytes = 0;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
@@ -273,6 +278,11 @@ cudaError_t launch_pdl(Kern kern, dim3 grid, cudaStream_t st, Args... args) {
     cfg.numAttrs = 1;
     count_launches(1);
     return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+template <typename Kern, typename... Args>
+cudaError_t launch_pdl(Kern kern, dim3 grid, cudaStream_t st, Args... args) {
+    return launch_pdl_block(kern, grid, kDecodeBlock, st, args...);
 }
 
 // One decode step with head coupling (Sec. 3.4) in a single launch, one block per
@@ -400,11 +410,15 @@ cudaError_t decode_t(const T *x_t, T *y_t, int B, int D, int M, float *s, const 
     const int64_t threads = BD * tpg;
     const unsigned grid = (unsigned)((threads + kDecodeBlock - 1) / kDecodeBlock);
     const float4 *cf = reinterpret_cast<const float4 *>(coef);
-    if (!kMix && M % 2 == 0 && 2 * tpg >= M && B >= 2) {
-        // Blocks of 8 batch rows sharing their channels' coefficient rows.
-        const dim3 gr((unsigned)((D + (32 >> log2_tpg) - 1) / (32 >> log2_tpg)),
-                      (unsigned)((B + kDecodeBlock / 32 - 1) / (kDecodeBlock / 32)));
-        return launch_pdl(k_decode_tile<T>, gr, st, x_t, y_t, B, D, M, log2_tpg, reinterpret_cast<float4 *>(s), cf);
+    if (!kMix && M % 2 == 0 && 2 * tpg >= M) {
+        // Blocks of R batch rows sharing their channels' coefficient rows.
+        const int R = B >= 16 && B <= 256 ? 16 : 8;
+        const dim3 gr((unsigned)((D + (32 >> log2_tpg) - 1) / (32 >> log2_tpg)), (unsigned)((B + R - 1) / R));
+        if (R == 16)
+            return launch_pdl_block(k_decode_tile<T, 16>, gr, 16 * 32, st, x_t, y_t, B, D, M, log2_tpg,
+                                    reinterpret_cast<float4 *>(s), cf);
+        return launch_pdl_block(k_decode_tile<T, 8>, gr, 8 * 32, st, x_t, y_t, B, D, M, log2_tpg,
+                                reinterpret_cast<float4 *>(s), cf);
     }
     if (!widened && M % 2 == 0 && 2 * tpg >= M)
         return launch_pdl(k_decode_vec2<T, kMix>, grid, st, x_t, y_t, BD, D, M, log2_tpg,
