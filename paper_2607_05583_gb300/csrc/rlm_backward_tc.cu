@@ -369,13 +369,20 @@ __global__ void __launch_bounds__(kThreads, 2)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
+    // The terminal-state pass (cconj given) runs on a drive that is zero except
+    // at token L-1, which lies in the first tile of the walk: its later tiles
+    // load only x and skip the products of the drive (projections, Q, T'); their
+    // projections are zero in the scan, and the up-projection starts the dx
+    // accumulator.
+    const bool unit = kGrad && args.cconj != nullptr;
     // Tile v of the reverse walk is tile ntiles - 1 - v of the sequence.
     auto load_tile = [&](int v) {
         const int slot = v % kSlots;
         const int chunk0 = (ntiles - 1 - v) * kNT;
         const uint32_t dst = sbase + kOffRing + slot * kSlotBytes;
-        bar_expect_tx(bar(kBarSlotFull + slot), kGrad ? kSlotBytes : kSlotBytes / 2);
-        tma_load_3d(dst, &tmap_dy, 0, chunk0, row, bar(kBarSlotFull + slot));
+        const bool dy_needed = !(unit && v > 0);
+        bar_expect_tx(bar(kBarSlotFull + slot), (dy_needed ? 4096u : 0u) + (kGrad ? 4096u : 0u));
+        if (dy_needed) tma_load_3d(dst, &tmap_dy, 0, chunk0, row, bar(kBarSlotFull + slot));
         if (kGrad) tma_load_3d(dst + 4096, &tmap_x, 0, chunk0, row, bar(kBarSlotFull + slot));
     };
     int issued = 0;
@@ -517,8 +524,13 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int h = 1; h >= 0; --h) {   // chunks 31 .. 0
                 uint32_t pv[16];
-                tmem_ld16(tl + kColP + 32 * bb + 16 * h, pv);
-                tmem_wait_ld();
+                if (unit && v > 0) {
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) pv[e] = 0u;
+                } else {
+                    tmem_ld16(tl + kColP + 32 * bb + 16 * h, pv);
+                    tmem_wait_ld();
+                }
                 if (h == 1) {
                     if (!wait_bar(bar(kBarBsEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) {
                         ok = false;
@@ -688,6 +700,10 @@ __global__ void __launch_bounds__(kThreads, 2)
                 tc_fence_after();
                 const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
                 const uint64_t ddy = desc_sw128(sdy, 16, 1024);
+                if (unit && v > 0) {   // a zero drive: nothing to project (the commit still orders)
+                    umma_commit(bar(kBarPFull + bb));
+                    continue;
+                }
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
                     umma_ss(tmem + kColP + 32 * bb, dap + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
@@ -723,9 +739,12 @@ __global__ void __launch_bounds__(kThreads, 2)
                 tc_fence_after();
                 const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
                 const uint64_t ddy = desc_sw128(sdy, 16, 1024), dxm = desc_sw128(sdy + 4096, 16, 1024);
+                const bool skip_t = unit && v > 0;   // zero drive: dx starts with the up-projection
+                if (!skip_t) {
 #pragma unroll
-                for (int ks = 0; ks < 4; ++ks)
-                    umma_ss(tmem + kColD + 32 * bb, dt + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
+                    for (int ks = 0; ks < 4; ++ks)
+                        umma_ss(tmem + kColD + 32 * bb, dt + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
+                }
                 if (!wait_bar(bar(kBarSFull + bb), (v >> 1) & 1, abort_flag)) {
                     umma_commit(bar(kBarDFull + bb));   // so that the drain below tracks T'
                     ++v;
@@ -740,7 +759,8 @@ __global__ void __launch_bounds__(kThreads, 2)
                     const uint64_t dbu = desc_plain(pp, 512, 128);
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks)
-                        umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dbu + ks * (2048 >> 4), kIdescU, 1u);
+                        umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dbu + ks * (2048 >> 4), kIdescU,
+                                (skip_t && part == 0 && ks == 0) ? 0u : 1u);
                     // E += [S^n ; R^n] X (K = chunks).
                     if (kGrad) {
                         const uint64_t dea = desc_plain(pp, 128, 512);
@@ -1032,11 +1052,20 @@ cudaError_t run_layout_and_scan(const CUtensorMap &mdy, const CUtensorMap &mx, B
 
 }  // namespace
 
-// The terminal-state pass's drive: 1 at token L-1 of every row, 0 elsewhere
-// (the rows were zeroed before).
-__global__ void k_unit_last(__nv_bfloat16 *dT, int64_t rows, int64_t Lp, int64_t L) {
-    const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (r < rows) dT[r * Lp + (L - 1)] = __float2bfloat16_rn(1.0f);
+// The terminal-state pass's drive in the last tile of every row: 1 at token L-1,
+// 0 elsewhere (the pass reads no other tile of it).  Block r writes row r's last
+// tile, 16 bytes per thread.
+__global__ void k_unit_last(__nv_bfloat16 *dT, int64_t Lp, int64_t L) {
+    const int64_t r = blockIdx.x;
+    const int64_t t0 = Lp - kTile + 8 * (int64_t)threadIdx.x;   // 256 threads x 8 tokens
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (L - 1 >= t0 && L - 1 < t0 + 8) {
+        __nv_bfloat16 e[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) e[k] = __float2bfloat16_rn(t0 + k == L - 1 ? 1.0f : 0.0f);
+        v = *reinterpret_cast<const uint4 *>(e);
+    }
+    *reinterpret_cast<uint4 *>(dT + r * Lp + t0) = v;
 }
 
 cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
@@ -1082,8 +1111,7 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
             static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp, 2, 0,
             0, 0, D);
         k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a);
-        if ((e = cudaMemsetAsync(dyT, 0, (size_t)rows * Lp * 2, st)) != cudaSuccess) return e;
-        k_unit_last<<<(unsigned)((rows + 255) / 256), 256, 0, st>>>(dyT, rows, Lp, L);
+        k_unit_last<<<(unsigned)rows, kTile / 8, 0, st>>>(dyT, Lp, L);
         BwdArgs a2 = a;
         a2.part_g = pg2;
         a2.part_p = pj;
@@ -1092,7 +1120,7 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
         k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a2);
         k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(
             dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp, 0, 0, 0, D);
-        count_launches(5);
+        count_launches(5);   // transpose, pass, unit drive, pass, transpose
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     return grad_reduce(rows / D, D, M, amp, phase, pg, pp, d_state_out ? pj : nullptr, g_decay, g_freq, g_amp,
