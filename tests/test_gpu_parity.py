@@ -627,6 +627,34 @@ def test_backward_training_workload_sampled():
         assert_close(getattr(g, k).cpu().numpy()[chans], g_ref[k], TOL["bf16"], "d" + k)
 
 
+@pytest.mark.parametrize("B,L,D,M,dtype", [
+    (4, 32768, 256, 16, "bf16"),     # the 16-mode tensor-core prefill (15-slot x ring)
+    (4, 32768, 512, 32, "bf16"),     # the 32-mode instance (7-slot x ring, two CTA waves)
+    (4, 32768, 256, 16, "f32"),      # the fp32 tensor-core prefill
+    (1, 2048 * 24 + 5, 64, 16, "bf16"),  # segmented, with published segment states
+])
+def test_prefill_is_bit_reproducible(B, L, D, M, dtype):
+    """Each call is a fixed sequence of fp32 operations, so repeated calls give
+    identical bits (y and the terminal state).  Runs each shape five times: a
+    pipeline hazard that lets a stage read a stale buffer shows up as a
+    difference between calls."""
+    inp = make_inputs(B, L, D, M, dtype, seed=21)
+    x = to_dev(inp.x, dtype)
+    p = rlm.Params.from_arrays(*inp.params())
+    ws = torch.empty(max(256, rlm.rlm_prefill_workspace_size(B, L, D, M, x.dtype)), dtype=torch.uint8,
+                     device=x.device)
+    ref_y, ref_s = None, None
+    for it in range(5):
+        y, st = torch.empty_like(x), rlm.State.empty(B, D, M)
+        rlm.rlm_mix_prefill(x, p, y, st, workspace=ws)
+        torch.cuda.synchronize()
+        if ref_y is None:
+            ref_y, ref_s = y, st.s.clone()
+        else:
+            assert torch.equal(y, ref_y), it
+            assert torch.equal(st.s, ref_s), it
+
+
 def test_backward_is_deterministic():
     inp = make_inputs(2, 5000, 64, 16, "bf16", seed=8, with_dy=True)
     dx1, g1 = _backward(inp)
