@@ -855,19 +855,28 @@ __global__ void __launch_bounds__(128) k_to_channel_major(const __nv_bfloat16 *_
     const int b = b0 + blockIdx.z / nf, f = blockIdx.z % nf;
     const __nv_bfloat16 *src = f ? src1 : src0;
     __nv_bfloat16 *dst = f ? dst1 : dst0;
-    for (int it = threadIdx.x; it < 512; it += 128) {
+    // Four 16-byte loads per thread, all issued before the tile is written.
+    uint4 val[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int it = threadIdx.x + 128 * k;
         const int r = it >> 3, vq = it & 7;
         const int64_t sp = t0 + r;
         const int c = c0 + 8 * vq;
-        uint4 val = make_uint4(0, 0, 0, 0);
+        val[k] = make_uint4(0, 0, 0, 0);
         if (sp < L && c < c_hi) {
             const int64_t t = rev ? L - 1 - sp : sp;
-            val = __ldg(reinterpret_cast<const uint4 *>(src + ((int64_t)b * L + t) * D + c));
+            val[k] = __ldg(reinterpret_cast<const uint4 *>(src + ((int64_t)b * L + t) * D + c));
         }
-        tile[r][4 * vq] = val.x;
-        tile[r][4 * vq + 1] = val.y;
-        tile[r][4 * vq + 2] = val.z;
-        tile[r][4 * vq + 3] = val.w;
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const int it = threadIdx.x + 128 * k;
+        const int r = it >> 3, vq = it & 7;
+        tile[r][4 * vq] = val[k].x;
+        tile[r][4 * vq + 1] = val[k].y;
+        tile[r][4 * vq + 2] = val[k].z;
+        tile[r][4 * vq + 3] = val[k].w;
     }
     __syncthreads();
     for (int it = threadIdx.x; it < 512; it += 128) {
@@ -898,17 +907,30 @@ __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__res
     const int b = b0 + blockIdx.z;
     // First position of the window: t0 itself, or the last 64 tokens' mirror rounded down.
     const int64_t s_lo = rev ? ((L - t0 - 64) >= 0 ? (L - t0 - 64) & ~(int64_t)7 : -((t0 + 64 - L + 7) & ~(int64_t)7)) : t0;
-    for (int it = threadIdx.x; it < 64 * 9; it += 128) {
-        const int cr = it / 9, vq = it % 9;
+    // A reversed window can straddle nine 8-position groups, a forward one is
+    // eight; a thread issues its (at most five) 16-byte loads before writing the
+    // tile.
+    const int nv = rev ? 9 : 8, nload = 64 * nv;
+    uint4 val[5];
+#pragma unroll
+    for (int k = 0; k < 5; ++k) {
+        const int it = threadIdx.x + 128 * k;
+        const int cr = it / nv, vq = it % nv;
         const int c = c0 + cr;
         const int64_t sp = s_lo + 8 * vq;
-        uint4 val = make_uint4(0, 0, 0, 0);
-        if (c < c_hi && sp >= 0 && sp < Lp)
-            val = __ldg(reinterpret_cast<const uint4 *>(srcT + ((int64_t)b * D + c) * Lp + sp));
-        tile[cr][4 * vq] = val.x;
-        tile[cr][4 * vq + 1] = val.y;
-        tile[cr][4 * vq + 2] = val.z;
-        tile[cr][4 * vq + 3] = val.w;
+        val[k] = make_uint4(0, 0, 0, 0);
+        if (it < nload && c < c_hi && sp >= 0 && sp < Lp)
+            val[k] = __ldg(reinterpret_cast<const uint4 *>(srcT + ((int64_t)b * D + c) * Lp + sp));
+    }
+#pragma unroll
+    for (int k = 0; k < 5; ++k) {
+        const int it = threadIdx.x + 128 * k;
+        if (it >= nload) break;
+        const int cr = it / nv, vq = it % nv;
+        tile[cr][4 * vq] = val[k].x;
+        tile[cr][4 * vq + 1] = val[k].y;
+        tile[cr][4 * vq + 2] = val[k].z;
+        tile[cr][4 * vq + 3] = val[k].w;
     }
     __syncthreads();
     for (int it = threadIdx.x; it < 512; it += 128) {
