@@ -123,8 +123,8 @@ constexpr int kSlotBytes = 8192;
 // K = the 16 S^n rows, LBO 512).
 constexpr int kOffBs = kOffRing + kSlots * kSlotBytes;   // [2] x (hi 8 KB, lo 8 KB)
 constexpr int kBsBuf = 16384;
-constexpr int kOffRho = kOffBs + 2 * kBsBuf;             // [2 warps][64] fp32
-constexpr int kOffBar = kOffRho + 2 * 64 * 4;
+constexpr int kOffRho = kOffBs + 2 * kBsBuf;             // [64] fp32: rho[n]
+constexpr int kOffBar = kOffRho + 64 * 4;
 constexpr int kNumBars = 32;
 constexpr int kOffMisc = kOffBar + kNumBars * 8;
 constexpr int kSmemBytes = kOffMisc + 64 + 1024;         // + alignment slack
@@ -137,6 +137,7 @@ constexpr int kOffPw = kOffBs;                                  // [32][65] floa
 constexpr int kOffCf = kOffPw + kMaxModes * kPwStride * 8;      // [32] float2
 constexpr int kOffK = kOffCf + kMaxModes * 8;                   // [64] float
 static_assert(kOffK + 64 * 4 <= kOffRho, "prologue scratch does not fit");
+static_assert(kC * 65 * 4 <= kSlots * kSlotBytes, "Q staging (end of the walk) does not fit in the ring");
 
 // Barrier indices.
 constexpr int kBarSlotFull = 0;                  // [kSlots]
@@ -420,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                 : args.cconj ? conj2(args.cconj[(int64_t)row * M + m])
                              : mode_coef(args.amp[d * M + m], args.phase[d * M + m]);
     }
-    if (tid < 128) reinterpret_cast<float *>(smem + kOffRho)[tid] = 0.0f;
+    if (tid < 64) reinterpret_cast<float *>(smem + kOffRho)[tid] = 0.0f;
     __syncthreads();
     // Stage 2: K[n] (Eq. 1 at integer lags, modes summed in a fixed order), the
     // projection table and the up-projection U', one 16-byte core-matrix row
@@ -656,23 +657,38 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
         }
         // Diagonal sums of Q (accumulated over the whole sequence; its last
-        // product precedes the last dx product): lane i of quarter q adds
-        // Q[i][j], j <= i, to rho_q[i - j].
-        if (kGrad && ok) {
-            tc_fence_after();
+        // product precedes the last dx product).  Both warps stage the rows of
+        // Q's lower triangle in the ring, which no load or product touches any
+        // more (row stride 65 words: the row writes and the diagonal reads each
+        // hit 32 banks), then thread n sums diagonal n: rho[n] = sum_k Q[n+k][k].
+        // (Adding row by row into rho, one dependent shared-memory update per
+        // element, cost ~3k cycles at the end of every CTA.)
+        if (kGrad) {
             const int i = 32 * q + lane;
-            float *rho = reinterpret_cast<float *>(smem + kOffRho) + 64 * q;
-            for (int h = 0; h < 2 + 2 * q; ++h) {
-                uint32_t qv[16];
-                tmem_ld16(tl + kColQ + 16 * h, qv);
-                tmem_wait_ld();
+            float *qs = reinterpret_cast<float *>(smem + kOffRing);
+            if (ok) {
+                tc_fence_after();
+                for (int h = 0; h < 2 + 2 * q; ++h) {
+                    uint32_t qv[16];
+                    tmem_ld16(tl + kColQ + 16 * h, qv);
+                    tmem_wait_ld();
 #pragma unroll
-                for (int e = 0; e < 16; ++e) {
-                    const int j = 16 * h + e;
-                    if (j <= i) rho[i - j] += __uint_as_float(qv[e]);
-                    __syncwarp();
+                    for (int e = 0; e < 16; ++e) qs[i * 65 + 16 * h + e] = __uint_as_float(qv[e]);
                 }
             }
+            // Both epilogue warps arrive here whether or not their loop completed.
+            asm volatile("bar.sync 1, 64;" ::: "memory");
+            float r0 = 0.0f, r1 = 0.0f, r2 = 0.0f, r3 = 0.0f;
+            int k = 0;
+            for (; k + 4 <= kC - i; k += 4) {
+                const float *p = qs + (i + k) * 65 + k;
+                r0 += p[0];
+                r1 += p[66];
+                r2 += p[132];
+                r3 += p[198];
+            }
+            for (; k < kC - i; ++k) r0 += qs[(i + k) * 65 + k];
+            if (ok) reinterpret_cast<float *>(smem + kOffRho)[i] = (r0 + r1) + (r2 + r3);
         }
     } else if (warp == w_prod) {
         // ---------------------------------------------------- TMA producer
@@ -790,7 +806,7 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll 4
         for (int e = 0; e < kC / 4; ++e) {
             const int n = 4 * e + s;
-            const float r = rho[n] + rho[64 + n];
+            const float r = rho[n];
             const float2 ln = lambda_pow(gamE, omgE, (float)n);
             gr = fmaf(r, ln.x, gr);
             gi = fmaf(r, ln.y, gi);
@@ -951,6 +967,67 @@ __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__res
     }
 }
 
+// [B*D][Lp] -> [B][L][D] without reversal: a 256-thread block covers 128 tokens x
+// 64 channels, so it reads 256 contiguous bytes of each channel row (the 64-token
+// tile above reads 128).  Measured on the backward at B = 4, L = 32768, D = 512:
+// the dx transpose 14 us shorter (0.380 -> 0.365 ms per call).  The same widening
+// of the channel-major transpose made it slower.
+constexpr int kRmTokens = 128, kRmChannels = 64;
+__global__ void __launch_bounds__(256) k_to_row_major_wide(const __nv_bfloat16 *__restrict__ srcT,
+                                                           __nv_bfloat16 *__restrict__ dst, int64_t L, int D,
+                                                           int64_t Lp) {
+    constexpr int kStride = kRmTokens / 2 + 1, kGroups = kRmTokens / 8;
+    constexpr int kLoads = kRmChannels * kGroups / 256, kStores = kRmTokens * (kRmChannels / 8) / 256;
+    __shared__ uint32_t tile[kRmChannels][kStride];   // [channel][position pair]
+    const int64_t t0 = (int64_t)blockIdx.x * kRmTokens;
+    const int c0 = blockIdx.y * kRmChannels;
+    const int b = blockIdx.z;
+    uint4 val[kLoads];
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k) {
+        const int it = threadIdx.x + 256 * k;
+        const int cr = it / kGroups, vq = it % kGroups;
+        const int c = c0 + cr;
+        const int64_t sp = t0 + 8 * vq;
+        val[k] = make_uint4(0, 0, 0, 0);
+        if (c < D && sp < Lp) val[k] = __ldg(reinterpret_cast<const uint4 *>(srcT + ((int64_t)b * D + c) * Lp + sp));
+    }
+#pragma unroll
+    for (int k = 0; k < kLoads; ++k) {
+        const int it = threadIdx.x + 256 * k;
+        const int cr = it / kGroups, vq = it % kGroups;
+        tile[cr][4 * vq] = val[k].x;
+        tile[cr][4 * vq + 1] = val[k].y;
+        tile[cr][4 * vq + 2] = val[k].z;
+        tile[cr][4 * vq + 3] = val[k].w;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < kStores; ++k) {
+        const int it = threadIdx.x + 256 * k;
+        const int r = it / (kRmChannels / 8), vq = it % (kRmChannels / 8);
+        const int64_t t = t0 + r;
+        const int c = c0 + 8 * vq;
+        if (t >= L || c >= D) continue;
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const uint32_t a = tile[8 * vq + 2 * e][r >> 1], bw = tile[8 * vq + 2 * e + 1][r >> 1];
+            const uint32_t lo = (r & 1) ? (a >> 16) : (a & 0xffffu);
+            const uint32_t hi = (r & 1) ? (bw >> 16) : (bw & 0xffffu);
+            w[e] = lo | (hi << 16);
+        }
+        *reinterpret_cast<uint4 *>(dst + ((int64_t)b * L + t) * D + c) = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+// Its launch (D % 8 == 0, which every tcgen05 backward shape has).
+void row_major_wide(const __nv_bfloat16 *srcT, __nv_bfloat16 *dst, int64_t B, int64_t L, int D, int64_t Lp,
+                    cudaStream_t st) {
+    k_to_row_major_wide<<<dim3((unsigned)((L + kRmTokens - 1) / kRmTokens),
+                               (unsigned)((D + kRmChannels - 1) / kRmChannels), (unsigned)B),
+                          256, 0, st>>>(srcT, dst, L, D, Lp);
+}
+
 // ------------------------------------------------------------ host side
 using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
                                    const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
@@ -1066,8 +1143,11 @@ cudaError_t run_layout_and_scan(const CUtensorMap &mdy, const CUtensorMap &mx, B
         src0, src1, dst0, dst1, L, D, Lp, nf, rev, 0, 0, D);
     a.row0 = 0;
     k_backward_tc<kGrad><<<(unsigned)(B * D), kThreads, kSmemBytes, st>>>(mdy, mx, a);
-    k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(outT, out, L, D, Lp, rev, 0,
-                                                                                     0, D);
+    if (rev)
+        k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(outT, out, L, D, Lp, rev,
+                                                                                         0, 0, D);
+    else
+        row_major_wide(outT, out, B, L, D, Lp, st);
     count_launches(3);
     return cudaGetLastError();
 }
@@ -1140,8 +1220,7 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
         a2.cconj = reinterpret_cast<const float2 *>(d_state_out);
         a2.acc_dx = 1;
         k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a2);
-        k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(
-            dxT, static_cast<__nv_bfloat16 *>(dx), L, D, Lp, 0, 0, 0, D);
+        row_major_wide(dxT, static_cast<__nv_bfloat16 *>(dx), B, L, D, Lp, st);
         count_launches(5);   // transpose, pass, unit drive, pass, transpose
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }

@@ -45,7 +45,7 @@ cudaError_t simt_backward(const void *dy, const void *x, void *dx, rlm_dtype dt,
                           float *g_freq, float *g_amp, float *g_phase, void *ws,
                           cudaStream_t st);
 
-// Fixed-order (fp64) sum of nparts partial (G, P) arrays of [D][M] each, then the
+// Fixed-order (compensated fp32) sum of nparts partial (G, P) arrays of [D][M] each, then the
 // four parameter gradients.  J (nullable): nparts partials of conj(g) J from a
 // terminal-state gradient g, whose sum's -Re and -Im join dgamma and domega.
 cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const float *phase,

@@ -354,9 +354,23 @@ __global__ void __launch_bounds__(kBlock) k_chunk_backward(
 }
 
 // Phase 4 (backward).  One thread per (d, m): fixed-order sum of the partials
-// over (b, k) in double, then the four gradients.
+// over (b, k), then the four gradients.  The sums are compensated (Kahan) fp32
+// sums, so the result is reproducible and its error stays near one rounding
+// however many chunk partials the SIMT path adds; the combination with
+// c = A e^{i phi} (formed as the forward forms it, fp32 sincosf) uses fmaf for
+// the differences.  Double precision made this launch 3-4x slower on this part
+// (low FP64 rate): 4.8 against 1.4 us at D = 512, M = 32, four partials.
 // ws_j (nullable): partials of conj(g) J from a terminal-state gradient, which
 // add -Re and -Im of their sum to dgamma and domega.
+struct KahanSum {
+    float s = 0.0f, c = 0.0f;
+    __device__ __forceinline__ void add(float v) {
+        const float y = v - c;
+        const float t = s + y;
+        c = (t - s) - y;
+        s = t;
+    }
+};
 __global__ void __launch_bounds__(256) k_grad_reduce(
     int64_t B, int D, int M, int nch, const float *__restrict__ amp,
     const float *__restrict__ phase, const float2 *__restrict__ ws_s,
@@ -364,27 +378,40 @@ __global__ void __launch_bounds__(256) k_grad_reduce(
     float *__restrict__ g_freq, float *__restrict__ g_amp, float *__restrict__ g_phase) {
     const int pm = blockIdx.x * blockDim.x + threadIdx.x;
     if (pm >= D * M) return;
-    double gr = 0, gi = 0, pr = 0, pi = 0, jr = 0, ji = 0;
-    for (int64_t bk = 0; bk < B * nch; ++bk) {
-        const int64_t off = bk * D * M + pm;
-        const float2 g = ws_s[off], p = ws_r[off];
-        gr += g.x;
-        gi += g.y;
-        pr += p.x;
-        pi += p.y;
-        if (ws_j) {
-            jr += ws_j[off].x;
-            ji += ws_j[off].y;
+    const float am = amp[pm], ph = phase[pm];
+    KahanSum gr, gi, pr, pi, jr, ji;
+    const int64_t n = B * nch, stride = (int64_t)D * M;
+    // Four partials' loads in flight before their adds (the sum order is fixed).
+    for (int64_t bk0 = 0; bk0 < n; bk0 += 4) {
+        float2 g[4], p[4], j[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t off = (bk0 + u) * stride + pm;
+            const bool in = bk0 + u < n;
+            g[u] = in ? ws_s[off] : make_float2(0.0f, 0.0f);
+            p[u] = in ? ws_r[off] : make_float2(0.0f, 0.0f);
+            j[u] = in && ws_j ? ws_j[off] : make_float2(0.0f, 0.0f);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (bk0 + u >= n) break;
+            gr.add(g[u].x);
+            gi.add(g[u].y);
+            pr.add(p[u].x);
+            pi.add(p[u].y);
+            if (ws_j) {
+                jr.add(j[u].x);
+                ji.add(j[u].y);
+            }
         }
     }
-    double sph, cph;
-    sincos((double)phase[pm], &sph, &cph);
-    const double a = amp[pm];
-    const double cr = a * cph, ci = a * sph;
-    g_amp[pm] = (float)(cph * gr - sph * gi);         // Re(e^{i phi} G)
-    g_phase[pm] = (float)(-(cr * gi + ci * gr));      // -Im(c G)
-    g_decay[pm] = (float)(-(cr * pr - ci * pi) - jr);   // -Re(c P) - Re(conj(g) J)
-    g_freq[pm] = (float)(-(cr * pi + ci * pr) - ji);    // -Im(c P) - Im(conj(g) J)
+    float sph, cph;
+    sincosf(ph, &sph, &cph);
+    const float cr = am * cph, ci = am * sph;
+    g_amp[pm] = fmaf(cph, gr.s, -sph * gi.s);            // Re(e^{i phi} G)
+    g_phase[pm] = -fmaf(cr, gi.s, ci * gr.s);            // -Im(c G)
+    g_decay[pm] = -fmaf(cr, pr.s, -ci * pi.s) - jr.s;    // -Re(c P) - Re(conj(g) J)
+    g_freq[pm] = -fmaf(cr, pi.s, ci * pr.s) - ji.s;      // -Im(c P) - Im(conj(g) J)
 }
 
 template <typename T>
