@@ -767,8 +767,8 @@ def _bench_backward(rlm, torch, dev, hbm_peak, args, flush):
     fms = _timed(lambda: rlm.rlm_mix_prefill(x, p, y, st, workspace=fw))
     del y, st, fw
     # Backward with the state terms of a segmented training step: an initial state
-    # (its gradient returned), and a terminal-state gradient as well (a second pass
-    # of the tcgen05 kernel).
+    # (its gradient returned), and a terminal-state gradient as well (one more
+    # launch that forms its terms in closed form).
     gen = torch.Generator(device="cpu").manual_seed(1)
     s_in, ds_out, ds_in = (rlm.State.empty(B, D, M, device=dev) for _ in range(3))
     s_in.s.copy_(torch.randn(B, D, M, 2, generator=gen))
@@ -787,8 +787,8 @@ def _bench_backward(rlm, torch, dev, hbm_peak, args, flush):
             "forward_ms": round(fms, 4), "forward_plus_backward_ms": round(fms + ms, 4),
             "with_state_in_ms": round(ms_init, 4),
             "with_state_in_and_d_state_out_ms": round(ms_term, 4),
-            "state_terms_route": "tcgen05; d_state_out adds a second pass of the same kernel on a unit "
-                                 "drive at token L-1 read through c = conj(d_state_out)"}
+            "state_terms_route": "tcgen05; d_state_out adds one launch (k_terminal_tc) forming "
+                                 "conj(g) lambda^(L-1-t) terms in closed form on the tensor cores"}
 
 
 def run_backward_only(args):

@@ -218,9 +218,9 @@ RLM_API rlm_status rlm_mix_backward(const rlm_tensor *dy, const rlm_tensor *x, c
  *                must not overlap dx, dparams, state_in or d_state_out.
  * dx and dparams as for rlm_mix_backward, with the state terms included.  Paths:
  * bf16 with M <= 32 runs the tcgen05 backward (state_in and d_state_in are
- * per-(b, d, m) terms at its end; a d_state_out adds a second pass of the same
- * kernel, on a unit drive at token L-1 read through c = conj(g)); fp32 or M > 32,
- * the SIMT backward.  rlm_backward_workspace_size covers the path taken. */
+ * per-(b, d, m) terms at its end; a d_state_out adds one launch that forms its
+ * terms in closed form, conj(g) lambda^(L-1-t), on the tensor cores); fp32 or
+ * M > 32, the SIMT backward.  rlm_backward_workspace_size covers the path taken. */
 RLM_API rlm_status rlm_mix_backward_from(const rlm_tensor *dy, const rlm_tensor *x, const rlm_params *p,
                                          const rlm_state *state_in, const rlm_state *d_state_out, rlm_tensor *dx,
                                          rlm_grads *dparams, rlm_state *d_state_in, const rlm_launch *launch);

@@ -307,11 +307,6 @@ struct BwdArgs {
     int row0;                 // first (b * D + d) row of this launch (0: the whole problem)
     float4 *coef_out;         // nullable, [D][M]   (time-reversed prefill)
     float2 *d_state_in;       // nullable, [B*D][M] (backward: gradient of the forward's state_in)
-    // nullable, [B*D][M]: the terminal-state pass (a unit drive at token L-1 read
-    // through c = conj(cconj[b * D + d][m]) per batch row); it writes c P as its P
-    // partial and adds to d_state_in.
-    const float2 *cconj;
-    int acc_dx;               // add this pass's dx to what dxT holds (the terminal-state pass)
     __nv_bfloat16 *dxT;       // [B*D][Lp]
     int64_t Lp;
     int D, M;
@@ -370,20 +365,13 @@ __global__ void __launch_bounds__(kThreads, 2)
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    // The terminal-state pass (cconj given) runs on a drive that is zero except
-    // at token L-1, which lies in the first tile of the walk: its later tiles
-    // load only x and skip the products of the drive (projections, Q, T'); their
-    // projections are zero in the scan, and the up-projection starts the dx
-    // accumulator.
-    const bool unit = kGrad && args.cconj != nullptr;
     // Tile v of the reverse walk is tile ntiles - 1 - v of the sequence.
     auto load_tile = [&](int v) {
         const int slot = v % kSlots;
         const int chunk0 = (ntiles - 1 - v) * kNT;
         const uint32_t dst = sbase + kOffRing + slot * kSlotBytes;
-        const bool dy_needed = !(unit && v > 0);
-        bar_expect_tx(bar(kBarSlotFull + slot), (dy_needed ? 4096u : 0u) + (kGrad ? 4096u : 0u));
-        if (dy_needed) tma_load_3d(dst, &tmap_dy, 0, chunk0, row, bar(kBarSlotFull + slot));
+        bar_expect_tx(bar(kBarSlotFull + slot), kGrad ? 8192u : 4096u);
+        tma_load_3d(dst, &tmap_dy, 0, chunk0, row, bar(kBarSlotFull + slot));
         if (kGrad) tma_load_3d(dst + 4096, &tmap_x, 0, chunk0, row, bar(kBarSlotFull + slot));
     };
     int issued = 0;
@@ -418,7 +406,6 @@ __global__ void __launch_bounds__(kThreads, 2)
     } else if (tid >= 288 && tid < 288 + kMaxModes) {
         const int m = tid - 288;
         cf[m] = m >= M ? make_float2(0.0f, 0.0f)
-                : args.cconj ? conj2(args.cconj[(int64_t)row * M + m])
                              : mode_coef(args.amp[d * M + m], args.phase[d * M + m]);
     }
     if (tid < 64) reinterpret_cast<float *>(smem + kOffRho)[tid] = 0.0f;
@@ -525,13 +512,8 @@ __global__ void __launch_bounds__(kThreads, 2)
 #pragma unroll
             for (int h = 1; h >= 0; --h) {   // chunks 31 .. 0
                 uint32_t pv[16];
-                if (unit && v > 0) {
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) pv[e] = 0u;
-                } else {
-                    tmem_ld16(tl + kColP + 32 * bb + 16 * h, pv);
-                    tmem_wait_ld();
-                }
+                tmem_ld16(tl + kColP + 32 * bb + 16 * h, pv);
+                tmem_wait_ld();
                 if (h == 1) {
                     if (!wait_bar(bar(kBarBsEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) {
                         ok = false;
@@ -633,27 +615,10 @@ __global__ void __launch_bounds__(kThreads, 2)
             }
             // Channel-major dx: each store instruction writes 64 contiguous bytes.
             __nv_bfloat16 *out = args.dxT + (int64_t)row * args.Lp + (int64_t)(last - v) * kTile + 32 * q + lane;
-            if (args.acc_dx) {
-                // Added to the first pass's dx (16 loads issued before their adds).
-                // That dx was already rounded to bf16, so the sum is rounded twice:
-                // one extra bf16 rounding of dx, well inside the bf16 tolerance.
 #pragma unroll
-                for (int hf = 0; hf < 2; ++hf) {
-                    const uint32_t *rv = hf ? r1 : r0;
-                    __nv_bfloat16 *oh = out + 16 * hf * kC;
-                    __nv_bfloat16 prev[16];
-#pragma unroll
-                    for (int k = 0; k < 16; ++k) prev[k] = oh[k * kC];
-#pragma unroll
-                    for (int k = 0; k < 16; ++k)
-                        oh[k * kC] = __float2bfloat16_rn(__bfloat162float(prev[k]) + __uint_as_float(rv[k]));
-                }
-            } else {
-#pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    out[k * kC] = __float2bfloat16_rn(__uint_as_float(r0[k]));
-                    out[(k + 16) * kC] = __float2bfloat16_rn(__uint_as_float(r1[k]));
-                }
+            for (int k = 0; k < 16; ++k) {
+                out[k * kC] = __float2bfloat16_rn(__uint_as_float(r0[k]));
+                out[(k + 16) * kC] = __float2bfloat16_rn(__uint_as_float(r1[k]));
             }
         }
         // Diagonal sums of Q (accumulated over the whole sequence; its last
@@ -716,10 +681,6 @@ __global__ void __launch_bounds__(kThreads, 2)
                 tc_fence_after();
                 const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
                 const uint64_t ddy = desc_sw128(sdy, 16, 1024);
-                if (unit && v > 0) {   // a zero drive: nothing to project (the commit still orders)
-                    umma_commit(bar(kBarPFull + bb));
-                    continue;
-                }
 #pragma unroll
                 for (int ks = 0; ks < 4; ++ks)
                     umma_ss(tmem + kColP + 32 * bb, dap + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
@@ -755,12 +716,9 @@ __global__ void __launch_bounds__(kThreads, 2)
                 tc_fence_after();
                 const uint32_t sdy = sbase + kOffRing + slot * kSlotBytes;
                 const uint64_t ddy = desc_sw128(sdy, 16, 1024), dxm = desc_sw128(sdy + 4096, 16, 1024);
-                const bool skip_t = unit && v > 0;   // zero drive: dx starts with the up-projection
-                if (!skip_t) {
 #pragma unroll
-                    for (int ks = 0; ks < 4; ++ks)
-                        umma_ss(tmem + kColD + 32 * bb, dt + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
-                }
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kColD + 32 * bb, dt + ks * 16, ddy + ks * 2, kIdescN32, ks > 0);
                 if (!wait_bar(bar(kBarSFull + bb), (v >> 1) & 1, abort_flag)) {
                     umma_commit(bar(kBarDFull + bb));   // so that the drain below tracks T'
                     ++v;
@@ -775,8 +733,7 @@ __global__ void __launch_bounds__(kThreads, 2)
                     const uint64_t dbu = desc_plain(pp, 512, 128);
 #pragma unroll
                     for (int ks = 0; ks < 4; ++ks)
-                        umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dbu + ks * (2048 >> 4), kIdescU,
-                                (skip_t && part == 0 && ks == 0) ? 0u : 1u);
+                        umma_ss(tmem + kColD + 32 * bb, du + ks * 16, dbu + ks * (2048 >> 4), kIdescU, 1u);
                     // E += [S^n ; R^n] X (K = chunks).
                     if (kGrad) {
                         const uint64_t dea = desc_plain(pp, 128, 512);
@@ -828,15 +785,9 @@ __global__ void __launch_bounds__(kThreads, 2)
                 pi += pin.y;
             }
             if (args.d_state_in) {
-                const float2 c = args.cconj ? conj2(args.cconj[(int64_t)row * M + mE])
-                                            : mode_coef(args.amp[d * M + mE], args.phase[d * M + mE]);
+                const float2 c = mode_coef(args.amp[d * M + mE], args.phase[d * M + mE]);
                 const float2 cls = cmul(c, ls);
-                float2 ds = make_float2(cls.x, -cls.y);
-                if (args.cconj) {
-                    const float2 prev = args.d_state_in[(int64_t)row * M + mE];
-                    ds = make_float2(prev.x + ds.x, prev.y + ds.y);
-                }
-                args.d_state_in[(int64_t)row * M + mE] = ds;
+                args.d_state_in[(int64_t)row * M + mE] = make_float2(cls.x, -cls.y);
             }
         }
 #pragma unroll
@@ -847,12 +798,453 @@ __global__ void __launch_bounds__(kThreads, 2)
             pi += __shfl_xor_sync(0xffffffffu, pi, o);
         }
         if (s == 0 && onE) {
-            float2 pp = make_float2(pr, pi);
-            if (args.cconj) pp = cmul(conj2(args.cconj[(int64_t)row * M + mE]), pp);   // conj(g) J
             args.part_g[(int64_t)row * M + mE] = make_float2(gr, gi);
-            args.part_p[(int64_t)row * M + mE] = pp;
+            args.part_p[(int64_t)row * M + mE] = make_float2(pr, pi);
         }
     }
+}
+
+// ------------------------------------------------------------ terminal-state gradient
+// The loss term Re(conj(g) s_L) of a terminal-state gradient g = d_state_out
+// (Sec. 3.2-3.3) adds, per (b, d) row and mode, with s = L - 1 - j:
+//   dx_j     += Re(sum_m conj(g_m) lambda_m^s),
+//   J_m       = sum_j x_j s lambda_m^s (+ L lambda^L s_in),  written as conj(g) J
+//               (the reduction subtracts its Re and Im from dgamma and domega),
+//   d_state_in += g conj(lambda^L).
+// Its adjoint state is the closed form conj(g) lambda^s, so no scan is needed.
+// Chunk n (tokens 64 n + i) lies fully before L when E_n = L - 64 - 64 n >= 0;
+// then lambda^s = lambda^E_n lambda^(63-i) with both exponents >= 0, and
+//   J += lambda^E_n (E_n p_n + q_n),  p_n = sum_i lambda^(63-i) x,  q_n = sum_i (63-i) lambda^(63-i) x
+//   dx[i][n] = Re(W_n lambda^(63-i)),  W_n = conj(g) lambda^E_n,
+// both on the tensor cores (p, q: the projections of the main pass with the
+// table reversed in i; dx: an up-projection of W).  The one chunk that holds
+// token L - 1 without ending there (L % 64 != 0) is evaluated directly in fp32,
+// so no negative power of lambda is ever formed.  One CTA per row, walking the
+// tiles from the end of the sequence:
+//   warps 0-3  per tile: the chunk weights lambda^E_n (an exact power at the
+//              tile's first full chunk, then steps of lambda^64), the W rows,
+//              and J from the projections (each lane weights its own TMEM row,
+//              the mode's four rows are added at the end);
+//   warps 4-5  dx epilogue: dxT += dx (positions 0-63; the old values come
+//              with the x tile, so no global read waits in the loop);
+//   warp 6     TMA producer (per slot: the x tile, swizzled for the product, and
+//              the dxT tile, plain), TMEM allocation;
+//   warp 7     MMA issue: projections into P, then the W up-projection into D.
+constexpr int kTmWarps = 8;
+constexpr int kTmThreads = kTmWarps * 32;
+constexpr int kTmSlots = 4;
+constexpr int kTmCols = 128;
+constexpr int kTmColP = 0;    // [2] x 32: projections (rows as in A_P)
+constexpr int kTmColD = 64;   // [2] x 32: dx (lanes 0-63)
+constexpr int kTmOffU = 0;                                  // U_g: 64 rows x K 64 (rows 64-127 of its M=128 product read kTmOffA)
+constexpr int kTmOffA = 8192;                               // reversed projection table, 128 rows
+constexpr int kTmOffAlo = 24576;                            // its low parts, 64 rows
+constexpr int kTmOffRing = 32768;                           // [kTmSlots] x (4 KB) + dxT (4 KB) tiles
+constexpr int kTmSlotBytes = 8192;
+constexpr int kTmOffW = kTmOffRing + kTmSlots * kTmSlotBytes;   // [2] W buffers, 8 KB each (pair layout)
+constexpr int kTmOffPw = kTmOffW + 2 * 8192;                // [32][65] float2: lambda^s, s = 0..64
+constexpr int kTmOffG = kTmOffPw + kMaxModes * kPwStride * 8;   // [32] float2: g
+constexpr int kTmOffXp = kTmOffG + kMaxModes * 8;          // [64] fp32: x of the chunk holding token L - 1
+constexpr int kTmOffBar = kTmOffXp + kC * 4;
+constexpr int kTmNumBars = 24;
+constexpr int kTmOffMisc = kTmOffBar + kTmNumBars * 8;
+constexpr int kTmSmemBytes = kTmOffMisc + 64 + 1024;        // + alignment slack
+static_assert(kTmOffRing % 1024 == 0, "swizzled tiles need 1024-byte alignment");
+static_assert(2 * (kTmSmemBytes + 1024) <= 233472, "two CTAs per SM");
+constexpr int kTmSlotFull = 0, kTmSlotEmpty = kTmSlots, kTmPFull = 2 * kTmSlots, kTmPEmpty = kTmPFull + 2,
+              kTmWFull = kTmPEmpty + 2, kTmWEmpty = kTmWFull + 2, kTmDFull = kTmWEmpty + 2,
+              kTmDEmpty = kTmDFull + 2;
+static_assert(kTmDEmpty + 2 <= kTmNumBars, "too many barriers");
+
+// SlotEmpty counts the projection commit and the two epilogue warps.
+struct TermArgs {
+    const float *decay, *freq;     // [D][M]
+    const float2 *g;               // d_state_out, [B*D][M]
+    const float2 *state_in;        // nullable, [B*D][M]
+    float2 *d_state_in;            // nullable, [B*D][M]: += g conj(lambda^L)
+    float2 *part_j;                // [B*D][M]: conj(g) J
+    const __nv_bfloat16 *xT;       // [B*D][Lp] channel-major x (the partial chunk's direct sum)
+    __nv_bfloat16 *dxT;            // [B*D][Lp]: += the g term of dx
+    int64_t L, Lp;
+    int D, M, ntiles;
+};
+
+__global__ void __launch_bounds__(kTmThreads, 2)
+    k_terminal_tc(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_dx,
+                  const TermArgs args) {
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t *smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+    const uint32_t sbase = smem_u32(smem);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int row = blockIdx.x;     // b * D + d
+    const int d = row % args.D;
+    const int M = args.M, ntiles = args.ntiles;
+    const int64_t L = args.L;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kTmOffBar);
+    auto bar = [&](int i) { return smem_u32(bars + i); };
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(smem + kTmOffMisc);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + kTmOffMisc + 16);
+    float2 *pw = reinterpret_cast<float2 *>(smem + kTmOffPw);
+    float2 *gs = reinterpret_cast<float2 *>(smem + kTmOffG);
+
+    if (tid == 0) {
+        *abort_flag = 0;
+        for (int i = 0; i < kTmSlots; ++i) {
+            bar_init(bar(kTmSlotFull + i), 1);
+            bar_init(bar(kTmSlotEmpty + i), 3);
+        }
+        for (int i = 0; i < 2; ++i) {
+            bar_init(bar(kTmPFull + i), 1);
+            bar_init(bar(kTmPEmpty + i), 4);
+            bar_init(bar(kTmWFull + i), 4);
+            bar_init(bar(kTmWEmpty + i), 1);
+            bar_init(bar(kTmDFull + i), 1);
+            bar_init(bar(kTmDEmpty + i), 2);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 6) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(kTmCols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    // lambda^s for s = 0..64 per mode slot (zero past M): thread (m, e) forms
+    // s = 8 e .. 8 e + 7 (and s = 64 for e = 7) as one exact power and products.
+    {
+        const int m = tid >> 3, e = tid & 7;
+        float2 *o = pw + m * kPwStride + 8 * e;
+        if (m < M) {
+            const float ga = args.decay[d * M + m], om = args.freq[d * M + m];
+            const float2 l1 = lambda_pow(ga, om, 1.0f);
+            float2 z = lambda_pow(ga, om, (float)(8 * e));
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                o[k] = z;
+                z = cmul(z, l1);
+            }
+            if (e == 7) o[8] = z;
+        } else {
+#pragma unroll
+            for (int k = 0; k < 8; ++k) o[k] = make_float2(0.0f, 0.0f);
+            if (e == 7) o[8] = make_float2(0.0f, 0.0f);
+        }
+        if (tid < kMaxModes) gs[tid] = tid < M ? args.g[(int64_t)row * M + tid] : make_float2(0.0f, 0.0f);
+        // x of the chunk holding token L - 1 when it does not end there.
+        if (tid >= 64 && tid < 64 + kC && (L % kC) != 0) {
+            const int64_t j = (L - 1) / kC * kC + (tid - 64);
+            reinterpret_cast<float *>(smem + kTmOffXp)[tid - 64] =
+                j < L ? __bfloat162float(args.xT[(int64_t)row * args.Lp + j]) : 0.0f;
+        }
+    }
+    __syncthreads();
+    // The tables (K index k = position i within the chunk; value at lambda^(63-k)):
+    //   A rows as A_P (row r: mode 8 (r / 32) + (r % 16) / 2, Re/Im by r % 2;
+    //   r % 32 < 16: lambda^(63-k), else (63-k) lambda^(63-k)), low parts of the
+    //   first kind into the M = 64 table;
+    //   U_g[k][2m + ri] = Re lambda_m^(63-k), -Im lambda_m^(63-k).
+    for (int t = tid; t < 1024 + 512; t += kTmThreads) {
+        if (t < 1024) {
+            const int kg = t >> 7, r = t & 127;
+            const int l = r & 31, m = 8 * (r >> 5) + ((l & 15) >> 1), ri = l & 1;
+            const bool jordan = l >= 16;
+            uint32_t hi[4], lo[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                float v[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int k = 8 * kg + 2 * e + u;
+                    const float2 p = pw[m * kPwStride + (kC - 1 - k)];
+                    const float w = ri ? p.y : p.x;
+                    v[u] = jordan ? (float)(kC - 1 - k) * w : w;
+                }
+                hi[e] = pack_bf16x2(v[0], v[1]);
+                lo[e] = pack_bf16x2(v[0] - __uint_as_float(hi[e] << 16), v[1] - __uint_as_float(hi[e] & 0xffff0000u));
+            }
+            st_shared_v4(sbase + kTmOffA + kmaj(r, 8 * kg), hi[0], hi[1], hi[2], hi[3]);
+            if (!jordan) st_shared_v4(sbase + kTmOffAlo + kmaj(16 * (r >> 5) + l, 8 * kg), lo[0], lo[1], lo[2], lo[3]);
+        } else {
+            const int u = t - 1024, kg = u >> 6, k = u & 63;
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float2 z = pw[(4 * kg + e) * kPwStride + (kC - 1 - k)];
+                w[e] = pack_bf16x2(z.x, -z.y);
+            }
+            st_shared_v4(sbase + kTmOffU + kmaj(k, 8 * kg), w[0], w[1], w[2], w[3]);
+        }
+    }
+    fence_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+    const int last = ntiles - 1;
+    // The chunk holding token L - 1 when it does not end there (-1: none).
+    const int64_t n_part = (L % kC) ? (L - 1) / kC : -1;
+
+    if (warp < 4) {
+        // ---------------------------------------------------- weights, W, J
+        const int q = warp, l = lane;
+        const int m = 8 * q + ((l & 15) >> 1), ri = l & 1;
+        const bool jordan = l >= 16, on = m < M;
+        const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
+        const float gam = on ? args.decay[d * M + m] : 0.0f, omg = on ? args.freq[d * M + m] : 0.0f;
+        const float2 l64 = lambda_pow(gam, omg, (float)kC), l2048 = lambda_pow(gam, omg, (float)kTile);
+        const float2 l512 = lambda_pow(gam, omg, 512.0f), l1024 = lambda_pow(gam, omg, 1024.0f),
+                     l1536 = lambda_pow(gam, omg, 1536.0f);
+        const float2 gc = on ? conj2(gs[m]) : make_float2(0.0f, 0.0f);
+        const int prow = 32 * q + l;     // this lane's W row (rows with l < 16)
+        // The last chunk that ends at or before token L - 1 (-1: none).
+        const int64_t nfull = L >= kC ? (L - kC) / kC : -1;
+        float jr[4] = {0.0f, 0.0f, 0.0f, 0.0f}, ji[4] = {0.0f, 0.0f, 0.0f, 0.0f};   // this lane's share of conj(g) J
+        float2 T = make_float2(0.0f, 0.0f);   // lambda^E of the next tile's chunk 31, once known
+        bool haveT = false;
+        bool ok = true;
+        for (int v = 0; v < ntiles && ok; ++v) {
+            const int bb = v & 1;
+            const int64_t n0 = (int64_t)(last - v) * kNT;   // the tile's first chunk
+            // Weights W_n = conj(g) lambda^E_n of the tile's chunks, E_n = L - 64 - 64 n
+            // (zero where E_n < 0), from the tile's last full chunk ctop down by steps
+            // of lambda^64.  lambda^E at ctop is an exact power in the first one or
+            // two tiles (E < 4200); after that chunk 31's comes from the previous
+            // tile's by one step of lambda^2048.
+            const int64_t ctop64 = nfull - n0;
+            const int ctop = ctop64 < 0 ? -1 : (ctop64 > kNT - 1 ? kNT - 1 : (int)ctop64);
+            float2 z = make_float2(0.0f, 0.0f);
+            if (ctop >= 0) {
+                const float2 a = (ctop == kNT - 1 && haveT) ? T : lambda_pow(gam, omg, (float)(L - kC - kC * (n0 + ctop)));
+                if (ctop == kNT - 1) {
+                    T = cmul(a, l2048);
+                    haveT = true;
+                }
+                z = cmul(gc, a);
+            }
+            float2 w[kNT];
+            if (ctop == kNT - 1) {
+                // A full tile: four independent chains of eight steps.
+                float2 z1 = cmul(z, l512), z2 = cmul(z, l1024), z3 = cmul(z, l1536);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    w[31 - k] = z;
+                    w[23 - k] = z1;
+                    w[15 - k] = z2;
+                    w[7 - k] = z3;
+                    z = cmul(z, l64);
+                    z1 = cmul(z1, l64);
+                    z2 = cmul(z2, l64);
+                    z3 = cmul(z3, l64);
+                }
+            } else {
+#pragma unroll
+                for (int c = kNT - 1; c >= 0; --c) {
+                    if (c > ctop) {
+                        w[c] = make_float2(0.0f, 0.0f);
+                    } else {
+                        w[c] = z;
+                        z = cmul(z, l64);
+                    }
+                }
+            }
+            // W rows (Re / Im of W_n) for the dx product.
+            if (!wait_bar(bar(kTmWEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
+            if (!jordan) {
+                const uint32_t wb = sbase + kTmOffW + bb * 8192;
+#pragma unroll
+                for (int g8 = 0; g8 < kNT / 8; ++g8) {
+                    uint32_t h[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 a0 = w[8 * g8 + 2 * e], a1 = w[8 * g8 + 2 * e + 1];
+                        h[e] = ri ? pack_bf16x2(a0.y, a1.y) : pack_bf16x2(a0.x, a1.x);
+                    }
+                    st_shared_v4(wb + pairoff(prow, g8), h[0], h[1], h[2], h[3]);
+                }
+            }
+            fence_async_smem();
+            __syncwarp();
+            if (lane == 0) bar_arrive(bar(kTmWFull + bb));
+            // conj(g) J from this lane's projection row: value v_n (Re or Im of p_n or
+            // q_n) enters as W_n f_n v_n (times i for an Im row), f_n = E_n for p, 1 for q.
+            if (!wait_bar(bar(kTmPFull + bb), (v >> 1) & 1, abort_flag)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            uint32_t pa[16], pb[16];
+            tmem_ld16(tl + kTmColP + 32 * bb, pa);
+            tmem_ld16(tl + kTmColP + 32 * bb + 16, pb);
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) bar_arrive(bar(kTmPEmpty + bb));
+            // E_n as fp32 (exact below 2^24): one 64-bit conversion per tile.
+            const float e0 = (float)(L - kC - kC * n0);
+#pragma unroll
+            for (int c = 0; c < kNT; ++c) {
+                const float f = jordan ? 1.0f : fmaf(-(float)kC, (float)c, e0);
+                const float val = __uint_as_float(c < 16 ? pa[c] : pb[c - 16]) * f;
+                // (ri ? i : 1) * w * val, four accumulators
+                jr[c & 3] = fmaf(ri ? -w[c].y : w[c].x, val, jr[c & 3]);
+                ji[c & 3] = fmaf(ri ? w[c].x : w[c].y, val, ji[c & 3]);
+            }
+        }
+        // The chunk holding token L - 1 (L % 64 != 0): its part of J directly, one
+        // lane per mode.
+        if (ok && on && !jordan && ri == 0 && n_part >= 0) {
+            const float *xp = reinterpret_cast<const float *>(smem + kTmOffXp);
+            const int cnt = (int)(L - n_part * kC);   // tokens of the chunk before L
+            float pr = 0.0f, pi = 0.0f;
+            for (int i = 0; i < cnt; ++i) {
+                const int s = cnt - 1 - i;
+                const float xv = xp[i] * (float)s;
+                const float2 p = pw[m * kPwStride + s];
+                pr = fmaf(p.x, xv, pr);
+                pi = fmaf(p.y, xv, pi);
+            }
+            const float2 t = cmul(gc, make_float2(pr, pi));
+            jr[0] += t.x;
+            ji[0] += t.y;
+        }
+        float jsr = (jr[0] + jr[1]) + (jr[2] + jr[3]), jsi = (ji[0] + ji[1]) + (ji[2] + ji[3]);
+        // The mode's four rows, then the state terms.
+        jsr += __shfl_xor_sync(0xffffffffu, jsr, 1);
+        jsi += __shfl_xor_sync(0xffffffffu, jsi, 1);
+        jsr += __shfl_xor_sync(0xffffffffu, jsr, 16);
+        jsi += __shfl_xor_sync(0xffffffffu, jsi, 16);
+        if (ok && on && !jordan && ri == 0) {
+            const float2 lL = lambda_pow(gam, omg, (float)L);
+            float2 J = make_float2(jsr, jsi);   // conj(g) J
+            const int64_t at = (int64_t)row * M + m;
+            if (args.state_in) {
+                const float2 t = cmul(gc, cmul(args.state_in[at], lL));
+                J = make_float2(fmaf((float)L, t.x, J.x), fmaf((float)L, t.y, J.y));
+            }
+            args.part_j[at] = J;
+            if (args.d_state_in) {
+                const float2 gg = gs[m], prev = args.d_state_in[at];
+                args.d_state_in[at] = cfma(gg, conj2(lL), prev);
+            }
+        }
+    } else if (warp < 6) {
+        // ---------------------------------------------------- dx epilogue
+        const int q = warp & 3;   // positions 32 q + lane
+        const int i = 32 * q + lane;
+        const uint32_t tl = tmem + ((uint32_t)(32 * q) << 16);
+        for (int v = 0; v < ntiles; ++v) {
+            const int bb = v & 1, slot = v % kTmSlots;
+            // The old dx values of this tile (plain [chunk][position] layout).
+            if (!wait_bar(bar(kTmSlotFull + slot), (v / kTmSlots) & 1, abort_flag)) break;
+            const __nv_bfloat16 *sdx =
+                reinterpret_cast<const __nv_bfloat16 *>(smem + kTmOffRing + slot * kTmSlotBytes + 4096) + i;
+            float prev[kNT];
+#pragma unroll
+            for (int c = 0; c < kNT; ++c) prev[c] = __bfloat162float(sdx[c * kC]);
+            __syncwarp();
+            if (lane == 0) bar_arrive(bar(kTmSlotEmpty + slot));
+            if (!wait_bar(bar(kTmDFull + bb), (v >> 1) & 1, abort_flag)) break;
+            tc_fence_after();
+            uint32_t r0[16], r1[16];
+            tmem_ld16(tl + kTmColD + 32 * bb, r0);
+            tmem_ld16(tl + kTmColD + 32 * bb + 16, r1);
+            tmem_wait_ld();
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) bar_arrive(bar(kTmDEmpty + bb));
+            const int64_t n0 = (int64_t)(last - v) * kNT;
+            float add[kNT];
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+                add[c] = __uint_as_float(r0[c]);
+                add[c + 16] = __uint_as_float(r1[c]);
+            }
+            // The chunk holding token L - 1 (weight zero in the product): direct sum.
+            if (n_part >= n0 && n_part < n0 + kNT) {
+                const int64_t j = n_part * kC + i;
+                float fx = 0.0f;
+                if (j < L) {
+                    const int s = (int)(L - 1 - j);
+                    for (int mm = 0; mm < M; ++mm) {
+                        const float2 p = pw[mm * kPwStride + s], gg = gs[mm];
+                        fx = fmaf(gg.x, p.x, fmaf(gg.y, p.y, fx));   // Re(conj(g) lambda^s)
+                    }
+                }
+                const int cp = (int)(n_part - n0);
+#pragma unroll
+                for (int c = 0; c < kNT; ++c)
+                    if (c == cp) add[c] += fx;
+            }
+            // dxT += add (one more bf16 rounding of the main pass's dx, well
+            // inside the bf16 tolerance).
+            __nv_bfloat16 *out = args.dxT + (int64_t)row * args.Lp + n0 * kC + i;
+#pragma unroll
+            for (int c = 0; c < kNT; ++c) out[c * kC] = __float2bfloat16_rn(prev[c] + add[c]);
+        }
+    } else if (warp == 6) {
+        // ---------------------------------------------------- TMA producer
+        if (lane == 0) {
+            int issued = 0;
+            for (; issued < ntiles; ++issued) {
+                const int slot = issued % kTmSlots;
+                if (!wait_bar(bar(kTmSlotEmpty + slot), ((issued / kTmSlots) & 1) ^ 1, abort_flag)) break;
+                bar_expect_tx(bar(kTmSlotFull + slot), 8192u);
+                tma_load_3d(sbase + kTmOffRing + slot * kTmSlotBytes, &tmap_x, 0, (last - issued) * kNT, row,
+                            bar(kTmSlotFull + slot));
+                tma_load_3d(sbase + kTmOffRing + slot * kTmSlotBytes + 4096, &tmap_dx, 0, (last - issued) * kNT, row,
+                            bar(kTmSlotFull + slot));
+            }
+            for (int k = issued > kTmSlots ? issued - kTmSlots : 0; k < issued; ++k)
+                drain_bar(bar(kTmSlotFull + k % kTmSlots), (k / kTmSlots) & 1);
+        }
+        __syncwarp();
+    } else {
+        // ---------------------------------------------------- MMA issue
+        if (lane == 0) {
+            const uint64_t da = desc_plain(sbase + kTmOffA, 128, 1024);
+            const uint64_t dal = desc_plain(sbase + kTmOffAlo, 128, 1024);
+            const uint64_t du = desc_plain(sbase + kTmOffU, 128, 1024);
+            int last_bar = -1;
+            uint32_t last_par = 0;
+            for (int v = 0; v < ntiles; ++v) {
+                const int slot = v % kTmSlots, bb = v & 1;
+                if (!wait_bar(bar(kTmSlotFull + slot), (v / kTmSlots) & 1, abort_flag)) break;
+                if (!wait_bar(bar(kTmPEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
+                tc_fence_after();
+                const uint64_t dx = desc_sw128(sbase + kTmOffRing + slot * kTmSlotBytes, 16, 1024);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kTmColP + 32 * bb, da + ks * 16, dx + ks * 2, kIdescN32, ks > 0);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kTmColP + 32 * bb, dal + ks * 16, dx + ks * 2, kIdescN32M64, 1u);
+                umma_commit(bar(kTmPFull + bb));
+                umma_commit(bar(kTmSlotEmpty + slot));
+                last_bar = kTmSlotEmpty + slot;
+                last_par = (v / kTmSlots) & 1;
+                if (!wait_bar(bar(kTmWFull + bb), (v >> 1) & 1, abort_flag)) break;
+                if (!wait_bar(bar(kTmDEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
+                tc_fence_after();
+                const uint64_t dw = desc_plain(sbase + kTmOffW + bb * 8192, 512, 128);
+#pragma unroll
+                for (int ks = 0; ks < 4; ++ks)
+                    umma_ss(tmem + kTmColD + 32 * bb, du + ks * 16, dw + ks * (2048 >> 4), kIdescU, ks > 0);
+                umma_commit(bar(kTmDFull + bb));
+                umma_commit(bar(kTmWEmpty + bb));
+                last_bar = kTmWEmpty + bb;
+                last_par = (v >> 1) & 1;
+            }
+            // Drain: the last commit's completion implies every earlier product's.
+            if (last_bar >= 0) drain_bar(bar(last_bar), last_par);
+        }
+        __syncwarp();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 6)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmCols));
 }
 
 // ------------------------------------------------------------ layout transposes
@@ -1050,8 +1442,8 @@ EncodeTiledFn encode_fn() {
 
 // 3-D map over a channel-major [rows][Lp] bf16 field viewed as (64 positions,
 // Lp / 64 chunks, rows); box = one tile of one row (64 x 32 x 1), loaded with the
-// 128-byte swizzle of the UMMA operand layout.
-bool make_chunk_map(CUtensorMap *map, const void *ptr, int64_t rows, int64_t Lp) {
+// 128-byte swizzle of the UMMA operand layout, or plain ([chunk][position]).
+bool make_chunk_map(CUtensorMap *map, const void *ptr, int64_t rows, int64_t Lp, bool swizzle = true) {
     EncodeTiledFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)kC, (cuuint64_t)(Lp / kC), (cuuint64_t)rows};
@@ -1059,7 +1451,7 @@ bool make_chunk_map(CUtensorMap *map, const void *ptr, int64_t rows, int64_t Lp)
     cuuint32_t box[3] = {(cuuint32_t)kC, (cuuint32_t)kNT, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(ptr), dims, strides, box, estr,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -1081,7 +1473,7 @@ bool tc_backward_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
 }
 
 size_t tc_backward_ws_bytes(int64_t B, int64_t L, int D, int M) {
-    return 3 * field_bytes(B, L, D) + 4 * part_bytes(B, D, M);   // + the terminal-state pass's partials
+    return 3 * field_bytes(B, L, D) + 3 * part_bytes(B, D, M);   // G, P and conj(g) J partials
 }
 
 namespace {
@@ -1097,6 +1489,8 @@ cudaError_t configure_once() {
         cudaError_t e = cudaFuncSetAttribute(k_backward_tc<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(k_backward_tc<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(k_terminal_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kTmSmemBytes);
         if (e != cudaSuccess) return e;
         configured[dev] = 1;
     }
@@ -1116,8 +1510,6 @@ BwdArgs base_args(const float *decay, const float *freq, const float *amp, const
     a.state_out = nullptr;
     a.coef_out = nullptr;
     a.d_state_in = nullptr;
-    a.cconj = nullptr;
-    a.acc_dx = 0;
     a.dxT = outT;
     a.Lp = Lp;
     a.D = D;
@@ -1154,21 +1546,6 @@ cudaError_t run_layout_and_scan(const CUtensorMap &mdy, const CUtensorMap &mx, B
 
 }  // namespace
 
-// The terminal-state pass's drive in the last tile of every row: 1 at token L-1,
-// 0 elsewhere (the pass reads no other tile of it).  Block r writes row r's last
-// tile, 16 bytes per thread.
-__global__ void k_unit_last(__nv_bfloat16 *dT, int64_t Lp, int64_t L) {
-    const int64_t r = blockIdx.x;
-    const int64_t t0 = Lp - kTile + 8 * (int64_t)threadIdx.x;   // 256 threads x 8 tokens
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (L - 1 >= t0 && L - 1 < t0 + 8) {
-        __nv_bfloat16 e[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) e[k] = __float2bfloat16_rn(t0 + k == L - 1 ? 1.0f : 0.0f);
-        v = *reinterpret_cast<const uint4 *>(e);
-    }
-    *reinterpret_cast<uint4 *>(dT + r * Lp + t0) = v;
-}
 
 cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int64_t L, int D, int M,
                         const float *decay, const float *freq, const float *amp, const float *phase,
@@ -1182,8 +1559,7 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     auto *dxT = reinterpret_cast<__nv_bfloat16 *>(w + 2 * field_bytes(B, L, D));
     auto *pg = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D));
     auto *pp = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + part_bytes(B, D, M));
-    auto *pg2 = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + 2 * part_bytes(B, D, M));
-    auto *pj = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + 3 * part_bytes(B, D, M));
+    auto *pj = reinterpret_cast<float2 *>(w + 3 * field_bytes(B, L, D) + 2 * part_bytes(B, D, M));
     const int64_t rows = B * (int64_t)D;
     CUtensorMap mdy, mx;
     if (!make_chunk_map(&mdy, dyT, rows, Lp) || !make_chunk_map(&mx, xT, rows, Lp)) return cudaErrorInvalidValue;
@@ -1202,26 +1578,34 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
     } else {
         // A terminal-state gradient g adds Re(conj(g) lambda^(L-1-t)) to dx_t,
         // conj(g) J to the decay / frequency products and g conj(lambda^L) to the
-        // gradient of s_in (Sec. 3.2-3.3).  These are exactly what the same
-        // backward gives for a unit drive at token L-1 read through c = conj(g)
-        // (per batch row): its dx, c P (P = J with the s_in term) and
-        // conj(c lambda S_0).  So a second pass of the kernel runs on that drive,
-        // reusing the channel-major x and adding its dx to the first pass's in
-        // the channel-major buffer; one transpose then writes the sum.
+        // gradient of s_in (Sec. 3.2-3.3).  After the main pass, k_terminal_tc
+        // forms them in closed form (no scan) from the channel-major x and adds
+        // its dx to the main pass's in the channel-major buffer; one transpose
+        // then writes the sum.
         const unsigned cg = (unsigned)((D + 63) / 64);
         k_to_channel_major<<<dim3((unsigned)(Lp / 64), cg, (unsigned)(B * 2)), 128, 0, st>>>(
             static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp, 2, 0,
             0, 0, D);
         k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a);
-        k_unit_last<<<(unsigned)rows, kTile / 8, 0, st>>>(dyT, Lp, L);
-        BwdArgs a2 = a;
-        a2.part_g = pg2;
-        a2.part_p = pj;
-        a2.cconj = reinterpret_cast<const float2 *>(d_state_out);
-        a2.acc_dx = 1;
-        k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a2);
+        TermArgs ta;
+        ta.decay = decay;
+        ta.freq = freq;
+        ta.g = reinterpret_cast<const float2 *>(d_state_out);
+        ta.state_in = reinterpret_cast<const float2 *>(state_in);
+        ta.d_state_in = reinterpret_cast<float2 *>(d_state_in);
+        ta.part_j = pj;
+        ta.xT = xT;
+        ta.dxT = dxT;
+        ta.L = L;
+        ta.Lp = Lp;
+        ta.D = D;
+        ta.M = M;
+        ta.ntiles = (int)(Lp / kTile);
+        CUtensorMap mdx;
+        if (!make_chunk_map(&mdx, dxT, rows, Lp, false)) return cudaErrorInvalidValue;
+        k_terminal_tc<<<(unsigned)rows, kTmThreads, kTmSmemBytes, st>>>(mx, mdx, ta);
         row_major_wide(dxT, static_cast<__nv_bfloat16 *>(dx), B, L, D, Lp, st);
-        count_launches(5);   // transpose, pass, unit drive, pass, transpose
+        count_launches(4);   // transpose, pass, terminal-state terms, transpose
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     return grad_reduce(rows / D, D, M, amp, phase, pg, pp, d_state_out ? pj : nullptr, g_decay, g_freq, g_amp,

@@ -301,15 +301,15 @@ def test_workspace_queries_are_host_only_and_monotone(lib):
 def test_tensor_core_backward_workspace(lib):
     # bf16 I/O with M <= 32 runs the tensor-core backward: channel-major copies of
     # x, dy and dx ([B*D][Lp] bf16, Lp = L rounded up to 2048-token tiles, each
-    # rounded up to 1 KiB) plus the per-(b, d, m) partial sums of G and P, for the
-    # main pass and for the terminal-state pass.
+    # rounded up to 1 KiB) plus the per-(b, d, m) partial sums of G and P of the
+    # main pass and of conj(g) J of the terminal-state terms.
     B, L, D, M = 4, 32768, 512, 32
     field = B * D * L * 2
-    parts = 4 * B * D * M * 8
+    parts = 3 * B * D * M * 8
     assert rlm.rlm_backward_workspace_size(B, L, D, M, rlm.RLM_BF16) == 3 * field + parts
     B, L, D, M = 1, 2049, 8, 5
     field = (B * D * 4096 * 2 + 1023) // 1024 * 1024
-    parts = 4 * ((B * D * M * 8 + 255) // 256 * 256)
+    parts = 3 * ((B * D * M * 8 + 255) // 256 * 256)
     assert rlm.rlm_backward_workspace_size(B, L, D, M, rlm.RLM_BF16) == 3 * field + parts
     # fp32 I/O and M > 32 keep the SIMT path and its chunk workspace.
     assert rlm.rlm_backward_workspace_size(4, 32768, 512, 32, rlm.RLM_F32) < 3 * 4 * 512 * 32768 * 2

@@ -499,7 +499,7 @@ def test_backward_matches_oracle(B, L, D, M, dtype):
     (1, 2 * 2048 + 1, 8, 32, "bf16", True, False),
     (3, 65, 8, 5, "bf16", True, False),
     (2, 3001, 16, 16, "bf16", False, False),
-    # ... with a terminal-state gradient (the second pass on a unit drive at L-1)
+    # ... with a terminal-state gradient (the closed-form terminal-state launch)
     (2, 3001, 16, 16, "bf16", True, True),
     (1, 700, 8, 32, "bf16", False, True),
     (3, 65, 8, 5, "bf16", True, True),
@@ -547,7 +547,8 @@ def test_backward_with_state_terms_matches_oracle(B, L, D, M, dtype, with_s, wit
 def test_terminal_gradient_with_silent_modes_matches_oracle(decay_scale, L):
     """A terminal-state gradient reaches modes with zero amplitude (c = 0: they add
     nothing to y, but the terminal state still depends on them), and fast decays
-    with a ragged sequence end (the tensor-core route's second pass)."""
+    with a ragged sequence end (the chunk holding token L - 1, summed directly
+    on the tensor-core route)."""
     B, D, M = 2, 16, 16
     inp = make_inputs(B, L, D, M, "bf16", seed=L, with_dy=True)
     decay, freq, amp, phase = (a.copy() for a in inp.params())
@@ -563,6 +564,37 @@ def test_terminal_gradient_with_silent_modes_matches_oracle(decay_scale, L):
     torch.cuda.synchronize()
     dx_ref, g_ref = oracle.backward_rec(inp.x, inp.dy, decay, freq, amp, phase, state_in=s_in,
                                         d_state_out=g_out)
+    assert_close(to_np(dx), dx_ref, TOL["bf16"], "dx")
+    for k in ("decay", "freq", "amp", "phase"):
+        assert_close(getattr(g, k).cpu().numpy(), g_ref[k], TOL["bf16"], "d" + k)
+    ds_np = ds.complex().cpu().numpy()
+    assert_close(ds_np.real, g_ref["state_in"].real, TOL["bf16"], "dstate_in re")
+    assert_close(ds_np.imag, g_ref["state_in"].imag, TOL["bf16"], "dstate_in im")
+
+
+@pytest.mark.parametrize("L,M,with_s", [
+    (63, 7, False),            # no chunk ends before L: all of it from the direct sum
+    (64, 32, True),            # one chunk ending exactly at L - 1
+    (2049, 32, False),         # the last tile holds only the one-token chunk
+    (4095, 5, True),           # a ragged chunk inside the last tile
+    (3 * 2048 + 100, 32, True),  # weights carried across tiles by lambda^2048
+])
+def test_terminal_state_terms_at_tile_edges(L, M, with_s):
+    """The terminal-state terms of the tcgen05 backward (dx, the decay and frequency
+    gradients through conj(g) J, the gradient of s_in) at the chunk and tile edges
+    of its closed form, against the recurrence oracle."""
+    B, D = 2, 8
+    inp = make_inputs(B, L, D, M, "bf16", seed=L + 3 * M, with_dy=True)
+    rng = np.random.default_rng(L + M)
+    g_out = rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M))
+    s_in = rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M)) if with_s else None
+    x, dy = to_dev(inp.x, "bf16"), to_dev(inp.dy, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    dx, g, ds = torch.empty_like(x), rlm.Grads.empty(D, M), rlm.State.empty(B, D, M)
+    rlm.rlm_mix_backward_from(dy, x, p, _state_from(inp, s_in) if with_s else None, _state_from(inp, g_out),
+                              dx, g, ds)
+    torch.cuda.synchronize()
+    dx_ref, g_ref = oracle.backward_rec(inp.x, inp.dy, *inp.params(), state_in=s_in, d_state_out=g_out)
     assert_close(to_np(dx), dx_ref, TOL["bf16"], "dx")
     for k in ("decay", "freq", "amp", "phase"):
         assert_close(getattr(g, k).cpu().numpy(), g_ref[k], TOL["bf16"], "d" + k)
