@@ -578,6 +578,7 @@ def test_terminal_gradient_with_silent_modes_matches_oracle(decay_scale, L):
     (2049, 32, False),         # the last tile holds only the one-token chunk
     (4095, 5, True),           # a ragged chunk inside the last tile
     (3 * 2048 + 100, 32, True),  # weights carried across tiles by lambda^2048
+    (2 ** 18 + 77, 8, True),   # ... over 128 tiles
 ])
 def test_terminal_state_terms_at_tile_edges(L, M, with_s):
     """The terminal-state terms of the tcgen05 backward (dx, the decay and frequency
