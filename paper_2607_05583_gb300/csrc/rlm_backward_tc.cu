@@ -757,18 +757,21 @@ __global__ void __launch_bounds__(kThreads, 2)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(kTmemCols));
     if (kGrad && warp < 4) {
-        // Within-chunk terms: lags n = s, s + 4, ... from rho (two partial arrays),
-        // then the sum over the mode's four lanes; role 0 writes the partials.
+        // Within-chunk terms: lags n = s, s + 4, ... from rho, then the sum over
+        // the mode's four lanes; role 0 writes the partials.  lambda^n by steps of
+        // lambda^4 from the exact lambda^s (at most 15 products).
         const float *rho = reinterpret_cast<const float *>(smem + kOffRho);
+        const float2 l4 = lambda_pow(gamE, omgE, 4.0f);
+        float2 ln = lambda_pow(gamE, omgE, (float)s);
 #pragma unroll 4
         for (int e = 0; e < kC / 4; ++e) {
             const int n = 4 * e + s;
             const float r = rho[n];
-            const float2 ln = lambda_pow(gamE, omgE, (float)n);
             gr = fmaf(r, ln.x, gr);
             gi = fmaf(r, ln.y, gi);
             pr = fmaf(r * (float)n, ln.x, pr);
             pi = fmaf(r * (float)n, ln.y, pi);
+            ln = cmul(ln, l4);
         }
         // The forward's initial state s_in (Sec. 3.2-3.3): G += s_in lambda S_0,
         // P += s_in lambda (R_0 + S_0), added once per mode before the lanes' sum; the
