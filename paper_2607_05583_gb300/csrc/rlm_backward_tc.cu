@@ -824,10 +824,11 @@ __global__ void __launch_bounds__(kThreads, 2)
 // token L - 1 without ending there (L % 64 != 0) is evaluated directly in fp32,
 // so no negative power of lambda is ever formed.  One CTA per row, walking the
 // tiles from the end of the sequence:
-//   warps 0-3  per tile: the chunk weights lambda^E_n (an exact power at the
-//              tile's first full chunk, then steps of lambda^64), the W rows,
-//              and J from the projections (each lane weights its own TMEM row,
-//              the mode's four rows are added at the end);
+//   warps 0-3  per tile: the chunk weights W_n = conj(g) lambda^E_n (steps of
+//              lambda^64 in four chains; each tile's first weight carried from
+//              the previous tile by lambda^2048), the W rows, and conj(g) J from
+//              the projections (each lane weights its own TMEM row, the mode's
+//              four rows are added at the end);
 //   warps 4-5  dx epilogue: dxT += dx (positions 0-63; the old values come
 //              with the x tile, so no global read waits in the loop);
 //   warp 6     TMA producer (per slot: the x tile, swizzled for the product, and
@@ -1252,18 +1253,17 @@ __global__ void __launch_bounds__(kTmThreads, 2)
 
 // ------------------------------------------------------------ layout transposes
 // [B][L][D] -> [B*D][Lp], zero for positions >= L.  Grid z = rows * nf: field f of
-// batch row b0 + z / nf is (src0, dst0) or (src1, dst1); channels from c_lo, below
-// c_hi.  rev: position s holds token L - 1 - s (time reversed within [0, L)).
+// batch row z / nf is (src0, dst0) or (src1, dst1).  rev: position s holds token
+// L - 1 - s (time reversed within [0, L)).
 __global__ void __launch_bounds__(128) k_to_channel_major(const __nv_bfloat16 *__restrict__ src0,
                                                           const __nv_bfloat16 *__restrict__ src1,
                                                           __nv_bfloat16 *__restrict__ dst0,
                                                           __nv_bfloat16 *__restrict__ dst1, int64_t L, int D,
-                                                          int64_t Lp, int nf, int rev, int b0, int c_lo,
-                                                          int c_hi) {
+                                                          int64_t Lp, int nf, int rev) {
     __shared__ uint32_t tile[64][33];   // [position][channel pair]
     const int64_t t0 = (int64_t)blockIdx.x * 64;
-    const int c0 = c_lo + blockIdx.y * 64;
-    const int b = b0 + blockIdx.z / nf, f = blockIdx.z % nf;
+    const int c0 = blockIdx.y * 64;
+    const int b = blockIdx.z / nf, f = blockIdx.z % nf;
     const __nv_bfloat16 *src = f ? src1 : src0;
     __nv_bfloat16 *dst = f ? dst1 : dst0;
     // Four 16-byte loads per thread, all issued before the tile is written.
@@ -1275,7 +1275,7 @@ __global__ void __launch_bounds__(128) k_to_channel_major(const __nv_bfloat16 *_
         const int64_t sp = t0 + r;
         const int c = c0 + 8 * vq;
         val[k] = make_uint4(0, 0, 0, 0);
-        if (sp < L && c < c_hi) {
+        if (sp < L && c < D) {
             const int64_t t = rev ? L - 1 - sp : sp;
             val[k] = __ldg(reinterpret_cast<const uint4 *>(src + ((int64_t)b * L + t) * D + c));
         }
@@ -1293,7 +1293,7 @@ __global__ void __launch_bounds__(128) k_to_channel_major(const __nv_bfloat16 *_
     for (int it = threadIdx.x; it < 512; it += 128) {
         const int cr = it >> 3, vq = it & 7;
         const int c = c0 + cr;
-        if (c >= c_hi) continue;
+        if (c >= D) continue;
         uint32_t w[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
@@ -1311,11 +1311,11 @@ __global__ void __launch_bounds__(128) k_to_channel_major(const __nv_bfloat16 *_
 // 8-aligned window of 72 positions that holds its (reversed) positions.
 __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__restrict__ srcT,
                                                       __nv_bfloat16 *__restrict__ dst, int64_t L, int D,
-                                                      int64_t Lp, int rev, int b0, int c_lo, int c_hi) {
+                                                      int64_t Lp, int rev) {
     __shared__ uint32_t tile[64][37];   // [channel][position pair]
     const int64_t t0 = (int64_t)blockIdx.x * 64;
-    const int c0 = c_lo + blockIdx.y * 64;
-    const int b = b0 + blockIdx.z;
+    const int c0 = blockIdx.y * 64;
+    const int b = blockIdx.z;
     // First position of the window: t0 itself, or the last 64 tokens' mirror rounded down.
     const int64_t s_lo = rev ? ((L - t0 - 64) >= 0 ? (L - t0 - 64) & ~(int64_t)7 : -((t0 + 64 - L + 7) & ~(int64_t)7)) : t0;
     // A reversed window can straddle nine 8-position groups, a forward one is
@@ -1330,7 +1330,7 @@ __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__res
         const int c = c0 + cr;
         const int64_t sp = s_lo + 8 * vq;
         val[k] = make_uint4(0, 0, 0, 0);
-        if (it < nload && c < c_hi && sp >= 0 && sp < Lp)
+        if (it < nload && c < D && sp >= 0 && sp < Lp)
             val[k] = __ldg(reinterpret_cast<const uint4 *>(srcT + ((int64_t)b * D + c) * Lp + sp));
     }
 #pragma unroll
@@ -1348,7 +1348,7 @@ __global__ void __launch_bounds__(128) k_to_row_major(const __nv_bfloat16 *__res
         const int r = it >> 3, vq = it & 7;
         const int64_t t = t0 + r;
         const int c = c0 + 8 * vq;
-        if (t >= L || c >= c_hi) continue;
+        if (t >= L || c >= D) continue;
         const int i = (int)((rev ? L - 1 - t : t) - s_lo);   // 0 <= i < 72
         uint32_t w[4];
 #pragma unroll
@@ -1535,12 +1535,11 @@ cudaError_t run_layout_and_scan(const CUtensorMap &mdy, const CUtensorMap &mx, B
                                 const __nv_bfloat16 *outT, __nv_bfloat16 *out, cudaStream_t st) {
     const unsigned cg = (unsigned)((D + 63) / 64);
     k_to_channel_major<<<dim3((unsigned)(Lp / 64), cg, (unsigned)(B * nf)), 128, 0, st>>>(
-        src0, src1, dst0, dst1, L, D, Lp, nf, rev, 0, 0, D);
+        src0, src1, dst0, dst1, L, D, Lp, nf, rev);
     a.row0 = 0;
     k_backward_tc<kGrad><<<(unsigned)(B * D), kThreads, kSmemBytes, st>>>(mdy, mx, a);
     if (rev)
-        k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(outT, out, L, D, Lp, rev,
-                                                                                         0, 0, D);
+        k_to_row_major<<<dim3((unsigned)((L + 63) / 64), cg, (unsigned)B), 128, 0, st>>>(outT, out, L, D, Lp, rev);
     else
         row_major_wide(outT, out, B, L, D, Lp, st);
     count_launches(3);
@@ -1587,8 +1586,7 @@ cudaError_t tc_backward(const void *dy, const void *x, void *dx, int64_t B, int6
         // then writes the sum.
         const unsigned cg = (unsigned)((D + 63) / 64);
         k_to_channel_major<<<dim3((unsigned)(Lp / 64), cg, (unsigned)(B * 2)), 128, 0, st>>>(
-            static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp, 2, 0,
-            0, 0, D);
+            static_cast<const __nv_bfloat16 *>(x), static_cast<const __nv_bfloat16 *>(dy), xT, dyT, L, D, Lp, 2, 0);
         k_backward_tc<true><<<(unsigned)rows, kThreads, kSmemBytes, st>>>(mdy, mx, a);
         TermArgs ta;
         ta.decay = decay;
