@@ -697,6 +697,29 @@ def test_backward_is_deterministic():
         assert torch.equal(getattr(g1, k), getattr(g2, k))
 
 
+def test_backward_with_state_terms_is_deterministic():
+    """The tcgen05 backward with state_in and d_state_out (the main pass, then the
+    closed-form terminal-state launch) gives the same bits on every call."""
+    B, L, D, M = 2, 5000, 64, 32
+    inp = make_inputs(B, L, D, M, "bf16", seed=9, with_dy=True)
+    rng = np.random.default_rng(9)
+    g_out = rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M))
+    s_in = rng.standard_normal((B, D, M)) + 1j * rng.standard_normal((B, D, M))
+    x, dy = to_dev(inp.x, "bf16"), to_dev(inp.dy, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    outs = []
+    for _ in range(3):
+        dx, g, ds = torch.empty_like(x), rlm.Grads.empty(D, M), rlm.State.empty(B, D, M)
+        rlm.rlm_mix_backward_from(dy, x, p, _state_from(inp, s_in), _state_from(inp, g_out), dx, g, ds)
+        outs.append((dx, g, ds))
+    torch.cuda.synchronize()
+    for dx, g, ds in outs[1:]:
+        assert torch.equal(dx, outs[0][0])
+        for k in ("decay", "freq", "amp", "phase"):
+            assert torch.equal(getattr(g, k), getattr(outs[0][1], k))
+        assert torch.equal(ds.s, outs[0][2].s)
+
+
 def test_backward_gpu_finite_differences_tiny():
     """Gradients against central differences of the GPU's own fp32 forward at a tiny
     size (loss sum(dy * y)); loose bound because the forward is fp32."""
