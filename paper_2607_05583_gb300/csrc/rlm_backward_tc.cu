@@ -999,7 +999,7 @@ __global__ void __launch_bounds__(kTmThreads, 2)
         const float2 l512 = lambda_pow(gam, omg, 512.0f), l1024 = lambda_pow(gam, omg, 1024.0f),
                      l1536 = lambda_pow(gam, omg, 1536.0f);
         const float2 gc = on ? conj2(gs[m]) : make_float2(0.0f, 0.0f);
-        const int prow = 32 * q + l;     // this lane's W row (rows with l < 16)
+        const int prow = 32 * q + (l & 15);   // this lane's W row
         // The last chunk that ends at or before token L - 1 (-1: none).
         const int64_t nfull = L >= kC ? (L - kC) / kC : -1;
         float jr[4] = {0.0f, 0.0f, 0.0f, 0.0f}, ji[4] = {0.0f, 0.0f, 0.0f, 0.0f};   // this lane's share of conj(g) J
@@ -1053,17 +1053,20 @@ __global__ void __launch_bounds__(kTmThreads, 2)
             }
             // W rows (Re / Im of W_n) for the dx product.
             if (!wait_bar(bar(kTmWEmpty + bb), ((v >> 1) & 1) ^ 1, abort_flag)) break;
-            if (!jordan) {
+            {
+                // Lane l < 16 stores chunk groups 0-1 of its row, lane l + 16 (the same
+                // mode and component, so the same weights) groups 2-3.
                 const uint32_t wb = sbase + kTmOffW + bb * 8192;
 #pragma unroll
-                for (int g8 = 0; g8 < kNT / 8; ++g8) {
+                for (int gg = 0; gg < 2; ++gg) {
                     uint32_t h[4];
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
-                        const float2 a0 = w[8 * g8 + 2 * e], a1 = w[8 * g8 + 2 * e + 1];
+                        const float2 a0 = jordan ? w[16 + 8 * gg + 2 * e] : w[8 * gg + 2 * e];
+                        const float2 a1 = jordan ? w[16 + 8 * gg + 2 * e + 1] : w[8 * gg + 2 * e + 1];
                         h[e] = ri ? pack_bf16x2(a0.y, a1.y) : pack_bf16x2(a0.x, a1.x);
                     }
-                    st_shared_v4(wb + pairoff(prow, g8), h[0], h[1], h[2], h[3]);
+                    st_shared_v4(wb + pairoff(prow, gg + (jordan ? 2 : 0)), h[0], h[1], h[2], h[3]);
                 }
             }
             fence_async_smem();
