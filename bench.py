@@ -812,12 +812,16 @@ def run_kernels_only(args):
     time, for their ncu captures: each case runs 3 warm-up and 5 timed calls (L2
     flushed before each) and the line reports its mean time and algorithmic
     bytes.  Cases and the kernels they launch:
-      fp32_prefill        B=4 L=32768 D=256 M=16 fp32: k_chunk_local, k_chunk_carry, k_chunk_output
-      decode_b64 / b1     one plain decode step: k_decode_tile (B=64), k_decode_vec2 (B=1)
+      fp32_prefill        B=4 L=32768 D=256 M=16 fp32: k_prefill_tc32
+      fp32_prefill_state  the same with an initial state (the SIMT chunked scan):
+                          k_chunk_local, k_chunk_carry, k_chunk_output
+      decode_b64 / b1     one plain decode step: k_decode_tile
+      mixer_decode_plain  mixer step without coupling, B=64 D=2048 K=4 (rows past the
+                          one-block step): k_decode_vec2 (mixer)
       mixer_decode_b64    coupled mixer step H=8 K=4 (D=256): k_decode_coupled
       mixer_prefill_d2048 coupled mixer prefill B=1 L=32768 D=2048 H=8 K=4 (4 KB rows):
                           k_prefill_tc, k_couple_small, k_mixer_epilogue, k_mixer_tail
-      mixer_decode_d2048  coupled mixer step B=64 D=2048 H=8 K=4: k_decode_vec2 (mixer), k_mixer_finish"""
+      mixer_decode_d2048  coupled mixer step B=64 D=2048 H=8 K=4: k_decode_tile, k_mixer_finish"""
     import torch
 
     import paper_2607_05583_gb300 as rlm
@@ -849,17 +853,22 @@ def run_kernels_only(args):
         out[name] = {"ms": round(ms, 5), "algorithmic_bytes": alg_bytes, "achieved_GBps": round(gbs, 1),
                      "frac_hbm": round(gbs / hbm_peak, 4)}
 
-    # fp32 prefill on the SIMT chunked scan
+    # fp32 prefill: from a zero state on the tensor cores, from an initial state on
+    # the SIMT chunked scan
     B, L, D, M = 4, 32768, 256, 16
     inp = make_inputs(B, L, D, M, "f32", seed=1)
     x = torch.from_numpy(inp.x).to(dev)
     p = rlm.Params.from_arrays(*inp.params(), device=dev)
     y = torch.empty_like(x)
     st = rlm.State.empty(B, D, M, device=dev)
+    s_in = rlm.State.empty(B, D, M, device=dev)
+    s_in.s.copy_(torch.randn(B, D, M, 2, generator=torch.Generator(device="cpu").manual_seed(2)))
     work = torch.empty(max(rlm.rlm_prefill_workspace_size(B, L, D, M, torch.float32), 256), dtype=torch.uint8,
                        device=dev)
     timed("fp32_prefill", lambda: rlm.rlm_mix_prefill(x, p, y, st, workspace=work), prefill_bytes(B, L, D, M, 4))
-    del x, y, work
+    timed("fp32_prefill_state", lambda: rlm.rlm_mix_prefill_from(x, p, s_in, y, st, workspace=work),
+          prefill_bytes(B, L, D, M, 4))
+    del x, y, work, s_in
 
     # plain decode steps
     for Bd in (64, 1):
@@ -871,8 +880,24 @@ def run_kernels_only(args):
         yt = torch.empty_like(tok)
         timed(f"decode_b{Bd}", lambda: rlm.rlm_mix_decode(tok, dst, yt), decode_bytes(Bd, D, M))
 
-    # coupled mixer decode step, fused (D = 256) and with the finishing pass (D = 2048)
+    # mixer decode step without coupling on rows past the one-block step (the
+    # recurrence step with gate and local path, k_decode_vec2)
     H, K = 8, 4
+    Bd, Dm = 64, 2048
+    dinp = make_inputs(Bd, 1, Dm, M, "bf16", seed=4, decode_steps=2)
+    dmx = make_mixer_inputs(dinp, K, seed=4)
+    dp = rlm.Params.from_arrays(*dinp.params(), device=dev)
+    dst = rlm.State.empty(Bd, Dm, M, device=dev)
+    rlm.rlm_state_init(dst, dp)
+    loc = rlm.Local.from_arrays(dmx.conv_w, dmx.scale, device=dev)
+    hist = rlm.ConvState(torch.zeros(Bd, K - 1, Dm, dtype=torch.bfloat16, device=dev))
+    tok = torch.from_numpy(dinp.tokens[0]).to(dev, torch.bfloat16)
+    gt = torch.randn(Bd, 1, Dm, device=dev).to(torch.bfloat16).view_as(tok)
+    zt = torch.empty_like(tok)
+    timed("mixer_decode_plain", lambda: rlm.rlm_mixer_decode(tok, gt, dst, loc, hist, zt),
+          decode_bytes(Bd, Dm, M) + 2 * Bd * Dm * (K - 1) * 2 + 2 * Bd * Dm)
+
+    # coupled mixer decode step, fused (D = 256) and with the finishing pass (D = 2048)
     for Dm in (256, 2048):
         Bd = 64
         dinp = make_inputs(Bd, 1, Dm, M, "bf16", seed=4, decode_steps=2)
