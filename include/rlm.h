@@ -31,7 +31,9 @@
  *    bounded number of iterations; on expiry they record RLM_ERR_TIMEOUT in a
  *    device status word and return without hanging.  rlm_get_device_status()
  *    reads and clears that word.
- *  - Shapes: B >= 1, L >= 1, D >= 8 with D % 8 == 0, 1 <= M <= 64.
+ *  - Shapes: B >= 1, L >= 1, D >= 8 with D % 8 == 0, 1 <= M <= 64.  Limits
+ *    (RLM_ERR_UNSUPPORTED beyond): B <= 65535, D <= 2^20, L <= 2^24 (the kernels
+ *    form lambda^n from fp32 token counts, which are exact up to 2^24).
  *  - Element types of x, y, dy, dx: RLM_F32 or RLM_BF16 (all four of one call
  *    share one type).  Parameters, gradients and the decode state are fp32.
  *  - Inputs and outputs of one call must not overlap.

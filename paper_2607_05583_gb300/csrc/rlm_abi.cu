@@ -83,8 +83,9 @@ rlm_status check_tensor(const rlm_tensor *t, const char *name) {
                     (long long)t->D);
     if (t->D > (1 << 20)) return fail(RLM_ERR_UNSUPPORTED, "%s has D=%lld > 2^20", name, (long long)t->D);
     if (t->B > 65535) return fail(RLM_ERR_UNSUPPORTED, "%s has B=%lld > 65535", name, (long long)t->B);
-    if (t->L > (int64_t)1 << 30)
-        return fail(RLM_ERR_UNSUPPORTED, "%s has L=%lld > 2^30", name, (long long)t->L);
+    // lambda^n is formed from fp32 token counts n, exact up to 2^24.
+    if (t->L > (int64_t)1 << 24)
+        return fail(RLM_ERR_UNSUPPORTED, "%s has L=%lld > 2^24", name, (long long)t->L);
     return RLM_OK;
 }
 

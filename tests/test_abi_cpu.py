@@ -122,6 +122,14 @@ def test_prefill_rejects_bad_arguments_on_host(lib, case):
     assert lib.rlm_last_error().decode()
 
 
+def test_sequences_past_2_to_24_tokens_are_unsupported(lib):
+    # The kernels form lambda^n from fp32 token counts, exact up to 2^24.
+    B, L, D, M = 1, (1 << 24) + 1, 8, 4
+    x, y = _t(FAKE, B, L, D), _t(FAKE + (1 << 36), B, L, D)
+    assert _prefill(lib, x, _p(D, M), y, None, None) == rlm.RLM_ERR_UNSUPPORTED
+    assert "2^24" in lib.rlm_last_error().decode()
+
+
 def test_prefill_from_rejects_bad_initial_states_on_host(lib):
     B, L, D, M = 2, 100, 64, 16
     x = _t(FAKE, B, L, D)
