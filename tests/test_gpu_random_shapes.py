@@ -30,8 +30,11 @@ def _config(i):
     H = int(r.choice([0, 0, 1, 2, 4, 8]))
     if H and D % H:
         H = 0
-    return dict(dtype=dtype, B=B, D=D, M=M, L=L, K=K, H=H, with_state=bool(r.random() < 0.5),
-                with_gate=bool(r.random() < 0.7), seed=1000 + i)
+    with_state = bool(r.random() < 0.5)
+    with_gate = bool(r.random() < 0.7)
+    with_gout = bool(r.random() < 0.5)   # drawn last: the earlier draws stay as they were
+    return dict(dtype=dtype, B=B, D=D, M=M, L=L, K=K, H=H, with_state=with_state, with_gate=with_gate,
+                with_gout=with_gout, seed=1000 + i)
 
 
 def _state_dev(B, D, M, s_np):
@@ -66,13 +69,17 @@ def test_random_configuration(i):
     assert_close(s.imag, st_ref.imag, tol, f"{c} state im")
 
     # backward with the state terms (the initial-state gradient whenever there is
-    # an initial state)
+    # an initial state or a terminal-state gradient)
+    g_out = None
+    if c["with_gout"]:
+        rg = np.random.default_rng(c["seed"] + 2)
+        g_out = rg.standard_normal((B, D, M)) + 1j * rg.standard_normal((B, D, M))
     dx = torch.empty_like(x)
     g = rlm.Grads.empty(D, M)
-    ds = rlm.State.empty(B, D, M) if s_in is not None else None
-    rlm.rlm_mix_backward_from(dy, x, p, si, None, dx, g, ds)
+    ds = rlm.State.empty(B, D, M) if (s_in is not None or g_out is not None) else None
+    rlm.rlm_mix_backward_from(dy, x, p, si, _state_dev(B, D, M, g_out) if g_out is not None else None, dx, g, ds)
     torch.cuda.synchronize()
-    dx_ref, g_ref = oracle.backward_rec(inp.x, inp.dy, *inp.params(), state_in=s_in)
+    dx_ref, g_ref = oracle.backward_rec(inp.x, inp.dy, *inp.params(), state_in=s_in, d_state_out=g_out)
     assert_close(to_np(dx), dx_ref, tol, f"{c} dx")
     for k in ("decay", "freq", "amp", "phase"):
         assert_close(getattr(g, k).cpu().numpy(), g_ref[k], tol, f"{c} d{k}")
