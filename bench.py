@@ -817,7 +817,7 @@ def run_kernels_only(args):
                           k_chunk_local, k_chunk_carry, k_chunk_output
       decode_b64 / b1     one plain decode step: k_decode_tile
       mixer_decode_plain  mixer step without coupling, B=64 D=2048 K=4 (rows past the
-                          one-block step): k_decode_vec2 (mixer)
+                          one-block step): k_decode_tile (mixer)
       mixer_decode_b64    coupled mixer step H=8 K=4 (D=256): k_decode_coupled
       mixer_prefill_d2048 coupled mixer prefill B=1 L=32768 D=2048 H=8 K=4 (4 KB rows):
                           k_prefill_tc, k_couple_small, k_mixer_epilogue, k_mixer_tail
@@ -881,7 +881,7 @@ def run_kernels_only(args):
         timed(f"decode_b{Bd}", lambda: rlm.rlm_mix_decode(tok, dst, yt), decode_bytes(Bd, D, M))
 
     # mixer decode step without coupling on rows past the one-block step (the
-    # recurrence step with gate and local path, k_decode_vec2)
+    # row-tiled recurrence step with gate and local path)
     H, K = 8, 4
     Bd, Dm = 64, 2048
     dinp = make_inputs(Bd, 1, Dm, M, "bf16", seed=4, decode_steps=2)

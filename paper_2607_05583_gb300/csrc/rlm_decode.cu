@@ -57,15 +57,13 @@ struct MixPart {
 };
 
 template <typename T>
-__device__ __forceinline__ MixPart<T> mix_part(const MixStep<T> &m, int64_t bd, int D, int g, int tpg,
-                                               const T *x_t) {
+__device__ __forceinline__ MixPart<T> mix_part(const MixStep<T> &m, int64_t b, int d, int64_t bd, int D,
+                                               int g, int tpg, const T *x_t) {
     MixPart<T> r;
     r.l = 0.0f;
     r.gate = 0.0f;
     if (m.g && g == 0) r.gate = ld_elem(m.g + bd);
     if (m.K > 0) {
-        const int d = (int)(bd % D);
-        const int64_t b = bd / D;
         const float *w = m.conv_w + (int64_t)d * m.K;
         if (g == 0) r.l = __ldg(w) * ld_elem(x_t + bd);
         const T *h = m.hist + b * (m.K - 1) * (int64_t)D + d;
@@ -85,11 +83,10 @@ __device__ __forceinline__ MixPart<T> mix_part(const MixStep<T> &m, int64_t bd, 
 // the old history are complete): shift the owned entries one slot down, rank 0
 // appends the current drive.
 template <typename T>
-__device__ __forceinline__ void mix_shift(const MixStep<T> &m, const MixPart<T> &r, int64_t bd, int D, int g,
-                                          int tpg, const T *x_t) {
+__device__ __forceinline__ void mix_shift(const MixStep<T> &m, const MixPart<T> &r, int64_t b, int d, int64_t bd,
+                                          int D, int g, int tpg, const T *x_t) {
     if (m.K < 2) return;
-    const int64_t b = bd / D;
-    T *h = m.hist + b * (m.K - 1) * (int64_t)D + (bd % D);
+    T *h = m.hist + b * (m.K - 1) * (int64_t)D + d;
 #pragma unroll
     for (int i = 0; i < 2; ++i) {
         const int j = g + i * tpg;
@@ -117,52 +114,7 @@ __device__ __forceinline__ void pdl_launch_dependents() {
     asm volatile("griddepcontrol.launch_dependents;" :::);
 }
 
-// MPT = 2 with M even: state and coefficients move as 16-byte vectors.
-template <typename T, bool kMix>
-__global__ void __launch_bounds__(kDecodeBlock) k_decode_vec2(
-    const T *__restrict__ x_t, T *__restrict__ y_t, int64_t BD, int D, int M, int log2_tpg,
-    float4 *__restrict__ s, const float4 *__restrict__ coef, MixStep<T> mix) {
-    const int64_t gid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    const int64_t bd = gid >> log2_tpg;
-    const int g = (int)(gid & ((1 << log2_tpg) - 1));
-    prefetch_step(x_t, mix, kMix, bd, BD, g);
-    pdl_wait();
-    pdl_launch_dependents();
-    const int tpg = 1 << log2_tpg;
-    const bool valid = bd < BD && 2 * g < M;
-    MixPart<T> mp{};
-    if (kMix && bd < BD) mp = mix_part(mix, bd, D, g, tpg, x_t);  // every rank, with or without modes
-    float acc = 0.0f;
-    if (valid) {
-        const int d = (int)(bd % D);
-        const float xv = ld_elem(x_t + bd);
-        const int64_t si = (bd * M) / 2 + g;  // pair index (M even)
-        float4 st = s[si];
-        const float4 c0 = __ldg(coef + d * M + 2 * g);
-        const float4 c1 = __ldg(coef + d * M + 2 * g + 1);
-        const float r0 = fmaf(c0.x, st.x, fmaf(-c0.y, st.y, xv));
-        const float i0 = fmaf(c0.x, st.y, c0.y * st.x);
-        const float r1 = fmaf(c1.x, st.z, fmaf(-c1.y, st.w, xv));
-        const float i1 = fmaf(c1.x, st.w, c1.y * st.z);
-        s[si] = make_float4(r0, i0, r1, i1);
-        acc = fmaf(c0.z, r0, fmaf(-c0.w, i0, fmaf(c1.z, r1, -c1.w * i1)));
-    }
-    float lsum = mp.l;
-    for (int o = tpg >> 1; o > 0; o >>= 1) {
-        acc += __shfl_xor_sync(0xffffffffu, acc, o);
-        if (kMix) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
-    }
-    if (kMix && bd < BD) {
-        mix_shift(mix, mp, bd, D, g, tpg, x_t);
-        if (g == 0) {
-            if (mix.g) acc *= 1.0f / (1.0f + expf(-mp.gate));
-            if (mix.K > 0) acc = fmaf(__ldg(mix.scale + bd % D), lsum, acc);
-        }
-    }
-    if (valid && g == 0) st_elem(y_t + bd, acc);
-}
-
-// The plain step (no mixer), M even with one mode pair per thread: a block of R
+// M even with one mode pair per thread: a block of R
 // warps covers the same 32 / tpg channels for R batch rows (warp w takes row
 // R * blockIdx.y + w), so the coefficient rows that every batch row needs are
 // fetched from L2 once per block and then hit in L1.  Within a warp the lanes
@@ -172,23 +124,33 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_vec2(
 // R = 16 against 1.97 (R = 8), 1.99 (R = 12), 1.97 (R = 24) and 2.03 (R = 32);
 // B = 8 took 1.16 with R = 8 and 1.29 with R = 16; B = 8192 (state above the L2
 // size, bandwidth-bound) 88.5 with R = 8 and 93.4 with R = 16.  A single row
-// (B = 1) took 1.05 us here against 1.37 on k_decode_vec2.
-template <typename T, int R>
+// (B = 1) took 1.05 us here against 1.37 with one block per 32 (b, d) pairs.
+// kMix adds the mixer step: the group's ranks share the history loads and the
+// shift, rank 0 takes the gate and the local path's sum; a group may then hold
+// ranks without modes.
+template <typename T, int R, bool kMix>
 __global__ void __launch_bounds__(R * 32) k_decode_tile(
     const T *__restrict__ x_t, T *__restrict__ y_t, int B, int D, int M, int log2_tpg,
-    float4 *__restrict__ s, const float4 *__restrict__ coef) {
+    float4 *__restrict__ s, const float4 *__restrict__ coef, MixStep<T> mix) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int g = lane & ((1 << log2_tpg) - 1);
+    const int tpg = 1 << log2_tpg;
+    const int g = lane & (tpg - 1);
     const int d = blockIdx.x * (32 >> log2_tpg) + (lane >> log2_tpg);
     const int b = blockIdx.y * R + warp;
-    const bool on = b < B && d < D && 2 * g < M;
+    const bool rowok = b < B && d < D;
+    const bool on = rowok && 2 * g < M;
     const int64_t bd = (int64_t)b * D + d;
-    if (on && g == 0 && (d & 63) == 0) prefetch_l2(x_t + bd);
+    if (rowok && g == 0 && (d & 63) == 0) {
+        prefetch_l2(x_t + bd);
+        if (kMix && mix.g) prefetch_l2(mix.g + bd);
+    }
     // The next step's grid may be scheduled before this one's wait returns (it
     // waits on this grid's completion in turn): measured 1.39 -> 1.15 us per step
     // at B = 8 with this kernel; neutral at B = 64.
     pdl_launch_dependents();
     pdl_wait();
+    MixPart<T> mp{};
+    if (kMix && rowok) mp = mix_part(mix, (int64_t)b, d, bd, D, g, tpg, x_t);  // every rank, with or without modes
     float acc = 0.0f;
     if (on) {
         const float4 c0 = __ldg(coef + d * M + 2 * g);
@@ -203,8 +165,19 @@ __global__ void __launch_bounds__(R * 32) k_decode_tile(
         s[si] = make_float4(r0, i0, r1, i1);
         acc = fmaf(c0.z, r0, fmaf(-c0.w, i0, fmaf(c1.z, r1, -c1.w * i1)));
     }
-    for (int o = (1 << log2_tpg) >> 1; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-    if (on && g == 0) st_elem(y_t + bd, acc);
+    float lsum = mp.l;
+    for (int o = tpg >> 1; o > 0; o >>= 1) {
+        acc += __shfl_xor_sync(0xffffffffu, acc, o);
+        if (kMix) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
+    }
+    if (kMix && rowok) {
+        mix_shift(mix, mp, (int64_t)b, d, bd, D, g, tpg, x_t);
+        if (g == 0) {
+            if (mix.g) acc *= 1.0f / (1.0f + expf(-mp.gate));
+            if (mix.K > 0) acc = fmaf(__ldg(mix.scale + d), lsum, acc);
+        }
+    }
+    if (rowok && g == 0) st_elem(y_t + bd, acc);
 }
 
 // Any M: each thread owns up to MPT modes, accessed as float2.
@@ -219,11 +192,12 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_any(
     pdl_wait();
     pdl_launch_dependents();
     const int tpg = 1 << log2_tpg;
+    const int64_t b = bd / D;
+    const int d = (int)(bd - b * D);
     MixPart<T> mp{};
-    if (kMix && bd < BD) mp = mix_part(mix, bd, D, g, tpg, x_t);
+    if (kMix && bd < BD) mp = mix_part(mix, b, d, bd, D, g, tpg, x_t);
     float acc = 0.0f;
     if (bd < BD) {
-        const int d = (int)(bd % D);
         const float xv = ld_elem(x_t + bd);
         for (int j = 0; j < mpt; ++j) {
             const int m = g * mpt + j;
@@ -242,10 +216,10 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_any(
         if (kMix) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
     }
     if (kMix && bd < BD) {
-        mix_shift(mix, mp, bd, D, g, tpg, x_t);
+        mix_shift(mix, mp, b, d, bd, D, g, tpg, x_t);
         if (g == 0) {
             if (mix.g) acc *= 1.0f / (1.0f + expf(-mp.gate));
-            if (mix.K > 0) acc = fmaf(__ldg(mix.scale + bd % D), lsum, acc);
+            if (mix.K > 0) acc = fmaf(__ldg(mix.scale + d), lsum, acc);
         }
     }
     if (bd < BD && g == 0) st_elem(y_t + bd, acc);
@@ -403,26 +377,24 @@ cudaError_t decode_t(const T *x_t, T *y_t, int B, int D, int M, float *s, const 
     while ((1 << log2_tpg) < pairs && log2_tpg < 5) ++log2_tpg;
     // The mixer step spreads the K - 1 <= 7 history entries over the group, two
     // at most per rank: at least 4 ranks (extra ranks own no modes).
-    const bool widened = kMix && log2_tpg < 2;
-    if (widened) log2_tpg = 2;
+    if (kMix && log2_tpg < 2) log2_tpg = 2;
     const int tpg = 1 << log2_tpg;
     const int64_t BD = (int64_t)B * D;
     const int64_t threads = BD * tpg;
     const unsigned grid = (unsigned)((threads + kDecodeBlock - 1) / kDecodeBlock);
     const float4 *cf = reinterpret_cast<const float4 *>(coef);
-    if (!kMix && M % 2 == 0 && 2 * tpg >= M) {
-        // Blocks of R batch rows sharing their channels' coefficient rows.
-        const int R = B >= 16 && B <= 256 ? 16 : 8;
+    if (M % 2 == 0 && 2 * tpg >= M) {
+        // Blocks of R batch rows sharing their channels' coefficient rows (the
+        // mixer step: 8 rows, 10.2 us a step at B = 64, D = 2048, M = 16, K = 4
+        // against 10.5 with 16 rows and 10.9 with 4).
+        const int R = !kMix && B >= 16 && B <= 256 ? 16 : 8;
         const dim3 gr((unsigned)((D + (32 >> log2_tpg) - 1) / (32 >> log2_tpg)), (unsigned)((B + R - 1) / R));
         if (R == 16)
-            return launch_pdl_block(k_decode_tile<T, 16>, gr, 16 * 32, st, x_t, y_t, B, D, M, log2_tpg,
-                                    reinterpret_cast<float4 *>(s), cf);
-        return launch_pdl_block(k_decode_tile<T, 8>, gr, 8 * 32, st, x_t, y_t, B, D, M, log2_tpg,
-                                reinterpret_cast<float4 *>(s), cf);
+            return launch_pdl_block(k_decode_tile<T, 16, kMix>, gr, 16 * 32, st, x_t, y_t, B, D, M, log2_tpg,
+                                    reinterpret_cast<float4 *>(s), cf, mix);
+        return launch_pdl_block(k_decode_tile<T, 8, kMix>, gr, 8 * 32, st, x_t, y_t, B, D, M, log2_tpg,
+                                reinterpret_cast<float4 *>(s), cf, mix);
     }
-    if (!widened && M % 2 == 0 && 2 * tpg >= M)
-        return launch_pdl(k_decode_vec2<T, kMix>, grid, st, x_t, y_t, BD, D, M, log2_tpg,
-                          reinterpret_cast<float4 *>(s), cf, mix);
     const int mpt = (M + tpg - 1) / tpg;
     return launch_pdl(k_decode_any<T, kMix>, grid, st, x_t, y_t, BD, D, M, log2_tpg, mpt,
                       reinterpret_cast<float2 *>(s), cf, mix);

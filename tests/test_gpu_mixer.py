@@ -123,12 +123,15 @@ def test_mixer_split_prefill_in_place_equals_whole(M):
     np.testing.assert_array_equal(to_np(cs.u), tr)
 
 
-@pytest.mark.parametrize("dtype,M,K", [("bf16", 16, 4), ("f32", 7, 3), ("bf16", 40, 8), ("bf16", 16, 1),
-                                     ("f32", 1, 8), ("bf16", 2, 6), ("bf16", 6, 8)])
-def test_mixer_decode_continues_the_prefill(dtype, M, K):
+@pytest.mark.parametrize("dtype,M,K,B", [("bf16", 16, 4, 3), ("f32", 7, 3, 3), ("bf16", 40, 8, 3), ("bf16", 16, 1, 3),
+                                       ("f32", 1, 8, 3), ("bf16", 2, 6, 3), ("bf16", 6, 8, 3),
+                                       ("bf16", 16, 4, 12), ("f32", 2, 6, 12), ("bf16", 40, 8, 12)])
+def test_mixer_decode_continues_the_prefill(dtype, M, K, B):
     """Prefill of 300 tokens then 40 fused mixer decode steps reproduce the oracle's
-    mixer output over all 340 tokens, and the final state and history."""
-    B, D, L0, T = 3, 32, 300, 40
+    mixer output over all 340 tokens, and the final state and history.  Up to 8
+    rows take the row-tiled step; 12 rows of at most 4096 modes take one block per
+    row (M = 40, twenty mode pairs, stays on row tiles)."""
+    D, L0, T = 32, 300, 40
     inp = make_inputs(B, L0 + T, D, M, dtype, seed=M + K)
     mx = make_mixer_inputs(inp, K, seed=M + K)
     x, g = to_dev(inp.x, dtype), to_dev(mx.g, dtype)
