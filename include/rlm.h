@@ -297,12 +297,11 @@ RLM_API rlm_status rlm_mixer_prefill(const rlm_tensor *x, const rlm_tensor *g, c
                                      rlm_conv_state *conv_out, const rlm_launch *launch);
 
 /* One decode step of the mixer: the recurrence step of rlm_mix_decode, the
- * coupling, the gate, and the local path over the cached history.  One kernel,
- * one block per batch row, where D <= 512, D * M <= 4096 and M / 2 is a power of
- * two, and the step is coupled or has more than 8 rows; otherwise the decode
- * kernel with the gate and the local path fused (with coupling: the recurrence
- * step, then one kernel per batch row for the coupling, the gate and the local
- * path).
+ * coupling, the gate, and the local path over the cached history.  Without
+ * coupling: the decode kernel with the gate and the local path fused.  With
+ * coupling: one kernel, one block per batch row, where D <= 512, D * M <= 4096
+ * and M / 2 is a power of two; otherwise the recurrence step, then one kernel per
+ * batch row for the coupling, the gate and the local path.
  *   x_t, g_t [B][1][D] (g_t nullable: no gate); state updated in place; conv
  *   ([B][K-1][D], required when K >= 2) shifted in place by one token; z_t
  *   [B][1][D] output.  No workspace. */

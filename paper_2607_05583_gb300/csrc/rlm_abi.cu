@@ -464,13 +464,9 @@ rlm_status rlm_mixer_decode(const rlm_tensor *x_t, const rlm_tensor *g_t, rlm_st
     }
     cudaStream_t st = static_cast<cudaStream_t>(ln->stream);
     cudaError_t e;
-    // One block per batch row serves the coupled step, and the uncoupled one where
-    // it measured faster than the row-tiled step: rows of at most 4096 modes in
-    // batches of more than 8 (a CUDA graph of steps with K = 4 and a gate, us per
-    // step, row block against row tiles: D = 256, M = 16 at B = 16 2.76 / 3.42,
-    // B = 64 3.10 / 3.63; D = 256, M = 2, B = 64 2.34 / 3.36; but B = 8 2.75 /
-    // 1.97 and D = 512, M = 32, B = 64 7.97 / 5.95).
-    const bool row_block = coupling || (x_t->B > 8 && x_t->D * state->M <= 4096);
+    // One block per batch row serves the coupled step; the uncoupled step runs on
+    // the row-tiled decode kernel.
+    const bool row_block = coupling != nullptr;
     if (row_block && mixer_decode_coupled_supported((int)x_t->D, state->M)) {
         // One launch: recurrence step, coupling (if any), gate, local path.
         e = mixer_decode_coupled(x_t->ptr, g_t ? g_t->ptr : nullptr, z_t->ptr, x_t->dtype, (int)x_t->B,

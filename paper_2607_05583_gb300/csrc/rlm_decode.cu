@@ -53,6 +53,8 @@ template <typename T>
 struct MixPart {
     float l;          // partial sum of w[k] u_{t-k}
     float gate;       // rank 0: g_t
+    float sc;         // rank 0: the channel's scale
+    T xr;             // rank 0: u_t as stored, appended to the history
     T hv[2];          // the history entries this thread owns (tpg >= 4 gives at most two)
 };
 
@@ -62,10 +64,16 @@ __device__ __forceinline__ MixPart<T> mix_part(const MixStep<T> &m, int64_t b, i
     MixPart<T> r;
     r.l = 0.0f;
     r.gate = 0.0f;
+    r.sc = 0.0f;
     if (m.g && g == 0) r.gate = ld_elem(m.g + bd);
     if (m.K > 0) {
         const float *w = m.conv_w + (int64_t)d * m.K;
-        if (g == 0) r.l = __ldg(w) * ld_elem(x_t + bd);
+        if (g == 0) {
+            // Every load of the step is issued here, before the reductions.
+            r.xr = x_t[bd];
+            r.sc = __ldg(m.scale + d);
+            r.l = __ldg(w) * as_float(r.xr);
+        }
         const T *h = m.hist + b * (m.K - 1) * (int64_t)D + d;
 #pragma unroll
         for (int i = 0; i < 2; ++i) {
@@ -83,8 +91,8 @@ __device__ __forceinline__ MixPart<T> mix_part(const MixStep<T> &m, int64_t b, i
 // the old history are complete): shift the owned entries one slot down, rank 0
 // appends the current drive.
 template <typename T>
-__device__ __forceinline__ void mix_shift(const MixStep<T> &m, const MixPart<T> &r, int64_t b, int d, int64_t bd,
-                                          int D, int g, int tpg, const T *x_t) {
+__device__ __forceinline__ void mix_shift(const MixStep<T> &m, const MixPart<T> &r, int64_t b, int d, int D, int g,
+                                          int tpg) {
     if (m.K < 2) return;
     T *h = m.hist + b * (m.K - 1) * (int64_t)D + d;
 #pragma unroll
@@ -92,7 +100,7 @@ __device__ __forceinline__ void mix_shift(const MixStep<T> &m, const MixPart<T> 
         const int j = g + i * tpg;
         if (j >= 1 && j < m.K - 1) h[(int64_t)(j - 1) * D] = r.hv[i];
     }
-    if (g == 0) h[(int64_t)(m.K - 2) * D] = x_t[bd];
+    if (g == 0) h[(int64_t)(m.K - 2) * D] = r.xr;
 }
 
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
@@ -128,8 +136,11 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 // kMix adds the mixer step: the group's ranks share the history loads and the
 // shift, rank 0 takes the gate and the local path's sum; a group may then hold
 // ranks without modes.
+// The launch bound holds the kernel to 32 registers, so 64 warps stay resident
+// per SM (the mixer step spills 8 bytes): at 40 registers the mixer step took
+// 11.1 us a step at B = 64, D = 2048, M = 16 against 10.6.
 template <typename T, int R, bool kMix>
-__global__ void __launch_bounds__(R * 32) k_decode_tile(
+__global__ void __launch_bounds__(R * 32, 2048 / (R * 32)) k_decode_tile(
     const T *__restrict__ x_t, T *__restrict__ y_t, int B, int D, int M, int log2_tpg,
     float4 *__restrict__ s, const float4 *__restrict__ coef, MixStep<T> mix) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -144,11 +155,12 @@ __global__ void __launch_bounds__(R * 32) k_decode_tile(
         prefetch_l2(x_t + bd);
         if (kMix && mix.g) prefetch_l2(mix.g + bd);
     }
-    // The next step's grid may be scheduled before this one's wait returns (it
-    // waits on this grid's completion in turn): measured 1.39 -> 1.15 us per step
-    // at B = 8 with this kernel; neutral at B = 64.
-    pdl_launch_dependents();
+    // The next step's grid is released once this one's wait has returned.  In a
+    // CUDA graph of steps (D = 256, M = 16, B = 8 / 64, us per step) that gave
+    // 1.05 / 1.95 for the plain step and 1.86 / 2.53 for the mixer step (K = 4,
+    // gate), against 1.20 / 2.08 and 1.95 / 3.91 with the release before the wait.
     pdl_wait();
+    pdl_launch_dependents();
     MixPart<T> mp{};
     if (kMix && rowok) mp = mix_part(mix, (int64_t)b, d, bd, D, g, tpg, x_t);  // every rank, with or without modes
     float acc = 0.0f;
@@ -171,10 +183,10 @@ __global__ void __launch_bounds__(R * 32) k_decode_tile(
         if (kMix) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
     }
     if (kMix && rowok) {
-        mix_shift(mix, mp, (int64_t)b, d, bd, D, g, tpg, x_t);
+        mix_shift(mix, mp, (int64_t)b, d, D, g, tpg);
         if (g == 0) {
             if (mix.g) acc *= 1.0f / (1.0f + expf(-mp.gate));
-            if (mix.K > 0) acc = fmaf(__ldg(mix.scale + d), lsum, acc);
+            if (mix.K > 0) acc = fmaf(mp.sc, lsum, acc);
         }
     }
     if (rowok && g == 0) st_elem(y_t + bd, acc);
@@ -216,10 +228,10 @@ __global__ void __launch_bounds__(kDecodeBlock) k_decode_any(
         if (kMix) lsum += __shfl_xor_sync(0xffffffffu, lsum, o);
     }
     if (kMix && bd < BD) {
-        mix_shift(mix, mp, b, d, bd, D, g, tpg, x_t);
+        mix_shift(mix, mp, b, d, D, g, tpg);
         if (g == 0) {
             if (mix.g) acc *= 1.0f / (1.0f + expf(-mp.gate));
-            if (mix.K > 0) acc = fmaf(__ldg(mix.scale + d), lsum, acc);
+            if (mix.K > 0) acc = fmaf(mp.sc, lsum, acc);
         }
     }
     if (bd < BD && g == 0) st_elem(y_t + bd, acc);

@@ -128,9 +128,9 @@ def test_mixer_split_prefill_in_place_equals_whole(M):
                                        ("bf16", 16, 4, 12), ("f32", 2, 6, 12), ("bf16", 40, 8, 12)])
 def test_mixer_decode_continues_the_prefill(dtype, M, K, B):
     """Prefill of 300 tokens then 40 fused mixer decode steps reproduce the oracle's
-    mixer output over all 340 tokens, and the final state and history.  Up to 8
-    rows take the row-tiled step; 12 rows of at most 4096 modes take one block per
-    row (M = 40, twenty mode pairs, stays on row tiles)."""
+    mixer output over all 340 tokens, and the final state and history (row-tiled
+    step: 3 rows in one block of 8, 12 rows over two; M = 1, 7 on the any-M
+    kernel)."""
     D, L0, T = 32, 300, 40
     inp = make_inputs(B, L0 + T, D, M, dtype, seed=M + K)
     mx = make_mixer_inputs(inp, K, seed=M + K)
