@@ -142,7 +142,7 @@ __device__ __forceinline__ void pdl_launch_dependents() {
 template <typename T, int R, bool kMix>
 __global__ void __launch_bounds__(R * 32, 2048 / (R * 32)) k_decode_tile(
     const T *__restrict__ x_t, T *__restrict__ y_t, int B, int D, int M, int log2_tpg,
-    float4 *__restrict__ s, const float4 *__restrict__ coef, MixStep<T> mix) {
+    float4 *__restrict__ s, const float4 *__restrict__ coef, MixStep<T> mix, bool late) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tpg = 1 << log2_tpg;
     const int g = lane & (tpg - 1);
@@ -155,12 +155,16 @@ __global__ void __launch_bounds__(R * 32, 2048 / (R * 32)) k_decode_tile(
         prefetch_l2(x_t + bd);
         if (kMix && mix.g) prefetch_l2(mix.g + bd);
     }
-    // The next step's grid is released once this one's wait has returned.  In a
-    // CUDA graph of steps (D = 256, M = 16, B = 8 / 64, us per step) that gave
-    // 1.05 / 1.95 for the plain step and 1.86 / 2.53 for the mixer step (K = 4,
-    // gate), against 1.20 / 2.08 and 1.95 / 3.91 with the release before the wait.
+    // The next step's grid is released once this one's wait has returned, or,
+    // for a plain step whose grid fits on the GPU at once (`late`), at the end.
+    // In a CUDA graph of steps (D = 256, M = 16, B = 8 / 64, us per step) the
+    // release after the wait gave 1.05 / 1.95 for the plain step and 1.86 / 2.53
+    // for the mixer step (K = 4, gate), against 1.20 / 2.08 and 1.95 / 3.91 with
+    // the release before the wait.  At the end, the plain step took 0.98 / 1.87
+    // against 1.24 / 1.97 in another harness, and the mixer step 1.72 / 2.76;
+    // grids of more than one wave lost 8-10 % (B = 256: 3.56 against 3.25).
     pdl_wait();
-    pdl_launch_dependents();
+    if (kMix || !late) pdl_launch_dependents();
     MixPart<T> mp{};
     if (kMix && rowok) mp = mix_part(mix, (int64_t)b, d, bd, D, g, tpg, x_t);  // every rank, with or without modes
     float acc = 0.0f;
@@ -190,6 +194,7 @@ __global__ void __launch_bounds__(R * 32, 2048 / (R * 32)) k_decode_tile(
         }
     }
     if (rowok && g == 0) st_elem(y_t + bd, acc);
+    if (!kMix && late) pdl_launch_dependents();
 }
 
 // Any M: each thread owns up to MPT modes, accessed as float2.
@@ -401,11 +406,13 @@ cudaError_t decode_t(const T *x_t, T *y_t, int B, int D, int M, float *s, const 
         // against 10.5 with 16 rows and 10.9 with 4).
         const int R = !kMix && B >= 16 && B <= 256 ? 16 : 8;
         const dim3 gr((unsigned)((D + (32 >> log2_tpg) - 1) / (32 >> log2_tpg)), (unsigned)((B + R - 1) / R));
+        // One wave: every block resident at once (32 registers: 2048 threads per SM).
+        const bool late = !kMix && (int64_t)gr.x * gr.y <= (int64_t)sm_count() * (2048 / (R * 32));
         if (R == 16)
             return launch_pdl_block(k_decode_tile<T, 16, kMix>, gr, 16 * 32, st, x_t, y_t, B, D, M, log2_tpg,
-                                    reinterpret_cast<float4 *>(s), cf, mix);
+                                    reinterpret_cast<float4 *>(s), cf, mix, late);
         return launch_pdl_block(k_decode_tile<T, 8, kMix>, gr, 8 * 32, st, x_t, y_t, B, D, M, log2_tpg,
-                                reinterpret_cast<float4 *>(s), cf, mix);
+                                reinterpret_cast<float4 *>(s), cf, mix, late);
     }
     const int mpt = (M + tpg - 1) / tpg;
     return launch_pdl(k_decode_any<T, kMix>, grid, st, x_t, y_t, BD, D, M, log2_tpg, mpt,
