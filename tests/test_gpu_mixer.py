@@ -156,6 +156,38 @@ def test_mixer_decode_continues_the_prefill(dtype, M, K, B):
         np.testing.assert_array_equal(to_np(cs.u), tr)
 
 
+@pytest.mark.parametrize("B,D", [(8, 256), (64, 2048)])
+def test_mixer_decode_on_one_and_several_waves(B, D):
+    """The row-tiled mixer step on a grid that fits on the GPU at once (8 x 256)
+    and on one of several waves (64 x 2048: 4096 blocks), chained over 5 steps
+    after a 6-token prefill: output, state and history against the oracle on
+    sampled channels, the first and last included."""
+    M, K, L0, T = 16, 4, 6, 5
+    inp = make_inputs(B, L0 + T, D, M, "bf16", seed=D)
+    mx = make_mixer_inputs(inp, K, seed=D)
+    x, g = to_dev(inp.x, "bf16"), to_dev(mx.g, "bf16")
+    p = rlm.Params.from_arrays(*inp.params())
+    local = rlm.Local.from_arrays(mx.conv_w, mx.scale)
+    st = rlm.State.empty(B, D, M)
+    cs = rlm.ConvState.empty(B, D, K, dtype=x.dtype)
+    z0 = torch.empty_like(x[:, :L0])
+    rlm.rlm_mixer_prefill(x[:, :L0].contiguous(), g[:, :L0].contiguous(), p, local, z0, state_out=st, conv_out=cs)
+    zs = []
+    for t in range(L0, L0 + T):
+        zt = torch.empty_like(x[:, t])
+        rlm.rlm_mixer_decode(x[:, t].contiguous(), g[:, t].contiguous(), st, local, cs, zt)
+        zs.append(zt)
+    torch.cuda.synchronize()
+    chans = np.unique(np.r_[np.random.default_rng(B).choice(D, 45, replace=False), 0, D - 1])
+    zr, sr, tr = oracle.mixer_prefill(inp.x[:, :, chans], mx.g[:, :, chans], inp.decay[chans], inp.freq[chans],
+                                      inp.amp[chans], inp.phase[chans], mx.conv_w[chans], mx.scale[chans])
+    assert_close(to_np(torch.stack(zs, 1))[:, :, chans], zr[:, L0:], TOL["bf16"], "decode z")
+    s = st.complex().cpu().numpy()[:, chans]
+    assert_close(s.real, sr.real, TOL["bf16"], "state re")
+    assert_close(s.imag, sr.imag, TOL["bf16"], "state im")
+    np.testing.assert_array_equal(to_np(cs.u)[:, :, chans], tr)
+
+
 def test_mixer_decode_without_gate_or_local_path_is_the_decode():
     inp = make_inputs(4, 1, 64, 16, "bf16", seed=2)
     x = to_dev(inp.x[:, 0], "bf16")

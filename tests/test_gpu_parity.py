@@ -432,6 +432,32 @@ def test_decode_after_32k_prefill(B):
     assert_close(s.real, st_ref.real, TOL["bf16"], "state re")
 
 
+@pytest.mark.parametrize("B,D", [(8, 1024), (8, 8192), (64, 4096)])
+def test_decode_grids_of_one_and_several_waves(B, D):
+    """The row-tiled step on a grid that fits on the GPU at once (8 x 1024: 256
+    blocks) and on grids of several waves (8 x 8192: 2048 blocks of 8 rows;
+    64 x 4096: 4096 blocks of 16 rows), which release the next step at different
+    points: chained steps after a short prefill against the oracle on sampled
+    channels, the first and last included."""
+    L, M, T = 5, 16, 6
+    inp = make_inputs(B, L, D, M, "bf16", seed=D + B, decode_steps=T)
+    _, st = _prefill(inp)
+    toks = to_dev(inp.tokens, "bf16")                  # [T][B][D]
+    out = torch.empty_like(toks)
+    for t in range(T):
+        rlm.rlm_mix_decode(toks[t], st, out[t])
+    torch.cuda.synchronize()
+    chans = np.unique(np.r_[np.random.default_rng(B).choice(D, 61, replace=False), 0, D // 2, D - 1])
+    xcat = np.concatenate([inp.x[:, :, chans], inp.tokens[:, :, chans].transpose(1, 0, 2)], 1)
+    ref, st_ref = oracle.rec_prefill(xcat, inp.decay[chans], inp.freq[chans], inp.amp[chans],
+                                     inp.phase[chans])
+    got = to_np(out)[:, :, chans].transpose(1, 0, 2)
+    assert_close(got, ref[:, L:], TOL["bf16"], "decode y_t")
+    s = st.complex().cpu().numpy()[:, chans]
+    assert_close(s.real, st_ref.real, TOL["bf16"], "state re")
+    assert_close(s.imag, st_ref.imag, TOL["bf16"], "state im")
+
+
 def test_state_init_then_decode_equals_prefill():
     inp = make_inputs(2, 50, 16, 16, "f32", seed=4)
     p = rlm.Params.from_arrays(*inp.params())
