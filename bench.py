@@ -364,7 +364,7 @@ def run_ours(args):
         # the 6M layer's prefill (B = 8, L = 2048)
         sweep["layer6m_B8_L2048"] = _time_prefill(rlm, torch, dev, 8, 2048, P["D"], P["M"], flush,
                                                   hbm_peak, reps=max(5, args.steps // 2))
-        # fp32 I/O on the headline shape (the SIMT chunked scan; 8 B per token-channel)
+        # fp32 I/O on the headline shape (the fp32 tcgen05 prefill; 8 B per token-channel)
         sweep[f"fp32_B{P['B']}_L{P['L']}"] = _time_prefill(rlm, torch, dev, P["B"], P["L"], P["D"], P["M"],
                                                            flush, hbm_peak, reps=max(5, args.steps // 2),
                                                            dtype="f32")
@@ -813,7 +813,8 @@ def run_kernels_only(args):
     flushed before each) and the line reports its mean time and algorithmic
     bytes.  Cases and the kernels they launch:
       fp32_prefill        B=4 L=32768 D=256 M=16 fp32: k_prefill_tc32
-      fp32_prefill_state  the same with an initial state (the SIMT chunked scan):
+      fp32_prefill_state  the same with an initial state: k_prefill_tc32
+      fp32_prefill_state_ragged  B=4 L=32767 with an initial state (the SIMT chunked scan):
                           k_chunk_local, k_chunk_carry, k_chunk_output
       decode_b64 / b1     one plain decode step: k_decode_tile
       mixer_decode_plain  mixer step without coupling, B=64 D=2048 K=4 (rows past the
@@ -853,8 +854,9 @@ def run_kernels_only(args):
         out[name] = {"ms": round(ms, 5), "algorithmic_bytes": alg_bytes, "achieved_GBps": round(gbs, 1),
                      "frac_hbm": round(gbs / hbm_peak, 4)}
 
-    # fp32 prefill: from a zero state on the tensor cores, from an initial state on
-    # the SIMT chunked scan
+    # fp32 prefill on the tensor cores, from a zero state and from an initial state;
+    # with an initial state and a length that is not a multiple of 64, the SIMT
+    # chunked scan
     B, L, D, M = 4, 32768, 256, 16
     inp = make_inputs(B, L, D, M, "f32", seed=1)
     x = torch.from_numpy(inp.x).to(dev)
@@ -868,7 +870,11 @@ def run_kernels_only(args):
     timed("fp32_prefill", lambda: rlm.rlm_mix_prefill(x, p, y, st, workspace=work), prefill_bytes(B, L, D, M, 4))
     timed("fp32_prefill_state", lambda: rlm.rlm_mix_prefill_from(x, p, s_in, y, st, workspace=work),
           prefill_bytes(B, L, D, M, 4))
-    del x, y, work, s_in
+    xr = x[:, :L - 1].contiguous()
+    yr = torch.empty_like(xr)
+    timed("fp32_prefill_state_ragged", lambda: rlm.rlm_mix_prefill_from(xr, p, s_in, yr, st, workspace=work),
+          prefill_bytes(B, L - 1, D, M, 4))
+    del x, y, xr, yr, work, s_in
 
     # plain decode steps
     for Bd in (64, 1):

@@ -127,8 +127,8 @@ typedef struct {
  *    no sequence segments (B * D / 8 of at least about the SM count); else the
  *    tcgen05 reverse-time scan of the reversed drive;
  *  - BF16, 32 < M <= 64 without segments: passes of 16 modes, each adding to y;
- *  - FP32, M <= 16, zero initial state: the tensor-core prefill with each
- *    product split into bf16 high and low parts (three MMAs);
+ *  - FP32, M <= 16: the tensor-core prefill with each product split into bf16
+ *    high and low parts (three MMAs);
  *  - other cases: the SIMT chunked scan. */
 RLM_API rlm_status rlm_mix_prefill(const rlm_tensor *x, const rlm_params *p, rlm_tensor *y,
                            rlm_state *state_out, const rlm_launch *launch);

@@ -182,8 +182,8 @@ rlm_status check_prefill_states(const rlm_tensor *x, const rlm_tensor *y, const 
 
 // The prefill path for a problem: the tcgen05 prefill (bf16, M <= 64), its
 // time-reversed form (other bf16 M <= 32), the tcgen05 prefill for fp32 I/O
-// (M <= 16, zero initial state), else the SIMT scan.  Both bf16 tcgen05 forms
-// work in 64-token chunks aligned to one end of the sequence; when L is not a
+// (M <= 16), else the SIMT scan.  The tcgen05 forms work in 64-token chunks
+// aligned to one end of the sequence; when L is not a
 // multiple of 64, an initial state enters them through a negative power of
 // lambda (up to lambda^-63), which overflows fp32 for decays above 88/63 per
 // token.  Such calls run on the SIMT scan, whose powers of lambda are all
@@ -197,7 +197,7 @@ PrefillPath prefill_path(const rlm_tensor *x, int M, bool with_state_in) {
     if (state_in_needs_simt(x->L, with_state_in)) return PrefillPath::kSimt;
     if (tc_prefill_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kTc;
     if (tc_prefill_rev_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kRev;
-    if (!with_state_in && tc32_prefill_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kTc32;
+    if (tc32_prefill_supported(x->B, x->L, D, M, x->dtype)) return PrefillPath::kTc32;
     return PrefillPath::kSimt;
 }
 
@@ -215,7 +215,7 @@ cudaError_t launch_prefill(PrefillPath path, const rlm_tensor *x, const rlm_para
                                   ln->workspace, st);
         case PrefillPath::kTc32:
             return tc32_prefill(static_cast<const float *>(x->ptr), static_cast<float *>(y), x->B, x->L, D, M,
-                                p->decay, p->freq, p->amp, p->phase, so, co, st);
+                                p->decay, p->freq, p->amp, p->phase, sin, so, co, st);
         default:
             return simt_prefill(x->ptr, y, x->dtype, x->B, x->L, D, M, p->decay, p->freq, p->amp, p->phase,
                                 sin, so, co, ln->workspace, st);

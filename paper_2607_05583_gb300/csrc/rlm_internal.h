@@ -53,12 +53,13 @@ cudaError_t grad_reduce(int64_t nparts, int D, int M, const float *amp, const fl
                         float *g_amp, float *g_phase, cudaStream_t st);
 
 // ---- tcgen05 prefill for fp32 I/O (rlm_prefill_tc32.cu) ----------------------
-// fp32 x and y, M <= 16, from a zero state; the contraction in three bf16 MMAs
-// per product (hi and lo parts).  No workspace.  state_out / coef_out may be null.
+// fp32 x and y, M <= 16, from a zero state or from state_in (L a multiple of
+// 64); the contraction in three bf16 MMAs per product (hi and lo parts).  No
+// workspace.  state_in / state_out / coef_out may be null.
 bool tc32_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt);
 cudaError_t tc32_prefill(const float *x, float *y, int64_t B, int64_t L, int D, int M, const float *decay,
-                         const float *freq, const float *amp, const float *phase, float *state_out, float *coef_out,
-                         cudaStream_t st);
+                         const float *freq, const float *amp, const float *phase, const float *state_in,
+                         float *state_out, float *coef_out, cudaStream_t st);
 cudaError_t read_and_clear_tc32_status(int *status, cudaStream_t st);
 
 // ---- tcgen05 backward (rlm_backward_tc.cu) -----------------------------------

@@ -18,6 +18,10 @@
 // 16 bits, against a tolerance of 1e-4.  The carry between chunks, the
 // accumulators and the output stay fp32.
 //
+// An initial state s_in (L a multiple of 64, so token 0 opens chunk n0 of tile
+// 0) enters as the state carried into chunk n0: the up-projection then gives
+// lambda^(i+1) s_in at its positions i and the scan carries lambda^64 s_in on.
+//
 // A CTA owns one batch row and a group of DG = 4 channels.  An fp32 token row of
 // 4 channels is 16 bytes, the same slice of the [B][L][D] row as the bf16
 // kernel's 8 channels, so loads and stores have the bf16 kernel's granularity
@@ -322,6 +326,7 @@ __device__ __forceinline__ int au_operand(int c) { return au_slot(c) * kAuStride
 
 struct Tc32Args {
     const float *decay, *freq, *amp, *phase;
+    const float2 *state_in;  // nullable, [B][D][M]; L % 64 == 0 when set
     float2 *state_out;   // nullable, [B][D][M]
     float4 *coef_out;    // nullable, [D][M]
     float *y;            // for the plain stores of boxes that start before t = 0
@@ -755,10 +760,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float m_decay = mreal ? args.decay[pm] : 0.0f, m_freq = mreal ? args.freq[pm] : 0.0f;
         const float2 LC = lambda_pow(m_decay, m_freq, (float)kC);
         float2 S = make_float2(0.0f, 0.0f);
+        // Chunk n0 of tile 0 opens at token 0; a batch row's initial state (zero
+        // without one) is the state carried into it.
+        const int n0 = (int)((-args.t0) >> 6);
+        auto state_in_of = [&](int row) {
+            return (args.state_in && mreal) ? args.state_in[((int64_t)row * D + d0 + ch) * args.M + m]
+                                            : make_float2(0.0f, 0.0f);
+        };
+        float2 inj = kPack ? make_float2(0.0f, 0.0f) : state_in_of(b);
         uint8_t *bs = smem + kOffBs + ch * kBsStride + ri * kBsPart + (m / 4) * kBsLbo + (m % 4) * 4;
         for (int v = 0; v < nV; ++v) {
             const int bb = v & 1, u = v >> 1;
-            if (kPack && real_tile(v) == 0) S = make_float2(0.0f, 0.0f);   // a new batch row starts from zero
+            if (kPack && real_tile(v) == 0) {
+                S = make_float2(0.0f, 0.0f);   // a new batch row starts from zero (or its own s_in)
+                inj = state_in_of(row_of(v));
+            }
+            const bool inj_tile = args.state_in != nullptr && real_tile(v) == 0;
             if (!wait_bar(bar(kBarTwDone + 2 * ch + bb), u & 1, abort_flag)) break;
             // The chain of tile v has completed, so its reads of B-operand buffer
             // v & 1 are done: release it (one arrival per channel).
@@ -778,6 +795,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const float other = __shfl_xor_sync(0xffffffffu, a, 1);
                     const float2 Ln = ri ? make_float2(other, a) : make_float2(a, other);
                     const int nn = 16 * h + n;
+                    if (inj_tile && nn == n0) S = make_float2(S.x + inj.x, S.y + inj.y);
                     uint32_t hi, lo;
                     split_pack(S.x, S.y, hi, lo);
                     *reinterpret_cast<uint32_t *>(bs + (nn >> 3) * kBsSbo + (nn & 7) * 16) = ri ? lo : hi;
@@ -908,8 +926,9 @@ bool tc32_prefill_supported(int64_t B, int64_t L, int D, int M, rlm_dtype dt) {
 }
 
 cudaError_t tc32_prefill(const float *x, float *y, int64_t B, int64_t L, int D, int M, const float *decay,
-                         const float *freq, const float *amp, const float *phase, float *state_out, float *coef_out,
-                         cudaStream_t st) {
+                         const float *freq, const float *amp, const float *phase, const float *state_in,
+                         float *state_out, float *coef_out, cudaStream_t st) {
+    if (state_in && L % kC != 0) return cudaErrorInvalidValue;
     CUtensorMap mx, my;
     if (!make_field_map32(&mx, x, B, L, D) || !make_field_map32(&my, y, B, L, D)) return cudaErrorInvalidValue;
     static std::mutex mu;
@@ -934,6 +953,7 @@ cudaError_t tc32_prefill(const float *x, float *y, int64_t B, int64_t L, int D, 
     a.freq = freq;
     a.amp = amp;
     a.phase = phase;
+    a.state_in = reinterpret_cast<const float2 *>(state_in);
     a.state_out = reinterpret_cast<float2 *>(state_out);
     a.coef_out = reinterpret_cast<float4 *>(coef_out);
     a.y = y;

@@ -208,7 +208,10 @@ def _state_from(inp, s_np):
     (1, 4096, 16, 20, "bf16"),            # time-reversed scan, L a chunk multiple
     (1, 4096, 16, 7, "bf16"),             # tcgen05 prefill, 7 modes padded to 16 (segmented)
     (4, 3001, 256, 1, "bf16"),            # ... one mode per channel, unsegmented
-    (2, 1000, 16, 7, "f32"),              # SIMT
+    (2, 1000, 16, 7, "f32"),              # SIMT (L not a multiple of 64)
+    (2, 4096, 16, 7, "f32"),              # fp32 tcgen05 prefill, 7 modes padded to 16
+    (3, 2048 + 64 * 5, 64, 16, "f32"),    # ... token 0 inside the first tile
+    (9, 704, 256, 16, "f32"),             # ... several rows per CTA, each from its own state
     (1, 500, 8, 40, "bf16"),              # SIMT, bf16 with M > 32
     (2, 4096, 640, 32, "bf16"),           # 32-mode tcgen05 instance, two rows per CTA
     (1, 2048 * 2 + 64 * 3, 1024, 24, "bf16"),  # ... one row per CTA, token 0 inside the first tile
