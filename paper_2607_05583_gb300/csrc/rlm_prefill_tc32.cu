@@ -282,6 +282,9 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
           "=r"(v[14]), "=r"(v[15])
         : "r"(taddr));
 }
+__device__ __forceinline__ void tmem_ld1(uint32_t taddr, uint32_t &v) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x1.b32 {%0}, [%1];" : "=r"(v) : "r"(taddr));
+}
 __device__ __forceinline__ void tmem_wait_ld() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -784,18 +787,37 @@ __global__ void __launch_bounds__(kThreads, 1)
             // up-projection must have read it before it is rewritten.
             if (v > 0 && !wait_bar(bar(kBarUDone + 2 * ch + (bb ^ 1)), ((v - 1) >> 1) & 1, abort_flag)) break;
             tc_fence_after();
+            if (!inj_tile) {
 #pragma unroll
-            for (int h = 0; h < kNT / 16; ++h) {
-                uint32_t va[16];
-                tmem_ld16(tmem + (st_lane << 16) + bb * 128 + ch * kNT + 16 * h, va);
-                tmem_wait_ld();
+                for (int h = 0; h < kNT / 16; ++h) {
+                    uint32_t va[16];
+                    tmem_ld16(tmem + (st_lane << 16) + bb * 128 + ch * kNT + 16 * h, va);
+                    tmem_wait_ld();
 #pragma unroll
-                for (int n = 0; n < 16; ++n) {
-                    const float a = __uint_as_float(va[n]);
+                    for (int n = 0; n < 16; ++n) {
+                        const float a = __uint_as_float(va[n]);
+                        const float other = __shfl_xor_sync(0xffffffffu, a, 1);
+                        const float2 Ln = ri ? make_float2(other, a) : make_float2(a, other);
+                        const int nn = 16 * h + n;
+                        uint32_t hi, lo;
+                        split_pack(S.x, S.y, hi, lo);
+                        *reinterpret_cast<uint32_t *>(bs + (nn >> 3) * kBsSbo + (nn & 7) * 16) = ri ? lo : hi;
+                        S = cfma(LC, S, Ln);
+                    }
+                }
+            } else {
+                // A row's first tile with an initial state: the same steps, one
+                // chunk at a time (compact code, off the other tiles' path), the
+                // state added where chunk n0 opens at token 0.
+#pragma unroll 1
+                for (int nn = 0; nn < kNT; ++nn) {
+                    uint32_t r;
+                    tmem_ld1(tmem + (st_lane << 16) + bb * 128 + ch * kNT + nn, r);
+                    tmem_wait_ld();
+                    const float a = __uint_as_float(r);
                     const float other = __shfl_xor_sync(0xffffffffu, a, 1);
                     const float2 Ln = ri ? make_float2(other, a) : make_float2(a, other);
-                    const int nn = 16 * h + n;
-                    if (inj_tile && nn == n0) S = make_float2(S.x + inj.x, S.y + inj.y);
+                    if (nn == n0) S = make_float2(S.x + inj.x, S.y + inj.y);
                     uint32_t hi, lo;
                     split_pack(S.x, S.y, hi, lo);
                     *reinterpret_cast<uint32_t *>(bs + (nn >> 3) * kBsSbo + (nn & 7) * 16) = ri ? lo : hi;
