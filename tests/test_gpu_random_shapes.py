@@ -104,3 +104,79 @@ def test_random_configuration(i):
     z_ref, _, _ = oracle.mixer_prefill(inp.x, mx.g if c["with_gate"] else None, *inp.params(), mx.conv_w,
                                        mx.scale, state_in=s_in, conv_in=mx.conv_in if K else None, coupling=cp)
     assert_close(to_np(z), z_ref, tol, f"{c} z")
+
+
+N_DECODE = 24
+
+
+def _decode_config(i):
+    r = np.random.default_rng([2026, i])
+    dtype = "bf16" if r.random() < 0.75 else "f32"
+    B = int(r.choice([1, 2, 7, 8, 9, 16, 33, 64, 200]))
+    D = int(r.choice([8, 24, 64, 256, 520, 2048, 4096]))
+    M = int(r.choice([1, 2, 5, 6, 8, 16, 17, 32, 40, 64]))
+    K = int(r.choice([0, 1, 3, 4, 8]))
+    H = int(r.choice([0, 0, 0, 2, 8]))
+    mixer = bool(r.random() < 0.6)
+    with_gate = bool(r.random() < 0.7)
+    if H and (D % H or (D // H) % 4 or B * D * M > (1 << 21)):
+        H = 0
+    return dict(dtype=dtype, B=B, D=D, M=M, K=K, H=H, mixer=mixer, with_gate=with_gate, seed=5000 + i)
+
+
+@pytest.mark.parametrize("i", range(N_DECODE))
+def test_random_decode_configuration(i):
+    """Seeded decode configurations: 1 to 200 batch rows (grids of one or several
+    waves, blocks of 8 or 16 rows), D up to 4096, M from 1 to 64 (one mode pair
+    per thread, widened groups, several modes per thread), plain steps or the
+    mixer's (gate, local path, coupling).  A 3-token prefill, then 4 chained
+    steps, against the oracle over the whole sequence on sampled channels (all
+    channels with coupling), outputs and terminal state."""
+    c = _decode_config(i)
+    dtype, B, D, M, K, H = c["dtype"], c["B"], c["D"], c["M"], c["K"], c["H"]
+    tol = TOL[dtype]
+    L0, T = 3, 4
+    inp = make_inputs(B, L0 + T, D, M, dtype, seed=c["seed"])
+    x = to_dev(inp.x, dtype)
+    p = rlm.Params.from_arrays(*inp.params())
+    st = rlm.State.empty(B, D, M)
+    if H:
+        chans = np.arange(D)
+    else:
+        pick = np.random.default_rng(c["seed"]).choice(D, min(D, 40), replace=False)
+        chans = np.unique(np.r_[pick, D - 1])
+    params = (inp.decay[chans], inp.freq[chans], inp.amp[chans], inp.phase[chans])
+    outs = []
+    if not c["mixer"]:
+        y0 = torch.empty_like(x[:, :L0])
+        rlm.rlm_mix_prefill(x[:, :L0].contiguous(), p, y0, st)
+        for t in range(L0, L0 + T):
+            yt = torch.empty_like(x[:, t])
+            rlm.rlm_mix_decode(x[:, t].contiguous(), st, yt)
+            outs.append(yt)
+        torch.cuda.synchronize()
+        ref, st_ref = oracle.rec_prefill(inp.x[:, :, chans], *params)
+    else:
+        mx = make_mixer_inputs(inp, K, seed=c["seed"])
+        g = to_dev(mx.g, dtype) if c["with_gate"] else None
+        local = rlm.Local.from_arrays(mx.conv_w, mx.scale) if K else None
+        cp = (np.random.default_rng(c["seed"]).standard_normal((H, H)), 0.6) if H else None
+        cpl = rlm.Coupling.from_arrays(*cp) if H else None
+        hin = rlm.ConvState(to_dev(mx.conv_in, dtype)) if K else None
+        hout = rlm.ConvState.empty(B, D, K, dtype=x.dtype) if K else None
+        z0 = torch.empty_like(x[:, :L0])
+        rlm.rlm_mixer_prefill(x[:, :L0].contiguous(), g[:, :L0].contiguous() if g is not None else None, p, local,
+                              z0, conv_in=hin, state_out=st, conv_out=hout, coupling=cpl)
+        for t in range(L0, L0 + T):
+            zt = torch.empty_like(x[:, t])
+            rlm.rlm_mixer_decode(x[:, t].contiguous(), g[:, t].contiguous() if g is not None else None, st, local,
+                                 hout, zt, coupling=cpl)
+            outs.append(zt)
+        torch.cuda.synchronize()
+        ref, st_ref, _ = oracle.mixer_prefill(inp.x[:, :, chans], mx.g[:, :, chans] if c["with_gate"] else None,
+                                              *params, mx.conv_w[chans], mx.scale[chans],
+                                              conv_in=mx.conv_in[:, :, chans] if K else None, coupling=cp)
+    assert_close(to_np(torch.stack(outs, 1))[:, :, chans], ref[:, L0:], tol, f"{c} outputs")
+    s = st.complex().cpu().numpy()[:, chans]
+    assert_close(s.real, st_ref.real, tol, f"{c} state re")
+    assert_close(s.imag, st_ref.imag, tol, f"{c} state im")
